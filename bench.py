@@ -1,0 +1,466 @@
+"""Benchmark: band-GGNN forward + backward on GB300 (arXiv 1906.11786 hot path).
+
+One step = one pass of the whole hot path over one supergraph: T GGNN steps forward (band
+propagation + GRU) and their backward (GRU backward + transposed-band propagation, all parameter
+gradients); the training workload adds the mean-pool readout, loss and Adam.  Metric: node-steps
+per second = real (non-padding) nodes x T / step time.  Default workload: 64 program-shaped graphs
+(~72k nodes) packed at S = 128, P = 20 edge types, H = 64, bf16, T = 8.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config 2] [--impl ours|reference]
+
+Under torchrun every rank plans its own supergraph (different seeds; the paper gives each core its
+own supergraph) and runs with no data-path collective (weak scaling); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "node-steps/s (fwd+bwd)"
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"hbm_gbs": d["hbm_gbs"], "bf16": d["bf16_tflops"],
+                "bf16_sustained": d["bf16_tflops_sustained"], "src": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "src": "fallback"}
+
+
+def _dist():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+class Clocks:
+    """Samples nvidia-smi clocks and throttle reasons while the timed region runs."""
+
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx = float(f[1])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[4:8]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------------- workload
+
+
+def workload(config: int, rank: int, S=None, H=None):
+    from paper_1906_11786_gb300 import synth
+    c = dict(synth.CONFIGS[config])
+    S = S or c["S"]
+    H = H or c["H"]
+    if rank == 0:
+        graphs = synth.config_graphs(config, S=S)
+    else:  # every rank gets its own supergraph of the same shape
+        graphs = synth.config_graphs(config, S=S)
+        graphs = [synth.gen_graph(g.n_nodes, c["F"], c["reverse"],
+                                  c["max_off"] or S // 2, c["tree_win"] or S // 2, c["lam"],
+                                  synth.graph_seed(config, i) + 7919 * rank)
+                  for i, g in enumerate(graphs)]
+    P = 2 * c["F"] if c["reverse"] else c["F"]
+    cap = 0
+    if c["sizes"][0] == "fill":
+        cap = -(-c["sizes"][1] // S)
+    return graphs, dict(c, S=S, H=H, P=P, cap=cap)
+
+
+class OursStep:
+    """Device buffers and one fwd+bwd step through the C ABI."""
+
+    def __init__(self, config, graphs, c, seed=0):
+        import torch
+
+        from paper_1906_11786_gb300 import _binding as L
+        from paper_1906_11786_gb300 import synth
+        self.L, self.torch = L, torch
+        self.c = c
+        P, S, H, T = c["P"], c["S"], c["H"], c["T"]
+        self.dt = c["dtype"]
+        tdt = torch.bfloat16 if self.dt == "bf16" else torch.float32
+        t0 = time.perf_counter()
+        self.plan = L.band_plan(graphs, P, S, c["cap"])
+        self.plan_ms = (time.perf_counter() - t0) * 1e3
+        t0 = time.perf_counter()
+        self.plan.upload()
+        torch.cuda.synchronize()
+        self.upload_ms = (time.perf_counter() - t0) * 1e3
+        self.info = self.plan.info()
+        N, n_real = self.info["n_pad"], self.info["n_real"]
+        self.N, self.n_real = N, n_real
+        n_all = sum(g.n_nodes for g in graphs)
+        self.n_all = n_all
+        E = torch.from_numpy(synth.gen_states(n_all, H, seed).astype(np.float32)).to(tdt)
+        self.E_orig_host = E.pin_memory()
+        self.E_orig_dev = E.cuda()
+        self.E0 = torch.empty((N, H), dtype=tdt, device="cuda")
+        L.pack_states(self.plan, self.dt, H, self.E_orig_dev, self.E0)
+        prm = synth.gen_params(P, H, seed + 1)
+        self.prm = {}
+        for k, v in prm.items():
+            t = torch.from_numpy(np.asarray(v, np.float32))
+            self.prm[k] = (t.to(tdt) if k in ("W", "W_ih", "W_hh") else t).cuda()
+        dET = np.random.default_rng(seed + 2).standard_normal((N, H)).astype(np.float32)
+        dET[n_real:] = 0
+        self.dET = torch.from_numpy(dET).cuda()
+        self.dET_host = torch.from_numpy(dET).pin_memory()
+        self.grads = {k: torch.empty(s, device="cuda") for k, s in
+                      (("dW", (P, H, H)), ("db", (P, H)), ("dW_ih", (3 * H, H)),
+                       ("dW_hh", (3 * H, H)), ("db_ih", (3 * H,)), ("db_hh", (3 * H,)))}
+        self.grads_host = {k: torch.empty(v.shape, pin_memory=True) for k, v in self.grads.items()}
+        self.dE0 = torch.empty((N, H), device="cuda")
+        self.dE0_orig = torch.zeros((n_all, H), device="cuda")
+        self.dE0_host = torch.empty((n_all, H), pin_memory=True)
+        self.Y = torch.empty((N, H), device="cuda")
+        self.train = bool(c.get("train"))
+        if c["gru"]:
+            self.saved = torch.empty(L.ggnn_saved_bytes(self.plan, self.dt, H, T), dtype=torch.uint8,
+                                     device="cuda")
+            self.ws_f = torch.empty(L.workspace_bytes(self.plan, self.dt, H, L.BG_OP_GGNN_FWD),
+                                    dtype=torch.uint8, device="cuda")
+            self.ws_b = torch.empty(L.workspace_bytes(self.plan, self.dt, H, L.BG_OP_GGNN_BWD),
+                                    dtype=torch.uint8, device="cuda")
+            self.ET = torch.empty((N, H), dtype=tdt, device="cuda")
+        else:
+            self.ws_f = torch.empty(L.workspace_bytes(self.plan, self.dt, H, L.BG_OP_PROPAGATE_FWD),
+                                    dtype=torch.uint8, device="cuda")
+            self.ws_b = torch.empty(L.workspace_bytes(self.plan, self.dt, H, L.BG_OP_PROPAGATE_BWD),
+                                    dtype=torch.uint8, device="cuda")
+        if self.train:
+            n_g = self.info["n_packed"]
+            self.target = torch.from_numpy(
+                np.random.default_rng(seed + 3).standard_normal(n_g).astype(np.float32)).cuda()
+            self.loss = torch.zeros(4, device="cuda")
+            self.dw_out = torch.empty(H, device="cuda")
+            self.ws_r = torch.empty(L.workspace_bytes(self.plan, self.dt, H, L.BG_OP_READOUT),
+                                    dtype=torch.uint8, device="cuda")
+            names = ["W", "b", "W_ih", "W_hh", "b_ih", "b_hh", "w_out"]
+            self.opt = {}
+            for k in names:
+                master = torch.from_numpy(np.asarray(prm[k], np.float32)).cuda().reshape(-1)
+                self.opt[k] = (master, torch.zeros_like(master), torch.zeros_like(master))
+            self.adam_t = 0
+
+    def step(self, E0=None, dET=None):
+        L, c = self.L, self.c
+        H, T = c["H"], c["T"]
+        E0 = self.E0 if E0 is None else E0
+        dET = self.dET if dET is None else dET
+        if not c["gru"]:
+            L.band_propagate_fwd(self.plan, self.dt, H, E0, self.prm["W"], self.prm["b"], self.Y,
+                                 self.ws_f)
+            L.band_propagate_bwd(self.plan, self.dt, H, E0, self.prm["W"], dET, self.dE0,
+                                 self.grads["dW"], self.grads["db"], self.ws_b)
+            return
+        L.ggnn_step(self.plan, self.dt, H, T, self.prm, E0, self.ET, self.saved, self.ws_f)
+        if self.train:
+            L.readout_loss(self.plan, self.dt, H, self.ET, self.prm["w_out"], self.target,
+                           self.loss, self.dET, self.dw_out, self.ws_r)
+            dET = self.dET
+        L.ggnn_step_bwd(self.plan, self.dt, H, T, self.prm, self.saved, dET, self.dE0, self.grads,
+                        self.ws_b)
+        if self.train:
+            self.adam_t += 1
+            gmap = dict(self.grads, w_out=self.dw_out)
+            for k, (master, m, v) in self.opt.items():
+                g = gmap["d" + k] if k != "w_out" else gmap["w_out"]
+                work = self.prm[k].reshape(-1)
+                L.adam_step(master, work if work.dtype != self.torch.float32 else work, m, v,
+                            g.reshape(-1), 1e-3, 0.9, 0.999, 1e-8, self.adam_t)
+
+    def step_e2e(self):
+        """The user's call sequence with host buffers: H2D inputs, pack, fwd+bwd, unpack, D2H."""
+        torch, L = self.torch, self.L
+        self.E_orig_dev.copy_(self.E_orig_host, non_blocking=True)
+        self.dET.copy_(self.dET_host, non_blocking=True)
+        L.pack_states(self.plan, self.dt, self.c["H"], self.E_orig_dev, self.E0)
+        self.step()
+        L.unpack_states(self.plan, "f32", self.c["H"], self.dE0, self.dE0_orig)
+        self.dE0_host.copy_(self.dE0_orig, non_blocking=True)
+        for k, v in self.grads.items():
+            self.grads_host[k].copy_(v, non_blocking=True)
+        return (self.E_orig_host.numel() * self.E_orig_host.element_size()
+                + self.dET_host.numel() * 4,
+                self.dE0_host.numel() * 4 + sum(v.numel() * 4 for v in self.grads_host.values()))
+
+
+# --------------------------------------------------------------------------------- CPU oracle
+
+
+def oracle_sample(config: int, c, budget_s: float = 15.0):
+    """The oracle as it stands (single-threaded fp64) on a bounded sample of the workload: the
+    leading graphs of the batch, as many as fit the time budget; returns node-steps/s."""
+    import oracle
+    from paper_1906_11786_gb300 import synth
+    graphs = synth.config_graphs(config, S=c["S"])
+    P, S, H, T = c["P"], c["S"], c["H"], c["T"]
+    done_nodes, spent, used = 0, 0.0, 0
+    rng = np.random.default_rng(0)
+    prm = synth.gen_params(P, H, 1)
+    t_start = time.perf_counter()
+    for g in graphs:
+        t0 = time.perf_counter()
+        lay = oracle.layout([g], P, S)
+        N = lay.n_pad
+        E0 = np.zeros((N, H)); E0[: lay.n_real] = rng.standard_normal((lay.n_real, H))
+        e = (lay.kept_dst, lay.kept_src, lay.kept_type)
+        if c["gru"]:
+            Es, Ys = oracle.ggnn_fwd(N, P, H, T, lay.n_real, *e, E0, prm)
+            oracle.ggnn_bwd(N, P, H, T, lay.n_real, *e, prm, Es, Ys, rng.standard_normal((N, H)))
+        else:
+            oracle.propagate_fwd(N, P, H, *e, E0, prm["W"], prm["b"])
+            oracle.propagate_bwd(N, P, H, *e, E0, prm["W"], rng.standard_normal((N, H)))
+        spent += time.perf_counter() - t0
+        done_nodes += g.n_nodes
+        used += 1
+        if time.perf_counter() - t_start > budget_s:
+            break
+    return done_nodes * T / spent, {"graphs": used, "nodes": done_nodes, "seconds": spent}
+
+
+# --------------------------------------------------------------------------------- main
+
+
+def run_reference(args):
+    rank, world, _ = _dist()
+    if rank != 0:
+        return 0
+    from paper_1906_11786_gb300 import synth
+    graphs, c = workload(args.config, 0, args.S, args.H)
+    n_real = sum(g.n_nodes for g in graphs)
+    times = []
+    for i in range(args.warmup + args.steps):
+        v, s = oracle_sample(args.config, c, budget_s=args.ref_budget)
+        if i >= args.warmup:
+            times.append(v)
+    value = statistics.median(times)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "node-steps/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": n_real * c["T"] / value * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": synth.CONFIGS[args.config]["name"], "S": c["S"], "H": c["H"],
+                   "P": c["P"], "T": c["T"]},
+        "cpu_baseline": {"value": value, "unit": "node-steps/s", "cores": 1, "kind": "oracle",
+                         "sample": f"leading graphs of the batch per step, ~{args.ref_budget}s "
+                                   f"of single-threaded fp64 work ({s['graphs']} graphs, "
+                                   f"{s['nodes']} nodes)"},
+        "e2e": {"value": value, "unit": "node-steps/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--config", type=int, default=2)
+    ap.add_argument("--S", type=int, default=None)
+    ap.add_argument("--H", type=int, default=None)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--ref-budget", type=float, default=15.0)
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    rank, world, local = _dist()
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_1906_11786_gb300 import _binding as L
+    from paper_1906_11786_gb300 import synth
+
+    graphs, c = workload(args.config, rank, args.S, args.H)
+    st = OursStep(args.config, graphs, c, seed=rank)
+    H, T = c["H"], c["T"]
+    units = st.n_real * T  # node-steps per step on this rank
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    for _ in range(max(args.warmup, 3)):
+        st.step()
+    torch.cuda.synchronize()
+    L.check_device()
+
+    # ---- timed region: device-resident inputs
+    L.profile_read(L.BG_KID_BAND_FWD, reset=True)
+    for k in range(5):
+        L.profile_read(k, reset=True)
+    L.profile_enable(True)
+    launches0 = L.launch_count()
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with Clocks(local) as clk:
+        barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for _ in range(args.steps):
+            st.step()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+    L.profile_enable(False)
+    launches = L.launch_count() - launches0
+    ms = ev0.elapsed_time(ev1)
+    L.check_device()
+    kt = {k: L.profile_read(k, reset=True) for k in range(5)}
+    if dist is not None:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        u = torch.tensor([float(units)], device="cuda")
+        dist.all_reduce(u)
+        total_units = float(u.item())
+    else:
+        total_units = float(units)
+    ms_step = ms / args.steps
+    value = total_units / (ms_step / 1e3)
+
+    # ---- e2e: host buffers, H2D + pack + step + unpack + D2H inside the timed region
+    for _ in range(2):
+        st.step_e2e()
+    torch.cuda.synchronize()
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        bi, bo = st.step_e2e()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e_ms = e0.elapsed_time(e1) / args.steps
+    if dist is not None:
+        t = torch.tensor([e_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e_ms = float(t.item())
+    e2e_value = total_units / (e_ms / 1e3)
+
+    # ---- roofline of the dominant kernel (band contraction)
+    pk = _peaks()
+    fwd_ms, fwd_n = kt[L.BG_KID_BAND_FWD]
+    bwd_ms, bwd_n = kt[L.BG_KID_BAND_BWD]
+    f_band = st.plan.flops(H, L.BG_FLOPS_BAND)
+    f_xf = st.plan.flops(H, L.BG_FLOPS_XFORM)
+    # algorithmic FLOPs per launch: band-dense contraction + the fused edge-type transform
+    flops_fwd = f_band + f_xf
+    kern = "band_fwd" if fwd_ms >= bwd_ms else "band_bwd"
+    if kern == "band_fwd":
+        avg_ms = fwd_ms / max(fwd_n, 1)
+        flops = flops_fwd
+    else:
+        avg_ms = bwd_ms / max(bwd_n, 1)
+        flops = f_band + 2 * f_xf
+    achieved = flops / (avg_ms / 1e3) / 1e12 if avg_ms > 0 else 0.0
+    peak = pk["bf16_sustained"]
+    roof = {"kernel": kern, "bound": "tensor", "achieved": achieved, "peak": peak,
+            "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+            "peak_src": f"{pk['src']} bf16 sustained",
+            "kernel_ms": {k: (kt[i][0] / max(kt[i][1], 1)) for i, k in
+                          enumerate(["band_fwd", "band_bwd", "gru_fwd", "gru_bwd", "dW"])},
+            "nnz_tflops": st.plan.flops(H, L.BG_FLOPS_NNZ) / (avg_ms / 1e3) / 1e12
+            if avg_ms > 0 else 0.0}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "node-steps/s", "n_gpus": world,
+        "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": c["dtype"], "data": "synthetic program-shaped graphs (seeded)",
+        "config": {"workload": synth.CONFIGS[args.config]["name"], "graphs": len(graphs),
+                   "packed": st.info["n_packed"], "n_real": st.n_real, "n_pad": st.N,
+                   "K": st.info["K"], "S": c["S"], "P": c["P"], "H": H, "T": T,
+                   "kept_edges": st.info["n_kept"], "dropped_edges": st.info["n_dropped"],
+                   "plan_ms": st.plan_ms, "upload_ms": st.upload_ms,
+                   "l2": "per-step working set (band tiles + saved activations) > 129 MB L2",
+                   "parallelism": f"dp{world} (one supergraph per GPU)"},
+        "e2e": {"value": e2e_value, "unit": "node-steps/s", "h2d_bytes_per_step": bi,
+                "d2h_bytes_per_step": bo},
+        "gpu_launches": launches,
+        "roofline": roof,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, s = oracle_sample(args.config, c)
+        line["cpu_baseline"] = {"value": v, "unit": "node-steps/s", "cores": 1, "kind": "oracle",
+                                "sample": f"leading {s['graphs']} graphs ({s['nodes']} nodes) of "
+                                          f"the same workload, fwd+bwd, {s['seconds']:.1f}s "
+                                          "single-threaded fp64"}
+    if rank == 0:
+        print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

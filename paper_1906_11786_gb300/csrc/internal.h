@@ -1,0 +1,45 @@
+// Library-internal declarations shared by the planner (plan.cpp) and the device code (*.cu).
+#pragma once
+
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include "bandggnn.h"
+
+struct bg_plan {
+  // shape
+  int32_t K = 0, S = 0, P = 0, W32 = 0;  // W32 = S / 32 mask words per tile row
+  int32_t n_graphs = 0, n_packed = 0, n_real = 0;
+  int64_t n_edges_in = 0, n_unique = 0, n_kept = 0, n_dropped = 0;
+  int64_t bw_before_max = 0, bw_after_max = 0;
+  // per input graph
+  std::vector<int32_t> n_nodes;
+  std::vector<int64_t> node_base;  // prefix sums of n_nodes
+  std::vector<int32_t> perm;       // concatenated perm[new] = old
+  std::vector<int32_t> offset;     // -1 if not packed
+  std::vector<int64_t> bw_before, bw_after;
+  // per packed position / graph
+  std::vector<int32_t> gather;          // [n_real] row of the concatenated input
+  std::vector<int32_t> seg_off, seg_cnt;  // packed graphs
+  // band tiles as bit rows: [K][3][P][S][W32] words, bit c of word c/32 (LSB first)
+  std::vector<uint32_t> masks;   // row = target r in block k, bits = source c in block k+d-1
+  std::vector<uint32_t> masksT;  // row = source c in block j, bits = target i in block j+e-1
+  // device copies (valid once uploaded)
+  int device = -1;
+  uint32_t* d_masks = nullptr;
+  uint32_t* d_masksT = nullptr;
+  int32_t* d_gather = nullptr;
+  int32_t* d_seg_off = nullptr;
+  int32_t* d_seg_cnt = nullptr;
+  int32_t* d_row_graph = nullptr;  // [n_pad] packed graph of each position, -1 for padding
+  int32_t n_pad() const { return K * S; }
+};
+
+// error plumbing (api.cu)
+int bg_fail(int code, const std::string& msg);
+void bg_clear_error();
+
+// planner entry (plan.cpp)
+int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S, int32_t cap,
+                  uint32_t flags, bg_plan** out);

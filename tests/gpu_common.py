@@ -1,0 +1,79 @@
+"""Shared set-up of the GPU parity tests: seeded inputs, device copies, oracle references and the
+parity measure (max-abs error relative to the reference's max-abs value, per tensor)."""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+from paper_1906_11786_gb300 import _binding as L
+from paper_1906_11786_gb300 import build as B
+from paper_1906_11786_gb300 import synth
+
+TOL = {"f32": 1e-4, "bf16": 2e-2}
+
+
+def ensure_built():
+    B.build()
+    L.load()
+
+
+def rel_err(got, ref) -> float:
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    assert got.shape == ref.shape, (got.shape, ref.shape)
+    return float(np.max(np.abs(got - ref)) / max(float(np.max(np.abs(ref))), 1e-30))
+
+
+def quantize(x: np.ndarray, dtype: str) -> np.ndarray:
+    """Round to the device dtype and back to float64 (both sides then start from equal values)."""
+    if dtype == "bf16":
+        return torch.from_numpy(np.asarray(x, np.float32)).to(torch.bfloat16).double().numpy()
+    return np.asarray(x, np.float32).astype(np.float64)
+
+
+def to_dev(x: np.ndarray, dtype: str) -> torch.Tensor:
+    t = torch.from_numpy(np.ascontiguousarray(x, np.float32))
+    if dtype == "bf16":
+        t = t.to(torch.bfloat16)
+    return t.cuda()
+
+
+def f32_dev(x) -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(x, np.float32)).cuda()
+
+
+class Case:
+    """A planned, uploaded supergraph with packed device states and the oracle's view of it."""
+
+    def __init__(self, graphs, P, S, H, dtype, seed=0, cap=0):
+        self.P, self.S, self.H, self.dtype = P, S, H, dtype
+        self.plan = L.band_plan(graphs, P, S, cap)
+        self.plan.upload()
+        self.ref = oracle.layout(graphs, P, S, cap)
+        info = self.plan.info()
+        self.info = info
+        self.N = info["n_pad"]
+        self.n_real = info["n_real"]
+        n_all = sum(g.n_nodes for g in graphs)
+        E_orig = quantize(synth.gen_states(n_all, H, seed), dtype)
+        self.E_orig = E_orig
+        self.E_orig_dev = to_dev(E_orig, dtype)
+        self.E_band_dev = torch.empty((self.N, H), dtype=self.E_orig_dev.dtype, device="cuda")
+        L.pack_states(self.plan, dtype, H, self.E_orig_dev, self.E_band_dev)
+        gi = self.ref.gather_index()
+        self.E_band = np.zeros((self.N, H))
+        self.E_band[: self.n_real] = E_orig[gi]
+        prm = synth.gen_params(P, H, seed + 1)
+        for k in ("W", "W_ih", "W_hh"):
+            prm[k] = quantize(prm[k], dtype)
+        for k in ("b", "b_ih", "b_hh", "w_out"):
+            prm[k] = quantize(prm[k], "f32")
+        self.prm = prm
+        self.dprm = {k: (to_dev(v, dtype) if k in ("W", "W_ih", "W_hh") else f32_dev(v))
+                     for k, v in prm.items()}
+        self.edges = (self.ref.kept_dst, self.ref.kept_src, self.ref.kept_type)
+
+    def ws(self, op):
+        n = L.workspace_bytes(self.plan, self.dtype, self.H, op)
+        return torch.empty(n, dtype=torch.uint8, device="cuda")

@@ -1,0 +1,212 @@
+"""GPU parity: the CUDA path, called through the C ABI, against the CPU oracle on the same seeded
+inputs.  Tolerances (max-abs error over the reference's max-abs value, per tensor): 1e-4 for the
+fp32 path, 2e-2 for the bf16 path (bf16 states/weights, fp32 accumulation); layout work is
+bit-exact."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_1906_11786_gb300 import _binding as L
+from paper_1906_11786_gb300 import synth
+
+from gpu_common import TOL, Case, ensure_built, f32_dev, quantize, rel_err
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    ensure_built()
+    torch.manual_seed(0)
+
+
+def _fwd(c: Case, with_bias=True):
+    Y = torch.empty((c.N, c.H), dtype=torch.float32, device="cuda")
+    L.band_propagate_fwd(c.plan, c.dtype, c.H, c.E_band_dev, c.dprm["W"],
+                         c.dprm["b"] if with_bias else None, Y, c.ws(L.BG_OP_PROPAGATE_FWD))
+    torch.cuda.synchronize()
+    L.check_device()
+    ref = oracle.propagate_fwd(c.N, c.P, c.H, *c.edges, c.E_band, c.prm["W"],
+                               c.prm["b"] if with_bias else None)
+    return Y.cpu().numpy(), ref
+
+
+def _bwd(c: Case, seed=7):
+    dY = quantize(np.random.default_rng(seed).standard_normal((c.N, c.H)), "f32")
+    dY[c.n_real:] = 0
+    dE = torch.empty((c.N, c.H), dtype=torch.float32, device="cuda")
+    dW = torch.empty((c.P, c.H, c.H), dtype=torch.float32, device="cuda")
+    db = torch.empty((c.P, c.H), dtype=torch.float32, device="cuda")
+    L.band_propagate_bwd(c.plan, c.dtype, c.H, c.E_band_dev, c.dprm["W"], f32_dev(dY), dE, dW, db,
+                         c.ws(L.BG_OP_PROPAGATE_BWD))
+    torch.cuda.synchronize()
+    L.check_device()
+    ref = oracle.propagate_bwd(c.N, c.P, c.H, *c.edges, c.E_band, c.prm["W"], dY)
+    return (dE.cpu().numpy(), dW.cpu().numpy(), db.cpu().numpy()), ref
+
+
+# ------------------------------------------------------------------------------------ layout
+
+
+def test_pack_unpack_bit_exact():
+    c = Case(synth.config_graphs(2, scale=0.1), 20, 128, 64, "bf16", seed=3)
+    got = c.E_band_dev.float().cpu().numpy()
+    np.testing.assert_array_equal(got, c.E_band)
+    back = torch.zeros_like(c.E_orig_dev)
+    L.unpack_states(c.plan, c.dtype, c.H, c.E_band_dev, back)
+    np.testing.assert_array_equal(back.float().cpu().numpy(), c.E_orig)
+
+
+# ------------------------------------------------------------------------------------ propagate
+
+
+def test_propagate_fp32_config1():
+    """Single 512-node graph, 4 types, S = 64, H = 64, fp32, fwd + bwd."""
+    c = Case(synth.config_graphs(1), 4, 64, 64, "f32", seed=11)
+    Y, ref = _fwd(c)
+    assert rel_err(Y, ref) < TOL["f32"]
+    got, ref = _bwd(c)
+    for g, r, name in zip(got, ref, ("dE", "dW", "db")):
+        assert rel_err(g, r) < TOL["f32"], name
+
+
+@pytest.mark.parametrize("S,H", [(128, 64), (64, 64), (32, 32), (256, 128), (128, 256)])
+def test_propagate_bf16_packed_batch(S, H):
+    """Several graphs packed into several block-rows with a ragged tail."""
+    gs = synth.gen_batch(7, 60, 400, 10, True, S // 2, S // 3, 2.0, 100 + S + H)
+    c = Case(gs, 20, S, H, "bf16", seed=S + H)
+    assert c.info["K"] >= 3 and c.n_real % S != 0
+    Y, ref = _fwd(c)
+    assert rel_err(Y, ref) < TOL["bf16"]
+    assert np.all(Y[c.n_real:] == 0)
+    got, ref = _bwd(c)
+    for g, r, name in zip(got, ref, ("dE", "dW", "db")):
+        assert rel_err(g, r) < TOL["bf16"], name
+
+
+def test_propagate_bf16_no_bias_and_single_block():
+    g = synth.gen_graph(100, 4, True, 20, 10, 1.0, 5)
+    c = Case([g], 8, 128, 64, "bf16", seed=2)
+    assert c.info["K"] == 1
+    Y, ref = _fwd(c, with_bias=False)
+    assert rel_err(Y, ref) < TOL["bf16"]
+
+
+def test_propagate_graph_without_edges():
+    g = synth.Graph(70, np.zeros(0, np.int32), np.zeros(0, np.int32), np.zeros(0, np.int32), 2)
+    c = Case([g], 2, 32, 32, "f32")
+    Y, ref = _fwd(c)
+    assert np.all(Y == 0) and np.all(ref == 0)
+
+
+def test_propagate_bf16_dropped_edges_config3_shape():
+    """Wide band: S = 256 < bandwidth, so some edges are dropped (coverage rule)."""
+    g = synth.gen_graph(3000, 10, True, 200, 133, 3.0, 17)
+    c = Case([g], 20, 256, 128, "bf16", seed=5)
+    Y, ref = _fwd(c)
+    assert rel_err(Y, ref) < TOL["bf16"]
+
+
+# ------------------------------------------------------------------------------------ GGNN
+
+
+def _ggnn(c: Case, T, seed=3):
+    saved = torch.empty(L.ggnn_saved_bytes(c.plan, c.dtype, c.H, T), dtype=torch.uint8,
+                        device="cuda")
+    ET = torch.empty_like(c.E_band_dev)
+    L.ggnn_step(c.plan, c.dtype, c.H, T, c.dprm, c.E_band_dev, ET, saved, c.ws(L.BG_OP_GGNN_FWD))
+    dET = quantize(np.random.default_rng(seed).standard_normal((c.N, c.H)), "f32")
+    dE0 = torch.empty((c.N, c.H), dtype=torch.float32, device="cuda")
+    grads = dict(dW=torch.empty((c.P, c.H, c.H), device="cuda"),
+                 db=torch.empty((c.P, c.H), device="cuda"),
+                 dW_ih=torch.empty((3 * c.H, c.H), device="cuda"),
+                 dW_hh=torch.empty((3 * c.H, c.H), device="cuda"),
+                 db_ih=torch.empty(3 * c.H, device="cuda"),
+                 db_hh=torch.empty(3 * c.H, device="cuda"))
+    L.ggnn_step_bwd(c.plan, c.dtype, c.H, T, c.dprm, saved, f32_dev(dET), dE0, grads,
+                    c.ws(L.BG_OP_GGNN_BWD))
+    torch.cuda.synchronize()
+    L.check_device()
+    Es, Ys = oracle.ggnn_fwd(c.N, c.P, c.H, T, c.n_real, *c.edges, c.E_band, c.prm)
+    ref = oracle.ggnn_bwd(c.N, c.P, c.H, T, c.n_real, *c.edges, c.prm, Es, Ys, dET)
+    return ET.float().cpu().numpy(), Es[T], {k: v.cpu().numpy() for k, v in grads.items()}, \
+        dE0.cpu().numpy(), ref
+
+
+@pytest.mark.parametrize("dtype,T", [("f32", 2), ("bf16", 3)])
+def test_ggnn_fwd_bwd(dtype, T):
+    gs = synth.gen_batch(5, 60, 300, 10, True, 48, 32, 2.0, 41)
+    c = Case(gs, 20, 64, 64, dtype, seed=9)
+    ET, ref_ET, grads, dE0, ref = _ggnn(c, T)
+    tol = TOL[dtype]
+    assert rel_err(ET, ref_ET) < tol
+    assert np.all(ET[c.n_real:] == 0)
+    assert rel_err(dE0, ref["dE0"]) < tol
+    for k, v in grads.items():
+        assert rel_err(v, ref[k]) < tol, k
+
+
+def test_ggnn_config2_shape_T8_reduced_batch():
+    """Config-2 shapes (P = 20, S = 128, H = 64, bf16, T = 8) on an 8-graph batch."""
+    c = Case(synth.config_graphs(2, scale=0.125), 20, 128, 64, "bf16", seed=2)
+    ET, ref_ET, grads, dE0, ref = _ggnn(c, 8)
+    assert rel_err(ET, ref_ET) < TOL["bf16"]
+    assert rel_err(dE0, ref["dE0"]) < TOL["bf16"]
+    for k, v in grads.items():
+        assert rel_err(v, ref[k]) < TOL["bf16"], k
+
+
+# ------------------------------------------------------------------------------------ readout, Adam
+
+
+def test_readout_loss_and_adam():
+    c = Case(synth.gen_batch(6, 50, 200, 3, True, 20, 10, 1.0, 8), 6, 64, 64, "bf16", seed=4)
+    n_g = c.info["n_packed"]
+    target = np.random.default_rng(1).standard_normal(n_g)
+    loss = torch.zeros(4, device="cuda")
+    dET = torch.empty((c.N, c.H), device="cuda")
+    dw = torch.empty(c.H, device="cuda")
+    L.readout_loss(c.plan, c.dtype, c.H, c.E_band_dev, c.dprm["w_out"], f32_dev(target), loss, dET,
+                   dw, c.ws(L.BG_OP_READOUT))
+    torch.cuda.synchronize()
+    off, cnt = c.ref.graph_segments()
+    rl, rdE, rdw = oracle.readout_loss(c.E_band, off, cnt, c.prm["w_out"], target)
+    assert abs(loss[0].item() - rl) / abs(rl) < 1e-4
+    assert rel_err(dET.cpu().numpy(), rdE) < 1e-4
+    assert rel_err(dw.cpu().numpy(), rdw) < 1e-4
+    # Adam on the edge weights: fp32 master, bf16 working copy
+    rng = np.random.default_rng(2)
+    p0 = rng.standard_normal(1000); g = rng.standard_normal(1000)
+    master = f32_dev(p0); work = master.to(torch.bfloat16)
+    m = torch.zeros_like(master); v = torch.zeros_like(master)
+    rp, rm, rv = p0, np.zeros(1000), np.zeros(1000)
+    for t in (1, 2):
+        L.adam_step(master, work, m, v, f32_dev(g), 1e-3, 0.9, 0.999, 1e-8, t)
+        rp, rm, rv = oracle.adam(rp, rm, rv, quantize(g, "f32"), 1e-3, 0.9, 0.999, 1e-8, t)
+    torch.cuda.synchronize()
+    assert rel_err(master.cpu().numpy(), rp) < 1e-5
+    assert rel_err(work.float().cpu().numpy(), rp) < 1e-2
+
+
+# ------------------------------------------------------------------------------------ full size
+
+
+def test_full_size_config2_propagate_sampled_rows():
+    """Config 2 at full size (64 graphs, ~72k nodes, P = 20, S = 128, H = 64, bf16): one forward
+    and backward propagation in the benchmark's launch configuration; the oracle computes a
+    seeded sample of output rows one by one (edges into sampled rows for Y; edges out of sampled
+    rows for dE) plus the exact dW and db."""
+    c = Case(synth.config_graphs(2), 20, 128, 64, "bf16", seed=21)
+    Y = torch.empty((c.N, c.H), dtype=torch.float32, device="cuda")
+    L.band_propagate_fwd(c.plan, c.dtype, c.H, c.E_band_dev, c.dprm["W"], c.dprm["b"], Y,
+                         c.ws(L.BG_OP_PROPAGATE_FWD))
+    torch.cuda.synchronize()
+    rows = np.unique(np.concatenate([np.random.default_rng(0).integers(0, c.n_real, 400),
+                                     [0, c.n_real - 1, c.N - 1]]))
+    d, s, t = c.edges
+    sel = np.isin(d, rows)
+    ref = oracle.propagate_fwd(c.N, c.P, c.H, d[sel], s[sel], t[sel], c.E_band, c.prm["W"],
+                               c.prm["b"])
+    assert rel_err(Y.cpu().numpy()[rows], ref[rows]) < TOL["bf16"]
+    L.check_device()

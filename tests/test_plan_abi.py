@@ -1,0 +1,143 @@
+"""The C-ABI library on the CPU: it loads, exports every declared symbol, and its host planner
+(RCM, packing, band tiles) is bit-exact against the oracle's independent implementation."""
+import ctypes
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_1906_11786_gb300 import _binding as L
+from paper_1906_11786_gb300 import build as B
+from paper_1906_11786_gb300 import synth
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    B.build()
+    L.load()
+
+
+def test_every_declared_symbol_is_exported():
+    lib = ctypes.CDLL(L.LIB_PATH)
+    names = L.declared_symbols()
+    assert len(names) >= 20
+    missing = [n for n in names if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def _compare(graphs, P, S, cap=0, flags=L.BG_RCM | L.BG_KEEP_IF_BETTER):
+    plan = L.band_plan(graphs, P, S, cap, flags)
+    ref = oracle.layout(graphs, P, S, cap, flags=flags)
+    info = plan.info()
+    assert info["K"] == ref.K and info["n_pad"] == ref.K * S
+    assert info["n_packed"] == ref.n_packed and info["n_real"] == ref.n_real
+    assert info["n_edges_unique"] == ref.n_unique
+    assert info["n_kept"] == ref.n_kept and info["n_dropped"] == ref.n_dropped
+    assert info["bw_before_max"] == ref.bw_before_max and info["bw_after_max"] == ref.bw_after_max
+    np.testing.assert_array_equal(plan.export(L.BG_EXPORT_PERM), ref.perm)
+    np.testing.assert_array_equal(plan.export(L.BG_EXPORT_OFFSETS), ref.offset)
+    bw = plan.export(L.BG_EXPORT_BW)
+    np.testing.assert_array_equal(bw[0], ref.bw_before)
+    np.testing.assert_array_equal(bw[1], ref.bw_after)
+    masks = plan.export(L.BG_EXPORT_MASKS)
+    assert masks.tobytes() == ref.masks.tobytes()
+    # transposed orientation: (j, e, p, c, i) set  <=>  forward (j+e-1, 2-e, p, i, c) set;
+    # checked on every block-row of small plans and on a seeded sample of block-rows otherwise
+    K = ref.K
+    mT = plan.export(L.BG_EXPORT_MASKS_T)
+    rows = range(K) if K * P * S * S <= 4_000_000 else \
+        sorted(set(np.random.default_rng(0).integers(0, K, 12).tolist()) | {0, K - 1})
+    for j in rows:
+        tb = np.unpackbits(mT[j], axis=-1, bitorder="little")            # [3,P,S,S]
+        for e in range(3):
+            k = j + e - 1
+            if 0 <= k < K:
+                fb = np.unpackbits(ref.masks[k, 2 - e], axis=-1, bitorder="little")
+                np.testing.assert_array_equal(tb[e], fb.transpose(0, 2, 1))
+            else:
+                assert not tb[e].any()
+    np.testing.assert_array_equal(plan.export(L.BG_EXPORT_GATHER), ref.gather_index())
+    return plan, ref
+
+
+def test_planner_bit_exact_config1():
+    _compare(synth.config_graphs(1), 4, 64)
+
+
+def test_planner_bit_exact_packed_batch_config2():
+    _compare(synth.config_graphs(2), 20, 128)
+
+
+def test_planner_bit_exact_single_large_config3():
+    _compare(synth.config_graphs(3), 20, 256)
+
+
+@pytest.mark.parametrize("S", [32, 64, 128, 256, 512])
+def test_planner_bit_exact_sweep_config4_capacity(S):
+    gs = synth.config_graphs(4, S=S, scale=0.25)
+    cap = max(1, (sum(g.n_nodes for g in gs) - 300) // S)  # the last graphs do not fit
+    plan, ref = _compare(gs, 20, S, cap)
+    assert ref.n_packed < len(gs)
+
+
+def test_planner_without_rcm_and_without_keep():
+    gs = synth.gen_batch(5, 40, 90, 3, True, 12, 8, 1.0, 3)
+    _compare(gs, 6, 32, flags=0)
+    _compare(gs, 6, 32, flags=L.BG_RCM)
+
+
+def test_planner_tiny_golden_rcm():
+    import json
+    import os
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "rcm_tiny.json")))
+    for c in g["cases"]:
+        e = np.array(c["edges"], np.int32)
+        gr = synth.Graph(c["n"], e[:, 0].copy(), e[:, 1].copy(), np.zeros(len(e), np.int32), 1)
+        plan = L.band_plan([gr], 1, 32)
+        assert plan.export(L.BG_EXPORT_PERM).tolist() == c["perm"], c["name"]
+
+
+def test_flop_counts():
+    plan = L.band_plan(synth.config_graphs(1), 4, 64)
+    i = plan.info()
+    K, S, P, H = i["K"], 64, 4, 64
+    assert plan.flops(H, L.BG_FLOPS_BAND) == 2 * (3 * K - 2) * P * S * S * H
+    assert plan.flops(H, L.BG_FLOPS_XFORM) == 2 * K * S * P * H * H
+    assert plan.flops(H, L.BG_FLOPS_NNZ) == 2 * H * i["n_kept"]
+
+
+@pytest.mark.parametrize("bad", ["id", "type", "S", "P", "capacity"])
+def test_invalid_inputs_return_einval_or_ecapacity(bad):
+    g = synth.gen_graph(50, 2, False, 5, 4, 1.0, 1)
+    P, S, cap = 2, 32, 0
+    if bad == "id":
+        g.dst = g.dst.copy(); g.dst[3] = 50
+    elif bad == "type":
+        g.etype = g.etype.copy(); g.etype[0] = 2
+    elif bad == "S":
+        S = 48
+    elif bad == "P":
+        P = 0
+    elif bad == "capacity":
+        cap = 1
+    with pytest.raises(L.BandGGNNError) as ei:
+        L.band_plan([g], P, S, cap)
+    assert ei.value.code == (-2 if bad == "capacity" else -1)
+    assert L.load().bg_last_error().decode()
+
+
+def test_device_calls_require_upload():
+    import torch
+    plan = L.band_plan(synth.config_graphs(1), 4, 64)
+    x = torch.zeros(16)
+    # a plan that was never uploaded is rejected before any CUDA call
+    rc = L.load().bg_band_propagate_fwd(plan.handle, 0, 64, x.data_ptr(), x.data_ptr(), None,
+                                        x.data_ptr(), x.data_ptr(), 64, None)
+    assert rc == -7
+
+
+def test_workspace_and_saved_sizes_are_positive():
+    plan = L.band_plan(synth.config_graphs(1), 4, 64)
+    for op in range(5):
+        assert L.workspace_bytes(plan, "f32", 64, op) > 0
+    assert L.ggnn_saved_bytes(plan, "bf16", 64, 8) >= 9 * 512 * 64 * 2 + 8 * 512 * 64 * 4
