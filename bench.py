@@ -156,7 +156,8 @@ class OursStep:
         self.E_orig_dev = E.cuda()
         self.E0 = torch.empty((N, H), dtype=tdt, device="cuda")
         L.pack_states(self.plan, self.dt, H, self.E_orig_dev, self.E0)
-        prm = synth.gen_params(P, H, seed + 1)
+        prm = synth.gen_params(P, H, seed + 1,
+                               mean_in_degree=self.info["n_kept"] / max(n_real, 1))
         self.prm = {}
         for k, v in prm.items():
             t = torch.from_numpy(np.asarray(v, np.float32))
@@ -257,7 +258,6 @@ def oracle_sample(config: int, c, budget_s: float = 15.0):
     P, S, H, T = c["P"], c["S"], c["H"], c["T"]
     done_nodes, spent, used = 0, 0.0, 0
     rng = np.random.default_rng(0)
-    prm = synth.gen_params(P, H, 1)
     t_start = time.perf_counter()
     for g in graphs:
         t0 = time.perf_counter()
@@ -265,6 +265,7 @@ def oracle_sample(config: int, c, budget_s: float = 15.0):
         N = lay.n_pad
         E0 = np.zeros((N, H)); E0[: lay.n_real] = rng.standard_normal((lay.n_real, H))
         e = (lay.kept_dst, lay.kept_src, lay.kept_type)
+        prm = synth.gen_params(P, H, 1, mean_in_degree=lay.n_kept / max(lay.n_real, 1))
         if c["gru"]:
             Es, Ys = oracle.ggnn_fwd(N, P, H, T, lay.n_real, *e, E0, prm)
             oracle.ggnn_bwd(N, P, H, T, lay.n_real, *e, prm, Es, Ys, rng.standard_normal((N, H)))

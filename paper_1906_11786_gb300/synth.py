@@ -175,13 +175,18 @@ def _xavier(rng, shape, fan_in, fan_out):
     return rng.uniform(-a, a, size=shape)
 
 
-def gen_params(P: int, H: int, seed: int, bias_scale: float = 0.1) -> dict:
+def gen_params(P: int, H: int, seed: int, bias_scale: float = 0.1,
+               mean_in_degree: float = 1.0) -> dict:
     """Edge-type transforms W [P, H, H] (message = state @ W[p]), per-type bias b [P, H],
     GRU weights W_ih, W_hh [3H, H] (gate rows r, z, n) and biases b_ih, b_hh [3H], readout
-    w_out [H].  Weights Xavier-uniform, biases uniform in +-bias_scale.  All float64."""
+    w_out [H].  Weights Xavier-uniform, biases uniform in +-bias_scale.  All float64.
+
+    Incoming messages are summed (Appendix D), so the message layer's fan-in is H times the mean
+    in-degree: W's Xavier bound uses fan_in = H * mean_in_degree (1.0 gives the plain H x H
+    bound)."""
     rng = np.random.default_rng(seed)
     return {
-        "W": _xavier(rng, (P, H, H), H, H),
+        "W": _xavier(rng, (P, H, H), H * max(mean_in_degree, 1.0), H),
         "b": rng.uniform(-bias_scale, bias_scale, size=(P, H)),
         "W_ih": _xavier(rng, (3 * H, H), H, 3 * H),
         "W_hh": _xavier(rng, (3 * H, H), H, 3 * H),

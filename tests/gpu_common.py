@@ -64,7 +64,8 @@ class Case:
         gi = self.ref.gather_index()
         self.E_band = np.zeros((self.N, H))
         self.E_band[: self.n_real] = E_orig[gi]
-        prm = synth.gen_params(P, H, seed + 1)
+        prm = synth.gen_params(P, H, seed + 1,
+                               mean_in_degree=self.ref.n_kept / max(self.ref.n_real, 1))
         for k in ("W", "W_ih", "W_hh"):
             prm[k] = quantize(prm[k], dtype)
         for k in ("b", "b_ih", "b_hh", "w_out"):
