@@ -442,6 +442,8 @@ def main():
                    "K": st.info["K"], "S": c["S"], "P": c["P"], "H": H, "T": T,
                    "kept_edges": st.info["n_kept"], "dropped_edges": st.info["n_dropped"],
                    "plan_ms": st.plan_ms, "upload_ms": st.upload_ms,
+                   "band_kernels": "tcgen05" if L.band_uses_tensor_cores(st.plan, c["dtype"], H)
+                   else "simt",
                    "l2": "per-step working set (band tiles + saved activations) > 129 MB L2",
                    "parallelism": f"dp{world} (one supergraph per GPU)"},
         "e2e": {"value": e2e_value, "unit": "node-steps/s", "h2d_bytes_per_step": bi,

@@ -233,6 +233,10 @@ int bg_profile_enable(int32_t on);
 int bg_profile_read(int32_t kid, double* ms_total, int64_t* launches, int32_t reset);
 /* Number of kernels this library has launched since load (all kinds). */
 int64_t bg_launch_count(void);
+/* 1 when band propagation for (plan, dtype, H) runs on the fused tcgen05 tensor-core kernels,
+ * 0 when it runs on the SIMT kernels (fp32 path and shapes the tensor-core kernels do not cover:
+ * S != 128, H not in {64, 128}, P > 32); negative status on error.  The plan must be uploaded. */
+int bg_band_uses_tensor_cores(const bg_plan* plan, bg_dtype dtype, int32_t H);
 
 #ifdef __cplusplus
 }

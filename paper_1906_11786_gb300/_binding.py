@@ -94,6 +94,7 @@ def load(path: str = LIB_PATH):
         "bg_profile_enable": (c.c_int, [i32]),
         "bg_profile_read": (c.c_int, [i32, vp, vp, i32]),
         "bg_launch_count": (i64, []),
+        "bg_band_uses_tensor_cores": (c.c_int, [vp, c.c_int, i32]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -315,6 +316,13 @@ def profile_read(kid, reset=False):
     n = ctypes.c_int64()
     _check(load().bg_profile_read(kid, ctypes.byref(ms), ctypes.byref(n), 1 if reset else 0))
     return ms.value, n.value
+
+
+def band_uses_tensor_cores(plan, dtype, H) -> bool:
+    rc = load().bg_band_uses_tensor_cores(plan.handle, dtype_code(dtype), H)
+    if rc < 0:
+        _check(rc)
+    return rc == 1
 
 
 def launch_count() -> int:

@@ -265,6 +265,10 @@ extern "C" int bg_plan_upload(bg_plan* p, void* stream) {
   }
   // host vectors must outlive the async copies
   BG_CUDA(cudaStreamSynchronize(st));
+  if (bg::band_tc_upload(p, st) != 0) {
+    free_device(p);
+    return bg_fail(BG_ENOMEM, "device allocation for the band tiles failed");
+  }
   return BG_OK;
 }
 
@@ -394,6 +398,13 @@ extern "C" size_t bg_workspace_bytes(const bg_plan* p, bg_dtype dt, int32_t H, i
 extern "C" size_t bg_ggnn_saved_bytes(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T) {
   if (!p || H <= 0 || T < 0) return 0;
   return saved_Y_off(p, dt, H, T, T);
+}
+
+extern "C" int bg_band_uses_tensor_cores(const bg_plan* p, bg_dtype dt, int32_t H) {
+  bg_clear_error();
+  BG_TRY(check_plan_dev(p));
+  BG_TRY(check_shape(p, dt, H));
+  return bg::band_tc_supported(p, (int)dt, H) ? 1 : 0;
 }
 
 // ---------------------------------------------------------------------------------- pack

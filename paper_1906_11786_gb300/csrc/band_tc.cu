@@ -1,16 +1,645 @@
+// Fused band contraction on the 5th-generation tensor cores (tcgen05, TMEM, TMA) for sm_103a.
+//
+// Forward (Algorithm 1's aggregate-first order, Eq. 3): for a 128-row tile of block-row k and
+// every edge type p,
+//     pre_p = sum_{d in -1,0,+1} A_{k,d,p} E_{k+d}        (128 x 3S  times  3S x H, fp32 in TMEM)
+//     Y_k  += bf16(pre_p) W_p                               (chained MMA, A operand read from TMEM)
+// and the per-type bias enters as one more product deg_k [128 x 2P] x [b_hi; b_lo] with exact
+// integer in-degrees and b split into two bf16 halves.  pre_p never leaves the SM.
+// Backward (transposed band): the same kernel with the transposed tiles, dY instead of E and W_p
+// instead of W_p^T gives dE_j += sum_p (A^T dY)_p W_p^T; dM_p = A_p^T dY is also written (bf16,
+// transposed) for the weight gradient.
+//
+// The 0/1 adjacency is the MMA's A operand.  It is stored as bits (the whole band costs
+// 3 P S^2 / 8 bytes per block-row) and expanded on chip straight into tensor memory: the bits of
+// each 32-column word are interleaved at upload (column 2j at bit j, column 2j+1 at bit 16+j) so
+// that one AND and one multiply give the packed bf16 pair {1.0 or 0, 1.0 or 0}.
+//
+// Roles (384 threads, one CTA per SM, persistent over tiles):
+//   warp 0      TMA producer: state blocks (B operand of the band product), W tiles, deg, bias
+//   warp 1      TMEM allocator; lane 0 issues every tcgen05.mma
+//   warps 4-7   expanders: thread r turns row r's mask bits into bf16 A tiles in TMEM
+//   warps 8-11  converters: pre_p fp32 -> bf16 in place; final epilogue TMEM -> global
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+
+#include <cstring>
+#include <mutex>
+#include <vector>
+
 #include "band_tc.h"
+#include "gemm_tc.h"
+#include "kernels.h"
+#include "tc_util.cuh"
 
 namespace bg {
-bool band_tc_supported(const bg_plan*, int, int) { return false; }
-size_t band_tc_fwd_ws_bytes(const bg_plan*, int, int) { return 0; }
-size_t band_tc_bwd_ws_bytes(const bg_plan*, int, int) { return 0; }
-cudaError_t band_tc_fwd(const bg_plan*, int, const void*, const void*, const float*, float*, char*,
-                        size_t, int*, cudaStream_t) {
-  return cudaErrorNotSupported;
+
+using namespace tc;
+
+namespace {
+
+constexpr int kTile = 128;     // rows per tile = UMMA M
+constexpr int kThreads = 384;
+constexpr int kAtom = 64;      // bf16 per 128-byte swizzle row
+
+template <int H>
+struct Cfg {
+  static constexpr int NXB = H <= 64 ? 2 : 1;                 // state-window buffers
+  static constexpr int NW = H <= 64 ? 4 : 2;                  // W ring stages
+  static constexpr int ATOM_X = H * 128;                      // 64 nodes x H rows
+  static constexpr int XWIN = 6 * ATOM_X;                     // 3 blocks x 2 atoms (S = 128)
+  static constexpr int WSTAGE = (H / kAtom) * H * 128;        // H x H bf16
+  static constexpr int DEG = kTile * 128;                     // 128 rows x 64 bf16
+  static constexpr int B2 = H * 128;                          // H rows x 64 bf16
+  static constexpr int OFF_X = 0;
+  static constexpr int OFF_W = OFF_X + NXB * XWIN;
+  static constexpr int OFF_DEG = OFF_W + NW * WSTAGE;
+  static constexpr int OFF_B2 = OFF_DEG + 2 * DEG;
+  static constexpr int OFF_BAR = OFF_B2 + B2;
+  static constexpr int SMEM = OFF_BAR + 1024 + 1024;          // barriers + 1 KB alignment slack
+  // TMEM columns
+  static constexpr int YCOL = 0;
+  static constexpr int D1COL0 = H;
+  static constexpr int ACOL = 3 * H;
+  static constexpr int NA = (512 - 3 * H) / 64;
+};
+
+struct Bars {
+  uint64_t x_full[2], x_empty[2];
+  uint64_t w_full[4], w_empty[4];
+  uint64_t deg_full[2], deg_empty[2];
+  uint64_t b2_full;
+  uint64_t a_full[8], a_empty[8];
+  uint64_t d1_full[2], pre_ready[2];
+  uint64_t y_full, y_empty;
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__device__ __forceinline__ uint32_t expand_pair(uint32_t w, int j) {
+  // w holds column 2j at bit j and column 2j+1 at bit 16+j (j < 8); result packs bf16 1.0/0.0
+  return (w & (0x00010001u << j)) * (0x3F80u >> j);
 }
-cudaError_t band_tc_bwd(const bg_plan*, int, const void*, const void*, const float*, float*,
-                        float*, float*, int, char*, size_t, int*, cudaStream_t) {
-  return cudaErrorNotSupported;
+
+// Expands one interleaved 32-bit mask word into 16 packed bf16 pairs.
+__device__ __forceinline__ void expand_word(uint32_t w, uint32_t* out) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j) out[j] = expand_pair(w, j);
+  const uint32_t w8 = w >> 8;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) out[8 + j] = expand_pair(w8, j);
 }
-void band_tc_release(bg_plan*) {}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+template <int H, bool BWD>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_band_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
+              const __grid_constant__ CUtensorMap tm_deg, const __grid_constant__ CUtensorMap tm_b2,
+              const uint32_t* __restrict__ maskI, float* __restrict__ out,
+              __nv_bfloat16* __restrict__ dMT, int K, int P, int n_pad, int has_bias,
+              int accumulate, int* status) {
+  using C = Cfg<H>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  Bars* bars = reinterpret_cast<Bars*>(smem + C::OFF_BAR);
+  uint8_t* xwin = smem + C::OFF_X;
+  uint8_t* wring = smem + C::OFF_W;
+  uint8_t* degs = smem + C::OFF_DEG;
+  uint8_t* b2s = smem + C::OFF_B2;
+  volatile int* abort = &bars->abort;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bars->x_full[i], 1); mbar_init(&bars->x_empty[i], 1);
+      mbar_init(&bars->deg_full[i], 1); mbar_init(&bars->deg_empty[i], 1);
+      mbar_init(&bars->d1_full[i], 1); mbar_init(&bars->pre_ready[i], kTile);
+    }
+    for (int i = 0; i < 4; ++i) { mbar_init(&bars->w_full[i], 1); mbar_init(&bars->w_empty[i], 1); }
+    for (int i = 0; i < 8; ++i) { mbar_init(&bars->a_full[i], kTile); mbar_init(&bars->a_empty[i], 1); }
+    mbar_init(&bars->b2_full, 1);
+    mbar_init(&bars->y_full, 1);
+    mbar_init(&bars->y_empty, kTile);
+    mbar_init(&bars->drain, 1);
+    bars->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&bars->tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem_base;
+  const int n_tiles = K;  // S = 128: one tile per block-row
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------------------ TMA producer
+    tma_prefetch_desc(&tm_x);
+    tma_prefetch_desc(&tm_w);
+    if (has_bias) {
+      tma_prefetch_desc(&tm_deg);
+      mbar_expect_tx(&bars->b2_full, C::B2);
+      tma_load_2d(b2s, &tm_b2, &bars->b2_full, 0, 0);
+    }
+    uint32_t widx = 0;
+    uint32_t n_x[2] = {0, 0}, n_deg[2] = {0, 0}, n_w[4] = {0, 0, 0, 0};
+    int i = 0;
+    for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x, ++i) {
+      const int xb = i % C::NXB;
+      if (!mbar_wait(&bars->x_empty[xb], ((i / C::NXB) & 1) ^ 1, status, 101, abort)) break;
+      ++n_x[xb];
+      uint32_t bytes = 0;
+      for (int d = 0; d < 3; ++d) {
+        const int kb = k + d - 1;
+        if (kb >= 0 && kb < K) bytes += 2 * C::ATOM_X;
+      }
+      mbar_expect_tx(&bars->x_full[xb], bytes);
+      for (int d = 0; d < 3; ++d) {
+        const int kb = k + d - 1;
+        if (kb < 0 || kb >= K) continue;
+        for (int a = 0; a < 2; ++a)
+          tma_load_2d(xwin + xb * C::XWIN + (d * 2 + a) * C::ATOM_X, &tm_x, &bars->x_full[xb],
+                      kb * kTile + a * kAtom, 0);
+      }
+      if (has_bias) {
+        const int db = i & 1;
+        if (!mbar_wait(&bars->deg_empty[db], ((i >> 1) & 1) ^ 1, status, 102, abort)) break;
+        ++n_deg[db];
+        mbar_expect_tx(&bars->deg_full[db], C::DEG);
+        tma_load_2d(degs + db * C::DEG, &tm_deg, &bars->deg_full[db], 0, k * kTile);
+      }
+      for (int p = 0; p < P; ++p, ++widx) {
+        const int ws = widx % C::NW;
+        if (!mbar_wait(&bars->w_empty[ws], ((widx / C::NW) & 1) ^ 1, status, 103, abort)) break;
+        ++n_w[ws];
+        mbar_expect_tx(&bars->w_full[ws], C::WSTAGE);
+        for (int a = 0; a < H / kAtom; ++a)
+          tma_load_2d(wring + ws * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws], a * kAtom,
+                      p * H);
+      }
+    }
+    if (*abort) {
+      // let this CTA's own copies land before shared memory is released (bounded)
+      auto settle = [](uint64_t* bar, uint32_t uses) {
+        if (!uses) return;
+        for (uint32_t t = 0; t < (1u << 22) && !mbar_try(bar, (uses - 1) & 1); ++t) {
+        }
+      };
+      for (int q = 0; q < 2; ++q) { settle(&bars->x_full[q], n_x[q]); settle(&bars->deg_full[q], n_deg[q]); }
+      for (int q = 0; q < 4; ++q) settle(&bars->w_full[q], n_w[q]);
+      if (has_bias) settle(&bars->b2_full, 1);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------------------------ MMA issuer
+    constexpr uint32_t idesc = idesc_bf16_f32(kTile, H);
+    uint32_t c = 0, aidx = 0, widx = 0;
+    bool ok = true;
+    int i = 0;
+    auto stage2 = [&](uint32_t cc, bool first_in_tile, int tile_i) -> bool {
+      const int b = cc & 1;
+      if (!mbar_wait(&bars->pre_ready[b], (cc >> 1) & 1, status, 201, abort)) return false;
+      const int ws = widx % C::NW;
+      if (!mbar_wait(&bars->w_full[ws], (widx / C::NW) & 1, status, 202, abort)) return false;
+      if (first_in_tile &&
+          !mbar_wait(&bars->y_empty, (tile_i & 1) ^ 1, status, 203, abort))
+        return false;
+      tc_fence_after();
+      const uint32_t wbase = smem_u32(wring + ws * C::WSTAGE);
+#pragma unroll
+      for (int kk = 0; kk < H / 16; ++kk) {
+        const uint64_t bdesc = desc_sw128_kmajor(wbase + (kk / 4) * H * 128 + (kk % 4) * 32);
+        mma_ts(tmem + C::YCOL, tmem + C::D1COL0 + b * H + kk * 8, bdesc, idesc,
+               (first_in_tile && kk == 0) ? 0u : 1u);
+      }
+      tc_commit(&bars->w_empty[ws]);
+      ++widx;
+      return true;
+    };
+    for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x, ++i) {
+      const int xb = i % C::NXB;
+      if (!mbar_wait(&bars->x_full[xb], (i / C::NXB) & 1, status, 204, abort)) break;
+      tc_fence_after();
+      const uint32_t xbase = smem_u32(xwin + xb * C::XWIN);
+      for (int p = 0; p < P && ok; ++p, ++c) {
+        const int b = c & 1;
+        uint32_t first = 1;
+        for (int d = 0; d < 3; ++d) {
+          const int kb = k + d - 1;
+          if (kb < 0 || kb >= K) continue;
+          const int slot = aidx % C::NA;
+          if (!mbar_wait(&bars->a_full[slot], (aidx / C::NA) & 1, status, 205, abort)) { ok = false; break; }
+          tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < kTile / 16; ++kk) {
+            const uint64_t bdesc =
+                desc_sw128_kmajor(xbase + (d * 2 + kk / 4) * C::ATOM_X + (kk % 4) * 32);
+            mma_ts(tmem + C::D1COL0 + b * H, tmem + C::ACOL + slot * 64 + kk * 8, bdesc, idesc,
+                   (first && kk == 0) ? 0u : 1u);
+          }
+          first = 0;
+          tc_commit(&bars->a_empty[slot]);
+          ++aidx;
+        }
+        if (!ok) break;
+        tc_commit(&bars->d1_full[b]);
+        if (p == P - 1) tc_commit(&bars->x_empty[xb]);
+        if (p >= 1 && !stage2(c - 1, p == 1, i)) { ok = false; break; }
+      }
+      if (!ok) break;
+      if (P == 1) {
+        if (!stage2(c - 1, true, i)) break;
+      } else if (!stage2(c - 1, false, i)) {
+        break;
+      }
+      if (has_bias) {
+        const int db = i & 1;
+        if (!mbar_wait(&bars->deg_full[db], (i >> 1) & 1, status, 206, abort)) break;
+        if (i == 0 && !mbar_wait(&bars->b2_full, 0, status, 207, abort)) break;
+        tc_fence_after();
+        const uint32_t dbase = smem_u32(degs + db * C::DEG), bbase = smem_u32(b2s);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          mma_ss(tmem + C::YCOL, desc_sw128_kmajor(dbase + kk * 32),
+                 desc_sw128_kmajor(bbase + kk * 32), idesc, 1u);
+        tc_commit(&bars->deg_empty[db]);
+      }
+      tc_commit(&bars->y_full);
+    }
+    // every MMA issued above has completed once this commit arrives (bounded wait)
+    tc_commit(&bars->drain);
+    for (uint32_t t = 0; t < (1u << 24) && !mbar_try(&bars->drain, 0); ++t) {
+    }
+  } else if (warp >= 4 && warp < 8) {
+    // ------------------------------------------------------------------ expanders
+    const int r = threadIdx.x - 128;
+    const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    uint32_t aidx = 0;
+    for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x) {
+      bool ok = true;
+      for (int p = 0; p < P && ok; ++p) {
+        for (int d = 0; d < 3; ++d) {
+          const int kb = k + d - 1;
+          if (kb < 0 || kb >= K) continue;
+          const uint4 m = *reinterpret_cast<const uint4*>(
+              maskI + ((((size_t)k * P + p) * 3 + d) * kTile + r) * 4);
+          const int slot = aidx % C::NA;
+          if (!mbar_wait(&bars->a_empty[slot], ((aidx / C::NA) & 1) ^ 1, status, 301, abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          uint32_t v[32];
+          expand_word(m.x, v);
+          expand_word(m.y, v + 16);
+          tmem_st32(tmem + lane_base + C::ACOL + slot * 64, v);
+          expand_word(m.z, v);
+          expand_word(m.w, v + 16);
+          tmem_st32(tmem + lane_base + C::ACOL + slot * 64 + 32, v);
+          tmem_wait_st();
+          tc_fence_before();
+          mbar_arrive(&bars->a_full[slot]);
+          ++aidx;
+        }
+      }
+      if (!ok) break;
+    }
+  } else if (warp >= 8) {
+    // ------------------------------------------------------------------ converters / epilogue
+    const int r = threadIdx.x - 256;
+    const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    uint32_t c = 0;
+    int i = 0;
+    for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x, ++i) {
+      const int row = k * kTile + r;
+      bool ok = true;
+      for (int p = 0; p < P; ++p, ++c) {
+        const int b = c & 1;
+        if (!mbar_wait(&bars->d1_full[b], (c >> 1) & 1, status, 401, abort)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t col = tmem + lane_base + C::D1COL0 + b * H;
+        uint32_t v[32], q[32];
+#pragma unroll
+        for (int h0 = 0; h0 < H; h0 += 64) {
+          tmem_ld32(col + h0, v);
+          tmem_ld32(col + h0 + 32, q);
+          tmem_wait_ld();
+          uint32_t pk[32];
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            pk[j] = pack_bf16(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            pk[16 + j] = pack_bf16(__uint_as_float(q[2 * j]), __uint_as_float(q[2 * j + 1]));
+          if (BWD) {
+            // dM_p (bf16) transposed: dMT[(p*H + h) * n_pad + row]
+            const __nv_bfloat16* hv = reinterpret_cast<const __nv_bfloat16*>(pk);
+#pragma unroll 8
+            for (int h = 0; h < 64; ++h)
+              dMT[((size_t)p * H + h0 + h) * n_pad + row] = hv[h];
+          }
+          // packed pairs of columns h0..h0+63 go to columns (h0/2)..(h0/2)+31 of the buffer
+          tmem_st32(col + h0 / 2, pk);
+        }
+        tmem_wait_st();
+        tc_fence_before();
+        mbar_arrive(&bars->pre_ready[b]);
+      }
+      if (!ok) break;
+      if (!mbar_wait(&bars->y_full, i & 1, status, 402, abort)) break;
+      tc_fence_after();
+      float4* o = reinterpret_cast<float4*>(out + (size_t)row * H);
+#pragma unroll
+      for (int h0 = 0; h0 < H; h0 += 32) {
+        uint32_t v[32];
+        tmem_ld32(tmem + lane_base + C::YCOL + h0, v);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          float4 a = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                 __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+          if (accumulate) {
+            const float4 prev = o[h0 / 4 + j];
+            a.x += prev.x; a.y += prev.y; a.z += prev.z; a.w += prev.w;
+          }
+          o[h0 / 4 + j] = a;
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&bars->y_empty);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ------------------------------------------------------------------------------------ prep
+// out[c][r] = bf16(in[r][c]) for an R x Cc row-major input (batched over blockIdx.z)
+template <typename T>
+__global__ void k_transpose_bf16(const T* __restrict__ in, __nv_bfloat16* __restrict__ out, int R,
+                                 int Cc, int64_t in_batch, int64_t out_batch) {
+  __shared__ float tile[32][33];
+  in += blockIdx.z * in_batch;
+  out += blockIdx.z * out_batch;
+  const int r0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
+  for (int dy = threadIdx.y; dy < 32; dy += blockDim.y) {
+    const int r = r0 + dy, c = c0 + threadIdx.x;
+    float v = 0.f;
+    if (r < R && c < Cc) {
+      if constexpr (sizeof(T) == 2)
+        v = __bfloat162float(in[(int64_t)r * Cc + c]);
+      else
+        v = in[(int64_t)r * Cc + c];
+    }
+    tile[dy][threadIdx.x] = v;
+  }
+  __syncthreads();
+  for (int dy = threadIdx.y; dy < 32; dy += blockDim.y) {
+    const int c = c0 + dy, r = r0 + threadIdx.x;
+    if (c < Cc && r < R) out[(int64_t)c * R + r] = __float2bfloat16_rn(tile[threadIdx.x][dy]);
+  }
+}
+
+// b2T[h][p] = bf16 hi part of b[p][h], b2T[h][32 + p] = bf16 of the remainder (zero beyond P)
+__global__ void k_bias_split(const float* __restrict__ b, __nv_bfloat16* __restrict__ b2T, int P,
+                             int H) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= H * 64) return;
+  const int h = t / 64, q = t % 64, p = q % 32;
+  float v = 0.f;
+  if (p < P && b) {
+    const float x = b[p * H + h];
+    const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+    v = q < 32 ? __bfloat162float(hi) : x - __bfloat162float(hi);
+  }
+  b2T[t] = __float2bfloat16_rn(v);
+}
+
+// ------------------------------------------------------------------------------------ host
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  return make_map_ld(m, base, rows, cols, cols, box_rows);
+}
+
+int num_sms() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+inline size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+template <int H, bool BWD>
+cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
+                   const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
+                   __nv_bfloat16* dMT, int has_bias, int accumulate, int* status,
+                   cudaStream_t st) {
+  using C = Cfg<H>;
+  cudaError_t e = cudaFuncSetAttribute(k_band_tc<H, BWD>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  const int grid = std::min(p->K, num_sms());
+  k_band_tc<H, BWD><<<grid, kThreads, C::SMEM, st>>>(
+      tx, tw, tdeg, tb2, BWD ? p->d_maskTI : p->d_maskI, out, dMT, p->K, p->P, p->n_pad(),
+      has_bias, accumulate, status);
+  note_launch();
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool make_map_ld(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
+                 uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+int gemm_tn_num_sms() { return num_sms(); }
+
+bool band_tc_supported(const bg_plan* p, int dtype, int H) {
+  return p && dtype == 1 && p->S == 128 && (H == 64 || H == 128) && p->P <= 32 && p->d_maskI &&
+         p->d_maskTI && p->d_deg2 && p->max_deg <= 256 && encode_fn() != nullptr;
+}
+
+size_t band_tc_fwd_ws_bytes(const bg_plan* p, int dtype, int H) {
+  if (!p || dtype != 1) return 0;
+  const size_t n = (size_t)p->n_pad();
+  return al256(n * H * 2) + al256((size_t)p->P * H * H * 2) + al256((size_t)H * 64 * 2);
+}
+
+size_t band_tc_bwd_ws_bytes(const bg_plan* p, int dtype, int H) {
+  if (!p || dtype != 1) return 0;
+  const size_t n = (size_t)p->n_pad();
+  return al256(n * H * 2) + al256((size_t)p->P * H * n * 2) + al256((size_t)(H + 16) * n * 2) +
+         al256((size_t)H * 64 * 2) +
+         al256(sizeof(float) * gemm_tn_part_floats(p->P * H, H + 16, (int64_t)n));
+}
+
+cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, const float* b,
+                        float* Y, char* ws, size_t ws_bytes, int* status, cudaStream_t st) {
+  if (ws_bytes < band_tc_fwd_ws_bytes(p, 1, H)) return cudaErrorInvalidValue;
+  const int n = p->n_pad(), P = p->P;
+  __nv_bfloat16* ET = reinterpret_cast<__nv_bfloat16*>(ws);
+  __nv_bfloat16* WT = reinterpret_cast<__nv_bfloat16*>(ws + al256((size_t)n * H * 2));
+  __nv_bfloat16* b2T = reinterpret_cast<__nv_bfloat16*>(ws + al256((size_t)n * H * 2) +
+                                                        al256((size_t)P * H * H * 2));
+  // E [n][H] -> ET [H][n];  W_p [H_in][H_out] -> WT_p [H_out][H_in];  bias split
+  k_transpose_bf16<__nv_bfloat16><<<dim3((H + 31) / 32, (n + 31) / 32, 1), dim3(32, 8), 0, st>>>(
+      static_cast<const __nv_bfloat16*>(E), ET, n, H, 0, 0);
+  note_launch();
+  k_transpose_bf16<__nv_bfloat16><<<dim3((H + 31) / 32, (H + 31) / 32, P), dim3(32, 8), 0, st>>>(
+      static_cast<const __nv_bfloat16*>(W), WT, H, H, (int64_t)H * H, (int64_t)H * H);
+  note_launch();
+  const int has_bias = b != nullptr;
+  if (has_bias) {
+    k_bias_split<<<(H * 64 + 255) / 256, 256, 0, st>>>(b, b2T, P, H);
+    note_launch();
+  }
+  CUtensorMap tx, tw, tdeg, tb2;
+  if (!make_map(&tx, ET, H, n, H) || !make_map(&tw, WT, (uint64_t)P * H, H, H) ||
+      !make_map(&tdeg, p->d_deg2, n, 64, kTile) || !make_map(&tb2, b2T, H, 64, H))
+    return cudaErrorInvalidValue;
+  if (H == 64) return launch<64, false>(p, tx, tw, tdeg, tb2, Y, nullptr, has_bias, 0, status, st);
+  return launch<128, false>(p, tx, tw, tdeg, tb2, Y, nullptr, has_bias, 0, status, st);
+}
+
+cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, const float* dY,
+                        float* dE, float* dW, float* db, int accum, char* ws, size_t ws_bytes,
+                        int* status, cudaStream_t st) {
+  if (ws_bytes < band_tc_bwd_ws_bytes(p, 1, H)) return cudaErrorInvalidValue;
+  const int n = p->n_pad(), P = p->P;
+  size_t o = 0;
+  __nv_bfloat16* dYT = reinterpret_cast<__nv_bfloat16*>(ws + o);
+  o += al256((size_t)n * H * 2);
+  __nv_bfloat16* dMT = reinterpret_cast<__nv_bfloat16*>(ws + o);
+  o += al256((size_t)P * H * n * 2);
+  __nv_bfloat16* ETa = reinterpret_cast<__nv_bfloat16*>(ws + o);
+  o += al256((size_t)(H + 16) * n * 2);
+  __nv_bfloat16* b2T = reinterpret_cast<__nv_bfloat16*>(ws + o);
+  o += al256((size_t)H * 64 * 2);
+  float* part = reinterpret_cast<float*>(ws + o);
+  const size_t part_floats = gemm_tn_part_floats(P * H, H + 16, (int64_t)n);
+  k_transpose_bf16<float><<<dim3((H + 31) / 32, (n + 31) / 32, 1), dim3(32, 8), 0, st>>>(dY, dYT,
+                                                                                         n, H, 0, 0);
+  note_launch();
+  CUtensorMap tx, tw, tdeg, tb2;
+  if (!make_map(&tx, dYT, H, n, H) || !make_map(&tw, W, (uint64_t)P * H, H, H) ||
+      !make_map(&tdeg, p->d_deg2, n, 64, kTile) || !make_map(&tb2, b2T, H, 64, H))
+    return cudaErrorInvalidValue;
+  cudaError_t e = H == 64
+                      ? launch<64, true>(p, tx, tw, tdeg, tb2, dE, dMT, 0, accum, status, st)
+                      : launch<128, true>(p, tx, tw, tdeg, tb2, dE, dMT, 0, accum, status, st);
+  if (e != cudaSuccess) return e;
+  // [E^T; 1; 0]: the ones row turns the bias gradient into column H of the same product
+  k_transpose_bf16<__nv_bfloat16><<<dim3((H + 31) / 32, (n + 31) / 32, 1), dim3(32, 8), 0, st>>>(
+      static_cast<const __nv_bfloat16*>(E), ETa, n, H, 0, 0);
+  note_launch();
+  e = fill_ones_rows(ETa, H, n, n, st);
+  if (e != cudaSuccess) return e;
+  // dW_p[h][h'] (+)= sum_nodes E[node][h] dM_p[node][h'],  db_p[h'] (+)= sum_nodes dM_p[node][h']
+  return gemm_tn(dMT, n, ETa, n, P * H, H, n, 1, dW, db, accum, part, part_floats, status, st);
+}
+
+int band_tc_upload(bg_plan* p, cudaStream_t st) {
+  if (p->S != 128 || p->P > 32) return 0;
+  const int K = p->K, P = p->P, S = p->S, W32 = p->W32;
+  const size_t n = (size_t)K * S;
+  // interleave bits of every word: column 2j -> bit j, column 2j+1 -> bit 16+j
+  auto inter = [](uint32_t w) {
+    uint32_t o = 0;
+    for (int j = 0; j < 16; ++j) {
+      o |= ((w >> (2 * j)) & 1u) << j;
+      o |= ((w >> (2 * j + 1)) & 1u) << (16 + j);
+    }
+    return o;
+  };
+  std::vector<uint32_t> mi((size_t)K * P * 3 * S * W32), mti(mi.size());
+  std::vector<uint16_t> deg(n * 64, 0);
+  int max_deg = 0;
+  for (int k = 0; k < K; ++k)
+    for (int d = 0; d < 3; ++d)
+      for (int q = 0; q < P; ++q)
+        for (int r = 0; r < S; ++r)
+          for (int w = 0; w < W32; ++w) {
+            const size_t src = ((((size_t)k * 3 + d) * P + q) * S + r) * W32 + w;
+            const size_t dst = ((((size_t)k * P + q) * 3 + d) * S + r) * W32 + w;
+            mi[dst] = inter(p->masks[src]);
+            mti[dst] = inter(p->masksT[src]);
+          }
+  for (int k = 0; k < K; ++k)
+    for (int q = 0; q < P; ++q)
+      for (int r = 0; r < S; ++r) {
+        int cnt = 0;
+        for (int d = 0; d < 3; ++d)
+          for (int w = 0; w < W32; ++w)
+            cnt += __builtin_popcount(p->masks[((((size_t)k * 3 + d) * P + q) * S + r) * W32 + w]);
+        max_deg = std::max(max_deg, cnt);
+        // bf16 bit pattern of a small integer (exact up to 256)
+        float f = (float)cnt;
+        uint32_t u;
+        std::memcpy(&u, &f, 4);
+        const uint16_t bfv = (uint16_t)(u >> 16);
+        deg[((size_t)k * S + r) * 64 + q] = bfv;
+        deg[((size_t)k * S + r) * 64 + 32 + q] = bfv;
+      }
+  p->max_deg = max_deg;
+  if (cudaMalloc(&p->d_maskI, mi.size() * 4) != cudaSuccess ||
+      cudaMalloc(&p->d_maskTI, mti.size() * 4) != cudaSuccess ||
+      cudaMalloc(&p->d_deg2, deg.size() * 2) != cudaSuccess)
+    return -1;
+  if (cudaMemcpyAsync(p->d_maskI, mi.data(), mi.size() * 4, cudaMemcpyHostToDevice, st) != cudaSuccess ||
+      cudaMemcpyAsync(p->d_maskTI, mti.data(), mti.size() * 4, cudaMemcpyHostToDevice, st) != cudaSuccess ||
+      cudaMemcpyAsync(p->d_deg2, deg.data(), deg.size() * 2, cudaMemcpyHostToDevice, st) != cudaSuccess)
+    return -1;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return -1;
+  return 0;
+}
+
+void band_tc_release(bg_plan* p) {
+  cudaFree(p->d_maskI);
+  cudaFree(p->d_maskTI);
+  cudaFree(p->d_deg2);
+  p->d_maskI = p->d_maskTI = nullptr;
+  p->d_deg2 = nullptr;
+}
+
 }  // namespace bg

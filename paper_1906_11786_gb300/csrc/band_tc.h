@@ -18,6 +18,8 @@ cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, c
 cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, const float* dY,
                         float* dE, float* dW, float* db, int accum, char* ws, size_t ws_bytes,
                         int* status, cudaStream_t st);
+// Builds and uploads the tensor-core path's plan data (no-op where unsupported); 0 on success.
+int band_tc_upload(bg_plan* p, cudaStream_t st);
 // Frees device data the tensor-core path keeps with the plan.
 void band_tc_release(bg_plan* p);
 

@@ -1,0 +1,235 @@
+// Split-K "TN" GEMM on tcgen05 for the weight-gradient reductions of the backward pass:
+//     part[s][m][n] = sum_{k in split s} A[m][k] B[n][k]        (A, B bf16, K contiguous; fp32)
+// followed by a deterministic reduction over the splits into the gradient layout.  The weight
+// gradients of Eq. 1's transforms and of the GRU are sums over every node (and every step) of
+// outer products, i.e. exactly such GEMMs with K = nodes; their bias gradients come out of the
+// same product through a row of ones appended to B.
+//
+// 192 threads: warp 0 issues TMA loads into a 4-stage ring, warp 1 allocates TMEM and issues the
+// MMAs (lane 0), warps 2-5 read the accumulator back (one TMEM lane quarter each).
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include <algorithm>
+
+#include "gemm_tc.h"
+#include "kernels.h"
+#include "tc_util.cuh"
+
+namespace bg {
+
+using namespace tc;
+
+namespace {
+
+constexpr int kStages = 4;
+
+template <int BN>
+struct GCfg {
+  static constexpr int A_BYTES = 128 * 128;  // 128 rows x 64 bf16
+  static constexpr int B_BYTES = BN * 128;
+  static constexpr int STAGE = A_BYTES + B_BYTES;
+  static constexpr int SMEM = kStages * STAGE + 1024 + 1024;
+  static constexpr int TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+};
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
+template <int BN>
+__global__ void __launch_bounds__(192, 1)
+    k_gemm_tn(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+              float* __restrict__ part, int M, int N, int kchunks, int per_split, int* status) {
+  using C = GCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * C::STAGE);
+  uint64_t* empty = full + kStages;
+  uint64_t* done = empty + kStages;
+  uint64_t* drain = done + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+  volatile int* abort = abort_flag;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int mt = blockIdx.x, split = blockIdx.z;
+  const int kc0 = split * per_split;
+  const int kc1 = min(kchunks, kc0 + per_split);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    mbar_init(done, 1);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TCOLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+    uint32_t issued[kStages] = {0, 0, 0, 0};
+    for (int kc = kc0, it = 0; kc < kc1; ++kc, ++it) {
+      const int s = it % kStages;
+      if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1, status, 501, abort)) break;
+      ++issued[s];
+      mbar_expect_tx(&full[s], C::STAGE);
+      uint8_t* st = smem + s * C::STAGE;
+      tma_load_2d(st, &tmA, &full[s], kc * 64, mt * 128);
+      tma_load_2d(st + C::A_BYTES, &tmB, &full[s], kc * 64, blockIdx.y * BN);
+    }
+    if (*abort)
+      for (int s = 0; s < kStages; ++s)
+        for (uint32_t t = 0; issued[s] && t < (1u << 22) && !mbar_try(&full[s], (issued[s] - 1) & 1); ++t) {
+        }
+  } else if (warp == 1 && lane == 0) {
+    constexpr uint32_t idesc = idesc_bf16_f32(128, BN);
+    for (int kc = kc0, it = 0; kc < kc1; ++kc, ++it) {
+      const int s = it % kStages;
+      if (!mbar_wait(&full[s], (it / kStages) & 1, status, 502, abort)) break;
+      tc_fence_after();
+      const uint32_t a = smem_u32(smem + s * C::STAGE), b = a + C::A_BYTES;
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)
+        mma_ss(tmem, desc_sw128_kmajor(a + kk * 32), desc_sw128_kmajor(b + kk * 32), idesc,
+               (kc > kc0 || kk > 0) ? 1u : 0u);
+      tc_commit(&empty[s]);
+    }
+    tc_commit(done);
+    tc_commit(drain);
+    for (uint32_t t = 0; t < (1u << 24) && !mbar_try(drain, 0); ++t) {
+    }
+  } else if (warp >= 2) {
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int m = mt * 128 + q * 32 + lane;
+    if (mbar_wait(done, 0, status, 503, abort)) {
+      tc_fence_after();
+      float* out = part + ((size_t)split * M + m) * N + blockIdx.y * BN;
+#pragma unroll
+      for (int c0 = 0; c0 < BN; c0 += 16) {
+        uint32_t v[16];
+        tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + c0, v);
+        tmem_wait_ld();
+        if (m < M && kc1 > kc0) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            if (blockIdx.y * BN + c0 + j < N) out[c0 + j] = __uint_as_float(v[j]);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TCOLS);
+  }
+}
+
+// mode 0: out[m][n] (+)= sum_s part[s][m][n] for n < Hout; bias[m] (+)= sum_s part[s][m][Hout]
+// mode 1: m = p*Hout + o: out[p][n][o] (+)= sum_s part[s][m][n]; bias[m] (+)= sum_s part[s][m][Hout]
+__global__ void k_gemm_tn_reduce(const float* __restrict__ part, int splits, int M, int N, int Hout,
+                                 int mode, float* __restrict__ out, float* __restrict__ bias,
+                                 int accumulate) {
+  const int64_t total = (int64_t)M * (Hout + 1);
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int m = (int)(t / (Hout + 1)), n = (int)(t % (Hout + 1));
+    float s = 0.f;
+    for (int q = 0; q < splits; ++q) s += part[((size_t)q * M + m) * N + n];
+    float* dst;
+    if (n == Hout) {
+      if (!bias) continue;
+      dst = bias + m;
+    } else if (mode == 0) {
+      dst = out + (size_t)m * Hout + n;
+    } else {
+      const int p = m / Hout, o = m % Hout;
+      dst = out + ((size_t)p * Hout + n) * Hout + o;
+    }
+    *dst = accumulate ? *dst + s : s;
+  }
+}
+
+}  // namespace
+
+namespace {
+__global__ void k_fill_ones_rows(__nv_bfloat16* base, int H, int64_t n, int64_t ld) {
+  const int64_t total = 16 * n;
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int r = (int)(t / n);
+    const int64_t c = t % n;
+    base[(int64_t)(H + r) * ld + c] = __float2bfloat16_rn(r == 0 ? 1.f : 0.f);
+  }
+}
+}  // namespace
+
+cudaError_t fill_ones_rows(__nv_bfloat16* base, int H, int64_t n, int64_t ld, cudaStream_t st) {
+  const int64_t total = 16 * n;
+  k_fill_ones_rows<<<(unsigned)std::min<int64_t>((total + 255) / 256, 8192), 256, 0, st>>>(base, H,
+                                                                                          n, ld);
+  note_launch();
+  return cudaGetLastError();
+}
+
+size_t gemm_tn_part_floats(int M, int N, int64_t K) {
+  const int64_t kchunks = (K + 63) / 64;
+  const int mt = (M + 127) / 128;
+  const int64_t splits = std::max<int64_t>(1, std::min<int64_t>(kchunks, (512 + mt - 1) / mt));
+  return (size_t)splits * M * N;
+}
+
+cudaError_t gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int Hout,
+                    int64_t K, int mode, float* out, float* bias, int accumulate, float* part,
+                    size_t part_floats, int* status, cudaStream_t st) {
+  const int N = Hout + 16;  // Hout gradient columns, one ones-column (bias), padding to 16
+  if (N != 48 && N != 80 && N != 144) return cudaErrorInvalidValue;
+  const int64_t kchunks = (K + 63) / 64;
+  const int mt = (M + 127) / 128;
+  const int sms = gemm_tn_num_sms();
+  int splits = (int)std::max<int64_t>(1, std::min<int64_t>(kchunks, (2 * sms + mt - 1) / mt));
+  while (splits > 1 && (size_t)splits * M * N > part_floats) --splits;
+  const int per = (int)((kchunks + splits - 1) / splits);
+  splits = (int)((kchunks + per - 1) / per);
+  CUtensorMap ta, tb;
+  if (!make_map_ld(&ta, A, M, K, lda, 128) || !make_map_ld(&tb, B, N, K, ldb, N))
+    return cudaErrorInvalidValue;
+  dim3 grid(mt, 1, splits);
+  cudaError_t e;
+#define BG_GEMM_CASE(BNV)                                                                      \
+  e = cudaFuncSetAttribute(k_gemm_tn<BNV>, cudaFuncAttributeMaxDynamicSharedMemorySize,        \
+                           GCfg<BNV>::SMEM);                                                   \
+  if (e != cudaSuccess) return e;                                                              \
+  k_gemm_tn<BNV><<<grid, 192, GCfg<BNV>::SMEM, st>>>(ta, tb, part, M, N, (int)kchunks, per, status);
+  if (N == 48) {
+    BG_GEMM_CASE(48)
+  } else if (N == 80) {
+    BG_GEMM_CASE(80)
+  } else {
+    BG_GEMM_CASE(144)
+  }
+#undef BG_GEMM_CASE
+  note_launch();
+  const int64_t total = (int64_t)M * (Hout + 1);
+  k_gemm_tn_reduce<<<(unsigned)std::min<int64_t>((total + 255) / 256, 4096), 256, 0, st>>>(
+      part, splits, M, N, Hout, mode, out, bias, accumulate);
+  note_launch();
+  return cudaGetLastError();
+}
+
+}  // namespace bg

@@ -1,0 +1,35 @@
+// Split-K tcgen05 GEMM for weight-gradient reductions (gemm_tc.cu).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+namespace bg {
+
+// Scratch floats gemm_tn needs for its split-K partial sums.
+size_t gemm_tn_part_floats(int M, int N, int64_t K);
+
+// Reduces over K (nodes, possibly several steps concatenated) the outer products
+//   G[m][n] = sum_k A[m][k] B[n][k]    A: [M][K] bf16 (row stride lda), B: [Hout+16][K] bf16
+// where B's row Hout is all ones and rows Hout+1.. are zero, so column Hout of G is the row sum
+// of A (a bias gradient).  Output (accumulate != 0 adds):
+//   mode 0: out[m][n] = G[m][n] (n < Hout), bias[m] = G[m][Hout]
+//   mode 1: m = p*Hout + o: out[p][n][o] = G[m][n], bias[m] = G[m][Hout]   (bias may be NULL)
+// Hout in {32, 64, 128}.  Deterministic: fixed split layout and summation order.
+cudaError_t gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int Hout,
+                    int64_t K, int mode, float* out, float* bias, int accumulate, float* part,
+                    size_t part_floats, int* status, cudaStream_t st);
+
+// 2-D bf16 tensor map over row-major [rows][cols] with row stride ld elements; box {64, box_rows};
+// 128-byte swizzle; reads outside the array return zero.
+bool make_map_ld(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
+                 uint32_t box_rows);
+int gemm_tn_num_sms();
+
+// rows [H, H+16) of a [H+16][ld] bf16 array: row H = 1.0, the rest 0 (cols [0, n)).
+cudaError_t fill_ones_rows(__nv_bfloat16* base, int H, int64_t n, int64_t ld, cudaStream_t st);
+
+}  // namespace bg

@@ -21,7 +21,14 @@ def built():
     torch.manual_seed(0)
 
 
+def _expect_path(c: Case):
+    """The fused tensor-core kernels must carry every bf16 case with S = 128, H in {64, 128}."""
+    want = c.dtype == "bf16" and c.S == 128 and c.H in (64, 128) and c.P <= 32
+    assert L.band_uses_tensor_cores(c.plan, c.dtype, c.H) == want
+
+
 def _fwd(c: Case, with_bias=True):
+    _expect_path(c)
     Y = torch.empty((c.N, c.H), dtype=torch.float32, device="cuda")
     L.band_propagate_fwd(c.plan, c.dtype, c.H, c.E_band_dev, c.dprm["W"],
                          c.dprm["b"] if with_bias else None, Y, c.ws(L.BG_OP_PROPAGATE_FWD))
