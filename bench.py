@@ -178,9 +178,9 @@ class OursStep:
         if c["gru"]:
             self.saved = torch.empty(L.ggnn_saved_bytes(self.plan, self.dt, H, T), dtype=torch.uint8,
                                      device="cuda")
-            self.ws_f = torch.empty(L.workspace_bytes(self.plan, self.dt, H, L.BG_OP_GGNN_FWD),
+            self.ws_f = torch.empty(L.ggnn_workspace_bytes(self.plan, self.dt, H, T, L.BG_OP_GGNN_FWD),
                                     dtype=torch.uint8, device="cuda")
-            self.ws_b = torch.empty(L.workspace_bytes(self.plan, self.dt, H, L.BG_OP_GGNN_BWD),
+            self.ws_b = torch.empty(L.ggnn_workspace_bytes(self.plan, self.dt, H, T, L.BG_OP_GGNN_BWD),
                                     dtype=torch.uint8, device="cuda")
             self.ET = torch.empty((N, H), dtype=tdt, device="cuda")
         else:

@@ -138,7 +138,11 @@ int bg_unpack_states(const bg_plan* plan, bg_dtype dtype, int32_t H, const void*
 #define BG_OP_GGNN_FWD 2
 #define BG_OP_GGNN_BWD 3
 #define BG_OP_READOUT 4
+/* Scratch of the propagate and readout ops (0 for the GGNN ops, whose size depends on T). */
 size_t bg_workspace_bytes(const bg_plan* plan, bg_dtype dtype, int32_t H, int32_t op);
+/* Scratch of bg_ggnn_step (op BG_OP_GGNN_FWD) or bg_ggnn_step_bwd (BG_OP_GGNN_BWD) for T steps. */
+size_t bg_ggnn_workspace_bytes(const bg_plan* plan, bg_dtype dtype, int32_t H, int32_t T,
+                               int32_t op);
 
 /* ---- propagation (device) -------------------------------------------------------------------
  * Forward (Eq. 1 / Eq. 3 with P types and per-type bias):

@@ -84,6 +84,7 @@ def load(path: str = LIB_PATH):
         "bg_band_propagate_bwd": (c.c_int, [vp, c.c_int, i32, vp, vp, vp, vp, vp, vp, c.c_uint32,
                                             vp, sz, vp]),
         "bg_ggnn_saved_bytes": (sz, [vp, c.c_int, i32, i32]),
+        "bg_ggnn_workspace_bytes": (sz, [vp, c.c_int, i32, i32, i32]),
         "bg_ggnn_step": (c.c_int, [vp, c.c_int, i32, i32, vp, vp, vp, vp, sz, vp, sz, vp]),
         "bg_ggnn_step_bwd": (c.c_int, [vp, c.c_int, i32, i32, vp, vp, sz, vp, vp, vp, c.c_uint32,
                                        vp, sz, vp]),
@@ -229,6 +230,10 @@ def band_plan(graphs, n_types, block_S, capacity_blocks=0, flags=BG_RCM | BG_KEE
 
 def workspace_bytes(plan, dtype, H, op) -> int:
     return int(load().bg_workspace_bytes(plan.handle, dtype_code(dtype), H, op))
+
+
+def ggnn_workspace_bytes(plan, dtype, H, T, op) -> int:
+    return int(load().bg_ggnn_workspace_bytes(plan.handle, dtype_code(dtype), H, T, op))
 
 
 def ggnn_saved_bytes(plan, dtype, H, T) -> int:

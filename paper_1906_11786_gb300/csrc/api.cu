@@ -10,6 +10,8 @@
 #include <vector>
 
 #include "band_tc.h"
+#include "gemm_tc.h"
+#include "gru_tc.h"
 #include "internal.h"
 #include "kernels.h"
 
@@ -381,6 +383,66 @@ size_t saved_E_off(const bg_plan* p, bg_dtype dt, int H, int t) {
 size_t saved_Y_off(const bg_plan* p, bg_dtype dt, int H, int T, int t) {
   return saved_E_off(p, dt, H, T + 1) + (size_t)t * al(sizeof(float) * (size_t)p->n_pad() * H);
 }
+
+// ---- fused tensor-core GGNN steps (bf16, S = 128, H = 64, P <= 32)
+bool tc_shape(const bg_plan* p, bg_dtype dt, int H) {
+  return p && dt == BG_BF16 && p->S == 128 && H == 64 && p->P <= 32;
+}
+bool tc_ggnn(const bg_plan* p, bg_dtype dt, int H) {
+  return tc_shape(p, dt, H) && bg::band_tc_supported(p, (int)dt, H) && bg::gru_tc_supported(H);
+}
+
+// Saved activations: E(0..T) [n][H]; [E(0..T-1)^T; 1; 0] as [H+16][T n]; Y(0..T-1) [n][H];
+// [Y(0..T-1)^T; 1; 0] as [H+16][T n]  (all bf16).  The transposed copies are the operands of the
+// band products (TMA, K contiguous) and of the weight-gradient GEMMs (ones row -> bias gradient).
+struct TcSaved {
+  size_t E, ETa, Y, YTa, total;
+};
+TcSaved tc_saved(const bg_plan* p, int H, int T) {
+  const size_t n = (size_t)p->n_pad(), TN = (size_t)T * n, st = al(n * H * 2);
+  TcSaved s{};
+  size_t o = 0;
+  s.E = o; o += (size_t)(T + 1) * st;
+  s.ETa = o; o += al((size_t)(H + 16) * TN * 2);
+  s.Y = o; o += (size_t)T * st;
+  s.YTa = o; o += al((size_t)(H + 16) * TN * 2);
+  s.total = o;
+  return s;
+}
+struct TcFwdWs {
+  size_t WT, b2T, total;
+};
+TcFwdWs tc_fwd_ws(const bg_plan* p, int H) {
+  TcFwdWs w{};
+  size_t o = 0;
+  w.WT = o; o += al((size_t)p->P * H * H * 2);
+  w.b2T = o; o += al((size_t)H * 64 * 2);
+  w.total = o;
+  return w;
+}
+struct TcBwdWs {
+  size_t g, dXT, dMT, dgiT, dghT, WihT, WhhT, part, total;
+};
+size_t tc_part_floats(const bg_plan* p, int H, int T) {
+  const int64_t K = (int64_t)T * p->n_pad();
+  return std::max(bg::gemm_tn_part_floats(p->P * H, H + 16, K),
+                  bg::gemm_tn_part_floats(3 * H, H + 16, K));
+}
+TcBwdWs tc_bwd_ws(const bg_plan* p, int H, int T) {
+  const size_t n = (size_t)p->n_pad(), TN = (size_t)T * n;
+  TcBwdWs w{};
+  size_t o = 0;
+  w.g = o; o += al(sizeof(float) * n * H);
+  w.dXT = o; o += al(n * H * 2);
+  w.dMT = o; o += al((size_t)p->P * H * TN * 2);
+  w.dgiT = o; o += al((size_t)3 * H * TN * 2);
+  w.dghT = o; o += al((size_t)3 * H * TN * 2);
+  w.WihT = o; o += al((size_t)3 * H * H * 2);
+  w.WhhT = o; o += al((size_t)3 * H * H * 2);
+  w.part = o; o += al(sizeof(float) * tc_part_floats(p, H, T));
+  w.total = o;
+  return w;
+}
 }  // namespace
 
 extern "C" size_t bg_workspace_bytes(const bg_plan* p, bg_dtype dt, int32_t H, int32_t op) {
@@ -388,16 +450,24 @@ extern "C" size_t bg_workspace_bytes(const bg_plan* p, bg_dtype dt, int32_t H, i
   switch (op) {
     case BG_OP_PROPAGATE_FWD: return fwd_ws(p, dt, H).total;
     case BG_OP_PROPAGATE_BWD: return bwd_ws(p, dt, H).total;
-    case BG_OP_GGNN_FWD: return ggnn_fwd_ws(p, dt, H).total;
-    case BG_OP_GGNN_BWD: return ggnn_bwd_ws(p, dt, H).total;
     case BG_OP_READOUT: return al(sizeof(float) * ((size_t)p->n_packed * H + p->n_packed + 64));
     default: return 0;
   }
 }
 
+extern "C" size_t bg_ggnn_workspace_bytes(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
+                                          int32_t op) {
+  if (!p || H <= 0 || T < 1) return 0;
+  const bool tc = tc_shape(p, dt, H);
+  if (op == BG_OP_GGNN_FWD) return std::max(ggnn_fwd_ws(p, dt, H).total, tc ? tc_fwd_ws(p, H).total : 0);
+  if (op == BG_OP_GGNN_BWD) return std::max(ggnn_bwd_ws(p, dt, H).total, tc ? tc_bwd_ws(p, H, T).total : 0);
+  return 0;
+}
+
 extern "C" size_t bg_ggnn_saved_bytes(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T) {
   if (!p || H <= 0 || T < 0) return 0;
-  return saved_Y_off(p, dt, H, T, T);
+  const size_t simt = saved_Y_off(p, dt, H, T, T);
+  return tc_shape(p, dt, H) && T >= 1 ? std::max(simt, tc_saved(p, H, T).total) : simt;
 }
 
 extern "C" int bg_band_uses_tensor_cores(const bg_plan* p, bg_dtype dt, int32_t H) {
@@ -570,9 +640,46 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
   if (T < 1 || T > 1024) return bg_fail(BG_EINVAL, "T must be in [1, 1024]");
   BG_PTR(E0, "E0"); BG_OPT_PTR(ET, "ET"); BG_PTR(saved, "saved"); BG_PTR(ws, "ws");
   if (saved_bytes < bg_ggnn_saved_bytes(p, dt, H, T)) return bg_fail(BG_ECAPACITY, "saved buffer too small");
-  GgnnFwdWs w = ggnn_fwd_ws(p, dt, H);
-  if (ws_bytes < w.total) return bg_fail(BG_ECAPACITY, "workspace too small");
+  if (ws_bytes < bg_ggnn_workspace_bytes(p, dt, H, T, BG_OP_GGNN_FWD))
+    return bg_fail(BG_ECAPACITY, "workspace too small");
   cudaStream_t st = (cudaStream_t)stream;
+  if (tc_ggnn(p, dt, H)) {
+    int* status = nullptr;
+    BG_TRY(status_word_ptr(&status));
+    const size_t n = (size_t)p->n_pad(), TN = (size_t)T * n, stE = al(n * H * 2);
+    const TcSaved sl = tc_saved(p, H, T);
+    const TcFwdWs wl = tc_fwd_ws(p, H);
+    char* sv = static_cast<char*>(saved);
+    char* wsc = static_cast<char*>(ws);
+    auto Ei = [&](int t) { return reinterpret_cast<__nv_bfloat16*>(sv + sl.E + (size_t)t * stE); };
+    auto Yi = [&](int t) { return reinterpret_cast<__nv_bfloat16*>(sv + sl.Y + (size_t)t * stE); };
+    __nv_bfloat16* ETa = reinterpret_cast<__nv_bfloat16*>(sv + sl.ETa);
+    __nv_bfloat16* YTa = reinterpret_cast<__nv_bfloat16*>(sv + sl.YTa);
+    __nv_bfloat16* WT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.WT);
+    __nv_bfloat16* b2T = reinterpret_cast<__nv_bfloat16*>(wsc + wl.b2T);
+    BG_CUDA(cudaMemcpyAsync(Ei(0), E0, n * H * 2, cudaMemcpyDeviceToDevice, st));
+    BG_CUDA(bg::prep_transpose_bf16(E0, 0, ETa, (int)n, H, 1, st, (int64_t)TN));
+    BG_CUDA(bg::fill_ones_rows(ETa, H, (int64_t)TN, (int64_t)TN, st));
+    BG_CUDA(bg::fill_ones_rows(YTa, H, (int64_t)TN, (int64_t)TN, st));
+    BG_CUDA(bg::prep_transpose_bf16(prm->W, 0, WT, H, H, p->P, st));
+    if (prm->b) BG_CUDA(bg::prep_bias_split(prm->b, b2T, p->P, H, st));
+    for (int t = 0; t < T; ++t) {
+      {
+        KTimer tm(BG_KID_BAND_FWD, st);
+        BG_CUDA(bg::band_tc_fwd_core(p, H, ETa + (size_t)t * n, (int64_t)TN, WT,
+                                     prm->b ? b2T : nullptr, nullptr, Yi(t), YTa + (size_t)t * n,
+                                     (int64_t)TN, status, st));
+      }
+      KTimer tm(BG_KID_GRU_FWD, st);
+      BG_CUDA(bg::gru_fwd_tc(
+          (int)n, p->n_real, Yi(t), Ei(t), static_cast<const __nv_bfloat16*>(prm->W_ih),
+          static_cast<const __nv_bfloat16*>(prm->W_hh), prm->b_ih, prm->b_hh, Ei(t + 1),
+          t + 1 < T ? ETa + (size_t)(t + 1) * n : nullptr, (int64_t)TN, status, st));
+    }
+    if (ET) BG_CUDA(cudaMemcpyAsync(ET, Ei(T), n * H * 2, cudaMemcpyDeviceToDevice, st));
+    return BG_OK;
+  }
+  GgnnFwdWs w = ggnn_fwd_ws(p, dt, H);
   const int bf = dt == BG_BF16;
   char* sv = static_cast<char*>(saved);
   char* wsc = static_cast<char*>(ws);
@@ -609,9 +716,60 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
   BG_PTR(gr->dW, "dW"); BG_OPT_PTR(gr->db, "db"); BG_PTR(gr->dW_ih, "dW_ih");
   BG_PTR(gr->dW_hh, "dW_hh"); BG_PTR(gr->db_ih, "db_ih"); BG_PTR(gr->db_hh, "db_hh");
   if (saved_bytes < bg_ggnn_saved_bytes(p, dt, H, T)) return bg_fail(BG_ECAPACITY, "saved buffer too small");
-  GgnnBwdWs w = ggnn_bwd_ws(p, dt, H);
-  if (ws_bytes < w.total) return bg_fail(BG_ECAPACITY, "workspace too small");
+  if (ws_bytes < bg_ggnn_workspace_bytes(p, dt, H, T, BG_OP_GGNN_BWD))
+    return bg_fail(BG_ECAPACITY, "workspace too small");
   cudaStream_t st = (cudaStream_t)stream;
+  if (tc_ggnn(p, dt, H)) {
+    int* status = nullptr;
+    BG_TRY(status_word_ptr(&status));
+    const size_t n = (size_t)p->n_pad(), TN = (size_t)T * n, stE = al(n * H * 2);
+    const TcSaved sl = tc_saved(p, H, T);
+    const TcBwdWs wl = tc_bwd_ws(p, H, T);
+    const char* sv = static_cast<const char*>(saved);
+    char* wsc = static_cast<char*>(ws);
+    auto Ei = [&](int t) { return reinterpret_cast<const __nv_bfloat16*>(sv + sl.E + (size_t)t * stE); };
+    auto Yi = [&](int t) { return reinterpret_cast<const __nv_bfloat16*>(sv + sl.Y + (size_t)t * stE); };
+    const __nv_bfloat16* ETa = reinterpret_cast<const __nv_bfloat16*>(sv + sl.ETa);
+    const __nv_bfloat16* YTa = reinterpret_cast<const __nv_bfloat16*>(sv + sl.YTa);
+    float* g = reinterpret_cast<float*>(wsc + wl.g);
+    __nv_bfloat16* dXT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.dXT);
+    __nv_bfloat16* dMT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.dMT);
+    __nv_bfloat16* dgiT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.dgiT);
+    __nv_bfloat16* dghT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.dghT);
+    __nv_bfloat16* WihT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.WihT);
+    __nv_bfloat16* WhhT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.WhhT);
+    float* part = reinterpret_cast<float*>(wsc + wl.part);
+    const size_t pf = tc_part_floats(p, H, T);
+    const auto* Wih = static_cast<const __nv_bfloat16*>(prm->W_ih);
+    const auto* Whh = static_cast<const __nv_bfloat16*>(prm->W_hh);
+    BG_CUDA(bg::prep_transpose_bf16(Wih, 0, WihT, 3 * H, H, 1, st));
+    BG_CUDA(bg::prep_transpose_bf16(Whh, 0, WhhT, 3 * H, H, 1, st));
+    const float* gin = dET;
+    for (int t = T - 1; t >= 0; --t) {
+      {
+        KTimer tm(BG_KID_GRU_BWD, st);
+        BG_CUDA(bg::gru_bwd_tc((int)n, p->n_real, Yi(t), Ei(t), Wih, Whh, WihT, WhhT, prm->b_ih,
+                               prm->b_hh, gin, g, dXT, (int64_t)n, dgiT + (size_t)t * n,
+                               dghT + (size_t)t * n, (int64_t)TN, status, st));
+      }
+      KTimer tm(BG_KID_BAND_BWD, st);
+      BG_CUDA(bg::band_tc_bwd_core(p, H, dXT, (int64_t)n, prm->W, g, 1, dMT + (size_t)t * n,
+                                   (int64_t)TN, status, st));
+      gin = g;
+    }
+    const int acc = (flags & BG_ACCUM) ? 1 : 0;
+    KTimer tm(BG_KID_DW, st);
+    // dW_p, db_p over all steps and nodes; dW_ih, db_ih; dW_hh, db_hh
+    BG_CUDA(bg::gemm_tn(dMT, (int64_t)TN, ETa, (int64_t)TN, p->P * H, H, (int64_t)TN, 1, gr->dW,
+                        gr->db, acc, part, pf, status, st));
+    BG_CUDA(bg::gemm_tn(dgiT, (int64_t)TN, YTa, (int64_t)TN, 3 * H, H, (int64_t)TN, 0, gr->dW_ih,
+                        gr->db_ih, acc, part, pf, status, st));
+    BG_CUDA(bg::gemm_tn(dghT, (int64_t)TN, ETa, (int64_t)TN, 3 * H, H, (int64_t)TN, 0, gr->dW_hh,
+                        gr->db_hh, acc, part, pf, status, st));
+    BG_CUDA(cudaMemcpyAsync(dE0, g, sizeof(float) * n * H, cudaMemcpyDeviceToDevice, st));
+    return BG_OK;
+  }
+  GgnnBwdWs w = ggnn_bwd_ws(p, dt, H);
   const int bf = dt == BG_BF16;
   const int n = p->n_pad();
   const char* sv = static_cast<const char*>(saved);

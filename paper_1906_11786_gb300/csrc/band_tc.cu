@@ -102,7 +102,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     k_band_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
               const __grid_constant__ CUtensorMap tm_deg, const __grid_constant__ CUtensorMap tm_b2,
               const uint32_t* __restrict__ maskI, float* __restrict__ out,
-              __nv_bfloat16* __restrict__ dMT, int K, int P, int n_pad, int has_bias,
+              __nv_bfloat16* __restrict__ outb, __nv_bfloat16* __restrict__ outT, int64_t ld_outT,
+              __nv_bfloat16* __restrict__ dMT, int64_t ld_mt, int K, int P, int has_bias,
               int accumulate, int* status) {
   using C = Cfg<H>;
   extern __shared__ uint8_t smem_raw[];
@@ -340,11 +341,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int j = 0; j < 16; ++j)
             pk[16 + j] = pack_bf16(__uint_as_float(q[2 * j]), __uint_as_float(q[2 * j + 1]));
           if (BWD) {
-            // dM_p (bf16) transposed: dMT[(p*H + h) * n_pad + row]
-            const __nv_bfloat16* hv = reinterpret_cast<const __nv_bfloat16*>(pk);
-#pragma unroll 8
-            for (int h = 0; h < 64; ++h)
-              dMT[((size_t)p * H + h0 + h) * n_pad + row] = hv[h];
+            // dM_p (bf16) transposed: dMT[(p*H + h) * ld_mt + row]
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+              const uint32_t w2 = pk[j];
+              __nv_bfloat16* d = dMT + ((size_t)p * H + h0 + 2 * j) * ld_mt + row;
+              d[0] = __ushort_as_bfloat16((unsigned short)(w2 & 0xFFFFu));
+              d[ld_mt] = __ushort_as_bfloat16((unsigned short)(w2 >> 16));
+            }
           }
           // packed pairs of columns h0..h0+63 go to columns (h0/2)..(h0/2)+31 of the buffer
           tmem_st32(col + h0 / 2, pk);
@@ -356,21 +360,43 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       if (!mbar_wait(&bars->y_full, i & 1, status, 402, abort)) break;
       tc_fence_after();
-      float4* o = reinterpret_cast<float4*>(out + (size_t)row * H);
 #pragma unroll
       for (int h0 = 0; h0 < H; h0 += 32) {
         uint32_t v[32];
         tmem_ld32(tmem + lane_base + C::YCOL + h0, v);
         tmem_wait_ld();
+        if (out) {
+          float4* o = reinterpret_cast<float4*>(out + (size_t)row * H + h0);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          float4 a = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
-                                 __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
-          if (accumulate) {
-            const float4 prev = o[h0 / 4 + j];
-            a.x += prev.x; a.y += prev.y; a.z += prev.z; a.w += prev.w;
+          for (int j = 0; j < 8; ++j) {
+            float4 a = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                   __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+            if (accumulate) {
+              const float4 prev = o[j];
+              a.x += prev.x; a.y += prev.y; a.z += prev.z; a.w += prev.w;
+            }
+            o[j] = a;
           }
-          o[h0 / 4 + j] = a;
+        }
+        if (outb || outT) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            pk[j] = pack_bf16(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+          if (outb) {
+            uint4* ob = reinterpret_cast<uint4*>(outb + (size_t)row * H + h0);
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              ob[j] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+          }
+          if (outT) {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              __nv_bfloat16* d = outT + (size_t)(h0 + 2 * j) * ld_outT + row;
+              d[0] = __ushort_as_bfloat16((unsigned short)(pk[j] & 0xFFFFu));
+              d[ld_outT] = __ushort_as_bfloat16((unsigned short)(pk[j] >> 16));
+            }
+          }
         }
       }
       tc_fence_before();
@@ -390,7 +416,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // out[c][r] = bf16(in[r][c]) for an R x Cc row-major input (batched over blockIdx.z)
 template <typename T>
 __global__ void k_transpose_bf16(const T* __restrict__ in, __nv_bfloat16* __restrict__ out, int R,
-                                 int Cc, int64_t in_batch, int64_t out_batch) {
+                                 int Cc, int64_t in_batch, int64_t out_batch, int64_t ld_out) {
   __shared__ float tile[32][33];
   in += blockIdx.z * in_batch;
   out += blockIdx.z * out_batch;
@@ -409,7 +435,7 @@ __global__ void k_transpose_bf16(const T* __restrict__ in, __nv_bfloat16* __rest
   __syncthreads();
   for (int dy = threadIdx.y; dy < 32; dy += blockDim.y) {
     const int c = c0 + dy, r = r0 + threadIdx.x;
-    if (c < Cc && r < R) out[(int64_t)c * R + r] = __float2bfloat16_rn(tile[threadIdx.x][dy]);
+    if (c < Cc && r < R) out[(int64_t)c * ld_out + r] = __float2bfloat16_rn(tile[threadIdx.x][dy]);
   }
 }
 
@@ -463,7 +489,8 @@ inline size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
 template <int H, bool BWD>
 cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
                    const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
-                   __nv_bfloat16* dMT, int has_bias, int accumulate, int* status,
+                   __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
+                   __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate, int* status,
                    cudaStream_t st) {
   using C = Cfg<H>;
   cudaError_t e = cudaFuncSetAttribute(k_band_tc<H, BWD>,
@@ -471,8 +498,8 @@ cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& t
   if (e != cudaSuccess) return e;
   const int grid = std::min(p->K, num_sms());
   k_band_tc<H, BWD><<<grid, kThreads, C::SMEM, st>>>(
-      tx, tw, tdeg, tb2, BWD ? p->d_maskTI : p->d_maskI, out, dMT, p->K, p->P, p->n_pad(),
-      has_bias, accumulate, status);
+      tx, tw, tdeg, tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt,
+      p->K, p->P, has_bias, accumulate, status);
   note_launch();
   return cudaGetLastError();
 }
@@ -514,6 +541,58 @@ size_t band_tc_bwd_ws_bytes(const bg_plan* p, int dtype, int H) {
          al256(sizeof(float) * gemm_tn_part_floats(p->P * H, H + 16, (int64_t)n));
 }
 
+cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, int64_t ld_x,
+                             const __nv_bfloat16* WT, const __nv_bfloat16* b2T, float* out,
+                             __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
+                             int* status, cudaStream_t st) {
+  const int n = p->n_pad(), P = p->P;
+  CUtensorMap tx, tw, tdeg, tb2;
+  if (!make_map_ld(&tx, XT, H, n, ld_x, H) || !make_map(&tw, WT, (uint64_t)P * H, H, H) ||
+      !make_map(&tdeg, p->d_deg2, n, 64, kTile) || !make_map(&tb2, b2T ? b2T : WT, H, 64, H))
+    return cudaErrorInvalidValue;
+  const int has_bias = b2T != nullptr;
+  if (H == 64)
+    return launch<64, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, has_bias,
+                             0, status, st);
+  return launch<128, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, has_bias,
+                            0, status, st);
+}
+
+cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, int64_t ld_y,
+                             const void* W, float* dE, int accumulate, __nv_bfloat16* dMT,
+                             int64_t ld_mt, int* status, cudaStream_t st) {
+  const int n = p->n_pad(), P = p->P;
+  CUtensorMap tx, tw;
+  if (!make_map_ld(&tx, dYT, H, n, ld_y, H) || !make_map(&tw, W, (uint64_t)P * H, H, H))
+    return cudaErrorInvalidValue;
+  if (H == 64)
+    return launch<64, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
+                            status, st);
+  return launch<128, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
+                           status, st);
+}
+
+cudaError_t prep_transpose_bf16(const void* in, int in_is_f32, __nv_bfloat16* out, int R, int Cc,
+                                int batch, cudaStream_t st, int64_t ld_out) {
+  dim3 grid((Cc + 31) / 32, (R + 31) / 32, batch);
+  if (ld_out <= 0) ld_out = R;
+  if (in_is_f32)
+    k_transpose_bf16<float><<<grid, dim3(32, 8), 0, st>>>(static_cast<const float*>(in), out, R, Cc,
+                                                          (int64_t)R * Cc, (int64_t)R * Cc, ld_out);
+  else
+    k_transpose_bf16<__nv_bfloat16><<<grid, dim3(32, 8), 0, st>>>(
+        static_cast<const __nv_bfloat16*>(in), out, R, Cc, (int64_t)R * Cc, (int64_t)R * Cc,
+        ld_out);
+  note_launch();
+  return cudaGetLastError();
+}
+
+cudaError_t prep_bias_split(const float* b, __nv_bfloat16* b2T, int P, int H, cudaStream_t st) {
+  k_bias_split<<<(H * 64 + 255) / 256, 256, 0, st>>>(b, b2T, P, H);
+  note_launch();
+  return cudaGetLastError();
+}
+
 cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, const float* b,
                         float* Y, char* ws, size_t ws_bytes, int* status, cudaStream_t st) {
   if (ws_bytes < band_tc_fwd_ws_bytes(p, 1, H)) return cudaErrorInvalidValue;
@@ -523,23 +602,11 @@ cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, c
   __nv_bfloat16* b2T = reinterpret_cast<__nv_bfloat16*>(ws + al256((size_t)n * H * 2) +
                                                         al256((size_t)P * H * H * 2));
   // E [n][H] -> ET [H][n];  W_p [H_in][H_out] -> WT_p [H_out][H_in];  bias split
-  k_transpose_bf16<__nv_bfloat16><<<dim3((H + 31) / 32, (n + 31) / 32, 1), dim3(32, 8), 0, st>>>(
-      static_cast<const __nv_bfloat16*>(E), ET, n, H, 0, 0);
-  note_launch();
-  k_transpose_bf16<__nv_bfloat16><<<dim3((H + 31) / 32, (H + 31) / 32, P), dim3(32, 8), 0, st>>>(
-      static_cast<const __nv_bfloat16*>(W), WT, H, H, (int64_t)H * H, (int64_t)H * H);
-  note_launch();
-  const int has_bias = b != nullptr;
-  if (has_bias) {
-    k_bias_split<<<(H * 64 + 255) / 256, 256, 0, st>>>(b, b2T, P, H);
-    note_launch();
-  }
-  CUtensorMap tx, tw, tdeg, tb2;
-  if (!make_map(&tx, ET, H, n, H) || !make_map(&tw, WT, (uint64_t)P * H, H, H) ||
-      !make_map(&tdeg, p->d_deg2, n, 64, kTile) || !make_map(&tb2, b2T, H, 64, H))
-    return cudaErrorInvalidValue;
-  if (H == 64) return launch<64, false>(p, tx, tw, tdeg, tb2, Y, nullptr, has_bias, 0, status, st);
-  return launch<128, false>(p, tx, tw, tdeg, tb2, Y, nullptr, has_bias, 0, status, st);
+  cudaError_t e = prep_transpose_bf16(E, 0, ET, n, H, 1, st);
+  if (e == cudaSuccess) e = prep_transpose_bf16(W, 0, WT, H, H, P, st);
+  if (e == cudaSuccess && b) e = prep_bias_split(b, b2T, P, H, st);
+  if (e != cudaSuccess) return e;
+  return band_tc_fwd_core(p, H, ET, n, WT, b ? b2T : nullptr, Y, nullptr, nullptr, 0, status, st);
 }
 
 cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, const float* dY,
@@ -554,26 +621,15 @@ cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, c
   o += al256((size_t)P * H * n * 2);
   __nv_bfloat16* ETa = reinterpret_cast<__nv_bfloat16*>(ws + o);
   o += al256((size_t)(H + 16) * n * 2);
-  __nv_bfloat16* b2T = reinterpret_cast<__nv_bfloat16*>(ws + o);
   o += al256((size_t)H * 64 * 2);
   float* part = reinterpret_cast<float*>(ws + o);
   const size_t part_floats = gemm_tn_part_floats(P * H, H + 16, (int64_t)n);
-  k_transpose_bf16<float><<<dim3((H + 31) / 32, (n + 31) / 32, 1), dim3(32, 8), 0, st>>>(dY, dYT,
-                                                                                         n, H, 0, 0);
-  note_launch();
-  CUtensorMap tx, tw, tdeg, tb2;
-  if (!make_map(&tx, dYT, H, n, H) || !make_map(&tw, W, (uint64_t)P * H, H, H) ||
-      !make_map(&tdeg, p->d_deg2, n, 64, kTile) || !make_map(&tb2, b2T, H, 64, H))
-    return cudaErrorInvalidValue;
-  cudaError_t e = H == 64
-                      ? launch<64, true>(p, tx, tw, tdeg, tb2, dE, dMT, 0, accum, status, st)
-                      : launch<128, true>(p, tx, tw, tdeg, tb2, dE, dMT, 0, accum, status, st);
+  cudaError_t e = prep_transpose_bf16(dY, 1, dYT, n, H, 1, st);
+  if (e == cudaSuccess) e = band_tc_bwd_core(p, H, dYT, n, W, dE, accum, dMT, n, status, st);
   if (e != cudaSuccess) return e;
   // [E^T; 1; 0]: the ones row turns the bias gradient into column H of the same product
-  k_transpose_bf16<__nv_bfloat16><<<dim3((H + 31) / 32, (n + 31) / 32, 1), dim3(32, 8), 0, st>>>(
-      static_cast<const __nv_bfloat16*>(E), ETa, n, H, 0, 0);
-  note_launch();
-  e = fill_ones_rows(ETa, H, n, n, st);
+  e = prep_transpose_bf16(E, 0, ETa, n, H, 1, st);
+  if (e == cudaSuccess) e = fill_ones_rows(ETa, H, n, n, st);
   if (e != cudaSuccess) return e;
   // dW_p[h][h'] (+)= sum_nodes E[node][h] dM_p[node][h'],  db_p[h'] (+)= sum_nodes dM_p[node][h']
   return gemm_tn(dMT, n, ETa, n, P * H, H, n, 1, dW, db, accum, part, part_floats, status, st);

@@ -1,6 +1,7 @@
 // Tensor-core (tcgen05 / TMEM / TMA) band contractions for sm_103a.
 #pragma once
 
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include "internal.h"
@@ -18,6 +19,24 @@ cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, c
 cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, const float* dY,
                         float* dE, float* dW, float* db, int accum, char* ws, size_t ws_bytes,
                         int* status, cudaStream_t st);
+// Kernel-level entry points used by the fused GGNN steps (operands already in kernel layout):
+//   XT: [H][>= n_pad] bf16 transposed states (row stride ld_x); WT: [P][H_out][H_in] bf16;
+//   b2T: [H][64] bf16 bias split or NULL.  Outputs (each optional): out fp32 [n][H],
+//   outb bf16 [n][H], outT bf16 [H][ld_outT].
+cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, int64_t ld_x,
+                             const __nv_bfloat16* WT, const __nv_bfloat16* b2T, float* out,
+                             __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
+                             int* status, cudaStream_t st);
+//   dYT: [H][>= n_pad] bf16; W: [P][H][H] bf16 as given; dE fp32 (+)=; dMT: [P*H][ld_mt] bf16.
+cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, int64_t ld_y,
+                             const void* W, float* dE, int accumulate, __nv_bfloat16* dMT,
+                             int64_t ld_mt, int* status, cudaStream_t st);
+// out[c * ld_out + r] = bf16(in[r][c]) for `batch` consecutive R x Cc matrices (in fp32 or bf16;
+// ld_out <= 0 means R; batches are R*Cc apart on both sides).
+cudaError_t prep_transpose_bf16(const void* in, int in_is_f32, __nv_bfloat16* out, int R, int Cc,
+                                int batch, cudaStream_t st, int64_t ld_out = 0);
+// [H][64] bf16: columns p / 32+p hold the bf16 high part / remainder of b[p][h].
+cudaError_t prep_bias_split(const float* b, __nv_bfloat16* b2T, int P, int H, cudaStream_t st);
 // Builds and uploads the tensor-core path's plan data (no-op where unsupported); 0 on success.
 int band_tc_upload(bg_plan* p, cudaStream_t st);
 // Frees device data the tensor-core path keeps with the plan.

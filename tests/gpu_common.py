@@ -75,6 +75,9 @@ class Case:
                      for k, v in prm.items()}
         self.edges = (self.ref.kept_dst, self.ref.kept_src, self.ref.kept_type)
 
-    def ws(self, op):
-        n = L.workspace_bytes(self.plan, self.dtype, self.H, op)
+    def ws(self, op, T=1):
+        if op in (L.BG_OP_GGNN_FWD, L.BG_OP_GGNN_BWD):
+            n = L.ggnn_workspace_bytes(self.plan, self.dtype, self.H, T, op)
+        else:
+            n = L.workspace_bytes(self.plan, self.dtype, self.H, op)
         return torch.empty(n, dtype=torch.uint8, device="cuda")

@@ -122,7 +122,7 @@ def _ggnn(c: Case, T, seed=3):
     saved = torch.empty(L.ggnn_saved_bytes(c.plan, c.dtype, c.H, T), dtype=torch.uint8,
                         device="cuda")
     ET = torch.empty_like(c.E_band_dev)
-    L.ggnn_step(c.plan, c.dtype, c.H, T, c.dprm, c.E_band_dev, ET, saved, c.ws(L.BG_OP_GGNN_FWD))
+    L.ggnn_step(c.plan, c.dtype, c.H, T, c.dprm, c.E_band_dev, ET, saved, c.ws(L.BG_OP_GGNN_FWD, T))
     dET = quantize(np.random.default_rng(seed).standard_normal((c.N, c.H)), "f32")
     dE0 = torch.empty((c.N, c.H), dtype=torch.float32, device="cuda")
     grads = dict(dW=torch.empty((c.P, c.H, c.H), device="cuda"),
@@ -132,7 +132,7 @@ def _ggnn(c: Case, T, seed=3):
                  db_ih=torch.empty(3 * c.H, device="cuda"),
                  db_hh=torch.empty(3 * c.H, device="cuda"))
     L.ggnn_step_bwd(c.plan, c.dtype, c.H, T, c.dprm, saved, f32_dev(dET), dE0, grads,
-                    c.ws(L.BG_OP_GGNN_BWD))
+                    c.ws(L.BG_OP_GGNN_BWD, T))
     torch.cuda.synchronize()
     L.check_device()
     Es, Ys = oracle.ggnn_fwd(c.N, c.P, c.H, T, c.n_real, *c.edges, c.E_band, c.prm)

@@ -138,6 +138,8 @@ def test_device_calls_require_upload():
 
 def test_workspace_and_saved_sizes_are_positive():
     plan = L.band_plan(synth.config_graphs(1), 4, 64)
-    for op in range(5):
+    for op in (L.BG_OP_PROPAGATE_FWD, L.BG_OP_PROPAGATE_BWD, L.BG_OP_READOUT):
         assert L.workspace_bytes(plan, "f32", 64, op) > 0
+    for op in (L.BG_OP_GGNN_FWD, L.BG_OP_GGNN_BWD):
+        assert L.ggnn_workspace_bytes(plan, "f32", 64, 8, op) > 0
     assert L.ggnn_saved_bytes(plan, "bf16", 64, 8) >= 9 * 512 * 64 * 2 + 8 * 512 * 64 * 4
