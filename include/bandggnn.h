@@ -164,6 +164,23 @@ int bg_band_propagate_bwd(const bg_plan* plan, bg_dtype dtype, int32_t H, const 
                           const void* W, const float* dY, float* dE, float* dW, float* db,
                           uint32_t flags, void* ws, size_t ws_bytes, void* stream);
 
+/* Same result as bg_band_propagate_fwd, for callers that cannot allocate device memory while they
+ * run (no allocator of their own for the workspace, or cudaMalloc forbidden at that point): the
+ * scratch comes from a fixed 32 MiB array inside the library (static device memory, reserved on
+ * every GPU where the library's device code is loaded, until the process exits) instead of a
+ * caller workspace, and the call itself allocates nothing -- no cudaMalloc, cudaFree or allocating
+ * library routine.  The paper has no counterpart; this is a deployment variant.
+ * The plan must already be uploaded (bg_plan_upload allocates).  The first call on each device
+ * resolves the array's device address (cudaGetSymbolAddress, that device current), so make it
+ * before any stream capture.  Returns BG_ECAPACITY, with a message giving both sizes, when the
+ * plan needs more scratch than the array holds (bg_workspace_bytes(..., BG_OP_PROPAGATE_FWD) >
+ * 32 MiB).  All calls share the array: calls that overlap on the GPU (different streams, or
+ * different host threads without ordering) race and corrupt each other's results; serialise them.
+ * Bounded device waits that give up are recorded in a status word private to this entry point and
+ * are not reported by bg_check_device. */
+int bg_band_propagate_fwd_noalloc(const bg_plan* plan, bg_dtype dtype, int32_t H, const void* E,
+                                  const void* W, const float* b, float* Y, void* stream);
+
 /* ---- GGNN steps (device) --------------------------------------------------------------------
  * T steps of E(t+1) = GRU(sum_p A_p (E(t) W_p + b_p), E(t)) (Eq. 1; GRU of Cho et al.:
  * r = sigma(W_ir x + b_ir + W_hr h + b_hr), z likewise, n = tanh(W_in x + b_in + r (W_hn h + b_hn)),

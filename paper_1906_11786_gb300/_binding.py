@@ -81,6 +81,7 @@ def load(path: str = LIB_PATH):
         "bg_unpack_states": (c.c_int, [vp, c.c_int, i32, vp, vp, vp]),
         "bg_workspace_bytes": (sz, [vp, c.c_int, i32, i32]),
         "bg_band_propagate_fwd": (c.c_int, [vp, c.c_int, i32, vp, vp, vp, vp, vp, sz, vp]),
+        "bg_band_propagate_fwd_noalloc": (c.c_int, [vp, c.c_int, i32, vp, vp, vp, vp, vp]),
         "bg_band_propagate_bwd": (c.c_int, [vp, c.c_int, i32, vp, vp, vp, vp, vp, vp, c.c_uint32,
                                             vp, sz, vp]),
         "bg_ggnn_saved_bytes": (sz, [vp, c.c_int, i32, i32]),
@@ -255,6 +256,12 @@ def band_propagate_fwd(plan, dtype, H, E, W, b, Y, ws, stream=None):
                                         _dev_ptr(W, "W"), _dev_ptr(b, "b"), _dev_ptr(Y, "Y"),
                                         _dev_ptr(ws, "ws"), ws.numel() * ws.element_size(),
                                         _stream(stream)))
+
+
+def band_propagate_fwd_noalloc(plan, dtype, H, E, W, b, Y, stream=None):
+    _check(load().bg_band_propagate_fwd_noalloc(plan.handle, dtype_code(dtype), H, _dev_ptr(E, "E"),
+                                                _dev_ptr(W, "W"), _dev_ptr(b, "b"),
+                                                _dev_ptr(Y, "Y"), _stream(stream)))
 
 
 def band_propagate_bwd(plan, dtype, H, E, W, dY, dE, dW, db, ws, flags=0, stream=None):
