@@ -314,6 +314,42 @@ def run_reference(args):
     return 0
 
 
+def run_op(args, st, c):
+    """One band propagation call per step (forward or backward) on the workload's supergraph."""
+    import torch
+
+    from paper_1906_11786_gb300 import _binding as L
+    H = c["H"]
+    ws_f = torch.empty(L.workspace_bytes(st.plan, st.dt, H, L.BG_OP_PROPAGATE_FWD),
+                       dtype=torch.uint8, device="cuda")
+    ws_b = torch.empty(L.workspace_bytes(st.plan, st.dt, H, L.BG_OP_PROPAGATE_BWD),
+                       dtype=torch.uint8, device="cuda")
+
+    def one():
+        if args.op == "band_fwd":
+            L.band_propagate_fwd(st.plan, st.dt, H, st.E0, st.prm["W"], st.prm["b"], st.Y, ws_f)
+        else:
+            L.band_propagate_bwd(st.plan, st.dt, H, st.E0, st.prm["W"], st.dET, st.dE0,
+                                 st.grads["dW"], st.grads["db"], ws_b)
+
+    for _ in range(max(args.warmup, 3)):
+        one()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        one()
+    e1.record()
+    torch.cuda.synchronize()
+    L.check_device()
+    ms = e0.elapsed_time(e1) / args.steps
+    f = st.plan.flops(H, L.BG_FLOPS_BAND) + st.plan.flops(H, L.BG_FLOPS_XFORM)
+    print(json.dumps({"op": args.op, "ms_per_call": ms, "tflops": f / (ms / 1e3) / 1e12,
+                      "band_kernels": "tcgen05" if L.band_uses_tensor_cores(st.plan, st.dt, H)
+                      else "simt"}))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -325,6 +361,9 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--ref-budget", type=float, default=15.0)
+    ap.add_argument("--op", default="step", choices=["step", "band_fwd", "band_bwd"],
+                    help="time one band propagation kernel call instead of the whole step "
+                         "(focused profiling of the same workload)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -345,6 +384,8 @@ def main():
     st = OursStep(args.config, graphs, c, seed=rank)
     H, T = c["H"], c["T"]
     units = st.n_real * T  # node-steps per step on this rank
+    if args.op != "step":
+        return run_op(args, st, c)
 
     def barrier():
         if dist is not None:
@@ -413,15 +454,11 @@ def main():
     bwd_ms, bwd_n = kt[L.BG_KID_BAND_BWD]
     f_band = st.plan.flops(H, L.BG_FLOPS_BAND)
     f_xf = st.plan.flops(H, L.BG_FLOPS_XFORM)
-    # algorithmic FLOPs per launch: band-dense contraction + the fused edge-type transform
-    flops_fwd = f_band + f_xf
+    # algorithmic FLOPs per launch of either band kernel: band-dense contraction plus the fused
+    # edge-type transform chain (forward: pre_p W_p; backward: dM_p W_p^T)
+    flops = f_band + f_xf
     kern = "band_fwd" if fwd_ms >= bwd_ms else "band_bwd"
-    if kern == "band_fwd":
-        avg_ms = fwd_ms / max(fwd_n, 1)
-        flops = flops_fwd
-    else:
-        avg_ms = bwd_ms / max(bwd_n, 1)
-        flops = f_band + 2 * f_xf
+    avg_ms = (fwd_ms / max(fwd_n, 1)) if kern == "band_fwd" else (bwd_ms / max(bwd_n, 1))
     achieved = flops / (avg_ms / 1e3) / 1e12 if avg_ms > 0 else 0.0
     peak = pk["bf16_sustained"]
     roof = {"kernel": kern, "bound": "tensor", "achieved": achieved, "peak": peak,

@@ -24,6 +24,7 @@
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <vector>
@@ -40,7 +41,6 @@ using namespace tc;
 namespace {
 
 constexpr int kTile = 128;     // rows per tile = UMMA M
-constexpr int kThreads = 384;
 constexpr int kAtom = 64;      // bf16 per 128-byte swizzle row
 
 template <int H>
@@ -56,13 +56,17 @@ struct Cfg {
   static constexpr int OFF_W = OFF_X + NXB * XWIN;
   static constexpr int OFF_DEG = OFF_W + NW * WSTAGE;
   static constexpr int OFF_B2 = OFF_DEG + 2 * DEG;
-  static constexpr int OFF_BAR = OFF_B2 + B2;
+  static constexpr int NM = H <= 64 ? 6 : 2;                  // mask ring stages (one type each)
+  static constexpr int MSTAGE = 3 * kTile * 16;               // 3 diagonals x 128 rows x 128 bits
+  static constexpr int OFF_M = OFF_B2 + B2;
+  static constexpr int OFF_BAR = OFF_M + NM * MSTAGE;
   static constexpr int SMEM = OFF_BAR + 1024 + 1024;          // barriers + 1 KB alignment slack
-  // TMEM columns
+  // TMEM columns: Y, NB pre_p buffers, then the A-tile slots
+  static constexpr int NB = H <= 64 ? 3 : 2;
   static constexpr int YCOL = 0;
   static constexpr int D1COL0 = H;
-  static constexpr int ACOL = 3 * H;
-  static constexpr int NA = (512 - 3 * H) / 64;
+  static constexpr int ACOL = (NB + 1) * H;
+  static constexpr int NA = (512 - ACOL) / 64;
 };
 
 struct Bars {
@@ -71,8 +75,9 @@ struct Bars {
   uint64_t deg_full[2], deg_empty[2];
   uint64_t b2_full;
   uint64_t a_full[8], a_empty[8];
-  uint64_t d1_full[2], pre_ready[2];
+  uint64_t d1_full[4], pre_ready[4];
   uint64_t y_full, y_empty;
+  uint64_t m_full[8], m_empty[8];
   uint64_t drain;
   uint32_t tmem_base;
   int abort;
@@ -97,8 +102,8 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
-template <int H, bool BWD>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int H, bool BWD, int NE, int NC>
+__global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
     k_band_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
               const __grid_constant__ CUtensorMap tm_deg, const __grid_constant__ CUtensorMap tm_b2,
               const uint32_t* __restrict__ maskI, float* __restrict__ out,
@@ -114,6 +119,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* wring = smem + C::OFF_W;
   uint8_t* degs = smem + C::OFF_DEG;
   uint8_t* b2s = smem + C::OFF_B2;
+  uint8_t* mring = smem + C::OFF_M;
   volatile int* abort = &bars->abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -121,14 +127,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bars->x_full[i], 1); mbar_init(&bars->x_empty[i], 1);
       mbar_init(&bars->deg_full[i], 1); mbar_init(&bars->deg_empty[i], 1);
-      mbar_init(&bars->d1_full[i], 1); mbar_init(&bars->pre_ready[i], kTile);
     }
+    for (int i = 0; i < 4; ++i) { mbar_init(&bars->d1_full[i], 1); mbar_init(&bars->pre_ready[i], kTile); }
     for (int i = 0; i < 4; ++i) { mbar_init(&bars->w_full[i], 1); mbar_init(&bars->w_empty[i], 1); }
     for (int i = 0; i < 8; ++i) { mbar_init(&bars->a_full[i], kTile); mbar_init(&bars->a_empty[i], 1); }
     mbar_init(&bars->b2_full, 1);
     mbar_init(&bars->y_full, 1);
     mbar_init(&bars->y_empty, kTile);
     mbar_init(&bars->drain, 1);
+    for (int i = 0; i < 8; ++i) { mbar_init(&bars->m_full[i], 1); mbar_init(&bars->m_empty[i], kTile * NE); }
     bars->abort = 0;
     fence_mbar_init();
   }
@@ -151,12 +158,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_expect_tx(&bars->b2_full, C::B2);
       tma_load_2d(b2s, &tm_b2, &bars->b2_full, 0, 0);
     }
-    uint32_t widx = 0;
-    uint32_t n_x[2] = {0, 0}, n_deg[2] = {0, 0}, n_w[4] = {0, 0, 0, 0};
+    uint32_t widx = 0, midx = 0;
+    uint32_t n_x[2] = {0, 0}, n_deg[2] = {0, 0}, n_w[4] = {0, 0, 0, 0}, n_m[8] = {0};
     int i = 0;
     for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x, ++i) {
       const int xb = i % C::NXB;
-      if (!mbar_wait(&bars->x_empty[xb], ((i / C::NXB) & 1) ^ 1, status, 101, abort)) break;
+      if (!mbar_wait(&bars->x_empty[xb], ((i / C::NXB) & 1) ^ 1, status, 101, abort, 64)) break;
       ++n_x[xb];
       uint32_t bytes = 0;
       for (int d = 0; d < 3; ++d) {
@@ -173,19 +180,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (has_bias) {
         const int db = i & 1;
-        if (!mbar_wait(&bars->deg_empty[db], ((i >> 1) & 1) ^ 1, status, 102, abort)) break;
+        if (!mbar_wait(&bars->deg_empty[db], ((i >> 1) & 1) ^ 1, status, 102, abort, 64)) break;
         ++n_deg[db];
         mbar_expect_tx(&bars->deg_full[db], C::DEG);
         tma_load_2d(degs + db * C::DEG, &tm_deg, &bars->deg_full[db], 0, k * kTile);
       }
       for (int p = 0; p < P; ++p, ++widx) {
         const int ws = widx % C::NW;
-        if (!mbar_wait(&bars->w_empty[ws], ((widx / C::NW) & 1) ^ 1, status, 103, abort)) break;
+        if (!mbar_wait(&bars->w_empty[ws], ((widx / C::NW) & 1) ^ 1, status, 103, abort, 64)) break;
         ++n_w[ws];
         mbar_expect_tx(&bars->w_full[ws], C::WSTAGE);
         for (int a = 0; a < H / kAtom; ++a)
           tma_load_2d(wring + ws * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws], a * kAtom,
                       p * H);
+        // this type's three bit tiles (contiguous [3][128][4] words) for the expanders
+        const int ms = midx % C::NM;
+        if (!mbar_wait(&bars->m_empty[ms], ((midx / C::NM) & 1) ^ 1, status, 104, abort, 64)) break;
+        ++n_m[ms];
+        ++midx;
+        mbar_expect_tx(&bars->m_full[ms], C::MSTAGE);
+        bulk_load(mring + ms * C::MSTAGE, maskI + ((size_t)k * P + p) * 3 * kTile * 4, C::MSTAGE,
+                  &bars->m_full[ms]);
       }
     }
     if (*abort) {
@@ -197,17 +212,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       for (int q = 0; q < 2; ++q) { settle(&bars->x_full[q], n_x[q]); settle(&bars->deg_full[q], n_deg[q]); }
       for (int q = 0; q < 4; ++q) settle(&bars->w_full[q], n_w[q]);
+      for (int q = 0; q < 8; ++q) settle(&bars->m_full[q], n_m[q]);
       if (has_bias) settle(&bars->b2_full, 1);
     }
-  } else if (warp == 1 && lane == 0) {
+  } else if (warp == 1) {
     // ------------------------------------------------------------------ MMA issuer
+    // the whole warp runs this loop (its operands stay warp-uniform); one elected lane issues
+    const bool leader = elect_one_sync();
     constexpr uint32_t idesc = idesc_bf16_f32(kTile, H);
     uint32_t c = 0, aidx = 0, widx = 0;
     bool ok = true;
     int i = 0;
     auto stage2 = [&](uint32_t cc, bool first_in_tile, int tile_i) -> bool {
-      const int b = cc & 1;
-      if (!mbar_wait(&bars->pre_ready[b], (cc >> 1) & 1, status, 201, abort)) return false;
+      const int b = cc % C::NB;
+      if (!mbar_wait(&bars->pre_ready[b], (cc / C::NB) & 1, status, 201, abort)) return false;
       const int ws = widx % C::NW;
       if (!mbar_wait(&bars->w_full[ws], (widx / C::NW) & 1, status, 202, abort)) return false;
       if (first_in_tile &&
@@ -218,20 +236,23 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int kk = 0; kk < H / 16; ++kk) {
         const uint64_t bdesc = desc_sw128_kmajor(wbase + (kk / 4) * H * 128 + (kk % 4) * 32);
-        mma_ts(tmem + C::YCOL, tmem + C::D1COL0 + b * H + kk * 8, bdesc, idesc,
+        if (leader) mma_ts(tmem + C::YCOL, tmem + C::D1COL0 + b * H + kk * 8, bdesc, idesc,
                (first_in_tile && kk == 0) ? 0u : 1u);
       }
-      tc_commit(&bars->w_empty[ws]);
+      if (leader) tc_commit(&bars->w_empty[ws]);
       ++widx;
       return true;
     };
+    constexpr int LAG = C::NB - 1;  // stage 2 of type p - LAG follows stage 1 of type p
     for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x, ++i) {
       const int xb = i % C::NXB;
       if (!mbar_wait(&bars->x_full[xb], (i / C::NXB) & 1, status, 204, abort)) break;
       tc_fence_after();
       const uint32_t xbase = smem_u32(xwin + xb * C::XWIN);
+      const uint32_t c0 = c;
+      int next_s2 = 0;
       for (int p = 0; p < P && ok; ++p, ++c) {
-        const int b = c & 1;
+        const int b = c % C::NB;
         uint32_t first = 1;
         for (int d = 0; d < 3; ++d) {
           const int kb = k + d - 1;
@@ -243,24 +264,22 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int kk = 0; kk < kTile / 16; ++kk) {
             const uint64_t bdesc =
                 desc_sw128_kmajor(xbase + (d * 2 + kk / 4) * C::ATOM_X + (kk % 4) * 32);
-            mma_ts(tmem + C::D1COL0 + b * H, tmem + C::ACOL + slot * 64 + kk * 8, bdesc, idesc,
+            if (leader) mma_ts(tmem + C::D1COL0 + b * H, tmem + C::ACOL + slot * 64 + kk * 8, bdesc, idesc,
                    (first && kk == 0) ? 0u : 1u);
           }
           first = 0;
-          tc_commit(&bars->a_empty[slot]);
+          if (leader) tc_commit(&bars->a_empty[slot]);
           ++aidx;
         }
         if (!ok) break;
-        tc_commit(&bars->d1_full[b]);
-        if (p == P - 1) tc_commit(&bars->x_empty[xb]);
-        if (p >= 1 && !stage2(c - 1, p == 1, i)) { ok = false; break; }
+        if (leader) tc_commit(&bars->d1_full[b]);
+        if (p == P - 1) if (leader) tc_commit(&bars->x_empty[xb]);
+        for (; ok && next_s2 <= p - LAG; ++next_s2)
+          if (!stage2(c0 + next_s2, next_s2 == 0, i)) ok = false;
       }
+      for (; ok && next_s2 < P; ++next_s2)
+        if (!stage2(c0 + next_s2, next_s2 == 0, i)) ok = false;
       if (!ok) break;
-      if (P == 1) {
-        if (!stage2(c - 1, true, i)) break;
-      } else if (!stage2(c - 1, false, i)) {
-        break;
-      }
       if (has_bias) {
         const int db = i & 1;
         if (!mbar_wait(&bars->deg_full[db], (i >> 1) & 1, status, 206, abort)) break;
@@ -269,31 +288,43 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t dbase = smem_u32(degs + db * C::DEG), bbase = smem_u32(b2s);
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk)
-          mma_ss(tmem + C::YCOL, desc_sw128_kmajor(dbase + kk * 32),
+          if (leader) mma_ss(tmem + C::YCOL, desc_sw128_kmajor(dbase + kk * 32),
                  desc_sw128_kmajor(bbase + kk * 32), idesc, 1u);
-        tc_commit(&bars->deg_empty[db]);
+        if (leader) tc_commit(&bars->deg_empty[db]);
       }
-      tc_commit(&bars->y_full);
+      if (leader) tc_commit(&bars->y_full);
     }
     // every MMA issued above has completed once this commit arrives (bounded wait)
-    tc_commit(&bars->drain);
+    if (leader) tc_commit(&bars->drain);
+    __syncwarp();
     for (uint32_t t = 0; t < (1u << 24) && !mbar_try(&bars->drain, 0); ++t) {
     }
-  } else if (warp >= 4 && warp < 8) {
+  } else if (warp >= 4 && warp < 4 + 4 * NE) {
     // ------------------------------------------------------------------ expanders
-    const int r = threadIdx.x - 128;
+    // NE warpgroups take the 128 x 128 chunks in turn, so NE chunks are in flight at once
+    const int eg = (warp - 4) / 4;
+    const int r = threadIdx.x - 128 * (1 + eg);
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
-    uint32_t aidx = 0;
+    uint32_t aidx = 0, midx = 0;
     for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x) {
       bool ok = true;
-      for (int p = 0; p < P && ok; ++p) {
+      for (int p = 0; p < P && ok; ++p, ++midx) {
+        const int ms = midx % C::NM;
+        if (!mbar_wait(&bars->m_full[ms], (midx / C::NM) & 1, status, 302, abort, 32)) {
+          ok = false;
+          break;
+        }
+        const uint8_t* mrow = mring + ms * C::MSTAGE + r * 16;
         for (int d = 0; d < 3; ++d) {
           const int kb = k + d - 1;
           if (kb < 0 || kb >= K) continue;
-          const uint4 m = *reinterpret_cast<const uint4*>(
-              maskI + ((((size_t)k * P + p) * 3 + d) * kTile + r) * 4);
+          if ((int)(aidx % NE) != eg) {
+            ++aidx;
+            continue;
+          }
+          const uint4 m = *reinterpret_cast<const uint4*>(mrow + d * kTile * 16);
           const int slot = aidx % C::NA;
-          if (!mbar_wait(&bars->a_empty[slot], ((aidx / C::NA) & 1) ^ 1, status, 301, abort)) {
+          if (!mbar_wait(&bars->a_empty[slot], ((aidx / C::NA) & 1) ^ 1, status, 301, abort, 32)) {
             ok = false;
             break;
           }
@@ -310,12 +341,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_arrive(&bars->a_full[slot]);
           ++aidx;
         }
+        mbar_arrive(&bars->m_empty[ms]);
       }
       if (!ok) break;
     }
-  } else if (warp >= 8) {
+  } else if (warp >= 4 + 4 * NE) {
     // ------------------------------------------------------------------ converters / epilogue
-    const int r = threadIdx.x - 256;
+    // NC warpgroups take the edge types in turn (conversions overlap); group 0 also writes Y
+    const int cg = (warp - 4 - 4 * NE) / 4;
+    const int r = threadIdx.x - 128 * (1 + NE + cg);
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     uint32_t c = 0;
     int i = 0;
@@ -323,8 +357,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int row = k * kTile + r;
       bool ok = true;
       for (int p = 0; p < P; ++p, ++c) {
-        const int b = c & 1;
-        if (!mbar_wait(&bars->d1_full[b], (c >> 1) & 1, status, 401, abort)) { ok = false; break; }
+        if ((int)(c % NC) != cg) continue;
+        const int b = c % C::NB;
+        if (!mbar_wait(&bars->d1_full[b], (c / C::NB) & 1, status, 401, abort, 64)) { ok = false; break; }
         tc_fence_after();
         const uint32_t col = tmem + lane_base + C::D1COL0 + b * H;
         uint32_t v[32], q[32];
@@ -340,6 +375,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int j = 0; j < 16; ++j)
             pk[16 + j] = pack_bf16(__uint_as_float(q[2 * j]), __uint_as_float(q[2 * j + 1]));
+          // packed pairs of columns h0..h0+63 go to columns (h0/2)..(h0/2)+31 of the buffer
+          tmem_st32(col + h0 / 2, pk);
           if (BWD) {
             // dM_p (bf16) transposed: dMT[(p*H + h) * ld_mt + row]
 #pragma unroll
@@ -350,15 +387,14 @@ __global__ void __launch_bounds__(kThreads, 1)
               d[ld_mt] = __ushort_as_bfloat16((unsigned short)(w2 >> 16));
             }
           }
-          // packed pairs of columns h0..h0+63 go to columns (h0/2)..(h0/2)+31 of the buffer
-          tmem_st32(col + h0 / 2, pk);
         }
         tmem_wait_st();
         tc_fence_before();
         mbar_arrive(&bars->pre_ready[b]);
       }
       if (!ok) break;
-      if (!mbar_wait(&bars->y_full, i & 1, status, 402, abort)) break;
+      if (cg != 0) continue;
+      if (!mbar_wait(&bars->y_full, i & 1, status, 402, abort, 64)) break;
       tc_fence_after();
 #pragma unroll
       for (int h0 = 0; h0 < H; h0 += 32) {
@@ -486,22 +522,50 @@ int num_sms() {
 
 inline size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
 
+template <int H, bool BWD, int NE, int NC>
+cudaError_t launch_ne(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
+                   const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
+                   __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
+                   __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate, int* status,
+                   cudaStream_t st) {
+  using C = Cfg<H>;
+  cudaError_t e = cudaFuncSetAttribute(k_band_tc<H, BWD, NE, NC>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  const int grid = std::min(p->K, num_sms());
+  k_band_tc<H, BWD, NE, NC><<<grid, 128 * (NE + NC + 1), C::SMEM, st>>>(
+      tx, tw, tdeg, tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt,
+      p->K, p->P, has_bias, accumulate, status);
+  note_launch();
+  return cudaGetLastError();
+}
+
+int group_config() {
+  static int cfg = -1;
+  if (cfg < 0) {
+    const char* v = getenv("BG_BAND_GROUPS");
+    cfg = v ? atoi(v) : 11;
+    if (cfg != 11 && cfg != 12 && cfg != 21 && cfg != 22) cfg = 11;
+  }
+  return cfg;
+}
+
 template <int H, bool BWD>
 cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
                    const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
                    __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
                    __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate, int* status,
                    cudaStream_t st) {
-  using C = Cfg<H>;
-  cudaError_t e = cudaFuncSetAttribute(k_band_tc<H, BWD>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-  if (e != cudaSuccess) return e;
-  const int grid = std::min(p->K, num_sms());
-  k_band_tc<H, BWD><<<grid, kThreads, C::SMEM, st>>>(
-      tx, tw, tdeg, tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt,
-      p->K, p->P, has_bias, accumulate, status);
-  note_launch();
-  return cudaGetLastError();
+#define BG_LAUNCH_NE(NEV, NCV)                                                                    \
+  return launch_ne<H, BWD, NEV, NCV>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, dMT, ld_mt, \
+                                     has_bias, accumulate, status, st);
+  switch (group_config()) {
+    case 21: BG_LAUNCH_NE(2, 1)
+    case 22: BG_LAUNCH_NE(2, 2)
+    case 12: BG_LAUNCH_NE(1, 2)
+    default: BG_LAUNCH_NE(1, 1)
+  }
+#undef BG_LAUNCH_NE
 }
 
 }  // namespace

@@ -56,16 +56,28 @@ __device__ __forceinline__ bool mbar_try(uint64_t* bar, uint32_t parity) {
 }
 
 // Waits for phase `parity` of `bar` to complete; false (and a recorded timeout) if the poll
-// limit is reached or another role already gave up (*abort set).
+// limit is reached or another role already gave up (*abort set).  backoff_ns > 0 sleeps between
+// polls so that waiting warps leave issue slots to the warps doing the work (the MMA issuer polls
+// with backoff_ns = 0).
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* status, int site,
-                                          volatile int* abort) {
+                                          volatile int* abort, uint32_t backoff_ns = 0) {
   for (uint32_t i = 0; i < kSpinLimit; ++i) {
     if (mbar_try(bar, parity)) return true;
     if ((i & 1023u) == 1023u && *abort) return false;
+    if (backoff_ns) __nanosleep(backoff_ns);
   }
   if (atomicCAS(status, 0, 1) == 0) atomicExch(status + 1, site);
   *abort = 1;
   return false;
+}
+
+// One lane of a converged warp (the lane that issues tcgen05.mma / commit for the whole warp).
+__device__ __forceinline__ bool elect_one_sync() {
+  uint32_t pred;
+  asm volatile(
+      "{\n.reg .pred P;\n.reg .b32 R;\nelect.sync R|P, 0xffffffff;\nselp.u32 %0, 1, 0, P;\n}"
+      : "=r"(pred));
+  return pred != 0;
 }
 
 // ------------------------------------------------------------------------------ TMA
@@ -79,6 +91,15 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* m, uin
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, "
       "%4}], [%2];" ::"r"(smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+
+// 1-D bulk copy global -> shared (16-byte aligned addresses, size a multiple of 16)
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
       : "memory");
 }
 
