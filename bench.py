@@ -39,6 +39,26 @@ def _peaks():
     return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "src": "fallback"}
 
 
+def _profiled_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary of `workload`, or None when
+    there is none or the kernel's source changed since it was captured."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"k_band_tc_{kernel}_{workload}.md")
+    if not os.path.exists(path):
+        return None
+    vals = {}
+    for line in open(path):
+        if ":" in line and line.split(":")[0] in ("dram_bytes_per_launch", "source_sha256_16"):
+            k, v = line.split(":", 1)
+            vals[k.strip()] = v.strip()
+    m = hashlib.sha256()
+    for f in ("band_tc.cu", "tc_util.cuh"):
+        m.update(open(os.path.join(ROOT, "paper_1906_11786_gb300", "csrc", f), "rb").read())
+    if vals.get("source_sha256_16") != m.hexdigest()[:16] or "dram_bytes_per_launch" not in vals:
+        return None
+    return int(vals["dram_bytes_per_launch"])
+
+
 def _dist():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -62,7 +82,7 @@ class Clocks:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
@@ -124,6 +144,18 @@ def workload(config: int, rank: int, S=None, H=None):
     if c["sizes"][0] == "fill":
         cap = -(-c["sizes"][1] // S)
     return graphs, dict(c, S=S, H=H, P=P, cap=cap)
+
+
+def reduce_over_ranks(dist, ms: float, units: float, device="cuda"):
+    """Whole-job aggregation: the slowest rank's time and the node-steps of all ranks."""
+    if dist is None:
+        return ms, units
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    u = torch.tensor([units], dtype=torch.float64, device=device)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u.item())
 
 
 class OursStep:
@@ -353,7 +385,7 @@ def run_op(args, st, c):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--config", type=int, default=2)
     ap.add_argument("--S", type=int, default=None)
@@ -418,15 +450,7 @@ def main():
     ms = ev0.elapsed_time(ev1)
     L.check_device()
     kt = {k: L.profile_read(k, reset=True) for k in range(5)}
-    if dist is not None:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-        u = torch.tensor([float(units)], device="cuda")
-        dist.all_reduce(u)
-        total_units = float(u.item())
-    else:
-        total_units = float(units)
+    ms, total_units = reduce_over_ranks(dist, ms, float(units))
     ms_step = ms / args.steps
     value = total_units / (ms_step / 1e3)
 
@@ -442,10 +466,7 @@ def main():
     e1.record(stream)
     torch.cuda.synchronize()
     e_ms = e0.elapsed_time(e1) / args.steps
-    if dist is not None:
-        t = torch.tensor([e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e_ms = float(t.item())
+    e_ms, _ = reduce_over_ranks(dist, e_ms, 0.0)
     e2e_value = total_units / (e_ms / 1e3)
 
     # ---- roofline of the dominant kernel (band contraction)
@@ -461,8 +482,11 @@ def main():
     avg_ms = (fwd_ms / max(fwd_n, 1)) if kern == "band_fwd" else (bwd_ms / max(bwd_n, 1))
     achieved = flops / (avg_ms / 1e3) / 1e12 if avg_ms > 0 else 0.0
     peak = pk["bf16_sustained"]
+    traffic = _profiled_traffic(kern.split("_")[1], synth.CONFIGS[args.config]["name"])
     roof = {"kernel": kern, "bound": "tensor", "achieved": achieved, "peak": peak,
-            "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+            "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
+            "traffic_src": "profiles/ ncu capture (dram read+write bytes per launch)"
+            if traffic else None,
             "peak_src": f"{pk['src']} bf16 sustained",
             "kernel_ms": {k: (kt[i][0] / max(kt[i][1], 1)) for i, k in
                           enumerate(["band_fwd", "band_bwd", "gru_fwd", "gru_bwd", "dW"])},

@@ -84,7 +84,7 @@ __global__ void __launch_bounds__(192, 1)
     uint32_t issued[kStages] = {0, 0, 0, 0};
     for (int kc = kc0, it = 0; kc < kc1; ++kc, ++it) {
       const int s = it % kStages;
-      if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1, status, 501, abort)) break;
+      if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1, status, 501, abort, 32)) break;
       ++issued[s];
       mbar_expect_tx(&full[s], C::STAGE);
       uint8_t* st = smem + s * C::STAGE;
@@ -95,7 +95,9 @@ __global__ void __launch_bounds__(192, 1)
       for (int s = 0; s < kStages; ++s)
         for (uint32_t t = 0; issued[s] && t < (1u << 22) && !mbar_try(&full[s], (issued[s] - 1) & 1); ++t) {
         }
-  } else if (warp == 1 && lane == 0) {
+  } else if (warp == 1) {
+    // the whole warp runs the loop (uniform operands); one elected lane issues
+    const bool leader = elect_one_sync();
     constexpr uint32_t idesc = idesc_bf16_f32(128, BN);
     for (int kc = kc0, it = 0; kc < kc1; ++kc, ++it) {
       const int s = it % kStages;
@@ -104,18 +106,23 @@ __global__ void __launch_bounds__(192, 1)
       const uint32_t a = smem_u32(smem + s * C::STAGE), b = a + C::A_BYTES;
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk)
-        mma_ss(tmem, desc_sw128_kmajor(a + kk * 32), desc_sw128_kmajor(b + kk * 32), idesc,
-               (kc > kc0 || kk > 0) ? 1u : 0u);
-      tc_commit(&empty[s]);
+        if (leader)
+          mma_ss(tmem, desc_sw128_kmajor(a + kk * 32), desc_sw128_kmajor(b + kk * 32), idesc,
+                 (kc > kc0 || kk > 0) ? 1u : 0u);
+      if (leader) tc_commit(&empty[s]);
+      __syncwarp();
     }
-    tc_commit(done);
-    tc_commit(drain);
+    if (leader) {
+      tc_commit(done);
+      tc_commit(drain);
+    }
+    __syncwarp();
     for (uint32_t t = 0; t < (1u << 24) && !mbar_try(drain, 0); ++t) {
     }
   } else if (warp >= 2) {
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int m = mt * 128 + q * 32 + lane;
-    if (mbar_wait(done, 0, status, 503, abort)) {
+    if (mbar_wait(done, 0, status, 503, abort, 256)) {
       tc_fence_after();
       float* out = part + ((size_t)split * M + m) * N + blockIdx.y * BN;
 #pragma unroll
