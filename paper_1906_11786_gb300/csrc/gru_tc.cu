@@ -1,18 +1,25 @@
-// GRU cell (Cho et al.; named in Section 2 and Algorithm 1) forward and backward on tcgen05, one
-// 128-row tile of nodes per CTA.  Gate convention: rows r, z, n of W_ih / W_hh;
+// GRU cell (Cho et al.; named in Section 2 and Algorithm 1) forward and backward on tcgen05.
+// Gate convention: rows r, z, n of W_ih / W_hh;
 //   r = sigma(Wi_r x + b_ir + Wh_r h + b_hr),  z = sigma(Wi_z x + b_iz + Wh_z h + b_hz),
 //   n = tanh(Wi_n x + b_in + r (Wh_n h + b_hn)),  h' = (1 - z) n + z h,
 // with x the summed messages Y and h the state E; padding rows stay 0.
 //
-// Pre-activations live in TMEM: [r|z] = Y Wi_rz^T + E Wh_rz^T (2H columns, both products
+// Pre-activations live in TMEM: [r|z] = Y Wi_rz^T + E Wh_rz^T (2H columns: both products
 // accumulate into one tile), Wi_n x (H) and Wh_n h (H).  The forward epilogue applies the gates
 // and writes E(t+1) row-major and transposed (the next band product's operand).  The backward
 // recomputes the same products, forms the gate gradients in registers, writes them back into the
 // TMEM columns it has just read as the bf16 A operand of dX = dgi W_ih and dH = dgh W_hh (chained
-// MMAs), and stores dX^T (the transposed-band operand), the running state gradient and dgi^T,
-// dgh^T for the weight-gradient GEMM.
+// MMAs that accumulate into the freed Wi_n x / Wh_n h columns), and stores dX^T (the
+// transposed-band operand), the running state gradient and dgi^T, dgh^T for the weight gradients.
+//
+// Both kernels are persistent (one CTA per SM) and warp-specialised: warp 0 streams 128-row
+// tiles of Y and E through a two-stage TMA ring (the weights stay resident), warp 1 issues the
+// MMAs into two TMEM accumulator sets, and two epilogue warpgroups (one per 32-column half) drain
+// them, so loads and MMAs of tile i+1 overlap the epilogue of tile i.
 #include <cuda.h>
 #include <cuda_bf16.h>
+
+#include <algorithm>
 
 #include "gemm_tc.h"
 #include "gru_tc.h"
@@ -25,16 +32,25 @@ using namespace tc;
 
 namespace {
 
-constexpr int kH = 64;  // state size handled by these kernels
+constexpr int kH = 64;        // state size handled by these kernels
+constexpr int kThreads = 384; // warp 0 TMA, warp 1 MMA, warps 4-11 epilogue (two groups)
+constexpr int kAcc = 4 * kH;  // TMEM columns per accumulator set
 
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t* r) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr),
+               "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]),
+               "r"(r[7])
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
   asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-      "%14,%15,%16};" ::"r"(taddr),
-      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
-      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
-      "r"(r[15])
-      : "memory");
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
 }
 
 __device__ __forceinline__ uint32_t pk2(float lo, float hi) {
@@ -61,99 +77,194 @@ __device__ __forceinline__ void read_sw128_row32(const uint8_t* tile, int r, int
   }
 }
 
+// 16 consecutive bf16 of row r (columns c0 .. c0+15, c0 % 16 == 0) of the same tile layout.
+__device__ __forceinline__ void read_sw128_row16(const uint8_t* tile, int r, int c0, float* out) {
+  const uint8_t* row = tile + (c0 / 64) * 128 * 128 + r * 128;
+  const int j0 = (c0 % 64) / 8;
+#pragma unroll
+  for (int q = 0; q < 2; ++q) {
+    const uint4 v = *reinterpret_cast<const uint4*>(row + (((j0 + q) ^ (r & 7)) << 4));
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      out[q * 8 + 2 * e] = __uint_as_float(w[e] << 16);
+      out[q * 8 + 2 * e + 1] = __uint_as_float(w[e] & 0xFFFF0000u);
+    }
+  }
+}
+
+// 8 bf16 pairs stored transposed: dst[(h0 + 2j + u) * ld + row]
+__device__ __forceinline__ void store_T8(__nv_bfloat16* dst, int64_t ld, int row, int h0,
+                                         const uint32_t* pk) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    __nv_bfloat16* t = dst + (size_t)(h0 + 2 * j) * ld + row;
+    t[0] = __ushort_as_bfloat16((unsigned short)(pk[j] & 0xFFFFu));
+    t[ld] = __ushort_as_bfloat16((unsigned short)(pk[j] >> 16));
+  }
+}
+
+// 32 bf16 pairs (64 values of consecutive rows) stored transposed: dst[(h0 + 2j + u) * ld + row]
+__device__ __forceinline__ void store_T16(__nv_bfloat16* dst, int64_t ld, int row, int h0,
+                                          const uint32_t* pk) {
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    __nv_bfloat16* t = dst + (size_t)(h0 + 2 * j) * ld + row;
+    t[0] = __ushort_as_bfloat16((unsigned short)(pk[j] & 0xFFFFu));
+    t[ld] = __ushort_as_bfloat16((unsigned short)(pk[j] >> 16));
+  }
+}
+
 struct GruSmem {
-  static constexpr int TILE = 128 * 128;           // 128 rows x 64 bf16
-  static constexpr int W = 3 * kH * 128;           // [3H][H] bf16
-  static constexpr int WT = 3 * kH * 128;          // [H][3H] bf16 as three 64-column atoms
-  static constexpr int OFF_Y = 0, OFF_E = TILE, OFF_WIH = 2 * TILE, OFF_WHH = OFF_WIH + W;
-  static constexpr int OFF_WIHT = OFF_WHH + W, OFF_WHHT = OFF_WIHT + WT;
-  static constexpr int FWD = OFF_WIHT + 1024 + 1024;
-  static constexpr int BWD = OFF_WHHT + WT + 1024 + 1024;
+  static constexpr int TILE = 128 * 128;  // 128 rows x 64 bf16
+  static constexpr int W = 3 * kH * 128;  // [3H][H] bf16 (also [H][3H] as three 64-column atoms)
+  static constexpr int FWD_T = 2 * W;     // tile ring after W_ih, W_hh
+  static constexpr int BWD_T = 4 * W;     // tile ring after W_ih, W_hh, W_ih^T, W_hh^T
+  static constexpr int FWD = FWD_T + 4 * TILE + 2048;
+  static constexpr int BWD = BWD_T + 4 * TILE + 2048;
 };
 
-// Issues [r|z], Wi_n x, Wh_n h for the tile (K = H = 64: four K=16 steps).
-__device__ __forceinline__ void gru_gate_mmas(uint32_t tmem, uint32_t sY, uint32_t sE, uint32_t sWih,
+struct GruBars {
+  uint64_t w_full, t_full[2], t_empty[2], acc_full[2], acc_empty[2], ops_ready[2], ph2_full[2];
+  uint64_t drain;
+  uint32_t tmem_slot;
+  int abort;
+};
+
+// Issues [r|z], Wi_n x, Wh_n h for one tile into the accumulator set at `acc` (K = H = 64).
+__device__ __forceinline__ void gru_gate_mmas(uint32_t acc, uint32_t sY, uint32_t sE, uint32_t sWih,
                                               uint32_t sWhh) {
   constexpr uint32_t id_rz = idesc_bf16_f32(128, 2 * kH), id_h = idesc_bf16_f32(128, kH);
 #pragma unroll
   for (int kk = 0; kk < 4; ++kk) {
     const uint64_t aY = desc_sw128_kmajor(sY + kk * 32), aE = desc_sw128_kmajor(sE + kk * 32);
-    mma_ss(tmem + 0, aY, desc_sw128_kmajor(sWih + kk * 32), id_rz, kk > 0);
-    mma_ss(tmem + 0, aE, desc_sw128_kmajor(sWhh + kk * 32), id_rz, 1u);
-    mma_ss(tmem + 2 * kH, aY, desc_sw128_kmajor(sWih + 2 * kH * 128 + kk * 32), id_h, kk > 0);
-    mma_ss(tmem + 3 * kH, aE, desc_sw128_kmajor(sWhh + 2 * kH * 128 + kk * 32), id_h, kk > 0);
+    mma_ss(acc + 0, aY, desc_sw128_kmajor(sWih + kk * 32), id_rz, kk > 0);
+    mma_ss(acc + 0, aE, desc_sw128_kmajor(sWhh + kk * 32), id_rz, 1u);
+    mma_ss(acc + 2 * kH, aY, desc_sw128_kmajor(sWih + 2 * kH * 128 + kk * 32), id_h, kk > 0);
+    mma_ss(acc + 3 * kH, aE, desc_sw128_kmajor(sWhh + 2 * kH * 128 + kk * 32), id_h, kk > 0);
   }
 }
 
-__global__ void __launch_bounds__(128, 1)
-    k_gru_fwd_tc(const __grid_constant__ CUtensorMap tY, const __grid_constant__ CUtensorMap tE,
-                 const __grid_constant__ CUtensorMap tWih, const __grid_constant__ CUtensorMap tWhh,
-                 const float* __restrict__ b_ih, const float* __restrict__ b_hh,
-                 __nv_bfloat16* __restrict__ En, __nv_bfloat16* __restrict__ EnT, int64_t ld_T,
-                 int n_real, int* status) {
-  using G = GruSmem;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~uintptr_t(1023));
-  __shared__ uint64_t full, done;
-  __shared__ uint32_t tmem_slot;
-  __shared__ int abort_flag;
-  __shared__ float bias[6 * kH];
-  volatile int* abort = &abort_flag;
-  const int warp = threadIdx.x >> 5, r = threadIdx.x;
+// Common prologue: barrier init, bias copy, TMEM allocation (512 columns: two accumulator sets).
+__device__ __forceinline__ void gru_setup(GruBars* b, float* bias, const float* b_ih,
+                                          const float* b_hh, int warp) {
   for (int t = threadIdx.x; t < 3 * kH; t += blockDim.x) {
     bias[t] = b_ih[t];
     bias[3 * kH + t] = b_hh[t];
   }
   if (threadIdx.x == 0) {
-    mbar_init(&full, 1);
-    mbar_init(&done, 1);
-    abort_flag = 0;
+    mbar_init(&b->w_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&b->t_full[i], 1);
+      mbar_init(&b->t_empty[i], 256);
+      mbar_init(&b->acc_full[i], 1);
+      mbar_init(&b->acc_empty[i], 256);
+      mbar_init(&b->ops_ready[i], 256);
+      mbar_init(&b->ph2_full[i], 1);
+    }
+    mbar_init(&b->drain, 1);
+    b->abort = 0;
     fence_mbar_init();
   }
-  if (warp == 0) {
-    tmem_alloc(&tmem_slot, 256);
+  if (warp == 1) {
+    tmem_alloc(&b->tmem_slot, 512);
     tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = tmem_slot;
-  const int tile = blockIdx.x;
-  bool ok = true;
-  if (threadIdx.x == 0) {
-    mbar_expect_tx(&full, 2 * G::TILE + 2 * G::W);
-    tma_load_2d(smem + G::OFF_Y, &tY, &full, 0, tile * 128);
-    tma_load_2d(smem + G::OFF_E, &tE, &full, 0, tile * 128);
-    tma_load_2d(smem + G::OFF_WIH, &tWih, &full, 0, 0);
-    tma_load_2d(smem + G::OFF_WHH, &tWhh, &full, 0, 0);
-    if (mbar_wait(&full, 0, status, 601, abort)) {
-      tc_fence_after();
-      gru_gate_mmas(tmem, smem_u32(smem + G::OFF_Y), smem_u32(smem + G::OFF_E),
-                    smem_u32(smem + G::OFF_WIH), smem_u32(smem + G::OFF_WHH));
-      tc_commit(&done);
-    } else {
-      for (uint32_t t = 0; t < (1u << 22) && !mbar_try(&full, 0); ++t) {
+}
+
+// Tile producer shared by both kernels: two-stage ring of (Y, E) tiles.
+__device__ __forceinline__ void gru_produce_tiles(GruBars* b, uint8_t* ring,
+                                                  const CUtensorMap* tY, const CUtensorMap* tE,
+                                                  int n_tiles, int* status, volatile int* abort) {
+  uint32_t issued[2] = {0, 0};
+  int i = 0;
+  for (int t = blockIdx.x; t < n_tiles && !*abort; t += gridDim.x, ++i) {
+    const int s = i & 1;
+    if (!mbar_wait(&b->t_empty[s], ((i >> 1) & 1) ^ 1, status, 611, abort, 64)) break;
+    ++issued[s];
+    mbar_expect_tx(&b->t_full[s], 2 * GruSmem::TILE);
+    tma_load_2d(ring + s * 2 * GruSmem::TILE, tY, &b->t_full[s], 0, t * 128);
+    tma_load_2d(ring + s * 2 * GruSmem::TILE + GruSmem::TILE, tE, &b->t_full[s], 0, t * 128);
+  }
+  if (*abort)
+    for (int s = 0; s < 2; ++s)
+      for (uint32_t k = 0; issued[s] && k < (1u << 22) && !mbar_try(&b->t_full[s], (issued[s] - 1) & 1); ++k) {
+      }
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_gru_fwd_tc(const __grid_constant__ CUtensorMap tY, const __grid_constant__ CUtensorMap tE,
+                 const __grid_constant__ CUtensorMap tWih, const __grid_constant__ CUtensorMap tWhh,
+                 const float* __restrict__ b_ih, const float* __restrict__ b_hh,
+                 __nv_bfloat16* __restrict__ En, __nv_bfloat16* __restrict__ EnT, int64_t ld_T,
+                 int n_tiles, int n_real, int* status) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  __shared__ GruBars bars;
+  __shared__ float bias[6 * kH];
+  volatile int* abort = &bars.abort;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  gru_setup(&bars, bias, b_ih, b_hh, warp);
+  const uint32_t tmem = bars.tmem_slot;
+  uint8_t* ring = smem + GruSmem::FWD_T;
+
+  if (warp == 0 && lane == 0) {
+    mbar_expect_tx(&bars.w_full, 2 * GruSmem::W);
+    tma_load_2d(smem, &tWih, &bars.w_full, 0, 0);
+    tma_load_2d(smem + GruSmem::W, &tWhh, &bars.w_full, 0, 0);
+    gru_produce_tiles(&bars, ring, &tY, &tE, n_tiles, status, abort);
+    if (*abort)
+      for (uint32_t k = 0; k < (1u << 22) && !mbar_try(&bars.w_full, 0); ++k) {
+      }
+  } else if (warp == 1) {
+    const bool leader = elect_one_sync();
+    if (mbar_wait(&bars.w_full, 0, status, 612, abort)) {
+      int i = 0;
+      for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
+        const int s = i & 1, a = i & 1;
+        if (!mbar_wait(&bars.t_full[s], (i >> 1) & 1, status, 613, abort)) break;
+        if (!mbar_wait(&bars.acc_empty[a], ((i >> 1) & 1) ^ 1, status, 614, abort)) break;
+        tc_fence_after();
+        const uint32_t sY = smem_u32(ring + s * 2 * GruSmem::TILE);
+        if (leader) {
+          gru_gate_mmas(tmem + a * kAcc, sY, sY + GruSmem::TILE, smem_u32(smem),
+                        smem_u32(smem + GruSmem::W));
+          tc_commit(&bars.acc_full[a]);
+        }
+        __syncwarp();
       }
     }
-  }
-  __syncwarp();
-  ok = mbar_wait(&done, 0, status, 602, abort);
-  if (ok) {
-    tc_fence_after();
-    const int row = tile * 128 + r;
-    const uint32_t lb = (uint32_t)(warp * 32) << 16;
-    const bool real = row < n_real;
-#pragma unroll
-    for (int h0 = 0; h0 < kH; h0 += 32) {
+    if (leader) tc_commit(&bars.drain);
+    __syncwarp();
+    for (uint32_t k = 0; k < (1u << 24) && !mbar_try(&bars.drain, 0); ++k) {
+    }
+  } else if (warp >= 4) {
+    const int g = (warp - 4) / 4, h0 = 32 * g;
+    const int r = (warp & 3) * 32 + lane;
+    const uint32_t lb = (uint32_t)((warp & 3) * 32) << 16;
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
+      const int s = i & 1, a = i & 1;
+      if (!mbar_wait(&bars.acc_full[a], (i >> 1) & 1, status, 615, abort, 64)) break;
+      tc_fence_after();
+      const uint32_t acc = tmem + lb + a * kAcc;
       uint32_t vr[32], vz[32], vn[32], vh[32];
-      tmem_ld32(tmem + lb + h0, vr);
-      tmem_ld32(tmem + lb + kH + h0, vz);
-      tmem_ld32(tmem + lb + 2 * kH + h0, vn);
-      tmem_ld32(tmem + lb + 3 * kH + h0, vh);
+      tmem_ld32(acc + h0, vr);
+      tmem_ld32(acc + kH + h0, vz);
+      tmem_ld32(acc + 2 * kH + h0, vn);
+      tmem_ld32(acc + 3 * kH + h0, vh);
       tmem_wait_ld();
       float e[32];
-      read_sw128_row32(smem + G::OFF_E, r, h0, e);
+      read_sw128_row32(ring + s * 2 * GruSmem::TILE + GruSmem::TILE, r, h0, e);
+      tc_fence_before();
+      mbar_arrive(&bars.acc_empty[a]);
+      mbar_arrive(&bars.t_empty[s]);
+      const int row = t * 128 + r;
+      const bool real = row < n_real;
       uint32_t pk[16];
 #pragma unroll
       for (int j = 0; j < 32; j += 2) {
@@ -172,209 +283,200 @@ __global__ void __launch_bounds__(128, 1)
       uint4* d = reinterpret_cast<uint4*>(En + (size_t)row * kH + h0);
 #pragma unroll
       for (int q = 0; q < 4; ++q) d[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
-      if (EnT) {
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          __nv_bfloat16* t = EnT + (size_t)(h0 + 2 * j) * ld_T + row;
-          t[0] = __ushort_as_bfloat16((unsigned short)(pk[j] & 0xFFFFu));
-          t[ld_T] = __ushort_as_bfloat16((unsigned short)(pk[j] >> 16));
-        }
-      }
+      if (EnT) store_T16(EnT, ld_T, row, h0, pk);
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) {
+  if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem, 256);
+    tmem_dealloc(tmem, 512);
   }
 }
 
-// TMEM columns of the backward kernel
-constexpr int kDX = 4 * kH, kDH = 5 * kH;
-// A-operand column of gate-gradient K step kk (16 values of one gate) after the in-place rewrite
+// A-operand column (relative to an accumulator set) of gate-gradient K step kk (16 values of one
+// gate) after the in-place rewrite.  Columns h in [32c + 16sb, +16) of chunk c, sub-chunk sb, are
+// read and then overwritten as: r window [32c + 16sb, +16) = (dgi_r | dgi_z) pairs, z window
+// [H + 32c + 16sb, +16) = (dgi_n | dgh_n) pairs; dgh_r = dgi_r and dgh_z = dgi_z.
 __device__ __forceinline__ uint32_t dg_col(int kk, bool hidden) {
   const int gate = kk / 4, hh = (kk % 4) * 16, c = hh / 32, sb = (hh % 32) / 16;
-  if (gate == 0) return c * 32 + sb * 8;
-  if (gate == 1) return c * 32 + 16 + sb * 8;
-  return kH + c * 32 + (hidden ? 16 : 0) + sb * 8;
+  const int base = c * 32 + sb * 16;
+  if (gate == 0) return base;
+  if (gate == 1) return base + 8;
+  return kH + base + (hidden ? 8 : 0);
 }
 
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     k_gru_bwd_tc(const __grid_constant__ CUtensorMap tY, const __grid_constant__ CUtensorMap tE,
                  const __grid_constant__ CUtensorMap tWih, const __grid_constant__ CUtensorMap tWhh,
                  const __grid_constant__ CUtensorMap tWihT, const __grid_constant__ CUtensorMap tWhhT,
                  const float* __restrict__ b_ih, const float* __restrict__ b_hh,
                  const float* __restrict__ gin, float* __restrict__ gout,
                  __nv_bfloat16* __restrict__ dXT, int64_t ld_x, __nv_bfloat16* __restrict__ dgiT,
-                 __nv_bfloat16* __restrict__ dghT, int64_t ld_g, int n_real, int* status) {
-  using G = GruSmem;
+                 __nv_bfloat16* __restrict__ dghT, int64_t ld_g, int n_tiles, int n_real,
+                 int* status) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  __shared__ uint64_t full, done1, done2;
-  __shared__ uint32_t tmem_slot;
-  __shared__ int abort_flag;
+  __shared__ GruBars bars;
   __shared__ float bias[6 * kH];
-  volatile int* abort = &abort_flag;
-  const int warp = threadIdx.x >> 5, r = threadIdx.x;
-  for (int t = threadIdx.x; t < 3 * kH; t += blockDim.x) {
-    bias[t] = b_ih[t];
-    bias[3 * kH + t] = b_hh[t];
-  }
-  if (threadIdx.x == 0) {
-    mbar_init(&full, 1);
-    mbar_init(&done1, 1);
-    mbar_init(&done2, 1);
-    abort_flag = 0;
-    fence_mbar_init();
-  }
-  if (warp == 0) {
-    tmem_alloc(&tmem_slot, 512);
-    tmem_relinquish();
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = tmem_slot;
-  const int tile = blockIdx.x;
-  if (threadIdx.x == 0) {
-    mbar_expect_tx(&full, 2 * G::TILE + 2 * G::W + 2 * G::WT);
-    tma_load_2d(smem + G::OFF_Y, &tY, &full, 0, tile * 128);
-    tma_load_2d(smem + G::OFF_E, &tE, &full, 0, tile * 128);
-    tma_load_2d(smem + G::OFF_WIH, &tWih, &full, 0, 0);
-    tma_load_2d(smem + G::OFF_WHH, &tWhh, &full, 0, 0);
+  volatile int* abort = &bars.abort;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  gru_setup(&bars, bias, b_ih, b_hh, warp);
+  const uint32_t tmem = bars.tmem_slot;
+  uint8_t* ring = smem + GruSmem::BWD_T;
+
+  if (warp == 0 && lane == 0) {
+    mbar_expect_tx(&bars.w_full, 4 * GruSmem::W);
+    tma_load_2d(smem, &tWih, &bars.w_full, 0, 0);
+    tma_load_2d(smem + GruSmem::W, &tWhh, &bars.w_full, 0, 0);
     for (int a = 0; a < 3; ++a) {
-      tma_load_2d(smem + G::OFF_WIHT + a * kH * 128, &tWihT, &full, a * 64, 0);
-      tma_load_2d(smem + G::OFF_WHHT + a * kH * 128, &tWhhT, &full, a * 64, 0);
+      tma_load_2d(smem + 2 * GruSmem::W + a * kH * 128, &tWihT, &bars.w_full, a * 64, 0);
+      tma_load_2d(smem + 3 * GruSmem::W + a * kH * 128, &tWhhT, &bars.w_full, a * 64, 0);
     }
-    if (mbar_wait(&full, 0, status, 701, abort)) {
-      tc_fence_after();
-      gru_gate_mmas(tmem, smem_u32(smem + G::OFF_Y), smem_u32(smem + G::OFF_E),
-                    smem_u32(smem + G::OFF_WIH), smem_u32(smem + G::OFF_WHH));
-      tc_commit(&done1);
-    } else {
-      for (uint32_t t = 0; t < (1u << 22) && !mbar_try(&full, 0); ++t) {
+    gru_produce_tiles(&bars, ring, &tY, &tE, n_tiles, status, abort);
+    if (*abort)
+      for (uint32_t k = 0; k < (1u << 22) && !mbar_try(&bars.w_full, 0); ++k) {
       }
-    }
-  }
-  __syncwarp();
-  const int row = tile * 128 + r;
-  const uint32_t lb = (uint32_t)(warp * 32) << 16;
-  const bool real = row < n_real;
-  float dhd[kH];
-  bool ok = mbar_wait(&done1, 0, status, 702, abort);
-  if (ok) {
-    tc_fence_after();
-#pragma unroll
-    for (int c = 0; c < 2; ++c) {
-      const int h0 = 32 * c;
-      uint32_t vr[32], vz[32], vn[32], vh[32];
-      tmem_ld32(tmem + lb + h0, vr);
-      tmem_ld32(tmem + lb + kH + h0, vz);
-      tmem_ld32(tmem + lb + 2 * kH + h0, vn);
-      tmem_ld32(tmem + lb + 3 * kH + h0, vh);
-      tmem_wait_ld();
-      float e[32];
-      read_sw128_row32(smem + G::OFF_E, r, h0, e);
-      const float4* g4 = reinterpret_cast<const float4*>(gin + (size_t)row * kH + h0);
-      uint32_t p_r[16], p_z[16], p_n[16], p_hn[16];
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const float4 gv = g4[q];
-        const float gg[4] = {gv.x, gv.y, gv.z, gv.w};
-        float dr[4], dz[4], dn[4], dhn[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int j = 4 * q + u, h = h0 + j;
-          const float rr = sigm(__uint_as_float(vr[j]) + bias[h] + bias[3 * kH + h]);
-          const float zz = sigm(__uint_as_float(vz[j]) + bias[kH + h] + bias[4 * kH + h]);
-          const float ghn = __uint_as_float(vh[j]) + bias[5 * kH + h];
-          const float nn = tanhf(__uint_as_float(vn[j]) + bias[2 * kH + h] + rr * ghn);
-          const float g = real ? gg[u] : 0.f;
-          const float an = g * (1.f - zz) * (1.f - nn * nn);
-          dn[u] = an;
-          dhn[u] = an * rr;
-          dr[u] = an * ghn * rr * (1.f - rr);
-          dz[u] = g * (e[j] - nn) * zz * (1.f - zz);
-          dhd[h] = g * zz;
-        }
-        p_r[2 * q] = pk2(dr[0], dr[1]); p_r[2 * q + 1] = pk2(dr[2], dr[3]);
-        p_z[2 * q] = pk2(dz[0], dz[1]); p_z[2 * q + 1] = pk2(dz[2], dz[3]);
-        p_n[2 * q] = pk2(dn[0], dn[1]); p_n[2 * q + 1] = pk2(dn[2], dn[3]);
-        p_hn[2 * q] = pk2(dhn[0], dhn[1]); p_hn[2 * q + 1] = pk2(dhn[2], dhn[3]);
-      }
-      // in-place rewrite into the columns read above (this chunk's windows only)
-      tmem_st16(tmem + lb + c * 32, p_r);
-      tmem_st16(tmem + lb + c * 32 + 16, p_z);
-      tmem_st16(tmem + lb + kH + c * 32, p_n);
-      tmem_st16(tmem + lb + kH + c * 32 + 16, p_hn);
-      // gate gradients transposed for the weight-gradient GEMM: rows o = gate*H + h
-#pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const int h = h0 + 2 * j;
-        const uint32_t w4[4] = {p_r[j], p_z[j], p_n[j], p_hn[j]};
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const unsigned short b_r = (unsigned short)(u ? w4[0] >> 16 : w4[0] & 0xFFFFu);
-          const unsigned short b_z = (unsigned short)(u ? w4[1] >> 16 : w4[1] & 0xFFFFu);
-          const unsigned short b_n = (unsigned short)(u ? w4[2] >> 16 : w4[2] & 0xFFFFu);
-          const unsigned short b_hn = (unsigned short)(u ? w4[3] >> 16 : w4[3] & 0xFFFFu);
-          const size_t col = (size_t)row;
-          dgiT[(size_t)(h + u) * ld_g + col] = __ushort_as_bfloat16(b_r);
-          dgiT[(size_t)(kH + h + u) * ld_g + col] = __ushort_as_bfloat16(b_z);
-          dgiT[(size_t)(2 * kH + h + u) * ld_g + col] = __ushort_as_bfloat16(b_n);
-          dghT[(size_t)(h + u) * ld_g + col] = __ushort_as_bfloat16(b_r);
-          dghT[(size_t)(kH + h + u) * ld_g + col] = __ushort_as_bfloat16(b_z);
-          dghT[(size_t)(2 * kH + h + u) * ld_g + col] = __ushort_as_bfloat16(b_hn);
-        }
-      }
-    }
-    tmem_wait_st();
-  }
-  tc_fence_before();
-  __syncthreads();
-  if (threadIdx.x == 0 && ok && !*abort) {
-    tc_fence_after();
+  } else if (warp == 1) {
+    const bool leader = elect_one_sync();
     constexpr uint32_t id_h = idesc_bf16_f32(128, kH);
-    const uint32_t sIT = smem_u32(smem + G::OFF_WIHT), sHT = smem_u32(smem + G::OFF_WHHT);
+    const uint32_t sIT = smem_u32(smem + 2 * GruSmem::W), sHT = smem_u32(smem + 3 * GruSmem::W);
+    // dX = dgi W_ih, dH = dgh W_hh for tile j (accumulating into the freed n columns)
+    auto phase2 = [&](int j) -> bool {
+      const int a = j & 1;
+      if (!mbar_wait(&bars.ops_ready[a], (j >> 1) & 1, status, 621, abort)) return false;
+      tc_fence_after();
+      if (leader) {
+        const uint32_t acc = tmem + a * kAcc;
 #pragma unroll
-    for (int kk = 0; kk < 12; ++kk) {
-      const uint32_t boff = (kk / 4) * kH * 128 + (kk % 4) * 32;
-      mma_ts(tmem + kDX, tmem + dg_col(kk, false), desc_sw128_kmajor(sIT + boff), id_h, kk > 0);
-      mma_ts(tmem + kDH, tmem + dg_col(kk, true), desc_sw128_kmajor(sHT + boff), id_h, kk > 0);
-    }
-    tc_commit(&done2);
-  }
-  __syncwarp();
-  if (ok && mbar_wait(&done2, 0, status, 703, abort)) {
-    tc_fence_after();
-#pragma unroll
-    for (int h0 = 0; h0 < kH; h0 += 32) {
-      uint32_t vx[32], vd[32];
-      tmem_ld32(tmem + lb + kDX + h0, vx);
-      tmem_ld32(tmem + lb + kDH + h0, vd);
-      tmem_wait_ld();
-#pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const uint32_t w = pk2(__uint_as_float(vx[2 * j]), __uint_as_float(vx[2 * j + 1]));
-        __nv_bfloat16* t = dXT + (size_t)(h0 + 2 * j) * ld_x + row;
-        t[0] = __ushort_as_bfloat16((unsigned short)(w & 0xFFFFu));
-        t[ld_x] = __ushort_as_bfloat16((unsigned short)(w >> 16));
+        for (int kk = 0; kk < 12; ++kk) {
+          const uint32_t boff = (kk / 4) * kH * 128 + (kk % 4) * 32;
+          mma_ts(acc + 2 * kH, acc + dg_col(kk, false), desc_sw128_kmajor(sIT + boff), id_h, kk > 0);
+          mma_ts(acc + 3 * kH, acc + dg_col(kk, true), desc_sw128_kmajor(sHT + boff), id_h, kk > 0);
+        }
+        tc_commit(&bars.ph2_full[a]);
       }
+      __syncwarp();
+      return true;
+    };
+    if (mbar_wait(&bars.w_full, 0, status, 622, abort)) {
+      int i = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++i) {
+        const int s = i & 1, a = i & 1;
+        if (!mbar_wait(&bars.t_full[s], (i >> 1) & 1, status, 623, abort)) break;
+        if (!mbar_wait(&bars.acc_empty[a], ((i >> 1) & 1) ^ 1, status, 624, abort)) break;
+        tc_fence_after();
+        const uint32_t sY = smem_u32(ring + s * 2 * GruSmem::TILE);
+        if (leader) {
+          gru_gate_mmas(tmem + a * kAcc, sY, sY + GruSmem::TILE, smem_u32(smem),
+                        smem_u32(smem + GruSmem::W));
+          tc_commit(&bars.acc_full[a]);
+        }
+        __syncwarp();
+        if (i >= 1) ok = phase2(i - 1);
+      }
+      if (ok && i >= 1) phase2(i - 1);
+    }
+    if (leader) tc_commit(&bars.drain);
+    __syncwarp();
+    for (uint32_t k = 0; k < (1u << 24) && !mbar_try(&bars.drain, 0); ++k) {
+    }
+  } else if (warp >= 4) {
+    const int c = (warp - 4) / 4, h0 = 32 * c;
+    const int r = (warp & 3) * 32 + lane;
+    const uint32_t lb = (uint32_t)((warp & 3) * 32) << 16;
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
+      const int s = i & 1, a = i & 1;
+      const int row = t * 128 + r;
+      const bool real = row < n_real;
+      if (!mbar_wait(&bars.acc_full[a], (i >> 1) & 1, status, 625, abort, 64)) break;
+      tc_fence_after();
+      const uint32_t acc = tmem + lb + a * kAcc;
+      const uint8_t* etile = ring + s * 2 * GruSmem::TILE + GruSmem::TILE;
+      float dhd[32];
+#pragma unroll
+      for (int sb = 0; sb < 2; ++sb) {
+        const int hs = h0 + 16 * sb;
+        uint32_t vr[16], vz[16], vn[16], vh[16];
+        tmem_ld16(acc + hs, vr);
+        tmem_ld16(acc + kH + hs, vz);
+        tmem_ld16(acc + 2 * kH + hs, vn);
+        tmem_ld16(acc + 3 * kH + hs, vh);
+        tmem_wait_ld();
+        float e[16];
+        read_sw128_row16(etile, r, hs, e);
+        const float4* g4 = reinterpret_cast<const float4*>(gin + (size_t)row * kH + hs);
+        uint32_t p_r[8], p_z[8], p_n[8], p_hn[8];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float4 gv = g4[q];
+          const float gg[4] = {gv.x, gv.y, gv.z, gv.w};
+          float dr[4], dz[4], dn[4], dhn[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int j = 4 * q + u, h = hs + j;
+            const float rr = sigm(__uint_as_float(vr[j]) + bias[h] + bias[3 * kH + h]);
+            const float zz = sigm(__uint_as_float(vz[j]) + bias[kH + h] + bias[4 * kH + h]);
+            const float ghn = __uint_as_float(vh[j]) + bias[5 * kH + h];
+            const float nn = tanhf(__uint_as_float(vn[j]) + bias[2 * kH + h] + rr * ghn);
+            const float gr = real ? gg[u] : 0.f;
+            const float an = gr * (1.f - zz) * (1.f - nn * nn);
+            dn[u] = an;
+            dhn[u] = an * rr;
+            dr[u] = an * ghn * rr * (1.f - rr);
+            dz[u] = gr * (e[j] - nn) * zz * (1.f - zz);
+            dhd[16 * sb + j] = gr * zz;
+          }
+          p_r[2 * q] = pk2(dr[0], dr[1]); p_r[2 * q + 1] = pk2(dr[2], dr[3]);
+          p_z[2 * q] = pk2(dz[0], dz[1]); p_z[2 * q + 1] = pk2(dz[2], dz[3]);
+          p_n[2 * q] = pk2(dn[0], dn[1]); p_n[2 * q + 1] = pk2(dn[2], dn[3]);
+          p_hn[2 * q] = pk2(dhn[0], dhn[1]); p_hn[2 * q + 1] = pk2(dhn[2], dhn[3]);
+        }
+        // in-place rewrite into the columns just read (see dg_col)
+        tmem_st8(acc + hs, p_r);
+        tmem_st8(acc + hs + 8, p_z);
+        tmem_st8(acc + kH + hs, p_n);
+        tmem_st8(acc + kH + hs + 8, p_hn);
+        // gate gradients transposed for the weight-gradient GEMM: rows o = gate*H + h
+        store_T8(dgiT, ld_g, row, hs, p_r);
+        store_T8(dgiT + (size_t)kH * ld_g, ld_g, row, hs, p_z);
+        store_T8(dgiT + (size_t)2 * kH * ld_g, ld_g, row, hs, p_n);
+        store_T8(dghT, ld_g, row, hs, p_r);
+        store_T8(dghT + (size_t)kH * ld_g, ld_g, row, hs, p_z);
+        store_T8(dghT + (size_t)2 * kH * ld_g, ld_g, row, hs, p_hn);
+      }
+      mbar_arrive(&bars.t_empty[s]);
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(&bars.ops_ready[a]);
+      if (!mbar_wait(&bars.ph2_full[a], (i >> 1) & 1, status, 626, abort, 64)) break;
+      tc_fence_after();
+      uint32_t vx[32], vd[32];
+      tmem_ld32(acc + 2 * kH + h0, vx);
+      tmem_ld32(acc + 3 * kH + h0, vd);
+      tmem_wait_ld();
+      tc_fence_before();
+      mbar_arrive(&bars.acc_empty[a]);
+      uint32_t px[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) px[j] = pk2(__uint_as_float(vx[2 * j]), __uint_as_float(vx[2 * j + 1]));
+      store_T16(dXT, ld_x, row, h0, px);
       float4* go = reinterpret_cast<float4*>(gout + (size_t)row * kH + h0);
 #pragma unroll
       for (int q = 0; q < 8; ++q)
-        go[q] = make_float4(dhd[h0 + 4 * q] + __uint_as_float(vd[4 * q]),
-                            dhd[h0 + 4 * q + 1] + __uint_as_float(vd[4 * q + 1]),
-                            dhd[h0 + 4 * q + 2] + __uint_as_float(vd[4 * q + 2]),
-                            dhd[h0 + 4 * q + 3] + __uint_as_float(vd[4 * q + 3]));
+        go[q] = make_float4(dhd[4 * q] + __uint_as_float(vd[4 * q]),
+                            dhd[4 * q + 1] + __uint_as_float(vd[4 * q + 1]),
+                            dhd[4 * q + 2] + __uint_as_float(vd[4 * q + 2]),
+                            dhd[4 * q + 3] + __uint_as_float(vd[4 * q + 3]));
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) {
+  if (warp == 1) {
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem, 512);
@@ -397,8 +499,10 @@ cudaError_t gru_fwd_tc(int n_pad, int n_real, const __nv_bfloat16* Y, const __nv
   cudaError_t e = cudaFuncSetAttribute(k_gru_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        GruSmem::FWD);
   if (e != cudaSuccess) return e;
-  k_gru_fwd_tc<<<n_pad / 128, 128, GruSmem::FWD, st>>>(tY, tE, tWi, tWh, b_ih, b_hh, En, EnT, ld_T,
-                                                      n_real, status);
+  const int n_tiles = n_pad / 128;
+  const int grid = std::min(n_tiles, gemm_tn_num_sms());
+  k_gru_fwd_tc<<<grid, kThreads, GruSmem::FWD, st>>>(tY, tE, tWi, tWh, b_ih, b_hh, En, EnT, ld_T,
+                                                     n_tiles, n_real, status);
   note_launch();
   return cudaGetLastError();
 }
@@ -419,9 +523,11 @@ cudaError_t gru_bwd_tc(int n_pad, int n_real, const __nv_bfloat16* Y, const __nv
   cudaError_t e = cudaFuncSetAttribute(k_gru_bwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        GruSmem::BWD);
   if (e != cudaSuccess) return e;
-  k_gru_bwd_tc<<<n_pad / 128, 128, GruSmem::BWD, st>>>(tY, tE, tWi, tWh, tWiT, tWhT, b_ih, b_hh,
-                                                      gin, gout, dXT, ld_x, dgiT, dghT, ld_g,
-                                                      n_real, status);
+  const int n_tiles = n_pad / 128;
+  const int grid = std::min(n_tiles, gemm_tn_num_sms());
+  k_gru_bwd_tc<<<grid, kThreads, GruSmem::BWD, st>>>(tY, tE, tWi, tWh, tWiT, tWhT, b_ih, b_hh, gin,
+                                                     gout, dXT, ld_x, dgiT, dghT, ld_g, n_tiles,
+                                                     n_real, status);
   note_launch();
   return cudaGetLastError();
 }
