@@ -15,11 +15,13 @@
 // each 32-column word are interleaved at upload (column 2j at bit j, column 2j+1 at bit 16+j) so
 // that one AND and one multiply give the packed bf16 pair {1.0 or 0, 1.0 or 0}.
 //
-// Roles (384 threads, one CTA per SM, persistent over tiles):
+// Roles (128 x (1 + NE + NC) threads, one CTA per SM, persistent over tiles):
 //   warp 0      TMA producer: state blocks (B operand of the band product), W tiles, deg, bias
-//   warp 1      TMEM allocator; lane 0 issues every tcgen05.mma
-//   warps 4-7   expanders: thread r turns row r's mask bits into bf16 A tiles in TMEM
-//   warps 8-11  converters: pre_p fp32 -> bf16 in place; final epilogue TMEM -> global
+//   warp 1      TMEM allocator; an elected lane of the converged warp issues every tcgen05.mma
+//   warp 2      mask producer: one bulk copy per (tile, type) of the bit tiles into an SMEM ring
+//   next NE warpgroups   expanders: thread r turns row r's mask bits into bf16 A tiles in TMEM
+//   last NC warpgroups   converters: pre_p fp32 -> bf16 in place; final epilogue TMEM -> global
+// Waiting roles sleep between polls so that the MMA issuer keeps its issue slots.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
@@ -56,7 +58,7 @@ struct Cfg {
   static constexpr int OFF_W = OFF_X + NXB * XWIN;
   static constexpr int OFF_DEG = OFF_W + NW * WSTAGE;
   static constexpr int OFF_B2 = OFF_DEG + 2 * DEG;
-  static constexpr int NM = H <= 64 ? 6 : 2;                  // mask ring stages (one type each)
+  static constexpr int NM = H <= 64 ? 8 : 2;                  // mask ring stages (one type each)
   static constexpr int MSTAGE = 3 * kTile * 16;               // 3 diagonals x 128 rows x 128 bits
   static constexpr int OFF_M = OFF_B2 + B2;
   static constexpr int OFF_BAR = OFF_M + NM * MSTAGE;
@@ -158,8 +160,8 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
       mbar_expect_tx(&bars->b2_full, C::B2);
       tma_load_2d(b2s, &tm_b2, &bars->b2_full, 0, 0);
     }
-    uint32_t widx = 0, midx = 0;
-    uint32_t n_x[2] = {0, 0}, n_deg[2] = {0, 0}, n_w[4] = {0, 0, 0, 0}, n_m[8] = {0};
+    uint32_t widx = 0;
+    uint32_t n_x[2] = {0, 0}, n_deg[2] = {0, 0}, n_w[4] = {0, 0, 0, 0};
     int i = 0;
     for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x, ++i) {
       const int xb = i % C::NXB;
@@ -193,14 +195,6 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
         for (int a = 0; a < H / kAtom; ++a)
           tma_load_2d(wring + ws * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws], a * kAtom,
                       p * H);
-        // this type's three bit tiles (contiguous [3][128][4] words) for the expanders
-        const int ms = midx % C::NM;
-        if (!mbar_wait(&bars->m_empty[ms], ((midx / C::NM) & 1) ^ 1, status, 104, abort, 64)) break;
-        ++n_m[ms];
-        ++midx;
-        mbar_expect_tx(&bars->m_full[ms], C::MSTAGE);
-        bulk_load(mring + ms * C::MSTAGE, maskI + ((size_t)k * P + p) * 3 * kTile * 4, C::MSTAGE,
-                  &bars->m_full[ms]);
       }
     }
     if (*abort) {
@@ -212,9 +206,31 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
       };
       for (int q = 0; q < 2; ++q) { settle(&bars->x_full[q], n_x[q]); settle(&bars->deg_full[q], n_deg[q]); }
       for (int q = 0; q < 4; ++q) settle(&bars->w_full[q], n_w[q]);
-      for (int q = 0; q < 8; ++q) settle(&bars->m_full[q], n_m[q]);
       if (has_bias) settle(&bars->b2_full, 1);
     }
+  } else if (warp == 2 && lane == 0) {
+    // ------------------------------------------------------------------ mask producer
+    // each type's three bit tiles (contiguous [3][128][4] words), NM types ahead of the expanders
+    uint32_t midx = 0, n_m[8] = {0};
+    for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x) {
+      bool ok = true;
+      for (int p = 0; p < P; ++p, ++midx) {
+        const int ms = midx % C::NM;
+        if (!mbar_wait(&bars->m_empty[ms], ((midx / C::NM) & 1) ^ 1, status, 104, abort, 64)) {
+          ok = false;
+          break;
+        }
+        ++n_m[ms];
+        mbar_expect_tx(&bars->m_full[ms], C::MSTAGE);
+        bulk_load(mring + ms * C::MSTAGE, maskI + ((size_t)k * P + p) * 3 * kTile * 4, C::MSTAGE,
+                  &bars->m_full[ms]);
+      }
+      if (!ok) break;
+    }
+    if (*abort)
+      for (int q = 0; q < 8; ++q)
+        for (uint32_t t = 0; n_m[q] && t < (1u << 22) && !mbar_try(&bars->m_full[q], (n_m[q] - 1) & 1); ++t) {
+        }
   } else if (warp == 1) {
     // ------------------------------------------------------------------ MMA issuer
     // the whole warp runs this loop (its operands stay warp-uniform); one elected lane issues
