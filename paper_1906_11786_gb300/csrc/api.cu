@@ -323,14 +323,20 @@ FwdWs fwd_ws(const bg_plan* p, bg_dtype dt, int H) {
   size_t n = (size_t)p->n_pad();
   w.M = 0;
   size_t band = bg::band_tc_fwd_ws_bytes(p, (int)dt, H);
-  size_t simt = al(sizeof(float) * (size_t)p->P * n * H);
+  size_t simt = al(sizeof(float) * (size_t)p->P * n * H) + al((size_t)p->P * H * H * 2);
   w.band = 0;
   w.total = std::max(band, simt);
   return w;
 }
 
+// bf16 shapes the fused kernels do not cover still run their products on the tensor cores (the
+// band sums stay SIMT gathers over the bit tiles); the split-K gradient GEMM needs H <= 128.
+bool tc_gemm_path(bg_dtype dt, int H) { return dt == BG_BF16 && H <= 128; }
+
 struct BwdWs {
-  size_t dM, Wt, part, total;
+  size_t dM, Wt, part;                 // fp32 SIMT path
+  size_t dMb, dMT, Wp, ETa, tpart;     // bf16 path with tensor-core GEMMs
+  size_t total;
 };
 BwdWs bwd_ws(const bg_plan* p, bg_dtype dt, int H) {
   BwdWs w{};
@@ -339,12 +345,22 @@ BwdWs bwd_ws(const bg_plan* p, bg_dtype dt, int H) {
   w.dM = o; o += al(sizeof(float) * n * p->P * H);
   w.Wt = o; o += al(sizeof(float) * (size_t)p->P * H * H);
   w.part = o; o += al(sizeof(float) * part_floats(p, H));
-  w.total = std::max(o, bg::band_tc_bwd_ws_bytes(p, (int)dt, H));
+  size_t total = o;
+  if (tc_gemm_path(dt, H)) {
+    size_t q = 0;
+    w.dMb = q; q += al(n * p->P * H * 2);
+    w.dMT = q; q += al(n * p->P * H * 2);
+    w.Wp = q; q += al((size_t)p->P * H * H * 2);
+    w.ETa = q; q += al((size_t)(H + 16) * n * 2);
+    w.tpart = q; q += al(sizeof(float) * bg::gemm_tn_part_floats(p->P * H, H + 16, (int64_t)n));
+    total = std::max(total, q);
+  }
+  w.total = std::max(total, bg::band_tc_bwd_ws_bytes(p, (int)dt, H));
   return w;
 }
 
 struct GgnnFwdWs {
-  size_t gi, gh, prop, part, total;
+  size_t gi, gh, Ybf, prop, part, total;
 };
 GgnnFwdWs ggnn_fwd_ws(const bg_plan* p, bg_dtype dt, int H) {
   GgnnFwdWs w{};
@@ -352,6 +368,7 @@ GgnnFwdWs ggnn_fwd_ws(const bg_plan* p, bg_dtype dt, int H) {
   size_t o = 0;
   w.gi = o; o += al(sizeof(float) * n * 3 * H);
   w.gh = o; o += al(sizeof(float) * n * 3 * H);
+  w.Ybf = o; o += al(n * H * 2);
   w.part = o; o += al(sizeof(float) * part_floats(p, H));
   w.prop = o; o += al(fwd_ws(p, dt, H).total);
   w.total = o;
@@ -359,12 +376,29 @@ GgnnFwdWs ggnn_fwd_ws(const bg_plan* p, bg_dtype dt, int H) {
 }
 
 struct GgnnBwdWs {
-  size_t gi, gh, dgi, dgh, dX, g, part, prop, total;
+  size_t gi, gh, dgi, dgh, dX, g, part, prop;
+  size_t Ybf, dgib, dghb, dgiT, dghT, YTa, ETa, WihT, WhhT, tpart;  // tensor-core GEMM path
+  size_t total;
 };
+size_t gru_tpart_floats(const bg_plan* p, int H) {
+  return bg::gemm_tn_part_floats(3 * H, H + 16, (int64_t)p->n_pad());
+}
 GgnnBwdWs ggnn_bwd_ws(const bg_plan* p, bg_dtype dt, int H) {
   GgnnBwdWs w{};
   size_t n = (size_t)p->n_pad();
   size_t o = 0;
+  if (tc_gemm_path(dt, H)) {
+    w.Ybf = o; o += al(n * H * 2);
+    w.dgib = o; o += al(n * 3 * H * 2);
+    w.dghb = o; o += al(n * 3 * H * 2);
+    w.dgiT = o; o += al(n * 3 * H * 2);
+    w.dghT = o; o += al(n * 3 * H * 2);
+    w.YTa = o; o += al((size_t)(H + 16) * n * 2);
+    w.ETa = o; o += al((size_t)(H + 16) * n * 2);
+    w.WihT = o; o += al((size_t)3 * H * H * 2);
+    w.WhhT = o; o += al((size_t)3 * H * H * 2);
+    w.tpart = o; o += al(sizeof(float) * gru_tpart_floats(p, H));
+  }
   w.gi = o; o += al(sizeof(float) * n * 3 * H);
   w.gh = o; o += al(sizeof(float) * n * 3 * H);
   w.dgi = o; o += al(sizeof(float) * n * 3 * H);
@@ -520,13 +554,23 @@ static int propagate_fwd_impl(const bg_plan* p, bg_dtype dt, int H, const void* 
   float* M = reinterpret_cast<float*>(ws);
   if (ws_bytes < sizeof(float) * (size_t)p->P * n * H) return bg_fail(BG_ECAPACITY, "workspace too small");
   KTimer t(BG_KID_BAND_FWD, st);
-  bg::Gemm g;
-  g.M = (int)n; g.N = H; g.K = H; g.batch = p->P;
-  g.A = E; g.a_bf16 = bf; g.sAb = 0; g.sAm = H; g.sAk = 1;
-  g.B = W; g.b_bf16 = bf; g.sBb = (int64_t)H * H; g.sBk = H; g.sBn = 1;
-  g.C = M; g.sCb = (int64_t)n * H; g.ldc = H;
-  g.bias = b; g.sBias = H;
-  BG_CUDA(bg::gemm(g, nullptr, 0, st));
+  if (bf) {
+    // transforms on the tensor cores: M_p = E W_p + b_p with W_p^T as the K-major operand
+    int* status = nullptr;
+    BG_TRY(status_word_ptr(&status));
+    auto* WT = reinterpret_cast<__nv_bfloat16*>(ws + al(sizeof(float) * (size_t)p->P * n * H));
+    BG_CUDA(bg::prep_transpose_bf16(W, 0, WT, H, H, p->P, st));
+    BG_CUDA(bg::gemm_bf16_tn(E, H, 0, WT, H, (int64_t)H * H, (int)n, H, H, p->P, M, H,
+                             (int64_t)n * H, b, H, 0, status, st));
+  } else {
+    bg::Gemm g;
+    g.M = (int)n; g.N = H; g.K = H; g.batch = p->P;
+    g.A = E; g.a_bf16 = bf; g.sAb = 0; g.sAm = H; g.sAk = 1;
+    g.B = W; g.b_bf16 = bf; g.sBb = (int64_t)H * H; g.sBk = H; g.sBn = 1;
+    g.C = M; g.sCb = (int64_t)n * H; g.ldc = H;
+    g.bias = b; g.sBias = H;
+    BG_CUDA(bg::gemm(g, nullptr, 0, st));
+  }
   BG_CUDA(bg::band_fwd_gather(p->d_masks, M, Y, p->K, p->S, p->P, H, st));
   return BG_OK;
 }
@@ -558,6 +602,33 @@ static int propagate_bwd_impl(const bg_plan* p, bg_dtype dt, int H, const void* 
   }
   BwdWs w = bwd_ws(p, dt, H);
   if (ws_bytes < w.total) return bg_fail(BG_ECAPACITY, "workspace too small");
+  if (tc_gemm_path(dt, H)) {
+    int* status = nullptr;
+    BG_TRY(status_word_ptr(&status));
+    auto* dMb = reinterpret_cast<__nv_bfloat16*>(ws + w.dMb);
+    auto* dMT = reinterpret_cast<__nv_bfloat16*>(ws + w.dMT);
+    auto* Wp = reinterpret_cast<__nv_bfloat16*>(ws + w.Wp);
+    auto* ETa = reinterpret_cast<__nv_bfloat16*>(ws + w.ETa);
+    float* tpart = reinterpret_cast<float*>(ws + w.tpart);
+    const size_t tpf = bg::gemm_tn_part_floats(p->P * H, H + 16, (int64_t)n);
+    const int PH = p->P * H;
+    {
+      KTimer t(BG_KID_BAND_BWD, st);
+      // dM_p = A_p^T dY over the transposed bit tiles; dE (+)= dM_cat [n][P*H] x Wp^T
+      BG_CUDA(bg::band_bwd_gather_bf16(p->d_masksT, dY, dMb, p->K, p->S, p->P, H, st));
+      BG_CUDA(bg::wperm(W, Wp, p->P, H, st));
+      BG_CUDA(bg::gemm_bf16_tn(dMb, PH, 0, Wp, PH, 0, (int)n, H, PH, 1, dE, H, 0, nullptr, 0,
+                               accum, status, st));
+    }
+    KTimer t(BG_KID_DW, st);
+    // dW_p, db_p from one split-K product of dM^T with [E^T; 1; 0]
+    BG_CUDA(bg::prep_transpose_bf16(dMb, 0, dMT, (int)n, PH, 1, st));
+    BG_CUDA(bg::prep_transpose_bf16(E, 0, ETa, (int)n, H, 1, st));
+    BG_CUDA(bg::fill_ones_rows(ETa, H, (int64_t)n, (int64_t)n, st));
+    BG_CUDA(bg::gemm_tn(dMT, (int64_t)n, ETa, (int64_t)n, PH, H, (int64_t)n, 1, dW, db, accum,
+                        tpart, tpf, status, st));
+    return BG_OK;
+  }
   float* dM = reinterpret_cast<float*>(ws + w.dM);
   float* Wt = reinterpret_cast<float*>(ws + w.Wt);
   float* part = reinterpret_cast<float*>(ws + w.part);
@@ -610,11 +681,22 @@ static int check_params(const bg_params* prm) {
   return BG_OK;
 }
 
-// gi = X W_ih^T + b_ih, gh = Hs W_hh^T + b_hh  ([n, 3H] fp32)
+// gi = X W_ih^T + b_ih, gh = Hs W_hh^T + b_hh  ([n, 3H] fp32).  With Xb (bf16 scratch [n][H]) the
+// products run on the tensor cores (W_ih, W_hh are already K-major [3H][H] operands).
 static int gru_gates_in(const bg_plan* p, int bf, int H, const float* X, const void* Hs,
                         const bg_params* prm, float* gi, float* gh, float* part, size_t pf,
-                        cudaStream_t st) {
+                        cudaStream_t st, __nv_bfloat16* Xb = nullptr) {
   const int n = p->n_pad();
+  if (Xb) {
+    int* status = nullptr;
+    BG_TRY(status_word_ptr(&status));
+    BG_CUDA(bg::f32_to_bf16(X, Xb, (int64_t)n * H, st));
+    BG_CUDA(bg::gemm_bf16_tn(Xb, H, 0, prm->W_ih, H, 0, n, 3 * H, H, 1, gi, 3 * H, 0, prm->b_ih, 0,
+                             0, status, st));
+    BG_CUDA(bg::gemm_bf16_tn(Hs, H, 0, prm->W_hh, H, 0, n, 3 * H, H, 1, gh, 3 * H, 0, prm->b_hh, 0,
+                             0, status, st));
+    return BG_OK;
+  }
   bg::Gemm g;
   g.M = n; g.N = 3 * H; g.K = H;
   g.A = X; g.sAm = H; g.sAk = 1;
@@ -695,7 +777,9 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
     float* Yt = reinterpret_cast<float*>(sv + saved_Y_off(p, dt, H, T, t));
     BG_TRY(propagate_fwd_impl(p, dt, H, Et, prm->W, prm->b, Yt, wsc + w.prop, w.total - w.prop, st));
     KTimer tm(BG_KID_GRU_FWD, st);
-    BG_TRY(gru_gates_in(p, bf, H, Yt, Et, prm, gi, gh, part, pf, st));
+    BG_TRY(gru_gates_in(p, bf, H, Yt, Et, prm, gi, gh, part, pf, st,
+                        tc_gemm_path(dt, H) ? reinterpret_cast<__nv_bfloat16*>(wsc + w.Ybf)
+                                            : nullptr));
     BG_CUDA(bg::gru_fwd_gates(bf, gi, gh, Et, En, p->n_real, p->n_pad(), H, st));
   }
   if (ET) BG_CUDA(cudaMemcpyAsync(ET, sv + saved_E_off(p, dt, H, T), ebytes, cudaMemcpyDeviceToDevice, st));
@@ -794,7 +878,44 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
   for (int t = T - 1; t >= 0; --t) {
     const void* Et = sv + saved_E_off(p, dt, H, t);
     const float* Yt = reinterpret_cast<const float*>(sv + saved_Y_off(p, dt, H, T, t));
-    {
+    if (tc_gemm_path(dt, H)) {
+      KTimer tm(BG_KID_GRU_BWD, st);
+      int* status = nullptr;
+      BG_TRY(status_word_ptr(&status));
+      auto* Ybf = reinterpret_cast<__nv_bfloat16*>(wsc + w.Ybf);
+      auto* dgib = reinterpret_cast<__nv_bfloat16*>(wsc + w.dgib);
+      auto* dghb = reinterpret_cast<__nv_bfloat16*>(wsc + w.dghb);
+      auto* dgiT = reinterpret_cast<__nv_bfloat16*>(wsc + w.dgiT);
+      auto* dghT = reinterpret_cast<__nv_bfloat16*>(wsc + w.dghT);
+      auto* YTa = reinterpret_cast<__nv_bfloat16*>(wsc + w.YTa);
+      auto* ETa = reinterpret_cast<__nv_bfloat16*>(wsc + w.ETa);
+      auto* WihT = reinterpret_cast<__nv_bfloat16*>(wsc + w.WihT);
+      auto* WhhT = reinterpret_cast<__nv_bfloat16*>(wsc + w.WhhT);
+      float* tpart = reinterpret_cast<float*>(wsc + w.tpart);
+      const size_t tpf = gru_tpart_floats(p, H);
+      BG_TRY(gru_gates_in(p, bf, H, Yt, Et, prm, gi, gh, part, pf, st, Ybf));
+      BG_CUDA(bg::gru_bwd_gates(bf, gi, gh, Et, gin, dgi, dgh, g, p->n_real, n, H, st));
+      BG_CUDA(bg::f32_to_bf16(dgi, dgib, (int64_t)n * 3 * H, st));
+      BG_CUDA(bg::f32_to_bf16(dgh, dghb, (int64_t)n * 3 * H, st));
+      // dX = dgi W_ih, g += dgh W_hh  (B operands W^T [H][3H])
+      BG_CUDA(bg::prep_transpose_bf16(prm->W_ih, 0, WihT, 3 * H, H, 1, st));
+      BG_CUDA(bg::prep_transpose_bf16(prm->W_hh, 0, WhhT, 3 * H, H, 1, st));
+      BG_CUDA(bg::gemm_bf16_tn(dgib, 3 * H, 0, WihT, 3 * H, 0, n, H, 3 * H, 1, dX, H, 0, nullptr,
+                               0, 0, status, st));
+      BG_CUDA(bg::gemm_bf16_tn(dghb, 3 * H, 0, WhhT, 3 * H, 0, n, H, 3 * H, 1, g, H, 0, nullptr,
+                               0, 1, status, st));
+      // dW_ih, db_ih and dW_hh, db_hh: split-K products with [Y^T; 1; 0] and [E^T; 1; 0]
+      BG_CUDA(bg::prep_transpose_bf16(dgib, 0, dgiT, n, 3 * H, 1, st));
+      BG_CUDA(bg::prep_transpose_bf16(dghb, 0, dghT, n, 3 * H, 1, st));
+      BG_CUDA(bg::prep_transpose_bf16(Yt, 1, YTa, n, H, 1, st));
+      BG_CUDA(bg::fill_ones_rows(YTa, H, n, n, st));
+      BG_CUDA(bg::prep_transpose_bf16(Et, 0, ETa, n, H, 1, st));
+      BG_CUDA(bg::fill_ones_rows(ETa, H, n, n, st));
+      BG_CUDA(bg::gemm_tn(dgiT, n, YTa, n, 3 * H, H, n, 0, gr->dW_ih, gr->db_ih, 1, tpart, tpf,
+                          status, st));
+      BG_CUDA(bg::gemm_tn(dghT, n, ETa, n, 3 * H, H, n, 0, gr->dW_hh, gr->db_hh, 1, tpart, tpf,
+                          status, st));
+    } else {
       KTimer tm(BG_KID_GRU_BWD, st);
       BG_TRY(gru_gates_in(p, bf, H, Yt, Et, prm, gi, gh, part, pf, st));
       // g <- direct term z * dE(t+1); dgi, dgh gate gradients

@@ -602,6 +602,20 @@ bool make_map_ld(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols,
 
 int gemm_tn_num_sms() { return num_sms(); }
 
+bool make_map_3d(CUtensorMap* m, const void* base, uint64_t batch, uint64_t rows, uint64_t cols,
+                 uint64_t ld, uint64_t sbatch, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {cols, rows, batch};
+  cuuint64_t strides[2] = {ld * 2, sbatch * 2};
+  cuuint32_t box[3] = {64, box_rows, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 bool band_tc_supported(const bg_plan* p, int dtype, int H) {
   return p && dtype == 1 && p->S == 128 && (H == 64 || H == 128) && p->P <= 32 && p->d_maskI &&
          p->d_maskTI && p->d_deg2 && p->max_deg <= 256 && encode_fn() != nullptr;

@@ -172,6 +172,141 @@ __global__ void k_gemm_tn_reduce(const float* __restrict__ part, int splits, int
   }
 }
 
+// ---------------------------------------------------------------------------------------------
+// Batched TN GEMM: C[b][m][n] (+)= sum_k A[b][m][k] B[b][n][k] (+ bias[b][n]); one 128 x BN output
+// tile per CTA, K streamed in 64-wide chunks through a 4-stage TMA ring.
+template <int BN>
+struct BCfg {
+  static constexpr int A_BYTES = 128 * 128;
+  static constexpr int B_BYTES = BN * 128;
+  static constexpr int STAGE = A_BYTES + B_BYTES;
+  static constexpr int SMEM = kStages * STAGE + 1024 + 1024;
+  static constexpr int TCOLS = BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+};
+
+struct BatchArgs {
+  int M, N, kchunks, a3d, b3d;
+  float* C;
+  int64_t ldc, sC;
+  const float* bias;
+  int64_t sBias;
+  int accumulate;
+};
+
+template <int BN>
+__global__ void __launch_bounds__(192, 1)
+    k_gemm_bf16(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                BatchArgs g, int* status) {
+  using C = BCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * C::STAGE);
+  uint64_t* empty = full + kStages;
+  uint64_t* done = empty + kStages;
+  uint64_t* drain = done + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+  volatile int* abort = abort_flag;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int mt = blockIdx.x, nt = blockIdx.y, b = blockIdx.z;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    mbar_init(done, 1);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TCOLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  if (warp == 0 && lane == 0) {
+    uint32_t issued[kStages] = {0, 0, 0, 0};
+    for (int kc = 0; kc < g.kchunks; ++kc) {
+      const int s = kc % kStages;
+      if (!mbar_wait(&empty[s], ((kc / kStages) & 1) ^ 1, status, 511, abort, 32)) break;
+      ++issued[s];
+      mbar_expect_tx(&full[s], C::STAGE);
+      uint8_t* st = smem + s * C::STAGE;
+      if (g.a3d) tma_load_3d(st, &tmA, &full[s], kc * 64, mt * 128, b);
+      else tma_load_2d(st, &tmA, &full[s], kc * 64, mt * 128);
+      if (g.b3d) tma_load_3d(st + C::A_BYTES, &tmB, &full[s], kc * 64, nt * BN, b);
+      else tma_load_2d(st + C::A_BYTES, &tmB, &full[s], kc * 64, nt * BN);
+    }
+    if (*abort)
+      for (int s = 0; s < kStages; ++s)
+        for (uint32_t t = 0; issued[s] && t < (1u << 22) && !mbar_try(&full[s], (issued[s] - 1) & 1); ++t) {
+        }
+  } else if (warp == 1) {
+    const bool leader = elect_one_sync();
+    constexpr uint32_t idesc = idesc_bf16_f32(128, BN);
+    for (int kc = 0; kc < g.kchunks; ++kc) {
+      const int s = kc % kStages;
+      if (!mbar_wait(&full[s], (kc / kStages) & 1, status, 512, abort)) break;
+      tc_fence_after();
+      const uint32_t a = smem_u32(smem + s * C::STAGE), bb = a + C::A_BYTES;
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)
+        if (leader)
+          mma_ss(tmem, desc_sw128_kmajor(a + kk * 32), desc_sw128_kmajor(bb + kk * 32), idesc,
+                 (kc > 0 || kk > 0) ? 1u : 0u);
+      if (leader) tc_commit(&empty[s]);
+      __syncwarp();
+    }
+    if (leader) {
+      tc_commit(done);
+      tc_commit(drain);
+    }
+    __syncwarp();
+    for (uint32_t t = 0; t < (1u << 24) && !mbar_try(drain, 0); ++t) {
+    }
+  } else if (warp >= 2) {
+    // each warp drains its 32 TMEM lanes (rows) 32 columns at a time through a padded SMEM
+    // transpose so that every global store instruction writes 32 consecutive columns of one row
+    const int q = warp & 3;
+    if (mbar_wait(done, 0, status, 513, abort, 128)) {
+      tc_fence_after();
+      float* sbuf = reinterpret_cast<float*>(smem) + (warp - 2) * 32 * 33;  // stages are idle now
+      const float* brow = g.bias ? g.bias + (size_t)b * g.sBias : nullptr;
+      float* cbase = g.C + (size_t)b * g.sC;
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        uint32_t v[32];
+        tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + c0, v);
+        tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + c0 + 16, v + 16);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) sbuf[lane * 33 + j] = __uint_as_float(v[j]);
+        __syncwarp();
+        const int n = nt * BN + c0 + lane;
+        const float bv = (brow && n < g.N) ? brow[n] : 0.f;
+#pragma unroll 4
+        for (int rr = 0; rr < 32; ++rr) {
+          const int m = mt * 128 + q * 32 + rr;
+          if (m < g.M && n < g.N) {
+            float* dst = cbase + (size_t)m * g.ldc + n;
+            const float x = sbuf[rr * 33 + lane] + bv;
+            *dst = g.accumulate ? *dst + x : x;
+          }
+        }
+        __syncwarp();
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TCOLS);
+  }
+}
+
 }  // namespace
 
 namespace {
@@ -190,6 +325,37 @@ cudaError_t fill_ones_rows(__nv_bfloat16* base, int H, int64_t n, int64_t ld, cu
   const int64_t total = 16 * n;
   k_fill_ones_rows<<<(unsigned)std::min<int64_t>((total + 255) / 256, 8192), 256, 0, st>>>(base, H,
                                                                                           n, ld);
+  note_launch();
+  return cudaGetLastError();
+}
+
+cudaError_t gemm_bf16_tn(const void* A, int64_t lda, int64_t sA, const void* B, int64_t ldb,
+                         int64_t sB, int M, int N, int K, int batch, float* Cout, int64_t ldc,
+                         int64_t sC, const float* bias, int64_t sBias, int accumulate, int* status,
+                         cudaStream_t st) {
+  if (M <= 0 || N <= 0 || batch <= 0) return cudaSuccess;
+  if (K <= 0 || (lda % 8) || (ldb % 8) || (sA % 8) || (sB % 8)) return cudaErrorInvalidValue;
+  const int BN = N <= 64 ? 64 : N <= 128 ? 128 : N <= 192 ? 192 : 256;
+  CUtensorMap ta, tb;
+  const bool a3 = batch > 1 && sA != 0, b3 = batch > 1 && sB != 0;
+  if (!(a3 ? make_map_3d(&ta, A, batch, M, K, lda, sA, 128) : make_map_ld(&ta, A, M, K, lda, 128)) ||
+      !(b3 ? make_map_3d(&tb, B, batch, N, K, ldb, sB, BN) : make_map_ld(&tb, B, N, K, ldb, BN)))
+    return cudaErrorInvalidValue;
+  BatchArgs g{M, N, (K + 63) / 64, a3 ? 1 : 0, b3 ? 1 : 0, Cout, ldc, sC, bias, sBias, accumulate};
+  dim3 grid((M + 127) / 128, (N + BN - 1) / BN, batch);
+  cudaError_t e;
+#define BG_GEMM16_CASE(BNV)                                                                    \
+  e = cudaFuncSetAttribute(k_gemm_bf16<BNV>, cudaFuncAttributeMaxDynamicSharedMemorySize,      \
+                           BCfg<BNV>::SMEM);                                                   \
+  if (e != cudaSuccess) return e;                                                              \
+  k_gemm_bf16<BNV><<<grid, 192, BCfg<BNV>::SMEM, st>>>(ta, tb, g, status);
+  switch (BN) {
+    case 64: BG_GEMM16_CASE(64) break;
+    case 128: BG_GEMM16_CASE(128) break;
+    case 192: BG_GEMM16_CASE(192) break;
+    default: BG_GEMM16_CASE(256) break;
+  }
+#undef BG_GEMM16_CASE
   note_launch();
   return cudaGetLastError();
 }

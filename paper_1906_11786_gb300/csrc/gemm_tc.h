@@ -23,11 +23,24 @@ cudaError_t gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int 
                     int64_t K, int mode, float* out, float* bias, int accumulate, float* part,
                     size_t part_floats, int* status, cudaStream_t st);
 
+// Batched TN GEMM on tcgen05 (fp32 accumulation):
+//   C[b][m][n] (+)= sum_k A[b][m][k] B[b][n][k] (+ bias[b*sBias + n])
+// A: [M][K] bf16, row stride lda, batch stride sA (0 = shared by all batches); B: [N][K] bf16, row
+// stride ldb, batch stride sB (0 = shared); C fp32 row stride ldc, batch stride sC.  Strides in
+// elements, multiples of 8; K > 0 (zero-padded to 64 by the tensor maps).
+cudaError_t gemm_bf16_tn(const void* A, int64_t lda, int64_t sA, const void* B, int64_t ldb,
+                         int64_t sB, int M, int N, int K, int batch, float* C, int64_t ldc,
+                         int64_t sC, const float* bias, int64_t sBias, int accumulate, int* status,
+                         cudaStream_t st);
+
 // 2-D bf16 tensor map over row-major [rows][cols] with row stride ld elements; box {64, box_rows};
 // 128-byte swizzle; reads outside the array return zero.
 bool make_map_ld(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
                  uint32_t box_rows);
 int gemm_tn_num_sms();
+// 3-D variant: [batch][rows][cols] with row stride ld and batch stride sbatch (elements).
+bool make_map_3d(CUtensorMap* m, const void* base, uint64_t batch, uint64_t rows, uint64_t cols,
+                 uint64_t ld, uint64_t sbatch, uint32_t box_rows);
 
 // rows [H, H+16) of a [H+16][ld] bf16 array: row H = 1.0, the rest 0 (cols [0, n)).
 cudaError_t fill_ones_rows(__nv_bfloat16* base, int H, int64_t n, int64_t ld, cudaStream_t st);

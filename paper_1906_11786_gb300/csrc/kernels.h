@@ -46,6 +46,13 @@ cudaError_t band_fwd_gather(const uint32_t* masks, const float* M, float* Y, int
 cudaError_t band_bwd_gather(const uint32_t* masksT, const float* dY, float* dM, int K, int S,
                             int P, int H, cudaStream_t st);
 
+// Same as band_bwd_gather with bf16 output dM [n_pad][P][H].
+cudaError_t band_bwd_gather_bf16(const uint32_t* masksT, const float* dY, __nv_bfloat16* dM, int K,
+                                 int S, int P, int H, cudaStream_t st);
+// Wp[h][p*H + o] = W[p][h][o] (bf16): W_p^T blocks side by side, the operand of dE = dM_cat Wp^T.
+cudaError_t wperm(const void* W, __nv_bfloat16* Wp, int P, int H, cudaStream_t st);
+cudaError_t f32_to_bf16(const float* x, __nv_bfloat16* y, int64_t n, cudaStream_t st);
+
 // Wt[(p*H + o)*H + i] = W[p][i][o] (fp32)
 cudaError_t transpose_weights(int bf16, const void* W, float* Wt, int P, int H, cudaStream_t st);
 

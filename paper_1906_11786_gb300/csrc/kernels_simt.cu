@@ -174,9 +174,10 @@ __global__ void __launch_bounds__(256) k_band_fwd_gather(const uint32_t* __restr
     if (q < HQ) Y[i * H + lane + 32 * q] = acc[q];
 }
 
+template <typename TO>
 __global__ void __launch_bounds__(256) k_band_bwd_gather(const uint32_t* __restrict__ masksT,
                                                          const float* __restrict__ dY,
-                                                         float* __restrict__ dM, int K, int S,
+                                                         TO* __restrict__ dM, int K, int S,
                                                          int P, int H) {
   const int lane = threadIdx.x & 31;
   const int64_t j = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
@@ -205,8 +206,27 @@ __global__ void __launch_bounds__(256) k_band_bwd_gather(const uint32_t* __restr
     }
 #pragma unroll
     for (int q = 0; q < 8; ++q)
-      if (q < HQ) dM[(j * P + p) * H + lane + 32 * q] = acc[q];
+      if (q < HQ) st(dM, (j * P + p) * H + lane + 32 * q, acc[q]);
   }
+}
+
+// Wperm[h][p*H + o] = W[p][h][o]  (the [H][P*H] B operand of dE = dM_cat W_perm^T)
+__global__ void k_wperm(const __nv_bfloat16* __restrict__ W, __nv_bfloat16* __restrict__ Wp, int P,
+                        int H) {
+  int64_t total = (int64_t)P * H * H;
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int o = (int)(t % H);
+    const int64_t ph = t / H;
+    const int h = (int)(ph % H), p = (int)(ph / H);
+    Wp[(int64_t)h * P * H + (int64_t)p * H + o] = W[t];
+  }
+}
+
+__global__ void k_f32_to_bf16(const float* __restrict__ x, __nv_bfloat16* __restrict__ y, int64_t n) {
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < n;
+       t += (int64_t)gridDim.x * blockDim.x)
+    y[t] = __float2bfloat16_rn(x[t]);
 }
 
 template <typename T>
@@ -445,7 +465,30 @@ cudaError_t band_fwd_gather(const uint32_t* masks, const float* M, float* Y, int
 cudaError_t band_bwd_gather(const uint32_t* masksT, const float* dY, float* dM, int K, int S,
                             int P, int H, cudaStream_t st) {
   int64_t rows = (int64_t)K * S;
-  k_band_bwd_gather<<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(masksT, dY, dM, K, S, P, H);
+  k_band_bwd_gather<float><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(masksT, dY, dM, K, S, P, H);
+  note_launch();
+  return cudaGetLastError();
+}
+
+cudaError_t band_bwd_gather_bf16(const uint32_t* masksT, const float* dY, __nv_bfloat16* dM, int K,
+                                 int S, int P, int H, cudaStream_t st) {
+  int64_t rows = (int64_t)K * S;
+  k_band_bwd_gather<__nv_bfloat16><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(masksT, dY, dM, K,
+                                                                               S, P, H);
+  note_launch();
+  return cudaGetLastError();
+}
+
+cudaError_t wperm(const void* W, __nv_bfloat16* Wp, int P, int H, cudaStream_t st) {
+  int64_t total = (int64_t)P * H * H;
+  k_wperm<<<grid_for(total, 256), 256, 0, st>>>(static_cast<const __nv_bfloat16*>(W), Wp, P, H);
+  note_launch();
+  return cudaGetLastError();
+}
+
+cudaError_t f32_to_bf16(const float* x, __nv_bfloat16* y, int64_t n, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  k_f32_to_bf16<<<grid_for(n, 256), 256, 0, st>>>(x, y, n);
   note_launch();
   return cudaGetLastError();
 }

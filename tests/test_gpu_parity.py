@@ -141,10 +141,14 @@ def _ggnn(c: Case, T, seed=3):
         dE0.cpu().numpy(), ref
 
 
-@pytest.mark.parametrize("dtype,T", [("f32", 2), ("bf16", 3)])
-def test_ggnn_fwd_bwd(dtype, T):
-    gs = synth.gen_batch(5, 60, 300, 10, True, 48, 32, 2.0, 41)
-    c = Case(gs, 20, 64, 64, dtype, seed=9)
+@pytest.mark.parametrize("dtype,T,S,H", [("f32", 2, 64, 64), ("bf16", 3, 64, 64),
+                                         ("bf16", 2, 128, 128), ("bf16", 2, 32, 32),
+                                         ("bf16", 2, 128, 256)])
+def test_ggnn_fwd_bwd(dtype, T, S, H):
+    """Every kernel family of the GGNN step: SIMT (fp32, H = 256), tensor-core GEMMs around the
+    SIMT band sums (S != 128), fused band kernels with GEMM-based GRU (H = 128)."""
+    gs = synth.gen_batch(5, 60, 300, 10, True, max(8, S // 2), max(8, S // 3), 2.0, 41)
+    c = Case(gs, 20, S, H, dtype, seed=9)
     ET, ref_ET, grads, dE0, ref = _ggnn(c, T)
     tol = TOL[dtype]
     assert rel_err(ET, ref_ET) < tol
