@@ -221,3 +221,59 @@ def test_full_size_config2_propagate_sampled_rows():
                                c.prm["b"])
     assert rel_err(Y.cpu().numpy()[rows], ref[rows]) < TOL["bf16"]
     L.check_device()
+
+
+
+def test_full_size_config2_ggnn_T8_fwd_bwd_sampled_graphs():
+    """The benchmark workload end to end: config 2 at full size (64 graphs, ~72k nodes, P = 20,
+    S = 128, H = 64, bf16, T = 8) through the fused tensor-core path, forward + backward.
+
+    Graphs share no edge, so (Eq. 1 and Eq. 2 act per graph) E(T) of a graph depends on that graph
+    alone, and a dE(T) that is zero outside a few sampled graphs leaves dE(0) zero outside them and
+    makes every parameter gradient a sum over the sampled graphs only.  The oracle therefore runs on
+    the sampled graphs, compacted, and is compared with the full-size launch on E(T) of the sampled
+    rows, on all of dE(0) and on all six parameter gradients."""
+    c = Case(synth.config_graphs(2), 20, 128, 64, "bf16", seed=23)
+    assert L.band_uses_tensor_cores(c.plan, c.dtype, c.H)
+    T = 8
+    saved = torch.empty(L.ggnn_saved_bytes(c.plan, c.dtype, c.H, T), dtype=torch.uint8,
+                        device="cuda")
+    ET = torch.empty_like(c.E_band_dev)
+    L.ggnn_step(c.plan, c.dtype, c.H, T, c.dprm, c.E_band_dev, ET, saved, c.ws(L.BG_OP_GGNN_FWD, T))
+    off, cnt = c.ref.graph_segments()
+    pick = np.random.default_rng(5).choice(len(off), 4, replace=False)
+    rows = np.concatenate([np.arange(off[g], off[g] + cnt[g]) for g in pick])
+    dET = np.zeros((c.N, c.H))
+    dET[rows] = quantize(np.random.default_rng(31).standard_normal((len(rows), c.H)), "f32")
+    dE0 = torch.empty((c.N, c.H), dtype=torch.float32, device="cuda")
+    grads = dict(dW=torch.empty((c.P, c.H, c.H), device="cuda"),
+                 db=torch.empty((c.P, c.H), device="cuda"),
+                 dW_ih=torch.empty((3 * c.H, c.H), device="cuda"),
+                 dW_hh=torch.empty((3 * c.H, c.H), device="cuda"),
+                 db_ih=torch.empty(3 * c.H, device="cuda"),
+                 db_hh=torch.empty(3 * c.H, device="cuda"))
+    L.ggnn_step_bwd(c.plan, c.dtype, c.H, T, c.dprm, saved, f32_dev(dET), dE0, grads,
+                    c.ws(L.BG_OP_GGNN_BWD, T))
+    torch.cuda.synchronize()
+    L.check_device()
+
+    # compact sub-problem: the sampled graphs' rows, renumbered 0..m-1, with their edges
+    m = len(rows)
+    new = np.full(c.N, -1, np.int64)
+    new[rows] = np.arange(m)
+    e_dst, e_src, e_type = c.edges
+    sel = new[e_dst] >= 0
+    assert np.all(new[e_src[sel]] >= 0)
+    sub = (new[e_dst[sel]], new[e_src[sel]], e_type[sel])
+    Es, Ys = oracle.ggnn_fwd(m, c.P, c.H, T, m, *sub, c.E_band[rows], c.prm)
+    ref = oracle.ggnn_bwd(m, c.P, c.H, T, m, *sub, c.prm, Es, Ys, dET[rows])
+
+    got_ET = ET.float().cpu().numpy()
+    assert rel_err(got_ET[rows], Es[T]) < TOL["bf16"]
+    got_dE0 = dE0.cpu().numpy()
+    assert rel_err(got_dE0[rows], ref["dE0"]) < TOL["bf16"]
+    rest = np.ones(c.N, bool)
+    rest[rows] = False
+    assert np.all(got_dE0[rest] == 0.0)
+    for k, v in grads.items():
+        assert rel_err(v.cpu().numpy(), ref[k]) < TOL["bf16"], k
