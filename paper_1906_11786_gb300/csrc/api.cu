@@ -449,13 +449,13 @@ struct TcFwdWs {
 TcFwdWs tc_fwd_ws(const bg_plan* p, int H) {
   TcFwdWs w{};
   size_t o = 0;
-  w.WT = o; o += al((size_t)p->P * H * H * 2);
+  w.WT = o; o += bg::band_tc_w_bytes(p, H);
   w.b2T = o; o += al((size_t)H * 64 * 2);
   w.total = o;
   return w;
 }
 struct TcBwdWs {
-  size_t g, dXT, dMT, dgiT, dghT, WihT, WhhT, part, total;
+  size_t g, dXT, dMT, dgiT, dghT, WihT, WhhT, Wk, part, total;
 };
 size_t tc_part_floats(const bg_plan* p, int H, int T) {
   const int64_t K = (int64_t)T * p->n_pad();
@@ -473,6 +473,7 @@ TcBwdWs tc_bwd_ws(const bg_plan* p, int H, int T) {
   w.dghT = o; o += al((size_t)3 * H * TN * 2);
   w.WihT = o; o += al((size_t)3 * H * H * 2);
   w.WhhT = o; o += al((size_t)3 * H * H * 2);
+  w.Wk = o; o += bg::band_tc_w_bytes(p, H);
   w.part = o; o += al(sizeof(float) * tc_part_floats(p, H, T));
   w.total = o;
   return w;
@@ -737,13 +738,13 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
     auto Yi = [&](int t) { return reinterpret_cast<__nv_bfloat16*>(sv + sl.Y + (size_t)t * stE); };
     __nv_bfloat16* ETa = reinterpret_cast<__nv_bfloat16*>(sv + sl.ETa);
     __nv_bfloat16* YTa = reinterpret_cast<__nv_bfloat16*>(sv + sl.YTa);
-    __nv_bfloat16* WT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.WT);
+    void* WT = wsc + wl.WT;
     __nv_bfloat16* b2T = reinterpret_cast<__nv_bfloat16*>(wsc + wl.b2T);
     BG_CUDA(cudaMemcpyAsync(Ei(0), E0, n * H * 2, cudaMemcpyDeviceToDevice, st));
     BG_CUDA(bg::prep_transpose_bf16(E0, 0, ETa, (int)n, H, 1, st, (int64_t)TN));
     BG_CUDA(bg::fill_ones_rows(ETa, H, (int64_t)TN, (int64_t)TN, st));
     BG_CUDA(bg::fill_ones_rows(YTa, H, (int64_t)TN, (int64_t)TN, st));
-    BG_CUDA(bg::prep_transpose_bf16(prm->W, 0, WT, H, H, p->P, st));
+    BG_CUDA(bg::band_tc_prep_w(p, H, prm->W, 0, WT, st));
     if (prm->b) BG_CUDA(bg::prep_bias_split(prm->b, b2T, p->P, H, st));
     for (int t = 0; t < T; ++t) {
       {
@@ -828,6 +829,8 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     const auto* Whh = static_cast<const __nv_bfloat16*>(prm->W_hh);
     BG_CUDA(bg::prep_transpose_bf16(Wih, 0, WihT, 3 * H, H, 1, st));
     BG_CUDA(bg::prep_transpose_bf16(Whh, 0, WhhT, 3 * H, H, 1, st));
+    void* Wk = wsc + wl.Wk;
+    BG_CUDA(bg::band_tc_prep_w(p, H, prm->W, 1, Wk, st));
     const float* gin = dET;
     for (int t = T - 1; t >= 0; --t) {
       {
@@ -837,7 +840,7 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
                                dghT + (size_t)t * n, (int64_t)TN, status, st));
       }
       KTimer tm(BG_KID_BAND_BWD, st);
-      BG_CUDA(bg::band_tc_bwd_core(p, H, dXT, (int64_t)n, prm->W, g, 1, dMT + (size_t)t * n,
+      BG_CUDA(bg::band_tc_bwd_core(p, H, dXT, (int64_t)n, Wk, g, 1, dMT + (size_t)t * n,
                                    (int64_t)TN, status, st));
       gin = g;
     }

@@ -3,25 +3,38 @@
 // Forward (Algorithm 1's aggregate-first order, Eq. 3): for a 128-row tile of block-row k and
 // every edge type p,
 //     pre_p = sum_{d in -1,0,+1} A_{k,d,p} E_{k+d}        (128 x 3S  times  3S x H, fp32 in TMEM)
-//     Y_k  += bf16(pre_p) W_p                               (chained MMA, A operand read from TMEM)
+//     Y_k  += pre_p W_p                                     (chained MMA, A operand read from TMEM)
 // and the per-type bias enters as one more product deg_k [128 x 2P] x [b_hi; b_lo] with exact
 // integer in-degrees and b split into two bf16 halves.  pre_p never leaves the SM.
 // Backward (transposed band): the same kernel with the transposed tiles, dY instead of E and W_p
 // instead of W_p^T gives dE_j += sum_p (A^T dY)_p W_p^T; dM_p = A_p^T dY is also written (bf16,
 // transposed) for the weight gradient.
 //
+// At H = 64 the second product runs as kind::tf32 straight from the fp32 pre_p (W_p staged as
+// fp32), so no thread touches pre_p between the two products and the MMA issuer never waits on
+// a conversion; at H = 128 pre_p is rounded to bf16 in place by the converter warps first.
+//
 // The 0/1 adjacency is the MMA's A operand.  It is stored as bits (the whole band costs
 // 3 P S^2 / 8 bytes per block-row) and expanded on chip straight into tensor memory: the bits of
 // each 32-column word are interleaved at upload (column 2j at bit j, column 2j+1 at bit 16+j) so
 // that one AND and one multiply give the packed bf16 pair {1.0 or 0, 1.0 or 0}.
 //
-// Roles (128 x (1 + NE + NC) threads, one CTA per SM, persistent over tiles):
+// Roles (384 threads, one CTA per SM, persistent over tiles):
 //   warp 0      TMA producer: state blocks (B operand of the band product), W tiles, deg, bias
-//   warp 1      TMEM allocator; an elected lane of the converged warp issues every tcgen05.mma
+//   warp 1      TMEM allocator and MMA issuer (an elected lane of the converged warp issues):
+//               at H = 64 the band products only, one wait per edge type; otherwise every MMA
 //   warp 2      mask producer: one bulk copy per (tile, type) of the bit tiles into an SMEM ring
-//   next NE warpgroups   expanders: thread r turns row r's mask bits into bf16 A tiles in TMEM
-//   last NC warpgroups   converters: pre_p fp32 -> bf16 in place; final epilogue TMEM -> global
-// Waiting roles sleep between polls so that the MMA issuer keeps its issue slots.
+//   warp 3      (H = 64) second MMA issuer: the pre_p W_p products and the bias product, so that
+//               their waits never stall the band-product stream
+//   warps 4-7   expanders: thread r turns row r's mask bits into bf16 A tiles in TMEM
+//   warps 8-11  converters: pre_p fp32 -> bf16 (H = 128), dM_p to global (backward), final
+//               epilogue TMEM -> global
+// A tcgen05.mma of N = 64 is about as long as its issue, so any wait on the band-product
+// issuer leaves the tensor pipe idle: at H = 64 that issuer waits once per edge type, on a
+// barrier that the expanders (all three A tiles in TMEM), the second issuer (the pre_p buffer is
+// free) and in the backward pass the converters complete together.
+// Consumer warps signal a barrier with one arrive per warp after __syncwarp.  Waiting roles other
+// than the expanders sleep between polls so that the MMA issuers keep their issue slots.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
@@ -47,11 +60,13 @@ constexpr int kAtom = 64;      // bf16 per 128-byte swizzle row
 
 template <int H>
 struct Cfg {
+  static constexpr bool TF = H <= 64;                         // split issuers, tf32 second product
   static constexpr int NXB = H <= 64 ? 2 : 1;                 // state-window buffers
-  static constexpr int NW = H <= 64 ? 4 : 2;                  // W ring stages
+  static constexpr int NW = 2;                                // W ring stages
   static constexpr int ATOM_X = H * 128;                      // 64 nodes x H rows
   static constexpr int XWIN = 6 * ATOM_X;                     // 3 blocks x 2 atoms (S = 128)
-  static constexpr int WSTAGE = (H / kAtom) * H * 128;        // H x H bf16
+  // H x H operand of the second product: fp32 (32 per 128-byte row) or bf16 (64 per row)
+  static constexpr int WSTAGE = (TF ? H / 32 : H / kAtom) * H * 128;
   static constexpr int DEG = kTile * 128;                     // 128 rows x 64 bf16
   static constexpr int B2 = H * 128;                          // H rows x 64 bf16
   static constexpr int OFF_X = 0;
@@ -64,11 +79,15 @@ struct Cfg {
   static constexpr int OFF_BAR = OFF_M + NM * MSTAGE;
   static constexpr int SMEM = OFF_BAR + 1024 + 1024;          // barriers + 1 KB alignment slack
   // TMEM columns: Y, NB pre_p buffers, then the A-tile slots
-  static constexpr int NB = H <= 64 ? 3 : 2;
+  static constexpr int NB = 2;
   static constexpr int YCOL = 0;
   static constexpr int D1COL0 = H;
   static constexpr int ACOL = (NB + 1) * H;
   static constexpr int NA = (512 - ACOL) / 64;
+  static constexpr int NT = 8;                                // per-type barrier ring (H = 64)
+  static_assert(NA >= 2 && NA <= 8, "A-slot ring");
+  static_assert(!TF || NA >= 3, "one edge type's three A tiles must fit");
+  static_assert(SMEM <= 232448, "shared memory");
 };
 
 struct Bars {
@@ -78,9 +97,10 @@ struct Bars {
   uint64_t b2_full;
   uint64_t a_full[8], a_empty[8];
   uint64_t d1_full[4], pre_ready[4];
+  uint64_t t_full[8];
   uint64_t y_full, y_empty;
   uint64_t m_full[8], m_empty[8];
-  uint64_t drain;
+  uint64_t drain, drain2;
   uint32_t tmem_base;
   int abort;
 };
@@ -104,8 +124,25 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
-template <int H, bool BWD, int NE, int NC>
-__global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
+// One arrive per warp once every lane of it is done (lanes' earlier operations are ordered
+// before lane 0's arrive by the warp barrier).
+__device__ __forceinline__ void warp_arrive(uint64_t* bar) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+}
+
+// Bounded wait for every MMA this thread issued (commit to an unused barrier).
+__device__ __forceinline__ void drain_mmas(bool leader, uint64_t* bar) {
+  if (leader) tc_commit(bar);
+  __syncwarp();
+  for (uint32_t t = 0; t < (1u << 24) && !mbar_try(bar, 0); ++t) {
+  }
+}
+
+constexpr int kThreads = 384;
+
+template <int H, bool BWD>
+__global__ void __launch_bounds__(kThreads, 1)
     k_band_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
               const __grid_constant__ CUtensorMap tm_deg, const __grid_constant__ CUtensorMap tm_b2,
               const uint32_t* __restrict__ maskI, float* __restrict__ out,
@@ -123,6 +160,9 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
   uint8_t* b2s = smem + C::OFF_B2;
   uint8_t* mring = smem + C::OFF_M;
   volatile int* abort = &bars->abort;
+  // arrivals that complete one type's t_full phase: 4 expander warps, the second issuer's commit
+  // and, backward, the 4 converter warps
+  constexpr int kTArrivals = 4 + 1 + (BWD ? 4 : 0);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -130,16 +170,23 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
       mbar_init(&bars->x_full[i], 1); mbar_init(&bars->x_empty[i], 1);
       mbar_init(&bars->deg_full[i], 1); mbar_init(&bars->deg_empty[i], 1);
     }
-    for (int i = 0; i < 4; ++i) { mbar_init(&bars->d1_full[i], 1); mbar_init(&bars->pre_ready[i], kTile); }
+    for (int i = 0; i < 4; ++i) { mbar_init(&bars->d1_full[i], 1); mbar_init(&bars->pre_ready[i], 4); }
     for (int i = 0; i < 4; ++i) { mbar_init(&bars->w_full[i], 1); mbar_init(&bars->w_empty[i], 1); }
-    for (int i = 0; i < 8; ++i) { mbar_init(&bars->a_full[i], kTile); mbar_init(&bars->a_empty[i], 1); }
+    for (int i = 0; i < 8; ++i) { mbar_init(&bars->a_full[i], 4); mbar_init(&bars->a_empty[i], 1); }
+    for (int i = 0; i < 8; ++i) mbar_init(&bars->t_full[i], kTArrivals);
     mbar_init(&bars->b2_full, 1);
     mbar_init(&bars->y_full, 1);
-    mbar_init(&bars->y_empty, kTile);
+    mbar_init(&bars->y_empty, 4);
     mbar_init(&bars->drain, 1);
-    for (int i = 0; i < 8; ++i) { mbar_init(&bars->m_full[i], 1); mbar_init(&bars->m_empty[i], kTile * NE); }
+    mbar_init(&bars->drain2, 1);
+    for (int i = 0; i < 8; ++i) { mbar_init(&bars->m_full[i], 1); mbar_init(&bars->m_empty[i], 4); }
     bars->abort = 0;
     fence_mbar_init();
+    if (C::TF) {
+      // the first NB types find their pre_p buffer free: stand in for the releases
+      for (int c = 0; c < C::NB; ++c)
+        for (int a = 0; a < kTArrivals - 4; ++a) mbar_arrive(&bars->t_full[c]);
+    }
   }
   if (warp == 1) {
     tmem_alloc(&bars->tmem_base, 512);
@@ -192,8 +239,10 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
         if (!mbar_wait(&bars->w_empty[ws], ((widx / C::NW) & 1) ^ 1, status, 103, abort, 64)) break;
         ++n_w[ws];
         mbar_expect_tx(&bars->w_full[ws], C::WSTAGE);
-        for (int a = 0; a < H / kAtom; ++a)
-          tma_load_2d(wring + ws * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws], a * kAtom,
+        // atoms of 128-byte rows along K: 32 fp32 (tf32 operand) or 64 bf16 each
+        constexpr int kw = C::TF ? 32 : kAtom;
+        for (int a = 0; a < H / kw; ++a)
+          tma_load_2d(wring + ws * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws], a * kw,
                       p * H);
       }
     }
@@ -231,14 +280,100 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
       for (int q = 0; q < 8; ++q)
         for (uint32_t t = 0; n_m[q] && t < (1u << 22) && !mbar_try(&bars->m_full[q], (n_m[q] - 1) & 1); ++t) {
         }
+  } else if (warp == 1 && C::TF) {
+    // ------------------------------------------------------------------ band-product issuer
+    // pre_p = sum_d A_{k,d,p} X_{k+d}: one t_full wait per type, then an unbroken MMA stream
+    const bool leader = elect_one_sync();
+    constexpr uint32_t idesc = idesc_bf16_f32(kTile, H);
+    uint32_t c = 0, aidx = 0;
+    bool ok = true;
+    int i = 0;
+    for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x, ++i) {
+      const int xb = i % C::NXB;
+      if (!mbar_wait(&bars->x_full[xb], (i / C::NXB) & 1, status, 204, abort)) break;
+      const uint32_t xbase = smem_u32(xwin + xb * C::XWIN);
+      for (int p = 0; p < P; ++p, ++c) {
+        const int b = c % C::NB;
+        if (!mbar_wait(&bars->t_full[c % C::NT], (c / C::NT) & 1, status, 210, abort)) { ok = false; break; }
+        tc_fence_after();
+        uint32_t first = 1;
+        for (int d = 0; d < 3; ++d) {
+          const int kb = k + d - 1;
+          if (kb < 0 || kb >= K) continue;
+          const int slot = aidx % C::NA;
+#pragma unroll
+          for (int kk = 0; kk < kTile / 16; ++kk) {
+            const uint64_t bdesc =
+                desc_sw128_kmajor(xbase + (d * 2 + kk / 4) * C::ATOM_X + (kk % 4) * 32);
+            if (leader) mma_ts(tmem + C::D1COL0 + b * H, tmem + C::ACOL + slot * 64 + kk * 8, bdesc, idesc,
+                   (first && kk == 0) ? 0u : 1u);
+          }
+          first = 0;
+          if (leader) tc_commit(&bars->a_empty[slot]);
+          ++aidx;
+        }
+        if (leader) tc_commit(&bars->d1_full[b]);
+        if (p == P - 1 && leader) tc_commit(&bars->x_empty[xb]);
+      }
+    }
+    drain_mmas(leader, &bars->drain);
+  } else if (warp == 3 && C::TF) {
+    // ------------------------------------------------------------------ second issuer
+    // Y (+)= pre_p W_p (kind::tf32, A = the fp32 pre_p in TMEM) and the bias product
+    const bool leader = elect_one_sync();
+    constexpr uint32_t idesc = idesc_bf16_f32(kTile, H);
+    constexpr uint32_t idesc2 = idesc_tf32_f32(kTile, H);
+    uint32_t c = 0, widx = 0;
+    bool ok = true;
+    int i = 0;
+    for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x, ++i) {
+      for (int p = 0; p < P; ++p, ++c, ++widx) {
+        const int b = c % C::NB;
+        const int ws = widx % C::NW;
+        if (!mbar_wait(&bars->d1_full[b], (c / C::NB) & 1, status, 208, abort) ||
+            !mbar_wait(&bars->w_full[ws], (widx / C::NW) & 1, status, 202, abort) ||
+            (p == 0 && !mbar_wait(&bars->y_empty, (i & 1) ^ 1, status, 203, abort))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t wbase = smem_u32(wring + ws * C::WSTAGE);
+#pragma unroll
+        for (int kk = 0; kk < H / 8; ++kk) {
+          const uint64_t bdesc = desc_sw128_kmajor(wbase + (kk / 4) * H * 128 + (kk % 4) * 32);
+          if (leader) mma_ts_tf32(tmem + C::YCOL, tmem + C::D1COL0 + b * H + kk * 8, bdesc, idesc2,
+                                  (p == 0 && kk == 0) ? 0u : 1u);
+        }
+        if (leader) {
+          tc_commit(&bars->w_empty[ws]);
+          tc_commit(&bars->t_full[(c + C::NB) % C::NT]);  // this pre_p buffer is free again
+        }
+      }
+      if (!ok) break;
+      if (has_bias) {
+        const int db = i & 1;
+        if (!mbar_wait(&bars->deg_full[db], (i >> 1) & 1, status, 206, abort)) break;
+        if (i == 0 && !mbar_wait(&bars->b2_full, 0, status, 207, abort)) break;
+        tc_fence_after();
+        const uint32_t dbase = smem_u32(degs + db * C::DEG), bbase = smem_u32(b2s);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          if (leader) mma_ss(tmem + C::YCOL, desc_sw128_kmajor(dbase + kk * 32),
+                 desc_sw128_kmajor(bbase + kk * 32), idesc, 1u);
+        if (leader) tc_commit(&bars->deg_empty[db]);
+      }
+      if (leader) tc_commit(&bars->y_full);
+    }
+    drain_mmas(leader, &bars->drain2);
   } else if (warp == 1) {
-    // ------------------------------------------------------------------ MMA issuer
+    // ------------------------------------------------------------------ MMA issuer (H = 128)
     // the whole warp runs this loop (its operands stay warp-uniform); one elected lane issues
     const bool leader = elect_one_sync();
     constexpr uint32_t idesc = idesc_bf16_f32(kTile, H);
     uint32_t c = 0, aidx = 0, widx = 0;
     bool ok = true;
     int i = 0;
+    // second product of type cc: Y (+)= bf16(pre_cc) W_cc, after the converters rounded pre_cc
     auto stage2 = [&](uint32_t cc, bool first_in_tile, int tile_i) -> bool {
       const int b = cc % C::NB;
       if (!mbar_wait(&bars->pre_ready[b], (cc / C::NB) & 1, status, 201, abort)) return false;
@@ -310,16 +445,10 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
       }
       if (leader) tc_commit(&bars->y_full);
     }
-    // every MMA issued above has completed once this commit arrives (bounded wait)
-    if (leader) tc_commit(&bars->drain);
-    __syncwarp();
-    for (uint32_t t = 0; t < (1u << 24) && !mbar_try(&bars->drain, 0); ++t) {
-    }
-  } else if (warp >= 4 && warp < 4 + 4 * NE) {
+    drain_mmas(leader, &bars->drain);
+  } else if (warp >= 4 && warp < 8) {
     // ------------------------------------------------------------------ expanders
-    // NE warpgroups take the 128 x 128 chunks in turn, so NE chunks are in flight at once
-    const int eg = (warp - 4) / 4;
-    const int r = threadIdx.x - 128 * (1 + eg);
+    const int r = threadIdx.x - 128;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     uint32_t aidx = 0, midx = 0;
     for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x) {
@@ -334,13 +463,9 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
         for (int d = 0; d < 3; ++d) {
           const int kb = k + d - 1;
           if (kb < 0 || kb >= K) continue;
-          if ((int)(aidx % NE) != eg) {
-            ++aidx;
-            continue;
-          }
           const uint4 m = *reinterpret_cast<const uint4*>(mrow + d * kTile * 16);
           const int slot = aidx % C::NA;
-          if (!mbar_wait(&bars->a_empty[slot], ((aidx / C::NA) & 1) ^ 1, status, 301, abort, 32)) {
+          if (!mbar_wait(&bars->a_empty[slot], ((aidx / C::NA) & 1) ^ 1, status, 301, abort)) {
             ok = false;
             break;
           }
@@ -352,35 +477,41 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
           expand_word(m.z, v);
           expand_word(m.w, v + 16);
           tmem_st32(tmem + lane_base + C::ACOL + slot * 64 + 32, v);
-          tmem_wait_st();
-          tc_fence_before();
-          mbar_arrive(&bars->a_full[slot]);
+          if (!C::TF) {
+            tmem_wait_st();
+            tc_fence_before();
+            warp_arrive(&bars->a_full[slot]);
+          }
           ++aidx;
         }
-        mbar_arrive(&bars->m_empty[ms]);
+        if (!ok) break;
+        if (C::TF) {
+          // all of this type's A tiles are in TMEM
+          tmem_wait_st();
+          tc_fence_before();
+          warp_arrive(&bars->t_full[midx % C::NT]);
+        }
+        warp_arrive(&bars->m_empty[ms]);
       }
       if (!ok) break;
     }
-  } else if (warp >= 4 + 4 * NE) {
+  } else if (warp >= 8) {
     // ------------------------------------------------------------------ converters / epilogue
-    // NC warpgroups take the edge types in turn (conversions overlap); group 0 also writes Y
-    const int cg = (warp - 4 - 4 * NE) / 4;
-    const int r = threadIdx.x - 128 * (1 + NE + cg);
+    const int r = threadIdx.x - 256;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     uint32_t c = 0;
     int i = 0;
     for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x, ++i) {
       const int row = k * kTile + r;
       bool ok = true;
-      for (int p = 0; p < P; ++p, ++c) {
-        if ((int)(c % NC) != cg) continue;
+      for (int p = 0; p < P && (BWD || !C::TF); ++p, ++c) {
         const int b = c % C::NB;
         if (!mbar_wait(&bars->d1_full[b], (c / C::NB) & 1, status, 401, abort, 64)) { ok = false; break; }
         tc_fence_after();
         const uint32_t col = tmem + lane_base + C::D1COL0 + b * H;
-        uint32_t v[32], q[32];
 #pragma unroll
         for (int h0 = 0; h0 < H; h0 += 64) {
+          uint32_t v[32], q[32];
           tmem_ld32(col + h0, v);
           tmem_ld32(col + h0 + 32, q);
           tmem_wait_ld();
@@ -391,8 +522,14 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
 #pragma unroll
           for (int j = 0; j < 16; ++j)
             pk[16 + j] = pack_bf16(__uint_as_float(q[2 * j]), __uint_as_float(q[2 * j + 1]));
-          // packed pairs of columns h0..h0+63 go to columns (h0/2)..(h0/2)+31 of the buffer
-          tmem_st32(col + h0 / 2, pk);
+          if (C::TF) {
+            // pre_p stays fp32 for the tf32 product: release the buffer before the stores
+            tc_fence_before();
+            warp_arrive(&bars->t_full[(c + C::NB) % C::NT]);
+          } else {
+            // packed pairs of columns h0..h0+63 go to columns (h0/2)..(h0/2)+31 of the buffer
+            tmem_st32(col + h0 / 2, pk);
+          }
           if (BWD) {
             // dM_p (bf16) transposed: dMT[(p*H + h) * ld_mt + row]
 #pragma unroll
@@ -404,12 +541,13 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
             }
           }
         }
-        tmem_wait_st();
-        tc_fence_before();
-        mbar_arrive(&bars->pre_ready[b]);
+        if (!C::TF) {
+          tmem_wait_st();
+          tc_fence_before();
+          warp_arrive(&bars->pre_ready[b]);
+        }
       }
       if (!ok) break;
-      if (cg != 0) continue;
       if (!mbar_wait(&bars->y_full, i & 1, status, 402, abort, 64)) break;
       tc_fence_after();
 #pragma unroll
@@ -417,6 +555,11 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
         uint32_t v[32];
         tmem_ld32(tmem + lane_base + C::YCOL + h0, v);
         tmem_wait_ld();
+        if (h0 + 32 >= H) {
+          // Y is in registers now: the next tile may start accumulating
+          tc_fence_before();
+          warp_arrive(&bars->y_empty);
+        }
         if (out) {
           float4* o = reinterpret_cast<float4*>(out + (size_t)row * H + h0);
 #pragma unroll
@@ -451,8 +594,6 @@ __global__ void __launch_bounds__(128 * (NE + NC + 1), 1)
           }
         }
       }
-      tc_fence_before();
-      mbar_arrive(&bars->y_empty);
     }
   }
   tc_fence_before();
@@ -491,6 +632,24 @@ __global__ void k_transpose_bf16(const T* __restrict__ in, __nv_bfloat16* __rest
   }
 }
 
+// Second-product weights in the band kernel's operand layout, for each type p:
+//   forward  out[p][o][i] = W[p][i][o]   (W_p^T, K-major in i)
+//   backward out[p][i][o] = W[p][i][o]   (W_p as given, K-major in o)
+// as fp32 (tf32 product) or bf16.
+template <typename TO>
+__global__ void k_prep_w(const __nv_bfloat16* __restrict__ W, TO* __restrict__ out, int P, int H,
+                         int transpose) {
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= (int64_t)P * H * H) return;
+  const int64_t p = t / ((int64_t)H * H);
+  const int a = (int)((t / H) % H), c = (int)(t % H);
+  const float v = __bfloat162float(transpose ? W[(p * H + c) * H + a] : W[(p * H + a) * H + c]);
+  if constexpr (sizeof(TO) == 4)
+    out[t] = v;
+  else
+    out[t] = __float2bfloat16_rn(v);
+}
+
 // b2T[h][p] = bf16 hi part of b[p][h], b2T[h][32 + p] = bf16 of the remainder (zero beyond P)
 __global__ void k_bias_split(const float* __restrict__ b, __nv_bfloat16* __restrict__ b2T, int P,
                              int H) {
@@ -525,6 +684,27 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, ui
   return make_map_ld(m, base, rows, cols, cols, box_rows);
 }
 
+// Row-major fp32 [rows][cols], boxes of 32 columns (one 128-byte swizzle row) x box_rows.
+bool make_map_f32(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols,
+                  uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 4};
+  cuuint32_t box[2] = {32, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// The W map of the band kernel: fp32 for the tf32 second product (H = 64), bf16 otherwise.
+bool make_map_w(CUtensorMap* m, const void* Wk, int P, int H) {
+  if (H <= 64) return make_map_f32(m, Wk, (uint64_t)P * H, H, H);
+  return make_map(m, Wk, (uint64_t)P * H, H, H);
+}
+
 int num_sms() {
   static int n = 0;
   if (!n) {
@@ -538,50 +718,22 @@ int num_sms() {
 
 inline size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-template <int H, bool BWD, int NE, int NC>
-cudaError_t launch_ne(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
-                   const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
-                   __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
-                   __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate, int* status,
-                   cudaStream_t st) {
-  using C = Cfg<H>;
-  cudaError_t e = cudaFuncSetAttribute(k_band_tc<H, BWD, NE, NC>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-  if (e != cudaSuccess) return e;
-  const int grid = std::min(p->K, num_sms());
-  k_band_tc<H, BWD, NE, NC><<<grid, 128 * (NE + NC + 1), C::SMEM, st>>>(
-      tx, tw, tdeg, tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt,
-      p->K, p->P, has_bias, accumulate, status);
-  note_launch();
-  return cudaGetLastError();
-}
-
-int group_config() {
-  static int cfg = -1;
-  if (cfg < 0) {
-    const char* v = getenv("BG_BAND_GROUPS");
-    cfg = v ? atoi(v) : 11;
-    if (cfg != 11 && cfg != 12 && cfg != 21 && cfg != 22) cfg = 11;
-  }
-  return cfg;
-}
-
 template <int H, bool BWD>
 cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
                    const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
                    __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
                    __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate, int* status,
                    cudaStream_t st) {
-#define BG_LAUNCH_NE(NEV, NCV)                                                                    \
-  return launch_ne<H, BWD, NEV, NCV>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, dMT, ld_mt, \
-                                     has_bias, accumulate, status, st);
-  switch (group_config()) {
-    case 21: BG_LAUNCH_NE(2, 1)
-    case 22: BG_LAUNCH_NE(2, 2)
-    case 12: BG_LAUNCH_NE(1, 2)
-    default: BG_LAUNCH_NE(1, 1)
-  }
-#undef BG_LAUNCH_NE
+  using C = Cfg<H>;
+  cudaError_t e = cudaFuncSetAttribute(k_band_tc<H, BWD>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  const int grid = std::min(p->K, num_sms());
+  k_band_tc<H, BWD><<<grid, kThreads, C::SMEM, st>>>(
+      tx, tw, tdeg, tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt,
+      p->K, p->P, has_bias, accumulate, status);
+  note_launch();
+  return cudaGetLastError();
 }
 
 }  // namespace
@@ -621,28 +773,46 @@ bool band_tc_supported(const bg_plan* p, int dtype, int H) {
          p->d_maskTI && p->d_deg2 && p->max_deg <= 256 && encode_fn() != nullptr;
 }
 
+size_t band_tc_w_bytes(const bg_plan* p, int H) {
+  return al256((size_t)p->P * H * H * (H <= 64 ? 4 : 2));
+}
+
+cudaError_t band_tc_prep_w(const bg_plan* p, int H, const void* W, int bwd, void* Wk,
+                           cudaStream_t st) {
+  const int64_t n = (int64_t)p->P * H * H;
+  const int blocks = (int)((n + 255) / 256);
+  const auto* w = static_cast<const __nv_bfloat16*>(W);
+  if (H <= 64)
+    k_prep_w<float><<<blocks, 256, 0, st>>>(w, static_cast<float*>(Wk), p->P, H, !bwd);
+  else
+    k_prep_w<__nv_bfloat16><<<blocks, 256, 0, st>>>(w, static_cast<__nv_bfloat16*>(Wk), p->P, H,
+                                                    !bwd);
+  note_launch();
+  return cudaGetLastError();
+}
+
 size_t band_tc_fwd_ws_bytes(const bg_plan* p, int dtype, int H) {
   if (!p || dtype != 1) return 0;
   const size_t n = (size_t)p->n_pad();
-  return al256(n * H * 2) + al256((size_t)p->P * H * H * 2) + al256((size_t)H * 64 * 2);
+  return al256(n * H * 2) + band_tc_w_bytes(p, H) + al256((size_t)H * 64 * 2);
 }
 
 size_t band_tc_bwd_ws_bytes(const bg_plan* p, int dtype, int H) {
   if (!p || dtype != 1) return 0;
   const size_t n = (size_t)p->n_pad();
   return al256(n * H * 2) + al256((size_t)p->P * H * n * 2) + al256((size_t)(H + 16) * n * 2) +
-         al256((size_t)H * 64 * 2) +
+         band_tc_w_bytes(p, H) +
          al256(sizeof(float) * gemm_tn_part_floats(p->P * H, H + 16, (int64_t)n));
 }
 
 cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, int64_t ld_x,
-                             const __nv_bfloat16* WT, const __nv_bfloat16* b2T, float* out,
+                             const void* Wk, const __nv_bfloat16* b2T, float* out,
                              __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
                              int* status, cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw, tdeg, tb2;
-  if (!make_map_ld(&tx, XT, H, n, ld_x, H) || !make_map(&tw, WT, (uint64_t)P * H, H, H) ||
-      !make_map(&tdeg, p->d_deg2, n, 64, kTile) || !make_map(&tb2, b2T ? b2T : WT, H, 64, H))
+  if (!make_map_ld(&tx, XT, H, n, ld_x, H) || !make_map_w(&tw, Wk, P, H) ||
+      !make_map(&tdeg, p->d_deg2, n, 64, kTile) || !make_map(&tb2, b2T ? b2T : XT, H, 64, H))
     return cudaErrorInvalidValue;
   const int has_bias = b2T != nullptr;
   if (H == 64)
@@ -653,11 +823,11 @@ cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, i
 }
 
 cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, int64_t ld_y,
-                             const void* W, float* dE, int accumulate, __nv_bfloat16* dMT,
+                             const void* Wk, float* dE, int accumulate, __nv_bfloat16* dMT,
                              int64_t ld_mt, int* status, cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw;
-  if (!make_map_ld(&tx, dYT, H, n, ld_y, H) || !make_map(&tw, W, (uint64_t)P * H, H, H))
+  if (!make_map_ld(&tx, dYT, H, n, ld_y, H) || !make_map_w(&tw, Wk, P, H))
     return cudaErrorInvalidValue;
   if (H == 64)
     return launch<64, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
@@ -692,12 +862,12 @@ cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, c
   if (ws_bytes < band_tc_fwd_ws_bytes(p, 1, H)) return cudaErrorInvalidValue;
   const int n = p->n_pad(), P = p->P;
   __nv_bfloat16* ET = reinterpret_cast<__nv_bfloat16*>(ws);
-  __nv_bfloat16* WT = reinterpret_cast<__nv_bfloat16*>(ws + al256((size_t)n * H * 2));
+  void* WT = ws + al256((size_t)n * H * 2);
   __nv_bfloat16* b2T = reinterpret_cast<__nv_bfloat16*>(ws + al256((size_t)n * H * 2) +
-                                                        al256((size_t)P * H * H * 2));
-  // E [n][H] -> ET [H][n];  W_p [H_in][H_out] -> WT_p [H_out][H_in];  bias split
+                                                        band_tc_w_bytes(p, H));
+  // E [n][H] -> ET [H][n];  W_p [H_in][H_out] -> W_p^T in the kernel's operand type;  bias split
   cudaError_t e = prep_transpose_bf16(E, 0, ET, n, H, 1, st);
-  if (e == cudaSuccess) e = prep_transpose_bf16(W, 0, WT, H, H, P, st);
+  if (e == cudaSuccess) e = band_tc_prep_w(p, H, W, 0, WT, st);
   if (e == cudaSuccess && b) e = prep_bias_split(b, b2T, P, H, st);
   if (e != cudaSuccess) return e;
   return band_tc_fwd_core(p, H, ET, n, WT, b ? b2T : nullptr, Y, nullptr, nullptr, 0, status, st);
@@ -715,11 +885,13 @@ cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, c
   o += al256((size_t)P * H * n * 2);
   __nv_bfloat16* ETa = reinterpret_cast<__nv_bfloat16*>(ws + o);
   o += al256((size_t)(H + 16) * n * 2);
-  o += al256((size_t)H * 64 * 2);
+  void* Wk = ws + o;
+  o += band_tc_w_bytes(p, H);
   float* part = reinterpret_cast<float*>(ws + o);
   const size_t part_floats = gemm_tn_part_floats(P * H, H + 16, (int64_t)n);
   cudaError_t e = prep_transpose_bf16(dY, 1, dYT, n, H, 1, st);
-  if (e == cudaSuccess) e = band_tc_bwd_core(p, H, dYT, n, W, dE, accum, dMT, n, status, st);
+  if (e == cudaSuccess) e = band_tc_prep_w(p, H, W, 1, Wk, st);
+  if (e == cudaSuccess) e = band_tc_bwd_core(p, H, dYT, n, Wk, dE, accum, dMT, n, status, st);
   if (e != cudaSuccess) return e;
   // [E^T; 1; 0]: the ones row turns the bias gradient into column H of the same product
   e = prep_transpose_bf16(E, 0, ETa, n, H, 1, st);

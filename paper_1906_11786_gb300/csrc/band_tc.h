@@ -19,17 +19,23 @@ cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, c
 cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, const float* dY,
                         float* dE, float* dW, float* db, int accum, char* ws, size_t ws_bytes,
                         int* status, cudaStream_t st);
+// The band kernel's second-product weights (band_tc_w_bytes): from W [P][H][H] bf16, the forward
+// operand W_p^T (bwd = 0) or the backward operand W_p (bwd = 1), fp32 at H = 64 (kind::tf32
+// product) and bf16 at H = 128.
+size_t band_tc_w_bytes(const bg_plan* p, int H);
+cudaError_t band_tc_prep_w(const bg_plan* p, int H, const void* W, int bwd, void* Wk,
+                           cudaStream_t st);
 // Kernel-level entry points used by the fused GGNN steps (operands already in kernel layout):
-//   XT: [H][>= n_pad] bf16 transposed states (row stride ld_x); WT: [P][H_out][H_in] bf16;
+//   XT: [H][>= n_pad] bf16 transposed states (row stride ld_x); Wk: band_tc_prep_w(bwd = 0);
 //   b2T: [H][64] bf16 bias split or NULL.  Outputs (each optional): out fp32 [n][H],
 //   outb bf16 [n][H], outT bf16 [H][ld_outT].
 cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, int64_t ld_x,
-                             const __nv_bfloat16* WT, const __nv_bfloat16* b2T, float* out,
+                             const void* Wk, const __nv_bfloat16* b2T, float* out,
                              __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
                              int* status, cudaStream_t st);
-//   dYT: [H][>= n_pad] bf16; W: [P][H][H] bf16 as given; dE fp32 (+)=; dMT: [P*H][ld_mt] bf16.
+//   dYT: [H][>= n_pad] bf16; Wk: band_tc_prep_w(bwd = 1); dE fp32 (+)=; dMT: [P*H][ld_mt] bf16.
 cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, int64_t ld_y,
-                             const void* W, float* dE, int accumulate, __nv_bfloat16* dMT,
+                             const void* Wk, float* dE, int accumulate, __nv_bfloat16* dMT,
                              int64_t ld_mt, int* status, cudaStream_t st);
 // out[c * ld_out + r] = bf16(in[r][c]) for `batch` consecutive R x Cc matrices (in fp32 or bf16;
 // ld_out <= 0 means R; batches are R*Cc apart on both sides).
