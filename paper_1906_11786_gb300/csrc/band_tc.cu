@@ -19,16 +19,17 @@
 // each 32-column word are interleaved at upload (column 2j at bit j, column 2j+1 at bit 16+j) so
 // that one AND and one multiply give the packed bf16 pair {1.0 or 0, 1.0 or 0}.
 //
-// Roles (384 threads, one CTA per SM, persistent over tiles):
+// Roles (128 x (2 + expander groups) threads, one CTA per SM, persistent over tiles):
 //   warp 0      TMA producer: state blocks (B operand of the band product), W tiles, deg, bias
 //   warp 1      TMEM allocator and MMA issuer (an elected lane of the converged warp issues):
 //               at H = 64 the band products only, one wait per edge type; otherwise every MMA
 //   warp 2      mask producer: one bulk copy per (tile, type) of the bit tiles into an SMEM ring
 //   warp 3      (H = 64) second MMA issuer: the pre_p W_p products and the bias product, so that
 //               their waits never stall the band-product stream
-//   warps 4-7   expanders: thread r turns row r's mask bits into bf16 A tiles in TMEM
-//   warps 8-11  converters: pre_p fp32 -> bf16 (H = 128), dM_p to global (backward), final
-//               epilogue TMEM -> global
+//   expanders   thread r of a warpgroup turns row r's mask bits into bf16 A tiles in TMEM; two
+//               warpgroups taking the edge types in turn at H = 64 (warps 4-11), one otherwise
+//   converters  the last warpgroup: pre_p fp32 -> bf16 (H = 128), dM_p to global (backward),
+//               final epilogue TMEM -> global
 // A tcgen05.mma of N = 64 is about as long as its issue, so any wait on the band-product
 // issuer leaves the tensor pipe idle: at H = 64 that issuer waits once per edge type, on a
 // barrier that the expanders (all three A tiles in TMEM), the second issuer (the pre_p buffer is
@@ -85,6 +86,9 @@ struct Cfg {
   static constexpr int ACOL = (NB + 1) * H;
   static constexpr int NA = (512 - ACOL) / 64;
   static constexpr int NT = 8;                                // per-type barrier ring (H = 64)
+  // expander warpgroups: at H = 64 two, taking the edge types in turn
+  static constexpr int NE = TF ? 2 : 1;
+  static constexpr int THREADS = 128 * (2 + NE);
   static_assert(NA >= 2 && NA <= 8, "A-slot ring");
   static_assert(!TF || NA >= 3, "one edge type's three A tiles must fit");
   static_assert(SMEM <= 232448, "shared memory");
@@ -139,10 +143,8 @@ __device__ __forceinline__ void drain_mmas(bool leader, uint64_t* bar) {
   }
 }
 
-constexpr int kThreads = 384;
-
 template <int H, bool BWD>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
     k_band_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
               const __grid_constant__ CUtensorMap tm_deg, const __grid_constant__ CUtensorMap tm_b2,
               const uint32_t* __restrict__ maskI, float* __restrict__ out,
@@ -446,14 +448,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (leader) tc_commit(&bars->y_full);
     }
     drain_mmas(leader, &bars->drain);
-  } else if (warp >= 4 && warp < 8) {
+  } else if (warp >= 4 && warp < 4 + 4 * C::NE) {
     // ------------------------------------------------------------------ expanders
-    const int r = threadIdx.x - 128;
+    const int eg = (warp - 4) / 4;
+    const int r = (threadIdx.x - 128) % 128;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     uint32_t aidx = 0, midx = 0;
     for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x) {
       bool ok = true;
+      const int n_diag = (k > 0) + 1 + (k + 1 < K);
       for (int p = 0; p < P && ok; ++p, ++midx) {
+        if (C::NE > 1 && (int)(midx % C::NE) != eg) {
+          aidx += n_diag;  // the other group's type
+          continue;
+        }
         const int ms = midx % C::NM;
         if (!mbar_wait(&bars->m_full[ms], (midx / C::NM) & 1, status, 302, abort, 32)) {
           ok = false;
@@ -495,9 +503,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!ok) break;
     }
-  } else if (warp >= 8) {
+  } else if (warp >= 4 + 4 * C::NE) {
     // ------------------------------------------------------------------ converters / epilogue
-    const int r = threadIdx.x - 256;
+    const int r = threadIdx.x - 128 * (1 + C::NE);
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     uint32_t c = 0;
     int i = 0;
@@ -729,7 +737,7 @@ cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& t
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
   const int grid = std::min(p->K, num_sms());
-  k_band_tc<H, BWD><<<grid, kThreads, C::SMEM, st>>>(
+  k_band_tc<H, BWD><<<grid, C::THREADS, C::SMEM, st>>>(
       tx, tw, tdeg, tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt,
       p->K, p->P, has_bias, accumulate, status);
   note_launch();
