@@ -58,7 +58,14 @@ __device__ __forceinline__ uint32_t pk2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
-__device__ __forceinline__ float sigm(float x) { return 1.f / (1.f + __expf(-x)); }
+// tanh on the special-function unit (tanh.approx.f32: relative error about 2^-11, below the bf16
+// rounding of the state) and the logistic function through sigma(x) = (1 + tanh(x / 2)) / 2
+__device__ __forceinline__ float tanh_fast(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float sigm(float x) { return fmaf(0.5f, tanh_fast(0.5f * x), 0.5f); }
 
 // 32 consecutive bf16 of row r (columns c0 .. c0+31, c0 % 32 == 0) of a 128-row K-major tile
 // stored with the 128-byte swizzle (16-byte chunk j of row r sits at chunk j ^ (r % 8)).
@@ -274,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int h = h0 + j + u;
           const float rr = sigm(__uint_as_float(vr[j + u]) + bias[h] + bias[3 * kH + h]);
           const float zz = sigm(__uint_as_float(vz[j + u]) + bias[kH + h] + bias[4 * kH + h]);
-          const float nn = tanhf(__uint_as_float(vn[j + u]) + bias[2 * kH + h] +
+          const float nn = tanh_fast(__uint_as_float(vn[j + u]) + bias[2 * kH + h] +
                                  rr * (__uint_as_float(vh[j + u]) + bias[5 * kH + h]));
           o[u] = real ? (1.f - zz) * nn + zz * e[j + u] : 0.f;
         }
@@ -422,7 +429,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float rr = sigm(__uint_as_float(vr[j]) + bias[h] + bias[3 * kH + h]);
             const float zz = sigm(__uint_as_float(vz[j]) + bias[kH + h] + bias[4 * kH + h]);
             const float ghn = __uint_as_float(vh[j]) + bias[5 * kH + h];
-            const float nn = tanhf(__uint_as_float(vn[j]) + bias[2 * kH + h] + rr * ghn);
+            const float nn = tanh_fast(__uint_as_float(vn[j]) + bias[2 * kH + h] + rr * ghn);
             const float gr = real ? gg[u] : 0.f;
             const float an = gr * (1.f - zz) * (1.f - nn * nn);
             dn[u] = an;
