@@ -375,7 +375,9 @@ cudaError_t gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int 
   const int64_t kchunks = (K + 63) / 64;
   const int mt = (M + 127) / 128;
   const int sms = gemm_tn_num_sms();
-  int splits = (int)std::max<int64_t>(1, std::min<int64_t>(kchunks, (2 * sms + mt - 1) / mt));
+  // two CTAs fit per SM: at most 2 * sms CTAs, so that all of them run in one wave (a partial
+  // second wave of even a few CTAs would nearly double the time of this HBM-bound pass)
+  int splits = (int)std::max<int64_t>(1, std::min<int64_t>(kchunks, std::max(1, 2 * sms / mt)));
   while (splits > 1 && (size_t)splits * M * N > part_floats) --splits;
   const int per = (int)((kchunks + splits - 1) / splits);
   splits = (int)((kchunks + per - 1) / per);

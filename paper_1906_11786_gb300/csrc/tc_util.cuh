@@ -55,12 +55,9 @@ __device__ __forceinline__ bool mbar_try(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Waits for phase `parity` of `bar` to complete; false (and a recorded timeout) if the poll
-// limit is reached or another role already gave up (*abort set).  backoff_ns > 0 sleeps between
-// polls so that waiting warps leave issue slots to the warps doing the work (the MMA issuer polls
-// with backoff_ns = 0).
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* status, int site,
-                                          volatile int* abort, uint32_t backoff_ns = 0) {
+// Slow path of mbar_wait: bounded polling after a first failed check.
+static __device__ __noinline__ bool mbar_wait_poll(uint64_t* bar, uint32_t parity, int* status, int site,
+                                            volatile int* abort, uint32_t backoff_ns) {
   for (uint32_t i = 0; i < kSpinLimit; ++i) {
     if (mbar_try(bar, parity)) return true;
     if ((i & 1023u) == 1023u && *abort) return false;
@@ -69,6 +66,17 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* s
   if (atomicCAS(status, 0, 1) == 0) atomicExch(status + 1, site);
   *abort = 1;
   return false;
+}
+
+// Waits for phase `parity` of `bar` to complete; false (and a recorded timeout) if the poll
+// limit is reached or another role already gave up (*abort set).  backoff_ns > 0 sleeps between
+// polls so that waiting warps leave issue slots to the warps doing the work (the MMA issuers poll
+// with backoff_ns = 0).  A phase that is already complete costs one check: the polling loop is out
+// of line so that it adds nothing to an MMA issuer's instruction stream.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* status, int site,
+                                          volatile int* abort, uint32_t backoff_ns = 0) {
+  if (mbar_try(bar, parity)) return true;
+  return mbar_wait_poll(bar, parity, status, site, abort, backoff_ns);
 }
 
 // One lane of a converged warp (the lane that issues tcgen05.mma / commit for the whole warp).
