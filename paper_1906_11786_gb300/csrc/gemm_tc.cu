@@ -153,11 +153,22 @@ __global__ void k_gemm_tn_reduce(const float* __restrict__ part, int splits, int
                                  int mode, float* __restrict__ out, float* __restrict__ bias,
                                  int accumulate) {
   const int64_t total = (int64_t)M * (Hout + 1);
+  const size_t stride = (size_t)M * N;
   for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total;
        t += (int64_t)gridDim.x * blockDim.x) {
     const int m = (int)(t / (Hout + 1)), n = (int)(t % (Hout + 1));
-    float s = 0.f;
-    for (int q = 0; q < splits; ++q) s += part[((size_t)q * M + m) * N + n];
+    const float* src = part + (size_t)m * N + n;
+    // four independent partial sums keep several loads in flight; fixed order, so deterministic
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+    int q = 0;
+    for (; q + 4 <= splits; q += 4) {
+      s0 += src[(size_t)q * stride];
+      s1 += src[(size_t)(q + 1) * stride];
+      s2 += src[(size_t)(q + 2) * stride];
+      s3 += src[(size_t)(q + 3) * stride];
+    }
+    for (; q < splits; ++q) s0 += src[(size_t)q * stride];
+    const float s = (s0 + s1) + (s2 + s3);
     float* dst;
     if (n == Hout) {
       if (!bias) continue;
@@ -311,18 +322,21 @@ __global__ void __launch_bounds__(192, 1)
 
 namespace {
 __global__ void k_fill_ones_rows(__nv_bfloat16* base, int H, int64_t n, int64_t ld) {
-  const int64_t total = 16 * n;
+  // row H: ones, rows H+1 .. H+15: zeros; 16-byte stores (ld and n are multiples of 8 elements)
+  const int64_t per_row = n / 8, total = 16 * per_row;
   for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total;
        t += (int64_t)gridDim.x * blockDim.x) {
-    const int r = (int)(t / n);
-    const int64_t c = t % n;
-    base[(int64_t)(H + r) * ld + c] = __float2bfloat16_rn(r == 0 ? 1.f : 0.f);
+    const int r = (int)(t / per_row);
+    const int64_t c = (t - r * per_row) * 8;
+    const uint32_t v = r == 0 ? 0x3F803F80u : 0u;  // bf16 1.0 pairs
+    *reinterpret_cast<uint4*>(base + (int64_t)(H + r) * ld + c) = make_uint4(v, v, v, v);
   }
 }
 }  // namespace
 
 cudaError_t fill_ones_rows(__nv_bfloat16* base, int H, int64_t n, int64_t ld, cudaStream_t st) {
-  const int64_t total = 16 * n;
+  if ((n % 8) || (ld % 8) || (reinterpret_cast<uintptr_t>(base) % 16)) return cudaErrorInvalidValue;
+  const int64_t total = 2 * n;  // 16 rows x n / 8 vectors
   k_fill_ones_rows<<<(unsigned)std::min<int64_t>((total + 255) / 256, 8192), 256, 0, st>>>(base, H,
                                                                                           n, ld);
   note_launch();
