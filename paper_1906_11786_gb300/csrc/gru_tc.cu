@@ -14,8 +14,8 @@
 //
 // Both kernels are persistent (one CTA per SM) and warp-specialised: warp 0 streams 128-row
 // tiles of Y and E through a two-stage TMA ring (the weights stay resident), warp 1 issues the
-// MMAs into two TMEM accumulator sets, and two epilogue warpgroups (one per 32-column half) drain
-// them, so loads and MMAs of tile i+1 overlap the epilogue of tile i.
+// MMAs into two TMEM accumulator sets, and four epilogue warpgroups (one per 16 state columns,
+// eight at a time) drain them, so loads and MMAs of tile i+1 overlap the epilogue of tile i.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -33,15 +33,9 @@ using namespace tc;
 namespace {
 
 constexpr int kH = 64;        // state size handled by these kernels
-constexpr int kThreads = 384; // warp 0 TMA, warp 1 MMA, warps 4-11 epilogue (two groups)
+constexpr int kEpiWarps = 16; // four epilogue warpgroups, 16 state columns each
+constexpr int kThreads = 128 + 32 * kEpiWarps;  // warp 0 TMA, warp 1 MMA, warps 4-19 epilogue
 constexpr int kAcc = 4 * kH;  // TMEM columns per accumulator set
-
-__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t* r) {
-  asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr),
-               "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]),
-               "r"(r[7])
-               : "memory");
-}
 
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
   asm volatile(
@@ -51,6 +45,25 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
         "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
         "=r"(r[14]), "=r"(r[15])
       : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t* r) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
+                 "=r"(r[6]), "=r"(r[7])
+               : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_st4(uint32_t taddr, const uint32_t* r) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1,%2,%3,%4};" ::"r"(taddr), "r"(r[0]),
+               "r"(r[1]), "r"(r[2]), "r"(r[3])
+               : "memory");
+}
+
+// One arrive per warp once every lane of it is done.
+__device__ __forceinline__ void warp_arrive(uint64_t* bar) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
 }
 
 __device__ __forceinline__ uint32_t pk2(float lo, float hi) {
@@ -67,36 +80,26 @@ __device__ __forceinline__ float tanh_fast(float x) {
 }
 __device__ __forceinline__ float sigm(float x) { return fmaf(0.5f, tanh_fast(0.5f * x), 0.5f); }
 
-// 32 consecutive bf16 of row r (columns c0 .. c0+31, c0 % 32 == 0) of a 128-row K-major tile
-// stored with the 128-byte swizzle (16-byte chunk j of row r sits at chunk j ^ (r % 8)).
-__device__ __forceinline__ void read_sw128_row32(const uint8_t* tile, int r, int c0, float* out) {
+// 8 consecutive bf16 of row r (columns c0 .. c0+7, c0 % 8 == 0): one swizzled 16-byte chunk.
+__device__ __forceinline__ void read_sw128_row8(const uint8_t* tile, int r, int c0, float* out) {
   const uint8_t* row = tile + (c0 / 64) * 128 * 128 + r * 128;
-  const int j0 = (c0 % 64) / 8;
+  const uint4 v = *reinterpret_cast<const uint4*>(row + ((((c0 % 64) / 8) ^ (r & 7)) << 4));
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const uint4 v = *reinterpret_cast<const uint4*>(row + (((j0 + q) ^ (r & 7)) << 4));
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      out[q * 8 + 2 * e] = __uint_as_float(w[e] << 16);
-      out[q * 8 + 2 * e + 1] = __uint_as_float(w[e] & 0xFFFF0000u);
-    }
+  for (int e = 0; e < 4; ++e) {
+    out[2 * e] = __uint_as_float(w[e] << 16);
+    out[2 * e + 1] = __uint_as_float(w[e] & 0xFFFF0000u);
   }
 }
 
-// 16 consecutive bf16 of row r (columns c0 .. c0+15, c0 % 16 == 0) of the same tile layout.
-__device__ __forceinline__ void read_sw128_row16(const uint8_t* tile, int r, int c0, float* out) {
-  const uint8_t* row = tile + (c0 / 64) * 128 * 128 + r * 128;
-  const int j0 = (c0 % 64) / 8;
+// 4 bf16 pairs stored transposed: dst[(h0 + 2j + u) * ld + row]
+__device__ __forceinline__ void store_T4(__nv_bfloat16* dst, int64_t ld, int row, int h0,
+                                         const uint32_t* pk) {
 #pragma unroll
-  for (int q = 0; q < 2; ++q) {
-    const uint4 v = *reinterpret_cast<const uint4*>(row + (((j0 + q) ^ (r & 7)) << 4));
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      out[q * 8 + 2 * e] = __uint_as_float(w[e] << 16);
-      out[q * 8 + 2 * e + 1] = __uint_as_float(w[e] & 0xFFFF0000u);
-    }
+  for (int j = 0; j < 4; ++j) {
+    __nv_bfloat16* t = dst + (size_t)(h0 + 2 * j) * ld + row;
+    t[0] = __ushort_as_bfloat16((unsigned short)(pk[j] & 0xFFFFu));
+    t[ld] = __ushort_as_bfloat16((unsigned short)(pk[j] >> 16));
   }
 }
 
@@ -105,17 +108,6 @@ __device__ __forceinline__ void store_T8(__nv_bfloat16* dst, int64_t ld, int row
                                          const uint32_t* pk) {
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    __nv_bfloat16* t = dst + (size_t)(h0 + 2 * j) * ld + row;
-    t[0] = __ushort_as_bfloat16((unsigned short)(pk[j] & 0xFFFFu));
-    t[ld] = __ushort_as_bfloat16((unsigned short)(pk[j] >> 16));
-  }
-}
-
-// 32 bf16 pairs (64 values of consecutive rows) stored transposed: dst[(h0 + 2j + u) * ld + row]
-__device__ __forceinline__ void store_T16(__nv_bfloat16* dst, int64_t ld, int row, int h0,
-                                          const uint32_t* pk) {
-#pragma unroll
-  for (int j = 0; j < 16; ++j) {
     __nv_bfloat16* t = dst + (size_t)(h0 + 2 * j) * ld + row;
     t[0] = __ushort_as_bfloat16((unsigned short)(pk[j] & 0xFFFFu));
     t[ld] = __ushort_as_bfloat16((unsigned short)(pk[j] >> 16));
@@ -163,10 +155,10 @@ __device__ __forceinline__ void gru_setup(GruBars* b, float* bias, const float* 
     mbar_init(&b->w_full, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&b->t_full[i], 1);
-      mbar_init(&b->t_empty[i], 256);
+      mbar_init(&b->t_empty[i], kEpiWarps);
       mbar_init(&b->acc_full[i], 1);
-      mbar_init(&b->acc_empty[i], 256);
-      mbar_init(&b->ops_ready[i], 256);
+      mbar_init(&b->acc_empty[i], kEpiWarps);
+      mbar_init(&b->ops_ready[i], kEpiWarps);
       mbar_init(&b->ph2_full[i], 1);
     }
     mbar_init(&b->drain, 1);
@@ -250,7 +242,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (uint32_t k = 0; k < (1u << 24) && !mbar_try(&bars.drain, 0); ++k) {
     }
   } else if (warp >= 4) {
-    const int g = (warp - 4) / 4, h0 = 32 * g;
+    const int g = (warp - 4) / 4, h0 = 16 * g;
     const int r = (warp & 3) * 32 + lane;
     const uint32_t lb = (uint32_t)((warp & 3) * 32) << 16;
     int i = 0;
@@ -259,38 +251,44 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!mbar_wait(&bars.acc_full[a], (i >> 1) & 1, status, 615, abort, 64)) break;
       tc_fence_after();
       const uint32_t acc = tmem + lb + a * kAcc;
-      uint32_t vr[32], vz[32], vn[32], vh[32];
-      tmem_ld32(acc + h0, vr);
-      tmem_ld32(acc + kH + h0, vz);
-      tmem_ld32(acc + 2 * kH + h0, vn);
-      tmem_ld32(acc + 3 * kH + h0, vh);
-      tmem_wait_ld();
-      float e[32];
-      read_sw128_row32(ring + s * 2 * GruSmem::TILE + GruSmem::TILE, r, h0, e);
-      tc_fence_before();
-      mbar_arrive(&bars.acc_empty[a]);
-      mbar_arrive(&bars.t_empty[s]);
+      const uint8_t* etile = ring + s * 2 * GruSmem::TILE + GruSmem::TILE;
       const int row = t * 128 + r;
       const bool real = row < n_real;
-      uint32_t pk[16];
 #pragma unroll
-      for (int j = 0; j < 32; j += 2) {
-        float o[2];
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const int h = h0 + j + u;
-          const float rr = sigm(__uint_as_float(vr[j + u]) + bias[h] + bias[3 * kH + h]);
-          const float zz = sigm(__uint_as_float(vz[j + u]) + bias[kH + h] + bias[4 * kH + h]);
-          const float nn = tanh_fast(__uint_as_float(vn[j + u]) + bias[2 * kH + h] +
-                                 rr * (__uint_as_float(vh[j + u]) + bias[5 * kH + h]));
-          o[u] = real ? (1.f - zz) * nn + zz * e[j + u] : 0.f;
+      for (int hh = 0; hh < 2; ++hh) {
+        const int hs = h0 + 8 * hh;
+        uint32_t vr[8], vz[8], vn[8], vh[8];
+        tmem_ld8(acc + hs, vr);
+        tmem_ld8(acc + kH + hs, vz);
+        tmem_ld8(acc + 2 * kH + hs, vn);
+        tmem_ld8(acc + 3 * kH + hs, vh);
+        tmem_wait_ld();
+        float e[8];
+        read_sw128_row8(etile, r, hs, e);
+        if (hh == 1) {
+          // accumulators and the state tile of this tile are no longer needed
+          tc_fence_before();
+          warp_arrive(&bars.acc_empty[a]);
+          warp_arrive(&bars.t_empty[s]);
         }
-        pk[j / 2] = pk2(o[0], o[1]);
-      }
-      uint4* d = reinterpret_cast<uint4*>(En + (size_t)row * kH + h0);
+        uint32_t pk[4];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) d[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
-      if (EnT) store_T16(EnT, ld_T, row, h0, pk);
+        for (int j = 0; j < 8; j += 2) {
+          float o[2];
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int h = hs + j + u;
+            const float rr = sigm(__uint_as_float(vr[j + u]) + bias[h] + bias[3 * kH + h]);
+            const float zz = sigm(__uint_as_float(vz[j + u]) + bias[kH + h] + bias[4 * kH + h]);
+            const float nn = tanh_fast(__uint_as_float(vn[j + u]) + bias[2 * kH + h] +
+                                       rr * (__uint_as_float(vh[j + u]) + bias[5 * kH + h]));
+            o[u] = real ? (1.f - zz) * nn + zz * e[j + u] : 0.f;
+          }
+          pk[j / 2] = pk2(o[0], o[1]);
+        }
+        *reinterpret_cast<uint4*>(En + (size_t)row * kH + hs) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        if (EnT) store_T4(EnT, ld_T, row, hs, pk);
+      }
     }
   }
   tc_fence_before();
@@ -392,7 +390,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (uint32_t k = 0; k < (1u << 24) && !mbar_try(&bars.drain, 0); ++k) {
     }
   } else if (warp >= 4) {
-    const int c = (warp - 4) / 4, h0 = 32 * c;
+    const int g = (warp - 4) / 4, h0 = 16 * g;
     const int r = (warp & 3) * 32 + lane;
     const uint32_t lb = (uint32_t)((warp & 3) * 32) << 16;
     int i = 0;
@@ -404,22 +402,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const uint32_t acc = tmem + lb + a * kAcc;
       const uint8_t* etile = ring + s * 2 * GruSmem::TILE + GruSmem::TILE;
-      float dhd[32];
+      float dhd[16];
+      // packed gate gradients of both halves: the in-place rewrite below overwrites columns that
+      // the second half still reads, so it waits until both halves are in registers
+      uint32_t p_r[8], p_z[8], p_n[8], p_hn[8];
 #pragma unroll
-      for (int sb = 0; sb < 2; ++sb) {
-        const int hs = h0 + 16 * sb;
-        uint32_t vr[16], vz[16], vn[16], vh[16];
-        tmem_ld16(acc + hs, vr);
-        tmem_ld16(acc + kH + hs, vz);
-        tmem_ld16(acc + 2 * kH + hs, vn);
-        tmem_ld16(acc + 3 * kH + hs, vh);
+      for (int hh = 0; hh < 2; ++hh) {
+        // columns hs .. hs+7: pairs 4hh .. 4hh+3 of this warpgroup's 16-column window h0
+        const int hs = h0 + 8 * hh;
+        uint32_t vr[8], vz[8], vn[8], vh[8];
+        tmem_ld8(acc + hs, vr);
+        tmem_ld8(acc + kH + hs, vz);
+        tmem_ld8(acc + 2 * kH + hs, vn);
+        tmem_ld8(acc + 3 * kH + hs, vh);
         tmem_wait_ld();
-        float e[16];
-        read_sw128_row16(etile, r, hs, e);
+        float e[8];
+        read_sw128_row8(etile, r, hs, e);
+        if (hh == 1) warp_arrive(&bars.t_empty[s]);
         const float4* g4 = reinterpret_cast<const float4*>(gin + (size_t)row * kH + hs);
-        uint32_t p_r[8], p_z[8], p_n[8], p_hn[8];
+        const int o = 4 * hh;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
+        for (int q = 0; q < 2; ++q) {
           const float4 gv = g4[q];
           const float gg[4] = {gv.x, gv.y, gv.z, gv.w};
           float dr[4], dz[4], dn[4], dhn[4];
@@ -436,45 +439,49 @@ __global__ void __launch_bounds__(kThreads, 1)
             dhn[u] = an * rr;
             dr[u] = an * ghn * rr * (1.f - rr);
             dz[u] = gr * (e[j] - nn) * zz * (1.f - zz);
-            dhd[16 * sb + j] = gr * zz;
+            dhd[8 * hh + j] = gr * zz;
           }
-          p_r[2 * q] = pk2(dr[0], dr[1]); p_r[2 * q + 1] = pk2(dr[2], dr[3]);
-          p_z[2 * q] = pk2(dz[0], dz[1]); p_z[2 * q + 1] = pk2(dz[2], dz[3]);
-          p_n[2 * q] = pk2(dn[0], dn[1]); p_n[2 * q + 1] = pk2(dn[2], dn[3]);
-          p_hn[2 * q] = pk2(dhn[0], dhn[1]); p_hn[2 * q + 1] = pk2(dhn[2], dhn[3]);
+          p_r[o + 2 * q] = pk2(dr[0], dr[1]); p_r[o + 2 * q + 1] = pk2(dr[2], dr[3]);
+          p_z[o + 2 * q] = pk2(dz[0], dz[1]); p_z[o + 2 * q + 1] = pk2(dz[2], dz[3]);
+          p_n[o + 2 * q] = pk2(dn[0], dn[1]); p_n[o + 2 * q + 1] = pk2(dn[2], dn[3]);
+          p_hn[o + 2 * q] = pk2(dhn[0], dhn[1]); p_hn[o + 2 * q + 1] = pk2(dhn[2], dhn[3]);
         }
-        // in-place rewrite into the columns just read (see dg_col)
-        tmem_st8(acc + hs, p_r);
-        tmem_st8(acc + hs + 8, p_z);
-        tmem_st8(acc + kH + hs, p_n);
-        tmem_st8(acc + kH + hs + 8, p_hn);
         // gate gradients transposed for the weight-gradient GEMM: rows o = gate*H + h
-        store_T8(dgiT, ld_g, row, hs, p_r);
-        store_T8(dgiT + (size_t)kH * ld_g, ld_g, row, hs, p_z);
-        store_T8(dgiT + (size_t)2 * kH * ld_g, ld_g, row, hs, p_n);
-        store_T8(dghT, ld_g, row, hs, p_r);
-        store_T8(dghT + (size_t)kH * ld_g, ld_g, row, hs, p_z);
-        store_T8(dghT + (size_t)2 * kH * ld_g, ld_g, row, hs, p_hn);
+        store_T4(dgiT, ld_g, row, hs, p_r + o);
+        store_T4(dgiT + (size_t)kH * ld_g, ld_g, row, hs, p_z + o);
+        store_T4(dgiT + (size_t)2 * kH * ld_g, ld_g, row, hs, p_n + o);
+        store_T4(dghT, ld_g, row, hs, p_r + o);
+        store_T4(dghT + (size_t)kH * ld_g, ld_g, row, hs, p_z + o);
+        store_T4(dghT + (size_t)2 * kH * ld_g, ld_g, row, hs, p_hn + o);
       }
-      mbar_arrive(&bars.t_empty[s]);
+      // in-place rewrite into the columns just read (see dg_col): within the 16-column window h0,
+      // r holds the 8 (dgi_r) pair columns then the 8 (dgi_z) ones, z the (dgi_n) then (dgh_n)
+      tmem_st4(acc + h0, p_r);
+      tmem_st4(acc + h0 + 4, p_r + 4);
+      tmem_st4(acc + h0 + 8, p_z);
+      tmem_st4(acc + h0 + 12, p_z + 4);
+      tmem_st4(acc + kH + h0, p_n);
+      tmem_st4(acc + kH + h0 + 4, p_n + 4);
+      tmem_st4(acc + kH + h0 + 8, p_hn);
+      tmem_st4(acc + kH + h0 + 12, p_hn + 4);
       tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(&bars.ops_ready[a]);
+      warp_arrive(&bars.ops_ready[a]);
       if (!mbar_wait(&bars.ph2_full[a], (i >> 1) & 1, status, 626, abort, 64)) break;
       tc_fence_after();
-      uint32_t vx[32], vd[32];
-      tmem_ld32(acc + 2 * kH + h0, vx);
-      tmem_ld32(acc + 3 * kH + h0, vd);
+      uint32_t vx[16], vd[16];
+      tmem_ld16(acc + 2 * kH + h0, vx);
+      tmem_ld16(acc + 3 * kH + h0, vd);
       tmem_wait_ld();
       tc_fence_before();
-      mbar_arrive(&bars.acc_empty[a]);
-      uint32_t px[16];
+      warp_arrive(&bars.acc_empty[a]);
+      uint32_t px[8];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) px[j] = pk2(__uint_as_float(vx[2 * j]), __uint_as_float(vx[2 * j + 1]));
-      store_T16(dXT, ld_x, row, h0, px);
+      for (int j = 0; j < 8; ++j) px[j] = pk2(__uint_as_float(vx[2 * j]), __uint_as_float(vx[2 * j + 1]));
+      store_T8(dXT, ld_x, row, h0, px);
       float4* go = reinterpret_cast<float4*>(gout + (size_t)row * kH + h0);
 #pragma unroll
-      for (int q = 0; q < 8; ++q)
+      for (int q = 0; q < 4; ++q)
         go[q] = make_float4(dhd[4 * q] + __uint_as_float(vd[4 * q]),
                             dhd[4 * q + 1] + __uint_as_float(vd[4 * q + 1]),
                             dhd[4 * q + 2] + __uint_as_float(vd[4 * q + 2]),
