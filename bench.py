@@ -158,10 +158,20 @@ def reduce_over_ranks(dist, ms: float, units: float, device="cuda"):
     return float(t.item()), float(u.item())
 
 
+def allreduce_grads(dist, flat):
+    """Data-parallel gradient exchange, the one collective of a step with N > 1: every rank's
+    gradients (one flat buffer) replaced in place by their mean over the ranks, as in the paper's
+    synchronous data-parallel training (one supergraph per core, Section 4.2)."""
+    if dist is None or dist.get_world_size() == 1:
+        return
+    dist.all_reduce(flat, op=dist.ReduceOp.SUM)
+    flat.mul_(1.0 / dist.get_world_size())
+
+
 class OursStep:
     """Device buffers and one fwd+bwd step through the C ABI."""
 
-    def __init__(self, config, graphs, c, seed=0):
+    def __init__(self, config, graphs, c, seed=0, dist=None):
         import torch
 
         from paper_1906_11786_gb300 import _binding as L
@@ -198,9 +208,18 @@ class OursStep:
         dET[n_real:] = 0
         self.dET = torch.from_numpy(dET).cuda()
         self.dET_host = torch.from_numpy(dET).pin_memory()
-        self.grads = {k: torch.empty(s, device="cuda") for k, s in
-                      (("dW", (P, H, H)), ("db", (P, H)), ("dW_ih", (3 * H, H)),
-                       ("dW_hh", (3 * H, H)), ("db_ih", (3 * H,)), ("db_hh", (3 * H,)))}
+        # every gradient is a view of one flat buffer: one all-reduce per step for N > 1
+        shapes = (("dW", (P, H, H)), ("db", (P, H)), ("dW_ih", (3 * H, H)), ("dW_hh", (3 * H, H)),
+                  ("db_ih", (3 * H,)), ("db_hh", (3 * H,)), ("dw_out", (H,)))
+        self.gflat = torch.zeros(sum(int(np.prod(sh)) for _, sh in shapes), device="cuda")
+        views, o = {}, 0
+        for k, sh in shapes:
+            n = int(np.prod(sh))
+            views[k] = self.gflat[o:o + n].view(sh)
+            o += n
+        self.dw_out = views.pop("dw_out")
+        self.grads = views
+        self.dist = dist
         self.grads_host = {k: torch.empty(v.shape, pin_memory=True) for k, v in self.grads.items()}
         self.dE0 = torch.empty((N, H), device="cuda")
         self.dE0_orig = torch.zeros((n_all, H), device="cuda")
@@ -225,7 +244,6 @@ class OursStep:
             self.target = torch.from_numpy(
                 np.random.default_rng(seed + 3).standard_normal(n_g).astype(np.float32)).cuda()
             self.loss = torch.zeros(4, device="cuda")
-            self.dw_out = torch.empty(H, device="cuda")
             self.ws_r = torch.empty(L.workspace_bytes(self.plan, self.dt, H, L.BG_OP_READOUT),
                                     dtype=torch.uint8, device="cuda")
             names = ["W", "b", "W_ih", "W_hh", "b_ih", "b_hh", "w_out"]
@@ -245,6 +263,7 @@ class OursStep:
                                  self.ws_f)
             L.band_propagate_bwd(self.plan, self.dt, H, E0, self.prm["W"], dET, self.dE0,
                                  self.grads["dW"], self.grads["db"], self.ws_b)
+            allreduce_grads(self.dist, self.gflat)
             return
         L.ggnn_step(self.plan, self.dt, H, T, self.prm, E0, self.ET, self.saved, self.ws_f)
         if self.train:
@@ -253,6 +272,7 @@ class OursStep:
             dET = self.dET
         L.ggnn_step_bwd(self.plan, self.dt, H, T, self.prm, self.saved, dET, self.dE0, self.grads,
                         self.ws_b)
+        allreduce_grads(self.dist, self.gflat)
         if self.train:
             self.adam_t += 1
             gmap = dict(self.grads, w_out=self.dw_out)
@@ -415,7 +435,7 @@ def main():
     from paper_1906_11786_gb300 import synth
 
     graphs, c = workload(args.config, rank, args.S, args.H)
-    st = OursStep(args.config, graphs, c, seed=rank)
+    st = OursStep(args.config, graphs, c, seed=rank, dist=dist)
     H, T = c["H"], c["T"]
     units = st.n_real * T  # node-steps per step on this rank
     if args.op != "step":
@@ -508,7 +528,8 @@ def main():
                    "band_kernels": "tcgen05" if L.band_uses_tensor_cores(st.plan, c["dtype"], H)
                    else "simt",
                    "l2": "per-step working set (band tiles + saved activations) > 129 MB L2",
-                   "parallelism": f"dp{world} (one supergraph per GPU)"},
+                   "parallelism": f"dp{world} (one supergraph per GPU"
+                                  + (", gradient all-reduce)" if world > 1 else ")")},
         "e2e": {"value": e2e_value, "unit": "node-steps/s", "h2d_bytes_per_step": bi,
                 "d2h_bytes_per_step": bo},
         "gpu_launches": launches,

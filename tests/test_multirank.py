@@ -1,6 +1,7 @@
 """Multi-GPU logic of the benchmark on CPU ranks (gloo, world size 2): every rank plans its own
-supergraph of the same shape (the paper gives each core its own supergraph), and the whole-job
-figures are the slowest rank's time and the sum of all ranks' node-steps.  No GPU is used."""
+supergraph of the same shape (the paper gives each core its own supergraph), the whole-job
+figures are the slowest rank's time and the sum of all ranks' node-steps, and the data-parallel
+gradient exchange leaves every rank with the mean of all ranks' gradients.  No GPU is used."""
 import os
 import socket
 
@@ -61,3 +62,40 @@ def test_two_cpu_ranks_plan_own_supergraphs_and_aggregate():
         assert same_shape and different_graphs
         assert ms_max == 10.0 + world - 1
         assert units_sum == units_expected
+
+
+def _grad_worker(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    import bench
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        # rank r's gradients are r + 1 + 0.5 k on element k; the mean over ranks is known exactly
+        flat = torch.arange(12, dtype=torch.float32) * 0.5 + (rank + 1)
+        view = flat[4:10].view(2, 3)  # gradients live as views of the flat buffer
+        bench.allreduce_grads(dist, flat)
+        out[rank] = (flat.tolist(), view.tolist())
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.timeout(300)
+def test_data_parallel_gradient_mean_over_cpu_ranks():
+    world = 2
+    port = _free_port()
+    mgr = mp.get_context("spawn").Manager()
+    out = mgr.dict()
+    mp.start_processes(_grad_worker, args=(world, port, out), nprocs=world, start_method="spawn")
+    mean_offset = sum(r + 1 for r in range(world)) / world
+    expect = [0.5 * k + mean_offset for k in range(12)]
+    for r in range(world):
+        flat, view = out[r]
+        assert flat == pytest.approx(expect, abs=0)
+        assert view == [expect[4:7], expect[7:10]]
+
+
+def test_single_process_gradients_untouched():
+    import bench
+    flat = torch.arange(5, dtype=torch.float32)
+    bench.allreduce_grads(None, flat)
+    assert flat.tolist() == [0.0, 1.0, 2.0, 3.0, 4.0]
