@@ -35,6 +35,9 @@ cudaError_t gemm_bf16_tn(const void* A, int64_t lda, int64_t sA, const void* B, 
 
 // 2-D bf16 tensor map over row-major [rows][cols] with row stride ld elements; box {64, box_rows};
 // 128-byte swizzle; reads outside the array return zero.
+// Row-major fp32 [rows][cols] with the 128-byte swizzle, boxes of 32 columns x box_rows.
+bool make_map_f32(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols,
+                  uint32_t box_rows);
 bool make_map_ld(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
                  uint32_t box_rows);
 int gemm_tn_num_sms();

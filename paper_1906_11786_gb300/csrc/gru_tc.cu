@@ -92,6 +92,15 @@ __device__ __forceinline__ void read_sw128_row8(const uint8_t* tile, int r, int 
   }
 }
 
+// 8 consecutive fp32 of row r (columns c0 .. c0+7, c0 % 8 == 0) of a 128-row tile stored as
+// 32-column boxes (128-byte rows) with the 128-byte swizzle.
+__device__ __forceinline__ void read_sw128_f32_row8(const uint8_t* tile, int r, int c0, float4* out) {
+  const uint8_t* row = tile + (c0 / 32) * 128 * 128 + r * 128;
+  const int j0 = (c0 % 32) / 4;
+  out[0] = *reinterpret_cast<const float4*>(row + (((j0) ^ (r & 7)) << 4));
+  out[1] = *reinterpret_cast<const float4*>(row + (((j0 + 1) ^ (r & 7)) << 4));
+}
+
 // 4 bf16 pairs stored transposed: dst[(h0 + 2j + u) * ld + row]
 __device__ __forceinline__ void store_T4(__nv_bfloat16* dst, int64_t ld, int row, int h0,
                                          const uint32_t* pk) {
@@ -116,11 +125,17 @@ __device__ __forceinline__ void store_T8(__nv_bfloat16* dst, int64_t ld, int row
 
 struct GruSmem {
   static constexpr int TILE = 128 * 128;  // 128 rows x 64 bf16
+  static constexpr int G = 128 * kH * 4;  // 128 rows x 64 fp32 (incoming state gradient, backward)
   static constexpr int W = 3 * kH * 128;  // [3H][H] bf16 (also [H][3H] as three 64-column atoms)
   static constexpr int FWD_T = 2 * W;     // tile ring after W_ih, W_hh
   static constexpr int BWD_T = 4 * W;     // tile ring after W_ih, W_hh, W_ih^T, W_hh^T
-  static constexpr int FWD = FWD_T + 4 * TILE + 2048;
-  static constexpr int BWD = BWD_T + 4 * TILE + 2048;
+  static constexpr int FWD_STAGE = 2 * TILE;      // Y, E
+  static constexpr int BWD_STAGE = 2 * TILE + G;  // Y, E, g
+  // dynamic shared memory: the ring plus 1 KB of slack for aligning its base to 1024 bytes; the
+  // barriers and biases are static (< 2 KB) and count toward the same 227 KB per block
+  static constexpr int FWD = FWD_T + 2 * FWD_STAGE + 1024;
+  static constexpr int BWD = BWD_T + 2 * BWD_STAGE + 1024;
+  static_assert(BWD + 2048 <= 232448, "shared memory");
 };
 
 struct GruBars {
@@ -174,19 +189,26 @@ __device__ __forceinline__ void gru_setup(GruBars* b, float* bias, const float* 
   tc_fence_after();
 }
 
-// Tile producer shared by both kernels: two-stage ring of (Y, E) tiles.
-__device__ __forceinline__ void gru_produce_tiles(GruBars* b, uint8_t* ring,
+// Tile producer shared by both kernels: two-stage ring of (Y, E) tiles and, backward, the fp32
+// incoming gradient tile (two 32-column boxes with the 128-byte swizzle).
+__device__ __forceinline__ void gru_produce_tiles(GruBars* b, uint8_t* ring, int stage,
                                                   const CUtensorMap* tY, const CUtensorMap* tE,
-                                                  int n_tiles, int* status, volatile int* abort) {
+                                                  const CUtensorMap* tG, int n_tiles, int* status,
+                                                  volatile int* abort) {
   uint32_t issued[2] = {0, 0};
   int i = 0;
   for (int t = blockIdx.x; t < n_tiles && !*abort; t += gridDim.x, ++i) {
     const int s = i & 1;
     if (!mbar_wait(&b->t_empty[s], ((i >> 1) & 1) ^ 1, status, 611, abort, 64)) break;
     ++issued[s];
-    mbar_expect_tx(&b->t_full[s], 2 * GruSmem::TILE);
-    tma_load_2d(ring + s * 2 * GruSmem::TILE, tY, &b->t_full[s], 0, t * 128);
-    tma_load_2d(ring + s * 2 * GruSmem::TILE + GruSmem::TILE, tE, &b->t_full[s], 0, t * 128);
+    uint8_t* st = ring + s * stage;
+    mbar_expect_tx(&b->t_full[s], 2 * GruSmem::TILE + (tG ? GruSmem::G : 0));
+    tma_load_2d(st, tY, &b->t_full[s], 0, t * 128);
+    tma_load_2d(st + GruSmem::TILE, tE, &b->t_full[s], 0, t * 128);
+    if (tG) {
+      tma_load_2d(st + 2 * GruSmem::TILE, tG, &b->t_full[s], 0, t * 128);
+      tma_load_2d(st + 2 * GruSmem::TILE + GruSmem::G / 2, tG, &b->t_full[s], 32, t * 128);
+    }
   }
   if (*abort)
     for (int s = 0; s < 2; ++s)
@@ -215,7 +237,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_expect_tx(&bars.w_full, 2 * GruSmem::W);
     tma_load_2d(smem, &tWih, &bars.w_full, 0, 0);
     tma_load_2d(smem + GruSmem::W, &tWhh, &bars.w_full, 0, 0);
-    gru_produce_tiles(&bars, ring, &tY, &tE, n_tiles, status, abort);
+    gru_produce_tiles(&bars, ring, GruSmem::FWD_STAGE, &tY, &tE, nullptr, n_tiles, status, abort);
     if (*abort)
       for (uint32_t k = 0; k < (1u << 22) && !mbar_try(&bars.w_full, 0); ++k) {
       }
@@ -316,8 +338,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     k_gru_bwd_tc(const __grid_constant__ CUtensorMap tY, const __grid_constant__ CUtensorMap tE,
                  const __grid_constant__ CUtensorMap tWih, const __grid_constant__ CUtensorMap tWhh,
                  const __grid_constant__ CUtensorMap tWihT, const __grid_constant__ CUtensorMap tWhhT,
+                 const __grid_constant__ CUtensorMap tG,
                  const float* __restrict__ b_ih, const float* __restrict__ b_hh,
-                 const float* __restrict__ gin, float* __restrict__ gout,
+                 float* __restrict__ gout,
                  __nv_bfloat16* __restrict__ dXT, int64_t ld_x, __nv_bfloat16* __restrict__ dgiT,
                  __nv_bfloat16* __restrict__ dghT, int64_t ld_g, int n_tiles, int n_real,
                  int* status) {
@@ -340,7 +363,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_load_2d(smem + 2 * GruSmem::W + a * kH * 128, &tWihT, &bars.w_full, a * 64, 0);
       tma_load_2d(smem + 3 * GruSmem::W + a * kH * 128, &tWhhT, &bars.w_full, a * 64, 0);
     }
-    gru_produce_tiles(&bars, ring, &tY, &tE, n_tiles, status, abort);
+    gru_produce_tiles(&bars, ring, GruSmem::BWD_STAGE, &tY, &tE, &tG, n_tiles, status, abort);
     if (*abort)
       for (uint32_t k = 0; k < (1u << 22) && !mbar_try(&bars.w_full, 0); ++k) {
       }
@@ -374,7 +397,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(&bars.t_full[s], (i >> 1) & 1, status, 623, abort)) break;
         if (!mbar_wait(&bars.acc_empty[a], ((i >> 1) & 1) ^ 1, status, 624, abort)) break;
         tc_fence_after();
-        const uint32_t sY = smem_u32(ring + s * 2 * GruSmem::TILE);
+        const uint32_t sY = smem_u32(ring + s * GruSmem::BWD_STAGE);
         if (leader) {
           gru_gate_mmas(tmem + a * kAcc, sY, sY + GruSmem::TILE, smem_u32(smem),
                         smem_u32(smem + GruSmem::W));
@@ -401,7 +424,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!mbar_wait(&bars.acc_full[a], (i >> 1) & 1, status, 625, abort, 64)) break;
       tc_fence_after();
       const uint32_t acc = tmem + lb + a * kAcc;
-      const uint8_t* etile = ring + s * 2 * GruSmem::TILE + GruSmem::TILE;
+      const uint8_t* etile = ring + s * GruSmem::BWD_STAGE + GruSmem::TILE;
+      const uint8_t* gtile = etile + GruSmem::TILE;
       float dhd[16];
       // packed gate gradients of both halves: the in-place rewrite below overwrites columns that
       // the second half still reads, so it waits until both halves are in registers
@@ -418,8 +442,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_wait_ld();
         float e[8];
         read_sw128_row8(etile, r, hs, e);
+        float4 g4[2];
+        read_sw128_f32_row8(gtile, r, hs, g4);
         if (hh == 1) warp_arrive(&bars.t_empty[s]);
-        const float4* g4 = reinterpret_cast<const float4*>(gin + (size_t)row * kH + hs);
         const int o = 4 * hh;
 #pragma unroll
         for (int q = 0; q < 2; ++q) {
@@ -527,19 +552,20 @@ cudaError_t gru_bwd_tc(int n_pad, int n_real, const __nv_bfloat16* Y, const __nv
                        const float* b_hh, const float* gin, float* gout, __nv_bfloat16* dXT,
                        int64_t ld_x, __nv_bfloat16* dgiT, __nv_bfloat16* dghT, int64_t ld_g,
                        int* status, cudaStream_t st) {
-  CUtensorMap tY, tE, tWi, tWh, tWiT, tWhT;
+  CUtensorMap tY, tE, tWi, tWh, tWiT, tWhT, tG;
   if (!make_map_ld(&tY, Y, n_pad, kH, kH, 128) || !make_map_ld(&tE, E, n_pad, kH, kH, 128) ||
       !make_map_ld(&tWi, W_ih, 3 * kH, kH, kH, 3 * kH) ||
       !make_map_ld(&tWh, W_hh, 3 * kH, kH, kH, 3 * kH) ||
       !make_map_ld(&tWiT, W_ihT, kH, 3 * kH, 3 * kH, kH) ||
-      !make_map_ld(&tWhT, W_hhT, kH, 3 * kH, 3 * kH, kH))
+      !make_map_ld(&tWhT, W_hhT, kH, 3 * kH, 3 * kH, kH) ||
+      !make_map_f32(&tG, gin, n_pad, kH, 128))
     return cudaErrorInvalidValue;
   cudaError_t e = cudaFuncSetAttribute(k_gru_bwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        GruSmem::BWD);
   if (e != cudaSuccess) return e;
   const int n_tiles = n_pad / 128;
   const int grid = std::min(n_tiles, gemm_tn_num_sms());
-  k_gru_bwd_tc<<<grid, kThreads, GruSmem::BWD, st>>>(tY, tE, tWi, tWh, tWiT, tWhT, b_ih, b_hh, gin,
+  k_gru_bwd_tc<<<grid, kThreads, GruSmem::BWD, st>>>(tY, tE, tWi, tWh, tWiT, tWhT, tG, b_ih, b_hh,
                                                      gout, dXT, ld_x, dgiT, dghT, ld_g, n_tiles,
                                                      n_real, status);
   note_launch();
