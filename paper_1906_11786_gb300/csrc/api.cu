@@ -459,8 +459,9 @@ struct TcBwdWs {
 };
 size_t tc_part_floats(const bg_plan* p, int H, int T) {
   const int64_t K = (int64_t)T * p->n_pad();
-  return std::max(bg::gemm_tn_part_floats(p->P * H, H + 16, K),
-                  bg::gemm_tn_part_floats(3 * H, H + 16, K));
+  return std::max({bg::gemm_tn_part_floats(p->P * H, H + 16, K),
+                   bg::gemm_tn_part_floats(3 * H, H + 16, K),
+                   bg::gemm_tn_part_floats(p->P * H + 6 * H, H + 16, K)});
 }
 TcBwdWs tc_bwd_ws(const bg_plan* p, int H, int T) {
   const size_t n = (size_t)p->n_pad(), TN = (size_t)T * n;
@@ -847,12 +848,11 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     const int acc = (flags & BG_ACCUM) ? 1 : 0;
     KTimer tm(BG_KID_DW, st);
     // dW_p, db_p over all steps and nodes; dW_ih, db_ih; dW_hh, db_hh
-    BG_CUDA(bg::gemm_tn(dMT, (int64_t)TN, ETa, (int64_t)TN, p->P * H, H, (int64_t)TN, 1, gr->dW,
-                        gr->db, acc, part, pf, status, st));
-    BG_CUDA(bg::gemm_tn(dgiT, (int64_t)TN, YTa, (int64_t)TN, 3 * H, H, (int64_t)TN, 0, gr->dW_ih,
-                        gr->db_ih, acc, part, pf, status, st));
-    BG_CUDA(bg::gemm_tn(dghT, (int64_t)TN, ETa, (int64_t)TN, 3 * H, H, (int64_t)TN, 0, gr->dW_hh,
-                        gr->db_hh, acc, part, pf, status, st));
+    const bg::TNProblem probs[3] = {
+        {dMT, (int64_t)TN, ETa, (int64_t)TN, p->P * H, 1, gr->dW, gr->db},
+        {dgiT, (int64_t)TN, YTa, (int64_t)TN, 3 * H, 0, gr->dW_ih, gr->db_ih},
+        {dghT, (int64_t)TN, ETa, (int64_t)TN, 3 * H, 0, gr->dW_hh, gr->db_hh}};
+    BG_CUDA(bg::gemm_tn_multi(probs, 3, H, (int64_t)TN, acc, part, pf, status, st));
     BG_CUDA(cudaMemcpyAsync(dE0, g, sizeof(float) * n * H, cudaMemcpyDeviceToDevice, st));
     return BG_OK;
   }

@@ -43,10 +43,20 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
       : "r"(taddr));
 }
 
+// Up to kMaxGroups problems with the same K and N in one launch: blockIdx.x runs over the M tiles
+// of all groups; group g's rows sit at rows prow[g] .. prow[g] + M[g] of the partial sums.
+constexpr int kMaxGroups = 3;
+struct TNGroups {
+  CUtensorMap a[kMaxGroups], b[kMaxGroups];
+  int mt_end[kMaxGroups];  // cumulative M-tile counts
+  int M[kMaxGroups];
+  int prow[kMaxGroups];
+};
+
 template <int BN>
 __global__ void __launch_bounds__(192, 1)
-    k_gemm_tn(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-              float* __restrict__ part, int M, int N, int kchunks, int per_split, int* status) {
+    k_gemm_tn(const __grid_constant__ TNGroups grp, float* __restrict__ part, int Mtot, int N,
+              int kchunks, int per_split, int* status) {
   using C = GCfg<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -59,7 +69,12 @@ __global__ void __launch_bounds__(192, 1)
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
   volatile int* abort = abort_flag;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int mt = blockIdx.x, split = blockIdx.z;
+  int g = 0;
+  while (g + 1 < kMaxGroups && (int)blockIdx.x >= grp.mt_end[g]) ++g;
+  const int mt = blockIdx.x - (g ? grp.mt_end[g - 1] : 0), split = blockIdx.z;
+  const int M = grp.M[g];
+  const CUtensorMap* tmA = &grp.a[g];
+  const CUtensorMap* tmB = &grp.b[g];
   const int kc0 = split * per_split;
   const int kc1 = min(kchunks, kc0 + per_split);
   if (threadIdx.x == 0) {
@@ -79,8 +94,8 @@ __global__ void __launch_bounds__(192, 1)
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&tmA);
-    tma_prefetch_desc(&tmB);
+    tma_prefetch_desc(tmA);
+    tma_prefetch_desc(tmB);
     uint32_t issued[kStages] = {0, 0, 0, 0};
     for (int kc = kc0, it = 0; kc < kc1; ++kc, ++it) {
       const int s = it % kStages;
@@ -88,8 +103,8 @@ __global__ void __launch_bounds__(192, 1)
       ++issued[s];
       mbar_expect_tx(&full[s], C::STAGE);
       uint8_t* st = smem + s * C::STAGE;
-      tma_load_2d(st, &tmA, &full[s], kc * 64, mt * 128);
-      tma_load_2d(st + C::A_BYTES, &tmB, &full[s], kc * 64, blockIdx.y * BN);
+      tma_load_2d(st, tmA, &full[s], kc * 64, mt * 128);
+      tma_load_2d(st + C::A_BYTES, tmB, &full[s], kc * 64, blockIdx.y * BN);
     }
     if (*abort)
       for (int s = 0; s < kStages; ++s)
@@ -124,7 +139,7 @@ __global__ void __launch_bounds__(192, 1)
     const int m = mt * 128 + q * 32 + lane;
     if (mbar_wait(done, 0, status, 503, abort, 256)) {
       tc_fence_after();
-      float* out = part + ((size_t)split * M + m) * N + blockIdx.y * BN;
+      float* out = part + ((size_t)split * Mtot + grp.prow[g] + m) * N + blockIdx.y * BN;
 #pragma unroll
       for (int c0 = 0; c0 < BN; c0 += 16) {
         uint32_t v[16];
@@ -147,17 +162,30 @@ __global__ void __launch_bounds__(192, 1)
   }
 }
 
+// Per group (rows prow .. prow + M of the partial sums):
 // mode 0: out[m][n] (+)= sum_s part[s][m][n] for n < Hout; bias[m] (+)= sum_s part[s][m][Hout]
 // mode 1: m = p*Hout + o: out[p][n][o] (+)= sum_s part[s][m][n]; bias[m] (+)= sum_s part[s][m][Hout]
-__global__ void k_gemm_tn_reduce(const float* __restrict__ part, int splits, int M, int N, int Hout,
-                                 int mode, float* __restrict__ out, float* __restrict__ bias,
-                                 int accumulate) {
-  const int64_t total = (int64_t)M * (Hout + 1);
-  const size_t stride = (size_t)M * N;
+struct TNOut {
+  float* out[kMaxGroups];
+  float* bias[kMaxGroups];
+  int mode[kMaxGroups];
+  int M[kMaxGroups];
+  int prow[kMaxGroups];
+  int n_groups;
+};
+
+__global__ void k_gemm_tn_reduce(const float* __restrict__ part, int splits, int Mtot, int N,
+                                 int Hout, TNOut o, int accumulate) {
+  const int64_t total = (int64_t)Mtot * (Hout + 1);
+  const size_t stride = (size_t)Mtot * N;
   for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total;
        t += (int64_t)gridDim.x * blockDim.x) {
-    const int m = (int)(t / (Hout + 1)), n = (int)(t % (Hout + 1));
-    const float* src = part + (size_t)m * N + n;
+    const int mm = (int)(t / (Hout + 1)), n = (int)(t % (Hout + 1));
+    int g = 0;
+    while (g + 1 < o.n_groups && mm >= o.prow[g + 1]) ++g;
+    const int m = mm - o.prow[g];
+    if (m >= o.M[g]) continue;
+    const float* src = part + (size_t)mm * N + n;
     // four independent partial sums keep several loads in flight; fixed order, so deterministic
     float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
     int q = 0;
@@ -171,13 +199,13 @@ __global__ void k_gemm_tn_reduce(const float* __restrict__ part, int splits, int
     const float s = (s0 + s1) + (s2 + s3);
     float* dst;
     if (n == Hout) {
-      if (!bias) continue;
-      dst = bias + m;
-    } else if (mode == 0) {
-      dst = out + (size_t)m * Hout + n;
+      if (!o.bias[g]) continue;
+      dst = o.bias[g] + m;
+    } else if (o.mode[g] == 0) {
+      dst = o.out[g] + (size_t)m * Hout + n;
     } else {
-      const int p = m / Hout, o = m % Hout;
-      dst = out + ((size_t)p * Hout + n) * Hout + o;
+      const int p = m / Hout, oo = m % Hout;
+      dst = o.out[g] + ((size_t)p * Hout + n) * Hout + oo;
     }
     *dst = accumulate ? *dst + s : s;
   }
@@ -381,30 +409,44 @@ size_t gemm_tn_part_floats(int M, int N, int64_t K) {
   return (size_t)splits * M * N;
 }
 
-cudaError_t gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int Hout,
-                    int64_t K, int mode, float* out, float* bias, int accumulate, float* part,
-                    size_t part_floats, int* status, cudaStream_t st) {
+cudaError_t gemm_tn_multi(const TNProblem* pr, int n, int Hout, int64_t K, int accumulate,
+                          float* part, size_t part_floats, int* status, cudaStream_t st) {
   const int N = Hout + 16;  // Hout gradient columns, one ones-column (bias), padding to 16
   if (N != 48 && N != 80 && N != 144) return cudaErrorInvalidValue;
+  if (n < 1 || n > kMaxGroups) return cudaErrorInvalidValue;
   const int64_t kchunks = (K + 63) / 64;
-  const int mt = (M + 127) / 128;
+  TNGroups grp{};
+  TNOut o{};
+  int mt = 0, Mtot = 0;
+  for (int g = 0; g < n; ++g) {
+    if (!make_map_ld(&grp.a[g], pr[g].A, pr[g].M, K, pr[g].lda, 128) ||
+        !make_map_ld(&grp.b[g], pr[g].B, N, K, pr[g].ldb, N))
+      return cudaErrorInvalidValue;
+    mt += (pr[g].M + 127) / 128;
+    grp.mt_end[g] = mt;
+    grp.M[g] = o.M[g] = pr[g].M;
+    grp.prow[g] = o.prow[g] = Mtot;
+    o.out[g] = pr[g].out;
+    o.bias[g] = pr[g].bias;
+    o.mode[g] = pr[g].mode;
+    Mtot += pr[g].M;
+  }
+  for (int g = n; g < kMaxGroups; ++g) grp.mt_end[g] = mt;
+  o.n_groups = n;
   const int sms = gemm_tn_num_sms();
   // two CTAs fit per SM: at most 2 * sms CTAs, so that all of them run in one wave (a partial
   // second wave of even a few CTAs would nearly double the time of this HBM-bound pass)
   int splits = (int)std::max<int64_t>(1, std::min<int64_t>(kchunks, std::max(1, 2 * sms / mt)));
-  while (splits > 1 && (size_t)splits * M * N > part_floats) --splits;
+  while (splits > 1 && (size_t)splits * Mtot * N > part_floats) --splits;
   const int per = (int)((kchunks + splits - 1) / splits);
   splits = (int)((kchunks + per - 1) / per);
-  CUtensorMap ta, tb;
-  if (!make_map_ld(&ta, A, M, K, lda, 128) || !make_map_ld(&tb, B, N, K, ldb, N))
-    return cudaErrorInvalidValue;
   dim3 grid(mt, 1, splits);
   cudaError_t e;
 #define BG_GEMM_CASE(BNV)                                                                      \
   e = cudaFuncSetAttribute(k_gemm_tn<BNV>, cudaFuncAttributeMaxDynamicSharedMemorySize,        \
                            GCfg<BNV>::SMEM);                                                   \
   if (e != cudaSuccess) return e;                                                              \
-  k_gemm_tn<BNV><<<grid, 192, GCfg<BNV>::SMEM, st>>>(ta, tb, part, M, N, (int)kchunks, per, status);
+  k_gemm_tn<BNV><<<grid, 192, GCfg<BNV>::SMEM, st>>>(grp, part, Mtot, N, (int)kchunks, per, status);
   if (N == 48) {
     BG_GEMM_CASE(48)
   } else if (N == 80) {
@@ -414,11 +456,18 @@ cudaError_t gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int 
   }
 #undef BG_GEMM_CASE
   note_launch();
-  const int64_t total = (int64_t)M * (Hout + 1);
+  const int64_t total = (int64_t)Mtot * (Hout + 1);
   k_gemm_tn_reduce<<<(unsigned)std::min<int64_t>((total + 255) / 256, 4096), 256, 0, st>>>(
-      part, splits, M, N, Hout, mode, out, bias, accumulate);
+      part, splits, Mtot, N, Hout, o, accumulate);
   note_launch();
   return cudaGetLastError();
+}
+
+cudaError_t gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int Hout,
+                    int64_t K, int mode, float* out, float* bias, int accumulate, float* part,
+                    size_t part_floats, int* status, cudaStream_t st) {
+  const TNProblem pr{A, lda, B, ldb, M, mode, out, bias};
+  return gemm_tn_multi(&pr, 1, Hout, K, accumulate, part, part_floats, status, st);
 }
 
 }  // namespace bg

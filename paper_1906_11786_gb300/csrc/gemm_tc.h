@@ -23,6 +23,21 @@ cudaError_t gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int 
                     int64_t K, int mode, float* out, float* bias, int accumulate, float* part,
                     size_t part_floats, int* status, cudaStream_t st);
 
+// Up to three such problems with the same K and Hout in one launch (one wave over all their M
+// tiles, one reduction); part_floats must cover gemm_tn_part_floats(sum of M, Hout + 16, K).
+struct TNProblem {
+  const void* A;
+  int64_t lda;
+  const void* B;
+  int64_t ldb;
+  int M;
+  int mode;
+  float* out;
+  float* bias;
+};
+cudaError_t gemm_tn_multi(const TNProblem* problems, int n, int Hout, int64_t K, int accumulate,
+                          float* part, size_t part_floats, int* status, cudaStream_t st);
+
 // Batched TN GEMM on tcgen05 (fp32 accumulation):
 //   C[b][m][n] (+)= sum_k A[b][m][k] B[b][n][k] (+ bias[b*sBias + n])
 // A: [M][K] bf16, row stride lda, batch stride sA (0 = shared by all batches); B: [N][K] bf16, row
