@@ -197,6 +197,8 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // TMEM is held: the next kernel in the stream may be scheduled on SMs as they free up
+  grid_dep_launch();
   const uint32_t tmem = bars->tmem_base;
   const int n_tiles = K;  // S = 128: one tile per block-row
 
@@ -209,6 +211,8 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
       mbar_expect_tx(&bars->b2_full, C::B2);
       tma_load_2d(b2s, &tm_b2, &bars->b2_full, 0, 0);
     }
+    // the state windows are the previous kernel's output (bit tiles, W, deg and b2 are not)
+    grid_dep_wait();
     uint32_t widx = 0;
     uint32_t n_x[2] = {0, 0}, n_deg[2] = {0, 0}, n_w[4] = {0, 0, 0, 0};
     int i = 0;
@@ -505,6 +509,7 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
     }
   } else if (warp >= 4 + 4 * C::NE) {
     // ------------------------------------------------------------------ converters / epilogue
+    grid_dep_wait();  // outputs (and the accumulated dE) may still be in use by the previous kernel
     const int r = threadIdx.x - 128 * (1 + C::NE);
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     uint32_t c = 0;
@@ -722,11 +727,11 @@ cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& t
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
   const int grid = std::min(p->K, num_sms());
-  k_band_tc<H, BWD><<<grid, C::THREADS, C::SMEM, st>>>(
-      tx, tw, tdeg, tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt,
-      p->K, p->P, has_bias, accumulate, status);
+  e = launch_pdl(k_band_tc<H, BWD>, dim3(grid), dim3(C::THREADS), C::SMEM, st, tx, tw, tdeg, tb2,
+                 BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt, p->K, p->P,
+                 has_bias, accumulate, status);
   note_launch();
-  return cudaGetLastError();
+  return e;
 }
 
 }  // namespace

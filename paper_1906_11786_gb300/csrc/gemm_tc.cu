@@ -91,11 +91,13 @@ __global__ void __launch_bounds__(192, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  grid_dep_launch();  // TMEM is held: the reduction may be scheduled as SMs free up
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(tmA);
     tma_prefetch_desc(tmB);
+    grid_dep_wait();  // A and B are the previous kernels' output
     uint32_t issued[kStages] = {0, 0, 0, 0};
     for (int kc = kc0, it = 0; kc < kc1; ++kc, ++it) {
       const int s = it % kStages;
@@ -135,6 +137,7 @@ __global__ void __launch_bounds__(192, 1)
     for (uint32_t t = 0; t < (1u << 24) && !mbar_try(drain, 0); ++t) {
     }
   } else if (warp >= 2) {
+    grid_dep_wait();  // the partial sums may still be read by the previous reduction
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int m = mt * 128 + q * 32 + lane;
     if (mbar_wait(done, 0, status, 503, abort, 256)) {
@@ -176,6 +179,7 @@ struct TNOut {
 
 __global__ void k_gemm_tn_reduce(const float* __restrict__ part, int splits, int Mtot, int N,
                                  int Hout, TNOut o, int accumulate) {
+  grid_dep_wait();
   const int64_t total = (int64_t)Mtot * (Hout + 1);
   const size_t stride = (size_t)Mtot * N;
   for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total;
@@ -446,7 +450,9 @@ cudaError_t gemm_tn_multi(const TNProblem* pr, int n, int Hout, int64_t K, int a
   e = cudaFuncSetAttribute(k_gemm_tn<BNV>, cudaFuncAttributeMaxDynamicSharedMemorySize,        \
                            GCfg<BNV>::SMEM);                                                   \
   if (e != cudaSuccess) return e;                                                              \
-  k_gemm_tn<BNV><<<grid, 192, GCfg<BNV>::SMEM, st>>>(grp, part, Mtot, N, (int)kchunks, per, status);
+  e = launch_pdl(k_gemm_tn<BNV>, grid, dim3(192), GCfg<BNV>::SMEM, st, grp, part, Mtot, N,        \
+                 (int)kchunks, per, status);                                                   \
+  if (e != cudaSuccess) return e;
   if (N == 48) {
     BG_GEMM_CASE(48)
   } else if (N == 80) {
@@ -457,10 +463,10 @@ cudaError_t gemm_tn_multi(const TNProblem* pr, int n, int Hout, int64_t K, int a
 #undef BG_GEMM_CASE
   note_launch();
   const int64_t total = (int64_t)Mtot * (Hout + 1);
-  k_gemm_tn_reduce<<<(unsigned)std::min<int64_t>((total + 255) / 256, 4096), 256, 0, st>>>(
-      part, splits, Mtot, N, Hout, o, accumulate);
+  e = launch_pdl(k_gemm_tn_reduce, dim3((unsigned)std::min<int64_t>((total + 255) / 256, 4096)),
+                 dim3(256), 0, st, (const float*)part, splits, Mtot, N, Hout, o, accumulate);
   note_launch();
-  return cudaGetLastError();
+  return e;
 }
 
 cudaError_t gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int Hout,

@@ -187,6 +187,8 @@ __device__ __forceinline__ void gru_setup(GruBars* b, float* bias, const float* 
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // TMEM is held: the next kernel in the stream may be scheduled on SMs as they free up
+  grid_dep_launch();
 }
 
 // Tile producer shared by both kernels: two-stage ring of (Y, E) tiles and, backward, the fp32
@@ -195,6 +197,8 @@ __device__ __forceinline__ void gru_produce_tiles(GruBars* b, uint8_t* ring, int
                                                   const CUtensorMap* tY, const CUtensorMap* tE,
                                                   const CUtensorMap* tG, int n_tiles, int* status,
                                                   volatile int* abort) {
+  // the tiles are the previous kernel's output (the weights, loaded before this, are not)
+  grid_dep_wait();
   uint32_t issued[2] = {0, 0};
   int i = 0;
   for (int t = blockIdx.x; t < n_tiles && !*abort; t += gridDim.x, ++i) {
@@ -264,6 +268,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (uint32_t k = 0; k < (1u << 24) && !mbar_try(&bars.drain, 0); ++k) {
     }
   } else if (warp >= 4) {
+    grid_dep_wait();  // outputs may still be in use by the previous kernel
     const int g = (warp - 4) / 4, h0 = 16 * g;
     const int r = (warp & 3) * 32 + lane;
     const uint32_t lb = (uint32_t)((warp & 3) * 32) << 16;
@@ -413,6 +418,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (uint32_t k = 0; k < (1u << 24) && !mbar_try(&bars.drain, 0); ++k) {
     }
   } else if (warp >= 4) {
+    grid_dep_wait();  // outputs may still be in use by the previous kernel
     const int g = (warp - 4) / 4, h0 = 16 * g;
     const int r = (warp & 3) * 32 + lane;
     const uint32_t lb = (uint32_t)((warp & 3) * 32) << 16;
@@ -540,10 +546,10 @@ cudaError_t gru_fwd_tc(int n_pad, int n_real, const __nv_bfloat16* Y, const __nv
   if (e != cudaSuccess) return e;
   const int n_tiles = n_pad / 128;
   const int grid = std::min(n_tiles, gemm_tn_num_sms());
-  k_gru_fwd_tc<<<grid, kThreads, GruSmem::FWD, st>>>(tY, tE, tWi, tWh, b_ih, b_hh, En, EnT, ld_T,
-                                                     n_tiles, n_real, status);
+  e = launch_pdl(k_gru_fwd_tc, dim3(grid), dim3(kThreads), GruSmem::FWD, st, tY, tE, tWi, tWh, b_ih,
+                 b_hh, En, EnT, ld_T, n_tiles, n_real, status);
   note_launch();
-  return cudaGetLastError();
+  return e;
 }
 
 cudaError_t gru_bwd_tc(int n_pad, int n_real, const __nv_bfloat16* Y, const __nv_bfloat16* E,
@@ -565,11 +571,10 @@ cudaError_t gru_bwd_tc(int n_pad, int n_real, const __nv_bfloat16* Y, const __nv
   if (e != cudaSuccess) return e;
   const int n_tiles = n_pad / 128;
   const int grid = std::min(n_tiles, gemm_tn_num_sms());
-  k_gru_bwd_tc<<<grid, kThreads, GruSmem::BWD, st>>>(tY, tE, tWi, tWh, tWiT, tWhT, tG, b_ih, b_hh,
-                                                     gout, dXT, ld_x, dgiT, dghT, ld_g, n_tiles,
-                                                     n_real, status);
+  e = launch_pdl(k_gru_bwd_tc, dim3(grid), dim3(kThreads), GruSmem::BWD, st, tY, tE, tWi, tWh, tWiT,
+                 tWhT, tG, b_ih, b_hh, gout, dXT, ld_x, dgiT, dghT, ld_g, n_tiles, n_real, status);
   note_launch();
-  return cudaGetLastError();
+  return e;
 }
 
 }  // namespace bg

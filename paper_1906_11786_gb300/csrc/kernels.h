@@ -12,6 +12,24 @@ namespace bg {
 // Counts every kernel this library launches (bg_launch_count).
 void note_launch();
 
+// Launches `kernel` with programmatic stream serialization: it may begin before the previous
+// kernel in `st` completes and must call grid_dep_wait() before touching that kernel's data.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // Generic fp32-accumulate GEMM with arbitrary element strides (covers transposed operands):
 //   C[b][m][n] (+)= sum_k A(b,m,k) B(b,k,n) + bias[b*sBias + n]
 // A(b,m,k) = A[b*sAb + m*sAm + k*sAk], B(b,k,n) = B[b*sBb + k*sBk + n*sBn]; C is row-major with

@@ -79,6 +79,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* s
   return mbar_wait_poll(bar, parity, status, site, abort, backoff_ns);
 }
 
+// Programmatic dependent launch.  A kernel launched with programmatic stream serialization may
+// start while the previous kernel in the stream is still running: grid_dep_wait() blocks until
+// that kernel has completed and its memory operations are visible, so every read of data it
+// produced, and every write that it might still read, must come after the wait.
+// grid_dep_launch() lets the next such kernel be scheduled as SMs free up.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // One lane of a converged warp (the lane that issues tcgen05.mma / commit for the whole warp).
 __device__ __forceinline__ bool elect_one_sync() {
   uint32_t pred;
