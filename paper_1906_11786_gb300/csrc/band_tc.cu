@@ -59,13 +59,20 @@ namespace {
 constexpr int kTile = 128;     // rows per tile = UMMA M
 constexpr int kAtom = 64;      // bf16 per 128-byte swizzle row
 
-template <int H>
+// Block size S: a 128-row tile sees a window of C1 128-column chunks of the state (and of its
+// bit tiles): rows [row0, row0 + 128) only couple to columns in block-rows kr - 1 .. kr + 1 of
+// their own block-row kr, which all lie in [ws, ws + 128 C1) with ws = (row0 / S) S - S.
+//   S <= 64: C1 = 2 (the tile spans 128 / S block-rows);  S = 128: C1 = 3;  S = 256: C1 = 6.
+__host__ __device__ constexpr int band_chunks(int S) { return S <= 64 ? 2 : 3 * (S / 128); }
+
+template <int H, int S>
 struct Cfg {
   static constexpr bool TF = H <= 64;                         // split issuers, tf32 second product
-  static constexpr int NXB = H <= 64 ? 2 : 1;                 // state-window buffers
-  static constexpr int NW = 2;                                // W ring stages
+  static constexpr int C1 = band_chunks(S);                   // 128-column chunks per type
   static constexpr int ATOM_X = H * 128;                      // 64 nodes x H rows
-  static constexpr int XWIN = 6 * ATOM_X;                     // 3 blocks x 2 atoms (S = 128)
+  static constexpr int XWIN = 2 * C1 * ATOM_X;                // the window, 64-node atoms
+  static constexpr int NXB = XWIN <= 48 * 1024 ? 2 : 1;       // state-window buffers
+  static constexpr int NW = 2;                                // W ring stages
   // H x H operand of the second product: fp32 (32 per 128-byte row) or bf16 (64 per row)
   static constexpr int WSTAGE = (TF ? H / 32 : H / kAtom) * H * 128;
   static constexpr int DEG = kTile * 128;                     // 128 rows x 64 bf16
@@ -74,8 +81,8 @@ struct Cfg {
   static constexpr int OFF_W = OFF_X + NXB * XWIN;
   static constexpr int OFF_DEG = OFF_W + NW * WSTAGE;
   static constexpr int OFF_B2 = OFF_DEG + 2 * DEG;
-  static constexpr int NM = H <= 64 ? 8 : 2;                  // mask ring stages (one type each)
-  static constexpr int MSTAGE = 3 * kTile * 16;               // 3 diagonals x 128 rows x 128 bits
+  static constexpr int MSTAGE = C1 * kTile * 16;              // C1 chunks x 128 rows x 128 bits
+  static constexpr int NM = H <= 64 ? (C1 <= 3 ? 8 : 4) : 2; // mask ring stages (one type each)
   static constexpr int OFF_M = OFF_B2 + B2;
   static constexpr int OFF_BAR = OFF_M + NM * MSTAGE;
   static constexpr int SMEM = OFF_BAR + 1024 + 1024;          // barriers + 1 KB alignment slack
@@ -85,12 +92,17 @@ struct Cfg {
   static constexpr int D1COL0 = H;
   static constexpr int ACOL = (NB + 1) * H;
   static constexpr int NA = (512 - ACOL) / 64;
-  static constexpr int NT = 8;                                // per-type barrier ring (H = 64)
+  // H = 64: a type's chunks come in CG-chunk groups (one barrier wait each), G groups per type
+  static constexpr int CG = C1 <= 3 ? C1 : 3;
+  static constexpr int G = C1 / CG;
+  static constexpr int NT = 8;                                // per-group barrier ring
   // expander warpgroups: at H = 64 two, taking the edge types in turn
   static constexpr int NE = TF ? 2 : 1;
   static constexpr int THREADS = 128 * (2 + NE);
+  static_assert(C1 % CG == 0 && NT % G == 0, "chunk groups");
   static_assert(NA >= 2 && NA <= 8, "A-slot ring");
-  static_assert(!TF || NA >= 3, "one edge type's three A tiles must fit");
+  static_assert(!TF || NA >= CG, "one group of A tiles must fit");
+  static_assert(NM <= 8, "mask ring");
   static_assert(SMEM <= 232448, "shared memory");
 };
 
@@ -143,15 +155,15 @@ __device__ __forceinline__ void drain_mmas(bool leader, uint64_t* bar) {
   }
 }
 
-template <int H, bool BWD>
-__global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
+template <int H, int S, bool BWD>
+__global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     k_band_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
               const __grid_constant__ CUtensorMap tm_deg, const __grid_constant__ CUtensorMap tm_b2,
               const uint32_t* __restrict__ maskI, float* __restrict__ out,
               __nv_bfloat16* __restrict__ outb, __nv_bfloat16* __restrict__ outT, int64_t ld_outT,
-              __nv_bfloat16* __restrict__ dMT, int64_t ld_mt, int K, int P, int has_bias,
+              __nv_bfloat16* __restrict__ dMT, int64_t ld_mt, int n_tiles, int P, int has_bias,
               int accumulate, int* status) {
-  using C = Cfg<H>;
+  using C = Cfg<H, S>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -162,9 +174,9 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
   uint8_t* b2s = smem + C::OFF_B2;
   uint8_t* mring = smem + C::OFF_M;
   volatile int* abort = &bars->abort;
-  // arrivals that complete one type's t_full phase: 4 expander warps, the second issuer's commit
-  // and, backward, the 4 converter warps
-  constexpr int kTArrivals = 4 + 1 + (BWD ? 4 : 0);
+  // releases of a pre_p buffer, which also complete the first group of a type (H = 64): the second
+  // issuer's commit and, backward, the 4 converter warps; every group also needs 4 expander warps
+  constexpr int kFree = 1 + (BWD ? 4 : 0);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -175,7 +187,8 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
     for (int i = 0; i < 4; ++i) { mbar_init(&bars->d1_full[i], 1); mbar_init(&bars->pre_ready[i], 4); }
     for (int i = 0; i < 4; ++i) { mbar_init(&bars->w_full[i], 1); mbar_init(&bars->w_empty[i], 1); }
     for (int i = 0; i < 8; ++i) { mbar_init(&bars->a_full[i], 4); mbar_init(&bars->a_empty[i], 1); }
-    for (int i = 0; i < 8; ++i) mbar_init(&bars->t_full[i], kTArrivals);
+    // group gi = G c + j of type c sits in slot gi % NT; first groups (j = 0) also take the release
+    for (int i = 0; i < 8; ++i) mbar_init(&bars->t_full[i], 4 + (i % C::G == 0 ? kFree : 0));
     mbar_init(&bars->b2_full, 1);
     mbar_init(&bars->y_full, 1);
     mbar_init(&bars->y_empty, 4);
@@ -187,7 +200,7 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
     if (C::TF) {
       // the first NB types find their pre_p buffer free: stand in for the releases
       for (int c = 0; c < C::NB; ++c)
-        for (int a = 0; a < kTArrivals - 4; ++a) mbar_arrive(&bars->t_full[c]);
+        for (int a = 0; a < kFree; ++a) mbar_arrive(&bars->t_full[(c * C::G) % C::NT]);
     }
   }
   if (warp == 1) {
@@ -200,7 +213,6 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
   // TMEM is held: the next kernel in the stream may be scheduled on SMs as they free up
   grid_dep_launch();
   const uint32_t tmem = bars->tmem_base;
-  const int n_tiles = K;  // S = 128: one tile per block-row
 
   if (warp == 0 && lane == 0) {
     // ------------------------------------------------------------------ TMA producer
@@ -220,35 +232,27 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
       const int xb = i % C::NXB;
       if (!mbar_wait(&bars->x_empty[xb], ((i / C::NXB) & 1) ^ 1, status, 101, abort, 64)) break;
       ++n_x[xb];
-      uint32_t bytes = 0;
-      for (int d = 0; d < 3; ++d) {
-        const int kb = k + d - 1;
-        if (kb >= 0 && kb < K) bytes += 2 * C::ATOM_X;
-      }
-      mbar_expect_tx(&bars->x_full[xb], bytes);
-      for (int d = 0; d < 3; ++d) {
-        const int kb = k + d - 1;
-        if (kb < 0 || kb >= K) continue;
-        for (int a = 0; a < 2; ++a)
-          tma_load_2d(xwin + xb * C::XWIN + (d * 2 + a) * C::ATOM_X, &tm_x, &bars->x_full[xb],
-                      kb * kTile + a * kAtom, 0);
-      }
+      // window rows ws .. ws + 128 C1; rows outside [0, n) arrive as zeros (TMA bounds fill)
+      const int row0 = k * kTile, ws = (row0 / S) * S - S;
+      mbar_expect_tx(&bars->x_full[xb], C::XWIN);
+      for (int a = 0; a < 2 * C::C1; ++a)
+        tma_load_2d(xwin + xb * C::XWIN + a * C::ATOM_X, &tm_x, &bars->x_full[xb], ws + a * kAtom, 0);
       if (has_bias) {
         const int db = i & 1;
         if (!mbar_wait(&bars->deg_empty[db], ((i >> 1) & 1) ^ 1, status, 102, abort, 64)) break;
         ++n_deg[db];
         mbar_expect_tx(&bars->deg_full[db], C::DEG);
-        tma_load_2d(degs + db * C::DEG, &tm_deg, &bars->deg_full[db], 0, k * kTile);
+        tma_load_2d(degs + db * C::DEG, &tm_deg, &bars->deg_full[db], 0, row0);
       }
       for (int p = 0; p < P; ++p, ++widx) {
-        const int ws = widx % C::NW;
-        if (!mbar_wait(&bars->w_empty[ws], ((widx / C::NW) & 1) ^ 1, status, 103, abort, 64)) break;
-        ++n_w[ws];
-        mbar_expect_tx(&bars->w_full[ws], C::WSTAGE);
+        const int ws2 = widx % C::NW;
+        if (!mbar_wait(&bars->w_empty[ws2], ((widx / C::NW) & 1) ^ 1, status, 103, abort, 64)) break;
+        ++n_w[ws2];
+        mbar_expect_tx(&bars->w_full[ws2], C::WSTAGE);
         // atoms of 128-byte rows along K: 32 fp32 (tf32 operand) or 64 bf16 each
         constexpr int kw = C::TF ? 32 : kAtom;
         for (int a = 0; a < H / kw; ++a)
-          tma_load_2d(wring + ws * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws], a * kw,
+          tma_load_2d(wring + ws2 * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws2], a * kw,
                       p * H);
       }
     }
@@ -265,7 +269,7 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
     }
   } else if (warp == 2 && lane == 0) {
     // ------------------------------------------------------------------ mask producer
-    // each type's three bit tiles (contiguous [3][128][4] words), NM types ahead of the expanders
+    // each type's C1 bit chunks (contiguous [C1][128][4] words), NM types ahead of the expanders
     uint32_t midx = 0, n_m[8] = {0};
     for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x) {
       bool ok = true;
@@ -277,8 +281,8 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
         }
         ++n_m[ms];
         mbar_expect_tx(&bars->m_full[ms], C::MSTAGE);
-        bulk_load(mring + ms * C::MSTAGE, maskI + ((size_t)k * P + p) * 3 * kTile * 4, C::MSTAGE,
-                  &bars->m_full[ms]);
+        bulk_load(mring + ms * C::MSTAGE, maskI + ((size_t)k * P + p) * C::C1 * kTile * 4,
+                  C::MSTAGE, &bars->m_full[ms]);
       }
       if (!ok) break;
     }
@@ -288,37 +292,37 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
         }
   } else if (warp == 1 && C::TF) {
     // ------------------------------------------------------------------ band-product issuer
-    // pre_p = sum_d A_{k,d,p} X_{k+d}: one t_full wait per type, then an unbroken MMA stream
+    // pre_p = sum over the window chunks of A_{tile,p,j} X_j: one t_full wait per group of chunks,
+    // then an unbroken MMA stream
     const bool leader = elect_one_sync();
     constexpr uint32_t idesc = idesc_bf16_f32(kTile, H);
-    uint32_t c = 0, aidx = 0;
+    uint32_t c = 0, slot = 0, gi = 0;
     bool ok = true;
     int i = 0;
     for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x, ++i) {
       const int xb = i % C::NXB;
       if (!mbar_wait(&bars->x_full[xb], (i / C::NXB) & 1, status, 204, abort)) break;
-      const uint32_t xbase = smem_u32(xwin + xb * C::XWIN);
-      for (int p = 0; p < P; ++p, ++c) {
-        const int b = c % C::NB;
-        if (!mbar_wait(&bars->t_full[c % C::NT], (c / C::NT) & 1, status, 210, abort)) { ok = false; break; }
-        tc_fence_after();
-        uint32_t first = 1;
-        for (int d = 0; d < 3; ++d) {
-          const int kb = k + d - 1;
-          if (kb < 0 || kb >= K) continue;
-          const int slot = aidx % C::NA;
+      // descriptors differ from the window's first one only in the start-address field
+      const uint64_t xdesc = desc_sw128_kmajor(smem_u32(xwin + xb * C::XWIN));
+      for (int p = 0; p < P && ok; ++p, ++c) {
+        const uint32_t d1 = tmem + C::D1COL0 + (c % C::NB) * H;
+        for (int g = 0; g < C::G; ++g, ++gi) {
+          if (!mbar_wait(&bars->t_full[gi % C::NT], (gi / C::NT) & 1, status, 210, abort)) { ok = false; break; }
+          tc_fence_after();
+          for (int j = g * C::CG; j < (g + 1) * C::CG; ++j) {
+            const uint32_t a = tmem + C::ACOL + slot * 64;
+            const uint64_t jdesc = xdesc + (uint64_t)((2 * j * C::ATOM_X) >> 4);
 #pragma unroll
-          for (int kk = 0; kk < kTile / 16; ++kk) {
-            const uint64_t bdesc =
-                desc_sw128_kmajor(xbase + (d * 2 + kk / 4) * C::ATOM_X + (kk % 4) * 32);
-            if (leader) mma_ts(tmem + C::D1COL0 + b * H, tmem + C::ACOL + slot * 64 + kk * 8, bdesc, idesc,
-                   (first && kk == 0) ? 0u : 1u);
+            for (int kk = 0; kk < kTile / 16; ++kk)
+              if (leader)
+                mma_ts(d1, a + kk * 8, jdesc + (uint64_t)(((kk / 4) * C::ATOM_X + (kk % 4) * 32) >> 4),
+                       idesc, (j == 0 && kk == 0) ? 0u : 1u);
+            if (leader) tc_commit(&bars->a_empty[slot]);
+            slot = slot + 1 == (uint32_t)C::NA ? 0 : slot + 1;
           }
-          first = 0;
-          if (leader) tc_commit(&bars->a_empty[slot]);
-          ++aidx;
         }
-        if (leader) tc_commit(&bars->d1_full[b]);
+        if (!ok) break;
+        if (leader) tc_commit(&bars->d1_full[c % C::NB]);
         if (p == P - 1 && leader) tc_commit(&bars->x_empty[xb]);
       }
     }
@@ -352,7 +356,8 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
         }
         if (leader) {
           tc_commit(&bars->w_empty[ws]);
-          tc_commit(&bars->t_full[(c + C::NB) % C::NT]);  // this pre_p buffer is free again
+          // this pre_p buffer is free again: part of type c + NB's first group
+          tc_commit(&bars->t_full[((c + C::NB) * C::G) % C::NT]);
         }
       }
       if (!ok) break;
@@ -410,21 +415,17 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
       int next_s2 = 0;
       for (int p = 0; p < P && ok; ++p, ++c) {
         const int b = c % C::NB;
-        uint32_t first = 1;
-        for (int d = 0; d < 3; ++d) {
-          const int kb = k + d - 1;
-          if (kb < 0 || kb >= K) continue;
+        for (int j = 0; j < C::C1; ++j) {
           const int slot = aidx % C::NA;
           if (!mbar_wait(&bars->a_full[slot], (aidx / C::NA) & 1, status, 205, abort)) { ok = false; break; }
           tc_fence_after();
 #pragma unroll
           for (int kk = 0; kk < kTile / 16; ++kk) {
             const uint64_t bdesc =
-                desc_sw128_kmajor(xbase + (d * 2 + kk / 4) * C::ATOM_X + (kk % 4) * 32);
+                desc_sw128_kmajor(xbase + (2 * j + kk / 4) * C::ATOM_X + (kk % 4) * 32);
             if (leader) mma_ts(tmem + C::D1COL0 + b * H, tmem + C::ACOL + slot * 64 + kk * 8, bdesc, idesc,
-                   (first && kk == 0) ? 0u : 1u);
+                   (j == 0 && kk == 0) ? 0u : 1u);
           }
-          first = 0;
           if (leader) tc_commit(&bars->a_empty[slot]);
           ++aidx;
         }
@@ -460,10 +461,9 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
     uint32_t aidx = 0, midx = 0;
     for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x) {
       bool ok = true;
-      const int n_diag = (k > 0) + 1 + (k + 1 < K);
       for (int p = 0; p < P && ok; ++p, ++midx) {
         if (C::NE > 1 && (int)(midx % C::NE) != eg) {
-          aidx += n_diag;  // the other group's type
+          aidx += C::C1;  // the other group's type
           continue;
         }
         const int ms = midx % C::NM;
@@ -472,10 +472,8 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
           break;
         }
         const uint8_t* mrow = mring + ms * C::MSTAGE + r * 16;
-        for (int d = 0; d < 3; ++d) {
-          const int kb = k + d - 1;
-          if (kb < 0 || kb >= K) continue;
-          const uint4 m = *reinterpret_cast<const uint4*>(mrow + d * kTile * 16);
+        for (int j = 0; j < C::C1; ++j) {
+          const uint4 m = *reinterpret_cast<const uint4*>(mrow + j * kTile * 16);
           const int slot = aidx % C::NA;
           if (!mbar_wait(&bars->a_empty[slot], ((aidx / C::NA) & 1) ^ 1, status, 301, abort)) {
             ok = false;
@@ -493,16 +491,16 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
             tmem_wait_st();
             tc_fence_before();
             warp_arrive(&bars->a_full[slot]);
+          } else if ((j + 1) % C::CG == 0) {
+            // all of this group's A tiles are in TMEM
+            tmem_wait_st();
+            tc_fence_before();
+            const uint32_t gi = midx * C::G + j / C::CG;
+            warp_arrive(&bars->t_full[gi % C::NT]);
           }
           ++aidx;
         }
         if (!ok) break;
-        if (C::TF) {
-          // all of this type's A tiles are in TMEM
-          tmem_wait_st();
-          tc_fence_before();
-          warp_arrive(&bars->t_full[midx % C::NT]);
-        }
         warp_arrive(&bars->m_empty[ms]);
       }
       if (!ok) break;
@@ -538,7 +536,7 @@ __global__ void __launch_bounds__(Cfg<H>::THREADS, 1)
           if (C::TF) {
             // pre_p stays fp32 for the tf32 product: release the buffer before the stores
             tc_fence_before();
-            warp_arrive(&bars->t_full[(c + C::NB) % C::NT]);
+            warp_arrive(&bars->t_full[((c + C::NB) * C::G) % C::NT]);
           } else {
             // packed pairs of columns h0..h0+63 go to columns (h0/2)..(h0/2)+31 of the buffer
             tmem_st32(col + h0 / 2, pk);
@@ -716,22 +714,46 @@ int num_sms() {
 
 inline size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
 
+template <int H, int S, bool BWD>
+cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
+                     const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
+                     __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
+                     __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate, int* status,
+                     cudaStream_t st) {
+  using C = Cfg<H, S>;
+  cudaError_t e = cudaFuncSetAttribute(k_band_tc<H, S, BWD>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  const int n_tiles = p->n_pad() / kTile;
+  const int grid = std::min(n_tiles, num_sms());
+  e = launch_pdl(k_band_tc<H, S, BWD>, dim3(grid), dim3(C::THREADS), C::SMEM, st, tx, tw, tdeg,
+                 tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt,
+                 n_tiles, p->P, has_bias, accumulate, status);
+  note_launch();
+  return e;
+}
+
+// The shapes with a tensor-core kernel: H = 64 at S in {32, 64, 128, 256}; H = 128 at S = 128.
 template <int H, bool BWD>
 cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
                    const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
                    __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
                    __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate, int* status,
                    cudaStream_t st) {
-  using C = Cfg<H>;
-  cudaError_t e = cudaFuncSetAttribute(k_band_tc<H, BWD>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-  if (e != cudaSuccess) return e;
-  const int grid = std::min(p->K, num_sms());
-  e = launch_pdl(k_band_tc<H, BWD>, dim3(grid), dim3(C::THREADS), C::SMEM, st, tx, tw, tdeg, tb2,
-                 BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt, p->K, p->P,
-                 has_bias, accumulate, status);
-  note_launch();
-  return e;
+#define BG_BAND_S(SV)                                                                            \
+  return launch_s<H, SV, BWD>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, dMT, ld_mt,      \
+                              has_bias, accumulate, status, st);
+  if constexpr (H == 64) {
+    switch (p->S) {
+      case 32: BG_BAND_S(32)
+      case 64: BG_BAND_S(64)
+      case 256: BG_BAND_S(256)
+      default: BG_BAND_S(128)
+    }
+  } else {
+    BG_BAND_S(128)
+  }
+#undef BG_BAND_S
 }
 
 }  // namespace
@@ -782,8 +804,11 @@ bool make_map_3d(CUtensorMap* m, const void* base, uint64_t batch, uint64_t rows
 }
 
 bool band_tc_supported(const bg_plan* p, int dtype, int H) {
-  return p && dtype == 1 && p->S == 128 && (H == 64 || H == 128) && p->P <= 32 && p->d_maskI &&
-         p->d_maskTI && p->d_deg2 && p->max_deg <= 256 && encode_fn() != nullptr;
+  if (!p || dtype != 1 || p->P > 32 || p->n_pad() % kTile) return false;
+  const bool shape = (H == 64 && (p->S == 32 || p->S == 64 || p->S == 128 || p->S == 256)) ||
+                     (H == 128 && p->S == 128);
+  return shape && p->d_maskI && p->d_maskTI && p->d_deg2 && p->max_deg <= 256 &&
+         encode_fn() != nullptr;
 }
 
 size_t band_tc_w_bytes(const bg_plan* p, int H) {
@@ -883,6 +908,7 @@ cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, c
   if (e == cudaSuccess) e = band_tc_prep_w(p, H, W, 0, WT, st);
   if (e == cudaSuccess && b) e = prep_bias_split(b, b2T, P, H, st);
   if (e != cudaSuccess) return e;
+  ProfSpan span(BG_KID_BAND_FWD, st);
   return band_tc_fwd_core(p, H, ET, n, WT, b ? b2T : nullptr, Y, nullptr, nullptr, 0, status, st);
 }
 
@@ -904,20 +930,27 @@ cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, c
   const size_t part_floats = gemm_tn_part_floats(P * H, H + 16, (int64_t)n);
   cudaError_t e = prep_transpose_bf16(dY, 1, dYT, n, H, 1, st);
   if (e == cudaSuccess) e = band_tc_prep_w(p, H, W, 1, Wk, st);
-  if (e == cudaSuccess) e = band_tc_bwd_core(p, H, dYT, n, Wk, dE, accum, dMT, n, status, st);
+  if (e == cudaSuccess) {
+    ProfSpan span(BG_KID_BAND_BWD, st);
+    e = band_tc_bwd_core(p, H, dYT, n, Wk, dE, accum, dMT, n, status, st);
+  }
   if (e != cudaSuccess) return e;
   // [E^T; 1; 0]: the ones row turns the bias gradient into column H of the same product
   e = prep_transpose_bf16(E, 0, ETa, n, H, 1, st);
   if (e == cudaSuccess) e = fill_ones_rows(ETa, H, n, n, st);
   if (e != cudaSuccess) return e;
   // dW_p[h][h'] (+)= sum_nodes E[node][h] dM_p[node][h'],  db_p[h'] (+)= sum_nodes dM_p[node][h']
+  ProfSpan span(BG_KID_DW, st);
   return gemm_tn(dMT, n, ETa, n, P * H, H, n, 1, dW, db, accum, part, part_floats, status, st);
 }
 
 int band_tc_upload(bg_plan* p, cudaStream_t st) {
-  if (p->S != 128 || p->P > 32) return 0;
-  const int K = p->K, P = p->P, S = p->S, W32 = p->W32;
+  const int S = p->S;
+  if (p->P > 32 || (S != 32 && S != 64 && S != 128 && S != 256)) return 0;
+  const int K = p->K, P = p->P, W32 = p->W32;
   const size_t n = (size_t)K * S;
+  if (n % kTile) return 0;
+  const int n_tiles = (int)(n / kTile), C1 = band_chunks(S);
   // interleave bits of every word: column 2j -> bit j, column 2j+1 -> bit 16+j
   auto inter = [](uint32_t w) {
     uint32_t o = 0;
@@ -927,19 +960,27 @@ int band_tc_upload(bg_plan* p, cudaStream_t st) {
     }
     return o;
   };
-  std::vector<uint32_t> mi((size_t)K * P * 3 * S * W32), mti(mi.size());
+  // per (tile, type): the C1 128-column chunks of the tile's window [ws, ws + 128 C1), 4 words per
+  // row per chunk; words outside the three block diagonals of the row's block-row are zero
+  std::vector<uint32_t> mi((size_t)n_tiles * P * C1 * kTile * 4), mti(mi.size());
   std::vector<uint16_t> deg(n * 64, 0);
   int max_deg = 0;
-  for (int k = 0; k < K; ++k)
-    for (int d = 0; d < 3; ++d)
-      for (int q = 0; q < P; ++q)
-        for (int r = 0; r < S; ++r)
-          for (int w = 0; w < W32; ++w) {
-            const size_t src = ((((size_t)k * 3 + d) * P + q) * S + r) * W32 + w;
-            const size_t dst = ((((size_t)k * P + q) * 3 + d) * S + r) * W32 + w;
+  for (int t = 0; t < n_tiles; ++t) {
+    const int64_t row0 = (int64_t)t * kTile, ws = (row0 / S) * S - S;
+    for (int q = 0; q < P; ++q)
+      for (int j = 0; j < C1; ++j)
+        for (int r = 0; r < kTile; ++r)
+          for (int w = 0; w < 4; ++w) {
+            const int64_t R = row0 + r, Cc = ws + j * kTile + 32 * w;
+            const size_t dst = ((((size_t)t * P + q) * C1 + j) * kTile + r) * 4 + w;
+            if (Cc < 0 || Cc >= (int64_t)n) continue;
+            const int64_t kr = R / S, kc = Cc / S, d = kc - kr + 1;
+            if (d < 0 || d > 2) continue;
+            const size_t src = ((((size_t)kr * 3 + d) * P + q) * S + R % S) * W32 + (Cc % S) / 32;
             mi[dst] = inter(p->masks[src]);
             mti[dst] = inter(p->masksT[src]);
           }
+  }
   for (int k = 0; k < K; ++k)
     for (int q = 0; q < P; ++q)
       for (int r = 0; r < S; ++r) {

@@ -33,8 +33,9 @@ struct bg_plan {
   int32_t* d_seg_off = nullptr;
   int32_t* d_seg_cnt = nullptr;
   int32_t* d_row_graph = nullptr;  // [n_pad] packed graph of each position, -1 for padding
-  // tensor-core path (S = 128): bit-interleaved tiles [K][P][3][S][W32] in both orientations and
-  // per-row in-degree counts [n_pad][64] bf16 (type p at columns p and 32 + p)
+  // tensor-core path: bit-interleaved window chunks [n_pad / 128][P][C1][128][4] (C1 128-column
+  // chunks per 128-row tile, band_tc.cu) in both orientations and per-row in-degree counts
+  // [n_pad][64] bf16 (type p at columns p and 32 + p)
   uint32_t* d_maskI = nullptr;
   uint32_t* d_maskTI = nullptr;
   uint16_t* d_deg2 = nullptr;

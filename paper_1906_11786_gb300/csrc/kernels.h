@@ -12,6 +12,21 @@ namespace bg {
 // Counts every kernel this library launches (bg_launch_count).
 void note_launch();
 
+// CUDA events around a span of launches on `st`, accumulated under kernel id `kid` (BG_KID_*)
+// while profiling is on (bg_profile_enable); no events otherwise.
+class ProfSpan {
+ public:
+  ProfSpan(int kid, cudaStream_t st);
+  ~ProfSpan();
+  ProfSpan(const ProfSpan&) = delete;
+  ProfSpan& operator=(const ProfSpan&) = delete;
+
+ private:
+  int kid_;
+  cudaStream_t st_;
+  cudaEvent_t a_ = nullptr, b_ = nullptr;
+};
+
 // Launches `kernel` with programmatic stream serialization: it may begin before the previous
 // kernel in `st` completes and must call grid_dep_wait() before touching that kernel's data.
 template <typename... KArgs, typename... Args>

@@ -21,10 +21,24 @@ def built():
     torch.manual_seed(0)
 
 
+def _tc_shape(c: Case) -> bool:
+    """Shapes the fused tensor-core band kernels carry: bf16, P <= 32, whole 128-row tiles, and
+    H = 64 at S in {32, 64, 128, 256} or H = 128 at S = 128."""
+    return (c.dtype == "bf16" and c.P <= 32 and c.N % 128 == 0 and
+            ((c.H == 64 and c.S in (32, 64, 128, 256)) or (c.H == 128 and c.S == 128)))
+
+
+def _cap_whole_tiles(gs, S):
+    """Capacity (blocks) that makes the padded size a whole number of 128-row tiles."""
+    n = sum(g.n_nodes for g in gs)
+    per_tile = max(1, 128 // S)
+    blocks = -(-n // S)
+    return -(-blocks // per_tile) * per_tile
+
+
 def _expect_path(c: Case):
-    """The fused tensor-core kernels must carry every bf16 case with S = 128, H in {64, 128}."""
-    want = c.dtype == "bf16" and c.S == 128 and c.H in (64, 128) and c.P <= 32
-    assert L.band_uses_tensor_cores(c.plan, c.dtype, c.H) == want
+    """The fused tensor-core kernels must carry every shape they support."""
+    assert L.band_uses_tensor_cores(c.plan, c.dtype, c.H) == _tc_shape(c)
 
 
 def _fwd(c: Case, with_bias=True):
@@ -78,11 +92,13 @@ def test_propagate_fp32_config1():
         assert rel_err(g, r) < TOL["f32"], name
 
 
-@pytest.mark.parametrize("S,H", [(128, 64), (64, 64), (32, 32), (256, 128), (128, 256)])
-def test_propagate_bf16_packed_batch(S, H):
-    """Several graphs packed into several block-rows with a ragged tail."""
+@pytest.mark.parametrize("S,H,whole", [(128, 64, 0), (64, 64, 1), (32, 32, 0), (256, 128, 0),
+                                       (128, 256, 0), (256, 64, 1), (32, 64, 1), (64, 64, 0)])
+def test_propagate_bf16_packed_batch(S, H, whole):
+    """Several graphs packed into several block-rows with a ragged tail (`whole`: capacity padded
+    to whole 128-row tiles, as the tensor-core kernels need below S = 128)."""
     gs = synth.gen_batch(7, 60, 400, 10, True, S // 2, S // 3, 2.0, 100 + S + H)
-    c = Case(gs, 20, S, H, "bf16", seed=S + H)
+    c = Case(gs, 20, S, H, "bf16", seed=S + H, cap=_cap_whole_tiles(gs, S) if whole else 0)
     assert c.info["K"] >= 3 and c.n_real % S != 0
     Y, ref = _fwd(c)
     assert rel_err(Y, ref) < TOL["bf16"]
@@ -141,14 +157,17 @@ def _ggnn(c: Case, T, seed=3):
         dE0.cpu().numpy(), ref
 
 
-@pytest.mark.parametrize("dtype,T,S,H", [("f32", 2, 64, 64), ("bf16", 3, 64, 64),
-                                         ("bf16", 2, 128, 128), ("bf16", 2, 32, 32),
-                                         ("bf16", 2, 128, 256)])
-def test_ggnn_fwd_bwd(dtype, T, S, H):
+@pytest.mark.parametrize("dtype,T,S,H,whole", [("f32", 2, 64, 64, 0), ("bf16", 3, 64, 64, 0),
+                                               ("bf16", 2, 128, 128, 0), ("bf16", 2, 32, 32, 0),
+                                               ("bf16", 2, 128, 256, 0), ("bf16", 2, 256, 64, 1),
+                                               ("bf16", 3, 64, 64, 1), ("bf16", 2, 32, 64, 1)])
+def test_ggnn_fwd_bwd(dtype, T, S, H, whole):
     """Every kernel family of the GGNN step: SIMT (fp32, H = 256), tensor-core GEMMs around the
-    SIMT band sums (S != 128), fused band kernels with GEMM-based GRU (H = 128)."""
+    SIMT band sums (ragged tiles, H = 32), fused band kernels with GEMM-based GRU (H = 128), fused
+    band and GRU kernels at S = 32, 64, 256 (H = 64)."""
     gs = synth.gen_batch(5, 60, 300, 10, True, max(8, S // 2), max(8, S // 3), 2.0, 41)
-    c = Case(gs, 20, S, H, dtype, seed=9)
+    c = Case(gs, 20, S, H, dtype, seed=9, cap=_cap_whole_tiles(gs, S) if whole else 0)
+    assert L.band_uses_tensor_cores(c.plan, c.dtype, c.H) == _tc_shape(c)
     ET, ref_ET, grads, dE0, ref = _ggnn(c, T)
     tol = TOL[dtype]
     assert rel_err(ET, ref_ET) < tol
