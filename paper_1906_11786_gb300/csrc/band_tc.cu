@@ -10,9 +10,12 @@
 // instead of W_p^T gives dE_j += sum_p (A^T dY)_p W_p^T; dM_p = A_p^T dY is also written (bf16,
 // transposed) for the weight gradient.
 //
-// At H = 64 the second product runs as kind::tf32 straight from the fp32 pre_p (W_p staged as
-// fp32), so no thread touches pre_p between the two products and the MMA issuer never waits on
-// a conversion; at H = 128 pre_p is rounded to bf16 in place by the converter warps first.
+// The second product runs as kind::tf32 straight from the fp32 pre_p (W_p staged as fp32), so no
+// thread touches pre_p between the two products and no MMA issuer waits on a conversion.  The
+// band product is N = 64: at H = 128 the tile makes two passes over 64-column halves of the state,
+// pass hh contracting the band with columns 64 hh .. of E and multiplying by rows 64 hh .. of W_p
+// (Y = sum_p sum_hh pre_p[:, hh] W_p[hh, :]); the (half, type) jobs alternate between two
+// 64-column pre_p units, so a job's band products overlap the previous job's W product.
 //
 // The 0/1 adjacency is the MMA's A operand.  It is stored as bits (the whole band costs
 // 3 P S^2 / 8 bytes per block-row) and expanded on chip straight into tensor memory: the bits of
@@ -21,19 +24,18 @@
 //
 // Roles (128 x (2 + expander groups) threads, one CTA per SM, persistent over tiles):
 //   warp 0      TMA producer: state blocks (B operand of the band product), W tiles, deg, bias
-//   warp 1      TMEM allocator and MMA issuer (an elected lane of the converged warp issues):
-//               at H = 64 the band products only, one wait per edge type; otherwise every MMA
+//   warp 1      TMEM allocator and band-product issuer (an elected lane of the converged warp
+//               issues), one wait per job (per chunk group at S = 256)
 //   warp 2      mask producer: one bulk copy per (tile, type) of the bit tiles into an SMEM ring
-//   warp 3      (H = 64) second MMA issuer: the pre_p W_p products and the bias product, so that
-//               their waits never stall the band-product stream
+//   warp 3      second MMA issuer: the pre_p W_p products and the bias product, so that their
+//               waits never stall the band-product stream
 //   expanders   thread r of a warpgroup turns row r's mask bits into bf16 A tiles in TMEM; two
-//               warpgroups taking the edge types in turn at H = 64 (warps 4-11), one otherwise
-//   converters  the last warpgroup: pre_p fp32 -> bf16 (H = 128), dM_p to global (backward),
-//               final epilogue TMEM -> global
+//               warpgroups taking the edge types in turn (warps 4-11)
+//   converters  the last warpgroup: dM_p to global (backward), final epilogue TMEM -> global
 // A tcgen05.mma of N = 64 is about as long as its issue, so any wait on the band-product
-// issuer leaves the tensor pipe idle: at H = 64 that issuer waits once per edge type, on a
-// barrier that the expanders (all three A tiles in TMEM), the second issuer (the pre_p buffer is
-// free) and in the backward pass the converters complete together.
+// issuer leaves the tensor pipe idle: that issuer waits once per job, on a barrier that the
+// expanders (all the job's A tiles are in TMEM), the second issuer (the pre_p unit is free) and
+// in the backward pass the converters complete together.
 // Consumer warps signal a barrier with one arrive per warp after __syncwarp.  Waiting roles other
 // than the expanders sleep between polls so that the MMA issuers keep their issue slots.
 #include <cuda.h>
@@ -67,42 +69,46 @@ __host__ __device__ constexpr int band_chunks(int S) { return S <= 64 ? 2 : 3 * 
 
 template <int H, int S>
 struct Cfg {
-  static constexpr bool TF = H <= 64;                         // split issuers, tf32 second product
+  // H = 128 runs as two passes over 64-column halves of the state: pass hh contracts the band with
+  // columns 64 hh .. 64 hh + 63 of E and multiplies the result by rows 64 hh .. of W_p, into Y
+  static constexpr int NH = H / 64;
   static constexpr int C1 = band_chunks(S);                   // 128-column chunks per type
-  static constexpr int ATOM_X = H * 128;                      // 64 nodes x H rows
-  static constexpr int XWIN = 2 * C1 * ATOM_X;                // the window, 64-node atoms
+  static constexpr int ATOM_X = 64 * 128;                     // 64 nodes x 64 state columns
+  static constexpr int XWIN = 2 * C1 * ATOM_X;                // one half's window, 64-node atoms
   static constexpr int NXB = XWIN <= 48 * 1024 ? 2 : 1;       // state-window buffers
   static constexpr int NW = 2;                                // W ring stages
-  // H x H operand of the second product: fp32 (32 per 128-byte row) or bf16 (64 per row)
-  static constexpr int WSTAGE = (TF ? H / 32 : H / kAtom) * H * 128;
+  // one W stage: the 64 K-columns of one half of W_p^T as fp32 (tf32 operand), two 32-column
+  // atoms of H rows
+  static constexpr int WSTAGE = 2 * H * 128;
   static constexpr int DEG = kTile * 128;                     // 128 rows x 64 bf16
+  static constexpr int NDEG = NH > 1 ? 1 : 2;                 // deg buffers
   static constexpr int B2 = H * 128;                          // H rows x 64 bf16
   static constexpr int OFF_X = 0;
   static constexpr int OFF_W = OFF_X + NXB * XWIN;
   static constexpr int OFF_DEG = OFF_W + NW * WSTAGE;
-  static constexpr int OFF_B2 = OFF_DEG + 2 * DEG;
+  static constexpr int OFF_B2 = OFF_DEG + NDEG * DEG;
   static constexpr int MSTAGE = C1 * kTile * 16;              // C1 chunks x 128 rows x 128 bits
-  static constexpr int NM = H <= 64 ? (C1 <= 3 ? 8 : 4) : 2; // mask ring stages (one type each)
+  static constexpr int NM = (C1 <= 3 ? 8 : 4) / NH;           // mask ring stages (one job each)
   static constexpr int OFF_M = OFF_B2 + B2;
   static constexpr int OFF_BAR = OFF_M + NM * MSTAGE;
   static constexpr int SMEM = OFF_BAR + 1024 + 1024;          // barriers + 1 KB alignment slack
-  // TMEM columns: Y, NB pre_p buffers, then the A-tile slots
+  // TMEM columns: Y (H), two 64-column pre_p units used by the jobs (half, type) in turn, so that
+  // a job's band products overlap the previous job's W product, then the A-tile slots
   static constexpr int NB = 2;
   static constexpr int YCOL = 0;
   static constexpr int D1COL0 = H;
-  static constexpr int ACOL = (NB + 1) * H;
+  static constexpr int ACOL = H + NB * 64;
   static constexpr int NA = (512 - ACOL) / 64;
-  // H = 64: a type's chunks come in CG-chunk groups (one barrier wait each), G groups per type
+  // a job's chunks come in CG-chunk groups (one barrier wait each), G groups per job
   static constexpr int CG = C1 <= 3 ? C1 : 3;
   static constexpr int G = C1 / CG;
   static constexpr int NT = 8;                                // per-group barrier ring
-  // expander warpgroups: at H = 64 two, taking the edge types in turn
-  static constexpr int NE = TF ? 2 : 1;
+  static constexpr int NE = 2;                                // expander warpgroups
   static constexpr int THREADS = 128 * (2 + NE);
+  static_assert(H == 64 || H == 128, "state size");
   static_assert(C1 % CG == 0 && NT % G == 0, "chunk groups");
-  static_assert(NA >= 2 && NA <= 8, "A-slot ring");
-  static_assert(!TF || NA >= CG, "one group of A tiles must fit");
-  static_assert(NM <= 8, "mask ring");
+  static_assert(NA >= CG + 1 && NA <= 8, "one group of A tiles and one more must fit");
+  static_assert(NM >= 2 && NM <= 8, "mask ring");
   static_assert(SMEM <= 232448, "shared memory");
 };
 
@@ -111,8 +117,8 @@ struct Bars {
   uint64_t w_full[4], w_empty[4];
   uint64_t deg_full[2], deg_empty[2];
   uint64_t b2_full;
-  uint64_t a_full[8], a_empty[8];
-  uint64_t d1_full[4], pre_ready[4];
+  uint64_t a_empty[8];
+  uint64_t d1_full[4];
   uint64_t t_full[8];
   uint64_t y_full, y_empty;
   uint64_t m_full[8], m_empty[8];
@@ -174,9 +180,12 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
   uint8_t* b2s = smem + C::OFF_B2;
   uint8_t* mring = smem + C::OFF_M;
   volatile int* abort = &bars->abort;
-  // releases of a pre_p buffer, which also complete the first group of a type (H = 64): the second
-  // issuer's commit and, backward, the 4 converter warps; every group also needs 4 expander warps
+  // A job is one (half, type) of a tile, in the order tile, half, type; job c writes pre_p unit
+  // c % 2.  Chunk group gi = G c + g waits on t_full[gi % NT]: the 4 warps of the expander group
+  // once its A tiles are in TMEM, and for first groups (g = 0) the release of the unit: the second
+  // issuer's commit and, backward, the 4 converter warps.
   constexpr int kFree = 1 + (BWD ? 4 : 0);
+  const int jobs = C::NH * P;  // per tile
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -184,10 +193,9 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
       mbar_init(&bars->x_full[i], 1); mbar_init(&bars->x_empty[i], 1);
       mbar_init(&bars->deg_full[i], 1); mbar_init(&bars->deg_empty[i], 1);
     }
-    for (int i = 0; i < 4; ++i) { mbar_init(&bars->d1_full[i], 1); mbar_init(&bars->pre_ready[i], 4); }
+    for (int i = 0; i < 4; ++i) mbar_init(&bars->d1_full[i], 1);
     for (int i = 0; i < 4; ++i) { mbar_init(&bars->w_full[i], 1); mbar_init(&bars->w_empty[i], 1); }
-    for (int i = 0; i < 8; ++i) { mbar_init(&bars->a_full[i], 4); mbar_init(&bars->a_empty[i], 1); }
-    // group gi = G c + j of type c sits in slot gi % NT; first groups (j = 0) also take the release
+    for (int i = 0; i < 8; ++i) mbar_init(&bars->a_empty[i], 1);
     for (int i = 0; i < 8; ++i) mbar_init(&bars->t_full[i], 4 + (i % C::G == 0 ? kFree : 0));
     mbar_init(&bars->b2_full, 1);
     mbar_init(&bars->y_full, 1);
@@ -197,11 +205,9 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     for (int i = 0; i < 8; ++i) { mbar_init(&bars->m_full[i], 1); mbar_init(&bars->m_empty[i], 4); }
     bars->abort = 0;
     fence_mbar_init();
-    if (C::TF) {
-      // the first NB types find their pre_p buffer free: stand in for the releases
-      for (int c = 0; c < C::NB; ++c)
-        for (int a = 0; a < kFree; ++a) mbar_arrive(&bars->t_full[(c * C::G) % C::NT]);
-    }
+    // the first NB jobs find their pre_p unit free: stand in for the releases
+    for (int c = 0; c < C::NB; ++c)
+      for (int a = 0; a < kFree; ++a) mbar_arrive(&bars->t_full[(c * C::G) % C::NT]);
   }
   if (warp == 1) {
     tmem_alloc(&bars->tmem_base, 512);
@@ -225,35 +231,45 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     }
     // the state windows are the previous kernel's output (bit tiles, W, deg and b2 are not)
     grid_dep_wait();
-    uint32_t widx = 0;
+    uint32_t widx = 0, xi = 0;
     uint32_t n_x[2] = {0, 0}, n_deg[2] = {0, 0}, n_w[4] = {0, 0, 0, 0};
     int i = 0;
-    for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x, ++i) {
-      const int xb = i % C::NXB;
-      if (!mbar_wait(&bars->x_empty[xb], ((i / C::NXB) & 1) ^ 1, status, 101, abort, 64)) break;
-      ++n_x[xb];
-      // window rows ws .. ws + 128 C1; rows outside [0, n) arrive as zeros (TMA bounds fill)
+    bool ok = true;
+    for (int k = blockIdx.x; k < n_tiles && ok && !*abort; k += gridDim.x, ++i) {
       const int row0 = k * kTile, ws = (row0 / S) * S - S;
-      mbar_expect_tx(&bars->x_full[xb], C::XWIN);
-      for (int a = 0; a < 2 * C::C1; ++a)
-        tma_load_2d(xwin + xb * C::XWIN + a * C::ATOM_X, &tm_x, &bars->x_full[xb], ws + a * kAtom, 0);
       if (has_bias) {
-        const int db = i & 1;
-        if (!mbar_wait(&bars->deg_empty[db], ((i >> 1) & 1) ^ 1, status, 102, abort, 64)) break;
+        const int db = i % C::NDEG;
+        if (!mbar_wait(&bars->deg_empty[db], ((i / C::NDEG) & 1) ^ 1, status, 102, abort, 64)) break;
         ++n_deg[db];
         mbar_expect_tx(&bars->deg_full[db], C::DEG);
         tma_load_2d(degs + db * C::DEG, &tm_deg, &bars->deg_full[db], 0, row0);
       }
-      for (int p = 0; p < P; ++p, ++widx) {
-        const int ws2 = widx % C::NW;
-        if (!mbar_wait(&bars->w_empty[ws2], ((widx / C::NW) & 1) ^ 1, status, 103, abort, 64)) break;
-        ++n_w[ws2];
-        mbar_expect_tx(&bars->w_full[ws2], C::WSTAGE);
-        // atoms of 128-byte rows along K: 32 fp32 (tf32 operand) or 64 bf16 each
-        constexpr int kw = C::TF ? 32 : kAtom;
-        for (int a = 0; a < H / kw; ++a)
-          tma_load_2d(wring + ws2 * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws2], a * kw,
-                      p * H);
+      for (int hh = 0; hh < C::NH && ok; ++hh, ++xi) {
+        // window rows ws .. ws + 128 C1 of state columns 64 hh ..; rows outside [0, n) arrive as
+        // zeros (TMA bounds fill)
+        const int xb = xi % C::NXB;
+        if (!mbar_wait(&bars->x_empty[xb], ((xi / C::NXB) & 1) ^ 1, status, 101, abort, 64)) {
+          ok = false;
+          break;
+        }
+        ++n_x[xb];
+        mbar_expect_tx(&bars->x_full[xb], C::XWIN);
+        for (int a = 0; a < 2 * C::C1; ++a)
+          tma_load_2d(xwin + xb * C::XWIN + a * C::ATOM_X, &tm_x, &bars->x_full[xb],
+                      ws + a * kAtom, 64 * hh);
+        // one W stage per job: K-columns 64 hh .. 64 hh + 63 of W_p^T, two 32-column atoms
+        for (int p = 0; p < P; ++p, ++widx) {
+          const int ws2 = widx % C::NW;
+          if (!mbar_wait(&bars->w_empty[ws2], ((widx / C::NW) & 1) ^ 1, status, 103, abort, 64)) {
+            ok = false;
+            break;
+          }
+          ++n_w[ws2];
+          mbar_expect_tx(&bars->w_full[ws2], C::WSTAGE);
+          for (int a = 0; a < 2; ++a)
+            tma_load_2d(wring + ws2 * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws2],
+                        64 * hh + 32 * a, p * H);
+        }
       }
     }
     if (*abort) {
@@ -269,11 +285,13 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     }
   } else if (warp == 2 && lane == 0) {
     // ------------------------------------------------------------------ mask producer
-    // each type's C1 bit chunks (contiguous [C1][128][4] words), NM types ahead of the expanders
+    // each job's C1 bit chunks (contiguous [C1][128][4] words of its type), NM jobs ahead of the
+    // expanders; both halves of a tile read the same bits
     uint32_t midx = 0, n_m[8] = {0};
     for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x) {
       bool ok = true;
-      for (int p = 0; p < P; ++p, ++midx) {
+      for (int jb = 0; jb < jobs; ++jb, ++midx) {
+        const int p = jb % P;
         const int ms = midx % C::NM;
         if (!mbar_wait(&bars->m_empty[ms], ((midx / C::NM) & 1) ^ 1, status, 104, abort, 64)) {
           ok = false;
@@ -290,80 +308,82 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
       for (int q = 0; q < 8; ++q)
         for (uint32_t t = 0; n_m[q] && t < (1u << 22) && !mbar_try(&bars->m_full[q], (n_m[q] - 1) & 1); ++t) {
         }
-  } else if (warp == 1 && C::TF) {
+  } else if (warp == 1) {
     // ------------------------------------------------------------------ band-product issuer
-    // pre_p = sum over the window chunks of A_{tile,p,j} X_j: one t_full wait per group of chunks,
-    // then an unbroken MMA stream
+    // pre_p = sum over the window chunks of A_{tile,p,j} X_j (N = 64): one t_full wait per group
+    // of chunks, then an unbroken MMA stream
     const bool leader = elect_one_sync();
-    constexpr uint32_t idesc = idesc_bf16_f32(kTile, H);
-    uint32_t c = 0, slot = 0, gi = 0;
+    constexpr uint32_t idesc = idesc_bf16_f32(kTile, 64);
+    uint32_t c = 0, slot = 0, gi = 0, xi = 0;
     bool ok = true;
-    int i = 0;
-    for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x, ++i) {
-      const int xb = i % C::NXB;
-      if (!mbar_wait(&bars->x_full[xb], (i / C::NXB) & 1, status, 204, abort)) break;
-      // descriptors differ from the window's first one only in the start-address field
-      const uint64_t xdesc = desc_sw128_kmajor(smem_u32(xwin + xb * C::XWIN));
-      for (int p = 0; p < P && ok; ++p, ++c) {
-        const uint32_t d1 = tmem + C::D1COL0 + (c % C::NB) * H;
-        for (int g = 0; g < C::G; ++g, ++gi) {
-          if (!mbar_wait(&bars->t_full[gi % C::NT], (gi / C::NT) & 1, status, 210, abort)) { ok = false; break; }
-          tc_fence_after();
-          for (int j = g * C::CG; j < (g + 1) * C::CG; ++j) {
-            const uint32_t a = tmem + C::ACOL + slot * 64;
-            const uint64_t jdesc = xdesc + (uint64_t)((2 * j * C::ATOM_X) >> 4);
+    for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x) {
+      for (int hh = 0; hh < C::NH && ok; ++hh, ++xi) {
+        const int xb = xi % C::NXB;
+        if (!mbar_wait(&bars->x_full[xb], (xi / C::NXB) & 1, status, 204, abort)) { ok = false; break; }
+        // descriptors differ from the window's first one only in the start-address field
+        const uint64_t xdesc = desc_sw128_kmajor(smem_u32(xwin + xb * C::XWIN));
+        for (int p = 0; p < P && ok; ++p, ++c) {
+          const uint32_t d1 = tmem + C::D1COL0 + (c % C::NB) * 64;
+          for (int g = 0; g < C::G; ++g, ++gi) {
+            if (!mbar_wait(&bars->t_full[gi % C::NT], (gi / C::NT) & 1, status, 210, abort)) { ok = false; break; }
+            tc_fence_after();
+            for (int j = g * C::CG; j < (g + 1) * C::CG; ++j) {
+              const uint32_t a = tmem + C::ACOL + slot * 64;
+              const uint64_t jdesc = xdesc + (uint64_t)((2 * j * C::ATOM_X) >> 4);
 #pragma unroll
-            for (int kk = 0; kk < kTile / 16; ++kk)
-              if (leader)
-                mma_ts(d1, a + kk * 8, jdesc + (uint64_t)(((kk / 4) * C::ATOM_X + (kk % 4) * 32) >> 4),
-                       idesc, (j == 0 && kk == 0) ? 0u : 1u);
-            if (leader) tc_commit(&bars->a_empty[slot]);
-            slot = slot + 1 == (uint32_t)C::NA ? 0 : slot + 1;
+              for (int kk = 0; kk < kTile / 16; ++kk)
+                if (leader)
+                  mma_ts(d1, a + kk * 8, jdesc + (uint64_t)(((kk / 4) * C::ATOM_X + (kk % 4) * 32) >> 4),
+                         idesc, (j == 0 && kk == 0) ? 0u : 1u);
+              if (leader) tc_commit(&bars->a_empty[slot]);
+              slot = slot + 1 == (uint32_t)C::NA ? 0 : slot + 1;
+            }
           }
+          if (!ok) break;
+          if (leader) tc_commit(&bars->d1_full[c % C::NB]);
+          if (p == P - 1 && leader) tc_commit(&bars->x_empty[xb]);
         }
-        if (!ok) break;
-        if (leader) tc_commit(&bars->d1_full[c % C::NB]);
-        if (p == P - 1 && leader) tc_commit(&bars->x_empty[xb]);
       }
     }
     drain_mmas(leader, &bars->drain);
-  } else if (warp == 3 && C::TF) {
+  } else if (warp == 3) {
     // ------------------------------------------------------------------ second issuer
-    // Y (+)= pre_p W_p (kind::tf32, A = the fp32 pre_p in TMEM) and the bias product
+    // Y (+)= pre_p W_p over the jobs (kind::tf32, A = the fp32 pre_p unit in TMEM, K = the 64 rows
+    // of W_p of the job's half), then the bias product
     const bool leader = elect_one_sync();
     constexpr uint32_t idesc = idesc_bf16_f32(kTile, H);
     constexpr uint32_t idesc2 = idesc_tf32_f32(kTile, H);
-    uint32_t c = 0, widx = 0;
+    uint32_t c = 0;
     bool ok = true;
     int i = 0;
     for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x, ++i) {
-      for (int p = 0; p < P; ++p, ++c, ++widx) {
+      for (int jb = 0; jb < jobs; ++jb, ++c) {
         const int b = c % C::NB;
-        const int ws = widx % C::NW;
+        const int ws = c % C::NW;
         if (!mbar_wait(&bars->d1_full[b], (c / C::NB) & 1, status, 208, abort) ||
-            !mbar_wait(&bars->w_full[ws], (widx / C::NW) & 1, status, 202, abort) ||
-            (p == 0 && !mbar_wait(&bars->y_empty, (i & 1) ^ 1, status, 203, abort))) {
+            !mbar_wait(&bars->w_full[ws], (c / C::NW) & 1, status, 202, abort) ||
+            (jb == 0 && !mbar_wait(&bars->y_empty, (i & 1) ^ 1, status, 203, abort))) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t wbase = smem_u32(wring + ws * C::WSTAGE);
 #pragma unroll
-        for (int kk = 0; kk < H / 8; ++kk) {
+        for (int kk = 0; kk < 8; ++kk) {
           const uint64_t bdesc = desc_sw128_kmajor(wbase + (kk / 4) * H * 128 + (kk % 4) * 32);
-          if (leader) mma_ts_tf32(tmem + C::YCOL, tmem + C::D1COL0 + b * H + kk * 8, bdesc, idesc2,
-                                  (p == 0 && kk == 0) ? 0u : 1u);
+          if (leader) mma_ts_tf32(tmem + C::YCOL, tmem + C::D1COL0 + b * 64 + kk * 8, bdesc, idesc2,
+                                  (jb == 0 && kk == 0) ? 0u : 1u);
         }
         if (leader) {
           tc_commit(&bars->w_empty[ws]);
-          // this pre_p buffer is free again: part of type c + NB's first group
+          // this unit is free again: part of job c + NB's first group
           tc_commit(&bars->t_full[((c + C::NB) * C::G) % C::NT]);
         }
       }
       if (!ok) break;
       if (has_bias) {
-        const int db = i & 1;
-        if (!mbar_wait(&bars->deg_full[db], (i >> 1) & 1, status, 206, abort)) break;
+        const int db = i % C::NDEG;
+        if (!mbar_wait(&bars->deg_full[db], (i / C::NDEG) & 1, status, 206, abort)) break;
         if (i == 0 && !mbar_wait(&bars->b2_full, 0, status, 207, abort)) break;
         tc_fence_after();
         const uint32_t dbase = smem_u32(degs + db * C::DEG), bbase = smem_u32(b2s);
@@ -376,94 +396,18 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
       if (leader) tc_commit(&bars->y_full);
     }
     drain_mmas(leader, &bars->drain2);
-  } else if (warp == 1) {
-    // ------------------------------------------------------------------ MMA issuer (H = 128)
-    // the whole warp runs this loop (its operands stay warp-uniform); one elected lane issues
-    const bool leader = elect_one_sync();
-    constexpr uint32_t idesc = idesc_bf16_f32(kTile, H);
-    uint32_t c = 0, aidx = 0, widx = 0;
-    bool ok = true;
-    int i = 0;
-    // second product of type cc: Y (+)= bf16(pre_cc) W_cc, after the converters rounded pre_cc
-    auto stage2 = [&](uint32_t cc, bool first_in_tile, int tile_i) -> bool {
-      const int b = cc % C::NB;
-      if (!mbar_wait(&bars->pre_ready[b], (cc / C::NB) & 1, status, 201, abort)) return false;
-      const int ws = widx % C::NW;
-      if (!mbar_wait(&bars->w_full[ws], (widx / C::NW) & 1, status, 202, abort)) return false;
-      if (first_in_tile &&
-          !mbar_wait(&bars->y_empty, (tile_i & 1) ^ 1, status, 203, abort))
-        return false;
-      tc_fence_after();
-      const uint32_t wbase = smem_u32(wring + ws * C::WSTAGE);
-#pragma unroll
-      for (int kk = 0; kk < H / 16; ++kk) {
-        const uint64_t bdesc = desc_sw128_kmajor(wbase + (kk / 4) * H * 128 + (kk % 4) * 32);
-        if (leader) mma_ts(tmem + C::YCOL, tmem + C::D1COL0 + b * H + kk * 8, bdesc, idesc,
-               (first_in_tile && kk == 0) ? 0u : 1u);
-      }
-      if (leader) tc_commit(&bars->w_empty[ws]);
-      ++widx;
-      return true;
-    };
-    constexpr int LAG = C::NB - 1;  // stage 2 of type p - LAG follows stage 1 of type p
-    for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x, ++i) {
-      const int xb = i % C::NXB;
-      if (!mbar_wait(&bars->x_full[xb], (i / C::NXB) & 1, status, 204, abort)) break;
-      tc_fence_after();
-      const uint32_t xbase = smem_u32(xwin + xb * C::XWIN);
-      const uint32_t c0 = c;
-      int next_s2 = 0;
-      for (int p = 0; p < P && ok; ++p, ++c) {
-        const int b = c % C::NB;
-        for (int j = 0; j < C::C1; ++j) {
-          const int slot = aidx % C::NA;
-          if (!mbar_wait(&bars->a_full[slot], (aidx / C::NA) & 1, status, 205, abort)) { ok = false; break; }
-          tc_fence_after();
-#pragma unroll
-          for (int kk = 0; kk < kTile / 16; ++kk) {
-            const uint64_t bdesc =
-                desc_sw128_kmajor(xbase + (2 * j + kk / 4) * C::ATOM_X + (kk % 4) * 32);
-            if (leader) mma_ts(tmem + C::D1COL0 + b * H, tmem + C::ACOL + slot * 64 + kk * 8, bdesc, idesc,
-                   (j == 0 && kk == 0) ? 0u : 1u);
-          }
-          if (leader) tc_commit(&bars->a_empty[slot]);
-          ++aidx;
-        }
-        if (!ok) break;
-        if (leader) tc_commit(&bars->d1_full[b]);
-        if (p == P - 1) if (leader) tc_commit(&bars->x_empty[xb]);
-        for (; ok && next_s2 <= p - LAG; ++next_s2)
-          if (!stage2(c0 + next_s2, next_s2 == 0, i)) ok = false;
-      }
-      for (; ok && next_s2 < P; ++next_s2)
-        if (!stage2(c0 + next_s2, next_s2 == 0, i)) ok = false;
-      if (!ok) break;
-      if (has_bias) {
-        const int db = i & 1;
-        if (!mbar_wait(&bars->deg_full[db], (i >> 1) & 1, status, 206, abort)) break;
-        if (i == 0 && !mbar_wait(&bars->b2_full, 0, status, 207, abort)) break;
-        tc_fence_after();
-        const uint32_t dbase = smem_u32(degs + db * C::DEG), bbase = smem_u32(b2s);
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk)
-          if (leader) mma_ss(tmem + C::YCOL, desc_sw128_kmajor(dbase + kk * 32),
-                 desc_sw128_kmajor(bbase + kk * 32), idesc, 1u);
-        if (leader) tc_commit(&bars->deg_empty[db]);
-      }
-      if (leader) tc_commit(&bars->y_full);
-    }
-    drain_mmas(leader, &bars->drain);
   } else if (warp >= 4 && warp < 4 + 4 * C::NE) {
     // ------------------------------------------------------------------ expanders
+    // the two groups take the jobs in turn
     const int eg = (warp - 4) / 4;
     const int r = (threadIdx.x - 128) % 128;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     uint32_t aidx = 0, midx = 0;
     for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x) {
       bool ok = true;
-      for (int p = 0; p < P && ok; ++p, ++midx) {
-        if (C::NE > 1 && (int)(midx % C::NE) != eg) {
-          aidx += C::C1;  // the other group's type
+      for (int jb = 0; jb < jobs && ok; ++jb, ++midx) {
+        if ((int)(midx % C::NE) != eg) {
+          aidx += C::C1;  // the other group's job
           continue;
         }
         const int ms = midx % C::NM;
@@ -487,11 +431,7 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
           expand_word(m.z, v);
           expand_word(m.w, v + 16);
           tmem_st32(tmem + lane_base + C::ACOL + slot * 64 + 32, v);
-          if (!C::TF) {
-            tmem_wait_st();
-            tc_fence_before();
-            warp_arrive(&bars->a_full[slot]);
-          } else if ((j + 1) % C::CG == 0) {
+          if ((j + 1) % C::CG == 0) {
             // all of this group's A tiles are in TMEM
             tmem_wait_st();
             tc_fence_before();
@@ -515,47 +455,32 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x, ++i) {
       const int row = k * kTile + r;
       bool ok = true;
-      for (int p = 0; p < P && (BWD || !C::TF); ++p, ++c) {
-        const int b = c % C::NB;
+      for (int jb = 0; BWD && jb < jobs; ++jb, ++c) {
+        const int b = c % C::NB, p = jb % P, hh = jb / P;
         if (!mbar_wait(&bars->d1_full[b], (c / C::NB) & 1, status, 401, abort, 64)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t col = tmem + lane_base + C::D1COL0 + b * H;
+        const uint32_t col = tmem + lane_base + C::D1COL0 + b * 64;
+        uint32_t v[32], w[32];
+        tmem_ld32(col, v);
+        tmem_ld32(col + 32, w);
+        tmem_wait_ld();
+        // pre_p stays fp32 for the tf32 product: release the unit before the stores
+        tc_fence_before();
+        warp_arrive(&bars->t_full[((c + C::NB) * C::G) % C::NT]);
+        uint32_t pk[32];
 #pragma unroll
-        for (int h0 = 0; h0 < H; h0 += 64) {
-          uint32_t v[32], q[32];
-          tmem_ld32(col + h0, v);
-          tmem_ld32(col + h0 + 32, q);
-          tmem_wait_ld();
-          uint32_t pk[32];
+        for (int j = 0; j < 16; ++j)
+          pk[j] = pack_bf16(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
 #pragma unroll
-          for (int j = 0; j < 16; ++j)
-            pk[j] = pack_bf16(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+        for (int j = 0; j < 16; ++j)
+          pk[16 + j] = pack_bf16(__uint_as_float(w[2 * j]), __uint_as_float(w[2 * j + 1]));
+        // dM_p (bf16) transposed: dMT[(p*H + h) * ld_mt + row]
 #pragma unroll
-          for (int j = 0; j < 16; ++j)
-            pk[16 + j] = pack_bf16(__uint_as_float(q[2 * j]), __uint_as_float(q[2 * j + 1]));
-          if (C::TF) {
-            // pre_p stays fp32 for the tf32 product: release the buffer before the stores
-            tc_fence_before();
-            warp_arrive(&bars->t_full[((c + C::NB) * C::G) % C::NT]);
-          } else {
-            // packed pairs of columns h0..h0+63 go to columns (h0/2)..(h0/2)+31 of the buffer
-            tmem_st32(col + h0 / 2, pk);
-          }
-          if (BWD) {
-            // dM_p (bf16) transposed: dMT[(p*H + h) * ld_mt + row]
-#pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              const uint32_t w2 = pk[j];
-              __nv_bfloat16* d = dMT + ((size_t)p * H + h0 + 2 * j) * ld_mt + row;
-              d[0] = __ushort_as_bfloat16((unsigned short)(w2 & 0xFFFFu));
-              d[ld_mt] = __ushort_as_bfloat16((unsigned short)(w2 >> 16));
-            }
-          }
-        }
-        if (!C::TF) {
-          tmem_wait_st();
-          tc_fence_before();
-          warp_arrive(&bars->pre_ready[b]);
+        for (int j = 0; j < 32; ++j) {
+          const uint32_t w2 = pk[j];
+          __nv_bfloat16* d = dMT + ((size_t)p * H + 64 * hh + 2 * j) * ld_mt + row;
+          d[0] = __ushort_as_bfloat16((unsigned short)(w2 & 0xFFFFu));
+          d[ld_mt] = __ushort_as_bfloat16((unsigned short)(w2 >> 16));
         }
       }
       if (!ok) break;
@@ -646,19 +571,14 @@ __global__ void k_transpose_bf16(const T* __restrict__ in, __nv_bfloat16* __rest
 // Second-product weights in the band kernel's operand layout, for each type p:
 //   forward  out[p][o][i] = W[p][i][o]   (W_p^T, K-major in i)
 //   backward out[p][i][o] = W[p][i][o]   (W_p as given, K-major in o)
-// as fp32 (tf32 product) or bf16.
-template <typename TO>
-__global__ void k_prep_w(const __nv_bfloat16* __restrict__ W, TO* __restrict__ out, int P, int H,
+// as fp32 (the tf32 product's B operand).
+__global__ void k_prep_w(const __nv_bfloat16* __restrict__ W, float* __restrict__ out, int P, int H,
                          int transpose) {
   const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= (int64_t)P * H * H) return;
   const int64_t p = t / ((int64_t)H * H);
   const int a = (int)((t / H) % H), c = (int)(t % H);
-  const float v = __bfloat162float(transpose ? W[(p * H + c) * H + a] : W[(p * H + a) * H + c]);
-  if constexpr (sizeof(TO) == 4)
-    out[t] = v;
-  else
-    out[t] = __float2bfloat16_rn(v);
+  out[t] = __bfloat162float(transpose ? W[(p * H + c) * H + a] : W[(p * H + a) * H + c]);
 }
 
 // b2T[h][p] = bf16 hi part of b[p][h], b2T[h][32 + p] = bf16 of the remainder (zero beyond P)
@@ -695,10 +615,9 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, ui
   return make_map_ld(m, base, rows, cols, cols, box_rows);
 }
 
-// The W map of the band kernel: fp32 for the tf32 second product (H = 64), bf16 otherwise.
+// The W map of the band kernel: fp32 (the tf32 second product), boxes of 32 columns x H rows.
 bool make_map_w(CUtensorMap* m, const void* Wk, int P, int H) {
-  if (H <= 64) return make_map_f32(m, Wk, (uint64_t)P * H, H, H);
-  return make_map(m, Wk, (uint64_t)P * H, H, H);
+  return make_map_f32(m, Wk, (uint64_t)P * H, H, H);
 }
 
 int num_sms() {
@@ -733,7 +652,7 @@ cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap&
   return e;
 }
 
-// The shapes with a tensor-core kernel: H = 64 at S in {32, 64, 128, 256}; H = 128 at S = 128.
+// The shapes with a tensor-core kernel: H in {64, 128} at S in {32, 64, 128, 256}.
 template <int H, bool BWD>
 cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
                    const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
@@ -743,15 +662,11 @@ cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& t
 #define BG_BAND_S(SV)                                                                            \
   return launch_s<H, SV, BWD>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, dMT, ld_mt,      \
                               has_bias, accumulate, status, st);
-  if constexpr (H == 64) {
-    switch (p->S) {
-      case 32: BG_BAND_S(32)
-      case 64: BG_BAND_S(64)
-      case 256: BG_BAND_S(256)
-      default: BG_BAND_S(128)
-    }
-  } else {
-    BG_BAND_S(128)
+  switch (p->S) {
+    case 32: BG_BAND_S(32)
+    case 64: BG_BAND_S(64)
+    case 256: BG_BAND_S(256)
+    default: BG_BAND_S(128)
   }
 #undef BG_BAND_S
 }
@@ -805,14 +720,14 @@ bool make_map_3d(CUtensorMap* m, const void* base, uint64_t batch, uint64_t rows
 
 bool band_tc_supported(const bg_plan* p, int dtype, int H) {
   if (!p || dtype != 1 || p->P > 32 || p->n_pad() % kTile) return false;
-  const bool shape = (H == 64 && (p->S == 32 || p->S == 64 || p->S == 128 || p->S == 256)) ||
-                     (H == 128 && p->S == 128);
+  const bool shape = (H == 64 || H == 128) &&
+                     (p->S == 32 || p->S == 64 || p->S == 128 || p->S == 256);
   return shape && p->d_maskI && p->d_maskTI && p->d_deg2 && p->max_deg <= 256 &&
          encode_fn() != nullptr;
 }
 
 size_t band_tc_w_bytes(const bg_plan* p, int H) {
-  return al256((size_t)p->P * H * H * (H <= 64 ? 4 : 2));
+  return al256((size_t)p->P * H * H * 4);
 }
 
 cudaError_t band_tc_prep_w(const bg_plan* p, int H, const void* W, int bwd, void* Wk,
@@ -820,11 +735,7 @@ cudaError_t band_tc_prep_w(const bg_plan* p, int H, const void* W, int bwd, void
   const int64_t n = (int64_t)p->P * H * H;
   const int blocks = (int)((n + 255) / 256);
   const auto* w = static_cast<const __nv_bfloat16*>(W);
-  if (H <= 64)
-    k_prep_w<float><<<blocks, 256, 0, st>>>(w, static_cast<float*>(Wk), p->P, H, !bwd);
-  else
-    k_prep_w<__nv_bfloat16><<<blocks, 256, 0, st>>>(w, static_cast<__nv_bfloat16*>(Wk), p->P, H,
-                                                    !bwd);
+  k_prep_w<<<blocks, 256, 0, st>>>(w, static_cast<float*>(Wk), p->P, H, !bwd);
   note_launch();
   return cudaGetLastError();
 }
@@ -849,7 +760,7 @@ cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, i
                              int* status, cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw, tdeg, tb2;
-  if (!make_map_ld(&tx, XT, H, n, ld_x, H) || !make_map_w(&tw, Wk, P, H) ||
+  if (!make_map_ld(&tx, XT, H, n, ld_x, 64) || !make_map_w(&tw, Wk, P, H) ||
       !make_map(&tdeg, p->d_deg2, n, 64, kTile) || !make_map(&tb2, b2T ? b2T : XT, H, 64, H))
     return cudaErrorInvalidValue;
   const int has_bias = b2T != nullptr;
@@ -865,7 +776,7 @@ cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, 
                              int64_t ld_mt, int* status, cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw;
-  if (!make_map_ld(&tx, dYT, H, n, ld_y, H) || !make_map_w(&tw, Wk, P, H))
+  if (!make_map_ld(&tx, dYT, H, n, ld_y, 64) || !make_map_w(&tw, Wk, P, H))
     return cudaErrorInvalidValue;
   if (H == 64)
     return launch<64, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,

@@ -20,8 +20,7 @@ cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, c
                         float* dE, float* dW, float* db, int accum, char* ws, size_t ws_bytes,
                         int* status, cudaStream_t st);
 // The band kernel's second-product weights (band_tc_w_bytes): from W [P][H][H] bf16, the forward
-// operand W_p^T (bwd = 0) or the backward operand W_p (bwd = 1), fp32 at H = 64 (kind::tf32
-// product) and bf16 at H = 128.
+// operand W_p^T (bwd = 0) or the backward operand W_p (bwd = 1), fp32 (kind::tf32 product).
 size_t band_tc_w_bytes(const bg_plan* p, int H);
 cudaError_t band_tc_prep_w(const bg_plan* p, int H, const void* W, int bwd, void* Wk,
                            cudaStream_t st);
