@@ -436,11 +436,11 @@ size_t saved_Y_off(const bg_plan* p, bg_dtype dt, int H, int T, int t) {
   return saved_E_off(p, dt, H, T + 1) + (size_t)t * al(sizeof(float) * (size_t)p->n_pad() * H);
 }
 
-// ---- fused tensor-core GGNN steps (bf16, S = 128, H = 64, P <= 32)
-// Shapes of the fused GGNN path (tensor-core band and GRU kernels): bf16, H = 64, P <= 32, a block
-// size the band kernel has, whole 128-row tiles.
+// ---- fused tensor-core GGNN steps (bf16, H in {64, 128}, P <= 32)
+// Shapes of the fused GGNN path (tensor-core band and GRU kernels): bf16, H in {64, 128},
+// P <= 32, a block size the band kernel has, whole 128-row tiles.
 bool tc_shape(const bg_plan* p, bg_dtype dt, int H) {
-  return p && dt == BG_BF16 && H == 64 && p->P <= 32 &&
+  return p && dt == BG_BF16 && (H == 64 || H == 128) && p->P <= 32 &&
          (p->S == 32 || p->S == 64 || p->S == 128 || p->S == 256) && p->n_pad() % 128 == 0;
 }
 bool tc_ggnn(const bg_plan* p, bg_dtype dt, int H) {
@@ -777,7 +777,7 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
       }
       KTimer tm(BG_KID_GRU_FWD, st);
       BG_CUDA(bg::gru_fwd_tc(
-          (int)n, p->n_real, Yi(t), Ei(t), static_cast<const __nv_bfloat16*>(prm->W_ih),
+          H, (int)n, p->n_real, Yi(t), Ei(t), static_cast<const __nv_bfloat16*>(prm->W_ih),
           static_cast<const __nv_bfloat16*>(prm->W_hh), prm->b_ih, prm->b_hh, Ei(t + 1),
           t + 1 < T ? ETa + (size_t)(t + 1) * n : nullptr, (int64_t)TN, status, st));
     }
@@ -857,7 +857,7 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     for (int t = T - 1; t >= 0; --t) {
       {
         KTimer tm(BG_KID_GRU_BWD, st);
-        BG_CUDA(bg::gru_bwd_tc((int)n, p->n_real, Yi(t), Ei(t), Wih, Whh, WihT, WhhT, prm->b_ih,
+        BG_CUDA(bg::gru_bwd_tc(H, (int)n, p->n_real, Yi(t), Ei(t), Wih, Whh, WihT, WhhT, prm->b_ih,
                                prm->b_hh, gin, g, dXT, (int64_t)n, dgiT + (size_t)t * n,
                                dghT + (size_t)t * n, (int64_t)TN, status, st));
       }

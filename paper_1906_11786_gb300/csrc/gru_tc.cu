@@ -528,51 +528,550 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+
+// ------------------------------------------------------------------------------------ H = 128
+// At H = 128, W_ih and W_hh (192 KB of bf16) do not fit in shared memory beside the tiles, so
+// these kernels stream them from L2 in pieces through a small TMA ring, and work on one 64-column
+// half of the state at a time (a job = (tile, half hh)): the gate pre-activations of the half's
+// columns h in [64 hh, 64 hh + 64) take 256 TMEM columns ([r|z] 128, Wi_n x 64, Wh_n h 64).
+//   gate piece (m, ka): rows {r, z, n} x [64 hh, +64) of W_m (m = ih, hh), K-columns [64 ka, +64):
+//                       192 rows x 128 B (three 64-row boxes), 24 KB
+//   backward piece (m, gate): W_m^T rows h' in [0, 128), K-columns gate*H + [64 hh, +64):
+//                       128 rows x 128 B, 16 KB
+namespace wide {
+
+constexpr int H = 128, NH = H / 64;
+constexpr int kTileB = 128 * H * 2;          // 128 rows x H bf16: NH 64-column atoms of 16 KB
+constexpr int kAtomB = 128 * 128;
+constexpr int kPiece = 192 * 128;            // ring slot (gate pieces; backward pieces use 16 KB)
+constexpr int kSlots = 3;
+constexpr int kGin = 128 * H * 4;            // 128 rows x H fp32 as 32-column boxes of 16 KB
+constexpr int kGates = 4 * 64;               // TMEM columns of one job's gate pre-activations
+
+struct Smem {
+  static constexpr int FWD_STAGE = 2 * kTileB;  // Y, E
+  static constexpr int FWD_PIECES = 2 * FWD_STAGE;
+  static constexpr int FWD = FWD_PIECES + kSlots * kPiece + 1024;
+  static constexpr int BWD_STAGE = 2 * kTileB + kGin;  // Y, E, incoming gradient (one stage)
+  static constexpr int BWD_PIECES = BWD_STAGE;
+  static constexpr int BWD = BWD_PIECES + kSlots * kPiece + 1024;
+  static_assert(FWD + 4096 <= 232448 && BWD + 4096 <= 232448, "shared memory");
+};
+
+struct Bars {
+  uint64_t t_full[2], t_empty[2], p_full[kSlots], p_empty[kSlots], g_full[2], g_empty[2];
+  uint64_t ops_ready, ph2_full, dx_empty, drain;
+  uint32_t tmem_slot;
+  int abort;
+};
+
+__device__ __forceinline__ void setup(Bars* b, float* bias, const float* b_ih, const float* b_hh,
+                                      int warp) {
+  for (int t = threadIdx.x; t < 3 * H; t += blockDim.x) {
+    bias[t] = b_ih[t];
+    bias[3 * H + t] = b_hh[t];
+  }
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&b->t_full[i], 1);
+      mbar_init(&b->t_empty[i], kEpiWarps);
+      mbar_init(&b->g_full[i], 1);
+      mbar_init(&b->g_empty[i], kEpiWarps);
+    }
+    for (int i = 0; i < kSlots; ++i) { mbar_init(&b->p_full[i], 1); mbar_init(&b->p_empty[i], 1); }
+    mbar_init(&b->ops_ready, kEpiWarps);
+    mbar_init(&b->ph2_full, 1);
+    mbar_init(&b->dx_empty, kEpiWarps);
+    mbar_init(&b->drain, 1);
+    b->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&b->tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  grid_dep_launch();
+}
+
+// Piece producer: for every job, the 2 NH gate pieces and (backward) the 6 backward pieces, in
+// the order the MMA issuer uses them.  The weights are not written by the kernels this one may
+// overlap under programmatic dependent launch (they change only between training steps).
+__device__ __forceinline__ void produce_pieces(Bars* b, uint8_t* ring, const CUtensorMap* tWih,
+                                               const CUtensorMap* tWhh, const CUtensorMap* tWihT,
+                                               const CUtensorMap* tWhhT, bool bwd, int n_tiles,
+                                               int* status, volatile int* abort) {
+  uint32_t pc = 0, issued[kSlots] = {0, 0, 0};
+  bool ok = true;
+  auto next = [&](int bytes) -> uint8_t* {
+    const int s = pc % kSlots;
+    if (!mbar_wait(&b->p_empty[s], ((pc / kSlots) & 1) ^ 1, status, 631, abort, 64)) return nullptr;
+    ++issued[s];
+    mbar_expect_tx(&b->p_full[s], bytes);
+    ++pc;
+    return ring + s * kPiece;
+  };
+  for (int t = blockIdx.x; t < n_tiles && ok && !*abort; t += gridDim.x) {
+    for (int hh = 0; hh < NH && ok; ++hh) {
+      for (int q = 0; q < 2 * NH && ok; ++q) {
+        const int m = q / NH, ka = q % NH, s = pc % kSlots;
+        uint8_t* dst = next(kPiece);
+        if (!dst) { ok = false; break; }
+        for (int g = 0; g < 3; ++g)
+          tma_load_2d(dst + g * 64 * 128, m ? tWhh : tWih, &b->p_full[s], 64 * ka, g * H + 64 * hh);
+      }
+      for (int q = 0; bwd && q < 6 && ok; ++q) {
+        const int m = q / 3, g = q % 3, s = pc % kSlots;
+        uint8_t* dst = next(128 * 128);
+        if (!dst) { ok = false; break; }
+        tma_load_2d(dst, m ? tWhhT : tWihT, &b->p_full[s], g * H + 64 * hh, 0);
+      }
+    }
+  }
+  if (*abort)
+    for (int s = 0; s < kSlots; ++s)
+      for (uint32_t k = 0; issued[s] && k < (1u << 22) && !mbar_try(&b->p_full[s], (issued[s] - 1) & 1); ++k) {
+      }
+}
+
+// Gate pre-activations of job (tile in `stage`, half hh) into TMEM columns g0 .. g0 + 255,
+// consuming 2 NH gate pieces.
+__device__ __forceinline__ bool gate_mmas(Bars* b, bool leader, uint32_t g0, uint32_t sY,
+                                          uint32_t sE, uint8_t* ring, uint32_t& pc, int* status,
+                                          volatile int* abort) {
+  constexpr uint32_t id_rz = idesc_bf16_f32(128, 128), id_n = idesc_bf16_f32(128, 64);
+  for (int q = 0; q < 2 * NH; ++q, ++pc) {
+    const int m = q / NH, ka = q % NH, s = pc % kSlots;
+    if (!mbar_wait(&b->p_full[s], (pc / kSlots) & 1, status, 632, abort)) return false;
+    tc_fence_after();
+    const uint32_t a0 = (m ? sE : sY) + ka * kAtomB, p0 = smem_u32(ring + s * kPiece);
+    if (leader) {
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+        const uint64_t ad = desc_sw128_kmajor(a0 + kk * 32);
+        mma_ss(g0, ad, desc_sw128_kmajor(p0 + kk * 32), id_rz, (q == 0 && kk == 0) ? 0u : 1u);
+        mma_ss(g0 + 128 + 64 * m, ad, desc_sw128_kmajor(p0 + 128 * 128 + kk * 32), id_n,
+               (ka == 0 && kk == 0) ? 0u : 1u);
+      }
+      tc_commit(&b->p_empty[s]);
+    }
+    __syncwarp();
+  }
+  return true;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_gru_fwd(const __grid_constant__ CUtensorMap tY, const __grid_constant__ CUtensorMap tE,
+              const __grid_constant__ CUtensorMap tWih, const __grid_constant__ CUtensorMap tWhh,
+              const float* __restrict__ b_ih, const float* __restrict__ b_hh,
+              __nv_bfloat16* __restrict__ En, __nv_bfloat16* __restrict__ EnT, int64_t ld_T,
+              int n_tiles, int n_real, int* status) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  __shared__ Bars bars;
+  __shared__ float bias[6 * H];
+  volatile int* abort = &bars.abort;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  setup(&bars, bias, b_ih, b_hh, warp);
+  const uint32_t tmem = bars.tmem_slot;
+  uint8_t* pieces = smem + Smem::FWD_PIECES;
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------------------ tile producer
+    grid_dep_wait();  // Y and E are the previous kernels' output
+    uint32_t issued[2] = {0, 0};
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles && !*abort; t += gridDim.x, ++i) {
+      const int s = i & 1;
+      if (!mbar_wait(&bars.t_empty[s], ((i >> 1) & 1) ^ 1, status, 633, abort, 64)) break;
+      ++issued[s];
+      uint8_t* st = smem + s * Smem::FWD_STAGE;
+      mbar_expect_tx(&bars.t_full[s], 2 * kTileB);
+      for (int a = 0; a < NH; ++a) {
+        tma_load_2d(st + a * kAtomB, &tY, &bars.t_full[s], 64 * a, t * 128);
+        tma_load_2d(st + kTileB + a * kAtomB, &tE, &bars.t_full[s], 64 * a, t * 128);
+      }
+    }
+    if (*abort)
+      for (int s = 0; s < 2; ++s)
+        for (uint32_t k = 0; issued[s] && k < (1u << 22) && !mbar_try(&bars.t_full[s], (issued[s] - 1) & 1); ++k) {
+        }
+  } else if (warp == 2 && lane == 0) {
+    produce_pieces(&bars, pieces, &tWih, &tWhh, nullptr, nullptr, false, n_tiles, status, abort);
+  } else if (warp == 1) {
+    // ------------------------------------------------------------------ MMA issuer
+    const bool leader = elect_one_sync();
+    uint32_t pc = 0, jn = 0;
+    bool ok = true;
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++i) {
+      const int s = i & 1;
+      if (!mbar_wait(&bars.t_full[s], (i >> 1) & 1, status, 634, abort)) break;
+      const uint32_t sY = smem_u32(smem + s * Smem::FWD_STAGE);
+      for (int hh = 0; hh < NH && ok; ++hh, ++jn) {
+        const int gb = jn & 1;
+        if (!mbar_wait(&bars.g_empty[gb], ((jn >> 1) & 1) ^ 1, status, 635, abort)) { ok = false; break; }
+        tc_fence_after();
+        if (!gate_mmas(&bars, leader, tmem + gb * kGates, sY, sY + kTileB, pieces, pc, status, abort)) {
+          ok = false;
+          break;
+        }
+        if (leader) tc_commit(&bars.g_full[gb]);
+        __syncwarp();
+      }
+    }
+    if (leader) tc_commit(&bars.drain);
+    __syncwarp();
+    for (uint32_t k = 0; k < (1u << 24) && !mbar_try(&bars.drain, 0); ++k) {
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------------------------ epilogue
+    grid_dep_wait();  // outputs may still be in use by the previous kernel
+    const int g = (warp - 4) / 4;
+    const int r = (warp & 3) * 32 + lane;
+    const uint32_t lb = (uint32_t)((warp & 3) * 32) << 16;
+    uint32_t jn = 0;
+    int i = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++i) {
+      const int s = i & 1;
+      const int row = t * 128 + r;
+      const bool real = row < n_real;
+      const uint8_t* etile = smem + s * Smem::FWD_STAGE + kTileB;
+      for (int hh = 0; hh < NH; ++hh, ++jn) {
+        const int gb = jn & 1;
+        if (!mbar_wait(&bars.g_full[gb], (jn >> 1) & 1, status, 636, abort, 64)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t acc = tmem + lb + gb * kGates;
+#pragma unroll
+        for (int h8 = 0; h8 < 2; ++h8) {
+          const int hs = 16 * g + 8 * h8, h = 64 * hh + hs;  // column within the half; global
+          uint32_t vr[8], vz[8], vn[8], vh[8];
+          tmem_ld8(acc + hs, vr);
+          tmem_ld8(acc + 64 + hs, vz);
+          tmem_ld8(acc + 128 + hs, vn);
+          tmem_ld8(acc + 192 + hs, vh);
+          tmem_wait_ld();
+          float e[8];
+          read_sw128_row8(etile, r, h, e);
+          if (h8 == 1) {
+            tc_fence_before();
+            warp_arrive(&bars.g_empty[gb]);
+            if (hh == NH - 1) warp_arrive(&bars.t_empty[s]);
+          }
+          uint32_t pk[4];
+#pragma unroll
+          for (int j = 0; j < 8; j += 2) {
+            float o[2];
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+              const int c = h + j + u;
+              const float rr = sigm(__uint_as_float(vr[j + u]) + bias[c] + bias[3 * H + c]);
+              const float zz = sigm(__uint_as_float(vz[j + u]) + bias[H + c] + bias[4 * H + c]);
+              const float nn = tanh_fast(__uint_as_float(vn[j + u]) + bias[2 * H + c] +
+                                         rr * (__uint_as_float(vh[j + u]) + bias[5 * H + c]));
+              o[u] = real ? (1.f - zz) * nn + zz * e[j + u] : 0.f;
+            }
+            pk[j / 2] = pk2(o[0], o[1]);
+          }
+          *reinterpret_cast<uint4*>(En + (size_t)row * H + h) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          if (EnT) store_T4(EnT, ld_T, row, h, pk);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// Backward.  TMEM: one job's gates (columns 0..255), dX (256..383) and dH (384..511), both
+// accumulated over the tile's two halves.  Per job: gate MMAs; the epilogue forms the gate
+// gradients of its columns and writes them back over the columns it read as the bf16 A operand
+// (window [16 g, +16) of r: dgi_r | dgi_z pairs; of z: dgi_n | dgh_n pairs; dgh_r = dgi_r,
+// dgh_z = dgi_z); then dX += dgi W_ih[half rows], dH += dgh W_hh[half rows] from the backward
+// pieces.  The next job's gate MMAs wait until those products have read the gradients.
+__global__ void __launch_bounds__(kThreads, 1)
+    k_gru_bwd(const __grid_constant__ CUtensorMap tY, const __grid_constant__ CUtensorMap tE,
+              const __grid_constant__ CUtensorMap tWih, const __grid_constant__ CUtensorMap tWhh,
+              const __grid_constant__ CUtensorMap tWihT, const __grid_constant__ CUtensorMap tWhhT,
+              const __grid_constant__ CUtensorMap tG, const float* __restrict__ b_ih,
+              const float* __restrict__ b_hh, float* __restrict__ gout,
+              __nv_bfloat16* __restrict__ dXT, int64_t ld_x, __nv_bfloat16* __restrict__ dgiT,
+              __nv_bfloat16* __restrict__ dghT, int64_t ld_g, int n_tiles, int n_real,
+              int* status) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  __shared__ Bars bars;
+  __shared__ float bias[6 * H];
+  volatile int* abort = &bars.abort;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  setup(&bars, bias, b_ih, b_hh, warp);
+  const uint32_t tmem = bars.tmem_slot;
+  uint8_t* pieces = smem + Smem::BWD_PIECES;
+  constexpr uint32_t kDX = kGates, kDH = kGates + H;
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------------------ tile producer (one stage)
+    grid_dep_wait();  // Y, E and the incoming gradient are earlier kernels' output
+    uint32_t issued = 0;
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles && !*abort; t += gridDim.x, ++i) {
+      if (!mbar_wait(&bars.t_empty[0], (i & 1) ^ 1, status, 641, abort, 64)) break;
+      ++issued;
+      mbar_expect_tx(&bars.t_full[0], Smem::BWD_STAGE);
+      for (int a = 0; a < NH; ++a) {
+        tma_load_2d(smem + a * kAtomB, &tY, &bars.t_full[0], 64 * a, t * 128);
+        tma_load_2d(smem + kTileB + a * kAtomB, &tE, &bars.t_full[0], 64 * a, t * 128);
+      }
+      for (int a = 0; a < H / 32; ++a)
+        tma_load_2d(smem + 2 * kTileB + a * kAtomB, &tG, &bars.t_full[0], 32 * a, t * 128);
+    }
+    if (*abort)
+      for (uint32_t k = 0; issued && k < (1u << 22) && !mbar_try(&bars.t_full[0], (issued - 1) & 1); ++k) {
+      }
+  } else if (warp == 2 && lane == 0) {
+    produce_pieces(&bars, pieces, &tWih, &tWhh, &tWihT, &tWhhT, true, n_tiles, status, abort);
+  } else if (warp == 1) {
+    // ------------------------------------------------------------------ MMA issuer
+    const bool leader = elect_one_sync();
+    constexpr uint32_t id_x = idesc_bf16_f32(128, H);
+    uint32_t pc = 0, jn = 0;
+    bool ok = true;
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++i) {
+      if (!mbar_wait(&bars.t_full[0], i & 1, status, 642, abort)) break;
+      const uint32_t sY = smem_u32(smem);
+      for (int hh = 0; hh < NH && ok; ++hh, ++jn) {
+        // the previous job's products have read the gate gradients out of columns 0..255
+        if (jn > 0 && !mbar_wait(&bars.ph2_full, (jn - 1) & 1, status, 643, abort)) { ok = false; break; }
+        tc_fence_after();
+        if (!gate_mmas(&bars, leader, tmem, sY, sY + kTileB, pieces, pc, status, abort)) {
+          ok = false;
+          break;
+        }
+        if (leader) tc_commit(&bars.g_full[0]);
+        __syncwarp();
+        if (!mbar_wait(&bars.ops_ready, jn & 1, status, 644, abort)) { ok = false; break; }
+        // dX and dH of the previous tile have been read out before the first job overwrites them
+        if (hh == 0 && i > 0 && !mbar_wait(&bars.dx_empty, (i - 1) & 1, status, 645, abort)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        for (int q = 0; q < 6; ++q, ++pc) {
+          const int m = q / 3, gate = q % 3, s = pc % kSlots;
+          if (!mbar_wait(&bars.p_full[s], (pc / kSlots) & 1, status, 646, abort)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t p0 = smem_u32(pieces + s * kPiece);
+          if (leader) {
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk) {
+              const uint32_t col = gate == 2 ? 64 + 16 * kk + 8 * m : 16 * kk + 8 * gate;
+              mma_ts(tmem + (m ? kDH : kDX), tmem + col, desc_sw128_kmajor(p0 + kk * 32), id_x,
+                     (hh == 0 && gate == 0 && kk == 0) ? 0u : 1u);
+            }
+            tc_commit(&bars.p_empty[s]);
+          }
+          __syncwarp();
+        }
+        if (!ok) break;
+        if (leader) tc_commit(&bars.ph2_full);
+        __syncwarp();
+      }
+    }
+    if (leader) tc_commit(&bars.drain);
+    __syncwarp();
+    for (uint32_t k = 0; k < (1u << 24) && !mbar_try(&bars.drain, 0); ++k) {
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------------------------ epilogue
+    grid_dep_wait();  // outputs may still be in use by the previous kernel
+    const int g = (warp - 4) / 4;
+    const int r = (warp & 3) * 32 + lane;
+    const uint32_t lb = (uint32_t)((warp & 3) * 32) << 16;
+    const uint8_t* etile = smem + kTileB;
+    const uint8_t* gtile = smem + 2 * kTileB;
+    uint32_t jn = 0;
+    int i = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++i) {
+      const int row = t * 128 + r;
+      const bool real = row < n_real;
+      for (int hh = 0; hh < NH; ++hh, ++jn) {
+        if (!mbar_wait(&bars.g_full[0], jn & 1, status, 647, abort, 64)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t acc = tmem + lb;
+        uint32_t p_r[8], p_z[8], p_n[8], p_hn[8];
+#pragma unroll
+        for (int h8 = 0; h8 < 2; ++h8) {
+          const int hs = 16 * g + 8 * h8, h = 64 * hh + hs;
+          float dhd[8];  // direct term z * dE(t+1), stored now and completed with dH below
+          uint32_t vr[8], vz[8], vn[8], vh[8];
+          tmem_ld8(acc + hs, vr);
+          tmem_ld8(acc + 64 + hs, vz);
+          tmem_ld8(acc + 128 + hs, vn);
+          tmem_ld8(acc + 192 + hs, vh);
+          tmem_wait_ld();
+          float e[8];
+          read_sw128_row8(etile, r, h, e);
+          float4 g4[2];
+          read_sw128_f32_row8(gtile, r, h, g4);
+          if (h8 == 1 && hh == NH - 1) warp_arrive(&bars.t_empty[0]);
+          const int o = 4 * h8;
+#pragma unroll
+          for (int q = 0; q < 2; ++q) {
+            const float4 gv = g4[q];
+            const float gg[4] = {gv.x, gv.y, gv.z, gv.w};
+            float dr[4], dz[4], dn[4], dhn[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const int j = 4 * q + u, c = h + j;
+              const float rr = sigm(__uint_as_float(vr[j]) + bias[c] + bias[3 * H + c]);
+              const float zz = sigm(__uint_as_float(vz[j]) + bias[H + c] + bias[4 * H + c]);
+              const float ghn = __uint_as_float(vh[j]) + bias[5 * H + c];
+              const float nn = tanh_fast(__uint_as_float(vn[j]) + bias[2 * H + c] + rr * ghn);
+              const float gr = real ? gg[u] : 0.f;
+              const float an = gr * (1.f - zz) * (1.f - nn * nn);
+              dn[u] = an;
+              dhn[u] = an * rr;
+              dr[u] = an * ghn * rr * (1.f - rr);
+              dz[u] = gr * (e[j] - nn) * zz * (1.f - zz);
+              dhd[j] = gr * zz;
+            }
+            p_r[o + 2 * q] = pk2(dr[0], dr[1]); p_r[o + 2 * q + 1] = pk2(dr[2], dr[3]);
+            p_z[o + 2 * q] = pk2(dz[0], dz[1]); p_z[o + 2 * q + 1] = pk2(dz[2], dz[3]);
+            p_n[o + 2 * q] = pk2(dn[0], dn[1]); p_n[o + 2 * q + 1] = pk2(dn[2], dn[3]);
+            p_hn[o + 2 * q] = pk2(dhn[0], dhn[1]); p_hn[o + 2 * q + 1] = pk2(dhn[2], dhn[3]);
+          }
+          float4* go = reinterpret_cast<float4*>(gout + (size_t)row * H + h);
+          go[0] = make_float4(dhd[0], dhd[1], dhd[2], dhd[3]);
+          go[1] = make_float4(dhd[4], dhd[5], dhd[6], dhd[7]);
+          // gate gradients transposed for the weight-gradient GEMM: rows o = gate*H + h
+          store_T4(dgiT, ld_g, row, h, p_r + o);
+          store_T4(dgiT + (size_t)H * ld_g, ld_g, row, h, p_z + o);
+          store_T4(dgiT + (size_t)2 * H * ld_g, ld_g, row, h, p_n + o);
+          store_T4(dghT, ld_g, row, h, p_r + o);
+          store_T4(dghT + (size_t)H * ld_g, ld_g, row, h, p_z + o);
+          store_T4(dghT + (size_t)2 * H * ld_g, ld_g, row, h, p_hn + o);
+        }
+        // in-place rewrite into the columns this warpgroup read (window 16 g of r and of z)
+        const uint32_t w0 = acc + 16 * g;
+        tmem_st4(w0, p_r);
+        tmem_st4(w0 + 4, p_r + 4);
+        tmem_st4(w0 + 8, p_z);
+        tmem_st4(w0 + 12, p_z + 4);
+        tmem_st4(w0 + 64, p_n);
+        tmem_st4(w0 + 68, p_n + 4);
+        tmem_st4(w0 + 72, p_hn);
+        tmem_st4(w0 + 76, p_hn + 4);
+        tmem_wait_st();
+        tc_fence_before();
+        warp_arrive(&bars.ops_ready);
+      }
+      if (!ok) break;
+      // dX and dH of the whole tile are complete once the last job's products are
+      if (!mbar_wait(&bars.ph2_full, (jn - 1) & 1, status, 648, abort, 64)) break;
+      tc_fence_after();
+#pragma unroll
+      for (int hh = 0; hh < NH; ++hh) {
+        const int h0 = 64 * hh + 16 * g;
+        uint32_t vx[16], vd[16];
+        tmem_ld16(tmem + lb + kDX + h0, vx);
+        tmem_ld16(tmem + lb + kDH + h0, vd);
+        tmem_wait_ld();
+        if (hh == NH - 1) {
+          tc_fence_before();
+          warp_arrive(&bars.dx_empty);
+        }
+        uint32_t px[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) px[j] = pk2(__uint_as_float(vx[2 * j]), __uint_as_float(vx[2 * j + 1]));
+        store_T8(dXT, ld_x, row, h0, px);
+        // this thread stored the direct term of these columns above
+        float4* go = reinterpret_cast<float4*>(gout + (size_t)row * H + h0);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float4 d = go[q];
+          go[q] = make_float4(d.x + __uint_as_float(vd[4 * q]), d.y + __uint_as_float(vd[4 * q + 1]),
+                              d.z + __uint_as_float(vd[4 * q + 2]), d.w + __uint_as_float(vd[4 * q + 3]));
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+}  // namespace wide
+
 }  // namespace
 
-bool gru_tc_supported(int H) { return H == kH; }
+bool gru_tc_supported(int H) { return H == kH || H == wide::H; }
 
-cudaError_t gru_fwd_tc(int n_pad, int n_real, const __nv_bfloat16* Y, const __nv_bfloat16* E,
-                       const __nv_bfloat16* W_ih, const __nv_bfloat16* W_hh, const float* b_ih,
-                       const float* b_hh, __nv_bfloat16* En, __nv_bfloat16* EnT, int64_t ld_T,
-                       int* status, cudaStream_t st) {
+cudaError_t gru_fwd_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y,
+                       const __nv_bfloat16* E, const __nv_bfloat16* W_ih,
+                       const __nv_bfloat16* W_hh, const float* b_ih, const float* b_hh,
+                       __nv_bfloat16* En, __nv_bfloat16* EnT, int64_t ld_T, int* status,
+                       cudaStream_t st) {
+  if (!gru_tc_supported(H) || n_pad % 128) return cudaErrorInvalidValue;
+  const bool w = H == wide::H;
   CUtensorMap tY, tE, tWi, tWh;
-  if (!make_map_ld(&tY, Y, n_pad, kH, kH, 128) || !make_map_ld(&tE, E, n_pad, kH, kH, 128) ||
-      !make_map_ld(&tWi, W_ih, 3 * kH, kH, kH, 3 * kH) ||
-      !make_map_ld(&tWh, W_hh, 3 * kH, kH, kH, 3 * kH))
+  if (!make_map_ld(&tY, Y, n_pad, H, H, 128) || !make_map_ld(&tE, E, n_pad, H, H, 128) ||
+      !make_map_ld(&tWi, W_ih, 3 * H, H, H, w ? 64 : 3 * H) ||
+      !make_map_ld(&tWh, W_hh, 3 * H, H, H, w ? 64 : 3 * H))
     return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(k_gru_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       GruSmem::FWD);
+  auto kern = w ? wide::k_gru_fwd : k_gru_fwd_tc;
+  const int smem = w ? wide::Smem::FWD : GruSmem::FWD;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const int n_tiles = n_pad / 128;
   const int grid = std::min(n_tiles, gemm_tn_num_sms());
-  e = launch_pdl(k_gru_fwd_tc, dim3(grid), dim3(kThreads), GruSmem::FWD, st, tY, tE, tWi, tWh, b_ih,
-                 b_hh, En, EnT, ld_T, n_tiles, n_real, status);
+  e = launch_pdl(kern, dim3(grid), dim3(kThreads), smem, st, tY, tE, tWi, tWh, b_ih, b_hh, En, EnT,
+                 ld_T, n_tiles, n_real, status);
   note_launch();
   return e;
 }
 
-cudaError_t gru_bwd_tc(int n_pad, int n_real, const __nv_bfloat16* Y, const __nv_bfloat16* E,
-                       const __nv_bfloat16* W_ih, const __nv_bfloat16* W_hh,
-                       const __nv_bfloat16* W_ihT, const __nv_bfloat16* W_hhT, const float* b_ih,
-                       const float* b_hh, const float* gin, float* gout, __nv_bfloat16* dXT,
-                       int64_t ld_x, __nv_bfloat16* dgiT, __nv_bfloat16* dghT, int64_t ld_g,
-                       int* status, cudaStream_t st) {
+cudaError_t gru_bwd_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y,
+                       const __nv_bfloat16* E, const __nv_bfloat16* W_ih,
+                       const __nv_bfloat16* W_hh, const __nv_bfloat16* W_ihT,
+                       const __nv_bfloat16* W_hhT, const float* b_ih, const float* b_hh,
+                       const float* gin, float* gout, __nv_bfloat16* dXT, int64_t ld_x,
+                       __nv_bfloat16* dgiT, __nv_bfloat16* dghT, int64_t ld_g, int* status,
+                       cudaStream_t st) {
+  if (!gru_tc_supported(H) || n_pad % 128) return cudaErrorInvalidValue;
+  const bool w = H == wide::H;
   CUtensorMap tY, tE, tWi, tWh, tWiT, tWhT, tG;
-  if (!make_map_ld(&tY, Y, n_pad, kH, kH, 128) || !make_map_ld(&tE, E, n_pad, kH, kH, 128) ||
-      !make_map_ld(&tWi, W_ih, 3 * kH, kH, kH, 3 * kH) ||
-      !make_map_ld(&tWh, W_hh, 3 * kH, kH, kH, 3 * kH) ||
-      !make_map_ld(&tWiT, W_ihT, kH, 3 * kH, 3 * kH, kH) ||
-      !make_map_ld(&tWhT, W_hhT, kH, 3 * kH, 3 * kH, kH) ||
-      !make_map_f32(&tG, gin, n_pad, kH, 128))
+  // H = 64: the transposed weights are loaded whole as three 64-column boxes; H = 128: pieces of
+  // 128 rows x 64 columns
+  if (!make_map_ld(&tY, Y, n_pad, H, H, 128) || !make_map_ld(&tE, E, n_pad, H, H, 128) ||
+      !make_map_ld(&tWi, W_ih, 3 * H, H, H, w ? 64 : 3 * H) ||
+      !make_map_ld(&tWh, W_hh, 3 * H, H, H, w ? 64 : 3 * H) ||
+      !make_map_ld(&tWiT, W_ihT, H, 3 * H, 3 * H, H) ||
+      !make_map_ld(&tWhT, W_hhT, H, 3 * H, 3 * H, H) || !make_map_f32(&tG, gin, n_pad, H, 128))
     return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(k_gru_bwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       GruSmem::BWD);
+  auto kern = w ? wide::k_gru_bwd : k_gru_bwd_tc;
+  const int smem = w ? wide::Smem::BWD : GruSmem::BWD;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const int n_tiles = n_pad / 128;
   const int grid = std::min(n_tiles, gemm_tn_num_sms());
-  e = launch_pdl(k_gru_bwd_tc, dim3(grid), dim3(kThreads), GruSmem::BWD, st, tY, tE, tWi, tWh, tWiT,
-                 tWhT, tG, b_ih, b_hh, gout, dXT, ld_x, dgiT, dghT, ld_g, n_tiles, n_real, status);
+  e = launch_pdl(kern, dim3(grid), dim3(kThreads), smem, st, tY, tE, tWi, tWh, tWiT, tWhT, tG, b_ih,
+                 b_hh, gout, dXT, ld_x, dgiT, dghT, ld_g, n_tiles, n_real, status);
   note_launch();
   return e;
 }

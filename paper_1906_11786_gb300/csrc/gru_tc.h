@@ -1,4 +1,4 @@
-// Fused GRU forward / backward on tcgen05 (gru_tc.cu); state size H = 64.
+// Fused GRU forward / backward on tcgen05 (gru_tc.cu); state size H in {64, 128}.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -10,9 +10,9 @@ namespace bg {
 
 bool gru_tc_supported(int H);
 
-// E(t+1) = GRU(Y, E) for all n_pad rows (rows >= n_real get 0).  Y, E, En: [n_pad][H] bf16;
+// E(t+1) = GRU(Y, E) for all n_pad rows (rows >= n_real get 0); n_pad a multiple of 128.  Y, E, En: [n_pad][H] bf16;
 // W_ih, W_hh: [3H][H] bf16; biases fp32 [3H]; EnT (may be NULL): [H][ld_T] bf16, transposed En.
-cudaError_t gru_fwd_tc(int n_pad, int n_real, const __nv_bfloat16* Y, const __nv_bfloat16* E,
+cudaError_t gru_fwd_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y, const __nv_bfloat16* E,
                        const __nv_bfloat16* W_ih, const __nv_bfloat16* W_hh, const float* b_ih,
                        const float* b_hh, __nv_bfloat16* En, __nv_bfloat16* EnT, int64_t ld_T,
                        int* status, cudaStream_t st);
@@ -21,7 +21,7 @@ cudaError_t gru_fwd_tc(int n_pad, int n_real, const __nv_bfloat16* Y, const __nv
 //   gout [n_pad][H] fp32 = dL/dE(t) through the GRU (direct and W_hh terms; may alias gin),
 //   dXT [H][ld_x] bf16 = (dL/dY)^T, dgiT / dghT [3H][ld_g] bf16 = gate gradients transposed.
 // W_ihT, W_hhT: [H][3H] bf16 transposes of W_ih, W_hh.
-cudaError_t gru_bwd_tc(int n_pad, int n_real, const __nv_bfloat16* Y, const __nv_bfloat16* E,
+cudaError_t gru_bwd_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y, const __nv_bfloat16* E,
                        const __nv_bfloat16* W_ih, const __nv_bfloat16* W_hh,
                        const __nv_bfloat16* W_ihT, const __nv_bfloat16* W_hhT, const float* b_ih,
                        const float* b_hh, const float* gin, float* gout, __nv_bfloat16* dXT,
