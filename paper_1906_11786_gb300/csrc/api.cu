@@ -349,7 +349,11 @@ FwdWs fwd_ws(const bg_plan* p, bg_dtype dt, int H) {
 
 // bf16 shapes the fused kernels do not cover still run their products on the tensor cores (the
 // band sums stay SIMT gathers over the bit tiles); the split-K gradient GEMM needs H <= 128.
-bool tc_gemm_path(bg_dtype dt, int H) { return dt == BG_BF16 && H <= 128; }
+// bf16 shapes whose GEMMs run on the tensor cores: the split-K weight-gradient GEMM takes
+// Hout in {32, 64, 128, 256}; other multiples of 32 use the SIMT GEMMs.
+bool tc_gemm_path(bg_dtype dt, int H) {
+  return dt == BG_BF16 && (H == 32 || H == 64 || H == 128 || H == 256);
+}
 
 struct BwdWs {
   size_t dM, Wt, part;                 // fp32 SIMT path

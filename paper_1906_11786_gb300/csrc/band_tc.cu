@@ -69,17 +69,19 @@ __host__ __device__ constexpr int band_chunks(int S) { return S <= 64 ? 2 : 3 * 
 
 template <int H, int S>
 struct Cfg {
-  // H = 128 runs as two passes over 64-column halves of the state: pass hh contracts the band with
-  // columns 64 hh .. 64 hh + 63 of E and multiplies the result by rows 64 hh .. of W_p, into Y
+  // H > 64 runs as H / 64 passes over 64-column slices of the state: pass hh contracts the band
+  // with columns 64 hh .. 64 hh + 63 of E and multiplies the result by rows 64 hh .. of W_p, into Y
   static constexpr int NH = H / 64;
   static constexpr int C1 = band_chunks(S);                   // 128-column chunks per type
   static constexpr int ATOM_X = 64 * 128;                     // 64 nodes x 64 state columns
   static constexpr int XWIN = 2 * C1 * ATOM_X;                // one half's window, 64-node atoms
   static constexpr int NXB = XWIN <= 48 * 1024 ? 2 : 1;       // state-window buffers
   static constexpr int NW = 2;                                // W ring stages
-  // one W stage: the 64 K-columns of one half of W_p^T as fp32 (tf32 operand), two 32-column
-  // atoms of H rows
-  static constexpr int WSTAGE = 2 * H * 128;
+  // W stages hold K-columns of W_p^T as fp32 (tf32 operand) in 32-column atoms of H rows: a job's
+  // 64 K-columns in one stage, or at H = 256 (64 KB) in two stages of one atom
+  static constexpr int WK = H <= 128 ? 64 : 32;               // K-columns per stage
+  static constexpr int WJ = 64 / WK;                          // stages per job
+  static constexpr int WSTAGE = (WK / 32) * H * 128;
   static constexpr int DEG = kTile * 128;                     // 128 rows x 64 bf16
   static constexpr int NDEG = NH > 1 ? 1 : 2;                 // deg buffers
   static constexpr int B2 = H * 128;                          // H rows x 64 bf16
@@ -99,13 +101,14 @@ struct Cfg {
   static constexpr int D1COL0 = H;
   static constexpr int ACOL = H + NB * 64;
   static constexpr int NA = (512 - ACOL) / 64;
-  // a job's chunks come in CG-chunk groups (one barrier wait each), G groups per job
-  static constexpr int CG = C1 <= 3 ? C1 : 3;
+  // a job's chunks come in CG-chunk groups (one barrier wait each), G groups per job; a group and
+  // one more A tile must fit in the NA slots (H = 256 has two slots: one chunk per group)
+  static constexpr int CG = (C1 <= 3 && NA > C1) ? C1 : (NA > 3 ? 3 : NA - 1);
   static constexpr int G = C1 / CG;
-  static constexpr int NT = 8;                                // per-group barrier ring
+  static constexpr int NT = (8 / G) * G;                      // per-group barrier ring
   static constexpr int NE = 2;                                // expander warpgroups
   static constexpr int THREADS = 128 * (2 + NE);
-  static_assert(H == 64 || H == 128, "state size");
+  static_assert(H == 64 || H == 128 || H == 256, "state size");
   static_assert(C1 % CG == 0 && NT % G == 0, "chunk groups");
   static_assert(NA >= CG + 1 && NA <= 8, "one group of A tiles and one more must fit");
   static_assert(NM >= 2 && NM <= 8, "mask ring");
@@ -117,7 +120,10 @@ struct Bars {
   uint64_t w_full[4], w_empty[4];
   uint64_t deg_full[2], deg_empty[2];
   uint64_t b2_full;
-  uint64_t a_empty[8];
+  // release of A slot s for the expander group that uses it next: each group waits only on its
+  // own barrier, once per use, so no waiter can fall two phases behind (the groups take jobs in
+  // turn, and slot uses alternate between them irregularly)
+  uint64_t a_empty[8][2];
   uint64_t d1_full[4];
   uint64_t t_full[8];
   uint64_t y_full, y_empty;
@@ -195,7 +201,7 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     }
     for (int i = 0; i < 4; ++i) mbar_init(&bars->d1_full[i], 1);
     for (int i = 0; i < 4; ++i) { mbar_init(&bars->w_full[i], 1); mbar_init(&bars->w_empty[i], 1); }
-    for (int i = 0; i < 8; ++i) mbar_init(&bars->a_empty[i], 1);
+    for (int i = 0; i < 8; ++i) { mbar_init(&bars->a_empty[i][0], 1); mbar_init(&bars->a_empty[i][1], 1); }
     for (int i = 0; i < 8; ++i) mbar_init(&bars->t_full[i], 4 + (i % C::G == 0 ? kFree : 0));
     mbar_init(&bars->b2_full, 1);
     mbar_init(&bars->y_full, 1);
@@ -205,9 +211,11 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     for (int i = 0; i < 8; ++i) { mbar_init(&bars->m_full[i], 1); mbar_init(&bars->m_empty[i], 4); }
     bars->abort = 0;
     fence_mbar_init();
-    // the first NB jobs find their pre_p unit free: stand in for the releases
+    // the first NB jobs find their pre_p unit free: stand in for the releases; likewise the first
+    // use of each A slot (chunk s, job s / C1)
     for (int c = 0; c < C::NB; ++c)
       for (int a = 0; a < kFree; ++a) mbar_arrive(&bars->t_full[(c * C::G) % C::NT]);
+    for (int sl = 0; sl < C::NA; ++sl) mbar_arrive(&bars->a_empty[sl][(sl / C::C1) % C::NE]);
   }
   if (warp == 1) {
     tmem_alloc(&bars->tmem_base, 512);
@@ -257,19 +265,20 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
         for (int a = 0; a < 2 * C::C1; ++a)
           tma_load_2d(xwin + xb * C::XWIN + a * C::ATOM_X, &tm_x, &bars->x_full[xb],
                       ws + a * kAtom, 64 * hh);
-        // one W stage per job: K-columns 64 hh .. 64 hh + 63 of W_p^T, two 32-column atoms
-        for (int p = 0; p < P; ++p, ++widx) {
-          const int ws2 = widx % C::NW;
-          if (!mbar_wait(&bars->w_empty[ws2], ((widx / C::NW) & 1) ^ 1, status, 103, abort, 64)) {
-            ok = false;
-            break;
+        // per job: K-columns 64 hh .. 64 hh + 63 of W_p^T in WJ stages of WK / 32 atoms
+        for (int p = 0; p < P && ok; ++p)
+          for (int wj = 0; wj < C::WJ; ++wj, ++widx) {
+            const int ws2 = widx % C::NW;
+            if (!mbar_wait(&bars->w_empty[ws2], ((widx / C::NW) & 1) ^ 1, status, 103, abort, 64)) {
+              ok = false;
+              break;
+            }
+            ++n_w[ws2];
+            mbar_expect_tx(&bars->w_full[ws2], C::WSTAGE);
+            for (int a = 0; a < C::WK / 32; ++a)
+              tma_load_2d(wring + ws2 * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws2],
+                          64 * hh + C::WK * wj + 32 * a, p * H);
           }
-          ++n_w[ws2];
-          mbar_expect_tx(&bars->w_full[ws2], C::WSTAGE);
-          for (int a = 0; a < 2; ++a)
-            tma_load_2d(wring + ws2 * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws2],
-                        64 * hh + 32 * a, p * H);
-        }
       }
     }
     if (*abort) {
@@ -315,6 +324,9 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     const bool leader = elect_one_sync();
     constexpr uint32_t idesc = idesc_bf16_f32(kTile, 64);
     uint32_t c = 0, slot = 0, gi = 0, xi = 0;
+    // expander group of chunk x + NA (the next user of the slot chunk x frees): job (x + NA) / C1
+    // mod 2, kept as a group and a position within the job
+    uint32_t nx_g = (C::NA / C::C1) & 1, nx_r = C::NA % C::C1;
     bool ok = true;
     for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x) {
       for (int hh = 0; hh < C::NH && ok; ++hh, ++xi) {
@@ -335,8 +347,9 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
                 if (leader)
                   mma_ts(d1, a + kk * 8, jdesc + (uint64_t)(((kk / 4) * C::ATOM_X + (kk % 4) * 32) >> 4),
                          idesc, (j == 0 && kk == 0) ? 0u : 1u);
-              if (leader) tc_commit(&bars->a_empty[slot]);
+              if (leader) tc_commit(&bars->a_empty[slot][nx_g]);
               slot = slot + 1 == (uint32_t)C::NA ? 0 : slot + 1;
+              if (++nx_r == (uint32_t)C::C1) { nx_r = 0; nx_g ^= 1; }
             }
           }
           if (!ok) break;
@@ -353,32 +366,36 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     const bool leader = elect_one_sync();
     constexpr uint32_t idesc = idesc_bf16_f32(kTile, H);
     constexpr uint32_t idesc2 = idesc_tf32_f32(kTile, H);
-    uint32_t c = 0;
+    uint32_t c = 0, widx = 0;
     bool ok = true;
     int i = 0;
     for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x, ++i) {
-      for (int jb = 0; jb < jobs; ++jb, ++c) {
+      for (int jb = 0; jb < jobs && ok; ++jb, ++c) {
         const int b = c % C::NB;
-        const int ws = c % C::NW;
         if (!mbar_wait(&bars->d1_full[b], (c / C::NB) & 1, status, 208, abort) ||
-            !mbar_wait(&bars->w_full[ws], (c / C::NW) & 1, status, 202, abort) ||
             (jb == 0 && !mbar_wait(&bars->y_empty, (i & 1) ^ 1, status, 203, abort))) {
           ok = false;
           break;
         }
-        tc_fence_after();
-        const uint32_t wbase = smem_u32(wring + ws * C::WSTAGE);
+        for (int wj = 0; wj < C::WJ; ++wj, ++widx) {
+          const int ws = widx % C::NW;
+          if (!mbar_wait(&bars->w_full[ws], (widx / C::NW) & 1, status, 202, abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t wbase = smem_u32(wring + ws * C::WSTAGE);
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t bdesc = desc_sw128_kmajor(wbase + (kk / 4) * H * 128 + (kk % 4) * 32);
-          if (leader) mma_ts_tf32(tmem + C::YCOL, tmem + C::D1COL0 + b * 64 + kk * 8, bdesc, idesc2,
-                                  (jb == 0 && kk == 0) ? 0u : 1u);
+          for (int kk = 0; kk < C::WK / 8; ++kk) {
+            const uint64_t bdesc = desc_sw128_kmajor(wbase + (kk / 4) * H * 128 + (kk % 4) * 32);
+            if (leader) mma_ts_tf32(tmem + C::YCOL, tmem + C::D1COL0 + b * 64 + C::WK * wj + kk * 8,
+                                    bdesc, idesc2, (jb == 0 && wj == 0 && kk == 0) ? 0u : 1u);
+          }
+          if (leader) tc_commit(&bars->w_empty[ws]);
         }
-        if (leader) {
-          tc_commit(&bars->w_empty[ws]);
-          // this unit is free again: part of job c + NB's first group
-          tc_commit(&bars->t_full[((c + C::NB) * C::G) % C::NT]);
-        }
+        if (!ok) break;
+        // this unit is free again: part of job c + NB's first group
+        if (leader) tc_commit(&bars->t_full[((c + C::NB) * C::G) % C::NT]);
       }
       if (!ok) break;
       if (has_bias) {
@@ -403,6 +420,7 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     const int r = (threadIdx.x - 128) % 128;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     uint32_t aidx = 0, midx = 0;
+    uint32_t par = 0;  // bit s: parity of this group's waits so far on A slot s
     for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x) {
       bool ok = true;
       for (int jb = 0; jb < jobs && ok; ++jb, ++midx) {
@@ -419,10 +437,11 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
         for (int j = 0; j < C::C1; ++j) {
           const uint4 m = *reinterpret_cast<const uint4*>(mrow + j * kTile * 16);
           const int slot = aidx % C::NA;
-          if (!mbar_wait(&bars->a_empty[slot], ((aidx / C::NA) & 1) ^ 1, status, 301, abort)) {
+          if (!mbar_wait(&bars->a_empty[slot][eg], (par >> slot) & 1, status, 301, abort)) {
             ok = false;
             break;
           }
+          par ^= 1u << slot;
           tc_fence_after();
           uint32_t v[32];
           expand_word(m.x, v);
@@ -652,7 +671,8 @@ cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap&
   return e;
 }
 
-// The shapes with a tensor-core kernel: H in {64, 128} at S in {32, 64, 128, 256}.
+// The shapes with a tensor-core kernel: H in {64, 128} at S in {32, 64, 128, 256}; H = 256 at
+// S in {32, 64, 128} (its state-slice window at S = 256 leaves no room for the mask ring).
 template <int H, bool BWD>
 cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
                    const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
@@ -665,7 +685,9 @@ cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& t
   switch (p->S) {
     case 32: BG_BAND_S(32)
     case 64: BG_BAND_S(64)
-    case 256: BG_BAND_S(256)
+    case 256:
+      if constexpr (H <= 128) { BG_BAND_S(256) }
+      return cudaErrorInvalidValue;
     default: BG_BAND_S(128)
   }
 #undef BG_BAND_S
@@ -720,8 +742,9 @@ bool make_map_3d(CUtensorMap* m, const void* base, uint64_t batch, uint64_t rows
 
 bool band_tc_supported(const bg_plan* p, int dtype, int H) {
   if (!p || dtype != 1 || p->P > 32 || p->n_pad() % kTile) return false;
-  const bool shape = (H == 64 || H == 128) &&
-                     (p->S == 32 || p->S == 64 || p->S == 128 || p->S == 256);
+  const bool shape = ((H == 64 || H == 128) &&
+                      (p->S == 32 || p->S == 64 || p->S == 128 || p->S == 256)) ||
+                     (H == 256 && (p->S == 32 || p->S == 64 || p->S == 128));
   return shape && p->d_maskI && p->d_maskTI && p->d_deg2 && p->max_deg <= 256 &&
          encode_fn() != nullptr;
 }
@@ -767,7 +790,10 @@ cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, i
   if (H == 64)
     return launch<64, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, has_bias,
                              0, status, st);
-  return launch<128, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, has_bias,
+  if (H == 128)
+    return launch<128, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, has_bias,
+                              0, status, st);
+  return launch<256, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, has_bias,
                             0, status, st);
 }
 
@@ -781,7 +807,10 @@ cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, 
   if (H == 64)
     return launch<64, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
                             status, st);
-  return launch<128, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
+  if (H == 128)
+    return launch<128, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
+                             status, st);
+  return launch<256, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
                            status, st);
 }
 

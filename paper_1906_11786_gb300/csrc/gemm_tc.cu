@@ -24,13 +24,25 @@ namespace {
 
 constexpr int kStages = 4;
 
+// Tile widths BN = Hout + 16 (48, 80, 144, 272), four stages each.  Up to BN = 80 two CTAs share
+// an SM; BN = 144 (138 KB) and BN = 272 (all 512 TMEM columns) run one per SM.  B boxes are at
+// most 256 rows: BN = 272 loads two boxes of 136 rows and issues an N = 256 and an N = 16 MMA per
+// K step.
 template <int BN>
 struct GCfg {
   static constexpr int A_BYTES = 128 * 128;  // 128 rows x 64 bf16
   static constexpr int B_BYTES = BN * 128;
   static constexpr int STAGE = A_BYTES + B_BYTES;
-  static constexpr int SMEM = kStages * STAGE + 1024 + 1024;
-  static constexpr int TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  static constexpr int STAGES = 4;
+  static constexpr int SMEM = STAGES * STAGE + 1024 + 1024;
+  static constexpr int TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : BN <= 256 ? 256 : 512;
+  static constexpr int PER_SM = BN <= 80 ? 2 : 1;
+  static constexpr int BOX = BN <= 256 ? BN : BN / 2;  // B rows per TMA box
+  static constexpr int N1 = BN <= 256 ? BN : 256;      // first MMA's N
+  static_assert(BN % 16 == 0 && BN <= 512, "tile width");
+  static_assert(PER_SM * (SMEM + 512) <= 232448, "shared memory");
+  static_assert(BOX * 128 % 1024 == 0, "box alignment");
+  static_assert(STAGES <= kStages, "stage count");
 };
 
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
@@ -61,9 +73,9 @@ __global__ void __launch_bounds__(192, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * C::STAGE);
-  uint64_t* empty = full + kStages;
-  uint64_t* done = empty + kStages;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* done = empty + C::STAGES;
   uint64_t* drain = done + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
@@ -78,7 +90,7 @@ __global__ void __launch_bounds__(192, 1)
   const int kc0 = split * per_split;
   const int kc1 = min(kchunks, kc0 + per_split);
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    for (int s = 0; s < C::STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
     mbar_init(done, 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -100,32 +112,38 @@ __global__ void __launch_bounds__(192, 1)
     grid_dep_wait();  // A and B are the previous kernels' output
     uint32_t issued[kStages] = {0, 0, 0, 0};
     for (int kc = kc0, it = 0; kc < kc1; ++kc, ++it) {
-      const int s = it % kStages;
-      if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1, status, 501, abort, 32)) break;
+      const int s = it % C::STAGES;
+      if (!mbar_wait(&empty[s], ((it / C::STAGES) & 1) ^ 1, status, 501, abort, 32)) break;
       ++issued[s];
       mbar_expect_tx(&full[s], C::STAGE);
       uint8_t* st = smem + s * C::STAGE;
       tma_load_2d(st, tmA, &full[s], kc * 64, mt * 128);
-      tma_load_2d(st + C::A_BYTES, tmB, &full[s], kc * 64, blockIdx.y * BN);
+      for (int r = 0; r < BN; r += C::BOX)
+        tma_load_2d(st + C::A_BYTES + r * 128, tmB, &full[s], kc * 64, blockIdx.y * BN + r);
     }
     if (*abort)
-      for (int s = 0; s < kStages; ++s)
+      for (int s = 0; s < C::STAGES; ++s)
         for (uint32_t t = 0; issued[s] && t < (1u << 22) && !mbar_try(&full[s], (issued[s] - 1) & 1); ++t) {
         }
   } else if (warp == 1) {
     // the whole warp runs the loop (uniform operands); one elected lane issues
     const bool leader = elect_one_sync();
-    constexpr uint32_t idesc = idesc_bf16_f32(128, BN);
+    constexpr uint32_t idesc = idesc_bf16_f32(128, C::N1);
+    constexpr uint32_t idesc2 = idesc_bf16_f32(128, BN > 256 ? BN - 256 : 16);
     for (int kc = kc0, it = 0; kc < kc1; ++kc, ++it) {
-      const int s = it % kStages;
-      if (!mbar_wait(&full[s], (it / kStages) & 1, status, 502, abort)) break;
+      const int s = it % C::STAGES;
+      if (!mbar_wait(&full[s], (it / C::STAGES) & 1, status, 502, abort)) break;
       tc_fence_after();
       const uint32_t a = smem_u32(smem + s * C::STAGE), b = a + C::A_BYTES;
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk)
-        if (leader)
-          mma_ss(tmem, desc_sw128_kmajor(a + kk * 32), desc_sw128_kmajor(b + kk * 32), idesc,
-                 (kc > kc0 || kk > 0) ? 1u : 0u);
+        if (leader) {
+          const uint64_t ad = desc_sw128_kmajor(a + kk * 32);
+          const uint32_t acc = (kc > kc0 || kk > 0) ? 1u : 0u;
+          mma_ss(tmem, ad, desc_sw128_kmajor(b + kk * 32), idesc, acc);
+          if (BN > 256)
+            mma_ss(tmem + 256, ad, desc_sw128_kmajor(b + 256 * 128 + kk * 32), idesc2, acc);
+        }
       if (leader) tc_commit(&empty[s]);
       __syncwarp();
     }
@@ -416,7 +434,7 @@ size_t gemm_tn_part_floats(int M, int N, int64_t K) {
 cudaError_t gemm_tn_multi(const TNProblem* pr, int n, int Hout, int64_t K, int accumulate,
                           float* part, size_t part_floats, int* status, cudaStream_t st) {
   const int N = Hout + 16;  // Hout gradient columns, one ones-column (bias), padding to 16
-  if (N != 48 && N != 80 && N != 144) return cudaErrorInvalidValue;
+  if (N != 48 && N != 80 && N != 144 && N != 272) return cudaErrorInvalidValue;
   if (n < 1 || n > kMaxGroups) return cudaErrorInvalidValue;
   const int64_t kchunks = (K + 63) / 64;
   TNGroups grp{};
@@ -424,7 +442,7 @@ cudaError_t gemm_tn_multi(const TNProblem* pr, int n, int Hout, int64_t K, int a
   int mt = 0, Mtot = 0;
   for (int g = 0; g < n; ++g) {
     if (!make_map_ld(&grp.a[g], pr[g].A, pr[g].M, K, pr[g].lda, 128) ||
-        !make_map_ld(&grp.b[g], pr[g].B, N, K, pr[g].ldb, N))
+        !make_map_ld(&grp.b[g], pr[g].B, N, K, pr[g].ldb, N <= 256 ? N : N / 2))
       return cudaErrorInvalidValue;
     mt += (pr[g].M + 127) / 128;
     grp.mt_end[g] = mt;
@@ -438,9 +456,11 @@ cudaError_t gemm_tn_multi(const TNProblem* pr, int n, int Hout, int64_t K, int a
   for (int g = n; g < kMaxGroups; ++g) grp.mt_end[g] = mt;
   o.n_groups = n;
   const int sms = gemm_tn_num_sms();
-  // two CTAs fit per SM: at most 2 * sms CTAs, so that all of them run in one wave (a partial
-  // second wave of even a few CTAs would nearly double the time of this HBM-bound pass)
-  int splits = (int)std::max<int64_t>(1, std::min<int64_t>(kchunks, std::max(1, 2 * sms / mt)));
+  // at most 2 * sms CTAs: one wave where two fit per SM (a partial second wave of even a few CTAs
+  // would nearly double the time of this HBM-bound pass); at N = 144 the same grid in two waves of
+  // one CTA per SM measured faster than one wave of two CTAs with three stages each
+  const int per_sm = N <= 144 ? 2 : 1;
+  int splits = (int)std::max<int64_t>(1, std::min<int64_t>(kchunks, std::max(1, per_sm * sms / mt)));
   while (splits > 1 && (size_t)splits * Mtot * N > part_floats) --splits;
   const int per = (int)((kchunks + splits - 1) / splits);
   splits = (int)((kchunks + per - 1) / per);
@@ -457,8 +477,10 @@ cudaError_t gemm_tn_multi(const TNProblem* pr, int n, int Hout, int64_t K, int a
     BG_GEMM_CASE(48)
   } else if (N == 80) {
     BG_GEMM_CASE(80)
-  } else {
+  } else if (N == 144) {
     BG_GEMM_CASE(144)
+  } else {
+    BG_GEMM_CASE(272)
   }
 #undef BG_GEMM_CASE
   note_launch();

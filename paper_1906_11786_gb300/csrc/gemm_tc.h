@@ -18,7 +18,7 @@ size_t gemm_tn_part_floats(int M, int N, int64_t K);
 // of A (a bias gradient).  Output (accumulate != 0 adds):
 //   mode 0: out[m][n] = G[m][n] (n < Hout), bias[m] = G[m][Hout]
 //   mode 1: m = p*Hout + o: out[p][n][o] = G[m][n], bias[m] = G[m][Hout]   (bias may be NULL)
-// Hout in {32, 64, 128}.  Deterministic: fixed split layout and summation order.
+// Hout in {32, 64, 128, 256}.  Deterministic: fixed split layout and summation order.
 cudaError_t gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int Hout,
                     int64_t K, int mode, float* out, float* bias, int accumulate, float* part,
                     size_t part_floats, int* status, cudaStream_t st);
