@@ -80,6 +80,32 @@ __device__ __forceinline__ float tanh_fast(float x) {
 }
 __device__ __forceinline__ float sigm(float x) { return fmaf(0.5f, tanh_fast(0.5f * x), 0.5f); }
 
+// Gate biases in shared memory as four H-vectors: b_ir + b_hr, b_iz + b_hz, b_in, b_hn (the r and z
+// biases enter only as sums); a thread reads those of its four columns c .. c+3 as one float4 each.
+struct GateBias {
+  float4 r, z, in, hn;
+};
+__device__ __forceinline__ GateBias gate_bias(const float* b, int H, int c) {
+  GateBias g;
+  g.r = *reinterpret_cast<const float4*>(b + c);
+  g.z = *reinterpret_cast<const float4*>(b + H + c);
+  g.in = *reinterpret_cast<const float4*>(b + 2 * H + c);
+  g.hn = *reinterpret_cast<const float4*>(b + 3 * H + c);
+  return g;
+}
+__device__ __forceinline__ float f4(const float4& v, int u) {
+  return u == 0 ? v.x : u == 1 ? v.y : u == 2 ? v.z : v.w;
+}
+__device__ __forceinline__ void fill_gate_bias(float* bias, const float* b_ih, const float* b_hh,
+                                               int H) {
+  for (int t = threadIdx.x; t < H; t += blockDim.x) {
+    bias[t] = b_ih[t] + b_hh[t];
+    bias[H + t] = b_ih[H + t] + b_hh[H + t];
+    bias[2 * H + t] = b_ih[2 * H + t];
+    bias[3 * H + t] = b_hh[2 * H + t];
+  }
+}
+
 // 8 consecutive bf16 of row r (columns c0 .. c0+7, c0 % 8 == 0): one swizzled 16-byte chunk.
 __device__ __forceinline__ void read_sw128_row8(const uint8_t* tile, int r, int c0, float* out) {
   const uint8_t* row = tile + (c0 / 64) * 128 * 128 + r * 128;
@@ -162,10 +188,7 @@ __device__ __forceinline__ void gru_gate_mmas(uint32_t acc, uint32_t sY, uint32_
 // Common prologue: barrier init, bias copy, TMEM allocation (512 columns: two accumulator sets).
 __device__ __forceinline__ void gru_setup(GruBars* b, float* bias, const float* b_ih,
                                           const float* b_hh, int warp) {
-  for (int t = threadIdx.x; t < 3 * kH; t += blockDim.x) {
-    bias[t] = b_ih[t];
-    bias[3 * kH + t] = b_hh[t];
-  }
+  fill_gate_bias(bias, b_ih, b_hh, kH);
   if (threadIdx.x == 0) {
     mbar_init(&b->w_full, 1);
     for (int i = 0; i < 2; ++i) {
@@ -230,7 +253,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   __shared__ GruBars bars;
-  __shared__ float bias[6 * kH];
+  __shared__ __align__(16) float bias[4 * kH];
   volatile int* abort = &bars.abort;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   gru_setup(&bars, bias, b_ih, b_hh, warp);
@@ -300,18 +323,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         uint32_t pk[4];
 #pragma unroll
-        for (int j = 0; j < 8; j += 2) {
-          float o[2];
+        for (int q = 0; q < 2; ++q) {
+          const GateBias gb = gate_bias(bias, kH, hs + 4 * q);
+          float o[4];
 #pragma unroll
-          for (int u = 0; u < 2; ++u) {
-            const int h = hs + j + u;
-            const float rr = sigm(__uint_as_float(vr[j + u]) + bias[h] + bias[3 * kH + h]);
-            const float zz = sigm(__uint_as_float(vz[j + u]) + bias[kH + h] + bias[4 * kH + h]);
-            const float nn = tanh_fast(__uint_as_float(vn[j + u]) + bias[2 * kH + h] +
-                                       rr * (__uint_as_float(vh[j + u]) + bias[5 * kH + h]));
-            o[u] = real ? (1.f - zz) * nn + zz * e[j + u] : 0.f;
+          for (int u = 0; u < 4; ++u) {
+            const int j = 4 * q + u;
+            const float rr = sigm(__uint_as_float(vr[j]) + f4(gb.r, u));
+            const float zz = sigm(__uint_as_float(vz[j]) + f4(gb.z, u));
+            const float nn = tanh_fast(__uint_as_float(vn[j]) + f4(gb.in, u) +
+                                       rr * (__uint_as_float(vh[j]) + f4(gb.hn, u)));
+            o[u] = real ? (1.f - zz) * nn + zz * e[j] : 0.f;
           }
-          pk[j / 2] = pk2(o[0], o[1]);
+          pk[2 * q] = pk2(o[0], o[1]);
+          pk[2 * q + 1] = pk2(o[2], o[3]);
         }
         *reinterpret_cast<uint4*>(En + (size_t)row * kH + hs) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
         if (EnT) store_T4(EnT, ld_T, row, hs, pk);
@@ -353,7 +378,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   __shared__ GruBars bars;
-  __shared__ float bias[6 * kH];
+  __shared__ __align__(16) float bias[4 * kH];
   volatile int* abort = &bars.abort;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   gru_setup(&bars, bias, b_ih, b_hh, warp);
@@ -456,14 +481,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int q = 0; q < 2; ++q) {
           const float4 gv = g4[q];
           const float gg[4] = {gv.x, gv.y, gv.z, gv.w};
+          const GateBias gb = gate_bias(bias, kH, hs + 4 * q);
           float dr[4], dz[4], dn[4], dhn[4];
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
-            const int j = 4 * q + u, h = hs + j;
-            const float rr = sigm(__uint_as_float(vr[j]) + bias[h] + bias[3 * kH + h]);
-            const float zz = sigm(__uint_as_float(vz[j]) + bias[kH + h] + bias[4 * kH + h]);
-            const float ghn = __uint_as_float(vh[j]) + bias[5 * kH + h];
-            const float nn = tanh_fast(__uint_as_float(vn[j]) + bias[2 * kH + h] + rr * ghn);
+            const int j = 4 * q + u;
+            const float rr = sigm(__uint_as_float(vr[j]) + f4(gb.r, u));
+            const float zz = sigm(__uint_as_float(vz[j]) + f4(gb.z, u));
+            const float ghn = __uint_as_float(vh[j]) + f4(gb.hn, u);
+            const float nn = tanh_fast(__uint_as_float(vn[j]) + f4(gb.in, u) + rr * ghn);
             const float gr = real ? gg[u] : 0.f;
             const float an = gr * (1.f - zz) * (1.f - nn * nn);
             dn[u] = an;
@@ -567,10 +593,7 @@ struct Bars {
 
 __device__ __forceinline__ void setup(Bars* b, float* bias, const float* b_ih, const float* b_hh,
                                       int warp) {
-  for (int t = threadIdx.x; t < 3 * H; t += blockDim.x) {
-    bias[t] = b_ih[t];
-    bias[3 * H + t] = b_hh[t];
-  }
+  fill_gate_bias(bias, b_ih, b_hh, H);
   if (threadIdx.x == 0) {
     for (int i = 0; i < 2; ++i) {
       mbar_init(&b->t_full[i], 1);
@@ -672,7 +695,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   __shared__ Bars bars;
-  __shared__ float bias[6 * H];
+  __shared__ __align__(16) float bias[4 * H];
   volatile int* abort = &bars.abort;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   setup(&bars, bias, b_ih, b_hh, warp);
@@ -764,18 +787,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           uint32_t pk[4];
 #pragma unroll
-          for (int j = 0; j < 8; j += 2) {
-            float o[2];
+          for (int q = 0; q < 2; ++q) {
+            const GateBias gb = gate_bias(bias, H, h + 4 * q);
+            float o[4];
 #pragma unroll
-            for (int u = 0; u < 2; ++u) {
-              const int c = h + j + u;
-              const float rr = sigm(__uint_as_float(vr[j + u]) + bias[c] + bias[3 * H + c]);
-              const float zz = sigm(__uint_as_float(vz[j + u]) + bias[H + c] + bias[4 * H + c]);
-              const float nn = tanh_fast(__uint_as_float(vn[j + u]) + bias[2 * H + c] +
-                                         rr * (__uint_as_float(vh[j + u]) + bias[5 * H + c]));
-              o[u] = real ? (1.f - zz) * nn + zz * e[j + u] : 0.f;
+            for (int u = 0; u < 4; ++u) {
+              const int j = 4 * q + u;
+              const float rr = sigm(__uint_as_float(vr[j]) + f4(gb.r, u));
+              const float zz = sigm(__uint_as_float(vz[j]) + f4(gb.z, u));
+              const float nn = tanh_fast(__uint_as_float(vn[j]) + f4(gb.in, u) +
+                                         rr * (__uint_as_float(vh[j]) + f4(gb.hn, u)));
+              o[u] = real ? (1.f - zz) * nn + zz * e[j] : 0.f;
             }
-            pk[j / 2] = pk2(o[0], o[1]);
+            pk[2 * q] = pk2(o[0], o[1]);
+            pk[2 * q + 1] = pk2(o[2], o[3]);
           }
           *reinterpret_cast<uint4*>(En + (size_t)row * H + h) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
           if (EnT) store_T4(EnT, ld_T, row, h, pk);
@@ -811,7 +836,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   __shared__ Bars bars;
-  __shared__ float bias[6 * H];
+  __shared__ __align__(16) float bias[4 * H];
   volatile int* abort = &bars.abort;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   setup(&bars, bias, b_ih, b_hh, warp);
@@ -931,14 +956,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int q = 0; q < 2; ++q) {
             const float4 gv = g4[q];
             const float gg[4] = {gv.x, gv.y, gv.z, gv.w};
+            const GateBias gb = gate_bias(bias, H, h + 4 * q);
             float dr[4], dz[4], dn[4], dhn[4];
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
-              const int j = 4 * q + u, c = h + j;
-              const float rr = sigm(__uint_as_float(vr[j]) + bias[c] + bias[3 * H + c]);
-              const float zz = sigm(__uint_as_float(vz[j]) + bias[H + c] + bias[4 * H + c]);
-              const float ghn = __uint_as_float(vh[j]) + bias[5 * H + c];
-              const float nn = tanh_fast(__uint_as_float(vn[j]) + bias[2 * H + c] + rr * ghn);
+              const int j = 4 * q + u;
+              const float rr = sigm(__uint_as_float(vr[j]) + f4(gb.r, u));
+              const float zz = sigm(__uint_as_float(vz[j]) + f4(gb.z, u));
+              const float ghn = __uint_as_float(vh[j]) + f4(gb.hn, u);
+              const float nn = tanh_fast(__uint_as_float(vn[j]) + f4(gb.in, u) + rr * ghn);
               const float gr = real ? gg[u] : 0.f;
               const float an = gr * (1.f - zz) * (1.f - nn * nn);
               dn[u] = an;
