@@ -71,16 +71,18 @@ template <int H, int S>
 struct Cfg {
   // H > 64 runs as H / 64 passes over 64-column slices of the state: pass hh contracts the band
   // with columns 64 hh .. 64 hh + 63 of E and multiplies the result by rows 64 hh .. of W_p, into Y
-  static constexpr int NH = H / 64;
+  // (H = 32: one pass over a 32-column slice)
+  static constexpr int SW = H < 64 ? H : 64;                  // state columns per pass
+  static constexpr int NH = H / SW;
   static constexpr int C1 = band_chunks(S);                   // 128-column chunks per type
-  static constexpr int ATOM_X = 64 * 128;                     // 64 nodes x 64 state columns
+  static constexpr int ATOM_X = SW * 128;                     // 64 nodes x SW state columns
   static constexpr int XWIN = 2 * C1 * ATOM_X;                // one half's window, 64-node atoms
   static constexpr int NXB = XWIN <= 48 * 1024 ? 2 : 1;       // state-window buffers
   static constexpr int NW = 2;                                // W ring stages
   // W stages hold K-columns of W_p^T as fp32 (tf32 operand) in 32-column atoms of H rows: a job's
   // 64 K-columns in one stage, or at H = 256 (64 KB) in two stages of one atom
-  static constexpr int WK = H <= 128 ? 64 : 32;               // K-columns per stage
-  static constexpr int WJ = 64 / WK;                          // stages per job
+  static constexpr int WK = H <= 128 ? SW : 32;               // K-columns per stage
+  static constexpr int WJ = SW / WK;                          // stages per job
   static constexpr int WSTAGE = (WK / 32) * H * 128;
   static constexpr int DEG = kTile * 128;                     // 128 rows x 64 bf16
   static constexpr int NDEG = NH > 1 ? 1 : 2;                 // deg buffers
@@ -98,8 +100,8 @@ struct Cfg {
   // a job's band products overlap the previous job's W product, then the A-tile slots
   static constexpr int NB = 2;
   static constexpr int YCOL = 0;
-  static constexpr int D1COL0 = H;
-  static constexpr int ACOL = H + NB * 64;
+  static constexpr int D1COL0 = H < 64 ? 64 : H;              // units start 64-column aligned
+  static constexpr int ACOL = D1COL0 + NB * 64;
   static constexpr int NA = (512 - ACOL) / 64;
   // a job's chunks come in CG-chunk groups (one barrier wait each), G groups per job; a group and
   // one more A tile must fit in the NA slots (H = 256 has two slots: one chunk per group)
@@ -108,7 +110,7 @@ struct Cfg {
   static constexpr int NT = (8 / G) * G;                      // per-group barrier ring
   static constexpr int NE = 2;                                // expander warpgroups
   static constexpr int THREADS = 128 * (2 + NE);
-  static_assert(H == 64 || H == 128 || H == 256, "state size");
+  static_assert(H == 32 || H == 64 || H == 128 || H == 256, "state size");
   static_assert(C1 % CG == 0 && NT % G == 0, "chunk groups");
   static_assert(NA >= CG + 1 && NA <= 8, "one group of A tiles and one more must fit");
   static_assert(NM >= 2 && NM <= 8, "mask ring");
@@ -264,7 +266,7 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
         mbar_expect_tx(&bars->x_full[xb], C::XWIN);
         for (int a = 0; a < 2 * C::C1; ++a)
           tma_load_2d(xwin + xb * C::XWIN + a * C::ATOM_X, &tm_x, &bars->x_full[xb],
-                      ws + a * kAtom, 64 * hh);
+                      ws + a * kAtom, C::SW * hh);
         // per job: K-columns 64 hh .. 64 hh + 63 of W_p^T in WJ stages of WK / 32 atoms
         for (int p = 0; p < P && ok; ++p)
           for (int wj = 0; wj < C::WJ; ++wj, ++widx) {
@@ -277,7 +279,7 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
             mbar_expect_tx(&bars->w_full[ws2], C::WSTAGE);
             for (int a = 0; a < C::WK / 32; ++a)
               tma_load_2d(wring + ws2 * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws2],
-                          64 * hh + C::WK * wj + 32 * a, p * H);
+                          C::SW * hh + C::WK * wj + 32 * a, p * H);
           }
       }
     }
@@ -319,10 +321,10 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
         }
   } else if (warp == 1) {
     // ------------------------------------------------------------------ band-product issuer
-    // pre_p = sum over the window chunks of A_{tile,p,j} X_j (N = 64): one t_full wait per group
+    // pre_p = sum over the window chunks of A_{tile,p,j} X_j (N = SW): one t_full wait per group
     // of chunks, then an unbroken MMA stream
     const bool leader = elect_one_sync();
-    constexpr uint32_t idesc = idesc_bf16_f32(kTile, 64);
+    constexpr uint32_t idesc = idesc_bf16_f32(kTile, C::SW);
     uint32_t c = 0, slot = 0, gi = 0, xi = 0;
     // expander group of chunk x + NA (the next user of the slot chunk x frees): job (x + NA) / C1
     // mod 2, kept as a group and a position within the job
@@ -479,25 +481,22 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
         if (!mbar_wait(&bars->d1_full[b], (c / C::NB) & 1, status, 401, abort, 64)) { ok = false; break; }
         tc_fence_after();
         const uint32_t col = tmem + lane_base + C::D1COL0 + b * 64;
-        uint32_t v[32], w[32];
+        uint32_t v[C::SW];
         tmem_ld32(col, v);
-        tmem_ld32(col + 32, w);
+        if constexpr (C::SW > 32) tmem_ld32(col + 32, v + 32);
         tmem_wait_ld();
         // pre_p stays fp32 for the tf32 product: release the unit before the stores
         tc_fence_before();
         warp_arrive(&bars->t_full[((c + C::NB) * C::G) % C::NT]);
-        uint32_t pk[32];
+        uint32_t pk[C::SW / 2];
 #pragma unroll
-        for (int j = 0; j < 16; ++j)
+        for (int j = 0; j < C::SW / 2; ++j)
           pk[j] = pack_bf16(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-          pk[16 + j] = pack_bf16(__uint_as_float(w[2 * j]), __uint_as_float(w[2 * j + 1]));
         // dM_p (bf16) transposed: dMT[(p*H + h) * ld_mt + row]
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
+        for (int j = 0; j < C::SW / 2; ++j) {
           const uint32_t w2 = pk[j];
-          __nv_bfloat16* d = dMT + ((size_t)p * H + 64 * hh + 2 * j) * ld_mt + row;
+          __nv_bfloat16* d = dMT + ((size_t)p * H + C::SW * hh + 2 * j) * ld_mt + row;
           d[0] = __ushort_as_bfloat16((unsigned short)(w2 & 0xFFFFu));
           d[ld_mt] = __ushort_as_bfloat16((unsigned short)(w2 >> 16));
         }
@@ -671,7 +670,7 @@ cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap&
   return e;
 }
 
-// The shapes with a tensor-core kernel: H in {64, 128} at S in {32, 64, 128, 256}; H = 256 at
+// The shapes with a tensor-core kernel: H in {32, 64, 128} at S in {32, 64, 128, 256}; H = 256 at
 // S in {32, 64, 128} (its state-slice window at S = 256 leaves no room for the mask ring).
 template <int H, bool BWD>
 cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
@@ -742,7 +741,7 @@ bool make_map_3d(CUtensorMap* m, const void* base, uint64_t batch, uint64_t rows
 
 bool band_tc_supported(const bg_plan* p, int dtype, int H) {
   if (!p || dtype != 1 || p->P > 32 || p->n_pad() % kTile) return false;
-  const bool shape = ((H == 64 || H == 128) &&
+  const bool shape = ((H == 32 || H == 64 || H == 128) &&
                       (p->S == 32 || p->S == 64 || p->S == 128 || p->S == 256)) ||
                      (H == 256 && (p->S == 32 || p->S == 64 || p->S == 128));
   return shape && p->d_maskI && p->d_maskTI && p->d_deg2 && p->max_deg <= 256 &&
@@ -783,10 +782,13 @@ cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, i
                              int* status, cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw, tdeg, tb2;
-  if (!make_map_ld(&tx, XT, H, n, ld_x, 64) || !make_map_w(&tw, Wk, P, H) ||
+  if (!make_map_ld(&tx, XT, H, n, ld_x, H < 64 ? H : 64) || !make_map_w(&tw, Wk, P, H) ||
       !make_map(&tdeg, p->d_deg2, n, 64, kTile) || !make_map(&tb2, b2T ? b2T : XT, H, 64, H))
     return cudaErrorInvalidValue;
   const int has_bias = b2T != nullptr;
+  if (H == 32)
+    return launch<32, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, has_bias,
+                             0, status, st);
   if (H == 64)
     return launch<64, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, has_bias,
                              0, status, st);
@@ -802,8 +804,11 @@ cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, 
                              int64_t ld_mt, int* status, cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw;
-  if (!make_map_ld(&tx, dYT, H, n, ld_y, 64) || !make_map_w(&tw, Wk, P, H))
+  if (!make_map_ld(&tx, dYT, H, n, ld_y, H < 64 ? H : 64) || !make_map_w(&tw, Wk, P, H))
     return cudaErrorInvalidValue;
+  if (H == 32)
+    return launch<32, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
+                            status, st);
   if (H == 64)
     return launch<64, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
                             status, st);

@@ -23,9 +23,9 @@ def built():
 
 def _tc_shape(c: Case) -> bool:
     """Shapes the fused tensor-core band kernels carry: bf16, P <= 32, whole 128-row tiles,
-    H in {64, 128} at S in {32, 64, 128, 256}, H = 256 at S in {32, 64, 128}."""
+    H in {32, 64, 128} at S in {32, 64, 128, 256}, H = 256 at S in {32, 64, 128}."""
     return (c.dtype == "bf16" and c.P <= 32 and c.N % 128 == 0 and
-            ((c.H in (64, 128) and c.S in (32, 64, 128, 256)) or
+            ((c.H in (32, 64, 128) and c.S in (32, 64, 128, 256)) or
              (c.H == 256 and c.S in (32, 64, 128))))
 
 
@@ -96,7 +96,8 @@ def test_propagate_fp32_config1():
 @pytest.mark.parametrize("S,H,whole", [(128, 64, 0), (64, 64, 1), (32, 32, 0), (256, 128, 0),
                                        (128, 256, 0), (256, 64, 1), (32, 64, 1), (64, 64, 0),
                                        (128, 128, 0), (64, 128, 1), (32, 128, 1),
-                                       (64, 256, 1), (32, 256, 1), (128, 96, 0)])
+                                       (64, 256, 1), (32, 256, 1), (128, 96, 0),
+                                       (128, 32, 0), (64, 32, 1), (256, 32, 0)])
 def test_propagate_bf16_packed_batch(S, H, whole):
     """Several graphs packed into several block-rows with a ragged tail (`whole`: capacity padded
     to whole 128-row tiles, as the tensor-core kernels need below S = 128)."""
@@ -164,12 +165,12 @@ def _ggnn(c: Case, T, seed=3):
                                                ("bf16", 2, 128, 128, 0), ("bf16", 2, 32, 32, 0),
                                                ("bf16", 2, 128, 256, 0), ("bf16", 2, 256, 64, 1),
                                                ("bf16", 2, 256, 128, 0), ("bf16", 3, 64, 128, 1),
-                                               ("bf16", 2, 32, 128, 0),
+                                               ("bf16", 2, 32, 128, 0), ("bf16", 2, 128, 32, 0),
                                                ("bf16", 3, 64, 64, 1), ("bf16", 2, 32, 64, 1)])
 def test_ggnn_fwd_bwd(dtype, T, S, H, whole):
     """Every kernel family of the GGNN step: SIMT (fp32), tensor-core GEMMs around the SIMT band
     sums (ragged tiles: H = 32, and H = 128 at S = 32), the band kernel with the tensor-core GEMM
-    GRU (H = 256), fused band and GRU kernels at H = 64 (S = 32, 64, 256) and H = 128 (S = 64,
+    GRU (H = 32, 256), fused band and GRU kernels at H = 64 (S = 32, 64, 256) and H = 128 (S = 64,
     128, 256; weights streamed through the GRU kernels' piece ring)."""
     gs = synth.gen_batch(5, 60, 300, 10, True, max(8, S // 2), max(8, S // 3), 2.0, 41)
     c = Case(gs, 20, S, H, dtype, seed=9, cap=_cap_whole_tiles(gs, S) if whole else 0)
