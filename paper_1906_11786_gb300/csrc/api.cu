@@ -440,11 +440,11 @@ size_t saved_Y_off(const bg_plan* p, bg_dtype dt, int H, int T, int t) {
   return saved_E_off(p, dt, H, T + 1) + (size_t)t * al(sizeof(float) * (size_t)p->n_pad() * H);
 }
 
-// ---- fused tensor-core GGNN steps (bf16, H in {64, 128}, P <= 32)
-// Shapes of the fused GGNN path (tensor-core band and GRU kernels): bf16, H in {64, 128},
+// ---- fused tensor-core GGNN steps (bf16, H in {32, 64, 128}, P <= 32)
+// Shapes of the fused GGNN path (tensor-core band and GRU kernels): bf16, H in {32, 64, 128},
 // P <= 32, a block size the band kernel has, whole 128-row tiles.
 bool tc_shape(const bg_plan* p, bg_dtype dt, int H) {
-  return p && dt == BG_BF16 && (H == 64 || H == 128) && p->P <= 32 &&
+  return p && dt == BG_BF16 && (H == 32 || H == 64 || H == 128) && p->P <= 32 &&
          (p->S == 32 || p->S == 64 || p->S == 128 || p->S == 256) && p->n_pad() % 128 == 0;
 }
 bool tc_ggnn(const bg_plan* p, bg_dtype dt, int H) {

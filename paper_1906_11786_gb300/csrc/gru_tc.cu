@@ -32,10 +32,13 @@ using namespace tc;
 
 namespace {
 
-constexpr int kH = 64;        // state size handled by these kernels
-constexpr int kEpiWarps = 16; // four epilogue warpgroups, 16 state columns each
+// The kernels below take H = KH in {32, 64}: the state fits one 64-column (128-byte) swizzle atom
+// of the tile, whose columns KH .. 63 the tensor maps fill with zeros at KH = 32, and only the
+// first KH / 16 K steps are issued.
+constexpr int kEpiWarps = 16; // four epilogue warpgroups of up to 16 state columns each
 constexpr int kThreads = 128 + 32 * kEpiWarps;  // warp 0 TMA, warp 1 MMA, warps 4-19 epilogue
-constexpr int kAcc = 4 * kH;  // TMEM columns per accumulator set
+template <int KH>
+__host__ __device__ constexpr int epi_warps() { return 4 * (KH / 16); }  // warps with columns
 
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
   asm volatile(
@@ -149,10 +152,12 @@ __device__ __forceinline__ void store_T8(__nv_bfloat16* dst, int64_t ld, int row
   }
 }
 
+template <int KH>
 struct GruSmem {
-  static constexpr int TILE = 128 * 128;  // 128 rows x 64 bf16
-  static constexpr int G = 128 * kH * 4;  // 128 rows x 64 fp32 (incoming state gradient, backward)
-  static constexpr int W = 3 * kH * 128;  // [3H][H] bf16 (also [H][3H] as three 64-column atoms)
+  static constexpr int TILE = 128 * 128;  // 128 rows x 64 bf16 (columns >= KH zero)
+  static constexpr int G = 128 * KH * 4;  // 128 rows x KH fp32 (incoming state gradient, backward)
+  static constexpr int W = 3 * KH * 128;  // [3H][64] bf16 (also [H][3H] as 64-column atoms)
+  static constexpr int WT_ATOMS = (3 * KH + 63) / 64;
   static constexpr int FWD_T = 2 * W;     // tile ring after W_ih, W_hh
   static constexpr int BWD_T = 4 * W;     // tile ring after W_ih, W_hh, W_ih^T, W_hh^T
   static constexpr int FWD_STAGE = 2 * TILE;      // Y, E
@@ -162,6 +167,7 @@ struct GruSmem {
   static constexpr int FWD = FWD_T + 2 * FWD_STAGE + 1024;
   static constexpr int BWD = BWD_T + 2 * BWD_STAGE + 1024;
   static_assert(BWD + 2048 <= 232448, "shared memory");
+  static_assert(WT_ATOMS * KH * 128 <= W, "transposed weights");
 };
 
 struct GruBars {
@@ -171,32 +177,34 @@ struct GruBars {
   int abort;
 };
 
-// Issues [r|z], Wi_n x, Wh_n h for one tile into the accumulator set at `acc` (K = H = 64).
+// Issues [r|z], Wi_n x, Wh_n h for one tile into the accumulator set at `acc` (K = H).
+template <int KH>
 __device__ __forceinline__ void gru_gate_mmas(uint32_t acc, uint32_t sY, uint32_t sE, uint32_t sWih,
                                               uint32_t sWhh) {
-  constexpr uint32_t id_rz = idesc_bf16_f32(128, 2 * kH), id_h = idesc_bf16_f32(128, kH);
+  constexpr uint32_t id_rz = idesc_bf16_f32(128, 2 * KH), id_h = idesc_bf16_f32(128, KH);
 #pragma unroll
-  for (int kk = 0; kk < 4; ++kk) {
+  for (int kk = 0; kk < KH / 16; ++kk) {
     const uint64_t aY = desc_sw128_kmajor(sY + kk * 32), aE = desc_sw128_kmajor(sE + kk * 32);
     mma_ss(acc + 0, aY, desc_sw128_kmajor(sWih + kk * 32), id_rz, kk > 0);
     mma_ss(acc + 0, aE, desc_sw128_kmajor(sWhh + kk * 32), id_rz, 1u);
-    mma_ss(acc + 2 * kH, aY, desc_sw128_kmajor(sWih + 2 * kH * 128 + kk * 32), id_h, kk > 0);
-    mma_ss(acc + 3 * kH, aE, desc_sw128_kmajor(sWhh + 2 * kH * 128 + kk * 32), id_h, kk > 0);
+    mma_ss(acc + 2 * KH, aY, desc_sw128_kmajor(sWih + 2 * KH * 128 + kk * 32), id_h, kk > 0);
+    mma_ss(acc + 3 * KH, aE, desc_sw128_kmajor(sWhh + 2 * KH * 128 + kk * 32), id_h, kk > 0);
   }
 }
 
 // Common prologue: barrier init, bias copy, TMEM allocation (512 columns: two accumulator sets).
+template <int KH>
 __device__ __forceinline__ void gru_setup(GruBars* b, float* bias, const float* b_ih,
                                           const float* b_hh, int warp) {
-  fill_gate_bias(bias, b_ih, b_hh, kH);
+  fill_gate_bias(bias, b_ih, b_hh, KH);
   if (threadIdx.x == 0) {
     mbar_init(&b->w_full, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&b->t_full[i], 1);
-      mbar_init(&b->t_empty[i], kEpiWarps);
+      mbar_init(&b->t_empty[i], epi_warps<KH>());
       mbar_init(&b->acc_full[i], 1);
-      mbar_init(&b->acc_empty[i], kEpiWarps);
-      mbar_init(&b->ops_ready[i], kEpiWarps);
+      mbar_init(&b->acc_empty[i], epi_warps<KH>());
+      mbar_init(&b->ops_ready[i], epi_warps<KH>());
       mbar_init(&b->ph2_full[i], 1);
     }
     mbar_init(&b->drain, 1);
@@ -215,7 +223,8 @@ __device__ __forceinline__ void gru_setup(GruBars* b, float* bias, const float* 
 }
 
 // Tile producer shared by both kernels: two-stage ring of (Y, E) tiles and, backward, the fp32
-// incoming gradient tile (two 32-column boxes with the 128-byte swizzle).
+// incoming gradient tile (KH / 32 boxes of 32 columns with the 128-byte swizzle).
+template <int KH>
 __device__ __forceinline__ void gru_produce_tiles(GruBars* b, uint8_t* ring, int stage,
                                                   const CUtensorMap* tY, const CUtensorMap* tE,
                                                   const CUtensorMap* tG, int n_tiles, int* status,
@@ -229,13 +238,13 @@ __device__ __forceinline__ void gru_produce_tiles(GruBars* b, uint8_t* ring, int
     if (!mbar_wait(&b->t_empty[s], ((i >> 1) & 1) ^ 1, status, 611, abort, 64)) break;
     ++issued[s];
     uint8_t* st = ring + s * stage;
-    mbar_expect_tx(&b->t_full[s], 2 * GruSmem::TILE + (tG ? GruSmem::G : 0));
+    using SM = GruSmem<KH>;
+    mbar_expect_tx(&b->t_full[s], 2 * SM::TILE + (tG ? SM::G : 0));
     tma_load_2d(st, tY, &b->t_full[s], 0, t * 128);
-    tma_load_2d(st + GruSmem::TILE, tE, &b->t_full[s], 0, t * 128);
-    if (tG) {
-      tma_load_2d(st + 2 * GruSmem::TILE, tG, &b->t_full[s], 0, t * 128);
-      tma_load_2d(st + 2 * GruSmem::TILE + GruSmem::G / 2, tG, &b->t_full[s], 32, t * 128);
-    }
+    tma_load_2d(st + SM::TILE, tE, &b->t_full[s], 0, t * 128);
+    if (tG)
+      for (int a = 0; a < KH / 32; ++a)
+        tma_load_2d(st + 2 * SM::TILE + a * 128 * 128, tG, &b->t_full[s], 32 * a, t * 128);
   }
   if (*abort)
     for (int s = 0; s < 2; ++s)
@@ -243,6 +252,7 @@ __device__ __forceinline__ void gru_produce_tiles(GruBars* b, uint8_t* ring, int
       }
 }
 
+template <int KH>
 __global__ void __launch_bounds__(kThreads, 1)
     k_gru_fwd_tc(const __grid_constant__ CUtensorMap tY, const __grid_constant__ CUtensorMap tE,
                  const __grid_constant__ CUtensorMap tWih, const __grid_constant__ CUtensorMap tWhh,
@@ -253,18 +263,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   __shared__ GruBars bars;
-  __shared__ __align__(16) float bias[4 * kH];
+  __shared__ __align__(16) float bias[4 * KH];
+  using SM = GruSmem<KH>;
+  constexpr int kAcc = 4 * KH;  // TMEM columns per accumulator set
   volatile int* abort = &bars.abort;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  gru_setup(&bars, bias, b_ih, b_hh, warp);
+  gru_setup<KH>(&bars, bias, b_ih, b_hh, warp);
   const uint32_t tmem = bars.tmem_slot;
-  uint8_t* ring = smem + GruSmem::FWD_T;
+  uint8_t* ring = smem + SM::FWD_T;
 
   if (warp == 0 && lane == 0) {
-    mbar_expect_tx(&bars.w_full, 2 * GruSmem::W);
+    mbar_expect_tx(&bars.w_full, 2 * SM::W);
     tma_load_2d(smem, &tWih, &bars.w_full, 0, 0);
-    tma_load_2d(smem + GruSmem::W, &tWhh, &bars.w_full, 0, 0);
-    gru_produce_tiles(&bars, ring, GruSmem::FWD_STAGE, &tY, &tE, nullptr, n_tiles, status, abort);
+    tma_load_2d(smem + SM::W, &tWhh, &bars.w_full, 0, 0);
+    gru_produce_tiles<KH>(&bars, ring, SM::FWD_STAGE, &tY, &tE, nullptr, n_tiles, status, abort);
     if (*abort)
       for (uint32_t k = 0; k < (1u << 22) && !mbar_try(&bars.w_full, 0); ++k) {
       }
@@ -277,10 +289,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(&bars.t_full[s], (i >> 1) & 1, status, 613, abort)) break;
         if (!mbar_wait(&bars.acc_empty[a], ((i >> 1) & 1) ^ 1, status, 614, abort)) break;
         tc_fence_after();
-        const uint32_t sY = smem_u32(ring + s * 2 * GruSmem::TILE);
+        const uint32_t sY = smem_u32(ring + s * 2 * SM::TILE);
         if (leader) {
-          gru_gate_mmas(tmem + a * kAcc, sY, sY + GruSmem::TILE, smem_u32(smem),
-                        smem_u32(smem + GruSmem::W));
+          gru_gate_mmas<KH>(tmem + a * kAcc, sY, sY + SM::TILE, smem_u32(smem),
+                        smem_u32(smem + SM::W));
           tc_commit(&bars.acc_full[a]);
         }
         __syncwarp();
@@ -290,7 +302,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
     for (uint32_t k = 0; k < (1u << 24) && !mbar_try(&bars.drain, 0); ++k) {
     }
-  } else if (warp >= 4) {
+  } else if (warp >= 4 && (warp - 4) / 4 < KH / 16) {
     grid_dep_wait();  // outputs may still be in use by the previous kernel
     const int g = (warp - 4) / 4, h0 = 16 * g;
     const int r = (warp & 3) * 32 + lane;
@@ -301,7 +313,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!mbar_wait(&bars.acc_full[a], (i >> 1) & 1, status, 615, abort, 64)) break;
       tc_fence_after();
       const uint32_t acc = tmem + lb + a * kAcc;
-      const uint8_t* etile = ring + s * 2 * GruSmem::TILE + GruSmem::TILE;
+      const uint8_t* etile = ring + s * 2 * SM::TILE + SM::TILE;
       const int row = t * 128 + r;
       const bool real = row < n_real;
 #pragma unroll
@@ -309,9 +321,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int hs = h0 + 8 * hh;
         uint32_t vr[8], vz[8], vn[8], vh[8];
         tmem_ld8(acc + hs, vr);
-        tmem_ld8(acc + kH + hs, vz);
-        tmem_ld8(acc + 2 * kH + hs, vn);
-        tmem_ld8(acc + 3 * kH + hs, vh);
+        tmem_ld8(acc + KH + hs, vz);
+        tmem_ld8(acc + 2 * KH + hs, vn);
+        tmem_ld8(acc + 3 * KH + hs, vh);
         tmem_wait_ld();
         float e[8];
         read_sw128_row8(etile, r, hs, e);
@@ -324,7 +336,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t pk[4];
 #pragma unroll
         for (int q = 0; q < 2; ++q) {
-          const GateBias gb = gate_bias(bias, kH, hs + 4 * q);
+          const GateBias gb = gate_bias(bias, KH, hs + 4 * q);
           float o[4];
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
@@ -338,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           pk[2 * q] = pk2(o[0], o[1]);
           pk[2 * q + 1] = pk2(o[2], o[3]);
         }
-        *reinterpret_cast<uint4*>(En + (size_t)row * kH + hs) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        *reinterpret_cast<uint4*>(En + (size_t)row * KH + hs) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
         if (EnT) store_T4(EnT, ld_T, row, hs, pk);
       }
     }
@@ -356,14 +368,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 // gate) after the in-place rewrite.  Columns h in [32c + 16sb, +16) of chunk c, sub-chunk sb, are
 // read and then overwritten as: r window [32c + 16sb, +16) = (dgi_r | dgi_z) pairs, z window
 // [H + 32c + 16sb, +16) = (dgi_n | dgh_n) pairs; dgh_r = dgi_r and dgh_z = dgi_z.
+template <int KH>
 __device__ __forceinline__ uint32_t dg_col(int kk, bool hidden) {
-  const int gate = kk / 4, hh = (kk % 4) * 16, c = hh / 32, sb = (hh % 32) / 16;
+  const int gate = kk / (KH / 16), hh = (kk % (KH / 16)) * 16, c = hh / 32, sb = (hh % 32) / 16;
   const int base = c * 32 + sb * 16;
   if (gate == 0) return base;
   if (gate == 1) return base + 8;
-  return kH + base + (hidden ? 8 : 0);
+  return KH + base + (hidden ? 8 : 0);
 }
 
+template <int KH>
 __global__ void __launch_bounds__(kThreads, 1)
     k_gru_bwd_tc(const __grid_constant__ CUtensorMap tY, const __grid_constant__ CUtensorMap tE,
                  const __grid_constant__ CUtensorMap tWih, const __grid_constant__ CUtensorMap tWhh,
@@ -378,29 +392,31 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   __shared__ GruBars bars;
-  __shared__ __align__(16) float bias[4 * kH];
+  __shared__ __align__(16) float bias[4 * KH];
+  using SM = GruSmem<KH>;
+  constexpr int kAcc = 4 * KH;  // TMEM columns per accumulator set
   volatile int* abort = &bars.abort;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  gru_setup(&bars, bias, b_ih, b_hh, warp);
+  gru_setup<KH>(&bars, bias, b_ih, b_hh, warp);
   const uint32_t tmem = bars.tmem_slot;
-  uint8_t* ring = smem + GruSmem::BWD_T;
+  uint8_t* ring = smem + SM::BWD_T;
 
   if (warp == 0 && lane == 0) {
-    mbar_expect_tx(&bars.w_full, 4 * GruSmem::W);
+    mbar_expect_tx(&bars.w_full, 2 * SM::W + 2 * SM::WT_ATOMS * KH * 128);
     tma_load_2d(smem, &tWih, &bars.w_full, 0, 0);
-    tma_load_2d(smem + GruSmem::W, &tWhh, &bars.w_full, 0, 0);
-    for (int a = 0; a < 3; ++a) {
-      tma_load_2d(smem + 2 * GruSmem::W + a * kH * 128, &tWihT, &bars.w_full, a * 64, 0);
-      tma_load_2d(smem + 3 * GruSmem::W + a * kH * 128, &tWhhT, &bars.w_full, a * 64, 0);
+    tma_load_2d(smem + SM::W, &tWhh, &bars.w_full, 0, 0);
+    for (int a = 0; a < SM::WT_ATOMS; ++a) {
+      tma_load_2d(smem + 2 * SM::W + a * KH * 128, &tWihT, &bars.w_full, a * 64, 0);
+      tma_load_2d(smem + 3 * SM::W + a * KH * 128, &tWhhT, &bars.w_full, a * 64, 0);
     }
-    gru_produce_tiles(&bars, ring, GruSmem::BWD_STAGE, &tY, &tE, &tG, n_tiles, status, abort);
+    gru_produce_tiles<KH>(&bars, ring, SM::BWD_STAGE, &tY, &tE, &tG, n_tiles, status, abort);
     if (*abort)
       for (uint32_t k = 0; k < (1u << 22) && !mbar_try(&bars.w_full, 0); ++k) {
       }
   } else if (warp == 1) {
     const bool leader = elect_one_sync();
-    constexpr uint32_t id_h = idesc_bf16_f32(128, kH);
-    const uint32_t sIT = smem_u32(smem + 2 * GruSmem::W), sHT = smem_u32(smem + 3 * GruSmem::W);
+    constexpr uint32_t id_h = idesc_bf16_f32(128, KH);
+    const uint32_t sIT = smem_u32(smem + 2 * SM::W), sHT = smem_u32(smem + 3 * SM::W);
     // dX = dgi W_ih, dH = dgh W_hh for tile j (accumulating into the freed n columns)
     auto phase2 = [&](int j) -> bool {
       const int a = j & 1;
@@ -409,10 +425,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (leader) {
         const uint32_t acc = tmem + a * kAcc;
 #pragma unroll
-        for (int kk = 0; kk < 12; ++kk) {
-          const uint32_t boff = (kk / 4) * kH * 128 + (kk % 4) * 32;
-          mma_ts(acc + 2 * kH, acc + dg_col(kk, false), desc_sw128_kmajor(sIT + boff), id_h, kk > 0);
-          mma_ts(acc + 3 * kH, acc + dg_col(kk, true), desc_sw128_kmajor(sHT + boff), id_h, kk > 0);
+        // K index 16 kk = gate * H + h of W^T: atom kk / 4, 32-byte step kk % 4
+        for (int kk = 0; kk < 3 * KH / 16; ++kk) {
+          const uint32_t boff = (kk / 4) * KH * 128 + (kk % 4) * 32;
+          mma_ts(acc + 2 * KH, acc + dg_col<KH>(kk, false), desc_sw128_kmajor(sIT + boff), id_h,
+                 kk > 0);
+          mma_ts(acc + 3 * KH, acc + dg_col<KH>(kk, true), desc_sw128_kmajor(sHT + boff), id_h,
+                 kk > 0);
         }
         tc_commit(&bars.ph2_full[a]);
       }
@@ -427,10 +446,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(&bars.t_full[s], (i >> 1) & 1, status, 623, abort)) break;
         if (!mbar_wait(&bars.acc_empty[a], ((i >> 1) & 1) ^ 1, status, 624, abort)) break;
         tc_fence_after();
-        const uint32_t sY = smem_u32(ring + s * GruSmem::BWD_STAGE);
+        const uint32_t sY = smem_u32(ring + s * SM::BWD_STAGE);
         if (leader) {
-          gru_gate_mmas(tmem + a * kAcc, sY, sY + GruSmem::TILE, smem_u32(smem),
-                        smem_u32(smem + GruSmem::W));
+          gru_gate_mmas<KH>(tmem + a * kAcc, sY, sY + SM::TILE, smem_u32(smem),
+                        smem_u32(smem + SM::W));
           tc_commit(&bars.acc_full[a]);
         }
         __syncwarp();
@@ -442,7 +461,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
     for (uint32_t k = 0; k < (1u << 24) && !mbar_try(&bars.drain, 0); ++k) {
     }
-  } else if (warp >= 4) {
+  } else if (warp >= 4 && (warp - 4) / 4 < KH / 16) {
     grid_dep_wait();  // outputs may still be in use by the previous kernel
     const int g = (warp - 4) / 4, h0 = 16 * g;
     const int r = (warp & 3) * 32 + lane;
@@ -455,8 +474,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!mbar_wait(&bars.acc_full[a], (i >> 1) & 1, status, 625, abort, 64)) break;
       tc_fence_after();
       const uint32_t acc = tmem + lb + a * kAcc;
-      const uint8_t* etile = ring + s * GruSmem::BWD_STAGE + GruSmem::TILE;
-      const uint8_t* gtile = etile + GruSmem::TILE;
+      const uint8_t* etile = ring + s * SM::BWD_STAGE + SM::TILE;
+      const uint8_t* gtile = etile + SM::TILE;
       float dhd[16];
       // packed gate gradients of both halves: the in-place rewrite below overwrites columns that
       // the second half still reads, so it waits until both halves are in registers
@@ -467,9 +486,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int hs = h0 + 8 * hh;
         uint32_t vr[8], vz[8], vn[8], vh[8];
         tmem_ld8(acc + hs, vr);
-        tmem_ld8(acc + kH + hs, vz);
-        tmem_ld8(acc + 2 * kH + hs, vn);
-        tmem_ld8(acc + 3 * kH + hs, vh);
+        tmem_ld8(acc + KH + hs, vz);
+        tmem_ld8(acc + 2 * KH + hs, vn);
+        tmem_ld8(acc + 3 * KH + hs, vh);
         tmem_wait_ld();
         float e[8];
         read_sw128_row8(etile, r, hs, e);
@@ -481,7 +500,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int q = 0; q < 2; ++q) {
           const float4 gv = g4[q];
           const float gg[4] = {gv.x, gv.y, gv.z, gv.w};
-          const GateBias gb = gate_bias(bias, kH, hs + 4 * q);
+          const GateBias gb = gate_bias(bias, KH, hs + 4 * q);
           float dr[4], dz[4], dn[4], dhn[4];
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
@@ -505,11 +524,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         // gate gradients transposed for the weight-gradient GEMM: rows o = gate*H + h
         store_T4(dgiT, ld_g, row, hs, p_r + o);
-        store_T4(dgiT + (size_t)kH * ld_g, ld_g, row, hs, p_z + o);
-        store_T4(dgiT + (size_t)2 * kH * ld_g, ld_g, row, hs, p_n + o);
+        store_T4(dgiT + (size_t)KH * ld_g, ld_g, row, hs, p_z + o);
+        store_T4(dgiT + (size_t)2 * KH * ld_g, ld_g, row, hs, p_n + o);
         store_T4(dghT, ld_g, row, hs, p_r + o);
-        store_T4(dghT + (size_t)kH * ld_g, ld_g, row, hs, p_z + o);
-        store_T4(dghT + (size_t)2 * kH * ld_g, ld_g, row, hs, p_hn + o);
+        store_T4(dghT + (size_t)KH * ld_g, ld_g, row, hs, p_z + o);
+        store_T4(dghT + (size_t)2 * KH * ld_g, ld_g, row, hs, p_hn + o);
       }
       // in-place rewrite into the columns just read (see dg_col): within the 16-column window h0,
       // r holds the 8 (dgi_r) pair columns then the 8 (dgi_z) ones, z the (dgi_n) then (dgh_n)
@@ -517,18 +536,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_st4(acc + h0 + 4, p_r + 4);
       tmem_st4(acc + h0 + 8, p_z);
       tmem_st4(acc + h0 + 12, p_z + 4);
-      tmem_st4(acc + kH + h0, p_n);
-      tmem_st4(acc + kH + h0 + 4, p_n + 4);
-      tmem_st4(acc + kH + h0 + 8, p_hn);
-      tmem_st4(acc + kH + h0 + 12, p_hn + 4);
+      tmem_st4(acc + KH + h0, p_n);
+      tmem_st4(acc + KH + h0 + 4, p_n + 4);
+      tmem_st4(acc + KH + h0 + 8, p_hn);
+      tmem_st4(acc + KH + h0 + 12, p_hn + 4);
       tmem_wait_st();
       tc_fence_before();
       warp_arrive(&bars.ops_ready[a]);
       if (!mbar_wait(&bars.ph2_full[a], (i >> 1) & 1, status, 626, abort, 64)) break;
       tc_fence_after();
       uint32_t vx[16], vd[16];
-      tmem_ld16(acc + 2 * kH + h0, vx);
-      tmem_ld16(acc + 3 * kH + h0, vd);
+      tmem_ld16(acc + 2 * KH + h0, vx);
+      tmem_ld16(acc + 3 * KH + h0, vd);
       tmem_wait_ld();
       tc_fence_before();
       warp_arrive(&bars.acc_empty[a]);
@@ -536,7 +555,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int j = 0; j < 8; ++j) px[j] = pk2(__uint_as_float(vx[2 * j]), __uint_as_float(vx[2 * j + 1]));
       store_T8(dXT, ld_x, row, h0, px);
-      float4* go = reinterpret_cast<float4*>(gout + (size_t)row * kH + h0);
+      float4* go = reinterpret_cast<float4*>(gout + (size_t)row * KH + h0);
 #pragma unroll
       for (int q = 0; q < 4; ++q)
         go[q] = make_float4(dhd[4 * q] + __uint_as_float(vd[4 * q]),
@@ -1046,7 +1065,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-bool gru_tc_supported(int H) { return H == kH || H == wide::H; }
+bool gru_tc_supported(int H) { return H == 32 || H == 64 || H == wide::H; }
 
 cudaError_t gru_fwd_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y,
                        const __nv_bfloat16* E, const __nv_bfloat16* W_ih,
@@ -1060,8 +1079,8 @@ cudaError_t gru_fwd_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y,
       !make_map_ld(&tWi, W_ih, 3 * H, H, H, w ? 64 : 3 * H) ||
       !make_map_ld(&tWh, W_hh, 3 * H, H, H, w ? 64 : 3 * H))
     return cudaErrorInvalidValue;
-  auto kern = w ? wide::k_gru_fwd : k_gru_fwd_tc;
-  const int smem = w ? wide::Smem::FWD : GruSmem::FWD;
+  auto kern = w ? wide::k_gru_fwd : H == 32 ? k_gru_fwd_tc<32> : k_gru_fwd_tc<64>;
+  const int smem = w ? wide::Smem::FWD : H == 32 ? GruSmem<32>::FWD : GruSmem<64>::FWD;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const int n_tiles = n_pad / 128;
@@ -1090,8 +1109,8 @@ cudaError_t gru_bwd_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y,
       !make_map_ld(&tWiT, W_ihT, H, 3 * H, 3 * H, H) ||
       !make_map_ld(&tWhT, W_hhT, H, 3 * H, 3 * H, H) || !make_map_f32(&tG, gin, n_pad, H, 128))
     return cudaErrorInvalidValue;
-  auto kern = w ? wide::k_gru_bwd : k_gru_bwd_tc;
-  const int smem = w ? wide::Smem::BWD : GruSmem::BWD;
+  auto kern = w ? wide::k_gru_bwd : H == 32 ? k_gru_bwd_tc<32> : k_gru_bwd_tc<64>;
+  const int smem = w ? wide::Smem::BWD : H == 32 ? GruSmem<32>::BWD : GruSmem<64>::BWD;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const int n_tiles = n_pad / 128;

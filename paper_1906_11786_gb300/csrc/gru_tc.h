@@ -1,4 +1,4 @@
-// Fused GRU forward / backward on tcgen05 (gru_tc.cu); state size H in {64, 128}.
+// Fused GRU forward / backward on tcgen05 (gru_tc.cu); state size H in {32, 64, 128}.
 #pragma once
 
 #include <cuda_bf16.h>

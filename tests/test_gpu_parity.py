@@ -166,12 +166,13 @@ def _ggnn(c: Case, T, seed=3):
                                                ("bf16", 2, 128, 256, 0), ("bf16", 2, 256, 64, 1),
                                                ("bf16", 2, 256, 128, 0), ("bf16", 3, 64, 128, 1),
                                                ("bf16", 2, 32, 128, 0), ("bf16", 2, 128, 32, 0),
-                                               ("bf16", 3, 64, 64, 1), ("bf16", 2, 32, 64, 1)])
+                                               ("bf16", 3, 64, 64, 1), ("bf16", 2, 32, 64, 1),
+                                               ("bf16", 3, 64, 32, 1)])
 def test_ggnn_fwd_bwd(dtype, T, S, H, whole):
     """Every kernel family of the GGNN step: SIMT (fp32), tensor-core GEMMs around the SIMT band
-    sums (ragged tiles: H = 32, and H = 128 at S = 32), the band kernel with the tensor-core GEMM
-    GRU (H = 32, 256), fused band and GRU kernels at H = 64 (S = 32, 64, 256) and H = 128 (S = 64,
-    128, 256; weights streamed through the GRU kernels' piece ring)."""
+    sums (ragged tiles: H = 32 at S = 32, and H = 128 at S = 32), the band kernel with the GEMM
+    GRU (H = 256), fused band and GRU kernels at H = 32 (S = 64, 128), H = 64 (S = 32, 64, 256) and
+    H = 128 (S = 64, 128, 256; weights streamed through the GRU kernels' piece ring)."""
     gs = synth.gen_batch(5, 60, 300, 10, True, max(8, S // 2), max(8, S // 3), 2.0, 41)
     c = Case(gs, 20, S, H, dtype, seed=9, cap=_cap_whole_tiles(gs, S) if whole else 0)
     assert L.band_uses_tensor_cores(c.plan, c.dtype, c.H) == _tc_shape(c)
