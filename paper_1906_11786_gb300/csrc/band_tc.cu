@@ -64,15 +64,16 @@ constexpr int kAtom = 64;      // bf16 per 128-byte swizzle row
 // Block size S: a 128-row tile sees a window of C1 128-column chunks of the state (and of its
 // bit tiles): rows [row0, row0 + 128) only couple to columns in block-rows kr - 1 .. kr + 1 of
 // their own block-row kr, which all lie in [ws, ws + 128 C1) with ws = (row0 / S) S - S.
-//   S <= 64: C1 = 2 (the tile spans 128 / S block-rows);  S = 128: C1 = 3;  S = 256: C1 = 6.
+//   S <= 64: C1 = 2 (the tile spans 128 / S block-rows);  S = 128: 3;  S = 256: 6;  S = 512: 12.
 __host__ __device__ constexpr int band_chunks(int S) { return S <= 64 ? 2 : 3 * (S / 128); }
 
 template <int H, int S>
 struct Cfg {
-  // H > 64 runs as H / 64 passes over 64-column slices of the state: pass hh contracts the band
-  // with columns 64 hh .. 64 hh + 63 of E and multiplies the result by rows 64 hh .. of W_p, into Y
-  // (H = 32: one pass over a 32-column slice)
-  static constexpr int SW = H < 64 ? H : 64;                  // state columns per pass
+  // H > SW runs as H / SW passes over SW-column slices of the state: pass hh contracts the band
+  // with columns SW hh .. SW hh + SW - 1 of E and multiplies the result by rows SW hh .. of W_p,
+  // into Y.  SW = 64, or 32 at H = 32 and at S = 512 (whose 1536-node window of 64 columns would
+  // take 192 KB)
+  static constexpr int SW = (H < 64 || S == 512) ? 32 : 64;   // state columns per pass
   static constexpr int NH = H / SW;
   static constexpr int C1 = band_chunks(S);                   // 128-column chunks per type
   static constexpr int ATOM_X = SW * 128;                     // 64 nodes x SW state columns
@@ -92,7 +93,9 @@ struct Cfg {
   static constexpr int OFF_DEG = OFF_W + NW * WSTAGE;
   static constexpr int OFF_B2 = OFF_DEG + NDEG * DEG;
   static constexpr int MSTAGE = C1 * kTile * 16;              // C1 chunks x 128 rows x 128 bits
-  static constexpr int NM = (C1 <= 3 ? 8 : 4) / NH;           // mask ring stages (one job each)
+  // mask ring stages (one job each): as many as fit beside the window, at least two
+  static constexpr int NM0 = (C1 <= 3 ? 8 : 4) / NH;
+  static constexpr int NM = C1 > 6 ? 2 : (NM0 > 2 ? NM0 : 2);
   static constexpr int OFF_M = OFF_B2 + B2;
   static constexpr int OFF_BAR = OFF_M + NM * MSTAGE;
   static constexpr int SMEM = OFF_BAR + 1024 + 1024;          // barriers + 1 KB alignment slack
@@ -670,8 +673,8 @@ cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap&
   return e;
 }
 
-// The shapes with a tensor-core kernel: H in {32, 64, 128} at S in {32, 64, 128, 256}; H = 256 at
-// S in {32, 64, 128} (its state-slice window at S = 256 leaves no room for the mask ring).
+// The shapes with a tensor-core kernel: H in {32, 64, 128} at S in {32, 64, 128, 256, 512}; H = 256
+// at S in {32, 64, 128} (its state-slice window at S = 256 leaves no room for the mask ring).
 template <int H, bool BWD>
 cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
                    const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
@@ -686,6 +689,9 @@ cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& t
     case 64: BG_BAND_S(64)
     case 256:
       if constexpr (H <= 128) { BG_BAND_S(256) }
+      return cudaErrorInvalidValue;
+    case 512:
+      if constexpr (H <= 128) { BG_BAND_S(512) }
       return cudaErrorInvalidValue;
     default: BG_BAND_S(128)
   }
@@ -742,7 +748,7 @@ bool make_map_3d(CUtensorMap* m, const void* base, uint64_t batch, uint64_t rows
 bool band_tc_supported(const bg_plan* p, int dtype, int H) {
   if (!p || dtype != 1 || p->P > 32 || p->n_pad() % kTile) return false;
   const bool shape = ((H == 32 || H == 64 || H == 128) &&
-                      (p->S == 32 || p->S == 64 || p->S == 128 || p->S == 256)) ||
+                      (p->S == 32 || p->S == 64 || p->S == 128 || p->S == 256 || p->S == 512)) ||
                      (H == 256 && (p->S == 32 || p->S == 64 || p->S == 128));
   return shape && p->d_maskI && p->d_maskTI && p->d_deg2 && p->max_deg <= 256 &&
          encode_fn() != nullptr;
@@ -782,7 +788,7 @@ cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, i
                              int* status, cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw, tdeg, tb2;
-  if (!make_map_ld(&tx, XT, H, n, ld_x, H < 64 ? H : 64) || !make_map_w(&tw, Wk, P, H) ||
+  if (!make_map_ld(&tx, XT, H, n, ld_x, (H < 64 || p->S == 512) ? 32 : 64) || !make_map_w(&tw, Wk, P, H) ||
       !make_map(&tdeg, p->d_deg2, n, 64, kTile) || !make_map(&tb2, b2T ? b2T : XT, H, 64, H))
     return cudaErrorInvalidValue;
   const int has_bias = b2T != nullptr;
@@ -804,7 +810,7 @@ cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, 
                              int64_t ld_mt, int* status, cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw;
-  if (!make_map_ld(&tx, dYT, H, n, ld_y, H < 64 ? H : 64) || !make_map_w(&tw, Wk, P, H))
+  if (!make_map_ld(&tx, dYT, H, n, ld_y, (H < 64 || p->S == 512) ? 32 : 64) || !make_map_w(&tw, Wk, P, H))
     return cudaErrorInvalidValue;
   if (H == 32)
     return launch<32, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
@@ -891,7 +897,7 @@ cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, c
 
 int band_tc_upload(bg_plan* p, cudaStream_t st) {
   const int S = p->S;
-  if (p->P > 32 || (S != 32 && S != 64 && S != 128 && S != 256)) return 0;
+  if (p->P > 32 || (S != 32 && S != 64 && S != 128 && S != 256 && S != 512)) return 0;
   const int K = p->K, P = p->P, W32 = p->W32;
   const size_t n = (size_t)K * S;
   if (n % kTile) return 0;

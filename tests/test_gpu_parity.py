@@ -23,9 +23,9 @@ def built():
 
 def _tc_shape(c: Case) -> bool:
     """Shapes the fused tensor-core band kernels carry: bf16, P <= 32, whole 128-row tiles,
-    H in {32, 64, 128} at S in {32, 64, 128, 256}, H = 256 at S in {32, 64, 128}."""
+    H in {32, 64, 128} at S in {32, 64, 128, 256, 512}, H = 256 at S in {32, 64, 128}."""
     return (c.dtype == "bf16" and c.P <= 32 and c.N % 128 == 0 and
-            ((c.H in (32, 64, 128) and c.S in (32, 64, 128, 256)) or
+            ((c.H in (32, 64, 128) and c.S in (32, 64, 128, 256, 512)) or
              (c.H == 256 and c.S in (32, 64, 128))))
 
 
@@ -97,7 +97,8 @@ def test_propagate_fp32_config1():
                                        (128, 256, 0), (256, 64, 1), (32, 64, 1), (64, 64, 0),
                                        (128, 128, 0), (64, 128, 1), (32, 128, 1),
                                        (64, 256, 1), (32, 256, 1), (128, 96, 0),
-                                       (128, 32, 0), (64, 32, 1), (256, 32, 0)])
+                                       (128, 32, 0), (64, 32, 1), (256, 32, 0),
+                                       (512, 64, 0), (512, 32, 0), (512, 128, 0)])
 def test_propagate_bf16_packed_batch(S, H, whole):
     """Several graphs packed into several block-rows with a ragged tail (`whole`: capacity padded
     to whole 128-row tiles, as the tensor-core kernels need below S = 128)."""
