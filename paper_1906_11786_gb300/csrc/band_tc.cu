@@ -507,46 +507,56 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
       if (!ok) break;
       if (!mbar_wait(&bars->y_full, i & 1, status, 402, abort, 64)) break;
       tc_fence_after();
+      // Y leaves TMEM in groups, each read completely before any global traffic of its own; after
+      // the last group's read the next tile may start accumulating.  Up to H = 64 one group, so
+      // the release does not wait on the accumulating backward's reads of the previous dE (wider
+      // groups at larger H measured slower: 32 columns there)
+      constexpr int YG = H <= 64 ? H : 32;
 #pragma unroll
-      for (int h0 = 0; h0 < H; h0 += 32) {
-        uint32_t v[32];
-        tmem_ld32(tmem + lane_base + C::YCOL + h0, v);
+      for (int g0 = 0; g0 < H; g0 += YG) {
+        uint32_t vg[YG];
+        tmem_ld32(tmem + lane_base + C::YCOL + g0, vg);
+        if constexpr (YG > 32) tmem_ld32(tmem + lane_base + C::YCOL + g0 + 32, vg + 32);
         tmem_wait_ld();
-        if (h0 + 32 >= H) {
-          // Y is in registers now: the next tile may start accumulating
+        if (g0 + YG >= H) {
           tc_fence_before();
           warp_arrive(&bars->y_empty);
         }
-        if (out) {
-          float4* o = reinterpret_cast<float4*>(out + (size_t)row * H + h0);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            float4 a = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
-                                   __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
-            if (accumulate) {
-              const float4 prev = o[j];
-              a.x += prev.x; a.y += prev.y; a.z += prev.z; a.w += prev.w;
+        for (int h1 = 0; h1 < YG; h1 += 32) {
+          const int h0 = g0 + h1;
+          const uint32_t* v = vg + h1;
+          if (out) {
+            float4* o = reinterpret_cast<float4*>(out + (size_t)row * H + h0);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              float4 a = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                     __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+              if (accumulate) {
+                const float4 prev = o[j];
+                a.x += prev.x; a.y += prev.y; a.z += prev.z; a.w += prev.w;
+              }
+              o[j] = a;
             }
-            o[j] = a;
           }
-        }
-        if (outb || outT) {
-          uint32_t pk[16];
+          if (outb || outT) {
+            uint32_t pk[16];
 #pragma unroll
-          for (int j = 0; j < 16; ++j)
-            pk[j] = pack_bf16(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
-          if (outb) {
-            uint4* ob = reinterpret_cast<uint4*>(outb + (size_t)row * H + h0);
+            for (int j = 0; j < 16; ++j)
+              pk[j] = pack_bf16(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+            if (outb) {
+              uint4* ob = reinterpret_cast<uint4*>(outb + (size_t)row * H + h0);
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
-              ob[j] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
-          }
-          if (outT) {
+              for (int j = 0; j < 4; ++j)
+                ob[j] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+            }
+            if (outT) {
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-              __nv_bfloat16* d = outT + (size_t)(h0 + 2 * j) * ld_outT + row;
-              d[0] = __ushort_as_bfloat16((unsigned short)(pk[j] & 0xFFFFu));
-              d[ld_outT] = __ushort_as_bfloat16((unsigned short)(pk[j] >> 16));
+              for (int j = 0; j < 16; ++j) {
+                __nv_bfloat16* d = outT + (size_t)(h0 + 2 * j) * ld_outT + row;
+                d[0] = __ushort_as_bfloat16((unsigned short)(pk[j] & 0xFFFFu));
+                d[ld_outT] = __ushort_as_bfloat16((unsigned short)(pk[j] >> 16));
+              }
             }
           }
         }
