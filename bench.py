@@ -282,20 +282,61 @@ class OursStep:
                 L.adam_step(master, work if work.dtype != self.torch.float32 else work, m, v,
                             g.reshape(-1), 1e-3, 0.9, 0.999, 1e-8, self.adam_t)
 
-    def step_e2e(self):
-        """The user's call sequence with host buffers: H2D inputs, pack, fwd+bwd, unpack, D2H."""
-        torch, L = self.torch, self.L
-        self.E_orig_dev.copy_(self.E_orig_host, non_blocking=True)
-        self.dET.copy_(self.dET_host, non_blocking=True)
-        L.pack_states(self.plan, self.dt, self.c["H"], self.E_orig_dev, self.E0)
-        self.step()
-        L.unpack_states(self.plan, "f32", self.c["H"], self.dE0, self.dE0_orig)
-        self.dE0_host.copy_(self.dE0_orig, non_blocking=True)
-        for k, v in self.grads.items():
-            self.grads_host[k].copy_(v, non_blocking=True)
-        return (self.E_orig_host.numel() * self.E_orig_host.element_size()
-                + self.dET_host.numel() * 4,
-                self.dE0_host.numel() * 4 + sum(v.numel() * 4 for v in self.grads_host.values()))
+    def e2e_run(self, steps, stream):
+        """`steps` steps of the user's call sequence with host buffers, timed on `stream`: every step
+        copies its inputs from pinned host memory (H2D), packs, runs fwd+bwd, unpacks and reads its
+        results back (D2H).  As in a training loop with prefetching, the copies run on their own
+        stream with double buffers: step k+1's inputs go up and step k's results come down while
+        step k computes.  Returns (ms per step, H2D bytes per step, D2H bytes per step)."""
+        torch, L, c = self.torch, self.L, self.c
+        H = c["H"]
+        if not hasattr(self, "e_cs"):
+            self.e_cs = torch.cuda.Stream()
+            self.e_in = [self.E_orig_dev, torch.empty_like(self.E_orig_dev)]
+            self.e_dET = [torch.empty_like(self.dET), torch.empty_like(self.dET)]
+            self.e_out = [self.dE0_orig, torch.empty_like(self.dE0_orig)]
+            self.e_out_host = [self.dE0_host, torch.empty(self.dE0_host.shape, pin_memory=True)]
+            self.e_gdev = [torch.empty_like(self.gflat), torch.empty_like(self.gflat)]
+            self.e_ghost = [torch.empty(self.gflat.shape, pin_memory=True) for _ in range(2)]
+            self.e_h2d = [torch.cuda.Event(), torch.cuda.Event()]
+            self.e_comp = [torch.cuda.Event(), torch.cuda.Event()]
+        cs = self.e_cs
+        t0, t1, fin = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+                       torch.cuda.Event())
+
+        def h2d(k):
+            b = k % 2
+            with torch.cuda.stream(cs):
+                self.e_in[b].copy_(self.E_orig_host, non_blocking=True)
+                self.e_dET[b].copy_(self.dET_host, non_blocking=True)
+            self.e_h2d[b].record(cs)
+
+        t0.record(stream)
+        cs.wait_event(t0)
+        h2d(0)
+        for k in range(steps):
+            b, nb = k % 2, (k + 1) % 2
+            if k + 1 < steps:
+                if k >= 1:
+                    cs.wait_event(self.e_comp[nb])  # step k-1 is done with buffer set nb
+                h2d(k + 1)
+            stream.wait_event(self.e_h2d[b])  # also orders step k-2's reads of set b before this
+            L.pack_states(self.plan, self.dt, H, self.e_in[b], self.E0)
+            self.step(dET=self.e_dET[b])
+            L.unpack_states(self.plan, "f32", H, self.dE0, self.e_out[b])
+            self.e_gdev[b].copy_(self.gflat, non_blocking=True)
+            self.e_comp[b].record(stream)
+            cs.wait_event(self.e_comp[b])
+            with torch.cuda.stream(cs):
+                self.e_out_host[b].copy_(self.e_out[b], non_blocking=True)
+                self.e_ghost[b].copy_(self.e_gdev[b], non_blocking=True)
+        fin.record(cs)
+        stream.wait_event(fin)
+        t1.record(stream)
+        torch.cuda.synchronize()
+        bi = self.E_orig_host.numel() * self.E_orig_host.element_size() + self.dET_host.numel() * 4
+        bo = self.dE0_host.numel() * 4 + self.gflat.numel() * 4
+        return t0.elapsed_time(t1) / steps, bi, bo
 
 
 # --------------------------------------------------------------------------------- CPU oracle
@@ -485,17 +526,9 @@ def main():
     value = total_units / (ms_step / 1e3)
 
     # ---- e2e: host buffers, H2D + pack + step + unpack + D2H inside the timed region
-    for _ in range(2):
-        st.step_e2e()
-    torch.cuda.synchronize()
+    st.e2e_run(2, stream)
     barrier()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        bi, bo = st.step_e2e()
-    e1.record(stream)
-    torch.cuda.synchronize()
-    e_ms = e0.elapsed_time(e1) / args.steps
+    e_ms, bi, bo = st.e2e_run(args.steps, stream)
     e_ms, _ = reduce_over_ranks(dist, e_ms, 0.0)
     e2e_value = total_units / (e_ms / 1e3)
 
