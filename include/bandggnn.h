@@ -240,6 +240,12 @@ const char* bg_last_error(void);
 /* Synchronise `stream` and read the device status word that bounded waits and in-kernel checks
  * write: BG_OK, BG_ETIMEOUT or BG_EDEVICE (the word is then cleared). */
 int bg_check_device(void* stream);
+/* Failure-path self test: launches (asynchronously, on `stream`) one block whose bounded
+ * mbarrier wait is never satisfied, so that it gives up after its poll cap (a fraction of a
+ * second), records BG_ETIMEOUT (site 901) in the status word and returns, as a stalled pipeline
+ * role would.  The next bg_check_device reports BG_ETIMEOUT and clears the word; the context stays
+ * usable.  Nothing faults or hangs. */
+int bg_selftest_device_wait(void* stream);
 /* Kernel timing with CUDA events recorded on the launching stream around every launch of the
  * listed kernels while enabled (adds two event records per launch). */
 #define BG_KID_BAND_FWD 0
@@ -256,7 +262,8 @@ int bg_profile_read(int32_t kid, double* ms_total, int64_t* launches, int32_t re
 int64_t bg_launch_count(void);
 /* 1 when band propagation for (plan, dtype, H) runs on the fused tcgen05 tensor-core kernels,
  * 0 when it runs on the SIMT kernels (fp32 path and shapes the tensor-core kernels do not cover:
- * S != 128, H not in {64, 128}, P > 32); negative status on error.  The plan must be uploaded. */
+ * H not in {32, 64, 128, 256}, H = 256 at S >= 256, P > 32, a padded size that is not a whole
+ * number of 128-row tiles); negative status on error.  The plan must be uploaded. */
 int bg_band_uses_tensor_cores(const bg_plan* plan, bg_dtype dtype, int32_t H);
 
 #ifdef __cplusplus

@@ -93,6 +93,7 @@ def load(path: str = LIB_PATH):
         "bg_adam_step": (c.c_int, [i64, vp, vp, c.c_int, vp, vp, vp, f32, f32, f32, f32, i32, vp]),
         "bg_last_error": (c.c_char_p, []),
         "bg_check_device": (c.c_int, [vp]),
+        "bg_selftest_device_wait": (c.c_int, [vp]),
         "bg_profile_enable": (c.c_int, [i32]),
         "bg_profile_read": (c.c_int, [i32, vp, vp, i32]),
         "bg_launch_count": (i64, []),
@@ -317,6 +318,12 @@ def adam_step(master, working, m, v, grad, lr, beta1, beta2, eps, step, stream=N
 
 def check_device(stream=None):
     _check(load().bg_check_device(_stream(stream)))
+
+
+def selftest_device_wait(stream=None):
+    """Launch the failure-path self test (a bounded wait that gives up); check_device() then
+    raises BG_ETIMEOUT."""
+    _check(load().bg_selftest_device_wait(_stream(stream)))
 
 
 def profile_enable(on: bool):

@@ -147,6 +147,14 @@ int status_word_ptr(int** out) {
 }
 }  // namespace
 
+extern "C" int bg_selftest_device_wait(void* stream) {
+  bg_clear_error();
+  int* d = nullptr;
+  BG_TRY(status_word_ptr(&d));
+  BG_CUDA(bg::wait_selftest(d, static_cast<cudaStream_t>(stream)));
+  return BG_OK;
+}
+
 extern "C" int bg_check_device(void* stream) {
   int* d = nullptr;
   BG_TRY(status_word_ptr(&d));

@@ -491,6 +491,31 @@ cudaError_t gemm_tn_multi(const TNProblem* pr, int n, int Hout, int64_t K, int a
   return e;
 }
 
+namespace {
+// One warp waits, through the same bounded wait as every pipeline role, on an mbarrier that
+// nothing arrives on: after the poll cap it records a timeout (site 901) in the status word and
+// returns, as a stalled kernel would.
+__global__ void k_wait_selftest(int* status) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  volatile int* abort = &abort_flag;
+  if (threadIdx.x == 0) mbar_wait(&bar, 0, status, 901, abort, 64);
+  __syncthreads();
+}
+}  // namespace
+
+cudaError_t wait_selftest(int* status, cudaStream_t st) {
+  k_wait_selftest<<<1, 32, 0, st>>>(status);
+  note_launch();
+  return cudaGetLastError();
+}
+
 cudaError_t gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int Hout,
                     int64_t K, int mode, float* out, float* bias, int accumulate, float* part,
                     size_t part_floats, int* status, cudaStream_t st) {

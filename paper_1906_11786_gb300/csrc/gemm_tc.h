@@ -60,6 +60,10 @@ int gemm_tn_num_sms();
 bool make_map_3d(CUtensorMap* m, const void* base, uint64_t batch, uint64_t rows, uint64_t cols,
                  uint64_t ld, uint64_t sbatch, uint32_t box_rows);
 
+// One block whose bounded mbarrier wait is never satisfied: it gives up after the poll cap and
+// records a timeout (site 901) in `status`, the path every stalled pipeline role takes.
+cudaError_t wait_selftest(int* status, cudaStream_t st);
+
 // rows [H, H+16) of a [H+16][ld] bf16 array: row H = 1.0, the rest 0 (cols [0, n)).
 cudaError_t fill_ones_rows(__nv_bfloat16* base, int H, int64_t n, int64_t ld, cudaStream_t st);
 

@@ -305,3 +305,20 @@ def test_full_size_config2_ggnn_T8_fwd_bwd_sampled_graphs():
     assert np.all(got_dE0[rest] == 0.0)
     for k, v in grads.items():
         assert rel_err(v.cpu().numpy(), ref[k]) < TOL["bf16"], k
+
+
+# ------------------------------------------------------------------------------------ failure path
+def test_device_wait_timeout_is_reported_and_the_context_survives():
+    """A bounded device wait that is never satisfied gives up after its poll cap, the status word
+    carries BG_ETIMEOUT with the wait's site to the host, the word is cleared, and the context
+    still runs and checks clean work (no fault, no hang: the wait returns by itself)."""
+    L.selftest_device_wait()
+    with pytest.raises(L.BandGGNNError) as err:
+        L.check_device()
+    assert "BG_ETIMEOUT" in str(err.value) and "901" in str(err.value)
+    L.check_device()  # cleared
+    g = synth.gen_graph(300, 4, True, 20, 10, 1.0, 11)
+    c = Case([g], 8, 128, 64, "bf16", seed=4)
+    Y, ref = _fwd(c)
+    assert rel_err(Y, ref) < TOL["bf16"]
+
