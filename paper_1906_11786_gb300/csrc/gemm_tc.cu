@@ -24,24 +24,27 @@ namespace {
 
 constexpr int kStages = 4;
 
-// Tile widths BN = Hout + 16 (48, 80, 144, 272), four stages each.  Up to BN = 80 two CTAs share
-// an SM; BN = 144 (138 KB) and BN = 272 (all 512 TMEM columns) run one per SM.  B boxes are at
-// most 256 rows: BN = 272 loads two boxes of 136 rows and issues an N = 256 and an N = 16 MMA per
-// K step.
+// Tile widths BN = Hout + 16 (48, 80, 144, 272), four stages each, one CTA per SM.  A CTA takes
+// MT = 2 consecutive 128-row M tiles of one problem (MT = 1 at BN = 272, whose accumulator takes all
+// 512 TMEM columns), so that each K chunk of B, which every M tile of the problem reads, is loaded
+// once per two tiles: the pass moves A once and B once per tile pair, instead of once per tile.
+// B boxes are at most 256 rows: BN = 272 loads two boxes of 136 rows and issues an N = 256 and an
+// N = 16 MMA per K step.
 template <int BN>
 struct GCfg {
+  static constexpr int MT = BN <= 256 ? 2 : 1;
   static constexpr int A_BYTES = 128 * 128;  // 128 rows x 64 bf16
   static constexpr int B_BYTES = BN * 128;
-  static constexpr int STAGE = A_BYTES + B_BYTES;
+  static constexpr int STAGE = MT * A_BYTES + B_BYTES;
   static constexpr int STAGES = 4;
   static constexpr int SMEM = STAGES * STAGE + 1024 + 1024;
   static constexpr int TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : BN <= 256 ? 256 : 512;
-  static constexpr int PER_SM = BN <= 80 ? 2 : 1;
   static constexpr int BOX = BN <= 256 ? BN : BN / 2;  // B rows per TMA box
   static constexpr int N1 = BN <= 256 ? BN : 256;      // first MMA's N
   static_assert(BN % 16 == 0 && BN <= 512, "tile width");
-  static_assert(PER_SM * (SMEM + 512) <= 232448, "shared memory");
-  static_assert(BOX * 128 % 1024 == 0, "box alignment");
+  static_assert(SMEM + 512 <= 232448, "shared memory");
+  static_assert(MT * TCOLS <= 512, "tensor memory");
+  static_assert(BOX * 128 % 1024 == 0 && A_BYTES % 1024 == 0, "box alignment");
   static_assert(STAGES <= kStages, "stage count");
 };
 
@@ -55,12 +58,13 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
       : "r"(taddr));
 }
 
-// Up to kMaxGroups problems with the same K and N in one launch: blockIdx.x runs over the M tiles
-// of all groups; group g's rows sit at rows prow[g] .. prow[g] + M[g] of the partial sums.
+// Up to kMaxGroups problems with the same K and N in one launch: blockIdx.x runs over the work
+// items (MT consecutive M tiles of one problem) of all groups; group g's rows sit at rows
+// prow[g] .. prow[g] + M[g] of the partial sums.
 constexpr int kMaxGroups = 3;
 struct TNGroups {
   CUtensorMap a[kMaxGroups], b[kMaxGroups];
-  int mt_end[kMaxGroups];  // cumulative M-tile counts
+  int it_end[kMaxGroups];  // cumulative work-item counts
   int M[kMaxGroups];
   int prow[kMaxGroups];
 };
@@ -82,9 +86,11 @@ __global__ void __launch_bounds__(192, 1)
   volatile int* abort = abort_flag;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   int g = 0;
-  while (g + 1 < kMaxGroups && (int)blockIdx.x >= grp.mt_end[g]) ++g;
-  const int mt = blockIdx.x - (g ? grp.mt_end[g - 1] : 0), split = blockIdx.z;
+  while (g + 1 < kMaxGroups && (int)blockIdx.x >= grp.it_end[g]) ++g;
+  const int item = blockIdx.x - (g ? grp.it_end[g - 1] : 0), split = blockIdx.z;
   const int M = grp.M[g];
+  const int mt0 = item * C::MT;                            // first M tile of this CTA
+  const int ntiles = min(C::MT, (M + 127) / 128 - mt0);    // 1 .. MT
   const CUtensorMap* tmA = &grp.a[g];
   const CUtensorMap* tmB = &grp.b[g];
   const int kc0 = split * per_split;
@@ -97,7 +103,7 @@ __global__ void __launch_bounds__(192, 1)
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, C::TCOLS);
+    tmem_alloc(tmem_slot, C::MT * C::TCOLS);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -115,11 +121,12 @@ __global__ void __launch_bounds__(192, 1)
       const int s = it % C::STAGES;
       if (!mbar_wait(&empty[s], ((it / C::STAGES) & 1) ^ 1, status, 501, abort, 32)) break;
       ++issued[s];
-      mbar_expect_tx(&full[s], C::STAGE);
+      mbar_expect_tx(&full[s], ntiles * C::A_BYTES + C::B_BYTES);
       uint8_t* st = smem + s * C::STAGE;
-      tma_load_2d(st, tmA, &full[s], kc * 64, mt * 128);
+      for (int m = 0; m < ntiles; ++m)
+        tma_load_2d(st + m * C::A_BYTES, tmA, &full[s], kc * 64, (mt0 + m) * 128);
       for (int r = 0; r < BN; r += C::BOX)
-        tma_load_2d(st + C::A_BYTES + r * 128, tmB, &full[s], kc * 64, blockIdx.y * BN + r);
+        tma_load_2d(st + C::MT * C::A_BYTES + r * 128, tmB, &full[s], kc * 64, blockIdx.y * BN + r);
     }
     if (*abort)
       for (int s = 0; s < C::STAGES; ++s)
@@ -134,15 +141,19 @@ __global__ void __launch_bounds__(192, 1)
       const int s = it % C::STAGES;
       if (!mbar_wait(&full[s], (it / C::STAGES) & 1, status, 502, abort)) break;
       tc_fence_after();
-      const uint32_t a = smem_u32(smem + s * C::STAGE), b = a + C::A_BYTES;
+      const uint32_t a = smem_u32(smem + s * C::STAGE), b = a + C::MT * C::A_BYTES;
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk)
         if (leader) {
-          const uint64_t ad = desc_sw128_kmajor(a + kk * 32);
           const uint32_t acc = (kc > kc0 || kk > 0) ? 1u : 0u;
-          mma_ss(tmem, ad, desc_sw128_kmajor(b + kk * 32), idesc, acc);
-          if (BN > 256)
-            mma_ss(tmem + 256, ad, desc_sw128_kmajor(b + 256 * 128 + kk * 32), idesc2, acc);
+          const uint64_t bd = desc_sw128_kmajor(b + kk * 32);
+          for (int m = 0; m < ntiles; ++m) {
+            const uint64_t ad = desc_sw128_kmajor(a + m * C::A_BYTES + kk * 32);
+            mma_ss(tmem + m * C::TCOLS, ad, bd, idesc, acc);
+            if (BN > 256)
+              mma_ss(tmem + m * C::TCOLS + 256, ad, desc_sw128_kmajor(b + 256 * 128 + kk * 32),
+                     idesc2, acc);
+          }
         }
       if (leader) tc_commit(&empty[s]);
       __syncwarp();
@@ -157,19 +168,21 @@ __global__ void __launch_bounds__(192, 1)
   } else if (warp >= 2) {
     grid_dep_wait();  // the partial sums may still be read by the previous reduction
     const int q = warp & 3;  // TMEM lane quarter this warp may access
-    const int m = mt * 128 + q * 32 + lane;
     if (mbar_wait(done, 0, status, 503, abort, 256)) {
       tc_fence_after();
-      float* out = part + ((size_t)split * Mtot + grp.prow[g] + m) * N + blockIdx.y * BN;
+      for (int mi = 0; mi < ntiles; ++mi) {
+        const int m = (mt0 + mi) * 128 + q * 32 + lane;
+        float* out = part + ((size_t)split * Mtot + grp.prow[g] + m) * N + blockIdx.y * BN;
 #pragma unroll
-      for (int c0 = 0; c0 < BN; c0 += 16) {
-        uint32_t v[16];
-        tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + c0, v);
-        tmem_wait_ld();
-        if (m < M && kc1 > kc0) {
+        for (int c0 = 0; c0 < BN; c0 += 16) {
+          uint32_t v[16];
+          tmem_ld16(tmem + mi * C::TCOLS + ((uint32_t)(q * 32) << 16) + c0, v);
+          tmem_wait_ld();
+          if (m < M && kc1 > kc0) {
 #pragma unroll
-          for (int j = 0; j < 16; ++j)
-            if (blockIdx.y * BN + c0 + j < N) out[c0 + j] = __uint_as_float(v[j]);
+            for (int j = 0; j < 16; ++j)
+              if (blockIdx.y * BN + c0 + j < N) out[c0 + j] = __uint_as_float(v[j]);
+          }
         }
       }
     }
@@ -179,7 +192,7 @@ __global__ void __launch_bounds__(192, 1)
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem, C::TCOLS);
+    tmem_dealloc(tmem, C::MT * C::TCOLS);
   }
 }
 
@@ -439,13 +452,14 @@ cudaError_t gemm_tn_multi(const TNProblem* pr, int n, int Hout, int64_t K, int a
   const int64_t kchunks = (K + 63) / 64;
   TNGroups grp{};
   TNOut o{};
+  const int MT = N <= 256 ? 2 : 1;  // M tiles per CTA (GCfg::MT)
   int mt = 0, Mtot = 0;
   for (int g = 0; g < n; ++g) {
     if (!make_map_ld(&grp.a[g], pr[g].A, pr[g].M, K, pr[g].lda, 128) ||
         !make_map_ld(&grp.b[g], pr[g].B, N, K, pr[g].ldb, N <= 256 ? N : N / 2))
       return cudaErrorInvalidValue;
-    mt += (pr[g].M + 127) / 128;
-    grp.mt_end[g] = mt;
+    mt += ((pr[g].M + 127) / 128 + MT - 1) / MT;
+    grp.it_end[g] = mt;
     grp.M[g] = o.M[g] = pr[g].M;
     grp.prow[g] = o.prow[g] = Mtot;
     o.out[g] = pr[g].out;
@@ -453,14 +467,12 @@ cudaError_t gemm_tn_multi(const TNProblem* pr, int n, int Hout, int64_t K, int a
     o.mode[g] = pr[g].mode;
     Mtot += pr[g].M;
   }
-  for (int g = n; g < kMaxGroups; ++g) grp.mt_end[g] = mt;
+  for (int g = n; g < kMaxGroups; ++g) grp.it_end[g] = mt;
   o.n_groups = n;
   const int sms = gemm_tn_num_sms();
-  // at most 2 * sms CTAs: one wave where two fit per SM (a partial second wave of even a few CTAs
-  // would nearly double the time of this HBM-bound pass); at N = 144 the same grid in two waves of
-  // one CTA per SM measured faster than one wave of two CTAs with three stages each
-  const int per_sm = N <= 144 ? 2 : 1;
-  int splits = (int)std::max<int64_t>(1, std::min<int64_t>(kchunks, std::max(1, per_sm * sms / mt)));
+  // at most one CTA per SM, so that all of them run in one wave (a partial second wave of even a
+  // few CTAs would nearly double the time of this HBM-bound pass)
+  int splits = (int)std::max<int64_t>(1, std::min<int64_t>(kchunks, std::max(1, sms / mt)));
   while (splits > 1 && (size_t)splits * Mtot * N > part_floats) --splits;
   const int per = (int)((kchunks + splits - 1) / splits);
   splits = (int)((kchunks + per - 1) / per);
