@@ -589,23 +589,25 @@ constexpr int H = 128, NH = H / 64;
 constexpr int kTileB = 128 * H * 2;          // 128 rows x H bf16: NH 64-column atoms of 16 KB
 constexpr int kAtomB = 128 * 128;
 constexpr int kPiece = 192 * 128;            // ring slot (gate pieces; backward pieces use 16 KB)
-constexpr int kSlots = 3;
-constexpr int kGin = 128 * H * 4;            // 128 rows x H fp32 as 32-column boxes of 16 KB
+constexpr int kSlots = 3;                    // forward piece ring
+constexpr int kSlotsB = 5;                   // backward piece ring
+constexpr int kGin = 128 * 64 * 4;           // one half of the incoming gradient: 2 boxes of 16 KB
 constexpr int kGates = 4 * 64;               // TMEM columns of one job's gate pre-activations
 
 struct Smem {
   static constexpr int FWD_STAGE = 2 * kTileB;  // Y, E
   static constexpr int FWD_PIECES = 2 * FWD_STAGE;
   static constexpr int FWD = FWD_PIECES + kSlots * kPiece + 1024;
-  static constexpr int BWD_STAGE = 2 * kTileB + kGin;  // Y, E, incoming gradient (one stage)
-  static constexpr int BWD_PIECES = BWD_STAGE;
-  static constexpr int BWD = BWD_PIECES + kSlots * kPiece + 1024;
+  static constexpr int BWD_STAGE = 2 * kTileB;       // Y, E (one stage)
+  static constexpr int BWD_GIN = BWD_STAGE;          // the job's half of the incoming gradient
+  static constexpr int BWD_PIECES = BWD_GIN + kGin;
+  static constexpr int BWD = BWD_PIECES + kSlotsB * kPiece + 1024;
   static_assert(FWD + 4096 <= 232448 && BWD + 4096 <= 232448, "shared memory");
 };
 
 struct Bars {
-  uint64_t t_full[2], t_empty[2], p_full[kSlots], p_empty[kSlots], g_full[2], g_empty[2];
-  uint64_t ops_ready, ph2_full, dx_empty, drain;
+  uint64_t t_full[2], t_empty[2], p_full[kSlotsB], p_empty[kSlotsB], g_full[2], g_empty[2];
+  uint64_t gin_full, gin_empty, ops_ready, ph2_full, dx_empty, drain;
   uint32_t tmem_slot;
   int abort;
 };
@@ -620,7 +622,9 @@ __device__ __forceinline__ void setup(Bars* b, float* bias, const float* b_ih, c
       mbar_init(&b->g_full[i], 1);
       mbar_init(&b->g_empty[i], kEpiWarps);
     }
-    for (int i = 0; i < kSlots; ++i) { mbar_init(&b->p_full[i], 1); mbar_init(&b->p_empty[i], 1); }
+    for (int i = 0; i < kSlotsB; ++i) { mbar_init(&b->p_full[i], 1); mbar_init(&b->p_empty[i], 1); }
+    mbar_init(&b->gin_full, 1);
+    mbar_init(&b->gin_empty, kEpiWarps);
     mbar_init(&b->ops_ready, kEpiWarps);
     mbar_init(&b->ph2_full, 1);
     mbar_init(&b->dx_empty, kEpiWarps);
@@ -641,15 +645,16 @@ __device__ __forceinline__ void setup(Bars* b, float* bias, const float* b_ih, c
 // Piece producer: for every job, the 2 NH gate pieces and (backward) the 6 backward pieces, in
 // the order the MMA issuer uses them.  The weights are not written by the kernels this one may
 // overlap under programmatic dependent launch (they change only between training steps).
+template <int NS>
 __device__ __forceinline__ void produce_pieces(Bars* b, uint8_t* ring, const CUtensorMap* tWih,
                                                const CUtensorMap* tWhh, const CUtensorMap* tWihT,
                                                const CUtensorMap* tWhhT, bool bwd, int n_tiles,
                                                int* status, volatile int* abort) {
-  uint32_t pc = 0, issued[kSlots] = {0, 0, 0};
+  uint32_t pc = 0, issued[NS] = {};
   bool ok = true;
   auto next = [&](int bytes) -> uint8_t* {
-    const int s = pc % kSlots;
-    if (!mbar_wait(&b->p_empty[s], ((pc / kSlots) & 1) ^ 1, status, 631, abort, 64)) return nullptr;
+    const int s = pc % NS;
+    if (!mbar_wait(&b->p_empty[s], ((pc / NS) & 1) ^ 1, status, 631, abort, 64)) return nullptr;
     ++issued[s];
     mbar_expect_tx(&b->p_full[s], bytes);
     ++pc;
@@ -658,14 +663,14 @@ __device__ __forceinline__ void produce_pieces(Bars* b, uint8_t* ring, const CUt
   for (int t = blockIdx.x; t < n_tiles && ok && !*abort; t += gridDim.x) {
     for (int hh = 0; hh < NH && ok; ++hh) {
       for (int q = 0; q < 2 * NH && ok; ++q) {
-        const int m = q / NH, ka = q % NH, s = pc % kSlots;
+        const int m = q / NH, ka = q % NH, s = pc % NS;
         uint8_t* dst = next(kPiece);
         if (!dst) { ok = false; break; }
         for (int g = 0; g < 3; ++g)
           tma_load_2d(dst + g * 64 * 128, m ? tWhh : tWih, &b->p_full[s], 64 * ka, g * H + 64 * hh);
       }
       for (int q = 0; bwd && q < 6 && ok; ++q) {
-        const int m = q / 3, g = q % 3, s = pc % kSlots;
+        const int m = q / 3, g = q % 3, s = pc % NS;
         uint8_t* dst = next(128 * 128);
         if (!dst) { ok = false; break; }
         tma_load_2d(dst, m ? tWhhT : tWihT, &b->p_full[s], g * H + 64 * hh, 0);
@@ -673,20 +678,21 @@ __device__ __forceinline__ void produce_pieces(Bars* b, uint8_t* ring, const CUt
     }
   }
   if (*abort)
-    for (int s = 0; s < kSlots; ++s)
+    for (int s = 0; s < NS; ++s)
       for (uint32_t k = 0; issued[s] && k < (1u << 22) && !mbar_try(&b->p_full[s], (issued[s] - 1) & 1); ++k) {
       }
 }
 
 // Gate pre-activations of job (tile in `stage`, half hh) into TMEM columns g0 .. g0 + 255,
 // consuming 2 NH gate pieces.
+template <int NS>
 __device__ __forceinline__ bool gate_mmas(Bars* b, bool leader, uint32_t g0, uint32_t sY,
                                           uint32_t sE, uint8_t* ring, uint32_t& pc, int* status,
                                           volatile int* abort) {
   constexpr uint32_t id_rz = idesc_bf16_f32(128, 128), id_n = idesc_bf16_f32(128, 64);
   for (int q = 0; q < 2 * NH; ++q, ++pc) {
-    const int m = q / NH, ka = q % NH, s = pc % kSlots;
-    if (!mbar_wait(&b->p_full[s], (pc / kSlots) & 1, status, 632, abort)) return false;
+    const int m = q / NH, ka = q % NH, s = pc % NS;
+    if (!mbar_wait(&b->p_full[s], (pc / NS) & 1, status, 632, abort)) return false;
     tc_fence_after();
     const uint32_t a0 = (m ? sE : sY) + ka * kAtomB, p0 = smem_u32(ring + s * kPiece);
     if (leader) {
@@ -742,7 +748,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (uint32_t k = 0; issued[s] && k < (1u << 22) && !mbar_try(&bars.t_full[s], (issued[s] - 1) & 1); ++k) {
         }
   } else if (warp == 2 && lane == 0) {
-    produce_pieces(&bars, pieces, &tWih, &tWhh, nullptr, nullptr, false, n_tiles, status, abort);
+    produce_pieces<kSlots>(&bars, pieces, &tWih, &tWhh, nullptr, nullptr, false, n_tiles, status,
+                           abort);
   } else if (warp == 1) {
     // ------------------------------------------------------------------ MMA issuer
     const bool leader = elect_one_sync();
@@ -757,7 +764,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int gb = jn & 1;
         if (!mbar_wait(&bars.g_empty[gb], ((jn >> 1) & 1) ^ 1, status, 635, abort)) { ok = false; break; }
         tc_fence_after();
-        if (!gate_mmas(&bars, leader, tmem + gb * kGates, sY, sY + kTileB, pieces, pc, status, abort)) {
+        if (!gate_mmas<kSlots>(&bars, leader, tmem + gb * kGates, sY, sY + kTileB, pieces, pc,
+                               status, abort)) {
           ok = false;
           break;
         }
@@ -866,9 +874,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0 && lane == 0) {
     // ------------------------------------------------------------------ tile producer (one stage)
     grid_dep_wait();  // Y, E and the incoming gradient are earlier kernels' output
-    uint32_t issued = 0;
+    uint32_t issued = 0, gissued = 0, jn = 0;
     int i = 0;
-    for (int t = blockIdx.x; t < n_tiles && !*abort; t += gridDim.x, ++i) {
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles && ok && !*abort; t += gridDim.x, ++i) {
       if (!mbar_wait(&bars.t_empty[0], (i & 1) ^ 1, status, 641, abort, 64)) break;
       ++issued;
       mbar_expect_tx(&bars.t_full[0], Smem::BWD_STAGE);
@@ -876,14 +885,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_2d(smem + a * kAtomB, &tY, &bars.t_full[0], 64 * a, t * 128);
         tma_load_2d(smem + kTileB + a * kAtomB, &tE, &bars.t_full[0], 64 * a, t * 128);
       }
-      for (int a = 0; a < H / 32; ++a)
-        tma_load_2d(smem + 2 * kTileB + a * kAtomB, &tG, &bars.t_full[0], 32 * a, t * 128);
+      // the incoming gradient one job (64-column half) at a time
+      for (int hh = 0; hh < NH; ++hh, ++jn) {
+        if (!mbar_wait(&bars.gin_empty, (jn & 1) ^ 1, status, 649, abort, 64)) { ok = false; break; }
+        ++gissued;
+        mbar_expect_tx(&bars.gin_full, kGin);
+        for (int a = 0; a < 2; ++a)
+          tma_load_2d(smem + Smem::BWD_GIN + a * kAtomB, &tG, &bars.gin_full, 64 * hh + 32 * a,
+                      t * 128);
+      }
     }
-    if (*abort)
+    if (*abort) {
       for (uint32_t k = 0; issued && k < (1u << 22) && !mbar_try(&bars.t_full[0], (issued - 1) & 1); ++k) {
       }
+      for (uint32_t k = 0; gissued && k < (1u << 22) && !mbar_try(&bars.gin_full, (gissued - 1) & 1); ++k) {
+      }
+    }
   } else if (warp == 2 && lane == 0) {
-    produce_pieces(&bars, pieces, &tWih, &tWhh, &tWihT, &tWhhT, true, n_tiles, status, abort);
+    produce_pieces<kSlotsB>(&bars, pieces, &tWih, &tWhh, &tWihT, &tWhhT, true, n_tiles, status,
+                            abort);
   } else if (warp == 1) {
     // ------------------------------------------------------------------ MMA issuer
     const bool leader = elect_one_sync();
@@ -898,7 +918,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // the previous job's products have read the gate gradients out of columns 0..255
         if (jn > 0 && !mbar_wait(&bars.ph2_full, (jn - 1) & 1, status, 643, abort)) { ok = false; break; }
         tc_fence_after();
-        if (!gate_mmas(&bars, leader, tmem, sY, sY + kTileB, pieces, pc, status, abort)) {
+        if (!gate_mmas<kSlotsB>(&bars, leader, tmem, sY, sY + kTileB, pieces, pc, status, abort)) {
           ok = false;
           break;
         }
@@ -912,8 +932,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_after();
         for (int q = 0; q < 6; ++q, ++pc) {
-          const int m = q / 3, gate = q % 3, s = pc % kSlots;
-          if (!mbar_wait(&bars.p_full[s], (pc / kSlots) & 1, status, 646, abort)) { ok = false; break; }
+          const int m = q / 3, gate = q % 3, s = pc % kSlotsB;
+          if (!mbar_wait(&bars.p_full[s], (pc / kSlotsB) & 1, status, 646, abort)) { ok = false; break; }
           tc_fence_after();
           const uint32_t p0 = smem_u32(pieces + s * kPiece);
           if (leader) {
@@ -943,7 +963,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = (warp & 3) * 32 + lane;
     const uint32_t lb = (uint32_t)((warp & 3) * 32) << 16;
     const uint8_t* etile = smem + kTileB;
-    const uint8_t* gtile = smem + 2 * kTileB;
+    const uint8_t* gtile = smem + Smem::BWD_GIN;
     uint32_t jn = 0;
     int i = 0;
     bool ok = true;
@@ -951,7 +971,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int row = t * 128 + r;
       const bool real = row < n_real;
       for (int hh = 0; hh < NH; ++hh, ++jn) {
-        if (!mbar_wait(&bars.g_full[0], jn & 1, status, 647, abort, 64)) { ok = false; break; }
+        if (!mbar_wait(&bars.g_full[0], jn & 1, status, 647, abort, 64) ||
+            !mbar_wait(&bars.gin_full, jn & 1, status, 650, abort, 64)) {
+          ok = false;
+          break;
+        }
         tc_fence_after();
         const uint32_t acc = tmem + lb;
         uint32_t p_r[8], p_z[8], p_n[8], p_hn[8];
@@ -968,8 +992,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           float e[8];
           read_sw128_row8(etile, r, h, e);
           float4 g4[2];
-          read_sw128_f32_row8(gtile, r, h, g4);
-          if (h8 == 1 && hh == NH - 1) warp_arrive(&bars.t_empty[0]);
+          read_sw128_f32_row8(gtile, r, hs, g4);  // column hs of the job's half
+          if (h8 == 1) {
+            warp_arrive(&bars.gin_empty);
+            if (hh == NH - 1) warp_arrive(&bars.t_empty[0]);
+          }
           const int o = 4 * h8;
 #pragma unroll
           for (int q = 0; q < 2; ++q) {
