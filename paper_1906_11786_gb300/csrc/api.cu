@@ -488,7 +488,7 @@ TcFwdWs tc_fwd_ws(const bg_plan* p, int H) {
   return w;
 }
 struct TcBwdWs {
-  size_t g, dXT, dMT, dgiT, dghT, WihT, WhhT, Wk, part, total;
+  size_t g, dXT, dMT, dgiT, dhnT, WihT, WhhT, Wk, part, total;
 };
 size_t tc_part_floats(const bg_plan* p, int H, int T) {
   const int64_t K = (int64_t)T * p->n_pad();
@@ -504,7 +504,7 @@ TcBwdWs tc_bwd_ws(const bg_plan* p, int H, int T) {
   w.dXT = o; o += al(n * H * 2);
   w.dMT = o; o += al((size_t)p->P * H * TN * 2);
   w.dgiT = o; o += al((size_t)3 * H * TN * 2);
-  w.dghT = o; o += al((size_t)3 * H * TN * 2);
+  w.dhnT = o; o += al((size_t)H * TN * 2);
   w.WihT = o; o += al((size_t)3 * H * H * 2);
   w.WhhT = o; o += al((size_t)3 * H * H * 2);
   w.Wk = o; o += bg::band_tc_w_bytes(p, H);
@@ -854,7 +854,7 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     __nv_bfloat16* dXT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.dXT);
     __nv_bfloat16* dMT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.dMT);
     __nv_bfloat16* dgiT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.dgiT);
-    __nv_bfloat16* dghT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.dghT);
+    __nv_bfloat16* dhnT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.dhnT);
     __nv_bfloat16* WihT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.WihT);
     __nv_bfloat16* WhhT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.WhhT);
     float* part = reinterpret_cast<float*>(wsc + wl.part);
@@ -871,7 +871,7 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
         KTimer tm(BG_KID_GRU_BWD, st);
         BG_CUDA(bg::gru_bwd_tc(H, (int)n, p->n_real, Yi(t), Ei(t), Wih, Whh, WihT, WhhT, prm->b_ih,
                                prm->b_hh, gin, g, dXT, (int64_t)n, dgiT + (size_t)t * n,
-                               dghT + (size_t)t * n, (int64_t)TN, status, st));
+                               dhnT + (size_t)t * n, (int64_t)TN, status, st));
       }
       KTimer tm(BG_KID_BAND_BWD, st);
       BG_CUDA(bg::band_tc_bwd_core(p, H, dXT, (int64_t)n, Wk, g, 1, dMT + (size_t)t * n,
@@ -880,12 +880,15 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     }
     const int acc = (flags & BG_ACCUM) ? 1 : 0;
     KTimer tm(BG_KID_DW, st);
-    // dW_p, db_p over all steps and nodes; dW_ih, db_ih; dW_hh, db_hh
-    const bg::TNProblem probs[3] = {
+    // dW_p, db_p over all steps and nodes; dW_ih, db_ih; dW_hh, db_hh, whose r and z rows take
+    // the input-side gate gradients (equal to the hidden-side ones there) and n rows dh_n
+    const bg::TNProblem probs[4] = {
         {dMT, (int64_t)TN, ETa, (int64_t)TN, p->P * H, 1, gr->dW, gr->db},
         {dgiT, (int64_t)TN, YTa, (int64_t)TN, 3 * H, 0, gr->dW_ih, gr->db_ih},
-        {dghT, (int64_t)TN, ETa, (int64_t)TN, 3 * H, 0, gr->dW_hh, gr->db_hh}};
-    BG_CUDA(bg::gemm_tn_multi(probs, 3, H, (int64_t)TN, acc, part, pf, status, st));
+        {dgiT, (int64_t)TN, ETa, (int64_t)TN, 2 * H, 0, gr->dW_hh, gr->db_hh},
+        {dhnT, (int64_t)TN, ETa, (int64_t)TN, H, 0, gr->dW_hh + (size_t)2 * H * H,
+         gr->db_hh + 2 * H}};
+    BG_CUDA(bg::gemm_tn_multi(probs, 4, H, (int64_t)TN, acc, part, pf, status, st));
     BG_CUDA(cudaMemcpyAsync(dE0, g, sizeof(float) * n * H, cudaMemcpyDeviceToDevice, st));
     return BG_OK;
   }

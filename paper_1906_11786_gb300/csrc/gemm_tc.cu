@@ -61,7 +61,7 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
 // Up to kMaxGroups problems with the same K and N in one launch: blockIdx.x runs over the work
 // items (MT consecutive M tiles of one problem) of all groups; group g's rows sit at rows
 // prow[g] .. prow[g] + M[g] of the partial sums.
-constexpr int kMaxGroups = 3;
+constexpr int kMaxGroups = 4;
 struct TNGroups {
   CUtensorMap a[kMaxGroups], b[kMaxGroups];
   int it_end[kMaxGroups];  // cumulative work-item counts

@@ -23,7 +23,7 @@ cudaError_t gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int 
                     int64_t K, int mode, float* out, float* bias, int accumulate, float* part,
                     size_t part_floats, int* status, cudaStream_t st);
 
-// Up to three such problems with the same K and Hout in one launch (one wave over all their M
+// Up to four such problems with the same K and Hout in one launch (one wave over all their M
 // tiles, one reduction); part_floats must cover gemm_tn_part_floats(sum of M, Hout + 16, K).
 struct TNProblem {
   const void* A;

@@ -386,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                  const float* __restrict__ b_ih, const float* __restrict__ b_hh,
                  float* __restrict__ gout,
                  __nv_bfloat16* __restrict__ dXT, int64_t ld_x, __nv_bfloat16* __restrict__ dgiT,
-                 __nv_bfloat16* __restrict__ dghT, int64_t ld_g, int n_tiles, int n_real,
+                 __nv_bfloat16* __restrict__ dhnT, int64_t ld_g, int n_tiles, int n_real,
                  int* status) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -522,13 +522,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           p_n[o + 2 * q] = pk2(dn[0], dn[1]); p_n[o + 2 * q + 1] = pk2(dn[2], dn[3]);
           p_hn[o + 2 * q] = pk2(dhn[0], dhn[1]); p_hn[o + 2 * q + 1] = pk2(dhn[2], dhn[3]);
         }
-        // gate gradients transposed for the weight-gradient GEMM: rows o = gate*H + h
+        // gate gradients transposed for the weight-gradient GEMM: dgi rows o = gate*H + h, and
+        // of dgh only the n rows (its r and z rows equal dgi's)
         store_T4(dgiT, ld_g, row, hs, p_r + o);
         store_T4(dgiT + (size_t)KH * ld_g, ld_g, row, hs, p_z + o);
         store_T4(dgiT + (size_t)2 * KH * ld_g, ld_g, row, hs, p_n + o);
-        store_T4(dghT, ld_g, row, hs, p_r + o);
-        store_T4(dghT + (size_t)KH * ld_g, ld_g, row, hs, p_z + o);
-        store_T4(dghT + (size_t)2 * KH * ld_g, ld_g, row, hs, p_hn + o);
+        store_T4(dhnT, ld_g, row, hs, p_hn + o);
       }
       // in-place rewrite into the columns just read (see dg_col): within the 16-column window h0,
       // r holds the 8 (dgi_r) pair columns then the 8 (dgi_z) ones, z the (dgi_n) then (dgh_n)
@@ -857,7 +856,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const __grid_constant__ CUtensorMap tG, const float* __restrict__ b_ih,
               const float* __restrict__ b_hh, float* __restrict__ gout,
               __nv_bfloat16* __restrict__ dXT, int64_t ld_x, __nv_bfloat16* __restrict__ dgiT,
-              __nv_bfloat16* __restrict__ dghT, int64_t ld_g, int n_tiles, int n_real,
+              __nv_bfloat16* __restrict__ dhnT, int64_t ld_g, int n_tiles, int n_real,
               int* status) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -1027,13 +1026,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           float4* go = reinterpret_cast<float4*>(gout + (size_t)row * H + h);
           go[0] = make_float4(dhd[0], dhd[1], dhd[2], dhd[3]);
           go[1] = make_float4(dhd[4], dhd[5], dhd[6], dhd[7]);
-          // gate gradients transposed for the weight-gradient GEMM: rows o = gate*H + h
+          // gate gradients transposed for the weight-gradient GEMM: dgi rows o = gate*H + h, and
+        // of dgh only the n rows (its r and z rows equal dgi's)
           store_T4(dgiT, ld_g, row, h, p_r + o);
           store_T4(dgiT + (size_t)H * ld_g, ld_g, row, h, p_z + o);
           store_T4(dgiT + (size_t)2 * H * ld_g, ld_g, row, h, p_n + o);
-          store_T4(dghT, ld_g, row, h, p_r + o);
-          store_T4(dghT + (size_t)H * ld_g, ld_g, row, h, p_z + o);
-          store_T4(dghT + (size_t)2 * H * ld_g, ld_g, row, h, p_hn + o);
+          store_T4(dhnT, ld_g, row, h, p_hn + o);
         }
         // in-place rewrite into the columns this warpgroup read (window 16 g of r and of z)
         const uint32_t w0 = acc + 16 * g;
@@ -1123,7 +1121,7 @@ cudaError_t gru_bwd_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y,
                        const __nv_bfloat16* W_hh, const __nv_bfloat16* W_ihT,
                        const __nv_bfloat16* W_hhT, const float* b_ih, const float* b_hh,
                        const float* gin, float* gout, __nv_bfloat16* dXT, int64_t ld_x,
-                       __nv_bfloat16* dgiT, __nv_bfloat16* dghT, int64_t ld_g, int* status,
+                       __nv_bfloat16* dgiT, __nv_bfloat16* dhnT, int64_t ld_g, int* status,
                        cudaStream_t st) {
   if (!gru_tc_supported(H) || n_pad % 128) return cudaErrorInvalidValue;
   const bool w = H == wide::H;
@@ -1143,7 +1141,7 @@ cudaError_t gru_bwd_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y,
   const int n_tiles = n_pad / 128;
   const int grid = std::min(n_tiles, gemm_tn_num_sms());
   e = launch_pdl(kern, dim3(grid), dim3(kThreads), smem, st, tY, tE, tWi, tWh, tWiT, tWhT, tG, b_ih,
-                 b_hh, gout, dXT, ld_x, dgiT, dghT, ld_g, n_tiles, n_real, status);
+                 b_hh, gout, dXT, ld_x, dgiT, dhnT, ld_g, n_tiles, n_real, status);
   note_launch();
   return e;
 }

@@ -19,13 +19,15 @@ cudaError_t gru_fwd_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y, con
 
 // Backward of gru_fwd_tc for one step.  gin: dL/dE(t+1) [n_pad][H] fp32.  Writes
 //   gout [n_pad][H] fp32 = dL/dE(t) through the GRU (direct and W_hh terms; may alias gin),
-//   dXT [H][ld_x] bf16 = (dL/dY)^T, dgiT / dghT [3H][ld_g] bf16 = gate gradients transposed.
+//   dXT [H][ld_x] bf16 = (dL/dY)^T, dgiT [3H][ld_g] bf16 = input-side gate gradients transposed
+//   (rows r, z, n), dhnT [H][ld_g] bf16 = the n rows of the hidden-side ones (the hidden-side r
+//   and z rows equal dgi's).
 // W_ihT, W_hhT: [H][3H] bf16 transposes of W_ih, W_hh.
 cudaError_t gru_bwd_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y, const __nv_bfloat16* E,
                        const __nv_bfloat16* W_ih, const __nv_bfloat16* W_hh,
                        const __nv_bfloat16* W_ihT, const __nv_bfloat16* W_hhT, const float* b_ih,
                        const float* b_hh, const float* gin, float* gout, __nv_bfloat16* dXT,
-                       int64_t ld_x, __nv_bfloat16* dgiT, __nv_bfloat16* dghT, int64_t ld_g,
+                       int64_t ld_x, __nv_bfloat16* dgiT, __nv_bfloat16* dhnT, int64_t ld_g,
                        int* status, cudaStream_t st);
 
 }  // namespace bg
