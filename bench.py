@@ -59,6 +59,38 @@ def _profiled_traffic(kernel: str, workload: str):
     return int(vals["dram_bytes_per_launch"])
 
 
+def _flops(L, plan, H):
+    """FLOPs of one forward pass over the plan: band-dense (all tiles of Eq. 3 as dense products),
+    edge-type transforms, GRU gates, and the useful count (one H-vector add per kept edge)."""
+    f = {k: plan.flops(H, c) for k, c in (("band_dense", L.BG_FLOPS_BAND),
+                                         ("xform", L.BG_FLOPS_XFORM), ("gru", L.BG_FLOPS_GRU),
+                                         ("nnz", L.BG_FLOPS_NNZ))}
+    f["nnz_over_band_dense"] = f["nnz"] / f["band_dense"] if f["band_dense"] else 0.0
+    return f
+
+
+def _host():
+    """The host cores the CPU baseline ran on: machine, core count, CPU model as /proc reports it."""
+    import platform
+    model = ""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name:"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        for line in open("/proc/cpuinfo") if not model else ():
+            key = line.split(":")[0].strip().lower()
+            if key in ("model name", "cpu part", "cpu implementer") and not model:
+                model = line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return {"machine": platform.machine(), "nproc": os.cpu_count(), "cpu_model": model}
+
+
 def _dist():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -568,6 +600,7 @@ def main():
                    "K": st.info["K"], "S": c["S"], "P": c["P"], "H": H, "T": T,
                    "kept_edges": st.info["n_kept"], "dropped_edges": st.info["n_dropped"],
                    "plan_ms": st.plan_ms, "upload_ms": st.upload_ms,
+                   "flops_per_pass": _flops(L, st.plan, H),
                    "band_kernels": "tcgen05" if L.band_uses_tensor_cores(st.plan, c["dtype"], H)
                    else "simt",
                    "l2": "per-step working set (band tiles + saved activations) > 129 MB L2",
@@ -584,7 +617,8 @@ def main():
         line["cpu_baseline"] = {"value": v, "unit": "node-steps/s", "cores": 1, "kind": "oracle",
                                 "sample": f"leading {s['graphs']} graphs ({s['nodes']} nodes) of "
                                           f"the same workload, fwd+bwd, {s['seconds']:.1f}s "
-                                          "single-threaded fp64"}
+                                          "single-threaded fp64",
+                                "host": _host()}
     if rank == 0:
         print(json.dumps(line))
     if dist is not None:
