@@ -347,9 +347,12 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
             for (int j = g * C::CG; j < (g + 1) * C::CG; ++j) {
               const uint32_t a = tmem + C::ACOL + slot * 64;
               const uint64_t jdesc = xdesc + (uint64_t)((2 * j * C::ATOM_X) >> 4);
+              // S = 32: the tile's rows couple to window columns [0, 192) only, so the last four
+              // K steps of the second chunk would multiply all-zero A tiles
+              const int kk_end = (S == 32 && j == C::C1 - 1) ? 4 : kTile / 16;
 #pragma unroll
               for (int kk = 0; kk < kTile / 16; ++kk)
-                if (leader)
+                if (leader && kk < kk_end)
                   mma_ts(d1, a + kk * 8, jdesc + (uint64_t)(((kk / 4) * C::ATOM_X + (kk % 4) * 32) >> 4),
                          idesc, (j == 0 && kk == 0) ? 0u : 1u);
               if (leader) tc_commit(&bars->a_empty[slot][nx_g]);
