@@ -80,6 +80,11 @@ def test_planner_bit_exact_sweep_config4_capacity(S):
     assert ref.n_packed < len(gs)
 
 
+def test_planner_bit_exact_training_batch_config5():
+    """Config 5's graphs (200 .. 5000 nodes, the largest RCM inputs of any config), full batch."""
+    _compare(synth.config_graphs(5), 20, 128)
+
+
 def test_planner_without_rcm_and_without_keep():
     gs = synth.gen_batch(5, 40, 90, 3, True, 12, 8, 1.0, 3)
     _compare(gs, 6, 32, flags=0)
