@@ -252,27 +252,25 @@ def test_full_size_config2_propagate_sampled_rows():
 
 
 
-def test_full_size_config2_ggnn_T8_fwd_bwd_sampled_graphs():
-    """The benchmark workload end to end: config 2 at full size (64 graphs, ~72k nodes, P = 20,
-    S = 128, H = 64, bf16, T = 8) through the fused tensor-core path, forward + backward.
+def _full_size_ggnn_sampled_graphs(c: Case, T: int, pick, seed: int):
+    """Runs T GGNN steps forward and backward on the whole plan (the benchmark's launches) with a
+    dE(T) that is zero outside the graphs `pick`, and checks them against the oracle run on those
+    graphs alone.
 
     Graphs share no edge, so (Eq. 1 and Eq. 2 act per graph) E(T) of a graph depends on that graph
     alone, and a dE(T) that is zero outside a few sampled graphs leaves dE(0) zero outside them and
     makes every parameter gradient a sum over the sampled graphs only.  The oracle therefore runs on
     the sampled graphs, compacted, and is compared with the full-size launch on E(T) of the sampled
     rows, on all of dE(0) and on all six parameter gradients."""
-    c = Case(synth.config_graphs(2), 20, 128, 64, "bf16", seed=23)
     assert L.band_uses_tensor_cores(c.plan, c.dtype, c.H)
-    T = 8
     saved = torch.empty(L.ggnn_saved_bytes(c.plan, c.dtype, c.H, T), dtype=torch.uint8,
                         device="cuda")
     ET = torch.empty_like(c.E_band_dev)
     L.ggnn_step(c.plan, c.dtype, c.H, T, c.dprm, c.E_band_dev, ET, saved, c.ws(L.BG_OP_GGNN_FWD, T))
     off, cnt = c.ref.graph_segments()
-    pick = np.random.default_rng(5).choice(len(off), 4, replace=False)
     rows = np.concatenate([np.arange(off[g], off[g] + cnt[g]) for g in pick])
     dET = np.zeros((c.N, c.H))
-    dET[rows] = quantize(np.random.default_rng(31).standard_normal((len(rows), c.H)), "f32")
+    dET[rows] = quantize(np.random.default_rng(seed).standard_normal((len(rows), c.H)), "f32")
     dE0 = torch.empty((c.N, c.H), dtype=torch.float32, device="cuda")
     grads = dict(dW=torch.empty((c.P, c.H, c.H), device="cuda"),
                  db=torch.empty((c.P, c.H), device="cuda"),
@@ -305,6 +303,26 @@ def test_full_size_config2_ggnn_T8_fwd_bwd_sampled_graphs():
     assert np.all(got_dE0[rest] == 0.0)
     for k, v in grads.items():
         assert rel_err(v.cpu().numpy(), ref[k]) < TOL["bf16"], k
+
+
+def test_full_size_config2_ggnn_T8_fwd_bwd_sampled_graphs():
+    """The benchmark workload end to end: config 2 at full size (64 graphs, ~72k nodes, P = 20,
+    S = 128, H = 64, bf16, T = 8) through the fused tensor-core path, forward + backward."""
+    c = Case(synth.config_graphs(2), 20, 128, 64, "bf16", seed=23)
+    off, _ = c.ref.graph_segments()
+    _full_size_ggnn_sampled_graphs(c, 8, np.random.default_rng(5).choice(len(off), 4, replace=False),
+                                   31)
+
+
+def test_full_size_config5_H128_ggnn_T8_fwd_bwd_sampled_graphs():
+    """Config 5's batch at full size and H = 128 (~100k nodes, 811 tiles, P = 20, S = 128, bf16,
+    T = 8): the band kernel's 64-column state passes and the GRU kernels with streamed weights,
+    forward + backward, against the oracle on three of the smaller graphs."""
+    c = Case(synth.config_graphs(5), 20, 128, 128, "bf16", seed=29)
+    off, cnt = c.ref.graph_segments()
+    small = np.flatnonzero(cnt <= 1500)
+    _full_size_ggnn_sampled_graphs(c, 8, np.random.default_rng(7).choice(small, 3, replace=False),
+                                   37)
 
 
 # ------------------------------------------------------------------------------------ failure path
