@@ -477,18 +477,19 @@ TcSaved tc_saved(const bg_plan* p, int H, int T) {
   return s;
 }
 struct TcFwdWs {
-  size_t WT, b2T, total;
+  size_t WT, b2T, split, total;
 };
 TcFwdWs tc_fwd_ws(const bg_plan* p, int H) {
   TcFwdWs w{};
   size_t o = 0;
   w.WT = o; o += bg::band_tc_w_bytes(p, H);
   w.b2T = o; o += al((size_t)H * 64 * 2);
+  w.split = o; o += al(sizeof(float) * bg::band_tc_split_floats(p, H));
   w.total = o;
   return w;
 }
 struct TcBwdWs {
-  size_t g, dXT, dMT, dgiT, dhnT, WihT, WhhT, Wk, part, total;
+  size_t g, dXT, dMT, dgiT, dhnT, WihT, WhhT, Wk, part, split, total;
 };
 size_t tc_part_floats(const bg_plan* p, int H, int T) {
   const int64_t K = (int64_t)T * p->n_pad();
@@ -509,6 +510,7 @@ TcBwdWs tc_bwd_ws(const bg_plan* p, int H, int T) {
   w.WhhT = o; o += al((size_t)3 * H * H * 2);
   w.Wk = o; o += bg::band_tc_w_bytes(p, H);
   w.part = o; o += al(sizeof(float) * tc_part_floats(p, H, T));
+  w.split = o; o += al(sizeof(float) * bg::band_tc_split_floats(p, H));
   w.total = o;
   return w;
 }
@@ -774,6 +776,8 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
     __nv_bfloat16* YTa = reinterpret_cast<__nv_bfloat16*>(sv + sl.YTa);
     void* WT = wsc + wl.WT;
     __nv_bfloat16* b2T = reinterpret_cast<__nv_bfloat16*>(wsc + wl.b2T);
+    float* split = bg::band_tc_split_floats(p, H) ? reinterpret_cast<float*>(wsc + wl.split)
+                                                   : nullptr;
     BG_CUDA(cudaMemcpyAsync(Ei(0), E0, n * H * 2, cudaMemcpyDeviceToDevice, st));
     BG_CUDA(bg::prep_transpose_bf16(E0, 0, ETa, (int)n, H, 1, st, (int64_t)TN));
     BG_CUDA(bg::fill_ones_rows(ETa, H, (int64_t)TN, (int64_t)TN, st));
@@ -785,7 +789,7 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
         KTimer tm(BG_KID_BAND_FWD, st);
         BG_CUDA(bg::band_tc_fwd_core(p, H, ETa + (size_t)t * n, (int64_t)TN, WT,
                                      prm->b ? b2T : nullptr, nullptr, Yi(t), YTa + (size_t)t * n,
-                                     (int64_t)TN, status, st));
+                                     (int64_t)TN, split, status, st));
       }
       KTimer tm(BG_KID_GRU_FWD, st);
       BG_CUDA(bg::gru_fwd_tc(
@@ -859,6 +863,8 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     __nv_bfloat16* WhhT = reinterpret_cast<__nv_bfloat16*>(wsc + wl.WhhT);
     float* part = reinterpret_cast<float*>(wsc + wl.part);
     const size_t pf = tc_part_floats(p, H, T);
+    float* split = bg::band_tc_split_floats(p, H) ? reinterpret_cast<float*>(wsc + wl.split)
+                                                   : nullptr;
     const auto* Wih = static_cast<const __nv_bfloat16*>(prm->W_ih);
     const auto* Whh = static_cast<const __nv_bfloat16*>(prm->W_hh);
     BG_CUDA(bg::prep_transpose_bf16(Wih, 0, WihT, 3 * H, H, 1, st));
@@ -875,7 +881,7 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
       }
       KTimer tm(BG_KID_BAND_BWD, st);
       BG_CUDA(bg::band_tc_bwd_core(p, H, dXT, (int64_t)n, Wk, g, 1, dMT + (size_t)t * n,
-                                   (int64_t)TN, status, st));
+                                   (int64_t)TN, split, status, st));
       gin = g;
     }
     const int acc = (flags & BG_ACCUM) ? 1 : 0;

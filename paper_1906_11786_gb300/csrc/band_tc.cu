@@ -172,13 +172,36 @@ __device__ __forceinline__ void drain_mmas(bool leader, uint64_t* bar) {
   }
 }
 
+// Work of one launch.  Items 0 .. n_full-1 are whole tiles; when the tiles do not fill the last
+// round of the grid evenly, each remaining tile is split into ksplit items over consecutive ranges
+// of its jobs, which write their partial Y (fp32) to their own slice of `part`, and a fix-up
+// kernel sums the slices in a fixed order into the outputs.
+struct Sched {
+  int n_items, n_full, ksplit, part_rows;
+  float* part;  // [ksplit][part_rows][H]: partial Y of split items, rows from tile n_full on
+};
+
+// Tile and job range [j0, j1) of item w; part -1 for a whole tile, else its slice.
+__device__ __forceinline__ void item_of(const Sched& sc, int w, int jobs, int& tile, int& j0,
+                                        int& j1, int& part) {
+  if (w < sc.n_full) {
+    tile = w, j0 = 0, j1 = jobs, part = -1;
+    return;
+  }
+  const int v = w - sc.n_full;
+  tile = sc.n_full + v / sc.ksplit;
+  part = v % sc.ksplit;
+  j0 = part * jobs / sc.ksplit;
+  j1 = (part + 1) * jobs / sc.ksplit;
+}
+
 template <int H, int S, bool BWD>
 __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     k_band_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
               const __grid_constant__ CUtensorMap tm_deg, const __grid_constant__ CUtensorMap tm_b2,
               const uint32_t* __restrict__ maskI, float* __restrict__ out,
               __nv_bfloat16* __restrict__ outb, __nv_bfloat16* __restrict__ outT, int64_t ld_outT,
-              __nv_bfloat16* __restrict__ dMT, int64_t ld_mt, int n_tiles, int P, int has_bias,
+              __nv_bfloat16* __restrict__ dMT, int64_t ld_mt, const Sched sc, int P, int has_bias,
               int accumulate, int* status) {
   using C = Cfg<H, S>;
   extern __shared__ uint8_t smem_raw[];
@@ -197,6 +220,7 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
   // issuer's commit and, backward, the 4 converter warps.
   constexpr int kFree = 1 + (BWD ? 4 : 0);
   const int jobs = C::NH * P;  // per tile
+  // bias: once per tile, by the whole tile or its first slice
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -244,34 +268,41 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     }
     // the state windows are the previous kernel's output (bit tiles, W, deg and b2 are not)
     grid_dep_wait();
-    uint32_t widx = 0, xi = 0;
+    uint32_t widx = 0, xi = 0, di = 0;
     uint32_t n_x[2] = {0, 0}, n_deg[2] = {0, 0}, n_w[4] = {0, 0, 0, 0};
-    int i = 0;
     bool ok = true;
-    for (int k = blockIdx.x; k < n_tiles && ok && !*abort; k += gridDim.x, ++i) {
+    for (int w = blockIdx.x; w < sc.n_items && ok && !*abort; w += gridDim.x) {
+      int k, j0, j1, part;
+      item_of(sc, w, jobs, k, j0, j1, part);
       const int row0 = k * kTile, ws = (row0 / S) * S - S;
-      if (has_bias) {
-        const int db = i % C::NDEG;
-        if (!mbar_wait(&bars->deg_empty[db], ((i / C::NDEG) & 1) ^ 1, status, 102, abort, 64)) break;
+      if (has_bias && part <= 0) {
+        const int db = di % C::NDEG;
+        if (!mbar_wait(&bars->deg_empty[db], ((di / C::NDEG) & 1) ^ 1, status, 102, abort, 64)) break;
         ++n_deg[db];
+        ++di;
         mbar_expect_tx(&bars->deg_full[db], C::DEG);
         tma_load_2d(degs + db * C::DEG, &tm_deg, &bars->deg_full[db], 0, row0);
       }
-      for (int hh = 0; hh < C::NH && ok; ++hh, ++xi) {
-        // window rows ws .. ws + 128 C1 of state columns 64 hh ..; rows outside [0, n) arrive as
-        // zeros (TMA bounds fill)
-        const int xb = xi % C::NXB;
-        if (!mbar_wait(&bars->x_empty[xb], ((xi / C::NXB) & 1) ^ 1, status, 101, abort, 64)) {
-          ok = false;
-          break;
+      // job jb = P hh + p, stepped without dividing (the issuers' loops are on the MMA issue path)
+      int hh = j0 / P, p = j0 - hh * P;
+      for (int jb = j0; jb < j1 && ok; ++jb, p = p + 1 == P ? (++hh, 0) : p + 1) {
+        if (jb == j0 || p == 0) {
+          // the window of the job's state slice: rows ws .. ws + 128 C1 of state columns SW hh ..;
+          // rows outside [0, n) arrive as zeros (TMA bounds fill)
+          const int xb = xi % C::NXB;
+          if (!mbar_wait(&bars->x_empty[xb], ((xi / C::NXB) & 1) ^ 1, status, 101, abort, 64)) {
+            ok = false;
+            break;
+          }
+          ++n_x[xb];
+          ++xi;
+          mbar_expect_tx(&bars->x_full[xb], C::XWIN);
+          for (int a = 0; a < 2 * C::C1; ++a)
+            tma_load_2d(xwin + xb * C::XWIN + a * C::ATOM_X, &tm_x, &bars->x_full[xb],
+                        ws + a * kAtom, C::SW * hh);
         }
-        ++n_x[xb];
-        mbar_expect_tx(&bars->x_full[xb], C::XWIN);
-        for (int a = 0; a < 2 * C::C1; ++a)
-          tma_load_2d(xwin + xb * C::XWIN + a * C::ATOM_X, &tm_x, &bars->x_full[xb],
-                      ws + a * kAtom, C::SW * hh);
-        // per job: K-columns 64 hh .. 64 hh + 63 of W_p^T in WJ stages of WK / 32 atoms
-        for (int p = 0; p < P && ok; ++p)
+        // per job: K-columns SW hh .. of W_p^T in WJ stages of WK / 32 atoms
+        {
           for (int wj = 0; wj < C::WJ; ++wj, ++widx) {
             const int ws2 = widx % C::NW;
             if (!mbar_wait(&bars->w_empty[ws2], ((widx / C::NW) & 1) ^ 1, status, 103, abort, 64)) {
@@ -284,6 +315,7 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
               tma_load_2d(wring + ws2 * C::WSTAGE + a * H * 128, &tm_w, &bars->w_full[ws2],
                           C::SW * hh + C::WK * wj + 32 * a, p * H);
           }
+        }
       }
     }
     if (*abort) {
@@ -302,10 +334,12 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     // each job's C1 bit chunks (contiguous [C1][128][4] words of its type), NM jobs ahead of the
     // expanders; both halves of a tile read the same bits
     uint32_t midx = 0, n_m[8] = {0};
-    for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x) {
+    for (int w = blockIdx.x; w < sc.n_items && !*abort; w += gridDim.x) {
+      int k, j0, j1, part;
+      item_of(sc, w, jobs, k, j0, j1, part);
       bool ok = true;
-      for (int jb = 0; jb < jobs; ++jb, ++midx) {
-        const int p = jb % P;
+      int p = j0 % P;
+      for (int jb = j0; jb < j1; ++jb, ++midx, p = p + 1 == P ? 0 : p + 1) {
         const int ms = midx % C::NM;
         if (!mbar_wait(&bars->m_empty[ms], ((midx / C::NM) & 1) ^ 1, status, 104, abort, 64)) {
           ok = false;
@@ -333,13 +367,18 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     // mod 2, kept as a group and a position within the job
     uint32_t nx_g = (C::NA / C::C1) & 1, nx_r = C::NA % C::C1;
     bool ok = true;
-    for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x) {
-      for (int hh = 0; hh < C::NH && ok; ++hh, ++xi) {
+    for (int w = blockIdx.x; w < sc.n_items && ok; w += gridDim.x) {
+      int k, j0, j1, part;
+      item_of(sc, w, jobs, k, j0, j1, part);
+      // segments of the item's jobs that share a state window (one slice each)
+      for (int jb = j0; jb < j1 && ok;) {
+        const int seg_end = min(j1, (jb / P + 1) * P);
         const int xb = xi % C::NXB;
         if (!mbar_wait(&bars->x_full[xb], (xi / C::NXB) & 1, status, 204, abort)) { ok = false; break; }
+        ++xi;
         // descriptors differ from the window's first one only in the start-address field
         const uint64_t xdesc = desc_sw128_kmajor(smem_u32(xwin + xb * C::XWIN));
-        for (int p = 0; p < P && ok; ++p, ++c) {
+        for (; jb < seg_end && ok; ++jb, ++c) {
           const uint32_t d1 = tmem + C::D1COL0 + (c % C::NB) * 64;
           for (int g = 0; g < C::G; ++g, ++gi) {
             if (!mbar_wait(&bars->t_full[gi % C::NT], (gi / C::NT) & 1, status, 210, abort)) { ok = false; break; }
@@ -362,8 +401,9 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
           }
           if (!ok) break;
           if (leader) tc_commit(&bars->d1_full[c % C::NB]);
-          if (p == P - 1 && leader) tc_commit(&bars->x_empty[xb]);
         }
+        if (!ok) break;
+        if (leader) tc_commit(&bars->x_empty[xb]);  // the segment's last job is issued
       }
     }
     drain_mmas(leader, &bars->drain);
@@ -374,14 +414,16 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     const bool leader = elect_one_sync();
     constexpr uint32_t idesc = idesc_bf16_f32(kTile, H);
     constexpr uint32_t idesc2 = idesc_tf32_f32(kTile, H);
-    uint32_t c = 0, widx = 0;
+    uint32_t c = 0, widx = 0, di = 0;
     bool ok = true;
     int i = 0;
-    for (int k = blockIdx.x; k < n_tiles && ok; k += gridDim.x, ++i) {
-      for (int jb = 0; jb < jobs && ok; ++jb, ++c) {
+    for (int w = blockIdx.x; w < sc.n_items && ok; w += gridDim.x, ++i) {
+      int k, j0, j1, part;
+      item_of(sc, w, jobs, k, j0, j1, part);
+      for (int jb = j0; jb < j1 && ok; ++jb, ++c) {
         const int b = c % C::NB;
         if (!mbar_wait(&bars->d1_full[b], (c / C::NB) & 1, status, 208, abort) ||
-            (jb == 0 && !mbar_wait(&bars->y_empty, (i & 1) ^ 1, status, 203, abort))) {
+            (jb == j0 && !mbar_wait(&bars->y_empty, (i & 1) ^ 1, status, 203, abort))) {
           ok = false;
           break;
         }
@@ -397,7 +439,7 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
           for (int kk = 0; kk < C::WK / 8; ++kk) {
             const uint64_t bdesc = desc_sw128_kmajor(wbase + (kk / 4) * H * 128 + (kk % 4) * 32);
             if (leader) mma_ts_tf32(tmem + C::YCOL, tmem + C::D1COL0 + b * 64 + C::WK * wj + kk * 8,
-                                    bdesc, idesc2, (jb == 0 && wj == 0 && kk == 0) ? 0u : 1u);
+                                    bdesc, idesc2, (jb == j0 && wj == 0 && kk == 0) ? 0u : 1u);
           }
           if (leader) tc_commit(&bars->w_empty[ws]);
         }
@@ -406,10 +448,11 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
         if (leader) tc_commit(&bars->t_full[((c + C::NB) * C::G) % C::NT]);
       }
       if (!ok) break;
-      if (has_bias) {
-        const int db = i % C::NDEG;
-        if (!mbar_wait(&bars->deg_full[db], (i / C::NDEG) & 1, status, 206, abort)) break;
-        if (i == 0 && !mbar_wait(&bars->b2_full, 0, status, 207, abort)) break;
+      if (has_bias && part <= 0) {
+        const int db = di % C::NDEG;
+        if (!mbar_wait(&bars->deg_full[db], (di / C::NDEG) & 1, status, 206, abort)) break;
+        if (di == 0 && !mbar_wait(&bars->b2_full, 0, status, 207, abort)) break;
+        ++di;
         tc_fence_after();
         const uint32_t dbase = smem_u32(degs + db * C::DEG), bbase = smem_u32(b2s);
 #pragma unroll
@@ -420,6 +463,9 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
       }
       if (leader) tc_commit(&bars->y_full);
     }
+    // a CTA whose items were all later slices of split tiles never used the bias rows it loaded:
+    // let that copy land before the CTA's shared memory is released
+    if (has_bias && di == 0) mbar_wait(&bars->b2_full, 0, status, 209, abort);
     drain_mmas(leader, &bars->drain2);
   } else if (warp >= 4 && warp < 4 + 4 * C::NE) {
     // ------------------------------------------------------------------ expanders
@@ -429,9 +475,11 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     uint32_t aidx = 0, midx = 0;
     uint32_t par = 0;  // bit s: parity of this group's waits so far on A slot s
-    for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x) {
+    for (int w = blockIdx.x; w < sc.n_items && !*abort; w += gridDim.x) {
+      int k, j0, j1, part;
+      item_of(sc, w, jobs, k, j0, j1, part);
       bool ok = true;
-      for (int jb = 0; jb < jobs && ok; ++jb, ++midx) {
+      for (int jb = j0; jb < j1 && ok; ++jb, ++midx) {
         if ((int)(midx % C::NE) != eg) {
           aidx += C::C1;  // the other group's job
           continue;
@@ -479,11 +527,14 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     uint32_t c = 0;
     int i = 0;
-    for (int k = blockIdx.x; k < n_tiles && !*abort; k += gridDim.x, ++i) {
+    for (int w = blockIdx.x; w < sc.n_items && !*abort; w += gridDim.x, ++i) {
+      int k, j0, j1, part;
+      item_of(sc, w, jobs, k, j0, j1, part);
       const int row = k * kTile + r;
       bool ok = true;
-      for (int jb = 0; BWD && jb < jobs; ++jb, ++c) {
-        const int b = c % C::NB, p = jb % P, hh = jb / P;
+      int hh = j0 / P, p = j0 - hh * P;
+      for (int jb = j0; BWD && jb < j1; ++jb, ++c, p = p + 1 == P ? (++hh, 0) : p + 1) {
+        const int b = c % C::NB;
         if (!mbar_wait(&bars->d1_full[b], (c / C::NB) & 1, status, 401, abort, 64)) { ok = false; break; }
         tc_fence_after();
         const uint32_t col = tmem + lane_base + C::D1COL0 + b * 64;
@@ -529,6 +580,16 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
         for (int h1 = 0; h1 < YG; h1 += 32) {
           const int h0 = g0 + h1;
           const uint32_t* v = vg + h1;
+          if (part >= 0) {
+            // a slice of a split tile: its partial Y, summed with the other slices' by the fix-up
+            float4* o = reinterpret_cast<float4*>(
+                sc.part + ((size_t)part * sc.part_rows + (size_t)(k - sc.n_full) * kTile + r) * H + h0);
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              o[j] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                 __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+            continue;
+          }
           if (out) {
             float4* o = reinterpret_cast<float4*>(out + (size_t)row * H + h0);
 #pragma unroll
@@ -615,6 +676,44 @@ __global__ void k_prep_w(const __nv_bfloat16* __restrict__ W, float* __restrict_
   out[t] = __bfloat162float(transpose ? W[(p * H + c) * H + a] : W[(p * H + a) * H + c]);
 }
 
+// Outputs of the split tiles: Y = sum over the ksplit slices of `part` (fixed order), written like
+// the band kernel's own epilogue (fp32 out, accumulating if asked; bf16 row-major; bf16
+// transposed).  Rows row0 .. row0 + part_rows.
+__global__ void k_band_split_fixup(const float* __restrict__ part, int ksplit, int part_rows,
+                                   int row0, int H, float* __restrict__ out,
+                                   __nv_bfloat16* __restrict__ outb,
+                                   __nv_bfloat16* __restrict__ outT, int64_t ld_outT,
+                                   int accumulate) {
+  grid_dep_wait();  // the partials are the band kernel's output
+  const int64_t n4 = (int64_t)part_rows * H / 4, slice = (int64_t)part_rows * H;
+  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < n4;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t e = 4 * t;
+    float4 y = *reinterpret_cast<const float4*>(part + e);
+    for (int q = 1; q < ksplit; ++q) {
+      const float4 v = *reinterpret_cast<const float4*>(part + q * slice + e);
+      y.x += v.x; y.y += v.y; y.z += v.z; y.w += v.w;
+    }
+    const int row = row0 + (int)(e / H), h = (int)(e % H);
+    if (out) {
+      float4* o = reinterpret_cast<float4*>(out + (size_t)row * H + h);
+      if (accumulate) {
+        const float4 prev = *o;
+        y.x += prev.x; y.y += prev.y; y.z += prev.z; y.w += prev.w;
+      }
+      *o = y;
+    }
+    const uint32_t p0 = pack_bf16(y.x, y.y), p1 = pack_bf16(y.z, y.w);
+    if (outb) *reinterpret_cast<uint2*>(outb + (size_t)row * H + h) = make_uint2(p0, p1);
+    if (outT) {
+      outT[(size_t)h * ld_outT + row] = __ushort_as_bfloat16((unsigned short)(p0 & 0xFFFFu));
+      outT[(size_t)(h + 1) * ld_outT + row] = __ushort_as_bfloat16((unsigned short)(p0 >> 16));
+      outT[(size_t)(h + 2) * ld_outT + row] = __ushort_as_bfloat16((unsigned short)(p1 & 0xFFFFu));
+      outT[(size_t)(h + 3) * ld_outT + row] = __ushort_as_bfloat16((unsigned short)(p1 >> 16));
+    }
+  }
+}
+
 // b2T[h][p] = bf16 hi part of b[p][h], b2T[h][32 + p] = bf16 of the remainder (zero beyond P)
 __global__ void k_bias_split(const float* __restrict__ b, __nv_bfloat16* __restrict__ b2T, int P,
                              int H) {
@@ -667,21 +766,58 @@ int num_sms() {
 
 inline size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
 
+// State columns per pass of the band kernel (Cfg::SW) and so its jobs per tile.
+int band_jobs(int H, int S, int P) { return H / ((H < 64 || S == 512) ? 32 : 64) * P; }
+
+// Work items of a launch over n_tiles tiles on `sms` SMs, one CTA per SM: whole tiles, and when
+// the last round of the grid would be mostly idle, its tiles split over k in {2, 4} job ranges
+// (rounds of a k-th of a tile: ceil(k tail / sms) / k).  A split tile costs extra window loads,
+// partial-sum traffic and the fix-up launch, measured at about half a tile round, so the split is
+// taken only when the tail then lasts less than half a round (single20k: 158 tiles on 152 SMs,
+// +28%; a tail of 110 of 152 tiles split four ways measured 9% slower).
+Sched make_sched(int n_tiles, int jobs, int sms, bool can_split) {
+  Sched sc{};
+  sc.n_items = sc.n_full = n_tiles;
+  sc.ksplit = 1;
+  const int full = (n_tiles / sms) * sms, tail = n_tiles - full;
+  if (!can_split || tail == 0) return sc;
+  int best = 1;
+  double best_t = 1.0;
+  for (int k = 2; k <= 4 && k <= jobs; k *= 2) {
+    const double t = (double)((k * tail + sms - 1) / sms) / k;
+    if (t < best_t - 1e-9) best_t = t, best = k;
+  }
+  if (best == 1 || best_t >= 0.5) return sc;
+  sc.n_full = full;
+  sc.ksplit = best;
+  sc.n_items = full + best * tail;
+  sc.part_rows = tail * kTile;
+  return sc;
+}
+
 template <int H, int S, bool BWD>
 cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
                      const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
                      __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
-                     __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate, int* status,
-                     cudaStream_t st) {
+                     __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate,
+                     float* split, int* status, cudaStream_t st) {
   using C = Cfg<H, S>;
   cudaError_t e = cudaFuncSetAttribute(k_band_tc<H, S, BWD>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
-  const int n_tiles = p->n_pad() / kTile;
-  const int grid = std::min(n_tiles, num_sms());
+  const int n_tiles = p->n_pad() / kTile, sms = num_sms();
+  Sched sc = make_sched(n_tiles, C::NH * p->P, sms, split != nullptr);
+  sc.part = split;
+  const int grid = std::min(sc.n_items, sms);
   e = launch_pdl(k_band_tc<H, S, BWD>, dim3(grid), dim3(C::THREADS), C::SMEM, st, tx, tw, tdeg,
-                 tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt,
-                 n_tiles, p->P, has_bias, accumulate, status);
+                 tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt, sc,
+                 p->P, has_bias, accumulate, status);
+  note_launch();
+  if (e != cudaSuccess || sc.ksplit == 1) return e;
+  const int64_t n4 = (int64_t)sc.part_rows * H / 4;
+  e = launch_pdl(k_band_split_fixup, dim3((unsigned)std::min<int64_t>((n4 + 255) / 256, 2048)),
+                 dim3(256), 0, st, (const float*)split, sc.ksplit, sc.part_rows,
+                 sc.n_full * kTile, H, out, outb, outT, ld_outT, accumulate);
   note_launch();
   return e;
 }
@@ -692,11 +828,11 @@ template <int H, bool BWD>
 cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& tw,
                    const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
                    __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
-                   __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate, int* status,
-                   cudaStream_t st) {
+                   __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate, float* split,
+                   int* status, cudaStream_t st) {
 #define BG_BAND_S(SV)                                                                            \
   return launch_s<H, SV, BWD>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, dMT, ld_mt,      \
-                              has_bias, accumulate, status, st);
+                              has_bias, accumulate, split, status, st);
   switch (p->S) {
     case 32: BG_BAND_S(32)
     case 64: BG_BAND_S(64)
@@ -784,7 +920,8 @@ cudaError_t band_tc_prep_w(const bg_plan* p, int H, const void* W, int bwd, void
 size_t band_tc_fwd_ws_bytes(const bg_plan* p, int dtype, int H) {
   if (!p || dtype != 1) return 0;
   const size_t n = (size_t)p->n_pad();
-  return al256(n * H * 2) + band_tc_w_bytes(p, H) + al256((size_t)H * 64 * 2);
+  return al256(n * H * 2) + band_tc_w_bytes(p, H) + al256((size_t)H * 64 * 2) +
+         al256(sizeof(float) * band_tc_split_floats(p, H));
 }
 
 size_t band_tc_bwd_ws_bytes(const bg_plan* p, int dtype, int H) {
@@ -792,50 +929,56 @@ size_t band_tc_bwd_ws_bytes(const bg_plan* p, int dtype, int H) {
   const size_t n = (size_t)p->n_pad();
   return al256(n * H * 2) + al256((size_t)p->P * H * n * 2) + al256((size_t)(H + 16) * n * 2) +
          band_tc_w_bytes(p, H) +
-         al256(sizeof(float) * gemm_tn_part_floats(p->P * H, H + 16, (int64_t)n));
+         al256(sizeof(float) * gemm_tn_part_floats(p->P * H, H + 16, (int64_t)n)) +
+         al256(sizeof(float) * band_tc_split_floats(p, H));
+}
+
+size_t band_tc_split_floats(const bg_plan* p, int H) {
+  const Sched sc = make_sched(p->n_pad() / kTile, band_jobs(H, p->S, p->P), num_sms(), true);
+  return sc.ksplit > 1 ? (size_t)sc.ksplit * sc.part_rows * H : 0;
 }
 
 cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, int64_t ld_x,
                              const void* Wk, const __nv_bfloat16* b2T, float* out,
                              __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
-                             int* status, cudaStream_t st) {
+                             float* split, int* status, cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw, tdeg, tb2;
-  if (!make_map_ld(&tx, XT, H, n, ld_x, (H < 64 || p->S == 512) ? 32 : 64) || !make_map_w(&tw, Wk, P, H) ||
-      !make_map(&tdeg, p->d_deg2, n, 64, kTile) || !make_map(&tb2, b2T ? b2T : XT, H, 64, H))
+  if (!make_map_ld(&tx, XT, H, n, ld_x, (H < 64 || p->S == 512) ? 32 : 64) ||
+      !make_map_w(&tw, Wk, P, H) || !make_map(&tdeg, p->d_deg2, n, 64, kTile) ||
+      !make_map(&tb2, b2T ? b2T : XT, H, 64, H))
     return cudaErrorInvalidValue;
-  const int has_bias = b2T != nullptr;
-  if (H == 32)
-    return launch<32, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, has_bias,
-                             0, status, st);
-  if (H == 64)
-    return launch<64, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, has_bias,
-                             0, status, st);
-  if (H == 128)
-    return launch<128, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, has_bias,
-                              0, status, st);
-  return launch<256, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, has_bias,
-                            0, status, st);
+  const int hb = b2T != nullptr;
+#define BG_FWD(HV)                                                                                \
+  return launch<HV, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, hb, 0,     \
+                           split, status, st);
+  switch (H) {
+    case 32: BG_FWD(32)
+    case 64: BG_FWD(64)
+    case 128: BG_FWD(128)
+    default: BG_FWD(256)
+  }
+#undef BG_FWD
 }
 
 cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, int64_t ld_y,
                              const void* Wk, float* dE, int accumulate, __nv_bfloat16* dMT,
-                             int64_t ld_mt, int* status, cudaStream_t st) {
+                             int64_t ld_mt, float* split, int* status, cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw;
-  if (!make_map_ld(&tx, dYT, H, n, ld_y, (H < 64 || p->S == 512) ? 32 : 64) || !make_map_w(&tw, Wk, P, H))
+  if (!make_map_ld(&tx, dYT, H, n, ld_y, (H < 64 || p->S == 512) ? 32 : 64) ||
+      !make_map_w(&tw, Wk, P, H))
     return cudaErrorInvalidValue;
-  if (H == 32)
-    return launch<32, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
-                            status, st);
-  if (H == 64)
-    return launch<64, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
-                            status, st);
-  if (H == 128)
-    return launch<128, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
-                             status, st);
-  return launch<256, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,
-                           status, st);
+#define BG_BWD(HV)                                                                                \
+  return launch<HV, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,  \
+                          split, status, st);
+  switch (H) {
+    case 32: BG_BWD(32)
+    case 64: BG_BWD(64)
+    case 128: BG_BWD(128)
+    default: BG_BWD(256)
+  }
+#undef BG_BWD
 }
 
 cudaError_t prep_transpose_bf16(const void* in, int in_is_f32, __nv_bfloat16* out, int R, int Cc,
@@ -867,13 +1010,16 @@ cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, c
   void* WT = ws + al256((size_t)n * H * 2);
   __nv_bfloat16* b2T = reinterpret_cast<__nv_bfloat16*>(ws + al256((size_t)n * H * 2) +
                                                         band_tc_w_bytes(p, H));
+  float* split = reinterpret_cast<float*>(ws + al256((size_t)n * H * 2) + band_tc_w_bytes(p, H) +
+                                          al256((size_t)H * 64 * 2));
   // E [n][H] -> ET [H][n];  W_p [H_in][H_out] -> W_p^T in the kernel's operand type;  bias split
   cudaError_t e = prep_transpose_bf16(E, 0, ET, n, H, 1, st);
   if (e == cudaSuccess) e = band_tc_prep_w(p, H, W, 0, WT, st);
   if (e == cudaSuccess && b) e = prep_bias_split(b, b2T, P, H, st);
   if (e != cudaSuccess) return e;
   ProfSpan span(BG_KID_BAND_FWD, st);
-  return band_tc_fwd_core(p, H, ET, n, WT, b ? b2T : nullptr, Y, nullptr, nullptr, 0, status, st);
+  return band_tc_fwd_core(p, H, ET, n, WT, b ? b2T : nullptr, Y, nullptr, nullptr, 0,
+                          band_tc_split_floats(p, H) ? split : nullptr, status, st);
 }
 
 cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, const float* dY,
@@ -892,11 +1038,13 @@ cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, c
   o += band_tc_w_bytes(p, H);
   float* part = reinterpret_cast<float*>(ws + o);
   const size_t part_floats = gemm_tn_part_floats(P * H, H + 16, (int64_t)n);
+  o += al256(sizeof(float) * part_floats);
+  float* split = band_tc_split_floats(p, H) ? reinterpret_cast<float*>(ws + o) : nullptr;
   cudaError_t e = prep_transpose_bf16(dY, 1, dYT, n, H, 1, st);
   if (e == cudaSuccess) e = band_tc_prep_w(p, H, W, 1, Wk, st);
   if (e == cudaSuccess) {
     ProfSpan span(BG_KID_BAND_BWD, st);
-    e = band_tc_bwd_core(p, H, dYT, n, Wk, dE, accum, dMT, n, status, st);
+    e = band_tc_bwd_core(p, H, dYT, n, Wk, dE, accum, dMT, n, split, status, st);
   }
   if (e != cudaSuccess) return e;
   // [E^T; 1; 0]: the ones row turns the bias gradient into column H of the same product

@@ -28,14 +28,17 @@ cudaError_t band_tc_prep_w(const bg_plan* p, int H, const void* W, int bwd, void
 //   XT: [H][>= n_pad] bf16 transposed states (row stride ld_x); Wk: band_tc_prep_w(bwd = 0);
 //   b2T: [H][64] bf16 bias split or NULL.  Outputs (each optional): out fp32 [n][H],
 //   outb bf16 [n][H], outT bf16 [H][ld_outT].
+//   split: fp32 scratch of band_tc_split_floats(p, H) floats (may be NULL: no tile splitting) for
+//   the partial outputs of tiles that the launch splits over several CTAs.
+size_t band_tc_split_floats(const bg_plan* p, int H);
 cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, int64_t ld_x,
                              const void* Wk, const __nv_bfloat16* b2T, float* out,
                              __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
-                             int* status, cudaStream_t st);
+                             float* split, int* status, cudaStream_t st);
 //   dYT: [H][>= n_pad] bf16; Wk: band_tc_prep_w(bwd = 1); dE fp32 (+)=; dMT: [P*H][ld_mt] bf16.
 cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, int64_t ld_y,
                              const void* Wk, float* dE, int accumulate, __nv_bfloat16* dMT,
-                             int64_t ld_mt, int* status, cudaStream_t st);
+                             int64_t ld_mt, float* split, int* status, cudaStream_t st);
 // out[c * ld_out + r] = bf16(in[r][c]) for `batch` consecutive R x Cc matrices (in fp32 or bf16;
 // ld_out <= 0 means R; batches are R*Cc apart on both sides).
 cudaError_t prep_transpose_bf16(const void* in, int in_is_f32, __nv_bfloat16* out, int R, int Cc,
