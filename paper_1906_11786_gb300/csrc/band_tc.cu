@@ -549,13 +549,16 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
 #pragma unroll
         for (int j = 0; j < C::SW / 2; ++j)
           pk[j] = pack_bf16(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
-        // dM_p (bf16) transposed: dMT[(p*H + h) * ld_mt + row]
+        // dM_p (bf16) transposed, dMT[(p*H + h) * ld_mt + row], as 4-byte words of two rows: a
+        // lane pair swaps its packed (h, h + 1) pairs, then the even lane stores column h of rows
+        // (row, row + 1) and the odd lane column h + 1 of rows (row - 1, row)
+        const bool odd = lane & 1;
 #pragma unroll
         for (int j = 0; j < C::SW / 2; ++j) {
-          const uint32_t w2 = pk[j];
-          __nv_bfloat16* d = dMT + ((size_t)p * H + C::SW * hh + 2 * j) * ld_mt + row;
-          d[0] = __ushort_as_bfloat16((unsigned short)(w2 & 0xFFFFu));
-          d[ld_mt] = __ushort_as_bfloat16((unsigned short)(w2 >> 16));
+          const uint32_t other = __shfl_xor_sync(0xffffffffu, pk[j], 1);
+          const uint32_t word = odd ? __byte_perm(other, pk[j], 0x7632) : __byte_perm(pk[j], other, 0x5410);
+          *reinterpret_cast<uint32_t*>(dMT + ((size_t)p * H + C::SW * hh + 2 * j + odd) * ld_mt +
+                                       (row & ~1)) = word;
         }
       }
       if (!ok) break;
