@@ -130,26 +130,30 @@ __device__ __forceinline__ void read_sw128_f32_row8(const uint8_t* tile, int r, 
   out[1] = *reinterpret_cast<const float4*>(row + (((j0 + 1) ^ (r & 7)) << 4));
 }
 
-// 4 bf16 pairs stored transposed: dst[(h0 + 2j + u) * ld + row]
-__device__ __forceinline__ void store_T4(__nv_bfloat16* dst, int64_t ld, int row, int h0,
-                                         const uint32_t* pk) {
+// N bf16 pairs (columns h0 + 2j, h0 + 2j + 1 of this lane's row) stored transposed,
+// dst[(h0 + 2j + u) * ld + row], as 4-byte words of two rows: the rows of a warp are consecutive
+// (row parity = lane parity), so a lane pair swaps its pairs with one shuffle and the even lane
+// writes column h0 + 2j of both rows, the odd lane column h0 + 2j + 1.  Every lane of the warp
+// calls it; ld and the row pair's first row are even.
+template <int N>
+__device__ __forceinline__ void store_T_pairs(__nv_bfloat16* dst, int64_t ld, int row, int h0,
+                                              const uint32_t* pk) {
+  const int odd = row & 1;
+  __nv_bfloat16* base = dst + (size_t)(h0 + odd) * ld + (row & ~1);
 #pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    __nv_bfloat16* t = dst + (size_t)(h0 + 2 * j) * ld + row;
-    t[0] = __ushort_as_bfloat16((unsigned short)(pk[j] & 0xFFFFu));
-    t[ld] = __ushort_as_bfloat16((unsigned short)(pk[j] >> 16));
+  for (int j = 0; j < N; ++j) {
+    const uint32_t other = __shfl_xor_sync(0xffffffffu, pk[j], 1);
+    const uint32_t word = odd ? __byte_perm(other, pk[j], 0x7632) : __byte_perm(pk[j], other, 0x5410);
+    *reinterpret_cast<uint32_t*>(base + (size_t)(2 * j) * ld) = word;
   }
 }
-
-// 8 bf16 pairs stored transposed: dst[(h0 + 2j + u) * ld + row]
+__device__ __forceinline__ void store_T4(__nv_bfloat16* dst, int64_t ld, int row, int h0,
+                                         const uint32_t* pk) {
+  store_T_pairs<4>(dst, ld, row, h0, pk);
+}
 __device__ __forceinline__ void store_T8(__nv_bfloat16* dst, int64_t ld, int row, int h0,
                                          const uint32_t* pk) {
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    __nv_bfloat16* t = dst + (size_t)(h0 + 2 * j) * ld + row;
-    t[0] = __ushort_as_bfloat16((unsigned short)(pk[j] & 0xFFFFu));
-    t[ld] = __ushort_as_bfloat16((unsigned short)(pk[j] >> 16));
-  }
+  store_T_pairs<8>(dst, ld, row, h0, pk);
 }
 
 template <int KH>
