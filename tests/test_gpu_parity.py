@@ -231,25 +231,81 @@ def test_readout_loss_and_adam():
 # ------------------------------------------------------------------------------------ full size
 
 
-def test_full_size_config2_propagate_sampled_rows():
-    """Config 2 at full size (64 graphs, ~72k nodes, P = 20, S = 128, H = 64, bf16): one forward
-    and backward propagation in the benchmark's launch configuration; the oracle computes a
-    seeded sample of output rows one by one (edges into sampled rows for Y; edges out of sampled
-    rows for dE) plus the exact dW and db."""
-    c = Case(synth.config_graphs(2), 20, 128, 64, "bf16", seed=21)
+def _full_size_propagation(c: Case, seed: int, n_rows: int = 400, types=(0, 7, 13)):
+    """One forward and one backward propagation through the C ABI on a full-size plan (the
+    benchmark's launches), checked on outputs the oracle computes one by one:
+      Y on sampled rows, from the kept edges into those rows (Eq. 1, Eq. 3);
+      dE on the same rows, from a compacted problem holding the rows and the targets of their
+      out-edges (dE[u] = sum_p (sum over edges u -> v of type p of dY[v]) W_p^T needs nothing else);
+      dW_p and db_p for sampled types p, from the edges of those types over all nodes.
+    Padding rows must come back as exact zeros in Y and dE."""
+    assert L.band_uses_tensor_cores(c.plan, c.dtype, c.H)
     Y = torch.empty((c.N, c.H), dtype=torch.float32, device="cuda")
     L.band_propagate_fwd(c.plan, c.dtype, c.H, c.E_band_dev, c.dprm["W"], c.dprm["b"], Y,
                          c.ws(L.BG_OP_PROPAGATE_FWD))
+    dY = quantize(np.random.default_rng(seed).standard_normal((c.N, c.H)), "f32")
+    dY[c.n_real:] = 0
+    dE = torch.empty((c.N, c.H), dtype=torch.float32, device="cuda")
+    dW = torch.empty((c.P, c.H, c.H), dtype=torch.float32, device="cuda")
+    db = torch.empty((c.P, c.H), dtype=torch.float32, device="cuda")
+    L.band_propagate_bwd(c.plan, c.dtype, c.H, c.E_band_dev, c.dprm["W"], f32_dev(dY), dE, dW, db,
+                         c.ws(L.BG_OP_PROPAGATE_BWD))
     torch.cuda.synchronize()
-    rows = np.unique(np.concatenate([np.random.default_rng(0).integers(0, c.n_real, 400),
-                                     [0, c.n_real - 1, c.N - 1]]))
+    L.check_device()
+    Y, dE, dW, db = (x.cpu().numpy() for x in (Y, dE, dW, db))
+    assert np.all(Y[c.n_real:] == 0) and np.all(dE[c.n_real:] == 0)
+
+    rows = np.unique(np.concatenate([np.random.default_rng(seed + 1).integers(0, c.n_real, n_rows),
+                                     [0, c.n_real - 1]]))
     d, s, t = c.edges
     sel = np.isin(d, rows)
     ref = oracle.propagate_fwd(c.N, c.P, c.H, d[sel], s[sel], t[sel], c.E_band, c.prm["W"],
                                c.prm["b"])
-    assert rel_err(Y.cpu().numpy()[rows], ref[rows]) < TOL["bf16"]
-    L.check_device()
+    assert rel_err(Y[rows], ref[rows]) < TOL["bf16"], "Y"
 
+    out = np.isin(s, rows)
+    nodes = np.unique(np.concatenate([rows, d[out]]))
+    new = np.full(c.N, -1, np.int64)
+    new[nodes] = np.arange(len(nodes))
+    ref_dE, _, _ = oracle.propagate_bwd(len(nodes), c.P, c.H, new[d[out]], new[s[out]], t[out],
+                                        c.E_band[nodes], c.prm["W"], dY[nodes])
+    assert rel_err(dE[rows], ref_dE[new[rows]]) < TOL["bf16"], "dE"
+
+    types = np.asarray(types)
+    tmap = np.full(c.P, -1, np.int64)
+    tmap[types] = np.arange(len(types))
+    ts = tmap[t] >= 0
+    _, ref_dW, ref_db = oracle.propagate_bwd(c.N, len(types), c.H, d[ts], s[ts], tmap[t[ts]],
+                                             c.E_band, c.prm["W"][types], dY)
+    assert rel_err(dW[types], ref_dW) < TOL["bf16"], "dW"
+    assert rel_err(db[types], ref_db) < TOL["bf16"], "db"
+
+
+def test_full_size_config2_propagate_sampled_rows():
+    """Config 2 at full size (64 graphs, ~72k nodes, 566 tiles, P = 20, S = 128, H = 64, bf16):
+    one forward and backward propagation, every tile whole."""
+    _full_size_propagation(Case(synth.config_graphs(2), 20, 128, 64, "bf16", seed=21), 41)
+
+
+def test_full_size_config3_propagate_sampled_rows():
+    """Config 3 at full size (one 20,000-node graph, S = 256, H = 128, 158 tiles): on a GPU with a
+    few SMs fewer than tiles, a whole round of tiles runs as whole tiles and the few tiles left are
+    split over several CTAs (partial sums and the fix-up kernel), the schedule the benchmark runs."""
+    c = Case(synth.config_graphs(3), 20, 256, 128, "bf16", seed=43)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    tiles = c.N // 128
+    assert tiles > sms and tiles % sms < sms // 2
+    _full_size_propagation(c, 47)
+
+
+@pytest.mark.parametrize("S", [32, 256, 512])
+def test_full_size_config4_propagate_sampled_rows(S):
+    """The block-size sweep at full size (131,072 positions, P = 20, H = 64, max offset S / 2):
+    S = 32 (four block-rows per tile), S = 256 (six window chunks) and S = 512 (32-column state
+    slices over a twelve-chunk window), with the sweep's capacity of 131,072 / S blocks."""
+    c = Case(synth.config_graphs(4, S=S), 20, S, 64, "bf16", seed=50 + S, cap=-(-131072 // S))
+    assert c.N == 131072
+    _full_size_propagation(c, 53 + S)
 
 
 def _full_size_ggnn_sampled_graphs(c: Case, T: int, pick, seed: int):
