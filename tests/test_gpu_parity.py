@@ -359,6 +359,7 @@ def _full_size_ggnn_sampled_graphs(c: Case, T: int, pick, seed: int):
     assert np.all(got_dE0[rest] == 0.0)
     for k, v in grads.items():
         assert rel_err(v.cpu().numpy(), ref[k]) < TOL["bf16"], k
+    return ET
 
 
 def test_full_size_config2_ggnn_T8_fwd_bwd_sampled_graphs():
@@ -370,15 +371,37 @@ def test_full_size_config2_ggnn_T8_fwd_bwd_sampled_graphs():
                                    31)
 
 
-def test_full_size_config5_H128_ggnn_T8_fwd_bwd_sampled_graphs():
-    """Config 5's batch at full size and H = 128 (~100k nodes, 811 tiles, P = 20, S = 128, bf16,
-    T = 8): the band kernel's 64-column state passes and the GRU kernels with streamed weights,
-    forward + backward, against the oracle on three of the smaller graphs."""
-    c = Case(synth.config_graphs(5), 20, 128, 128, "bf16", seed=29)
+@pytest.mark.parametrize("H", [32, 128, 256])
+def test_full_size_config5_ggnn_T8_fwd_bwd_sampled_graphs(H):
+    """Config 5's batch at full size with the benchmark's capacity (100,000 positions rounded up to
+    whole blocks: 782 tiles, P = 20, S = 128, bf16, T = 8), forward + backward against the oracle on
+    a few of the smaller graphs: H = 32 (32-column band products, resident-weight GRU kernels),
+    H = 128 (64-column state passes, GRU weights streamed), H = 256 (four state passes, the GRU on
+    tensor-core GEMMs); H = 64 runs at full size as config 2.  On a 152-SM GB300 the band kernels
+    run five whole rounds of tiles and split the 22-tile tail four ways.  The training step's mean-pool readout and loss are checked over the whole batch on the E(T) the
+    launch produced."""
+    cap = -(-synth.CONFIGS[5]["sizes"][1] // 128)
+    c = Case(synth.config_graphs(5), 20, 128, H, "bf16", seed=29, cap=cap)
+    assert c.N == cap * 128
     off, cnt = c.ref.graph_segments()
-    small = np.flatnonzero(cnt <= 1500)
-    _full_size_ggnn_sampled_graphs(c, 8, np.random.default_rng(7).choice(small, 3, replace=False),
-                                   37)
+    if H <= 128:
+        pick = np.random.default_rng(7).choice(np.flatnonzero(cnt <= 1500), 3, replace=False)
+    else:
+        pick = np.argsort(cnt, kind="stable")[:2]  # the oracle's cost grows with H^2
+    ET = _full_size_ggnn_sampled_graphs(c, 8, pick, 37)
+    target = np.random.default_rng(11).standard_normal(len(off))
+    loss = torch.zeros(4, device="cuda")
+    dET = torch.empty((c.N, c.H), device="cuda")
+    dw = torch.empty(c.H, device="cuda")
+    L.readout_loss(c.plan, c.dtype, c.H, ET, c.dprm["w_out"], f32_dev(target), loss, dET, dw,
+                   c.ws(L.BG_OP_READOUT))
+    torch.cuda.synchronize()
+    L.check_device()
+    rl, rdE, rdw = oracle.readout_loss(ET.float().cpu().numpy().astype(np.float64), off, cnt,
+                                       c.prm["w_out"], target)
+    assert abs(loss[0].item() - rl) / abs(rl) < 1e-4
+    assert rel_err(dET.cpu().numpy(), rdE) < 1e-4
+    assert rel_err(dw.cpu().numpy(), rdw) < 1e-4
 
 
 # ------------------------------------------------------------------------------------ failure path
