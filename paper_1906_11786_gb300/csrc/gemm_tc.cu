@@ -249,13 +249,20 @@ __global__ void k_gemm_tn_reduce(const float* __restrict__ part, int splits, int
 // ---------------------------------------------------------------------------------------------
 // Batched TN GEMM: C[b][m][n] (+)= sum_k A[b][m][k] B[b][n][k] (+ bias[b][n]); one 128 x BN output
 // tile per CTA, K streamed in 64-wide chunks through a 4-stage TMA ring.
+// One 128 x BN output tile per CTA.  Two stages keep a CTA under half of the SM's shared memory
+// (96 KB at BN = 256) and its accumulator at most 256 TMEM columns, so two CTAs share an SM and one's
+// epilogue overlaps the other's loads and MMAs (with four stages, one CTA per SM ran its load,
+// MMA and epilogue back to back).
+constexpr int kStagesB = 2;
 template <int BN>
 struct BCfg {
   static constexpr int A_BYTES = 128 * 128;
   static constexpr int B_BYTES = BN * 128;
   static constexpr int STAGE = A_BYTES + B_BYTES;
-  static constexpr int SMEM = kStages * STAGE + 1024 + 1024;
+  static constexpr int SMEM = kStagesB * STAGE + 1024 + 1024;
   static constexpr int TCOLS = BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  static_assert(2 * (SMEM + 1024) <= 233472 && 2 * TCOLS <= 512, "two CTAs per SM");
+  static_assert(4 * 32 * 33 * 4 <= kStagesB * STAGE, "epilogue transpose buffers");
 };
 
 struct BatchArgs {
@@ -268,16 +275,16 @@ struct BatchArgs {
 };
 
 template <int BN>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(192, 2)
     k_gemm_bf16(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 BatchArgs g, int* status) {
   using C = BCfg<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * C::STAGE);
-  uint64_t* empty = full + kStages;
-  uint64_t* done = empty + kStages;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStagesB * C::STAGE);
+  uint64_t* empty = full + kStagesB;
+  uint64_t* done = empty + kStagesB;
   uint64_t* drain = done + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
@@ -285,7 +292,7 @@ __global__ void __launch_bounds__(192, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int mt = blockIdx.x, nt = blockIdx.y, b = blockIdx.z;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    for (int s = 0; s < kStagesB; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
     mbar_init(done, 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -300,10 +307,10 @@ __global__ void __launch_bounds__(192, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   if (warp == 0 && lane == 0) {
-    uint32_t issued[kStages] = {0, 0, 0, 0};
+    uint32_t issued[kStagesB] = {};
     for (int kc = 0; kc < g.kchunks; ++kc) {
-      const int s = kc % kStages;
-      if (!mbar_wait(&empty[s], ((kc / kStages) & 1) ^ 1, status, 511, abort, 32)) break;
+      const int s = kc % kStagesB;
+      if (!mbar_wait(&empty[s], ((kc / kStagesB) & 1) ^ 1, status, 511, abort, 32)) break;
       ++issued[s];
       mbar_expect_tx(&full[s], C::STAGE);
       uint8_t* st = smem + s * C::STAGE;
@@ -313,15 +320,15 @@ __global__ void __launch_bounds__(192, 1)
       else tma_load_2d(st + C::A_BYTES, &tmB, &full[s], kc * 64, nt * BN);
     }
     if (*abort)
-      for (int s = 0; s < kStages; ++s)
+      for (int s = 0; s < kStagesB; ++s)
         for (uint32_t t = 0; issued[s] && t < (1u << 22) && !mbar_try(&full[s], (issued[s] - 1) & 1); ++t) {
         }
   } else if (warp == 1) {
     const bool leader = elect_one_sync();
     constexpr uint32_t idesc = idesc_bf16_f32(128, BN);
     for (int kc = 0; kc < g.kchunks; ++kc) {
-      const int s = kc % kStages;
-      if (!mbar_wait(&full[s], (kc / kStages) & 1, status, 512, abort)) break;
+      const int s = kc % kStagesB;
+      if (!mbar_wait(&full[s], (kc / kStagesB) & 1, status, 512, abort)) break;
       tc_fence_after();
       const uint32_t a = smem_u32(smem + s * C::STAGE), bb = a + C::A_BYTES;
 #pragma unroll
