@@ -410,24 +410,26 @@ struct GgnnBwdWs {
   size_t Ybf, dgib, dghb, dgiT, dghT, YTa, ETa, WihT, WhhT, tpart;  // tensor-core GEMM path
   size_t total;
 };
-size_t gru_tpart_floats(const bg_plan* p, int H) {
-  return bg::gemm_tn_part_floats(3 * H, H + 16, (int64_t)p->n_pad());
+// The GRU weight gradients of the GEMM path are reduced once over all T steps: the gate gradients
+// and the [Y^T; 1; 0], [E^T; 1; 0] operands of every step are kept side by side, [rows][T n].
+size_t gru_tpart_floats(const bg_plan* p, int H, int T) {
+  return bg::gemm_tn_part_floats(6 * H, H + 16, (int64_t)T * p->n_pad());
 }
-GgnnBwdWs ggnn_bwd_ws(const bg_plan* p, bg_dtype dt, int H) {
+GgnnBwdWs ggnn_bwd_ws(const bg_plan* p, bg_dtype dt, int H, int T) {
   GgnnBwdWs w{};
-  size_t n = (size_t)p->n_pad();
+  size_t n = (size_t)p->n_pad(), TN = (size_t)T * n;
   size_t o = 0;
   if (tc_gemm_path(dt, H)) {
     w.Ybf = o; o += al(n * H * 2);
     w.dgib = o; o += al(n * 3 * H * 2);
     w.dghb = o; o += al(n * 3 * H * 2);
-    w.dgiT = o; o += al(n * 3 * H * 2);
-    w.dghT = o; o += al(n * 3 * H * 2);
-    w.YTa = o; o += al((size_t)(H + 16) * n * 2);
-    w.ETa = o; o += al((size_t)(H + 16) * n * 2);
+    w.dgiT = o; o += al(TN * 3 * H * 2);
+    w.dghT = o; o += al(TN * 3 * H * 2);
+    w.YTa = o; o += al((size_t)(H + 16) * TN * 2);
+    w.ETa = o; o += al((size_t)(H + 16) * TN * 2);
     w.WihT = o; o += al((size_t)3 * H * H * 2);
     w.WhhT = o; o += al((size_t)3 * H * H * 2);
-    w.tpart = o; o += al(sizeof(float) * gru_tpart_floats(p, H));
+    w.tpart = o; o += al(sizeof(float) * gru_tpart_floats(p, H, T));
   }
   w.gi = o; o += al(sizeof(float) * n * 3 * H);
   w.gh = o; o += al(sizeof(float) * n * 3 * H);
@@ -531,7 +533,7 @@ extern "C" size_t bg_ggnn_workspace_bytes(const bg_plan* p, bg_dtype dt, int32_t
   if (!p || H <= 0 || T < 1) return 0;
   const bool tc = tc_shape(p, dt, H);
   if (op == BG_OP_GGNN_FWD) return std::max(ggnn_fwd_ws(p, dt, H).total, tc ? tc_fwd_ws(p, H).total : 0);
-  if (op == BG_OP_GGNN_BWD) return std::max(ggnn_bwd_ws(p, dt, H).total, tc ? tc_bwd_ws(p, H, T).total : 0);
+  if (op == BG_OP_GGNN_BWD) return std::max(ggnn_bwd_ws(p, dt, H, T).total, tc ? tc_bwd_ws(p, H, T).total : 0);
   return 0;
 }
 
@@ -898,7 +900,7 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     BG_CUDA(cudaMemcpyAsync(dE0, g, sizeof(float) * n * H, cudaMemcpyDeviceToDevice, st));
     return BG_OK;
   }
-  GgnnBwdWs w = ggnn_bwd_ws(p, dt, H);
+  GgnnBwdWs w = ggnn_bwd_ws(p, dt, H, T);
   const int bf = dt == BG_BF16;
   const int n = p->n_pad();
   const char* sv = static_cast<const char*>(saved);
@@ -920,46 +922,45 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     BG_CUDA(bg::fill_zero_f32(gr->db_hh, 3LL * H, st));
   }
   const float* gin = dET;  // gradient arriving at E(t+1)
+  const bool tcg = tc_gemm_path(dt, H);
+  const int64_t TN = (int64_t)T * n;
+  int* status = nullptr;
+  auto* Ybf = reinterpret_cast<__nv_bfloat16*>(wsc + w.Ybf);
+  auto* dgib = reinterpret_cast<__nv_bfloat16*>(wsc + w.dgib);
+  auto* dghb = reinterpret_cast<__nv_bfloat16*>(wsc + w.dghb);
+  auto* dgiT = reinterpret_cast<__nv_bfloat16*>(wsc + w.dgiT);
+  auto* dghT = reinterpret_cast<__nv_bfloat16*>(wsc + w.dghT);
+  auto* YTa = reinterpret_cast<__nv_bfloat16*>(wsc + w.YTa);
+  auto* ETa = reinterpret_cast<__nv_bfloat16*>(wsc + w.ETa);
+  auto* WihT = reinterpret_cast<__nv_bfloat16*>(wsc + w.WihT);
+  auto* WhhT = reinterpret_cast<__nv_bfloat16*>(wsc + w.WhhT);
+  if (tcg) {
+    BG_TRY(status_word_ptr(&status));
+    // B operands W^T [H][3H] of dX = dgi W_ih and g += dgh W_hh; the ones rows of [Y^T; 1; 0] and
+    // [E^T; 1; 0] over all T steps (their bias-gradient column)
+    BG_CUDA(bg::prep_transpose_bf16(prm->W_ih, 0, WihT, 3 * H, H, 1, st));
+    BG_CUDA(bg::prep_transpose_bf16(prm->W_hh, 0, WhhT, 3 * H, H, 1, st));
+    BG_CUDA(bg::fill_ones_rows(YTa, H, TN, TN, st));
+    BG_CUDA(bg::fill_ones_rows(ETa, H, TN, TN, st));
+  }
   for (int t = T - 1; t >= 0; --t) {
     const void* Et = sv + saved_E_off(p, dt, H, t);
     const float* Yt = reinterpret_cast<const float*>(sv + saved_Y_off(p, dt, H, T, t));
-    if (tc_gemm_path(dt, H)) {
+    if (tcg) {
       KTimer tm(BG_KID_GRU_BWD, st);
-      int* status = nullptr;
-      BG_TRY(status_word_ptr(&status));
-      auto* Ybf = reinterpret_cast<__nv_bfloat16*>(wsc + w.Ybf);
-      auto* dgib = reinterpret_cast<__nv_bfloat16*>(wsc + w.dgib);
-      auto* dghb = reinterpret_cast<__nv_bfloat16*>(wsc + w.dghb);
-      auto* dgiT = reinterpret_cast<__nv_bfloat16*>(wsc + w.dgiT);
-      auto* dghT = reinterpret_cast<__nv_bfloat16*>(wsc + w.dghT);
-      auto* YTa = reinterpret_cast<__nv_bfloat16*>(wsc + w.YTa);
-      auto* ETa = reinterpret_cast<__nv_bfloat16*>(wsc + w.ETa);
-      auto* WihT = reinterpret_cast<__nv_bfloat16*>(wsc + w.WihT);
-      auto* WhhT = reinterpret_cast<__nv_bfloat16*>(wsc + w.WhhT);
-      float* tpart = reinterpret_cast<float*>(wsc + w.tpart);
-      const size_t tpf = gru_tpart_floats(p, H);
       BG_TRY(gru_gates_in(p, bf, H, Yt, Et, prm, gi, gh, part, pf, st, Ybf));
       BG_CUDA(bg::gru_bwd_gates(bf, gi, gh, Et, gin, dgi, dgh, g, p->n_real, n, H, st));
       BG_CUDA(bg::f32_to_bf16(dgi, dgib, (int64_t)n * 3 * H, st));
       BG_CUDA(bg::f32_to_bf16(dgh, dghb, (int64_t)n * 3 * H, st));
-      // dX = dgi W_ih, g += dgh W_hh  (B operands W^T [H][3H])
-      BG_CUDA(bg::prep_transpose_bf16(prm->W_ih, 0, WihT, 3 * H, H, 1, st));
-      BG_CUDA(bg::prep_transpose_bf16(prm->W_hh, 0, WhhT, 3 * H, H, 1, st));
       BG_CUDA(bg::gemm_bf16_tn(dgib, 3 * H, 0, WihT, 3 * H, 0, n, H, 3 * H, 1, dX, H, 0, nullptr,
                                0, 0, status, st));
       BG_CUDA(bg::gemm_bf16_tn(dghb, 3 * H, 0, WhhT, 3 * H, 0, n, H, 3 * H, 1, g, H, 0, nullptr,
                                0, 1, status, st));
-      // dW_ih, db_ih and dW_hh, db_hh: split-K products with [Y^T; 1; 0] and [E^T; 1; 0]
-      BG_CUDA(bg::prep_transpose_bf16(dgib, 0, dgiT, n, 3 * H, 1, st));
-      BG_CUDA(bg::prep_transpose_bf16(dghb, 0, dghT, n, 3 * H, 1, st));
-      BG_CUDA(bg::prep_transpose_bf16(Yt, 1, YTa, n, H, 1, st));
-      BG_CUDA(bg::fill_ones_rows(YTa, H, n, n, st));
-      BG_CUDA(bg::prep_transpose_bf16(Et, 0, ETa, n, H, 1, st));
-      BG_CUDA(bg::fill_ones_rows(ETa, H, n, n, st));
-      BG_CUDA(bg::gemm_tn(dgiT, n, YTa, n, 3 * H, H, n, 0, gr->dW_ih, gr->db_ih, 1, tpart, tpf,
-                          status, st));
-      BG_CUDA(bg::gemm_tn(dghT, n, ETa, n, 3 * H, H, n, 0, gr->dW_hh, gr->db_hh, 1, tpart, tpf,
-                          status, st));
+      // step t's columns of the weight-gradient operands (reduced after the loop)
+      BG_CUDA(bg::prep_transpose_bf16(dgib, 0, dgiT + (size_t)t * n, n, 3 * H, 1, st, TN));
+      BG_CUDA(bg::prep_transpose_bf16(dghb, 0, dghT + (size_t)t * n, n, 3 * H, 1, st, TN));
+      BG_CUDA(bg::prep_transpose_bf16(Yt, 1, YTa + (size_t)t * n, n, H, 1, st, TN));
+      BG_CUDA(bg::prep_transpose_bf16(Et, 0, ETa + (size_t)t * n, n, H, 1, st, TN));
     } else {
       KTimer tm(BG_KID_GRU_BWD, st);
       BG_TRY(gru_gates_in(p, bf, H, Yt, Et, prm, gi, gh, part, pf, st));
@@ -996,6 +997,15 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
       BG_CUDA(cudaMemcpyAsync(dX, g, sizeof(float) * (size_t)n * H, cudaMemcpyDeviceToDevice, st));
       gin = dX;
     }
+  }
+  if (tcg) {
+    // dW_ih, db_ih += dgi^T [Y; 1] and dW_hh, db_hh += dgh^T [E; 1] over all T steps at once
+    KTimer tm(BG_KID_DW, st);
+    const bg::TNProblem probs[2] = {
+        {dgiT, TN, YTa, TN, 3 * H, 0, gr->dW_ih, gr->db_ih},
+        {dghT, TN, ETa, TN, 3 * H, 0, gr->dW_hh, gr->db_hh}};
+    BG_CUDA(bg::gemm_tn_multi(probs, 2, H, TN, 1, reinterpret_cast<float*>(wsc + w.tpart),
+                              gru_tpart_floats(p, H, T), status, st));
   }
   BG_CUDA(cudaMemcpyAsync(dE0, g, sizeof(float) * (size_t)n * H, cudaMemcpyDeviceToDevice, st));
   return BG_OK;
