@@ -523,7 +523,9 @@ extern "C" size_t bg_workspace_bytes(const bg_plan* p, bg_dtype dt, int32_t H, i
   switch (op) {
     case BG_OP_PROPAGATE_FWD: return fwd_ws(p, dt, H).total;
     case BG_OP_PROPAGATE_BWD: return bwd_ws(p, dt, H).total;
-    case BG_OP_READOUT: return al(sizeof(float) * ((size_t)p->n_packed * H + p->n_packed + 64));
+    case BG_OP_READOUT:
+      return al(sizeof(float) * ((size_t)p->n_packed * H + p->n_packed + 64)) +
+             al(sizeof(float) * (size_t)p->n_packed * bg::kPoolSplit * H);
     default: return 0;
   }
 }
@@ -1023,9 +1025,11 @@ extern "C" int bg_readout_loss(const bg_plan* p, bg_dtype dt, int32_t H, const v
   if (ws_bytes < bg_workspace_bytes(p, dt, H, BG_OP_READOUT)) return bg_fail(BG_ECAPACITY, "workspace too small");
   float* pool = static_cast<float*>(ws);
   float* resid = pool + (size_t)p->n_packed * H;
+  float* part = reinterpret_cast<float*>(static_cast<char*>(ws) +
+                                         al(sizeof(float) * ((size_t)p->n_packed * H + p->n_packed + 64)));
   BG_CUDA(bg::readout_loss(dt == BG_BF16, ET, w_out, target, p->d_seg_off, p->d_seg_cnt,
-                           p->d_row_graph, p->n_packed, p->n_pad(), H, pool, resid, loss, dET,
-                           dw_out, (cudaStream_t)stream));
+                           p->d_row_graph, p->n_packed, p->n_pad(), H, pool, resid, part, loss,
+                           dET, dw_out, (cudaStream_t)stream));
   return BG_OK;
 }
 

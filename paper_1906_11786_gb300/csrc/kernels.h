@@ -102,11 +102,13 @@ cudaError_t gru_bwd_gates(int bf16, const float* gi, const float* gh, const void
                           const float* dHn, float* dgi, float* dgh, float* dHd, int n_real,
                           int n_pad, int H, cudaStream_t st);
 
-// Mean-pool readout and squared loss.
+// Mean-pool readout and squared loss.  pool [n_seg][H], resid [n_seg] and part
+// [n_seg][kPoolSplit][H] (per-graph partial sums) are scratch; H <= 256.
+constexpr int kPoolSplit = 32;
 cudaError_t readout_loss(int bf16, const void* ET, const float* w_out, const float* target,
                          const int32_t* seg_off, const int32_t* seg_cnt, const int32_t* row_graph,
-                         int n_seg, int n_pad, int H, float* pool, float* resid, float* loss,
-                         float* dET, float* dw_out, cudaStream_t st);
+                         int n_seg, int n_pad, int H, float* pool, float* resid, float* part,
+                         float* loss, float* dET, float* dw_out, cudaStream_t st);
 
 cudaError_t adam(int64_t n, float* master, void* working, int working_bf16, float* m, float* v,
                  const float* grad, float lr, float b1, float b2, float eps, int step,

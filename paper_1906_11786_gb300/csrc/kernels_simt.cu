@@ -323,15 +323,36 @@ __global__ void k_gru_bwd(const float* gi, const float* gh, const T* E, const fl
 }
 
 // ------------------------------------------------------------------------------------ readout
+// Mean pool in two passes so that every graph's rows are read by many blocks at once (one block
+// per graph walked each graph's rows one load after another): block (g, k) sums rows
+// [off + k cnt / kPoolSplit, off + (k + 1) cnt / kPoolSplit) of graph g, 256 / H rows at a time, into
+// part[g][k][H]; k_pool_finish adds the kPoolSplit partial sums in a fixed order.
 template <typename T>
-__global__ void k_pool(const T* ET, const float* w_out, const float* target,
-                       const int32_t* seg_off, const int32_t* seg_cnt, int H, float* pool,
-                       float* resid) {
+__global__ void k_pool_part(const T* ET, const int32_t* seg_off, const int32_t* seg_cnt, int H,
+                            float* part) {
+  __shared__ float red[256];
+  const int g = blockIdx.x, k = blockIdx.y;
+  const int R = blockDim.x / H, r = threadIdx.x / H, h = threadIdx.x - r * H;
+  const int64_t off = seg_off[g], cnt = seg_cnt[g];
+  const int64_t r0 = off + k * cnt / kPoolSplit, r1 = off + (k + 1) * cnt / kPoolSplit;
+  float s = 0.f;
+  if (r < R)
+    for (int64_t i = r0 + r; i < r1; i += R) s += ld(ET, i * H + h);
+  red[threadIdx.x] = s;
+  __syncthreads();
+  if (r == 0) {
+    for (int q = 1; q < R; ++q) s += red[q * H + h];
+    part[((int64_t)g * kPoolSplit + k) * H + h] = s;
+  }
+}
+
+__global__ void k_pool_finish(const float* part, const float* w_out, const float* target,
+                              const int32_t* seg_cnt, int H, float* pool, float* resid) {
   __shared__ float red[256];
   const int g = blockIdx.x, h = threadIdx.x;
   float s = 0.f;
   if (h < H) {
-    for (int i = seg_off[g]; i < seg_off[g] + seg_cnt[g]; ++i) s += ld(ET, (int64_t)i * H + h);
+    for (int k = 0; k < kPoolSplit; ++k) s += part[((int64_t)g * kPoolSplit + k) * H + h];
     s /= (float)seg_cnt[g];
     pool[(int64_t)g * H + h] = s;
   }
@@ -359,15 +380,15 @@ __global__ void k_readout_tail(const float* pool, const float* resid, int n_seg,
   }
 }
 
+// dE(T) of the readout, one warp per row (no per-element division of the flat index).
 __global__ void k_readout_grad(const float* w_out, const float* resid, const int32_t* seg_cnt,
-                               const int32_t* row_graph, int64_t total, int H, float* dET) {
-  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total;
-       t += (int64_t)gridDim.x * blockDim.x) {
-    int64_t i = t / H;
-    int h = (int)(t % H);
-    int g = row_graph[i];
-    dET[t] = g < 0 ? 0.f : resid[g] * w_out[h] / (float)seg_cnt[g];
-  }
+                               const int32_t* row_graph, int64_t n_rows, int H, float* dET) {
+  const int64_t i = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+  if (i >= n_rows) return;
+  const int g = row_graph[i];
+  float* d = dET + i * H;
+  for (int h = threadIdx.x & 31; h < H; h += 32)
+    d[h] = g < 0 ? 0.f : resid[g] * w_out[h] / (float)seg_cnt[g];
 }
 
 // ------------------------------------------------------------------------------------ Adam
@@ -569,20 +590,24 @@ cudaError_t gru_bwd_gates(int bf16, const float* gi, const float* gh, const void
 
 cudaError_t readout_loss(int bf16, const void* ET, const float* w_out, const float* target,
                          const int32_t* seg_off, const int32_t* seg_cnt, const int32_t* row_graph,
-                         int n_seg, int n_pad, int H, float* pool, float* resid, float* loss,
-                         float* dET, float* dw_out, cudaStream_t st) {
-  if (bf16)
-    k_pool<<<n_seg, 256, 0, st>>>(static_cast<const __nv_bfloat16*>(ET), w_out, target, seg_off,
-                                  seg_cnt, H, pool, resid);
-  else
-    k_pool<<<n_seg, 256, 0, st>>>(static_cast<const float*>(ET), w_out, target, seg_off, seg_cnt,
-                                  H, pool, resid);
-  note_launch();
+                         int n_seg, int n_pad, int H, float* pool, float* resid, float* part,
+                         float* loss, float* dET, float* dw_out, cudaStream_t st) {
+  if (H < 1 || H > 256) return cudaErrorInvalidValue;
+  if (n_seg > 0) {
+    const dim3 grid(n_seg, kPoolSplit);
+    if (bf16)
+      k_pool_part<<<grid, 256, 0, st>>>(static_cast<const __nv_bfloat16*>(ET), seg_off, seg_cnt, H,
+                                        part);
+    else
+      k_pool_part<<<grid, 256, 0, st>>>(static_cast<const float*>(ET), seg_off, seg_cnt, H, part);
+    note_launch();
+    k_pool_finish<<<n_seg, 256, 0, st>>>(part, w_out, target, seg_cnt, H, pool, resid);
+    note_launch();
+  }
   k_readout_tail<<<1, 256, 0, st>>>(pool, resid, n_seg, H, loss, dw_out);
   note_launch();
-  int64_t total = (int64_t)n_pad * H;
-  k_readout_grad<<<grid_for(total, 256), 256, 0, st>>>(w_out, resid, seg_cnt, row_graph, total, H,
-                                                       dET);
+  k_readout_grad<<<(unsigned)((n_pad + 7) / 8), 256, 0, st>>>(w_out, resid, seg_cnt, row_graph,
+                                                              n_pad, H, dET);
   note_launch();
   return cudaGetLastError();
 }
