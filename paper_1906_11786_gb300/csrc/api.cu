@@ -108,17 +108,22 @@ extern "C" int bg_profile_enable(int32_t on) {
 extern "C" int bg_profile_read(int32_t kid, double* ms_total, int64_t* launches, int32_t reset) {
   if (kid < 0 || kid >= BG_KID_COUNT) return bg_fail(BG_EINVAL, "bad kernel id");
   std::lock_guard<std::mutex> g(g_prof_mu);
-  std::vector<EvPair> keep;
+  // every pending pair is read (when it can be) and destroyed exactly once, then dropped
+  bool failed = false;
   for (auto& e : g_prof_events) {
     float ms = 0.f;
-    if (cudaEventSynchronize(e.b) != cudaSuccess || cudaEventElapsedTime(&ms, e.a, e.b) != cudaSuccess)
-      return bg_fail(BG_ECUDA, "event timing failed");
-    g_prof_ms[e.kid] += ms;
-    g_prof_n[e.kid] += 1;
+    if (!failed && cudaEventSynchronize(e.b) == cudaSuccess &&
+        cudaEventElapsedTime(&ms, e.a, e.b) == cudaSuccess) {
+      g_prof_ms[e.kid] += ms;
+      g_prof_n[e.kid] += 1;
+    } else {
+      failed = true;
+    }
     cudaEventDestroy(e.a);
     cudaEventDestroy(e.b);
   }
   g_prof_events.clear();
+  if (failed) return bg_fail(BG_ECUDA, "event timing failed");
   if (ms_total) *ms_total = g_prof_ms[kid];
   if (launches) *launches = g_prof_n[kid];
   if (reset) {
