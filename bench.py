@@ -6,7 +6,7 @@ gradients); the training workload adds the mean-pool readout, loss and Adam.  Me
 per second = real (non-padding) nodes x T / step time.  Default workload: 64 program-shaped graphs
 (~72k nodes) packed at S = 128, P = 20 edge types, H = 64, bf16, T = 8.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--config 2] [--impl ours|reference]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload packed64] [--impl ours|reference]
 
 Under torchrun every rank plans its own supergraph (different seeds; the paper gives each core its
 own supergraph) and runs with no data-path collective (weak scaling); rank 0 prints one JSON line.
@@ -28,6 +28,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "node-steps/s (fwd+bwd)"
+WORKLOAD_NAMES = ("single512", "packed64", "single20k", "sweep131k", "train100k")
 
 
 def _peaks():
@@ -158,18 +159,18 @@ class Clocks:
 # --------------------------------------------------------------------------------- workload
 
 
-def workload(config: int, rank: int, S=None, H=None):
+def workload(name: str, rank: int, S=None, H=None):
     from paper_1906_11786_gb300 import synth
-    c = dict(synth.CONFIGS[config])
+    c = dict(synth.WORKLOADS[name])
     S = S or c["S"]
     H = H or c["H"]
     if rank == 0:
-        graphs = synth.config_graphs(config, S=S)
+        graphs = synth.workload_graphs(name, S=S)
     else:  # every rank gets its own supergraph of the same shape
-        graphs = synth.config_graphs(config, S=S)
+        graphs = synth.workload_graphs(name, S=S)
         graphs = [synth.gen_graph(g.n_nodes, c["F"], c["reverse"],
                                   c["max_off"] or S // 2, c["tree_win"] or S // 2, c["lam"],
-                                  synth.graph_seed(config, i) + 7919 * rank)
+                                  synth.graph_seed(name, i) + 7919 * rank)
                   for i, g in enumerate(graphs)]
     P = 2 * c["F"] if c["reverse"] else c["F"]
     cap = 0
@@ -203,7 +204,7 @@ def allreduce_grads(dist, flat):
 class OursStep:
     """Device buffers and one fwd+bwd step through the C ABI."""
 
-    def __init__(self, config, graphs, c, seed=0, dist=None):
+    def __init__(self, graphs, c, seed=0, dist=None):
         import torch
 
         from paper_1906_11786_gb300 import _binding as L
@@ -374,12 +375,12 @@ class OursStep:
 # --------------------------------------------------------------------------------- CPU oracle
 
 
-def oracle_sample(config: int, c, budget_s: float = 15.0):
+def oracle_sample(name: str, c, budget_s: float = 15.0):
     """The oracle as it stands (single-threaded fp64) on a bounded sample of the workload: the
     leading graphs of the batch, as many as fit the time budget; returns node-steps/s."""
     import oracle
     from paper_1906_11786_gb300 import synth
-    graphs = synth.config_graphs(config, S=c["S"])
+    graphs = synth.workload_graphs(name, S=c["S"])
     P, S, H, T = c["P"], c["S"], c["H"], c["T"]
     done_nodes, spent, used = 0, 0.0, 0
     rng = np.random.default_rng(0)
@@ -413,13 +414,13 @@ def run_reference(args):
     if rank != 0:
         return 0
     from paper_1906_11786_gb300 import synth
-    graphs, c = workload(args.config, 0, args.S, args.H)
+    graphs, c = workload(args.workload, 0, args.S, args.H)
     n_real = sum(g.n_nodes for g in graphs)
     times = []
     # keep the whole run within a few minutes whatever K and W are
     budget = max(0.5, min(args.ref_budget, 150.0 / max(1, args.warmup + args.steps)))
     for i in range(args.warmup + args.steps):
-        v, s = oracle_sample(args.config, c, budget_s=budget)
+        v, s = oracle_sample(args.workload, c, budget_s=budget)
         if i >= args.warmup:
             times.append(v)
     value = statistics.median(times)
@@ -428,7 +429,7 @@ def run_reference(args):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": n_real * c["T"] / value * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": synth.CONFIGS[args.config]["name"], "S": c["S"], "H": c["H"],
+        "config": {"workload": args.workload, "S": c["S"], "H": c["H"],
                    "P": c["P"], "T": c["T"]},
         "cpu_baseline": {"value": value, "unit": "node-steps/s", "cores": 1, "kind": "oracle",
                          "sample": f"leading graphs of the batch per step, ~{budget:.1f}s "
@@ -482,7 +483,14 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--config", type=int, default=2)
+    ap.add_argument("--workload", default="packed64", choices=list(WORKLOAD_NAMES),
+                    help="single512: one 512-node graph, S 64, fp32, one propagation; packed64: 64 "
+                         "graphs of 200-2000 nodes, S 128, H 64, T 8; single20k: one 20,000-node "
+                         "graph, S 256, H 128, T 8; sweep131k: 131,072 packed positions, one "
+                         "propagation (set --S); train100k: ~100k nodes, T 8 with readout, loss "
+                         "and Adam (set --H)")
+    # the position of the workload in the list above, as earlier command lines name it
+    ap.add_argument("--config", type=int, default=None, help=argparse.SUPPRESS)
     ap.add_argument("--S", type=int, default=None)
     ap.add_argument("--H", type=int, default=None)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
@@ -492,6 +500,8 @@ def main():
                     help="time one band propagation kernel call instead of the whole step "
                          "(focused profiling of the same workload)")
     args = ap.parse_args()
+    if args.config is not None:
+        args.workload = WORKLOAD_NAMES[args.config - 1]
     if args.impl == "reference":
         return run_reference(args)
 
@@ -505,10 +515,9 @@ def main():
     import __graft_entry__
     __graft_entry__.build()
     from paper_1906_11786_gb300 import _binding as L
-    from paper_1906_11786_gb300 import synth
 
-    graphs, c = workload(args.config, rank, args.S, args.H)
-    st = OursStep(args.config, graphs, c, seed=rank, dist=dist)
+    graphs, c = workload(args.workload, rank, args.S, args.H)
+    st = OursStep(graphs, c, seed=rank, dist=dist)
     H, T = c["H"], c["T"]
     units = st.n_real * T  # node-steps per step on this rank
     if args.op != "step":
@@ -577,7 +586,7 @@ def main():
     avg_ms = (fwd_ms / max(fwd_n, 1)) if kern == "band_fwd" else (bwd_ms / max(bwd_n, 1))
     achieved = flops / (avg_ms / 1e3) / 1e12 if avg_ms > 0 else 0.0
     peak = pk["bf16_sustained"]
-    traffic = _profiled_traffic(kern.split("_")[1], synth.CONFIGS[args.config]["name"])
+    traffic = _profiled_traffic(kern.split("_")[1], args.workload)
     roof = {"kernel": kern, "bound": "tensor", "achieved": achieved, "peak": peak,
             "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
             "traffic_src": "profiles/ ncu capture (dram read+write bytes per launch)"
@@ -595,7 +604,7 @@ def main():
         "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms_step,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": c["dtype"], "data": "synthetic program-shaped graphs (seeded)",
-        "config": {"workload": synth.CONFIGS[args.config]["name"], "graphs": len(graphs),
+        "config": {"workload": args.workload, "graphs": len(graphs),
                    "packed": st.info["n_packed"], "n_real": st.n_real, "n_pad": st.N,
                    "K": st.info["K"], "S": c["S"], "P": c["P"], "H": H, "T": T,
                    "kept_edges": st.info["n_kept"], "dropped_edges": st.info["n_dropped"],
@@ -613,7 +622,7 @@ def main():
         "clocks": clk.summary(),
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, s = oracle_sample(args.config, c)
+        v, s = oracle_sample(args.workload, c)
         line["cpu_baseline"] = {"value": v, "unit": "node-steps/s", "cores": 1, "kind": "oracle",
                                 "sample": f"leading {s['graphs']} graphs ({s['nodes']} nodes) of "
                                           f"the same workload, fwd+bwd, {s['seconds']:.1f}s "

@@ -17,7 +17,7 @@ from dataclasses import dataclass, field
 import numpy as np
 
 __all__ = [
-    "Graph", "gen_graph", "gen_batch", "gen_states", "gen_params", "CONFIGS", "config_graphs",
+    "Graph", "gen_graph", "gen_batch", "gen_states", "gen_params", "WORKLOADS", "workload_graphs",
     "graph_seed",
 ]
 
@@ -38,9 +38,9 @@ class Graph:
         return int(self.src.shape[0])
 
 
-def graph_seed(config: int, graph_index: int) -> int:
-    """Seed of graph `graph_index` in workload `config`."""
-    return 1906 + 1000 * config + 17 * graph_index
+def graph_seed(workload: str, graph_index: int) -> int:
+    """Seed of graph `graph_index` of the named workload."""
+    return WORKLOADS[workload]["seed"] + 17 * graph_index
 
 
 def gen_graph(n: int, n_families: int, reverse: bool, max_off: int, tree_win: int, lam: float,
@@ -107,26 +107,30 @@ def gen_graph(n: int, n_families: int, reverse: bool, max_off: int, tree_win: in
 
 
 # Workloads: sizes follow the paper's program graphs (Section 4: up to ~20k nodes per graph,
-# P = 22 edge types; Appendix A.1: 70,272-node supergraphs at S = 128) with P = 20.
-CONFIGS = {
-    1: dict(name="single512", sizes=("fixed", [512]), F=4, reverse=False, max_off=48, tree_win=32,
-            lam=1.0, S=64, H=64, T=1, dtype="f32", gru=False),
-    2: dict(name="packed64", sizes=("uniform", 64, 200, 2000), F=10, reverse=True, max_off=96,
-            tree_win=64, lam=3.0, S=128, H=64, T=8, dtype="bf16", gru=True),
-    3: dict(name="single20k", sizes=("fixed", [20000]), F=10, reverse=True, max_off=200,
-            tree_win=133, lam=3.0, S=256, H=128, T=8, dtype="bf16", gru=True),
-    4: dict(name="sweep131k", sizes=("fill", 131072, 200, 2000), F=10, reverse=True, max_off=None,
-            tree_win=None, lam=3.0, S=128, H=64, T=1, dtype="bf16", gru=False),
-    5: dict(name="train100k", sizes=("fill", 100000, 200, 5000), F=10, reverse=True, max_off=96,
-            tree_win=64, lam=3.0, S=128, H=64, T=8, dtype="bf16", gru=True, train=True),
+# P = 22 edge types; Appendix A.1: 70,272-node supergraphs at S = 128) with P = 20.  `seed` is the
+# base of the workload's random streams (graph sizes, and graph g from seed + 17 g).
+WORKLOADS = {
+    "single512": dict(seed=2906, sizes=("fixed", [512]), F=4, reverse=False, max_off=48,
+                      tree_win=32, lam=1.0, S=64, H=64, T=1, dtype="f32", gru=False),
+    "packed64": dict(seed=3906, sizes=("uniform", 64, 200, 2000), F=10, reverse=True, max_off=96,
+                     tree_win=64, lam=3.0, S=128, H=64, T=8, dtype="bf16", gru=True),
+    "single20k": dict(seed=4906, sizes=("fixed", [20000]), F=10, reverse=True, max_off=200,
+                      tree_win=133, lam=3.0, S=256, H=128, T=8, dtype="bf16", gru=True),
+    "sweep131k": dict(seed=5906, sizes=("fill", 131072, 200, 2000), F=10, reverse=True,
+                      max_off=None, tree_win=None, lam=3.0, S=128, H=64, T=1, dtype="bf16",
+                      gru=False),
+    "train100k": dict(seed=6906, sizes=("fill", 100000, 200, 5000), F=10, reverse=True, max_off=96,
+                      tree_win=64, lam=3.0, S=128, H=64, T=8, dtype="bf16", gru=True, train=True),
 }
+for _name, _w in WORKLOADS.items():
+    _w["name"] = _name
 
 
-def _sizes(config: int, spec) -> list[int]:
+def _sizes(workload: str, spec) -> list[int]:
     kind = spec[0]
     if kind == "fixed":
         return list(spec[1])
-    rng = np.random.default_rng(1906 + 1000 * config)
+    rng = np.random.default_rng(WORKLOADS[workload]["seed"])
     if kind == "uniform":
         _, count, lo, hi = spec
         return [int(x) for x in rng.integers(lo, hi + 1, size=count)]
@@ -142,17 +146,18 @@ def _sizes(config: int, spec) -> list[int]:
     raise ValueError(kind)
 
 
-def config_graphs(config: int, S: int | None = None, scale: float = 1.0, **over) -> list[Graph]:
-    """Graphs of a workload.  `S` overrides the block size (the sweep sets max_off = tree_win = S/2);
-    `scale` < 1 keeps only a leading fraction of the graph list (small parity cases)."""
-    c = dict(CONFIGS[config]); c.update(over)
+def workload_graphs(workload: str, S: int | None = None, scale: float = 1.0, **over) -> list[Graph]:
+    """Graphs of the named workload.  `S` overrides the block size (the sweep sets max_off =
+    tree_win = S/2); `scale` < 1 keeps only a leading fraction of the graph list (small parity
+    cases)."""
+    c = dict(WORKLOADS[workload]); c.update(over)
     S = S or c["S"]
     max_off = c["max_off"] if c["max_off"] is not None else max(1, S // 2)
     tree_win = c["tree_win"] if c["tree_win"] is not None else max(1, S // 2)
-    sizes = _sizes(config, c["sizes"])
+    sizes = _sizes(workload, c["sizes"])
     if scale < 1.0:
         sizes = sizes[:max(1, int(round(len(sizes) * scale)))]
-    return [gen_graph(n, c["F"], c["reverse"], max_off, tree_win, c["lam"], graph_seed(config, g))
+    return [gen_graph(n, c["F"], c["reverse"], max_off, tree_win, c["lam"], graph_seed(workload, g))
             for g, n in enumerate(sizes)]
 
 

@@ -72,7 +72,7 @@ def _bwd(c: Case, seed=7):
 
 
 def test_pack_unpack_bit_exact():
-    c = Case(synth.config_graphs(2, scale=0.1), 20, 128, 64, "bf16", seed=3)
+    c = Case(synth.workload_graphs("packed64", scale=0.1), 20, 128, 64, "bf16", seed=3)
     got = c.E_band_dev.float().cpu().numpy()
     np.testing.assert_array_equal(got, c.E_band)
     back = torch.zeros_like(c.E_orig_dev)
@@ -83,9 +83,9 @@ def test_pack_unpack_bit_exact():
 # ------------------------------------------------------------------------------------ propagate
 
 
-def test_propagate_fp32_config1():
+def test_propagate_fp32_single512():
     """Single 512-node graph, 4 types, S = 64, H = 64, fp32, fwd + bwd."""
-    c = Case(synth.config_graphs(1), 4, 64, 64, "f32", seed=11)
+    c = Case(synth.workload_graphs("single512"), 4, 64, 64, "f32", seed=11)
     Y, ref = _fwd(c)
     assert rel_err(Y, ref) < TOL["f32"]
     got, ref = _bwd(c)
@@ -128,7 +128,7 @@ def test_propagate_graph_without_edges():
     assert np.all(Y == 0) and np.all(ref == 0)
 
 
-def test_propagate_bf16_dropped_edges_config3_shape():
+def test_propagate_bf16_dropped_edges_single20k_shape():
     """Wide band: S = 256 < bandwidth, so some edges are dropped (coverage rule)."""
     g = synth.gen_graph(3000, 10, True, 200, 133, 3.0, 17)
     c = Case([g], 20, 256, 128, "bf16", seed=5)
@@ -186,9 +186,9 @@ def test_ggnn_fwd_bwd(dtype, T, S, H, whole):
         assert rel_err(v, ref[k]) < tol, k
 
 
-def test_ggnn_config2_shape_T8_reduced_batch():
-    """Config-2 shapes (P = 20, S = 128, H = 64, bf16, T = 8) on an 8-graph batch."""
-    c = Case(synth.config_graphs(2, scale=0.125), 20, 128, 64, "bf16", seed=2)
+def test_ggnn_packed64_shape_T8_reduced_batch():
+    """The packed64 workload's shapes (P = 20, S = 128, H = 64, bf16, T = 8) on an 8-graph batch."""
+    c = Case(synth.workload_graphs("packed64", scale=0.125), 20, 128, 64, "bf16", seed=2)
     ET, ref_ET, grads, dE0, ref = _ggnn(c, 8)
     assert rel_err(ET, ref_ET) < TOL["bf16"]
     assert rel_err(dE0, ref["dE0"]) < TOL["bf16"]
@@ -281,17 +281,17 @@ def _full_size_propagation(c: Case, seed: int, n_rows: int = 400, types=(0, 7, 1
     assert rel_err(db[types], ref_db) < TOL["bf16"], "db"
 
 
-def test_full_size_config2_propagate_sampled_rows():
-    """Config 2 at full size (64 graphs, ~72k nodes, 566 tiles, P = 20, S = 128, H = 64, bf16):
+def test_full_size_packed64_propagate_sampled_rows():
+    """The packed64 workload at full size (64 graphs, ~72k nodes, 566 tiles, P = 20, S = 128, H = 64, bf16):
     one forward and backward propagation, every tile whole."""
-    _full_size_propagation(Case(synth.config_graphs(2), 20, 128, 64, "bf16", seed=21), 41)
+    _full_size_propagation(Case(synth.workload_graphs("packed64"), 20, 128, 64, "bf16", seed=21), 41)
 
 
-def test_full_size_config3_propagate_sampled_rows():
-    """Config 3 at full size (one 20,000-node graph, S = 256, H = 128, 158 tiles): on a GPU with a
+def test_full_size_single20k_propagate_sampled_rows():
+    """The single20k workload at full size (one 20,000-node graph, S = 256, H = 128, 158 tiles): on a GPU with a
     few SMs fewer than tiles, a whole round of tiles runs as whole tiles and the few tiles left are
     split over several CTAs (partial sums and the fix-up kernel), the schedule the benchmark runs."""
-    c = Case(synth.config_graphs(3), 20, 256, 128, "bf16", seed=43)
+    c = Case(synth.workload_graphs("single20k"), 20, 256, 128, "bf16", seed=43)
     sms = torch.cuda.get_device_properties(0).multi_processor_count
     tiles = c.N // 128
     assert tiles > sms and tiles % sms < sms // 2
@@ -299,11 +299,11 @@ def test_full_size_config3_propagate_sampled_rows():
 
 
 @pytest.mark.parametrize("S", [32, 256, 512])
-def test_full_size_config4_propagate_sampled_rows(S):
+def test_full_size_sweep131k_propagate_sampled_rows(S):
     """The block-size sweep at full size (131,072 positions, P = 20, H = 64, max offset S / 2):
     S = 32 (four block-rows per tile), S = 256 (six window chunks) and S = 512 (32-column state
     slices over a twelve-chunk window), with the sweep's capacity of 131,072 / S blocks."""
-    c = Case(synth.config_graphs(4, S=S), 20, S, 64, "bf16", seed=50 + S, cap=-(-131072 // S))
+    c = Case(synth.workload_graphs("sweep131k", S=S), 20, S, 64, "bf16", seed=50 + S, cap=-(-131072 // S))
     assert c.N == 131072
     _full_size_propagation(c, 53 + S)
 
@@ -362,26 +362,26 @@ def _full_size_ggnn_sampled_graphs(c: Case, T: int, pick, seed: int):
     return ET
 
 
-def test_full_size_config2_ggnn_T8_fwd_bwd_sampled_graphs():
-    """The benchmark workload end to end: config 2 at full size (64 graphs, ~72k nodes, P = 20,
+def test_full_size_packed64_ggnn_T8_fwd_bwd_sampled_graphs():
+    """The benchmark workload end to end: packed64 at full size (64 graphs, ~72k nodes, P = 20,
     S = 128, H = 64, bf16, T = 8) through the fused tensor-core path, forward + backward."""
-    c = Case(synth.config_graphs(2), 20, 128, 64, "bf16", seed=23)
+    c = Case(synth.workload_graphs("packed64"), 20, 128, 64, "bf16", seed=23)
     off, _ = c.ref.graph_segments()
     _full_size_ggnn_sampled_graphs(c, 8, np.random.default_rng(5).choice(len(off), 4, replace=False),
                                    31)
 
 
 @pytest.mark.parametrize("H", [32, 128, 256])
-def test_full_size_config5_ggnn_T8_fwd_bwd_sampled_graphs(H):
-    """Config 5's batch at full size with the benchmark's capacity (100,000 positions rounded up to
+def test_full_size_train100k_ggnn_T8_fwd_bwd_sampled_graphs(H):
+    """The train100k batch at full size with the benchmark's capacity (100,000 positions rounded up to
     whole blocks: 782 tiles, P = 20, S = 128, bf16, T = 8), forward + backward against the oracle on
     a few of the smaller graphs: H = 32 (32-column band products, resident-weight GRU kernels),
     H = 128 (64-column state passes, GRU weights streamed), H = 256 (four state passes, the GRU on
-    tensor-core GEMMs); H = 64 runs at full size as config 2.  On a 152-SM GB300 the band kernels
+    tensor-core GEMMs); H = 64 runs at full size as packed64.  On a 152-SM GB300 the band kernels
     run five whole rounds of tiles and split the 22-tile tail four ways.  The training step's mean-pool readout and loss are checked over the whole batch on the E(T) the
     launch produced."""
-    cap = -(-synth.CONFIGS[5]["sizes"][1] // 128)
-    c = Case(synth.config_graphs(5), 20, 128, H, "bf16", seed=29, cap=cap)
+    cap = -(-synth.WORKLOADS["train100k"]["sizes"][1] // 128)
+    c = Case(synth.workload_graphs("train100k"), 20, 128, H, "bf16", seed=29, cap=cap)
     assert c.N == cap * 128
     off, cnt = c.ref.graph_segments()
     if H <= 128:

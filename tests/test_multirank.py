@@ -26,7 +26,7 @@ def _worker(rank, world, port, out):
     from paper_1906_11786_gb300 import _binding as L
     dist.init_process_group("gloo", rank=rank, world_size=world)
     try:
-        graphs, c = bench.workload(2, rank)
+        graphs, c = bench.workload("packed64", rank)
         # same workload shape on every rank, different graphs
         sig = torch.tensor([len(graphs), sum(g.n_nodes for g in graphs), c["S"], c["P"], c["H"]],
                            dtype=torch.float64)

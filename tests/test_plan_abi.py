@@ -60,29 +60,29 @@ def _compare(graphs, P, S, cap=0, flags=L.BG_RCM | L.BG_KEEP_IF_BETTER):
     return plan, ref
 
 
-def test_planner_bit_exact_config1():
-    _compare(synth.config_graphs(1), 4, 64)
+def test_planner_bit_exact_single512():
+    _compare(synth.workload_graphs("single512"), 4, 64)
 
 
-def test_planner_bit_exact_packed_batch_config2():
-    _compare(synth.config_graphs(2), 20, 128)
+def test_planner_bit_exact_packed64():
+    _compare(synth.workload_graphs("packed64"), 20, 128)
 
 
-def test_planner_bit_exact_single_large_config3():
-    _compare(synth.config_graphs(3), 20, 256)
+def test_planner_bit_exact_single20k():
+    _compare(synth.workload_graphs("single20k"), 20, 256)
 
 
 @pytest.mark.parametrize("S", [32, 64, 128, 256, 512])
-def test_planner_bit_exact_sweep_config4_capacity(S):
-    gs = synth.config_graphs(4, S=S, scale=0.25)
+def test_planner_bit_exact_sweep131k_capacity(S):
+    gs = synth.workload_graphs("sweep131k", S=S, scale=0.25)
     cap = max(1, (sum(g.n_nodes for g in gs) - 300) // S)  # the last graphs do not fit
     plan, ref = _compare(gs, 20, S, cap)
     assert ref.n_packed < len(gs)
 
 
-def test_planner_bit_exact_training_batch_config5():
-    """Config 5's graphs (200 .. 5000 nodes, the largest RCM inputs of any config), full batch."""
-    _compare(synth.config_graphs(5), 20, 128)
+def test_planner_bit_exact_train100k():
+    """The train100k graphs (200 .. 5000 nodes, the largest RCM inputs of any workload), full batch."""
+    _compare(synth.workload_graphs("train100k"), 20, 128)
 
 
 def test_planner_without_rcm_and_without_keep():
@@ -103,7 +103,7 @@ def test_planner_tiny_golden_rcm():
 
 
 def test_flop_counts():
-    plan = L.band_plan(synth.config_graphs(1), 4, 64)
+    plan = L.band_plan(synth.workload_graphs("single512"), 4, 64)
     i = plan.info()
     K, S, P, H = i["K"], 64, 4, 64
     assert plan.flops(H, L.BG_FLOPS_BAND) == 2 * (3 * K - 2) * P * S * S * H
@@ -133,7 +133,7 @@ def test_invalid_inputs_return_einval_or_ecapacity(bad):
 
 def test_device_calls_require_upload():
     import torch
-    plan = L.band_plan(synth.config_graphs(1), 4, 64)
+    plan = L.band_plan(synth.workload_graphs("single512"), 4, 64)
     x = torch.zeros(16)
     # a plan that was never uploaded is rejected before any CUDA call
     rc = L.load().bg_band_propagate_fwd(plan.handle, 0, 64, x.data_ptr(), x.data_ptr(), None,
@@ -142,7 +142,7 @@ def test_device_calls_require_upload():
 
 
 def test_workspace_and_saved_sizes_are_positive():
-    plan = L.band_plan(synth.config_graphs(1), 4, 64)
+    plan = L.band_plan(synth.workload_graphs("single512"), 4, 64)
     for op in (L.BG_OP_PROPAGATE_FWD, L.BG_OP_PROPAGATE_BWD, L.BG_OP_READOUT):
         assert L.workspace_bytes(plan, "f32", 64, op) > 0
     for op in (L.BG_OP_GGNN_FWD, L.BG_OP_GGNN_BWD):
