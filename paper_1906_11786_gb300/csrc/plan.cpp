@@ -224,52 +224,78 @@ int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S
   worker();
   for (auto& t : pool) t.join();
 
-  // gather table, segments, and the deduplicated edge keys in supergraph positions
+  // gather table and segments
   pl->gather.resize(pl->n_real);
-  std::vector<uint64_t> keys;
   for (int32_t g = 0; g < pl->n_packed; ++g) {
     const bg_graph& gr = graphs[g];
     const int32_t* pg = pl->perm.data() + pl->node_base[g];
-    int32_t o = pl->offset[g];
-    std::vector<int32_t> where(gr.n_nodes);
-    for (int32_t i = 0; i < gr.n_nodes; ++i) {
-      where[pg[i]] = i;
-      pl->gather[o + i] = (int32_t)(pl->node_base[g] + pg[i]);
-    }
+    const int32_t o = pl->offset[g];
+    for (int32_t i = 0; i < gr.n_nodes; ++i) pl->gather[o + i] = (int32_t)(pl->node_base[g] + pg[i]);
     pl->seg_off.push_back(o);
     pl->seg_cnt.push_back(gr.n_nodes);
     pl->bw_before_max = std::max(pl->bw_before_max, pl->bw_before[g]);
     pl->bw_after_max = std::max(pl->bw_after_max, pl->bw_after[g]);
     pl->n_edges_in += gr.n_edges;
-    for (int64_t e = 0; e < gr.n_edges; ++e) {
-      uint64_t tgt = (uint64_t)(o + where[gr.dst[e]]);
-      uint64_t srcp = (uint64_t)(o + where[gr.src[e]]);
-      // target (28 bits) | source (28 bits) | type (6 bits) -> unique key, sorted by target
-      keys.push_back((tgt << 34) | (srcp << 6) | (uint64_t)gr.etype[e]);
-    }
   }
-  std::sort(keys.begin(), keys.end());
-  keys.erase(std::unique(keys.begin(), keys.end()), keys.end());
-  pl->n_unique = (int64_t)keys.size();
 
+  // Deduplicated edges in supergraph positions and their bits, graph by graph on the host
+  // threads.  Packed graphs share no node, so each graph's sorted unique keys are a contiguous
+  // run of the global sorted order, and every mask word a graph sets (forward: a row of one of its
+  // targets; transposed: a row of one of its sources) belongs to that graph alone.
   const size_t tile_words = (size_t)S * pl->W32;
   const size_t nwords = (size_t)pl->K * 3 * P * tile_words;
   pl->masks.assign(nwords, 0u);
   pl->masksT.assign(nwords, 0u);
-  for (uint64_t key : keys) {
-    int64_t i = (int64_t)(key >> 34);
-    int64_t j = (int64_t)((key >> 6) & ((1ull << 28) - 1));
-    int32_t p = (int32_t)(key & 63);
-    int64_t bi = i / S, bj = j / S;
-    if (bj - bi < -1 || bj - bi > 1) { ++pl->n_dropped; continue; }
-    ++pl->n_kept;
-    int64_t ri = i % S, cj = j % S;
-    // forward: block-row bi, diagonal slot (bj - bi + 1), row ri, bit cj
-    size_t f = ((((size_t)bi * 3 + (size_t)(bj - bi + 1)) * P + p) * S + ri) * pl->W32 + cj / 32;
-    pl->masks[f] |= 1u << (cj % 32);
-    // transposed: source block bj, target slot (bi - bj + 1), row cj, bit ri
-    size_t t = ((((size_t)bj * 3 + (size_t)(bi - bj + 1)) * P + p) * S + cj) * pl->W32 + ri / 32;
-    pl->masksT[t] |= 1u << (ri % 32);
+  std::vector<int64_t> uniq(pl->n_packed, 0), kept(pl->n_packed, 0), dropped(pl->n_packed, 0);
+  std::atomic<int32_t> next_g{0};
+  auto edge_worker = [&]() {
+    std::vector<uint64_t> keys;
+    std::vector<int32_t> where;
+    for (;;) {
+      const int32_t g = next_g.fetch_add(1);
+      if (g >= pl->n_packed) return;
+      const bg_graph& gr = graphs[g];
+      const int32_t* pg = pl->perm.data() + pl->node_base[g];
+      const int32_t o = pl->offset[g];
+      where.resize(gr.n_nodes);
+      for (int32_t i = 0; i < gr.n_nodes; ++i) where[pg[i]] = i;
+      keys.clear();
+      for (int64_t e = 0; e < gr.n_edges; ++e) {
+        const uint64_t tgt = (uint64_t)(o + where[gr.dst[e]]);
+        const uint64_t srcp = (uint64_t)(o + where[gr.src[e]]);
+        // target (28 bits) | source (28 bits) | type (6 bits) -> unique key, sorted by target
+        keys.push_back((tgt << 34) | (srcp << 6) | (uint64_t)gr.etype[e]);
+      }
+      std::sort(keys.begin(), keys.end());
+      keys.erase(std::unique(keys.begin(), keys.end()), keys.end());
+      uniq[g] = (int64_t)keys.size();
+      for (uint64_t key : keys) {
+        const int64_t i = (int64_t)(key >> 34);
+        const int64_t j = (int64_t)((key >> 6) & ((1ull << 28) - 1));
+        const int32_t p = (int32_t)(key & 63);
+        const int64_t bi = i / S, bj = j / S;
+        if (bj - bi < -1 || bj - bi > 1) { ++dropped[g]; continue; }
+        ++kept[g];
+        const int64_t ri = i % S, cj = j % S;
+        // forward: block-row bi, diagonal slot (bj - bi + 1), row ri, bit cj
+        const size_t f = ((((size_t)bi * 3 + (size_t)(bj - bi + 1)) * P + p) * S + ri) * pl->W32 + cj / 32;
+        pl->masks[f] |= 1u << (cj % 32);
+        // transposed: source block bj, target slot (bi - bj + 1), row cj, bit ri
+        const size_t t = ((((size_t)bj * 3 + (size_t)(bi - bj + 1)) * P + p) * S + cj) * pl->W32 + ri / 32;
+        pl->masksT[t] |= 1u << (ri % 32);
+      }
+    }
+  };
+  unsigned ne = std::max(1u, std::min(std::thread::hardware_concurrency(), 16u));
+  ne = std::min<unsigned>(ne, (unsigned)pl->n_packed);
+  std::vector<std::thread> epool;
+  for (unsigned t = 1; t < ne; ++t) epool.emplace_back(edge_worker);
+  edge_worker();
+  for (auto& t : epool) t.join();
+  for (int32_t g = 0; g < pl->n_packed; ++g) {
+    pl->n_unique += uniq[g];
+    pl->n_kept += kept[g];
+    pl->n_dropped += dropped[g];
   }
   *out = pl;
   return BG_OK;
