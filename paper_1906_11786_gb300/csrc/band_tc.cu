@@ -1062,56 +1062,11 @@ cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, c
 int band_tc_upload(bg_plan* p, cudaStream_t st) {
   const int S = p->S;
   if (p->P > 32 || (S != 32 && S != 64 && S != 128 && S != 256 && S != 512)) return 0;
-  const int K = p->K, P = p->P, W32 = p->W32;
-  const size_t n = (size_t)K * S;
+  const size_t n = (size_t)p->K * S;
   if (n % kTile) return 0;
-  const int n_tiles = (int)(n / kTile), C1 = band_chunks(S);
-  // interleave bits of every word: column 2j -> bit j, column 2j+1 -> bit 16+j
-  auto inter = [](uint32_t w) {
-    uint32_t o = 0;
-    for (int j = 0; j < 16; ++j) {
-      o |= ((w >> (2 * j)) & 1u) << j;
-      o |= ((w >> (2 * j + 1)) & 1u) << (16 + j);
-    }
-    return o;
-  };
-  // per (tile, type): the C1 128-column chunks of the tile's window [ws, ws + 128 C1), 4 words per
-  // row per chunk; words outside the three block diagonals of the row's block-row are zero
-  std::vector<uint32_t> mi((size_t)n_tiles * P * C1 * kTile * 4), mti(mi.size());
-  std::vector<uint16_t> deg(n * 64, 0);
-  int max_deg = 0;
-  for (int t = 0; t < n_tiles; ++t) {
-    const int64_t row0 = (int64_t)t * kTile, ws = (row0 / S) * S - S;
-    for (int q = 0; q < P; ++q)
-      for (int j = 0; j < C1; ++j)
-        for (int r = 0; r < kTile; ++r)
-          for (int w = 0; w < 4; ++w) {
-            const int64_t R = row0 + r, Cc = ws + j * kTile + 32 * w;
-            const size_t dst = ((((size_t)t * P + q) * C1 + j) * kTile + r) * 4 + w;
-            if (Cc < 0 || Cc >= (int64_t)n) continue;
-            const int64_t kr = R / S, kc = Cc / S, d = kc - kr + 1;
-            if (d < 0 || d > 2) continue;
-            const size_t src = ((((size_t)kr * 3 + d) * P + q) * S + R % S) * W32 + (Cc % S) / 32;
-            mi[dst] = inter(p->masks[src]);
-            mti[dst] = inter(p->masksT[src]);
-          }
-  }
-  for (int k = 0; k < K; ++k)
-    for (int q = 0; q < P; ++q)
-      for (int r = 0; r < S; ++r) {
-        int cnt = 0;
-        for (int d = 0; d < 3; ++d)
-          for (int w = 0; w < W32; ++w)
-            cnt += __builtin_popcount(p->masks[((((size_t)k * 3 + d) * P + q) * S + r) * W32 + w]);
-        max_deg = std::max(max_deg, cnt);
-        // bf16 bit pattern of a small integer (exact up to 256)
-        float f = (float)cnt;
-        uint32_t u;
-        std::memcpy(&u, &f, 4);
-        const uint16_t bfv = (uint16_t)(u >> 16);
-        deg[((size_t)k * S + r) * 64 + q] = bfv;
-        deg[((size_t)k * S + r) * 64 + 32 + q] = bfv;
-      }
+  std::vector<uint32_t> mi, mti;
+  std::vector<uint16_t> deg;
+  const int max_deg = band_tc_host_tiles(p, band_chunks(S), mi, mti, deg);
   p->max_deg = max_deg;
   if (cudaMalloc(&p->d_maskI, mi.size() * 4) != cudaSuccess ||
       cudaMalloc(&p->d_maskTI, mti.size() * 4) != cudaSuccess ||

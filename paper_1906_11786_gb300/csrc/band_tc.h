@@ -47,6 +47,11 @@ cudaError_t prep_transpose_bf16(const void* in, int in_is_f32, __nv_bfloat16* ou
 cudaError_t prep_bias_split(const float* b, __nv_bfloat16* b2T, int P, int H, cudaStream_t st);
 // Builds and uploads the tensor-core path's plan data (no-op where unsupported); 0 on success.
 int band_tc_upload(bg_plan* p, cudaStream_t st);
+// Host side of band_tc_upload (band_tiles.cpp): the bit-interleaved window chunks of every
+// 128-row tile, [n_pad / 128][P][C1][128][4] words for C1 128-column chunks per tile, in both
+// orientations, and the per-row in-degrees [n_pad][64] as bf16; returns the largest in-degree.
+int band_tc_host_tiles(const bg_plan* p, int C1, std::vector<uint32_t>& mi,
+                       std::vector<uint32_t>& mti, std::vector<uint16_t>& deg);
 // Frees device data the tensor-core path keeps with the plan.
 void band_tc_release(bg_plan* p);
 
