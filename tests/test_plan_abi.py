@@ -148,3 +148,97 @@ def test_workspace_and_saved_sizes_are_positive():
     for op in (L.BG_OP_GGNN_FWD, L.BG_OP_GGNN_BWD):
         assert L.ggnn_workspace_bytes(plan, "f32", 64, 8, op) > 0
     assert L.ggnn_saved_bytes(plan, "bf16", 64, 8) >= 9 * 512 * 64 * 2 + 8 * 512 * 64 * 4
+
+
+def _probe_binary(tmp_path_factory):
+    """Compiles tests/tiles_probe.cpp against the in-tree library (g++, host code only)."""
+    import os
+    import shutil
+    import subprocess
+    gxx = shutil.which("g++")
+    if gxx is None:
+        pytest.skip("g++ not available")
+    here = os.path.dirname(os.path.abspath(__file__))
+    root = os.path.dirname(here)
+    pkg = os.path.dirname(L.LIB_PATH)
+    exe = str(tmp_path_factory.mktemp("probe") / "tiles_probe")
+    subprocess.run([gxx, "-O1", "-std=c++17", "-I", os.path.join(root, "include"), "-I",
+                    os.path.join(pkg, "csrc"), os.path.join(here, "tiles_probe.cpp"), "-L", pkg,
+                    "-lbandggnn", f"-Wl,-rpath,{pkg}", "-lpthread", "-o", exe], check=True)
+    return exe
+
+
+def _interleave(w):
+    """Column 2j of a 32-column word to bit j, column 2j+1 to bit 16+j (the bf16-pair expansion
+    order of the tensor-core kernels' A operand)."""
+    w = w.astype(np.uint64)
+    out = np.zeros_like(w)
+    for j in range(16):
+        out |= ((w >> np.uint64(2 * j)) & np.uint64(1)) << np.uint64(j)
+        out |= ((w >> np.uint64(2 * j + 1)) & np.uint64(1)) << np.uint64(16 + j)
+    return out.astype(np.uint32)
+
+
+@pytest.mark.parametrize("S", [32, 64, 128, 256, 512])
+def test_tensor_core_upload_layout_from_the_bit_tiles(S, tmp_path_factory, tmp_path):
+    """The host-built operands of the tensor-core band kernels, rebuilt from the plan's bit tiles
+    (themselves bit-exact against the oracle): for each 128-row tile and type, C1 window chunks
+    of 128 columns starting one block before the tile's block-row, 4 interleaved words per row,
+    zero outside the row's three block diagonals; the transposed orientation likewise from the
+    transposed tiles; and per row and type the in-degree over the three diagonals as bf16."""
+    exe = _probe_binary(tmp_path_factory)
+    P = 6
+    gs = synth.gen_batch(5, 40, 3 * S, 6, False, max(2, S // 2), max(2, S // 3), 1.5, 300 + S)
+    n = sum(g.n_nodes for g in gs)
+    K0 = -(-n // S)
+    if K0 * S % 128:  # whole 128-row tiles, as the tensor-core path requires: pad with a graph
+        gs.append(synth.Graph(128 * (-(-K0 * S // 128)) - n, np.zeros(0, np.int32),
+                              np.zeros(0, np.int32), np.zeros(0, np.int32), P))
+    blob = [np.int32(len(gs)).tobytes()]
+    for g in gs:
+        blob += [np.int32(g.n_nodes).tobytes(), np.int64(g.n_edges).tobytes(),
+                 np.asarray(g.src, np.int32).tobytes(), np.asarray(g.dst, np.int32).tobytes(),
+                 np.asarray(g.etype, np.int32).tobytes()]
+    (tmp_path / "in.bin").write_bytes(b"".join(blob))
+    C1 = 2 if S <= 64 else 3 * S // 128
+    import subprocess
+    subprocess.run([exe, str(tmp_path / "in.bin"), str(tmp_path / "out.bin"), str(P), str(S),
+                    str(C1)], check=True)
+    raw = (tmp_path / "out.bin").read_bytes()
+    K, max_deg = np.frombuffer(raw[:8], np.int32)
+    nm, nI, nTI, nd = np.frombuffer(raw[8:40], np.int64)
+    o = 40
+    masks = np.frombuffer(raw[o:o + 4 * nm], np.uint32); o += 4 * nm
+    masksT = np.frombuffer(raw[o:o + 4 * nm], np.uint32); o += 4 * nm
+    mI = np.frombuffer(raw[o:o + 4 * nI], np.uint32); o += 4 * nI
+    mTI = np.frombuffer(raw[o:o + 4 * nTI], np.uint32); o += 4 * nTI
+    deg = np.frombuffer(raw[o:o + 2 * nd], np.uint16)
+    W32 = S // 32
+    N = int(K) * S
+    T = N // 128
+    assert N % 128 == 0 and nI == T * P * C1 * 128 * 4 and nd == N * 64
+    for tiles, got in ((masks, mI), (masksT, mTI)):
+        tiles = tiles.reshape(int(K), 3, P, S, W32)
+        exp = np.zeros((T, P, C1, 128, 4), np.uint32)
+        for t in range(T):
+            R = 128 * t + np.arange(128)
+            kr = R // S
+            ws = (128 * t // S) * S - S
+            for j in range(C1):
+                for w in range(4):
+                    c = ws + 128 * j + 32 * w
+                    if not 0 <= c < N:
+                        continue
+                    d = c // S - kr + 1
+                    ok = (d >= 0) & (d <= 2)
+                    words = tiles[kr[ok], d[ok], :, R[ok] % S, (c % S) // 32]   # [rows, P]
+                    exp[t, :, j, np.flatnonzero(ok), w] = _interleave(words)  # [rows, P]
+        np.testing.assert_array_equal(got.reshape(T, P, C1, 128, 4), exp)
+    bits = np.unpackbits(masks.reshape(int(K), 3, P, S, W32).view(np.uint8), axis=-1)
+    cnt = bits.reshape(int(K), 3, P, S, -1).sum(axis=(1, 4))                    # [K, P, S]
+    as_bf16 = (cnt.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    exp_deg = np.zeros((N, 64), np.uint16)
+    exp_deg[:, :P] = as_bf16.transpose(0, 2, 1).reshape(N, P)
+    exp_deg[:, 32:32 + P] = exp_deg[:, :P]
+    np.testing.assert_array_equal(deg.reshape(N, 64), exp_deg)
+    assert max_deg == cnt.max()
