@@ -150,7 +150,10 @@ size_t bg_ggnn_workspace_bytes(const bg_plan* plan, bg_dtype dtype, int32_t H, i
  * computed per block-row as Algorithm 1 does: the three diagonals' tiles aggregate the
  * neighbouring state blocks per type, then one contraction with the concatenated [P*H, H] edge
  * weights.  E [n_pad, H] (dtype), W [P, H, H] (dtype, W[p][h_in][h_out]), b [P, H] fp32 or NULL,
- * Y [n_pad, H] fp32 (overwritten). */
+ * Y [n_pad, H] fp32 (overwritten).  The bf16 tensor-core path adds the bias as in-degree x bias
+ * products on the tensor cores; on a plan where some node has more than 256 in-edges of one type
+ * these run in fp16, which holds |b| <= 65504: a larger finite bias is reported by
+ * bg_check_device as BG_EDEVICE (site 120). */
 int bg_band_propagate_fwd(const bg_plan* plan, bg_dtype dtype, int32_t H, const void* E,
                           const void* W, const float* b, float* Y, void* ws, size_t ws_bytes,
                           void* stream);
@@ -167,17 +170,21 @@ int bg_band_propagate_bwd(const bg_plan* plan, bg_dtype dtype, int32_t H, const 
 /* Same result as bg_band_propagate_fwd, for callers that cannot allocate device memory while they
  * run (no allocator of their own for the workspace, or cudaMalloc forbidden at that point): the
  * scratch comes from a fixed 32 MiB array inside the library (static device memory, reserved on
- * every GPU where the library's device code is loaded, until the process exits) instead of a
- * caller workspace, and the call itself allocates nothing -- no cudaMalloc, cudaFree or allocating
- * library routine.  The paper has no counterpart; this is a deployment variant.
- * The plan must already be uploaded (bg_plan_upload allocates).  The first call on each device
- * resolves the array's device address (cudaGetSymbolAddress, that device current), so make it
- * before any stream capture.  Returns BG_ECAPACITY, with a message giving both sizes, when the
- * plan needs more scratch than the array holds (bg_workspace_bytes(..., BG_OP_PROPAGATE_FWD) >
- * 32 MiB).  All calls share the array: calls that overlap on the GPU (different streams, or
+ * every GPU where this part of the library's device code is loaded, until the process exits)
+ * instead of a caller workspace, and the call itself allocates nothing -- no cudaMalloc, cudaFree
+ * or allocating library routine.  The paper has no counterpart; this is a deployment variant.
+ * Set-up: bg_plan_upload (which allocates anyway, and must precede this call on the same device)
+ * resolves the array's device address (cudaGetSymbolAddress with that device current, which also
+ * reserves the array there), creates the library's status word and loads the forward kernels of
+ * the plan's block size, so no set-up is left for the first call.
+ * Scratch needed: the tensor-core path (bg_band_uses_tensor_cores = 1) needs about
+ * n_pad H 2 + P H^2 4 bytes plus the split-tile partials; the SIMT path n_pad P H 4 bytes.  A plan
+ * that needs more than 32 MiB is refused with BG_ECAPACITY and a message giving both sizes.
+ * All calls share the array, which keeps the previous call's contents (every byte a call reads is
+ * written earlier in the same call): calls that overlap on the GPU (different streams, or
  * different host threads without ordering) race and corrupt each other's results; serialise them.
- * Bounded device waits that give up are recorded in a status word private to this entry point and
- * are not reported by bg_check_device. */
+ * Bounded device waits that give up are recorded in the library's status word, as for every other
+ * entry point: bg_check_device reports them (BG_ETIMEOUT) and clears the word. */
 int bg_band_propagate_fwd_noalloc(const bg_plan* plan, bg_dtype dtype, int32_t H, const void* E,
                                   const void* W, const float* b, float* Y, void* stream);
 

@@ -152,6 +152,12 @@ int status_word_ptr(int** out) {
 }
 }  // namespace
 
+int* bg_status_word_if_created(int dev) {
+  if (dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> g(g_status_mu);
+  return g_status[dev];
+}
+
 extern "C" int bg_selftest_device_wait(void* stream) {
   bg_clear_error();
   int* d = nullptr;
@@ -301,6 +307,13 @@ extern "C" int bg_plan_upload(bg_plan* p, void* stream) {
   if (bg::band_tc_upload(p, st) != 0) {
     free_device(p);
     return bg_fail(BG_ENOMEM, "device allocation for the band tiles failed");
+  }
+  // everything a device call may need to create on this device is created here, so that the
+  // allocation-free entry point finds it: the status word, its static scratch, the kernels
+  int* status = nullptr;
+  if ((rc = status_word_ptr(&status)) != BG_OK || (rc = bg_noalloc_prepare(p)) != BG_OK) {
+    free_device(p);
+    return rc;
   }
   return BG_OK;
 }
@@ -792,7 +805,7 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
     BG_CUDA(bg::fill_ones_rows(ETa, H, (int64_t)TN, (int64_t)TN, st));
     BG_CUDA(bg::fill_ones_rows(YTa, H, (int64_t)TN, (int64_t)TN, st));
     BG_CUDA(bg::band_tc_prep_w(p, H, prm->W, 0, WT, st));
-    if (prm->b) BG_CUDA(bg::prep_bias_split(prm->b, b2T, p->P, H, st));
+    if (prm->b) BG_CUDA(bg::prep_bias_split(p, prm->b, b2T, H, status, st));
     for (int t = 0; t < T; ++t) {
       {
         KTimer tm(BG_KID_BAND_FWD, st);

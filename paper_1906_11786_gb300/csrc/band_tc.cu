@@ -5,7 +5,8 @@
 //     pre_p = sum_{d in -1,0,+1} A_{k,d,p} E_{k+d}        (128 x 3S  times  3S x H, fp32 in TMEM)
 //     Y_k  += pre_p W_p                                     (chained MMA, A operand read from TMEM)
 // and the per-type bias enters as one more product deg_k [128 x 2P] x [b_hi; b_lo] with exact
-// integer in-degrees and b split into two bf16 halves.  pre_p never leaves the SM.
+// integer in-degrees and b split into two bf16 halves (fp16 for a plan with an in-degree above
+// 256, where bf16 integers stop being exact).  pre_p never leaves the SM.
 // Backward (transposed band): the same kernel with the transposed tiles, dY instead of E and W_p
 // instead of W_p^T gives dE_j += sum_p (A^T dY)_p W_p^T; dM_p = A_p^T dY is also written (bf16,
 // transposed) for the weight gradient.
@@ -40,6 +41,7 @@
 // than the expanders sleep between polls so that the MMA issuers keep their issue slots.
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cudaTypedefs.h>
 
 #include <cstdlib>
@@ -202,7 +204,7 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
               const uint32_t* __restrict__ maskI, float* __restrict__ out,
               __nv_bfloat16* __restrict__ outb, __nv_bfloat16* __restrict__ outT, int64_t ld_outT,
               __nv_bfloat16* __restrict__ dMT, int64_t ld_mt, const Sched sc, int P, int has_bias,
-              int accumulate, int* status) {
+              int bias_f16, int accumulate, int* status) {
   using C = Cfg<H, S>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -412,7 +414,9 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     // Y (+)= pre_p W_p over the jobs (kind::tf32, A = the fp32 pre_p unit in TMEM, K = the 64 rows
     // of W_p of the job's half), then the bias product
     const bool leader = elect_one_sync();
-    constexpr uint32_t idesc = idesc_bf16_f32(kTile, H);
+    // the bias product: in-degrees and bias halves as bf16, or as fp16 when an in-degree exceeds
+    // 256 (the plan's hub rows)
+    const uint32_t idesc = bias_f16 ? idesc_f16_f32(kTile, H) : idesc_bf16_f32(kTile, H);
     constexpr uint32_t idesc2 = idesc_tf32_f32(kTile, H);
     uint32_t c = 0, widx = 0, di = 0;
     bool ok = true;
@@ -717,19 +721,25 @@ __global__ void k_band_split_fixup(const float* __restrict__ part, int ksplit, i
   }
 }
 
-// b2T[h][p] = bf16 hi part of b[p][h], b2T[h][32 + p] = bf16 of the remainder (zero beyond P)
-__global__ void k_bias_split(const float* __restrict__ b, __nv_bfloat16* __restrict__ b2T, int P,
-                             int H) {
+// b2T[h][p] = high part of b[p][h], b2T[h][32 + p] = the remainder (zero beyond P), both bf16, or
+// both fp16 (f16 != 0; the in-degrees are then fp16 too).  fp16 holds magnitudes up to 65504: a
+// finite bias beyond that is recorded in the status word (code 2, site 120) and the product is
+// then not to be trusted.
+__global__ void k_bias_split(const float* __restrict__ b, uint16_t* __restrict__ b2T, int P, int H,
+                             int f16, int* status) {
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= H * 64) return;
   const int h = t / 64, q = t % 64, p = q % 32;
-  float v = 0.f;
-  if (p < P && b) {
-    const float x = b[p * H + h];
+  float x = 0.f;
+  if (p < P && b) x = b[p * H + h];
+  if (f16) {
+    if (fabsf(x) > 65504.f && isfinite(x) && atomicCAS(status, 0, 2) == 0) atomicExch(status + 1, 120);
+    const __half hi = __float2half_rn(x);
+    b2T[t] = __half_as_ushort(q < 32 ? hi : __float2half_rn(x - __half2float(hi)));
+  } else {
     const __nv_bfloat16 hi = __float2bfloat16_rn(x);
-    v = q < 32 ? __bfloat162float(hi) : x - __bfloat162float(hi);
+    b2T[t] = __bfloat16_as_ushort(q < 32 ? hi : __float2bfloat16_rn(x - __bfloat162float(hi)));
   }
-  b2T[t] = __float2bfloat16_rn(v);
 }
 
 // ------------------------------------------------------------------------------------ host
@@ -814,7 +824,7 @@ cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap&
   const int grid = std::min(sc.n_items, sms);
   e = launch_pdl(k_band_tc<H, S, BWD>, dim3(grid), dim3(C::THREADS), C::SMEM, st, tx, tw, tdeg,
                  tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt, sc,
-                 p->P, has_bias, accumulate, status);
+                 p->P, has_bias, p->max_deg > 256 ? 1 : 0, accumulate, status);
   note_launch();
   if (e != cudaSuccess || sc.ksplit == 1) return e;
   const int64_t n4 = (int64_t)sc.part_rows * H / 4;
@@ -902,7 +912,7 @@ bool band_tc_supported(const bg_plan* p, int dtype, int H) {
   const bool shape = ((H == 32 || H == 64 || H == 128) &&
                       (p->S == 32 || p->S == 64 || p->S == 128 || p->S == 256 || p->S == 512)) ||
                      (H == 256 && (p->S == 32 || p->S == 64 || p->S == 128));
-  return shape && p->d_maskI && p->d_maskTI && p->d_deg2 && p->max_deg <= 256 &&
+  return shape && p->d_maskI && p->d_maskTI && p->d_deg2 && p->max_deg < 2048 &&
          encode_fn() != nullptr;
 }
 
@@ -999,8 +1009,10 @@ cudaError_t prep_transpose_bf16(const void* in, int in_is_f32, __nv_bfloat16* ou
   return cudaGetLastError();
 }
 
-cudaError_t prep_bias_split(const float* b, __nv_bfloat16* b2T, int P, int H, cudaStream_t st) {
-  k_bias_split<<<(H * 64 + 255) / 256, 256, 0, st>>>(b, b2T, P, H);
+cudaError_t prep_bias_split(const bg_plan* p, const float* b, __nv_bfloat16* b2T, int H,
+                            int* status, cudaStream_t st) {
+  k_bias_split<<<(H * 64 + 255) / 256, 256, 0, st>>>(b, reinterpret_cast<uint16_t*>(b2T), p->P, H,
+                                                     p->max_deg > 256 ? 1 : 0, status);
   note_launch();
   return cudaGetLastError();
 }
@@ -1018,7 +1030,7 @@ cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, c
   // E [n][H] -> ET [H][n];  W_p [H_in][H_out] -> W_p^T in the kernel's operand type;  bias split
   cudaError_t e = prep_transpose_bf16(E, 0, ET, n, H, 1, st);
   if (e == cudaSuccess) e = band_tc_prep_w(p, H, W, 0, WT, st);
-  if (e == cudaSuccess && b) e = prep_bias_split(b, b2T, P, H, st);
+  if (e == cudaSuccess && b) e = prep_bias_split(p, b, b2T, H, status, st);
   if (e != cudaSuccess) return e;
   ProfSpan span(BG_KID_BAND_FWD, st);
   return band_tc_fwd_core(p, H, ET, n, WT, b ? b2T : nullptr, Y, nullptr, nullptr, 0,
@@ -1078,6 +1090,30 @@ int band_tc_upload(bg_plan* p, cudaStream_t st) {
     return -1;
   if (cudaStreamSynchronize(st) != cudaSuccess) return -1;
   return 0;
+}
+
+cudaError_t band_tc_preload_fwd(const bg_plan* p) {
+  if (!encode_fn()) return cudaErrorNotSupported;
+  cudaFuncAttributes a;
+  cudaError_t e = cudaSuccess;
+  auto take = [&](cudaError_t r) { if (e == cudaSuccess) e = r; };
+  take(cudaFuncGetAttributes(&a, k_transpose_bf16<__nv_bfloat16>));
+  take(cudaFuncGetAttributes(&a, k_prep_w));
+  take(cudaFuncGetAttributes(&a, k_bias_split));
+  take(cudaFuncGetAttributes(&a, k_band_split_fixup));
+#define BG_PRELOAD(HV, SV) take(cudaFuncGetAttributes(&a, k_band_tc<HV, SV, false>));
+#define BG_PRELOAD_S(SV) BG_PRELOAD(32, SV) BG_PRELOAD(64, SV) BG_PRELOAD(128, SV)
+  switch (p->S) {
+    case 32: BG_PRELOAD_S(32) BG_PRELOAD(256, 32) break;
+    case 64: BG_PRELOAD_S(64) BG_PRELOAD(256, 64) break;
+    case 128: BG_PRELOAD_S(128) BG_PRELOAD(256, 128) break;
+    case 256: BG_PRELOAD_S(256) break;
+    case 512: BG_PRELOAD_S(512) break;
+    default: break;
+  }
+#undef BG_PRELOAD_S
+#undef BG_PRELOAD
+  return e;
 }
 
 void band_tc_release(bg_plan* p) {

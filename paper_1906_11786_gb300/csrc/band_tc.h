@@ -43,8 +43,11 @@ cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, 
 // ld_out <= 0 means R; batches are R*Cc apart on both sides).
 cudaError_t prep_transpose_bf16(const void* in, int in_is_f32, __nv_bfloat16* out, int R, int Cc,
                                 int batch, cudaStream_t st, int64_t ld_out = 0);
-// [H][64] bf16: columns p / 32+p hold the bf16 high part / remainder of b[p][h].
-cudaError_t prep_bias_split(const float* b, __nv_bfloat16* b2T, int P, int H, cudaStream_t st);
+// [H][64] 16-bit: columns p / 32+p hold the high part / remainder of b[p][h], as bf16, or as fp16
+// for a plan whose in-degrees exceed 256 (the in-degree table is fp16 then; a finite |b| above
+// 65504 is recorded in `status`).
+cudaError_t prep_bias_split(const bg_plan* p, const float* b, __nv_bfloat16* b2T, int H,
+                            int* status, cudaStream_t st);
 // Builds and uploads the tensor-core path's plan data (no-op where unsupported); 0 on success.
 int band_tc_upload(bg_plan* p, cudaStream_t st);
 // Host side of band_tc_upload (band_tiles.cpp): the bit-interleaved window chunks of every
@@ -52,6 +55,9 @@ int band_tc_upload(bg_plan* p, cudaStream_t st);
 // orientations, and the per-row in-degrees [n_pad][64] as bf16; returns the largest in-degree.
 int band_tc_host_tiles(const bg_plan* p, int C1, std::vector<uint32_t>& mi,
                        std::vector<uint32_t>& mti, std::vector<uint16_t>& deg);
+// Loads (CUDA lazy loading) every kernel band_tc_fwd can launch for this plan's block size, at
+// any H, on the current device.
+cudaError_t band_tc_preload_fwd(const bg_plan* p);
 // Frees device data the tensor-core path keeps with the plan.
 void band_tc_release(bg_plan* p);
 

@@ -5,7 +5,8 @@
 // with the bits of each word interleaved (column 2j at bit j, column 2j+1 at bit 16+j) so that the
 // kernel turns a word into packed bf16 pairs with one AND and one multiply; words outside the three
 // block diagonals of the row's block-row are zero.  And per row and type the in-degree over the
-// three diagonals as a bf16 integer (columns p and 32 + p), the bias product's A operand.
+// three diagonals (columns p and 32 + p), the bias product's A operand: bf16 integers when every
+// in-degree is at most 256, fp16 integers otherwise (a hub node; fp16 is exact up to 2048).
 #include <algorithm>
 #include <cstring>
 #include <thread>
@@ -45,9 +46,27 @@ void parallel_ranges(int64_t n, F f) {
   for (auto& th : pool) th.join();
 }
 
+// bf16 bit pattern of a count (exact up to 256).
+inline uint16_t bf16_bits_of_count(int c) {
+  const float f = (float)c;
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  return (uint16_t)(u >> 16);
+}
+
+// IEEE fp16 bit pattern of a count in [0, 2048) (exact: at most 11 significant bits).
+inline uint16_t f16_bits_of_count(int c) {
+  if (c == 0) return 0;
+  int e = 0;
+  while ((c >> (e + 1)) != 0) ++e;  // floor(log2 c)
+  const uint32_t mant = ((uint32_t)c << (10 - e)) & 0x3FFu;
+  return (uint16_t)(((uint32_t)(e + 15) << 10) | mant);
+}
+
 }  // namespace
 
-// mi, mti: [n_tiles][P][C1][128][4] words; deg: [n_pad][64] bf16.  Returns the largest in-degree.
+// mi, mti: [n_tiles][P][C1][128][4] words; deg: [n_pad][64] in-degrees (type q at columns q and
+// 32 + q) as bf16 when the largest is at most 256, else as fp16.  Returns the largest in-degree.
 int band_tc_host_tiles(const bg_plan* p, int C1, std::vector<uint32_t>& mi,
                        std::vector<uint32_t>& mti, std::vector<uint16_t>& deg) {
   constexpr int kTile = 128;
@@ -74,29 +93,37 @@ int band_tc_host_tiles(const bg_plan* p, int C1, std::vector<uint32_t>& mi,
             }
     }
   });
+  // in-degrees first, then their encoding: bf16 while every count is at most 256 (exact), else
+  // fp16 (exact up to 2048 > 3 S for every block size)
+  std::vector<uint16_t> cnt((size_t)n * P, 0);
   std::vector<int> part_max(K, 0);
   parallel_ranges(K, [&](int64_t k0, int64_t k1) {
     for (int64_t k = k0; k < k1; ++k) {
       int mx = 0;
       for (int q = 0; q < P; ++q)
         for (int r = 0; r < S; ++r) {
-          int cnt = 0;
+          int c = 0;
           for (int d = 0; d < 3; ++d)
             for (int w = 0; w < W32; ++w)
-              cnt += __builtin_popcount(p->masks[((((size_t)k * 3 + d) * P + q) * S + r) * W32 + w]);
-          mx = std::max(mx, cnt);
-          // bf16 bit pattern of a small integer (exact up to 256)
-          const float f = (float)cnt;
-          uint32_t u;
-          std::memcpy(&u, &f, 4);
-          const uint16_t bfv = (uint16_t)(u >> 16);
-          deg[((size_t)k * S + r) * 64 + q] = bfv;
-          deg[((size_t)k * S + r) * 64 + 32 + q] = bfv;
+              c += __builtin_popcount(p->masks[((((size_t)k * 3 + d) * P + q) * S + r) * W32 + w]);
+          mx = std::max(mx, c);
+          cnt[((size_t)k * S + r) * P + q] = (uint16_t)c;
         }
       part_max[k] = mx;
     }
   });
-  return *std::max_element(part_max.begin(), part_max.end());
+  const int max_deg = *std::max_element(part_max.begin(), part_max.end());
+  const bool f16 = max_deg > 256;
+  parallel_ranges(n, [&](int64_t r0, int64_t r1) {
+    for (int64_t r = r0; r < r1; ++r)
+      for (int q = 0; q < P; ++q) {
+        const uint16_t v = f16 ? f16_bits_of_count(cnt[(size_t)r * P + q])
+                               : bf16_bits_of_count(cnt[(size_t)r * P + q]);
+        deg[(size_t)r * 64 + q] = v;
+        deg[(size_t)r * 64 + 32 + q] = v;
+      }
+  });
+  return max_deg;
 }
 
 }  // namespace bg

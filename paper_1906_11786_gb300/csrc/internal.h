@@ -35,7 +35,7 @@ struct bg_plan {
   int32_t* d_row_graph = nullptr;  // [n_pad] packed graph of each position, -1 for padding
   // tensor-core path: bit-interleaved window chunks [n_pad / 128][P][C1][128][4] (C1 128-column
   // chunks per 128-row tile, band_tc.cu) in both orientations and per-row in-degree counts
-  // [n_pad][64] bf16 (type p at columns p and 32 + p)
+  // [n_pad][64] (type p at columns p and 32 + p), bf16 while max_deg <= 256, else fp16
   uint32_t* d_maskI = nullptr;
   uint32_t* d_maskTI = nullptr;
   uint16_t* d_deg2 = nullptr;
@@ -46,6 +46,13 @@ struct bg_plan {
 // error plumbing (api.cu)
 int bg_fail(int code, const std::string& msg);
 void bg_clear_error();
+// The device status word of device `dev` that bounded waits write and bg_check_device reads, or
+// NULL when it has not been created yet (api.cu; bg_plan_upload creates it).  Never allocates.
+int* bg_status_word_if_created(int dev);
+// Device-side set-up of the allocation-free entry point for the current device (noalloc.cu):
+// resolves its static scratch array's address and loads the forward kernels of this plan's block
+// size.  Called by bg_plan_upload, which allocates anyway.
+int bg_noalloc_prepare(const bg_plan* p);
 
 // planner entry (plan.cpp)
 int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S, int32_t cap,

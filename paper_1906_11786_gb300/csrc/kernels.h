@@ -74,6 +74,8 @@ cudaError_t unpack_states(int bf16, const void* Eb, void* Eo, const int32_t* gat
 // Band aggregation over bit tiles: out[i] = sum_{slot, p, set bits c} X_p[(k+slot-1)S + c]
 //   forward  (rows = targets):  X = M [P][n_pad][H], out = Y [n_pad][H]
 //   backward (rows = sources):  X = dY [n_pad][H] shared by all p, out = dM [n_pad][P][H]
+// Loads (CUDA lazy loading) every kernel band_fwd_gather and gemm can launch on this device.
+cudaError_t preload_fwd_simt();
 cudaError_t band_fwd_gather(const uint32_t* masks, const float* M, float* Y, int K, int S, int P,
                             int H, cudaStream_t st);
 cudaError_t band_bwd_gather(const uint32_t* masksT, const float* dY, float* dM, int K, int S,

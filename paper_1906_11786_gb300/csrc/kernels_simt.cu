@@ -486,6 +486,20 @@ cudaError_t unpack_states(int bf16, const void* Eb, void* Eo, const int32_t* gat
   return cudaGetLastError();
 }
 
+cudaError_t preload_fwd_simt() {
+  // CUDA loads kernels lazily, on first launch; this loads the ones the SIMT forward launches
+  cudaFuncAttributes a;
+  cudaError_t e = cudaSuccess;
+  auto take = [&](cudaError_t r) { if (e == cudaSuccess) e = r; };
+  take(cudaFuncGetAttributes(&a, k_gemm<__nv_bfloat16, __nv_bfloat16>));
+  take(cudaFuncGetAttributes(&a, k_gemm<__nv_bfloat16, float>));
+  take(cudaFuncGetAttributes(&a, k_gemm<float, __nv_bfloat16>));
+  take(cudaFuncGetAttributes(&a, k_gemm<float, float>));
+  take(cudaFuncGetAttributes(&a, k_gemm_reduce));
+  take(cudaFuncGetAttributes(&a, k_band_fwd_gather));
+  return e;
+}
+
 cudaError_t band_fwd_gather(const uint32_t* masks, const float* M, float* Y, int K, int S, int P,
                             int H, cudaStream_t st) {
   int64_t rows = (int64_t)K * S;

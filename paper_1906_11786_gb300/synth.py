@@ -18,7 +18,7 @@ import numpy as np
 
 __all__ = [
     "Graph", "gen_graph", "gen_batch", "gen_states", "gen_params", "WORKLOADS", "workload_graphs",
-    "graph_seed",
+    "graph_seed", "hub_graph", "with_self_loops",
 ]
 
 
@@ -168,6 +168,40 @@ def gen_batch(count: int, n_lo: int, n_hi: int, n_families: int, reverse: bool, 
     sizes = rng.integers(n_lo, n_hi + 1, size=count)
     return [gen_graph(int(n), n_families, reverse, max_off, tree_win, lam, seed * 7919 + 13 * g)
             for g, n in enumerate(sizes)]
+
+
+def hub_graph(n_leaves: int, n_types: int, seed: int, lam: float = 1.0) -> Graph:
+    """A program-shaped graph with one hub: a chain (type 1) over n_leaves + 1 nodes, every node
+    also sending a type-0 edge to node 0 (in-degree n_leaves of one type, as a much-used variable
+    or a shared declaration would receive), plus round(lam n) short-range edges of types
+    2..n_types-1 at offsets up to 8; then a uniform random relabelling."""
+    n = n_leaves + 1
+    rng = np.random.default_rng(seed)
+    src = [np.arange(1, n), np.arange(n - 1)]
+    dst = [np.zeros(n - 1, np.int64), np.arange(1, n)]
+    et = [np.zeros(n - 1, np.int64), np.ones(n - 1, np.int64)]
+    m = int(round(lam * n)) if n_types > 2 else 0
+    if m:
+        s = rng.integers(0, n, size=m)
+        t = np.clip(s + rng.integers(-8, 9, size=m), 0, n - 1)
+        src.append(s); dst.append(t); et.append(rng.integers(2, n_types, size=m))
+    src, dst, et = (np.concatenate(x).astype(np.int64) for x in (src, dst, et))
+    key = (et * n + src) * n + dst
+    _, first = np.unique(key, return_index=True)
+    first.sort()
+    relabel = rng.permutation(n)
+    return Graph(n, relabel[src[first]].astype(np.int32), relabel[dst[first]].astype(np.int32),
+                 et[first].astype(np.int32), n_types)
+
+
+def with_self_loops(g: Graph, frac: float, n_types: int, seed: int) -> Graph:
+    """`g` plus a self-loop u -> u of a uniform type on a uniform random `frac` of its nodes."""
+    rng = np.random.default_rng(seed)
+    k = int(round(frac * g.n_nodes))
+    u = rng.choice(g.n_nodes, size=k, replace=False).astype(np.int32)
+    t = rng.integers(0, n_types, size=k).astype(np.int32)
+    return Graph(g.n_nodes, np.concatenate([g.src, u]), np.concatenate([g.dst, u]),
+                 np.concatenate([g.etype, t]), max(g.n_types, n_types), dict(g.meta))
 
 
 def gen_states(n: int, H: int, seed: int) -> np.ndarray:

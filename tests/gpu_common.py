@@ -25,6 +25,26 @@ def rel_err(got, ref) -> float:
     return float(np.max(np.abs(got - ref)) / max(float(np.max(np.abs(ref))), 1e-30))
 
 
+def med_rel_err(got, ref) -> float:
+    """Element-wise median relative error |g - o| / |o| over the entries with |o| > 1e-3 max|o|
+    (reading c14's second measure: an error confined to small entries, such as the rows of
+    low-degree nodes, is under-weighted by the max-norm measure)."""
+    got = np.asarray(got, np.float64).ravel()
+    ref = np.asarray(ref, np.float64).ravel()
+    big = np.abs(ref) > 1e-3 * max(float(np.max(np.abs(ref))), 1e-30)
+    if not big.any():
+        return 0.0
+    return float(np.median(np.abs(got[big] - ref[big]) / np.abs(ref[big])))
+
+
+def assert_close(got, ref, tol: float, what: str = ""):
+    """Both parity measures of reading c14 under the same tolerance: the max-abs error over the
+    reference's max-abs value, and the element-wise median relative error."""
+    e_inf, e_med = rel_err(got, ref), med_rel_err(got, ref)
+    assert e_inf < tol and e_med < tol, \
+        f"{what}: max-norm rel {e_inf:.3e}, median rel {e_med:.3e}, tolerance {tol:g}"
+
+
 def quantize(x: np.ndarray, dtype: str) -> np.ndarray:
     """Round to the device dtype and back to float64 (both sides then start from equal values)."""
     if dtype == "bf16":
@@ -46,7 +66,7 @@ def f32_dev(x) -> torch.Tensor:
 class Case:
     """A planned, uploaded supergraph with packed device states and the oracle's view of it."""
 
-    def __init__(self, graphs, P, S, H, dtype, seed=0, cap=0):
+    def __init__(self, graphs, P, S, H, dtype, seed=0, cap=0, plain_xavier=False):
         self.P, self.S, self.H, self.dtype = P, S, H, dtype
         self.plan = L.band_plan(graphs, P, S, cap)
         self.plan.upload()
@@ -64,8 +84,10 @@ class Case:
         gi = self.ref.gather_index()
         self.E_band = np.zeros((self.N, H))
         self.E_band[: self.n_real] = E_orig[gi]
-        prm = synth.gen_params(P, H, seed + 1,
-                               mean_in_degree=self.ref.n_kept / max(self.ref.n_real, 1))
+        # plain_xavier: the H x H Xavier bound for W_p, as the workloads state it; otherwise the
+        # message layer's fan-in H x mean in-degree (reading r1, for the T = 8 recurrences)
+        prm = synth.gen_params(P, H, seed + 1, mean_in_degree=1.0 if plain_xavier else
+                               self.ref.n_kept / max(self.ref.n_real, 1))
         for k in ("W", "W_ih", "W_hh"):
             prm[k] = quantize(prm[k], dtype)
         for k in ("b", "b_ih", "b_hh", "w_out"):

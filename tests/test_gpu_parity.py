@@ -10,7 +10,7 @@ import oracle
 from paper_1906_11786_gb300 import _binding as L
 from paper_1906_11786_gb300 import synth
 
-from gpu_common import TOL, Case, ensure_built, f32_dev, quantize, rel_err
+from gpu_common import TOL, Case, assert_close, ensure_built, f32_dev, quantize, rel_err
 
 pytestmark = pytest.mark.gpu
 
@@ -87,10 +87,10 @@ def test_propagate_fp32_single512():
     """Single 512-node graph, 4 types, S = 64, H = 64, fp32, fwd + bwd."""
     c = Case(synth.workload_graphs("single512"), 4, 64, 64, "f32", seed=11)
     Y, ref = _fwd(c)
-    assert rel_err(Y, ref) < TOL["f32"]
+    assert_close(Y, ref, TOL["f32"], "")
     got, ref = _bwd(c)
     for g, r, name in zip(got, ref, ("dE", "dW", "db")):
-        assert rel_err(g, r) < TOL["f32"], name
+        assert_close(g, r, TOL["f32"], name)
 
 
 @pytest.mark.parametrize("S,H,whole", [(128, 64, 0), (64, 64, 1), (32, 32, 0), (256, 128, 0),
@@ -106,11 +106,11 @@ def test_propagate_bf16_packed_batch(S, H, whole):
     c = Case(gs, 20, S, H, "bf16", seed=S + H, cap=_cap_whole_tiles(gs, S) if whole else 0)
     assert c.info["K"] >= 3 and c.n_real % S != 0
     Y, ref = _fwd(c)
-    assert rel_err(Y, ref) < TOL["bf16"]
+    assert_close(Y, ref, TOL["bf16"], "")
     assert np.all(Y[c.n_real:] == 0)
     got, ref = _bwd(c)
     for g, r, name in zip(got, ref, ("dE", "dW", "db")):
-        assert rel_err(g, r) < TOL["bf16"], name
+        assert_close(g, r, TOL["bf16"], name)
 
 
 def test_propagate_bf16_no_bias_and_single_block():
@@ -118,7 +118,7 @@ def test_propagate_bf16_no_bias_and_single_block():
     c = Case([g], 8, 128, 64, "bf16", seed=2)
     assert c.info["K"] == 1
     Y, ref = _fwd(c, with_bias=False)
-    assert rel_err(Y, ref) < TOL["bf16"]
+    assert_close(Y, ref, TOL["bf16"], "")
 
 
 def test_propagate_graph_without_edges():
@@ -133,7 +133,7 @@ def test_propagate_bf16_dropped_edges_single20k_shape():
     g = synth.gen_graph(3000, 10, True, 200, 133, 3.0, 17)
     c = Case([g], 20, 256, 128, "bf16", seed=5)
     Y, ref = _fwd(c)
-    assert rel_err(Y, ref) < TOL["bf16"]
+    assert_close(Y, ref, TOL["bf16"], "")
 
 
 # ------------------------------------------------------------------------------------ GGNN
@@ -179,21 +179,21 @@ def test_ggnn_fwd_bwd(dtype, T, S, H, whole):
     assert L.band_uses_tensor_cores(c.plan, c.dtype, c.H) == _tc_shape(c)
     ET, ref_ET, grads, dE0, ref = _ggnn(c, T)
     tol = TOL[dtype]
-    assert rel_err(ET, ref_ET) < tol
+    assert_close(ET, ref_ET, tol, "")
     assert np.all(ET[c.n_real:] == 0)
-    assert rel_err(dE0, ref["dE0"]) < tol
+    assert_close(dE0, ref["dE0"], tol, "")
     for k, v in grads.items():
-        assert rel_err(v, ref[k]) < tol, k
+        assert_close(v, ref[k], tol, k)
 
 
 def test_ggnn_packed64_shape_T8_reduced_batch():
     """The packed64 workload's shapes (P = 20, S = 128, H = 64, bf16, T = 8) on an 8-graph batch."""
     c = Case(synth.workload_graphs("packed64", scale=0.125), 20, 128, 64, "bf16", seed=2)
     ET, ref_ET, grads, dE0, ref = _ggnn(c, 8)
-    assert rel_err(ET, ref_ET) < TOL["bf16"]
-    assert rel_err(dE0, ref["dE0"]) < TOL["bf16"]
+    assert_close(ET, ref_ET, TOL["bf16"], "")
+    assert_close(dE0, ref["dE0"], TOL["bf16"], "")
     for k, v in grads.items():
-        assert rel_err(v, ref[k]) < TOL["bf16"], k
+        assert_close(v, ref[k], TOL["bf16"], k)
 
 
 # ------------------------------------------------------------------------------------ readout, Adam
@@ -261,7 +261,7 @@ def _full_size_propagation(c: Case, seed: int, n_rows: int = 400, types=(0, 7, 1
     sel = np.isin(d, rows)
     ref = oracle.propagate_fwd(c.N, c.P, c.H, d[sel], s[sel], t[sel], c.E_band, c.prm["W"],
                                c.prm["b"])
-    assert rel_err(Y[rows], ref[rows]) < TOL["bf16"], "Y"
+    assert_close(Y[rows], ref[rows], TOL["bf16"], "Y")
 
     out = np.isin(s, rows)
     nodes = np.unique(np.concatenate([rows, d[out]]))
@@ -269,7 +269,7 @@ def _full_size_propagation(c: Case, seed: int, n_rows: int = 400, types=(0, 7, 1
     new[nodes] = np.arange(len(nodes))
     ref_dE, _, _ = oracle.propagate_bwd(len(nodes), c.P, c.H, new[d[out]], new[s[out]], t[out],
                                         c.E_band[nodes], c.prm["W"], dY[nodes])
-    assert rel_err(dE[rows], ref_dE[new[rows]]) < TOL["bf16"], "dE"
+    assert_close(dE[rows], ref_dE[new[rows]], TOL["bf16"], "dE")
 
     types = np.asarray(types)
     tmap = np.full(c.P, -1, np.int64)
@@ -277,8 +277,8 @@ def _full_size_propagation(c: Case, seed: int, n_rows: int = 400, types=(0, 7, 1
     ts = tmap[t] >= 0
     _, ref_dW, ref_db = oracle.propagate_bwd(c.N, len(types), c.H, d[ts], s[ts], tmap[t[ts]],
                                              c.E_band, c.prm["W"][types], dY)
-    assert rel_err(dW[types], ref_dW) < TOL["bf16"], "dW"
-    assert rel_err(db[types], ref_db) < TOL["bf16"], "db"
+    assert_close(dW[types], ref_dW, TOL["bf16"], "dW")
+    assert_close(db[types], ref_db, TOL["bf16"], "db")
 
 
 def test_full_size_packed64_propagate_sampled_rows():
@@ -351,14 +351,14 @@ def _full_size_ggnn_sampled_graphs(c: Case, T: int, pick, seed: int):
     ref = oracle.ggnn_bwd(m, c.P, c.H, T, m, *sub, c.prm, Es, Ys, dET[rows])
 
     got_ET = ET.float().cpu().numpy()
-    assert rel_err(got_ET[rows], Es[T]) < TOL["bf16"]
+    assert_close(got_ET[rows], Es[T], TOL["bf16"], "")
     got_dE0 = dE0.cpu().numpy()
-    assert rel_err(got_dE0[rows], ref["dE0"]) < TOL["bf16"]
+    assert_close(got_dE0[rows], ref["dE0"], TOL["bf16"], "")
     rest = np.ones(c.N, bool)
     rest[rows] = False
     assert np.all(got_dE0[rest] == 0.0)
     for k, v in grads.items():
-        assert rel_err(v.cpu().numpy(), ref[k]) < TOL["bf16"], k
+        assert_close(v.cpu().numpy(), ref[k], TOL["bf16"], k)
     return ET
 
 
@@ -417,5 +417,5 @@ def test_device_wait_timeout_is_reported_and_the_context_survives():
     g = synth.gen_graph(300, 4, True, 20, 10, 1.0, 11)
     c = Case([g], 8, 128, 64, "bf16", seed=4)
     Y, ref = _fwd(c)
-    assert rel_err(Y, ref) < TOL["bf16"]
+    assert_close(Y, ref, TOL["bf16"], "")
 

@@ -72,6 +72,18 @@ def test_planner_bit_exact_single20k():
     _compare(synth.workload_graphs("single20k"), 20, 256)
 
 
+@pytest.mark.parametrize("S", [32, 128, 512])
+def test_planner_bit_exact_self_loops_and_hubs(S):
+    """Self-loops (reading c6: allowed, on the diagonal tile) and a hub node with more in-edges
+    of one type than the block size: the planner stays bit-exact against the oracle."""
+    gs = synth.gen_batch(4, 50, 2 * S, 5, True, max(2, S // 2), max(2, S // 3), 1.5, 900 + S)
+    gs = [synth.with_self_loops(g, 0.2, 10, 31 + i) for i, g in enumerate(gs)]
+    gs.insert(2, synth.with_self_loops(synth.hub_graph(S + 40, 10, 5 + S), 0.1, 10, 3))
+    plan, ref = _compare(gs, 10, S)
+    loops = sum(int(np.sum(g.src == g.dst)) for g in gs)
+    assert loops > 0 and ref.n_kept > 0
+
+
 @pytest.mark.parametrize("S", [32, 64, 128, 256, 512])
 def test_planner_bit_exact_sweep131k_capacity(S):
     gs = synth.workload_graphs("sweep131k", S=S, scale=0.25)
@@ -179,8 +191,9 @@ def _interleave(w):
     return out.astype(np.uint32)
 
 
-@pytest.mark.parametrize("S", [32, 64, 128, 256, 512])
-def test_tensor_core_upload_layout_from_the_bit_tiles(S, tmp_path_factory, tmp_path):
+@pytest.mark.parametrize("S,hub", [(32, 0), (64, 0), (128, 0), (256, 0), (512, 0), (256, 1),
+                                   (512, 1)])
+def test_tensor_core_upload_layout_from_the_bit_tiles(S, hub, tmp_path_factory, tmp_path):
     """The host-built operands of the tensor-core band kernels, rebuilt from the plan's bit tiles
     (themselves bit-exact against the oracle): for each 128-row tile and type, C1 window chunks
     of 128 columns starting one block before the tile's block-row, 4 interleaved words per row,
@@ -189,6 +202,8 @@ def test_tensor_core_upload_layout_from_the_bit_tiles(S, tmp_path_factory, tmp_p
     exe = _probe_binary(tmp_path_factory)
     P = 6
     gs = synth.gen_batch(5, 40, 3 * S, 6, False, max(2, S // 2), max(2, S // 3), 1.5, 300 + S)
+    if hub:  # in-degrees above 256: the table switches to fp16
+        gs.insert(1, synth.hub_graph(S + S // 4, 2, 7 + S))
     n = sum(g.n_nodes for g in gs)
     K0 = -(-n // S)
     if K0 * S % 128:  # whole 128-row tiles, as the tensor-core path requires: pad with a graph
@@ -236,9 +251,13 @@ def test_tensor_core_upload_layout_from_the_bit_tiles(S, tmp_path_factory, tmp_p
         np.testing.assert_array_equal(got.reshape(T, P, C1, 128, 4), exp)
     bits = np.unpackbits(masks.reshape(int(K), 3, P, S, W32).view(np.uint8), axis=-1)
     cnt = bits.reshape(int(K), 3, P, S, -1).sum(axis=(1, 4))                    # [K, P, S]
-    as_bf16 = (cnt.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    if cnt.max() > 256:  # a hub: fp16 integers (exact up to 2048)
+        enc = cnt.astype(np.float16).view(np.uint16)
+    else:
+        enc = (cnt.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
     exp_deg = np.zeros((N, 64), np.uint16)
-    exp_deg[:, :P] = as_bf16.transpose(0, 2, 1).reshape(N, P)
+    exp_deg[:, :P] = enc.transpose(0, 2, 1).reshape(N, P)
     exp_deg[:, 32:32 + P] = exp_deg[:, :P]
     np.testing.assert_array_equal(deg.reshape(N, 64), exp_deg)
     assert max_deg == cnt.max()
+    assert (max_deg > 256) == bool(hub)
