@@ -17,6 +17,7 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "oracle.cpp")
+_SRC_PAR = os.path.join(_HERE, "oracle_par.cpp")
 _LIB = os.path.join(_HERE, "liboracle.so")
 _lock = threading.Lock()
 _lib = None
@@ -28,11 +29,17 @@ _u8p = np.ctypeslib.ndpointer(np.uint8, flags="C_CONTIGUOUS")
 
 
 def build(force: bool = False) -> str:
-    """Compile oracle.cpp into liboracle.so (g++ -O2, portable flags only)."""
+    """Compile oracle.cpp and its multi-threaded variant oracle_par.cpp into liboracle.so (g++ -O2,
+    portable flags only; no floating-point contraction, so that both files evaluate every
+    expression exactly as written on every host; OpenMP when the compiler has it)."""
     with _lock:
-        if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        newest = max(os.path.getmtime(_SRC), os.path.getmtime(_SRC_PAR))
+        if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < newest:
             tmp = _LIB + f".tmp{os.getpid()}"
-            subprocess.check_call(["g++", "-O2", "-std=c++17", "-shared", "-fPIC", "-o", tmp, _SRC])
+            base = ["g++", "-O2", "-std=c++17", "-ffp-contract=off", "-shared", "-fPIC", "-o", tmp,
+                    _SRC, _SRC_PAR]
+            if subprocess.call(base + ["-fopenmp"], stderr=subprocess.DEVNULL) != 0:
+                subprocess.check_call(base)
             os.replace(tmp, _LIB)
     return _LIB
 
@@ -72,6 +79,20 @@ def _load():
     lib.orc_readout_loss.restype = None
     lib.orc_readout_loss.argtypes = [c.c_int32] * 3 + [_i32p, _i32p, _f64p, _f64p, _f64p, _f64p,
                                                         _f64p, _f64p]
+    lib.orc_par_propagate_fwd.restype = None
+    lib.orc_par_propagate_fwd.argtypes = ([c.c_int32] * 3 + [c.c_int64, _i32p, _i32p, _i32p, _f64p,
+                                          _f64p, c.c_void_p, _f64p, c.c_int32])
+    lib.orc_par_propagate_bwd.restype = None
+    lib.orc_par_propagate_bwd.argtypes = ([c.c_int32] * 3 + [c.c_int64, _i32p, _i32p, _i32p, _f64p,
+                                          _f64p, _f64p, _f64p, _f64p, c.c_void_p, c.c_int32])
+    lib.orc_par_ggnn_fwd.restype = None
+    lib.orc_par_ggnn_fwd.argtypes = ([c.c_int32] * 5 + [c.c_int64, _i32p, _i32p, _i32p] +
+                                     [_f64p] * 8 + [c.c_int32])
+    lib.orc_par_ggnn_bwd.restype = None
+    lib.orc_par_ggnn_bwd.argtypes = ([c.c_int32] * 5 + [c.c_int64, _i32p, _i32p, _i32p] +
+                                     [_f64p] * 16 + [c.c_int32])
+    lib.orc_par_max_threads.restype = c.c_int32
+    lib.orc_par_max_threads.argtypes = []
     lib.orc_adam.restype = None
     lib.orc_adam.argtypes = [c.c_int64, _f64p, _f64p, _f64p, _f64p, c.c_double, c.c_double,
                              c.c_double, c.c_double, c.c_int32]
@@ -278,3 +299,58 @@ def adam(param, m, v, grad, lr, b1, b2, eps, t):
     p, mm, vv = _f64(param).copy(), _f64(m).copy(), _f64(v).copy()
     lib.orc_adam(p.size, p, mm, vv, _f64(grad), lr, b1, b2, eps, t)
     return p, mm, vv
+
+
+# ---------------------------------------------------------------------------------------------
+# multi-threaded pull-based variant (CPU baseline on all host cores; equal to the last bit to the
+# functions above)
+
+
+def par_max_threads() -> int:
+    """Threads the multi-threaded variant uses by default (1 when built without OpenMP)."""
+    return int(_load().orc_par_max_threads())
+
+
+def par_propagate_fwd(N, P, H, e_dst, e_src, e_type, E, W, b=None, threads=0) -> np.ndarray:
+    lib = _load()
+    e_dst, e_src, e_type = _i32(e_dst), _i32(e_src), _i32(e_type)
+    bb = None if b is None else _f64(b)
+    Y = np.zeros((N, H))
+    lib.orc_par_propagate_fwd(N, P, H, e_dst.shape[0], e_dst, e_src, e_type, _f64(E), _f64(W),
+                              None if bb is None else bb.ctypes.data_as(ctypes.c_void_p), Y,
+                              threads)
+    return Y
+
+
+def par_propagate_bwd(N, P, H, e_dst, e_src, e_type, E, W, dY, threads=0):
+    lib = _load()
+    e_dst, e_src, e_type = _i32(e_dst), _i32(e_src), _i32(e_type)
+    dE = np.zeros((N, H)); dW = np.zeros((P, H, H)); db = np.zeros((P, H))
+    lib.orc_par_propagate_bwd(N, P, H, e_dst.shape[0], e_dst, e_src, e_type, _f64(E), _f64(W),
+                              _f64(dY), dE, dW, db.ctypes.data_as(ctypes.c_void_p), threads)
+    return dE, dW, db
+
+
+def par_ggnn_fwd(N, P, H, T, n_real, e_dst, e_src, e_type, E0, prm, threads=0):
+    lib = _load()
+    Es = np.zeros((T + 1, N, H)); Es[0] = E0
+    Ys = np.zeros((max(T, 1), N, H))
+    e_dst, e_src, e_type = _i32(e_dst), _i32(e_src), _i32(e_type)
+    lib.orc_par_ggnn_fwd(N, P, H, T, n_real, e_dst.shape[0], e_dst, e_src, e_type, _f64(prm["W"]),
+                         _f64(prm["b"]), _f64(prm["W_ih"]), _f64(prm["W_hh"]), _f64(prm["b_ih"]),
+                         _f64(prm["b_hh"]), Es, Ys, threads)
+    return Es, Ys
+
+
+def par_ggnn_bwd(N, P, H, T, n_real, e_dst, e_src, e_type, prm, Es, Ys, dET, threads=0):
+    lib = _load()
+    e_dst, e_src, e_type = _i32(e_dst), _i32(e_src), _i32(e_type)
+    out = dict(dE0=np.zeros((N, H)), dW=np.zeros((P, H, H)), db=np.zeros((P, H)),
+               dW_ih=np.zeros((3 * H, H)), dW_hh=np.zeros((3 * H, H)), db_ih=np.zeros(3 * H),
+               db_hh=np.zeros(3 * H))
+    lib.orc_par_ggnn_bwd(N, P, H, T, n_real, e_dst.shape[0], e_dst, e_src, e_type, _f64(prm["W"]),
+                         _f64(prm["b"]), _f64(prm["W_ih"]), _f64(prm["W_hh"]), _f64(prm["b_ih"]),
+                         _f64(prm["b_hh"]), _f64(Es), _f64(Ys), _f64(dET), out["dE0"], out["dW"],
+                         out["db"], out["dW_ih"], out["dW_hh"], out["db_ih"], out["db_hh"],
+                         threads)
+    return out

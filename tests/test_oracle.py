@@ -437,3 +437,37 @@ def test_invalid_input_is_rejected():
     g = _graph(3, [(0, 1)], types=[3])
     with pytest.raises(ValueError):
         oracle.layout([g], 2, 8)
+
+
+# ------------------------------------------------------------------------ multi-threaded variant
+
+
+def test_parallel_oracle_equals_the_oracle_to_the_last_bit():
+    """The pull-based multi-threaded oracle (the CPU baseline on all host cores) adds every sum's
+    terms in the single-threaded oracle's order, so its outputs are identical to the last bit:
+    propagation forward and backward, and a T = 2 GGNN step forward and backward, with 4 threads
+    on a packed batch with self-loops and a hub."""
+    gs = synth.gen_batch(5, 50, 300, 4, True, 20, 12, 2.0, 404)
+    gs = [synth.with_self_loops(g, 0.1, 8, 5 + i) for i, g in enumerate(gs)]
+    gs.append(synth.hub_graph(150, 8, 9))
+    lay = oracle.layout(gs, 8, 64)
+    N, P, H, T = lay.n_pad, 8, 12, 2
+    e = (lay.kept_dst, lay.kept_src, lay.kept_type)
+    rng = np.random.default_rng(3)
+    E = np.zeros((N, H)); E[:lay.n_real] = rng.standard_normal((lay.n_real, H))
+    prm = synth.gen_params(P, H, 4)
+    dY = rng.standard_normal((N, H))
+    np.testing.assert_array_equal(oracle.par_propagate_fwd(N, P, H, *e, E, prm["W"], prm["b"], 4),
+                                  oracle.propagate_fwd(N, P, H, *e, E, prm["W"], prm["b"]))
+    for a, b in zip(oracle.par_propagate_bwd(N, P, H, *e, E, prm["W"], dY, 4),
+                    oracle.propagate_bwd(N, P, H, *e, E, prm["W"], dY)):
+        np.testing.assert_array_equal(a, b)
+    Es, Ys = oracle.ggnn_fwd(N, P, H, T, lay.n_real, *e, E, prm)
+    Es2, Ys2 = oracle.par_ggnn_fwd(N, P, H, T, lay.n_real, *e, E, prm, 4)
+    np.testing.assert_array_equal(Es2, Es)
+    np.testing.assert_array_equal(Ys2, Ys)
+    r = oracle.ggnn_bwd(N, P, H, T, lay.n_real, *e, prm, Es, Ys, dY)
+    r2 = oracle.par_ggnn_bwd(N, P, H, T, lay.n_real, *e, prm, Es, Ys, dY, 4)
+    for k in r:
+        np.testing.assert_array_equal(r2[k], r[k], err_msg=k)
+    assert oracle.par_max_threads() >= 1
