@@ -36,8 +36,10 @@ def _peaks():
     if os.path.exists(p):
         d = json.load(open(p))
         return {"hbm_gbs": d["hbm_gbs"], "bf16": d["bf16_tflops"],
-                "bf16_sustained": d["bf16_tflops_sustained"], "src": "measured"}
-    return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "src": "fallback"}
+                "bf16_sustained": d["bf16_tflops_sustained"],
+                "sm_max_mhz": d.get("sm_max_mhz", 2070.0), "src": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "sm_max_mhz": 2070.0,
+            "src": "fallback"}
 
 
 def _profiled_traffic(kernel: str, workload: str):
@@ -100,7 +102,9 @@ def _dist():
 
 
 class Clocks:
-    """Samples nvidia-smi clocks and throttle reasons while the timed region runs."""
+    """Samples nvidia-smi clocks and throttle reasons every 50 ms from before the warm-up to the
+    end of the end-to-end run (the timed steps, then a profiled pass of at least two seconds under
+    the same load); marks bracket the timed steps."""
 
     Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -110,6 +114,7 @@ class Clocks:
         self.index = index
         self.proc = None
         self.lines = []
+        self.marks = {}
 
     def __enter__(self):
         try:
@@ -125,10 +130,14 @@ class Clocks:
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.perf_counter(), line.strip()))
+
+    def mark(self, tag: str):
+        self.marks[tag] = time.perf_counter()
 
     def __exit__(self, *a):
         if self.proc:
+            time.sleep(0.1)  # the sample in flight
             self.proc.terminate()
             try:
                 self.proc.wait(timeout=5)
@@ -136,24 +145,31 @@ class Clocks:
                 self.proc.kill()
 
     def summary(self):
-        sm, mx, reasons = [], None, set()
+        sm, timed, mx, reasons = [], [], None, set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
+        t0, t1 = self.marks.get("timed_start"), self.marks.get("timed_end")
+        for t, ln in self.lines:
             f = [x.strip() for x in ln.split(",")]
             if len(f) < 8:
                 continue
             try:
-                sm.append(float(f[0]))
+                v = float(f[0])
                 mx = float(f[1])
             except ValueError:
                 continue
-            for n, v in zip(names, f[4:8]):
-                if v.lower() == "active":
+            sm.append(v)
+            if t0 is not None and t1 is not None and t0 <= t <= t1 + 0.05:
+                timed.append(v)
+            for n, r in zip(names, f[4:8]):
+                if r.lower() == "active":
                     reasons.add(n)
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
-                "samples": len(sm)}
+                "samples": len(sm), "samples_timed": len(timed),
+                "sm_mhz_timed": statistics.median(timed) if timed else None,
+                "window": "warm-up, the timed steps, the profiled pass (>= 2 s) and the "
+                          "end-to-end run, every 50 ms"}
 
 
 # --------------------------------------------------------------------------------- workload
@@ -375,66 +391,119 @@ class OursStep:
 # --------------------------------------------------------------------------------- CPU oracle
 
 
-def oracle_sample(name: str, c, budget_s: float = 15.0):
-    """The oracle as it stands (single-threaded fp64) on a bounded sample of the workload: the
-    leading graphs of the batch, as many as fit the time budget; returns node-steps/s."""
+def oracle_sample(name: str, c, budget_s: float = 15.0, parallel: bool = False,
+                  smallest_first: bool = False, graphs=None):
+    """The oracle as it stands on a bounded sample of the workload: fp64 forward + backward of the
+    workload's step (T GGNN steps with the GRU, or one propagation), timed without the layout
+    (the GPU number excludes the plan too).  Single-threaded: one graph at a time, leading graphs
+    first (or smallest first); parallel: the pull-based multi-threaded oracle on all host cores,
+    on supergraphs of eight graphs at a time.  A problem larger than the rest of the budget allows
+    (at the per-node cost measured so far, or before the first measurement at 1e9 multiply-adds
+    per second and thread) is cut to a prefix of its band positions: the subgraph the first m
+    positions induce, nodes of the same degree mix.  The graphs are taken in turn (again from the
+    first when the list ends) until the budget is spent.  Returns (node-steps/s, sample
+    description)."""
     import oracle
     from paper_1906_11786_gb300 import synth
-    graphs = synth.workload_graphs(name, S=c["S"])
+    graphs = graphs if graphs is not None else synth.workload_graphs(name, S=c["S"])
     P, S, H, T = c["P"], c["S"], c["H"], c["T"]
-    done_nodes, spent, used = 0, 0.0, 0
+    order = sorted(range(len(graphs)), key=lambda i: graphs[i].n_nodes) if smallest_first \
+        else list(range(len(graphs)))
+    group = 8 if parallel else 1
+    threads = oracle.par_max_threads() if parallel else 1
+    done_nodes, spent, used, cut = 0, 0.0, 0, 0
     rng = np.random.default_rng(0)
-    t_start = time.perf_counter()
-    for g in graphs:
-        t0 = time.perf_counter()
-        lay = oracle.layout([g], P, S)
-        N = lay.n_pad
-        E0 = np.zeros((N, H)); E0[: lay.n_real] = rng.standard_normal((lay.n_real, H))
-        e = (lay.kept_dst, lay.kept_src, lay.kept_type)
+    n_chunks = -(-len(order) // group)
+    for it in range(1 << 20):
+        i0 = (it % n_chunks) * group
+        chunk = [graphs[i] for i in order[i0:i0 + group]]
+        lay = oracle.layout(chunk, P, S, with_masks=False)
+        N, n_real = lay.n_pad, lay.n_real
+        d, s_, t_ = lay.kept_dst, lay.kept_src, lay.kept_type
+        if done_nodes == 0:  # before any measurement: about 1e9 multiply-adds per second
+            cap = int(budget_s * 1e9 * max(1, threads // 2) / (6.0 * T * (P + 6) * H * H))
+        else:
+            cap = int((budget_s - spent) / (spent / done_nodes))
+        cap = max(32, cap)
+        if n_real > cap:
+            keep = (d < cap) & (s_ < cap)
+            d, s_, t_ = d[keep], s_[keep], t_[keep]
+            N = n_real = cap
+            cut += 1
+        E0 = np.zeros((N, H)); E0[:n_real] = rng.standard_normal((n_real, H))
+        dY = rng.standard_normal((N, H))
+        e = (d, s_, t_)
         prm = synth.gen_params(P, H, 1, mean_in_degree=lay.n_kept / max(lay.n_real, 1))
-        if c["gru"]:
-            Es, Ys = oracle.ggnn_fwd(N, P, H, T, lay.n_real, *e, E0, prm)
-            oracle.ggnn_bwd(N, P, H, T, lay.n_real, *e, prm, Es, Ys, rng.standard_normal((N, H)))
+        t0 = time.perf_counter()
+        if c["gru"] and parallel:
+            Es, Ys = oracle.par_ggnn_fwd(N, P, H, T, n_real, *e, E0, prm, threads)
+            oracle.par_ggnn_bwd(N, P, H, T, n_real, *e, prm, Es, Ys, dY, threads)
+        elif c["gru"]:
+            Es, Ys = oracle.ggnn_fwd(N, P, H, T, n_real, *e, E0, prm)
+            oracle.ggnn_bwd(N, P, H, T, n_real, *e, prm, Es, Ys, dY)
+        elif parallel:
+            oracle.par_propagate_fwd(N, P, H, *e, E0, prm["W"], prm["b"], threads)
+            oracle.par_propagate_bwd(N, P, H, *e, E0, prm["W"], dY, threads)
         else:
             oracle.propagate_fwd(N, P, H, *e, E0, prm["W"], prm["b"])
-            oracle.propagate_bwd(N, P, H, *e, E0, prm["W"], rng.standard_normal((N, H)))
+            oracle.propagate_bwd(N, P, H, *e, E0, prm["W"], dY)
         spent += time.perf_counter() - t0
-        done_nodes += g.n_nodes
-        used += 1
-        if time.perf_counter() - t_start > budget_s:
+        done_nodes += n_real
+        used += len(chunk)
+        if spent > 0.95 * budget_s:
             break
-    return done_nodes * T / spent, {"graphs": used, "nodes": done_nodes, "seconds": spent}
+    value = done_nodes * T / spent
+    desc = {"graphs": used, "nodes": done_nodes, "seconds": spent, "threads": threads,
+            "kind": "parallel" if parallel else "single",
+            "text": (f"{'smallest' if smallest_first else 'leading'} graphs, {used} taken "
+                     + (f"({cut} cut to a prefix of band positions) " if cut else "")
+                     + f"({done_nodes} nodes) of the same workload, fwd+bwd, {spent:.1f}s of "
+                     + (f"pull-based fp64 on {threads} host threads" if parallel
+                        else "single-threaded fp64") + ", layout not timed")}
+    return value, desc
 
 
 # --------------------------------------------------------------------------------- main
 
 
+def fixed_config(name, graphs, c, world, n_packed, n_real, n_pad, K):
+    """The workload's identity, the same for both arms: what ran, not how fast."""
+    return {"workload": name, "graphs": len(graphs), "packed": n_packed, "n_real": n_real,
+            "n_pad": n_pad, "K": K, "S": c["S"], "P": c["P"], "H": c["H"], "T": c["T"],
+            "l2": "per-step working set (band tiles + saved activations) > 129 MB L2",
+            "parallelism": f"dp{world} (one supergraph per GPU"
+                           + (", gradient all-reduce)" if world > 1 else ")")}
+
+
 def run_reference(args):
+    """The reference arm: the fp64 CPU oracle as it stands, on the host cores, each step a bounded
+    sample of the same workload; its step time is the sample's measured time."""
     rank, world, _ = _dist()
     if rank != 0:
         return 0
-    from paper_1906_11786_gb300 import synth
+    import oracle
     graphs, c = workload(args.workload, 0, args.S, args.H)
-    n_real = sum(g.n_nodes for g in graphs)
-    times = []
-    # keep the whole run within a few minutes whatever K and W are
-    budget = max(0.5, min(args.ref_budget, 150.0 / max(1, args.warmup + args.steps)))
+    lay = oracle.layout(graphs, c["P"], c["S"], c["cap"], with_masks=False)
+    per_step = max(0.5, min(args.ref_budget, 150.0 / max(1, args.warmup + args.steps)))
+    secs, units, last = [], [], None
     for i in range(args.warmup + args.steps):
-        v, s = oracle_sample(args.workload, c, budget_s=budget)
+        v, s = oracle_sample(args.workload, c, budget_s=per_step, graphs=graphs)
         if i >= args.warmup:
-            times.append(v)
-    value = statistics.median(times)
+            secs.append(s["seconds"])
+            units.append(s["nodes"] * c["T"])
+            last = s
+    value = sum(units) / sum(secs)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "node-steps/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": n_real * c["T"] / value * 1e3, "higher_is_better": True,
+        "ms_per_step": 1e3 * sum(secs) / len(secs), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": args.workload, "S": c["S"], "H": c["H"],
-                   "P": c["P"], "T": c["T"]},
+        "config": fixed_config(args.workload, graphs, c, world, lay.n_packed, lay.n_real,
+                               lay.n_pad, lay.K),
         "cpu_baseline": {"value": value, "unit": "node-steps/s", "cores": 1, "kind": "oracle",
-                         "sample": f"leading graphs of the batch per step, ~{budget:.1f}s "
-                                   f"of single-threaded fp64 work ({s['graphs']} graphs, "
-                                   f"{s['nodes']} nodes)"},
+                         "sample": f"per step: {last['text']} (about {per_step:.1f}s); "
+                                   f"ms_per_step is the sample's measured time, value the "
+                                   f"sample's node-steps over it"},
         "e2e": {"value": value, "unit": "node-steps/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -478,6 +547,155 @@ def run_op(args, st, c):
     return 0
 
 
+KNAMES = ["band_fwd", "band_bwd", "gru_fwd", "gru_bwd", "dW"]
+
+
+def roofline(L, st, c, kt, pk, workload_name):
+    """Roofline of the dominant band kernel (the one with the larger share of the step): its
+    algorithmic FLOPs per launch (band-dense contraction plus the fused edge-type transform chain)
+    over its average CUDA-event duration.  Tensor-core kernels against the measured bf16 peak
+    (burst; the sustained fraction beside it); the fp32 SIMT path against the fp32 FMA rate of the
+    SMs (an ALU bound: 128 lanes x 2 FLOP x SMs x the measured maximum SM clock)."""
+    import torch
+    H = c["H"]
+    fwd_ms, fwd_n = kt[L.BG_KID_BAND_FWD]
+    bwd_ms, bwd_n = kt[L.BG_KID_BAND_BWD]
+    kern = "band_fwd" if fwd_ms >= bwd_ms else "band_bwd"
+    avg_ms = (fwd_ms / max(fwd_n, 1)) if kern == "band_fwd" else (bwd_ms / max(bwd_n, 1))
+    flops = st.plan.flops(H, L.BG_FLOPS_BAND) + st.plan.flops(H, L.BG_FLOPS_XFORM)
+    achieved = flops / (avg_ms / 1e3) / 1e12 if avg_ms > 0 else 0.0
+    tc = L.band_uses_tensor_cores(st.plan, c["dtype"], H)
+    if tc:
+        bound, peak = "tensor", pk["bf16"]
+        peak_src = f"{pk['src']} bf16 burst (kernel timed per launch)"
+    else:
+        sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+        bound, peak = "alu", sms * 128 * 2 * pk["sm_max_mhz"] * 1e6 / 1e12
+        peak_src = f"fp32 FMA rate: {sms} SMs x 128 lanes x 2 FLOP x {pk['sm_max_mhz']:.0f} MHz"
+    traffic = _profiled_traffic(kern.split("_")[1], workload_name) if tc else None
+    roof = {"kernel": kern, "bound": bound, "achieved": achieved, "peak": peak,
+            "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
+            "traffic_src": "profiles/ ncu capture (dram read+write bytes per launch)"
+            if traffic else None, "peak_src": peak_src,
+            "kernel_ms": {k: (kt[i][0] / max(kt[i][1], 1)) for i, k in enumerate(KNAMES)},
+            "nnz_tflops": st.plan.flops(H, L.BG_FLOPS_NNZ) / (avg_ms / 1e3) / 1e12
+            if avg_ms > 0 else 0.0}
+    if tc:
+        roof["frac_sustained"] = achieved / pk["bf16_sustained"]
+    return roof
+
+
+def measure(L, graphs, c, name, steps, warmup, prof_min_s, e2e_steps, dist=None, rank=0,
+            clocks=None):
+    """Plans and runs one workload: W warm-up steps, then exactly `steps` timed steps (CUDA events
+    on the stream, no per-launch events), then a profiled pass of the same steps with per-kernel
+    CUDA events lasting at least prof_min_s, then the end-to-end run with host buffers."""
+    import torch
+    st = OursStep(graphs, c, seed=rank, dist=dist)
+    units = st.n_real * c["T"]
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    for _ in range(max(warmup, 3)):
+        st.step()
+    torch.cuda.synchronize()
+    L.check_device()
+    launches0 = L.launch_count()
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if clocks is not None:
+        clocks.mark("timed_start")
+    barrier()
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for _ in range(steps):
+        st.step()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    if clocks is not None:
+        clocks.mark("timed_end")
+    launches = L.launch_count() - launches0
+    ms = ev0.elapsed_time(ev1)
+    L.check_device()
+    # per-kernel durations: CUDA events around every launch, on its stream
+    for k in range(len(KNAMES)):
+        L.profile_read(k, reset=True)
+    L.profile_enable(True)
+    t0, prof_steps = time.perf_counter(), 0
+    while prof_steps < min(steps, 20) or time.perf_counter() - t0 < prof_min_s:
+        st.step()
+        prof_steps += 1
+        if prof_steps % 10 == 0:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
+    prof_s = time.perf_counter() - t0
+    L.profile_enable(False)
+    L.check_device()
+    kt = {k: L.profile_read(k, reset=True) for k in range(len(KNAMES))}
+    ms, total_units = reduce_over_ranks(dist, ms, float(units))
+    ms_step = ms / steps
+    st.e2e_run(2, stream)
+    barrier()
+    e_ms, bi, bo = st.e2e_run(e2e_steps, stream)
+    e_ms, _ = reduce_over_ranks(dist, e_ms, 0.0)
+    return {"st": st, "ms_step": ms_step, "value": total_units / (ms_step / 1e3),
+            "units": total_units, "launches": launches, "kt": kt, "prof_steps": prof_steps,
+            "prof_s": prof_s, "e2e": {"value": total_units / (e_ms / 1e3), "unit": "node-steps/s",
+                                      "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo}}
+
+
+# workloads of the sweep beside the headline (the configurations of the workload list that the
+# headline does not cover): (name, S, H)
+SWEEP = ([("single512", None, None), ("single20k", None, None)] +
+         [("sweep131k", s, None) for s in (32, 64, 128, 256, 512)] +
+         [("train100k", None, h) for h in (32, 64, 128, 256)])
+
+
+def sweep_rows(L, args, pk, budget_s):
+    """Every other workload of the list at a short fixed length: node-steps/s, end-to-end, the
+    band kernel's roofline fraction and the oracle on the host cores (single-threaded, and for the
+    three large workloads the multi-threaded variant too)."""
+    import torch
+    rows = []
+    t_all = time.perf_counter()
+    for name, S, H in SWEEP:
+        if time.perf_counter() - t_all > budget_s:
+            rows.append({"workload": name, "S": S, "H": H, "skipped": "sweep time budget spent"})
+            continue
+        t_row = time.perf_counter()
+        graphs, c = workload(name, 0, S, H)
+        m = measure(L, graphs, c, name, steps=10, warmup=3, prof_min_s=0.3, e2e_steps=5)
+        t_gpu = time.perf_counter() - t_row
+        st = m["st"]
+        roof = roofline(L, st, c, m["kt"], pk, name)
+        row = {"workload": name, "S": c["S"], "H": c["H"], "T": c["T"], "P": c["P"],
+               "dtype": c["dtype"], "n_real": st.n_real, "n_pad": st.N, "value": m["value"],
+               "ms_per_step": m["ms_step"], "e2e": m["e2e"]["value"],
+               "band_kernels": "tcgen05" if L.band_uses_tensor_cores(st.plan, c["dtype"], c["H"])
+               else "simt",
+               "roofline": {k: roof[k] for k in ("kernel", "bound", "achieved", "peak", "frac")},
+               "kernel_ms": roof["kernel_ms"],
+               "nnz_over_band_dense": st.plan.flops(c["H"], L.BG_FLOPS_NNZ) /
+               max(st.plan.flops(c["H"], L.BG_FLOPS_BAND), 1.0),
+               "dropped_edges": st.info["n_dropped"], "kept_edges": st.info["n_kept"]}
+        del m, st
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+        wide = c["H"] >= 128 and c["gru"]
+        v, s = oracle_sample(name, c, budget_s=2.0, smallest_first=wide, graphs=graphs)
+        row["cpu_oracle"] = {"value": v, "cores": 1, "sample": s["text"]}
+        if name in ("single20k", "sweep131k", "train100k"):
+            v, s = oracle_sample(name, c, budget_s=2.0, parallel=True, smallest_first=wide,
+                                 graphs=graphs)
+            row["cpu_oracle_parallel"] = {"value": v, "cores": s["threads"], "sample": s["text"]}
+        row["seconds"] = {"plan_and_gpu": t_gpu, "total": time.perf_counter() - t_row}
+        rows.append(row)
+    return rows
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -495,7 +713,13 @@ def main():
     ap.add_argument("--H", type=int, default=None)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true",
+                    help="skip the sweep over the other workloads (run at N = 1 on rank 0 only)")
+    ap.add_argument("--sweep-budget", type=float, default=180.0,
+                    help="seconds after which the sweep skips its remaining workloads")
     ap.add_argument("--ref-budget", type=float, default=15.0)
+    ap.add_argument("--prof-seconds", type=float, default=2.0,
+                    help="minimum length of the profiled pass that times every kernel launch")
     ap.add_argument("--op", default="step", choices=["step", "band_fwd", "band_bwd"],
                     help="time one band propagation kernel call instead of the whole step "
                          "(focused profiling of the same workload)")
@@ -517,117 +741,43 @@ def main():
     from paper_1906_11786_gb300 import _binding as L
 
     graphs, c = workload(args.workload, rank, args.S, args.H)
-    st = OursStep(graphs, c, seed=rank, dist=dist)
-    H, T = c["H"], c["T"]
-    units = st.n_real * T  # node-steps per step on this rank
     if args.op != "step":
-        return run_op(args, st, c)
+        return run_op(args, OursStep(graphs, c, seed=rank, dist=dist), c)
 
-    def barrier():
-        if dist is not None:
-            dist.barrier()
-
-    for _ in range(max(args.warmup, 3)):
-        st.step()
-    torch.cuda.synchronize()
-    L.check_device()
-
-    # ---- timed region: device-resident inputs, no per-launch events (a timing event between two
-    # launches waits for the first to drain and exposes the next one's launch latency: +6% here)
-    launches0 = L.launch_count()
-    stream = torch.cuda.current_stream()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with Clocks(local) as clk:
-        barrier()
-        torch.cuda.synchronize()
-        ev0.record(stream)
-        for _ in range(args.steps):
-            st.step()
-        ev1.record(stream)
-        torch.cuda.synchronize()
-        barrier()
-    launches = L.launch_count() - launches0
-    ms = ev0.elapsed_time(ev1)
-    L.check_device()
-
-    # ---- per-kernel durations: CUDA events around every launch, on its stream, in a profiled pass
-    # of the same steps right after the timed region (same process, buffers and launches)
-    prof_steps = min(args.steps, 20)
-    for k in range(5):
-        L.profile_read(k, reset=True)
-    L.profile_enable(True)
-    for _ in range(prof_steps):
-        st.step()
-    torch.cuda.synchronize()
-    L.profile_enable(False)
-    L.check_device()
-    kt = {k: L.profile_read(k, reset=True) for k in range(5)}
-    ms, total_units = reduce_over_ranks(dist, ms, float(units))
-    ms_step = ms / args.steps
-    value = total_units / (ms_step / 1e3)
-
-    # ---- e2e: host buffers, H2D + pack + step + unpack + D2H inside the timed region
-    st.e2e_run(2, stream)
-    barrier()
-    e_ms, bi, bo = st.e2e_run(args.steps, stream)
-    e_ms, _ = reduce_over_ranks(dist, e_ms, 0.0)
-    e2e_value = total_units / (e_ms / 1e3)
-
-    # ---- roofline of the dominant kernel (band contraction)
     pk = _peaks()
-    fwd_ms, fwd_n = kt[L.BG_KID_BAND_FWD]
-    bwd_ms, bwd_n = kt[L.BG_KID_BAND_BWD]
-    f_band = st.plan.flops(H, L.BG_FLOPS_BAND)
-    f_xf = st.plan.flops(H, L.BG_FLOPS_XFORM)
-    # algorithmic FLOPs per launch of either band kernel: band-dense contraction plus the fused
-    # edge-type transform chain (forward: pre_p W_p; backward: dM_p W_p^T)
-    flops = f_band + f_xf
-    kern = "band_fwd" if fwd_ms >= bwd_ms else "band_bwd"
-    avg_ms = (fwd_ms / max(fwd_n, 1)) if kern == "band_fwd" else (bwd_ms / max(bwd_n, 1))
-    achieved = flops / (avg_ms / 1e3) / 1e12 if avg_ms > 0 else 0.0
-    peak = pk["bf16_sustained"]
-    traffic = _profiled_traffic(kern.split("_")[1], args.workload)
-    roof = {"kernel": kern, "bound": "tensor", "achieved": achieved, "peak": peak,
-            "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
-            "traffic_src": "profiles/ ncu capture (dram read+write bytes per launch)"
-            if traffic else None,
-            "peak_src": f"{pk['src']} bf16 sustained",
-            "kernel_ms": {k: (kt[i][0] / max(kt[i][1], 1)) for i, k in
-                          enumerate(["band_fwd", "band_bwd", "gru_fwd", "gru_bwd", "dW"])},
-            "kernel_timing": f"CUDA events around every launch on its stream, in a profiled pass "
-                             f"of {prof_steps} steps right after the timed region",
-            "nnz_tflops": st.plan.flops(H, L.BG_FLOPS_NNZ) / (avg_ms / 1e3) / 1e12
-            if avg_ms > 0 else 0.0}
-
+    with Clocks(local) as clk:
+        m = measure(L, graphs, c, args.workload, args.steps, args.warmup, args.prof_seconds,
+                    args.steps, dist=dist, rank=rank, clocks=clk)
+    st = m["st"]
+    roof = roofline(L, st, c, m["kt"], pk, args.workload)
+    roof["kernel_timing"] = (f"CUDA events around every launch on its stream, in a profiled pass "
+                             f"of {m['prof_steps']} steps ({m['prof_s']:.1f}s) right after the "
+                             f"timed region")
     line = {
-        "metric": METRIC, "value": value, "unit": "node-steps/s", "n_gpus": world,
-        "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms_step,
+        "metric": METRIC, "value": m["value"], "unit": "node-steps/s", "n_gpus": world,
+        "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": m["ms_step"],
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": c["dtype"], "data": "synthetic program-shaped graphs (seeded)",
-        "config": {"workload": args.workload, "graphs": len(graphs),
-                   "packed": st.info["n_packed"], "n_real": st.n_real, "n_pad": st.N,
-                   "K": st.info["K"], "S": c["S"], "P": c["P"], "H": H, "T": T,
-                   "kept_edges": st.info["n_kept"], "dropped_edges": st.info["n_dropped"],
-                   "plan_ms": st.plan_ms, "upload_ms": st.upload_ms,
-                   "flops_per_pass": _flops(L, st.plan, H),
-                   "band_kernels": "tcgen05" if L.band_uses_tensor_cores(st.plan, c["dtype"], H)
-                   else "simt",
-                   "l2": "per-step working set (band tiles + saved activations) > 129 MB L2",
-                   "parallelism": f"dp{world} (one supergraph per GPU"
-                                  + (", gradient all-reduce)" if world > 1 else ")")},
-        "e2e": {"value": e2e_value, "unit": "node-steps/s", "h2d_bytes_per_step": bi,
-                "d2h_bytes_per_step": bo},
-        "gpu_launches": launches,
+        "config": fixed_config(args.workload, graphs, c, world, st.info["n_packed"], st.n_real,
+                               st.N, st.info["K"]),
+        "plan": {"kept_edges": st.info["n_kept"], "dropped_edges": st.info["n_dropped"],
+                 "plan_ms": st.plan_ms, "upload_ms": st.upload_ms,
+                 "flops_per_pass": _flops(L, st.plan, c["H"]),
+                 "band_kernels": "tcgen05" if L.band_uses_tensor_cores(st.plan, c["dtype"], c["H"])
+                 else "simt"},
+        "e2e": m["e2e"],
+        "gpu_launches": m["launches"],
         "roofline": roof,
         "clocks": clk.summary(),
     }
+    del m, st
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, s = oracle_sample(args.workload, c)
+        v, s = oracle_sample(args.workload, c, graphs=graphs)
         line["cpu_baseline"] = {"value": v, "unit": "node-steps/s", "cores": 1, "kind": "oracle",
-                                "sample": f"leading {s['graphs']} graphs ({s['nodes']} nodes) of "
-                                          f"the same workload, fwd+bwd, {s['seconds']:.1f}s "
-                                          "single-threaded fp64",
-                                "host": _host()}
+                                "sample": s["text"], "host": _host()}
+    if rank == 0 and world == 1 and not args.no_sweep:
+        torch.cuda.empty_cache()
+        line["sweep"] = sweep_rows(L, args, pk, args.sweep_budget)
     if rank == 0:
         print(json.dumps(line))
     if dist is not None:
