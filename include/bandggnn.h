@@ -95,6 +95,18 @@ int bg_band_plan(const bg_graph* graphs, int32_t n_graphs, int32_t n_types, int3
 void bg_plan_free(bg_plan* plan); /* frees host and device memory of the plan; NULL is a no-op */
 int bg_plan_info(const bg_plan* plan, bg_info* out);
 
+/* Reachability preprocessing (Section 4 "Reachability preprocessing"), host only: with T
+ * propagation steps, only nodes from which some candidate node is reachable along at most T edges
+ * (any types, in edge direction) can change the candidates' final states; the others are dropped.
+ * g: the input graph; cand [n_cand]: candidate node ids.  Writes node_map [g->n_nodes] (new id of
+ * a kept node -- kept nodes keep their relative order -- or -1), *n_nodes_out (kept nodes),
+ * *n_edges_out (kept edges: both ends kept) and, where the arrays are non-NULL (capacity
+ * g->n_edges each), the kept edges renumbered, in input order.  Candidates are always kept; T = 0
+ * keeps only them.  Errors: BG_EINVAL (ids out of range, NULL arrays, negative T). */
+int bg_reach_filter(const bg_graph* g, const int32_t* cand, int32_t n_cand, int32_t T,
+                    int32_t* node_map, int32_t* n_nodes_out, int64_t* n_edges_out,
+                    int32_t* src_out, int32_t* dst_out, int32_t* etype_out);
+
 /* FLOPs of one forward propagation pass at state size H (the backward pass has the same band
  * and twice the transform FLOPs).  which: */
 #define BG_FLOPS_BAND 0  /* band-dense: 2 (3K-2) P S^2 H (all tiles of Eq. 3 as dense products) */

@@ -56,6 +56,8 @@ def _load():
     lib.orc_bandwidth.argtypes = [c.c_int32, c.c_int64, _i32p, _i32p, c.c_void_p]
     lib.orc_rcm.restype = c.c_int
     lib.orc_rcm.argtypes = [c.c_int32, c.c_int64, _i32p, _i32p, c.c_int, _i32p]
+    lib.orc_reach.restype = c.c_int32
+    lib.orc_reach.argtypes = [c.c_int32, c.c_int64, _i32p, _i32p, _i32p, c.c_int32, c.c_int32, _u8p]
     lib.orc_num_blocks.restype = c.c_int32
     lib.orc_num_blocks.argtypes = [c.c_int32, _i32p, c.c_int32, c.c_int32]
     lib.orc_layout.restype = c.c_int
@@ -130,6 +132,28 @@ def rcm(n, src, dst, keep_if_better=True) -> np.ndarray:
     if lib.orc_rcm(n, src.shape[0], src, dst, int(bool(keep_if_better)), perm):
         raise ValueError("invalid graph")
     return perm
+
+
+def reach(n, src, dst, candidates, T) -> np.ndarray:
+    """Reachability preprocessing (Section 4): bool [n], True for nodes from which a candidate is
+    reachable along at most T edges."""
+    lib = _load()
+    keep = np.zeros(n, np.uint8)
+    src, dst, cand = _i32(src), _i32(dst), _i32(candidates)
+    if lib.orc_reach(n, src.shape[0], src, dst, cand, cand.shape[0], T, keep) < 0:
+        raise ValueError("invalid graph or candidates")
+    return keep.astype(bool)
+
+
+def reach_filter(graph, candidates, T):
+    """The graph reduced to its kept nodes (renumbered in ascending old id) and the edges between
+    them (input order): (node_map [n] new id or -1, n_kept, src, dst, etype)."""
+    keep = reach(graph.n_nodes, graph.src, graph.dst, candidates, T)
+    node_map = np.full(graph.n_nodes, -1, np.int32)
+    node_map[keep] = np.arange(int(keep.sum()), dtype=np.int32)
+    ek = keep[graph.src] & keep[graph.dst]
+    return (node_map, int(keep.sum()), node_map[graph.src[ek]], node_map[graph.dst[ek]],
+            np.asarray(graph.etype)[ek].astype(np.int32))
 
 
 FLAG_RCM = 1

@@ -152,6 +152,35 @@ int orc_rcm(int32_t n, int64_t m, const int32_t* src, const int32_t* dst, int ke
   return 0;
 }
 
+// Reachability preprocessing (Section 4 "Reachability preprocessing"): with T propagation steps
+// only nodes from which some candidate node is reachable along at most T edges affect the
+// candidates' final states, so the others are discarded.  Written as the definition: R_0 = the
+// candidates; R_k = R_{k-1} plus every source u of an edge u -> v with v in R_{k-1}; keep R_T.
+// keep[v] = 1 for kept nodes.  Returns the number kept, or -1 on invalid input.
+int32_t orc_reach(int32_t n, int64_t m, const int32_t* src, const int32_t* dst,
+                  const int32_t* cand, int32_t n_cand, int32_t T, uint8_t* keep) {
+  if (n < 0 || m < 0 || n_cand < 0 || T < 0) return -1;
+  for (int64_t e = 0; e < m; ++e)
+    if (src[e] < 0 || src[e] >= n || dst[e] < 0 || dst[e] >= n) return -1;
+  std::vector<uint8_t> in(n, 0);
+  for (int32_t i = 0; i < n_cand; ++i) {
+    if (cand[i] < 0 || cand[i] >= n) return -1;
+    in[cand[i]] = 1;
+  }
+  for (int32_t k = 1; k <= T; ++k) {
+    std::vector<uint8_t> next(in);
+    for (int64_t e = 0; e < m; ++e)
+      if (in[dst[e]]) next[src[e]] = 1;
+    in.swap(next);
+  }
+  int32_t kept = 0;
+  for (int32_t v = 0; v < n; ++v) {
+    keep[v] = in[v];
+    kept += in[v];
+  }
+  return kept;
+}
+
 // Number of blocks K the supergraph gets: capacity_blocks, or ceil(sum n / S) when 0.
 int32_t orc_num_blocks(int32_t n_graphs, const int32_t* n_nodes, int32_t S, int32_t capacity_blocks) {
   if (capacity_blocks > 0) return capacity_blocks;

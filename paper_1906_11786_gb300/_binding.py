@@ -98,6 +98,7 @@ def load(path: str = LIB_PATH):
         "bg_profile_read": (c.c_int, [i32, vp, vp, i32]),
         "bg_launch_count": (i64, []),
         "bg_band_uses_tensor_cores": (c.c_int, [vp, c.c_int, i32]),
+        "bg_reach_filter": (c.c_int, [vp, vp, i32, i32, vp, vp, vp, vp, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -225,6 +226,25 @@ def band_plan(graphs, n_types, block_S, capacity_blocks=0, flags=BG_RCM | BG_KEE
     _check(lib.bg_band_plan(arr, len(graphs), n_types, block_S, capacity_blocks, flags,
                             ctypes.byref(h)))
     return Plan(h.value, n_types)
+
+
+def reach_filter(graph, candidates, T):
+    """bg_reach_filter: (node_map [n] new id or -1, n_kept, src, dst, etype) of the graph reduced
+    to the nodes that reach a candidate within T steps."""
+    lib = load()
+    s = np.ascontiguousarray(graph.src, np.int32)
+    d = np.ascontiguousarray(graph.dst, np.int32)
+    t = np.ascontiguousarray(graph.etype, np.int32)
+    cand = np.ascontiguousarray(candidates, np.int32)
+    g = bg_graph(int(graph.n_nodes), int(s.shape[0]), s.ctypes.data, d.ctypes.data, t.ctypes.data)
+    node_map = np.zeros(max(graph.n_nodes, 1), np.int32)
+    so, do, to = (np.zeros(max(s.shape[0], 1), np.int32) for _ in range(3))
+    nn, ne = ctypes.c_int32(), ctypes.c_int64()
+    _check(lib.bg_reach_filter(ctypes.byref(g), cand.ctypes.data, cand.shape[0], T,
+                               node_map.ctypes.data, ctypes.byref(nn), ctypes.byref(ne),
+                               so.ctypes.data, do.ctypes.data, to.ctypes.data))
+    m = ne.value
+    return node_map[:graph.n_nodes], nn.value, so[:m].copy(), do[:m].copy(), to[:m].copy()
 
 
 # --------------------------------------------------------------------------------- device calls

@@ -18,7 +18,7 @@ import numpy as np
 
 __all__ = [
     "Graph", "gen_graph", "gen_batch", "gen_states", "gen_params", "WORKLOADS", "workload_graphs",
-    "graph_seed", "hub_graph", "with_self_loops",
+    "graph_seed", "hub_graph", "with_self_loops", "gen_candidates",
 ]
 
 
@@ -202,6 +202,13 @@ def with_self_loops(g: Graph, frac: float, n_types: int, seed: int) -> Graph:
     t = rng.integers(0, n_types, size=k).astype(np.int32)
     return Graph(g.n_nodes, np.concatenate([g.src, u]), np.concatenate([g.dst, u]),
                  np.concatenate([g.etype, t]), max(g.n_types, n_types), dict(g.meta))
+
+
+def gen_candidates(g: Graph, k: int, seed: int) -> np.ndarray:
+    """k distinct candidate nodes of `g` drawn uniformly (the synthetic stand-in for the
+    VarMisuse hole's type-correct in-scope variables, Section 4 "Data"), ascending."""
+    rng = np.random.default_rng(seed)
+    return np.sort(rng.choice(g.n_nodes, size=min(k, g.n_nodes), replace=False)).astype(np.int32)
 
 
 def gen_states(n: int, H: int, seed: int) -> np.ndarray:

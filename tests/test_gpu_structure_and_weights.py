@@ -147,3 +147,59 @@ def test_self_loops(dtype, S, H):
     assert L.band_uses_tensor_cores(c.plan, dtype, H) == (dtype == "bf16")
     _check_propagation(c, 93)
     _ggnn_check(c, 2, 95)
+
+
+# ------------------------------------------------------------------------ reachability
+
+
+def test_reach_filtered_batch_gives_the_full_graphs_candidate_states():
+    """Reachability preprocessing (Section 4) in front of the whole GPU path: each graph is cut
+    to the nodes that reach one of its seeded candidates within T = 8 steps (bg_reach_filter),
+    the reduced graphs are planned, packed and run through T = 8 GGNN steps on the tensor-core
+    path, and the candidates' states E(T) match the oracle's exact sparse GGNN on the full,
+    unreduced graphs (nothing is dropped by the band cover here, so both sides see every edge)."""
+    T, P, S, H = 8, 20, 128, 64
+    gs = synth.gen_batch(10, 300, 1500, 10, True, 24, 24, 3.0, 1234)
+    cands = [synth.gen_candidates(g, 5, 40 + i) for i, g in enumerate(gs)]
+    red, maps = [], []
+    for g, cand in zip(gs, cands):
+        node_map, nk, s2, d2, t2 = L.reach_filter(g, cand, T)
+        red.append(synth.Graph(nk, s2, d2, t2, P))
+        maps.append(node_map)
+    assert sum(r.n_nodes for r in red) < sum(g.n_nodes for g in gs)
+    plan = L.band_plan(red, P, S)
+    plan.upload()
+    info = plan.info()
+    assert info["n_dropped"] == 0 and info["n_packed"] == len(red)
+    assert L.band_uses_tensor_cores(plan, "bf16", H)
+    N = info["n_pad"]
+    full_E = [quantize(synth.gen_states(g.n_nodes, H, 70 + i), "bf16") for i, g in enumerate(gs)]
+    E_red = np.concatenate([E[m >= 0] for E, m in zip(full_E, maps)])
+    prm = synth.gen_params(P, H, 71, mean_in_degree=info["n_kept"] / info["n_real"])
+    for k in ("W", "W_ih", "W_hh"):
+        prm[k] = quantize(prm[k], "bf16")
+    for k in ("b", "b_ih", "b_hh"):
+        prm[k] = quantize(prm[k], "f32")
+    dprm = {k: (torch.from_numpy(np.asarray(v, np.float32)).to(torch.bfloat16).cuda()
+                if k in ("W", "W_ih", "W_hh") else f32_dev(v)) for k, v in prm.items()}
+    E0 = torch.empty((N, H), dtype=torch.bfloat16, device="cuda")
+    L.pack_states(plan, "bf16", H, torch.from_numpy(E_red.astype(np.float32)).to(torch.bfloat16)
+                  .cuda(), E0)
+    saved = torch.empty(L.ggnn_saved_bytes(plan, "bf16", H, T), dtype=torch.uint8, device="cuda")
+    ws = torch.empty(L.ggnn_workspace_bytes(plan, "bf16", H, T, L.BG_OP_GGNN_FWD),
+                     dtype=torch.uint8, device="cuda")
+    ET = torch.empty_like(E0)
+    L.ggnn_step(plan, "bf16", H, T, dprm, E0, ET, saved, ws)
+    ET_red = torch.empty((E_red.shape[0], H), dtype=torch.bfloat16, device="cuda")
+    L.unpack_states(plan, "bf16", H, ET, ET_red)
+    torch.cuda.synchronize()
+    L.check_device()
+    got = ET_red.float().cpu().numpy()
+    off = np.concatenate([[0], np.cumsum([r.n_nodes for r in red])])
+    got_c, want_c = [], []
+    for i, (g, cand, m) in enumerate(zip(gs, cands, maps)):
+        Es, _ = oracle.ggnn_fwd(g.n_nodes, P, H, T, g.n_nodes, g.dst, g.src, g.etype, full_E[i],
+                                prm)
+        got_c.append(got[off[i] + m[cand]])
+        want_c.append(Es[T][cand])
+    assert_close(np.concatenate(got_c), np.concatenate(want_c), TOL["bf16"], "E(T) at candidates")

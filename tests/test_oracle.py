@@ -471,3 +471,62 @@ def test_parallel_oracle_equals_the_oracle_to_the_last_bit():
     for k in r:
         np.testing.assert_array_equal(r2[k], r[k], err_msg=k)
     assert oracle.par_max_threads() >= 1
+
+
+# ------------------------------------------------------------------------ reachability (Section 4)
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2, 3])
+def test_reach_matches_all_pairs_shortest_paths(seed):
+    """Brute force: directed shortest-path lengths by Floyd-Warshall on a small random graph; a
+    node is kept iff its distance to the nearest candidate is at most T."""
+    rng = np.random.default_rng(seed)
+    n = 25
+    m = 45
+    src = rng.integers(0, n, m).astype(np.int32)
+    dst = rng.integers(0, n, m).astype(np.int32)
+    cand = np.unique(rng.integers(0, n, 3)).astype(np.int32)
+    D = np.full((n, n), np.inf)
+    np.fill_diagonal(D, 0)
+    D[src, dst] = np.minimum(D[src, dst], 1)
+    for k in range(n):
+        D = np.minimum(D, D[:, [k]] + D[[k], :])
+    for T in (0, 1, 2, 3, 6):
+        want = D[:, cand].min(axis=1) <= T
+        np.testing.assert_array_equal(oracle.reach(n, src, dst, cand, T), want)
+
+
+def test_reach_on_a_chain_keeps_the_last_T_plus_one_nodes():
+    """Chain 0 -> 1 -> ... -> n-1 with the last node the only candidate: exactly the T + 1 nodes
+    n-1-T .. n-1 reach it within T steps; reversing the edges keeps only the candidate's
+    successors-side nodes (none here)."""
+    n = 40
+    src = np.arange(n - 1, dtype=np.int32)
+    dst = src + 1
+    for T in (0, 1, 5, 8):
+        keep = oracle.reach(n, src, dst, [n - 1], T)
+        assert keep.sum() == T + 1 and keep[n - 1 - T:].all()
+        rev = oracle.reach(n, dst, src, [n - 1], T)
+        assert rev.sum() == 1 and rev[n - 1]
+
+
+def test_reach_filter_leaves_candidate_states_unchanged():
+    """The reason the preprocessing is lossless (Section 4): after T GGNN steps the candidates'
+    states on the reduced graph equal those on the full graph (fp64, up to summation order)."""
+    g = synth.gen_graph(300, 4, True, 12, 8, 1.0, 21)
+    cand = synth.gen_candidates(g, 4, 5)
+    T, H, P = 3, 8, 8
+    node_map, nk, s2, d2, t2 = oracle.reach_filter(g, cand, T)
+    assert 0 < nk < g.n_nodes
+    prm = synth.gen_params(P, H, 6)
+    E = synth.gen_states(g.n_nodes, H, 7)
+    Es, _ = oracle.ggnn_fwd(g.n_nodes, P, H, T, g.n_nodes, g.dst, g.src, g.etype, E, prm)
+    keep = node_map >= 0
+    Er, _ = oracle.ggnn_fwd(nk, P, H, T, nk, d2, s2, t2, E[keep], prm)
+    np.testing.assert_allclose(Er[T][node_map[cand]], Es[T][cand], rtol=1e-12, atol=1e-12)
+    # and a node the preprocessing dropped would have changed nothing: perturbing it leaves the
+    # candidates' final states as they were
+    dropped = np.flatnonzero(~keep)[0]
+    E2 = E.copy(); E2[dropped] += 10.0
+    Es2, _ = oracle.ggnn_fwd(g.n_nodes, P, H, T, g.n_nodes, g.dst, g.src, g.etype, E2, prm)
+    np.testing.assert_array_equal(Es2[T][cand], Es[T][cand])

@@ -261,3 +261,19 @@ def test_tensor_core_upload_layout_from_the_bit_tiles(S, hub, tmp_path_factory, 
     np.testing.assert_array_equal(deg.reshape(N, 64), exp_deg)
     assert max_deg == cnt.max()
     assert (max_deg > 256) == bool(hub)
+
+
+@pytest.mark.parametrize("T", [0, 1, 3, 8])
+def test_reach_filter_bit_exact_against_the_oracle(T):
+    """Reachability preprocessing (Section 4): the library's kept nodes, renumbering and kept
+    edges equal the oracle's, on program-shaped graphs with seeded candidates, at several T."""
+    for i, g in enumerate(synth.gen_batch(6, 50, 1500, 10, True, 96, 64, 3.0, 77 + T)):
+        cand = synth.gen_candidates(g, 5, 100 + i)
+        got = L.reach_filter(g, cand, T)
+        want = oracle.reach_filter(g, cand, T)
+        np.testing.assert_array_equal(got[0], want[0])
+        assert got[1] == want[1]
+        for a, b in zip(got[2:], want[2:]):
+            np.testing.assert_array_equal(a, b)
+    with pytest.raises(L.BandGGNNError):
+        L.reach_filter(g, [g.n_nodes], T)
