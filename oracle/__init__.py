@@ -63,7 +63,8 @@ def _load():
     lib.orc_layout.restype = c.c_int
     lib.orc_layout.argtypes = [c.c_int32, _i32p, _i64p, _i32p, _i32p, _i32p, c.c_int32, c.c_int32,
                                c.c_int32, c.c_int32, _i32p, _i32p, _i64p, c.c_void_p, c.c_void_p,
-                               c.c_void_p, c.c_void_p, _i64p, _i64p]
+                               c.c_void_p, c.c_void_p, _i64p, _i64p, c.c_int32, c.c_int32,
+                               c.c_void_p, c.c_void_p]
     lib.orc_propagate_fwd.restype = None
     lib.orc_propagate_fwd.argtypes = [c.c_int32] * 3 + [c.c_int64, _i32p, _i32p, _i32p, _f64p,
                                                          _f64p, c.c_void_p, _f64p]
@@ -158,6 +159,7 @@ def reach_filter(graph, candidates, T):
 
 FLAG_RCM = 1
 FLAG_KEEP_IF_BETTER = 2
+FLAG_SUPERNODES = 4
 
 
 @dataclass
@@ -181,6 +183,8 @@ class Layout:
     bw_before: np.ndarray
     bw_after: np.ndarray
     n_nodes: np.ndarray
+    kept_super: np.ndarray = None  # bool per kept edge: has a supernode end
+    is_super: np.ndarray = None    # bool per position: a supernode
 
     @property
     def n_pad(self) -> int:
@@ -205,8 +209,10 @@ class Layout:
 
 
 def layout(graphs, P, S, capacity_blocks=0, flags=FLAG_RCM | FLAG_KEEP_IF_BETTER,
-           with_masks=True) -> Layout:
-    """Supergraph layout of `graphs` (objects with n_nodes, src, dst, etype)."""
+           with_masks=True, super_min_degree=0, max_super=0) -> Layout:
+    """Supergraph layout of `graphs` (objects with n_nodes, src, dst, etype); with
+    FLAG_SUPERNODES, nodes of at least super_min_degree distinct neighbours (at most max_super per
+    graph) become supernodes."""
     lib = _load()
     n_nodes = _i32([g.n_nodes for g in graphs])
     counts = np.array([g.n_edges for g in graphs], np.int64)
@@ -223,9 +229,12 @@ def layout(graphs, P, S, capacity_blocks=0, flags=FLAG_RCM | FLAG_KEEP_IF_BETTER
     kd, ks, kt = (np.zeros(max(m, 1), np.int32) for _ in range(3))
     bwb = np.zeros(len(graphs), np.int64)
     bwa = np.zeros(len(graphs), np.int64)
+    ksup = np.zeros(max(m, 1), np.uint8)
+    isup = np.zeros(max(K * S, 1), np.uint8)
     vp = lambda a: None if a is None else a.ctypes.data_as(ctypes.c_void_p)  # noqa: E731
     rc = lib.orc_layout(len(graphs), n_nodes, edge_off, src, dst, et, P, S, capacity_blocks, flags,
-                        perm, offset, info, vp(masks), vp(kd), vp(ks), vp(kt), bwb, bwa)
+                        perm, offset, info, vp(masks), vp(kd), vp(ks), vp(kt), bwb, bwa,
+                        super_min_degree, max_super, vp(ksup), vp(isup))
     if rc:
         raise ValueError("invalid graphs for layout")
     nk = int(info[4])
@@ -233,7 +242,8 @@ def layout(graphs, P, S, capacity_blocks=0, flags=FLAG_RCM | FLAG_KEEP_IF_BETTER
                   n_unique=int(info[3]), n_kept=nk, n_dropped=int(info[5]),
                   bw_before_max=int(info[6]), bw_after_max=int(info[7]), perm=perm, offset=offset,
                   masks=masks, kept_dst=kd[:nk].copy(), kept_src=ks[:nk].copy(),
-                  kept_type=kt[:nk].copy(), bw_before=bwb, bw_after=bwa, n_nodes=n_nodes)
+                  kept_type=kt[:nk].copy(), bw_before=bwb, bw_after=bwa, n_nodes=n_nodes,
+                  kept_super=ksup[:nk].astype(bool), is_super=isup[:K * S].astype(bool))
 
 
 # ---------------------------------------------------------------------------------------------

@@ -193,23 +193,35 @@ int32_t orc_num_blocks(int32_t n_graphs, const int32_t* n_nodes, int32_t S, int3
 // block-tridiagonal cover of Eq. 3.
 //
 // Graph g's edges are src/dst/etype[edge_off[g] .. edge_off[g+1]) with graph-local ids.
-// flags bit 0: reorder each graph by RCM; bit 1: keep-if-better.
+// flags bit 0: reorder each graph by RCM; bit 1: keep-if-better; bit 2: supernodes.
+// Supernodes (the "supernode" propagation primitive of Section 6: some nodes may exchange
+// messages with every node, through the first rows and columns of the adjacency): a node with at
+// least super_min_degree distinct neighbours (edges of any type and direction, self-loops not
+// counted) is a supernode, at most max_super per graph, highest degree first (ties: lower id).  A
+// graph's supernodes take its first positions in that order, the RCM order of the graph without
+// them follows, and every edge with a supernode end is kept whatever its block distance; the
+// band masks hold the other kept edges only.  bw_after then measures the edges without a
+// supernode end.
 // Outputs (caller-owned):
 //   perm[node_off[g] + new] = old          (node_off = prefix sums of n_nodes; every graph)
 //   offset[g] = first supergraph position of g, or -1 if it was not packed
 //   info[0..7] = K, n_packed, n_real, n_unique_edges, n_kept, n_dropped, bw_before_max, bw_after_max
 //   masks: bit (k, d+1, p, r, c) of byte ((((k*3 + d+1)*P + p)*S + r)*(S/8) + c/8), bit c%8, is 1
-//          iff the supergraph has a type-p edge from position (k+d)*S + c to position k*S + r;
-//          masks may be NULL.
+//          iff the supergraph has a type-p band edge from position (k+d)*S + c to position
+//          k*S + r; masks may be NULL.
 //   kept_dst/kept_src/kept_type (capacity = total edges): the kept, deduplicated edges in
-//          supergraph positions, sorted by (dst, src, type); may be NULL.
+//          supergraph positions, sorted by (dst, src, type); may be NULL.  kept_super (may be
+//          NULL) marks those with a supernode end.
+//   is_super (K*S bytes, may be NULL): 1 at the positions of supernodes.
 //   bw_before/bw_after per graph (may be NULL).
 // Returns 0, or -1 on invalid input.
 int orc_layout(int32_t n_graphs, const int32_t* n_nodes, const int64_t* edge_off,
                const int32_t* src, const int32_t* dst, const int32_t* etype, int32_t P, int32_t S,
                int32_t capacity_blocks, int32_t flags, int32_t* perm, int32_t* offset,
                int64_t* info, uint8_t* masks, int32_t* kept_dst, int32_t* kept_src,
-               int32_t* kept_type, int64_t* bw_before, int64_t* bw_after) {
+               int32_t* kept_type, int64_t* bw_before, int64_t* bw_after,
+               int32_t super_min_degree, int32_t max_super, uint8_t* kept_super,
+               uint8_t* is_super) {
   if (n_graphs < 0 || P < 1 || S < 8 || S % 8 != 0) return -1;
   int32_t K = orc_num_blocks(n_graphs, n_nodes, S, capacity_blocks);
   int64_t cap = (int64_t)K * S;
@@ -218,6 +230,7 @@ int orc_layout(int32_t n_graphs, const int32_t* n_nodes, const int64_t* edge_off
   int32_t n_packed = 0;
   int64_t bwb_max = 0, bwa_max = 0;
   std::vector<std::pair<std::pair<int64_t, int64_t>, int32_t>> edges;  // ((dst, src), type)
+  std::vector<uint8_t> sup_at((size_t)cap, 0);
   for (int32_t g = 0; g < n_graphs; ++g) {
     int32_t n = n_nodes[g];
     int64_t e0 = edge_off[g], e1 = edge_off[g + 1];
@@ -226,17 +239,43 @@ int orc_layout(int32_t n_graphs, const int32_t* n_nodes, const int64_t* edge_off
       if (src[e] < 0 || src[e] >= n || dst[e] < 0 || dst[e] >= n || etype[e] < 0 ||
           etype[e] >= P)
         return -1;
-    std::vector<int32_t> p(n);
-    if (flags & 1) {
-      if (orc_rcm(n, e1 - e0, src + e0, dst + e0, (flags & 2) ? 1 : 0, p.data())) return -1;
-    } else {
-      for (int32_t i = 0; i < n; ++i) p[i] = i;
+    // supernodes first (bit 2), then the rest in RCM (bit 0) or input order
+    std::vector<int32_t> sup;
+    if (flags & 4) {
+      NbrLists nb = symmetric_neighbours(n, e1 - e0, src + e0, dst + e0);
+      for (int32_t v = 0; v < n; ++v)
+        if ((int64_t)nb[v].size() >= super_min_degree) sup.push_back(v);
+      std::sort(sup.begin(), sup.end(), [&](int32_t a, int32_t b) {
+        return nb[a].size() != nb[b].size() ? nb[a].size() > nb[b].size() : a < b;
+      });
+      if ((int32_t)sup.size() > max_super) sup.resize(std::max(0, max_super));
     }
+    std::vector<char> sflag(n, 0);
+    for (int32_t v : sup) sflag[v] = 1;
+    std::vector<int32_t> rest, rid(n, -1);
+    for (int32_t v = 0; v < n; ++v)
+      if (!sflag[v]) { rid[v] = (int32_t)rest.size(); rest.push_back(v); }
+    std::vector<int32_t> rs, rd;
+    for (int64_t e = e0; e < e1; ++e)
+      if (!sflag[src[e]] && !sflag[dst[e]]) { rs.push_back(rid[src[e]]); rd.push_back(rid[dst[e]]); }
+    const int32_t nr = (int32_t)rest.size();
+    std::vector<int32_t> pr(nr);
+    if (flags & 1) {
+      if (orc_rcm(nr, (int64_t)rs.size(), rs.data(), rd.data(), (flags & 2) ? 1 : 0, pr.data()))
+        return -1;
+    } else {
+      for (int32_t i = 0; i < nr; ++i) pr[i] = i;
+    }
+    std::vector<int32_t> p(sup);
+    for (int32_t i = 0; i < nr; ++i) p.push_back(rest[pr[i]]);
     std::memcpy(perm + node_off, p.data(), sizeof(int32_t) * n);
     std::vector<int32_t> pos(n);
     for (int32_t i = 0; i < n; ++i) pos[p[i]] = i;
     int64_t bwb = orc_bandwidth(n, e1 - e0, src + e0, dst + e0, nullptr);
-    int64_t bwa = orc_bandwidth(n, e1 - e0, src + e0, dst + e0, pos.data());
+    int64_t bwa = 0;
+    for (int64_t e = e0; e < e1; ++e)
+      if (!sflag[src[e]] && !sflag[dst[e]])
+        bwa = std::max<int64_t>(bwa, std::abs((int64_t)pos[dst[e]] - (int64_t)pos[src[e]]));
     if (bw_before) bw_before[g] = bwb;
     if (bw_after) bw_after[g] = bwa;
     if (!stopped && next_pos + n <= cap) {
@@ -244,6 +283,7 @@ int orc_layout(int32_t n_graphs, const int32_t* n_nodes, const int64_t* edge_off
       ++n_packed;
       bwb_max = std::max(bwb_max, bwb);
       bwa_max = std::max(bwa_max, bwa);
+      for (size_t i = 0; i < sup.size(); ++i) sup_at[(size_t)next_pos + i] = 1;
       for (int64_t e = e0; e < e1; ++e)
         edges.push_back({{next_pos + pos[dst[e]], next_pos + pos[src[e]]}, etype[e]});
       next_pos += n;
@@ -256,13 +296,15 @@ int orc_layout(int32_t n_graphs, const int32_t* n_nodes, const int64_t* edge_off
   std::sort(edges.begin(), edges.end());
   edges.erase(std::unique(edges.begin(), edges.end()), edges.end());
   if (masks) std::memset(masks, 0, (size_t)K * 3 * P * S * (S / 8));
+  if (is_super) std::memcpy(is_super, sup_at.data(), (size_t)cap);
   int64_t kept = 0, dropped = 0;
   for (const auto& ed : edges) {
     int64_t i = ed.first.first, j = ed.first.second;
     int32_t t = ed.second;
     int64_t k = i / S, c = j / S, d = c - k;
-    if (d < -1 || d > 1) { ++dropped; continue; }
-    if (masks) {
+    const bool via_super = sup_at[(size_t)i] || sup_at[(size_t)j];
+    if (!via_super && (d < -1 || d > 1)) { ++dropped; continue; }
+    if (masks && !via_super) {
       int64_t r = i % S, cc = j % S;
       size_t byte = ((((size_t)k * 3 + (size_t)(d + 1)) * P + t) * S + r) * (S / 8) + cc / 8;
       masks[byte] |= (uint8_t)(1u << (cc % 8));
@@ -272,6 +314,7 @@ int orc_layout(int32_t n_graphs, const int32_t* n_nodes, const int64_t* edge_off
       kept_src[kept] = (int32_t)j;
       kept_type[kept] = t;
     }
+    if (kept_super) kept_super[kept] = via_super ? 1 : 0;
     ++kept;
   }
   info[0] = K; info[1] = n_packed; info[2] = next_pos; info[3] = (int64_t)edges.size();

@@ -530,3 +530,64 @@ def test_reach_filter_leaves_candidate_states_unchanged():
     E2 = E.copy(); E2[dropped] += 10.0
     Es2, _ = oracle.ggnn_fwd(g.n_nodes, P, H, T, g.n_nodes, g.dst, g.src, g.etype, E2, prm)
     np.testing.assert_array_equal(Es2[T][cand], Es[T][cand])
+
+
+# ------------------------------------------------------------------------ supernodes (Section 6)
+
+
+def _star_chain(n_leaves, seed):
+    """A chain over n_leaves + 1 nodes plus a hub (node 0) that every node sends a type-0 edge to
+    and that sends a type-2 edge back to every node, relabelled at random."""
+    g = synth.hub_graph(n_leaves, 3, seed, lam=0.0)
+    hub = int(np.bincount(g.dst[g.etype == 0]).argmax())
+    back = g.src[g.etype == 0]
+    return synth.Graph(g.n_nodes, np.concatenate([g.src, np.full(len(back), hub, np.int32)]),
+                       np.concatenate([g.dst, back]),
+                       np.concatenate([g.etype, np.full(len(back), 2, np.int32)]), 3), hub
+
+
+def test_supernode_selection_rule_and_positions():
+    """Degrees are distinct neighbours over all types and both directions; nodes at or above the
+    threshold become supernodes, highest degree first, ties by lower id, at most max_super; they
+    take the graph's first positions in that order."""
+    # node 0: 5 neighbours, node 1: 4, node 2: 4, others fewer; node 0 -> node 0 self-loop ignored
+    src = np.array([0, 0, 0, 0, 0, 1, 1, 1, 2, 2, 2, 0, 7], np.int32)
+    dst = np.array([1, 2, 3, 4, 5, 6, 7, 8, 6, 7, 8, 0, 2], np.int32)
+    g = synth.Graph(9, src, dst, np.zeros(13, np.int32), 1)
+    F = oracle.FLAG_RCM | oracle.FLAG_KEEP_IF_BETTER | oracle.FLAG_SUPERNODES
+    lay = oracle.layout([g], 1, 32, flags=F, super_min_degree=4, max_super=8)
+    assert list(lay.perm[:3]) == [0, 1, 2] and lay.is_super[:3].all() and not lay.is_super[3:].any()
+    lay = oracle.layout([g], 1, 32, flags=F, super_min_degree=4, max_super=2)
+    assert list(lay.perm[:2]) == [0, 1] and lay.is_super.sum() == 2
+    lay = oracle.layout([g], 1, 32, flags=F, super_min_degree=6, max_super=8)
+    plain = oracle.layout([g], 1, 32)
+    assert not lay.is_super.any() and np.array_equal(lay.perm, plain.perm)
+
+
+def test_supernodes_keep_every_hub_edge_and_restore_a_narrow_band():
+    """A hub connected both ways to 300 chain nodes: without supernodes RCM cannot give a band
+    narrower than about half the graph and the cover at S = 32 drops most hub edges; as a
+    supernode the hub takes position 0, the rest is a chain of bandwidth 1, and nothing is
+    dropped, so the band propagation equals dense brute force over all edges (Eq. 1)."""
+    g, hub = _star_chain(300, 3)
+    plain = oracle.layout([g], 3, 32)
+    assert plain.n_dropped > 300 and plain.bw_after_max > 100
+    F = oracle.FLAG_RCM | oracle.FLAG_KEEP_IF_BETTER | oracle.FLAG_SUPERNODES
+    lay = oracle.layout([g], 3, 32, flags=F, super_min_degree=64, max_super=4)
+    assert lay.perm[0] == hub and lay.is_super.sum() == 1
+    assert lay.n_dropped == 0 and lay.bw_after_max == 1
+    assert lay.kept_super.sum() == np.sum((g.src == hub) | (g.dst == hub))  # 300 in, 301 out
+    # the band masks hold exactly the kept edges without a supernode end
+    bits = np.unpackbits(lay.masks, bitorder="little").sum()
+    assert bits == lay.n_kept - lay.kept_super.sum()
+    H, P = 6, 3
+    rng = np.random.default_rng(1)
+    E = np.zeros((lay.n_pad, H)); E[:lay.n_real] = rng.standard_normal((lay.n_real, H))
+    prm = synth.gen_params(P, H, 2)
+    Y = oracle.propagate_fwd(lay.n_pad, P, H, lay.kept_dst, lay.kept_src, lay.kept_type, E,
+                             prm["W"], prm["b"])
+    pos = np.empty(g.n_nodes, np.int64); pos[lay.perm] = np.arange(g.n_nodes)
+    A = np.zeros((P, lay.n_pad, lay.n_pad))
+    A[g.etype, pos[g.dst], pos[g.src]] = 1.0
+    want = sum(A[p] @ (E @ prm["W"][p]) + A[p].sum(1, keepdims=True) * prm["b"][p] for p in range(P))
+    np.testing.assert_allclose(Y, want, rtol=1e-12, atol=1e-12)
