@@ -47,6 +47,7 @@ extern "C" {
 /* ---- plan flags (bg_band_plan) ---------------------------------------------------------- */
 #define BG_RCM 1u            /* reorder every graph by Reverse Cuthill-McKee (Section 3.1) */
 #define BG_KEEP_IF_BETTER 2u /* keep a graph's input order when RCM does not lower its bandwidth */
+#define BG_SUPERNODES 4u     /* supernodes (bg_band_plan_opts): see bg_plan_opts */
 
 /* ---- backward flags --------------------------------------------------------------------- */
 #define BG_ACCUM 1u /* add into dE/dW/db (and GRU gradients) instead of overwriting them */
@@ -78,7 +79,10 @@ typedef struct bg_info {
   int64_t n_kept;         /* edges inside the block-tridiagonal cover (Eq. 3) */
   int64_t n_dropped;      /* edges whose block distance exceeds one (coverage rule, Section 3.2) */
   int64_t bw_before_max;  /* max over packed graphs of the input-order bandwidth (Section 2) */
-  int64_t bw_after_max;   /* max over packed graphs of the bandwidth after reordering */
+  int64_t bw_after_max;   /* max over packed graphs of the bandwidth after reordering (edges
+                             without a supernode end) */
+  int32_t n_super;        /* supernodes of the packed graphs (BG_SUPERNODES) */
+  int64_t n_super_edges;  /* kept edges with a supernode end (included in n_kept) */
 } bg_info;
 
 /* ---- compile step (host) ------------------------------------------------------------------
@@ -92,6 +96,22 @@ typedef struct bg_info {
  * BG_ECAPACITY (not even the first graph fits), BG_ENOMEM. */
 int bg_band_plan(const bg_graph* graphs, int32_t n_graphs, int32_t n_types, int32_t block_S,
                  int32_t capacity_blocks, uint32_t flags, bg_plan** out);
+/* bg_band_plan with options.  Supernodes (flag BG_SUPERNODES; the "supernode" propagation
+ * primitive of Section 6: some nodes exchange messages with every node, through dense first rows
+ * and columns of the adjacency): a node with at least supernode_min_degree distinct neighbours
+ * (edges of any type and direction; self-loops not counted) is a supernode, at most
+ * max_supernodes per graph, highest degree first (ties: lower id).  A graph's supernodes take its
+ * first positions in that order, and RCM orders the graph without them after them, so a hub no
+ * longer widens the band.  Every edge with a supernode end is kept whatever the block distance
+ * and is propagated by the supernode rows and columns (a per-node gather over those edges, on
+ * the device), not by the band tiles; the other edges follow the band cover as before. */
+typedef struct bg_plan_opts {
+  uint32_t flags;               /* BG_RCM | BG_KEEP_IF_BETTER | BG_SUPERNODES */
+  int32_t supernode_min_degree; /* >= 1 when BG_SUPERNODES is set */
+  int32_t max_supernodes;       /* per graph, >= 0 */
+} bg_plan_opts;
+int bg_band_plan_opts(const bg_graph* graphs, int32_t n_graphs, int32_t n_types, int32_t block_S,
+                      int32_t capacity_blocks, const bg_plan_opts* opts, bg_plan** out);
 void bg_plan_free(bg_plan* plan); /* frees host and device memory of the plan; NULL is a no-op */
 int bg_plan_info(const bg_plan* plan, bg_info* out);
 
@@ -125,6 +145,10 @@ double bg_plan_flops(const bg_plan* plan, int32_t H, int32_t which);
 #define BG_EXPORT_BW 4      /* int64 [2][n_graphs]: bandwidth before / after reordering */
 #define BG_EXPORT_GATHER 5  /* int32 [n_real]: row of the caller's concatenated state array held
                                by each supergraph position */
+#define BG_EXPORT_SUPER_EDGES 6 /* int32 [n_super_edges][3]: (target position, source position,
+                               type) of the kept edges with a supernode end, sorted */
+#define BG_EXPORT_SUPER_COUNT 7 /* int32 [n_graphs]: supernodes of each graph (its first
+                               positions) */
 size_t bg_plan_export_bytes(const bg_plan* plan, int32_t which);
 int bg_plan_export(const bg_plan* plan, int32_t which, void* out, size_t out_bytes);
 

@@ -18,11 +18,11 @@ LIB_PATH = os.path.join(_PKG, "libbandggnn.so")
 HEADER = os.path.join(os.path.dirname(_PKG), "include", "bandggnn.h")
 
 BG_F32, BG_BF16 = 0, 1
-BG_RCM, BG_KEEP_IF_BETTER = 1, 2
+BG_RCM, BG_KEEP_IF_BETTER, BG_SUPERNODES = 1, 2, 4
 BG_ACCUM = 1
 BG_FLOPS_BAND, BG_FLOPS_XFORM, BG_FLOPS_GRU, BG_FLOPS_NNZ = 0, 1, 2, 3
 (BG_EXPORT_PERM, BG_EXPORT_OFFSETS, BG_EXPORT_MASKS, BG_EXPORT_MASKS_T, BG_EXPORT_BW,
- BG_EXPORT_GATHER) = range(6)
+ BG_EXPORT_GATHER, BG_EXPORT_SUPER_EDGES, BG_EXPORT_SUPER_COUNT) = range(8)
 BG_OP_PROPAGATE_FWD, BG_OP_PROPAGATE_BWD, BG_OP_GGNN_FWD, BG_OP_GGNN_BWD, BG_OP_READOUT = range(5)
 BG_KID_BAND_FWD, BG_KID_BAND_BWD, BG_KID_GRU_FWD, BG_KID_GRU_BWD, BG_KID_DW = range(5)
 STATUS = {0: "BG_OK", -1: "BG_EINVAL", -2: "BG_ECAPACITY", -3: "BG_ENOMEM", -4: "BG_ECUDA",
@@ -44,7 +44,13 @@ class bg_info(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in ("K", "S", "P", "n_graphs", "n_packed", "n_real",
                                               "n_pad")] + \
                [(n, ctypes.c_int64) for n in ("n_edges_in", "n_edges_unique", "n_kept",
-                                              "n_dropped", "bw_before_max", "bw_after_max")]
+                                              "n_dropped", "bw_before_max", "bw_after_max")] + \
+               [("n_super", ctypes.c_int32), ("n_super_edges", ctypes.c_int64)]
+
+
+class bg_plan_opts(ctypes.Structure):
+    _fields_ = [("flags", ctypes.c_uint32), ("supernode_min_degree", ctypes.c_int32),
+                ("max_supernodes", ctypes.c_int32)]
 
 
 class bg_params(ctypes.Structure):
@@ -71,6 +77,7 @@ def load(path: str = LIB_PATH):
     vp, i32, i64, sz, f32 = c.c_void_p, c.c_int32, c.c_int64, c.c_size_t, c.c_float
     sig = {
         "bg_band_plan": (c.c_int, [vp, i32, i32, i32, i32, c.c_uint32, vp]),
+        "bg_band_plan_opts": (c.c_int, [vp, i32, i32, i32, i32, vp, vp]),
         "bg_plan_free": (None, [vp]),
         "bg_plan_info": (c.c_int, [vp, vp]),
         "bg_plan_flops": (c.c_double, [vp, i32, i32]),
@@ -199,8 +206,10 @@ class Plan:
         buf = np.zeros(max(n, 1), np.uint8)
         _check(lib.bg_plan_export(self.handle, which, buf.ctypes.data, n))
         buf = buf[:n]
-        if which in (BG_EXPORT_PERM, BG_EXPORT_OFFSETS, BG_EXPORT_GATHER):
+        if which in (BG_EXPORT_PERM, BG_EXPORT_OFFSETS, BG_EXPORT_GATHER, BG_EXPORT_SUPER_COUNT):
             return buf.view(np.int32)
+        if which == BG_EXPORT_SUPER_EDGES:
+            return buf.view(np.int32).reshape(-1, 3)
         if which == BG_EXPORT_BW:
             return buf.view(np.int64).reshape(2, -1)
         i = self.info()
@@ -210,8 +219,10 @@ class Plan:
         _check(load().bg_plan_upload(self.handle, _stream(stream)))
 
 
-def band_plan(graphs, n_types, block_S, capacity_blocks=0, flags=BG_RCM | BG_KEEP_IF_BETTER) -> Plan:
-    """bg_band_plan on a list of objects with n_nodes, src, dst, etype (int32 arrays)."""
+def band_plan(graphs, n_types, block_S, capacity_blocks=0, flags=BG_RCM | BG_KEEP_IF_BETTER,
+              supernode_min_degree=0, max_supernodes=0) -> Plan:
+    """bg_band_plan (bg_band_plan_opts with BG_SUPERNODES) on a list of objects with n_nodes, src,
+    dst, etype (int32 arrays)."""
     lib = load()
     keep = []
     arr = (bg_graph * len(graphs))()
@@ -223,8 +234,13 @@ def band_plan(graphs, n_types, block_S, capacity_blocks=0, flags=BG_RCM | BG_KEE
         arr[i] = bg_graph(int(g.n_nodes), int(s.shape[0]), s.ctypes.data, d.ctypes.data,
                           t.ctypes.data)
     h = ctypes.c_void_p()
-    _check(lib.bg_band_plan(arr, len(graphs), n_types, block_S, capacity_blocks, flags,
-                            ctypes.byref(h)))
+    if flags & BG_SUPERNODES:
+        opts = bg_plan_opts(flags, supernode_min_degree, max_supernodes)
+        _check(lib.bg_band_plan_opts(arr, len(graphs), n_types, block_S, capacity_blocks,
+                                     ctypes.byref(opts), ctypes.byref(h)))
+    else:
+        _check(lib.bg_band_plan(arr, len(graphs), n_types, block_S, capacity_blocks, flags,
+                                ctypes.byref(h)))
     return Plan(h.value, n_types)
 
 

@@ -14,6 +14,7 @@
 #include "gru_tc.h"
 #include "internal.h"
 #include "kernels.h"
+#include "super.h"
 
 namespace bg {
 long long launch_total();
@@ -186,8 +187,22 @@ extern "C" int bg_band_plan(const bg_graph* graphs, int32_t n_graphs, int32_t n_
                             int32_t block_S, int32_t capacity_blocks, uint32_t flags,
                             bg_plan** out) {
   bg_clear_error();
+  if (flags & BG_SUPERNODES) return bg_fail(BG_EINVAL, "supernodes need bg_band_plan_opts");
   try {
-    return bg_plan_build(graphs, n_graphs, n_types, block_S, capacity_blocks, flags, out);
+    return bg_plan_build(graphs, n_graphs, n_types, block_S, capacity_blocks, flags, 0, 0, out);
+  } catch (const std::bad_alloc&) {
+    return bg_fail(BG_ENOMEM, "host allocation failed");
+  }
+}
+
+extern "C" int bg_band_plan_opts(const bg_graph* graphs, int32_t n_graphs, int32_t n_types,
+                                 int32_t block_S, int32_t capacity_blocks, const bg_plan_opts* opts,
+                                 bg_plan** out) {
+  bg_clear_error();
+  if (!opts) return bg_fail(BG_EINVAL, "opts is NULL");
+  try {
+    return bg_plan_build(graphs, n_graphs, n_types, block_S, capacity_blocks, opts->flags,
+                         opts->supernode_min_degree, opts->max_supernodes, out);
   } catch (const std::bad_alloc&) {
     return bg_fail(BG_ENOMEM, "host allocation failed");
   }
@@ -205,6 +220,7 @@ static void free_device(bg_plan* p) {
   cudaFree(p->d_seg_cnt);
   cudaFree(p->d_row_graph);
   bg::band_tc_release(p);
+  bg::super_release(p);
   cudaSetDevice(prev);
   p->d_masks = p->d_masksT = nullptr;
   p->d_gather = p->d_seg_off = p->d_seg_cnt = p->d_row_graph = nullptr;
@@ -223,6 +239,7 @@ extern "C" int bg_plan_info(const bg_plan* p, bg_info* o) {
   o->n_real = p->n_real; o->n_pad = p->n_pad(); o->n_edges_in = p->n_edges_in;
   o->n_edges_unique = p->n_unique; o->n_kept = p->n_kept; o->n_dropped = p->n_dropped;
   o->bw_before_max = p->bw_before_max; o->bw_after_max = p->bw_after_max;
+  o->n_super = p->n_super; o->n_super_edges = p->n_super_edges();
   return BG_OK;
 }
 
@@ -247,6 +264,8 @@ extern "C" size_t bg_plan_export_bytes(const bg_plan* p, int32_t which) {
     case BG_EXPORT_MASKS_T: return p->masks.size() * 4;
     case BG_EXPORT_BW: return p->bw_before.size() * 16;
     case BG_EXPORT_GATHER: return p->gather.size() * 4;
+    case BG_EXPORT_SUPER_EDGES: return p->sup_edges.size() * 4;
+    case BG_EXPORT_SUPER_COUNT: return p->nsup.size() * 4;
     default: return 0;
   }
 }
@@ -254,7 +273,8 @@ extern "C" size_t bg_plan_export_bytes(const bg_plan* p, int32_t which) {
 extern "C" int bg_plan_export(const bg_plan* p, int32_t which, void* out, size_t out_bytes) {
   if (!p || !out) return bg_fail(BG_EINVAL, "NULL argument");
   size_t need = bg_plan_export_bytes(p, which);
-  if (need == 0 && which != BG_EXPORT_GATHER) return bg_fail(BG_EINVAL, "unknown export kind");
+  if (which < BG_EXPORT_PERM || which > BG_EXPORT_SUPER_COUNT)
+    return bg_fail(BG_EINVAL, "unknown export kind");
   if (out_bytes < need) return bg_fail(BG_ECAPACITY, "export buffer too small");
   switch (which) {
     case BG_EXPORT_PERM: std::memcpy(out, p->perm.data(), need); break;
@@ -269,6 +289,8 @@ extern "C" int bg_plan_export(const bg_plan* p, int32_t which, void* out, size_t
       break;
     }
     case BG_EXPORT_GATHER: std::memcpy(out, p->gather.data(), need); break;
+    case BG_EXPORT_SUPER_EDGES: std::memcpy(out, p->sup_edges.data(), need); break;
+    case BG_EXPORT_SUPER_COUNT: std::memcpy(out, p->nsup.data(), need); break;
   }
   return BG_OK;
 }
@@ -304,7 +326,7 @@ extern "C" int bg_plan_upload(bg_plan* p, void* stream) {
   }
   // host vectors must outlive the async copies
   BG_CUDA(cudaStreamSynchronize(st));
-  if (bg::band_tc_upload(p, st) != 0) {
+  if (bg::band_tc_upload(p, st) != 0 || bg::super_upload(p, st) != 0) {
     free_device(p);
     return bg_fail(BG_ENOMEM, "device allocation for the band tiles failed");
   }
@@ -384,6 +406,7 @@ bool tc_gemm_path(bg_dtype dt, int H) {
 struct BwdWs {
   size_t dM, Wt, part;                 // fp32 SIMT path
   size_t dMb, dMT, Wp, ETa, tpart;     // bf16 path with tensor-core GEMMs
+  size_t super;                        // supernode edges (after everything else)
   size_t total;
 };
 BwdWs bwd_ws(const bg_plan* p, bg_dtype dt, int H) {
@@ -404,6 +427,8 @@ BwdWs bwd_ws(const bg_plan* p, bg_dtype dt, int H) {
     total = std::max(total, q);
   }
   w.total = std::max(total, bg::band_tc_bwd_ws_bytes(p, (int)dt, H));
+  w.super = al(w.total);
+  w.total = w.super + bg::super_bwd_ws_bytes(p, H);
   return w;
 }
 
@@ -497,7 +522,7 @@ TcSaved tc_saved(const bg_plan* p, int H, int T) {
   return s;
 }
 struct TcFwdWs {
-  size_t WT, b2T, split, total;
+  size_t WT, b2T, split, addend, total;
 };
 TcFwdWs tc_fwd_ws(const bg_plan* p, int H) {
   TcFwdWs w{};
@@ -505,11 +530,12 @@ TcFwdWs tc_fwd_ws(const bg_plan* p, int H) {
   w.WT = o; o += bg::band_tc_w_bytes(p, H);
   w.b2T = o; o += al((size_t)H * 64 * 2);
   w.split = o; o += al(sizeof(float) * bg::band_tc_split_floats(p, H));
+  w.addend = o; o += al(sizeof(float) * (size_t)p->sup_rows_in * H);
   w.total = o;
   return w;
 }
 struct TcBwdWs {
-  size_t g, dXT, dMT, dgiT, dhnT, WihT, WhhT, Wk, part, split, total;
+  size_t g, dXT, dMT, dgiT, dhnT, WihT, WhhT, Wk, part, split, sup, dWs, dbs, total;
 };
 size_t tc_part_floats(const bg_plan* p, int H, int T) {
   const int64_t K = (int64_t)T * p->n_pad();
@@ -531,6 +557,10 @@ TcBwdWs tc_bwd_ws(const bg_plan* p, int H, int T) {
   w.Wk = o; o += bg::band_tc_w_bytes(p, H);
   w.part = o; o += al(sizeof(float) * tc_part_floats(p, H, T));
   w.split = o; o += al(sizeof(float) * bg::band_tc_split_floats(p, H));
+  const bool sup = p->n_super_edges() > 0;
+  w.sup = o; o += bg::super_bwd_ws_bytes(p, H);
+  w.dWs = o; o += sup ? al(sizeof(float) * (size_t)p->P * H * H) : 0;
+  w.dbs = o; o += sup ? al(sizeof(float) * (size_t)p->P * H) : 0;
   w.total = o;
   return w;
 }
@@ -606,6 +636,8 @@ static int propagate_fwd_impl(const bg_plan* p, bg_dtype dt, int H, const void* 
     BG_TRY(status_word_ptr(&status));
     // the band kernel alone is timed inside (its operand preparation is not)
     BG_CUDA(bg::band_tc_fwd(p, H, E, W, b, Y, ws, ws_bytes, status, st));
+    // the supernode rows and columns (Section 6), added to the band's sums
+    BG_CUDA(bg::super_fwd(p, bf, H, E, W, b, Y, 0, st));
     return BG_OK;
   }
   // SIMT path: messages M_p = E W_p + b_p for all p, then the band sum over the bit tiles
@@ -631,6 +663,7 @@ static int propagate_fwd_impl(const bg_plan* p, bg_dtype dt, int H, const void* 
     BG_CUDA(bg::gemm(g, nullptr, 0, st));
   }
   BG_CUDA(bg::band_fwd_gather(p->d_masks, M, Y, p->K, p->S, p->P, H, st));
+  BG_CUDA(bg::super_fwd(p, bf, H, E, W, b, Y, 0, st));
   return BG_OK;
 }
 
@@ -646,8 +679,25 @@ extern "C" int bg_band_propagate_fwd(const bg_plan* p, bg_dtype dt, int32_t H, c
                             (cudaStream_t)stream);
 }
 
+static int propagate_bwd_band(const bg_plan* p, bg_dtype dt, int H, const void* E, const void* W,
+                              const float* dY, float* dE, float* dW, float* db, int accum,
+                              char* ws, size_t ws_bytes, cudaStream_t st);
+
 // dE/dW/db accumulate when accum != 0 (callers zero them first otherwise).
 static int propagate_bwd_impl(const bg_plan* p, bg_dtype dt, int H, const void* E, const void* W,
+                              const float* dY, float* dE, float* dW, float* db, int accum,
+                              char* ws, size_t ws_bytes, cudaStream_t st) {
+  const int bf = dt == BG_BF16;
+  BwdWs w = bwd_ws(p, dt, H);
+  if (ws_bytes < w.total) return bg_fail(BG_ECAPACITY, "workspace too small");
+  BG_TRY(propagate_bwd_band(p, dt, H, E, W, dY, dE, dW, db, accum, ws, ws_bytes, st));
+  // the supernode rows and columns (Section 6), added to the band's gradients
+  BG_CUDA(bg::super_bwd(p, bf, H, E, W, dY, nullptr, 0, dE, dW, db, ws + w.super, st));
+  return BG_OK;
+}
+
+// The band part of propagate_bwd_impl.
+static int propagate_bwd_band(const bg_plan* p, bg_dtype dt, int H, const void* E, const void* W,
                               const float* dY, float* dE, float* dW, float* db, int accum,
                               char* ws, size_t ws_bytes, cudaStream_t st) {
   const int bf = dt == BG_BF16;
@@ -660,7 +710,6 @@ static int propagate_bwd_impl(const bg_plan* p, bg_dtype dt, int H, const void* 
     return BG_OK;
   }
   BwdWs w = bwd_ws(p, dt, H);
-  if (ws_bytes < w.total) return bg_fail(BG_ECAPACITY, "workspace too small");
   if (tc_gemm_path(dt, H)) {
     int* status = nullptr;
     BG_TRY(status_word_ptr(&status));
@@ -800,6 +849,7 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
     __nv_bfloat16* b2T = reinterpret_cast<__nv_bfloat16*>(wsc + wl.b2T);
     float* split = bg::band_tc_split_floats(p, H) ? reinterpret_cast<float*>(wsc + wl.split)
                                                    : nullptr;
+    float* addend = p->sup_rows_in ? reinterpret_cast<float*>(wsc + wl.addend) : nullptr;
     BG_CUDA(cudaMemcpyAsync(Ei(0), E0, n * H * 2, cudaMemcpyDeviceToDevice, st));
     BG_CUDA(bg::prep_transpose_bf16(E0, 0, ETa, (int)n, H, 1, st, (int64_t)TN));
     BG_CUDA(bg::fill_ones_rows(ETa, H, (int64_t)TN, (int64_t)TN, st));
@@ -807,11 +857,13 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
     BG_CUDA(bg::band_tc_prep_w(p, H, prm->W, 0, WT, st));
     if (prm->b) BG_CUDA(bg::prep_bias_split(p, prm->b, b2T, H, status, st));
     for (int t = 0; t < T; ++t) {
+      // the supernode rows' messages, which the band kernel adds before it rounds Y
+      if (addend) BG_CUDA(bg::super_fwd(p, 1, H, Ei(t), prm->W, prm->b, addend, 1, st));
       {
         KTimer tm(BG_KID_BAND_FWD, st);
         BG_CUDA(bg::band_tc_fwd_core(p, H, ETa + (size_t)t * n, (int64_t)TN, WT,
                                      prm->b ? b2T : nullptr, nullptr, Yi(t), YTa + (size_t)t * n,
-                                     (int64_t)TN, split, status, st));
+                                     (int64_t)TN, split, addend, status, st));
       }
       KTimer tm(BG_KID_GRU_FWD, st);
       BG_CUDA(bg::gru_fwd_tc(
@@ -893,6 +945,13 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     BG_CUDA(bg::prep_transpose_bf16(Whh, 0, WhhT, 3 * H, H, 1, st));
     void* Wk = wsc + wl.Wk;
     BG_CUDA(bg::band_tc_prep_w(p, H, prm->W, 1, Wk, st));
+    const bool sup = p->n_super_edges() > 0;
+    float* dWs = reinterpret_cast<float*>(wsc + wl.dWs);
+    float* dbs = reinterpret_cast<float*>(wsc + wl.dbs);
+    if (sup) {
+      BG_CUDA(bg::fill_zero_f32(dWs, (int64_t)p->P * H * H, st));
+      BG_CUDA(bg::fill_zero_f32(dbs, (int64_t)p->P * H, st));
+    }
     const float* gin = dET;
     for (int t = T - 1; t >= 0; --t) {
       {
@@ -901,9 +960,15 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
                                prm->b_hh, gin, g, dXT, (int64_t)n, dgiT + (size_t)t * n,
                                dhnT + (size_t)t * n, (int64_t)TN, status, st));
       }
-      KTimer tm(BG_KID_BAND_BWD, st);
-      BG_CUDA(bg::band_tc_bwd_core(p, H, dXT, (int64_t)n, Wk, g, 1, dMT + (size_t)t * n,
-                                   (int64_t)TN, split, status, st));
+      {
+        KTimer tm(BG_KID_BAND_BWD, st);
+        BG_CUDA(bg::band_tc_bwd_core(p, H, dXT, (int64_t)n, Wk, g, 1, dMT + (size_t)t * n,
+                                     (int64_t)TN, split, status, st));
+      }
+      // the supernode rows and columns: dE(t) and their share of dW, db (summed over the steps)
+      if (sup)
+        BG_CUDA(bg::super_bwd(p, 1, H, Ei(t), prm->W, nullptr, dXT, (int64_t)n, g, dWs, dbs,
+                              wsc + wl.sup, st, t < T - 1));
       gin = g;
     }
     const int acc = (flags & BG_ACCUM) ? 1 : 0;
@@ -917,6 +982,10 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
         {dhnT, (int64_t)TN, ETa, (int64_t)TN, H, 0, gr->dW_hh + (size_t)2 * H * H,
          gr->db_hh + 2 * H}};
     BG_CUDA(bg::gemm_tn_multi(probs, 4, H, (int64_t)TN, acc, part, pf, status, st));
+    if (sup) {
+      BG_CUDA(bg::add_inplace_f32(gr->dW, dWs, (int64_t)p->P * H * H, st));
+      if (gr->db) BG_CUDA(bg::add_inplace_f32(gr->db, dbs, (int64_t)p->P * H, st));
+    }
     BG_CUDA(cudaMemcpyAsync(dE0, g, sizeof(float) * n * H, cudaMemcpyDeviceToDevice, st));
     return BG_OK;
   }

@@ -181,6 +181,10 @@ __device__ __forceinline__ void drain_mmas(bool leader, uint64_t* bar) {
 struct Sched {
   int n_items, n_full, ksplit, part_rows;
   float* part;  // [ksplit][part_rows][H]: partial Y of split items, rows from tile n_full on
+  // forward: a row r with slot[r] >= 0 gets addend[slot[r]][:] added to its Y before the outputs
+  // are written (the supernode rows' messages); NULL for none
+  const float* addend;
+  const int32_t* slot;
 };
 
 // Tile and job range [j0, j1) of item w; part -1 for a whole tile, else its slice.
@@ -535,6 +539,7 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
       int k, j0, j1, part;
       item_of(sc, w, jobs, k, j0, j1, part);
       const int row = k * kTile + r;
+      const int asl = (!BWD && sc.addend && part < 0) ? sc.slot[row] : -1;
       bool ok = true;
       int hh = j0 / P, p = j0 - hh * P;
       for (int jb = j0; BWD && jb < j1; ++jb, ++c, p = p + 1 == P ? (++hh, 0) : p + 1) {
@@ -582,6 +587,11 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
         if (g0 + YG >= H) {
           tc_fence_before();
           warp_arrive(&bars->y_empty);
+        }
+        if (asl >= 0) {
+          const float* ad = sc.addend + (size_t)asl * H + g0;
+#pragma unroll
+          for (int j = 0; j < YG; ++j) vg[j] = __float_as_uint(__uint_as_float(vg[j]) + ad[j]);
         }
 #pragma unroll
         for (int h1 = 0; h1 < YG; h1 += 32) {
@@ -690,7 +700,8 @@ __global__ void k_band_split_fixup(const float* __restrict__ part, int ksplit, i
                                    int row0, int H, float* __restrict__ out,
                                    __nv_bfloat16* __restrict__ outb,
                                    __nv_bfloat16* __restrict__ outT, int64_t ld_outT,
-                                   int accumulate) {
+                                   int accumulate, const float* __restrict__ addend,
+                                   const int32_t* __restrict__ slot) {
   grid_dep_wait();  // the partials are the band kernel's output
   const int64_t n4 = (int64_t)part_rows * H / 4, slice = (int64_t)part_rows * H;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < n4;
@@ -702,6 +713,10 @@ __global__ void k_band_split_fixup(const float* __restrict__ part, int ksplit, i
       y.x += v.x; y.y += v.y; y.z += v.z; y.w += v.w;
     }
     const int row = row0 + (int)(e / H), h = (int)(e % H);
+    if (addend && slot[row] >= 0) {
+      const float4 a = *reinterpret_cast<const float4*>(addend + (size_t)slot[row] * H + h);
+      y.x += a.x; y.y += a.y; y.z += a.z; y.w += a.w;
+    }
     if (out) {
       float4* o = reinterpret_cast<float4*>(out + (size_t)row * H + h);
       if (accumulate) {
@@ -813,7 +828,7 @@ cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap&
                      const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
                      __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
                      __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate,
-                     float* split, int* status, cudaStream_t st) {
+                     float* split, const float* addend, int* status, cudaStream_t st) {
   using C = Cfg<H, S>;
   cudaError_t e = cudaFuncSetAttribute(k_band_tc<H, S, BWD>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
@@ -821,6 +836,8 @@ cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap&
   const int n_tiles = p->n_pad() / kTile, sms = num_sms();
   Sched sc = make_sched(n_tiles, C::NH * p->P, sms, split != nullptr);
   sc.part = split;
+  sc.addend = BWD ? nullptr : addend;
+  sc.slot = p->d_sin_slot;
   const int grid = std::min(sc.n_items, sms);
   e = launch_pdl(k_band_tc<H, S, BWD>, dim3(grid), dim3(C::THREADS), C::SMEM, st, tx, tw, tdeg,
                  tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt, sc,
@@ -830,7 +847,7 @@ cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap&
   const int64_t n4 = (int64_t)sc.part_rows * H / 4;
   e = launch_pdl(k_band_split_fixup, dim3((unsigned)std::min<int64_t>((n4 + 255) / 256, 2048)),
                  dim3(256), 0, st, (const float*)split, sc.ksplit, sc.part_rows,
-                 sc.n_full * kTile, H, out, outb, outT, ld_outT, accumulate);
+                 sc.n_full * kTile, H, out, outb, outT, ld_outT, accumulate, sc.addend, sc.slot);
   note_launch();
   return e;
 }
@@ -842,10 +859,10 @@ cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& t
                    const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
                    __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
                    __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate, float* split,
-                   int* status, cudaStream_t st) {
+                   const float* addend, int* status, cudaStream_t st) {
 #define BG_BAND_S(SV)                                                                            \
   return launch_s<H, SV, BWD>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, dMT, ld_mt,      \
-                              has_bias, accumulate, split, status, st);
+                              has_bias, accumulate, split, addend, status, st);
   switch (p->S) {
     case 32: BG_BAND_S(32)
     case 64: BG_BAND_S(64)
@@ -954,7 +971,7 @@ size_t band_tc_split_floats(const bg_plan* p, int H) {
 cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, int64_t ld_x,
                              const void* Wk, const __nv_bfloat16* b2T, float* out,
                              __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
-                             float* split, int* status, cudaStream_t st) {
+                             float* split, const float* addend, int* status, cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw, tdeg, tb2;
   if (!make_map_ld(&tx, XT, H, n, ld_x, (H < 64 || p->S == 512) ? 32 : 64) ||
@@ -964,7 +981,7 @@ cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, i
   const int hb = b2T != nullptr;
 #define BG_FWD(HV)                                                                                \
   return launch<HV, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, hb, 0,     \
-                           split, status, st);
+                           split, addend, status, st);
   switch (H) {
     case 32: BG_FWD(32)
     case 64: BG_FWD(64)
@@ -984,7 +1001,7 @@ cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, 
     return cudaErrorInvalidValue;
 #define BG_BWD(HV)                                                                                \
   return launch<HV, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,  \
-                          split, status, st);
+                          split, nullptr, status, st);
   switch (H) {
     case 32: BG_BWD(32)
     case 64: BG_BWD(64)
@@ -1020,7 +1037,7 @@ cudaError_t prep_bias_split(const bg_plan* p, const float* b, __nv_bfloat16* b2T
 cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, const float* b,
                         float* Y, char* ws, size_t ws_bytes, int* status, cudaStream_t st) {
   if (ws_bytes < band_tc_fwd_ws_bytes(p, 1, H)) return cudaErrorInvalidValue;
-  const int n = p->n_pad(), P = p->P;
+  const int n = p->n_pad();
   __nv_bfloat16* ET = reinterpret_cast<__nv_bfloat16*>(ws);
   void* WT = ws + al256((size_t)n * H * 2);
   __nv_bfloat16* b2T = reinterpret_cast<__nv_bfloat16*>(ws + al256((size_t)n * H * 2) +
@@ -1034,7 +1051,7 @@ cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, c
   if (e != cudaSuccess) return e;
   ProfSpan span(BG_KID_BAND_FWD, st);
   return band_tc_fwd_core(p, H, ET, n, WT, b ? b2T : nullptr, Y, nullptr, nullptr, 0,
-                          band_tc_split_floats(p, H) ? split : nullptr, status, st);
+                          band_tc_split_floats(p, H) ? split : nullptr, nullptr, status, st);
 }
 
 cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, const float* dY,

@@ -25,6 +25,29 @@ struct bg_plan {
   // band tiles as bit rows: [K][3][P][S][W32] words, bit c of word c/32 (LSB first)
   std::vector<uint32_t> masks;   // row = target r in block k, bits = source c in block k+d-1
   std::vector<uint32_t> masksT;  // row = source c in block j, bits = target i in block j+e-1
+  // supernodes: count per input graph (its first positions); kept edges with a supernode end,
+  // (target, source, type) in positions, sorted
+  int32_t n_super = 0;
+  std::vector<int32_t> nsup;
+  std::vector<int32_t> sup_edges;  // [n_super_edges][3]
+  // device copies of the supernode edges (super.cu): in-edges by target row, out-edges by source
+  // row, the (source row, type) pairs of the out-edges and those pairs grouped by type
+  int32_t sup_rows_in = 0, sup_rows_out = 0, sup_pairs = 0;
+  int32_t* d_sup = nullptr;        // one allocation holding the arrays below
+  int32_t* d_sin_rows = nullptr;   // [rows_in] target positions
+  int32_t* d_sin_off = nullptr;    // [rows_in + 1]
+  int32_t* d_sin_src = nullptr;    // [n_super_edges] sorted by (type, source) within a row
+  int32_t* d_sin_type = nullptr;
+  int32_t* d_sin_slot = nullptr;   // [n_pad] row index of a target position, or -1
+  int32_t* d_sout_rows = nullptr;  // [rows_out] source positions
+  int32_t* d_sout_poff = nullptr;  // [rows_out + 1] pair ranges of each row
+  int32_t* d_pair_type = nullptr;  // [pairs]
+  int32_t* d_pair_off = nullptr;   // [pairs + 1] edge ranges of each pair
+  int32_t* d_pair_row = nullptr;   // [pairs] index into rows_out
+  int32_t* d_sout_dst = nullptr;   // [n_super_edges] sorted by (type, target) within a row
+  int32_t* d_type_off = nullptr;   // [P + 1] ranges of d_type_pairs per type
+  int32_t* d_type_pairs = nullptr; // [pairs] pair ids grouped by type, ascending row
+  int64_t n_super_edges() const { return (int64_t)sup_edges.size() / 3; }
   // device copies (valid once uploaded)
   int device = -1;
   uint32_t* d_masks = nullptr;
@@ -56,4 +79,4 @@ int bg_noalloc_prepare(const bg_plan* p);
 
 // planner entry (plan.cpp)
 int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S, int32_t cap,
-                  uint32_t flags, bg_plan** out);
+                  uint32_t flags, int32_t super_min_degree, int32_t max_super, bg_plan** out);

@@ -20,6 +20,7 @@
 #include "band_tc.h"
 #include "internal.h"
 #include "kernels.h"
+#include "super.h"
 
 namespace {
 
@@ -68,6 +69,7 @@ int bg_noalloc_prepare(const bg_plan* p) {
   if (rc != BG_OK) return rc;
   e = bg::preload_fwd_simt();
   if (e == cudaSuccess && p->d_maskI) e = bg::band_tc_preload_fwd(p);
+  if (e == cudaSuccess) e = bg::super_preload_fwd();
   if (e != cudaSuccess) return bg_fail(BG_ECUDA, std::string("kernel load: ") + cudaGetErrorString(e));
   return BG_OK;
 }
@@ -122,6 +124,8 @@ extern "C" int bg_band_propagate_fwd_noalloc(const bg_plan* p, bg_dtype dt, int3
       e = bg::band_fwd_gather(p->d_masks, reinterpret_cast<float*>(scratch), Y, p->K, p->S, p->P,
                               H, st);
   }
+  // the supernode rows and columns (no scratch: added to Y in place)
+  if (e == cudaSuccess) e = bg::super_fwd(p, dt == BG_BF16, H, E, W, b, Y, 0, st);
   if (e != cudaSuccess) return bg_fail(BG_ECUDA, std::string("launch: ") + cudaGetErrorString(e));
   return BG_OK;
 }

@@ -142,7 +142,7 @@ void reverse_cuthill_mckee(int32_t n, int64_t m, const int32_t* src, const int32
 }  // namespace
 
 int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S, int32_t cap,
-                  uint32_t flags, bg_plan** out) {
+                  uint32_t flags, int32_t super_min_degree, int32_t max_super, bg_plan** out) {
   if (!out) return bg_fail(BG_EINVAL, "out is NULL");
   *out = nullptr;
   if (n_graphs < 1 || (!graphs)) return bg_fail(BG_EINVAL, "need at least one graph");
@@ -150,6 +150,9 @@ int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S
     return bg_fail(BG_EINVAL, "block size S must be one of 32, 64, 128, 256, 512");
   if (P < 1 || P > 64) return bg_fail(BG_EINVAL, "n_types must be in [1, 64]");
   if (cap < 0) return bg_fail(BG_EINVAL, "capacity_blocks must be >= 0");
+  const bool supernodes = (flags & BG_SUPERNODES) != 0;
+  if (supernodes && (super_min_degree < 1 || max_super < 0))
+    return bg_fail(BG_EINVAL, "supernodes need supernode_min_degree >= 1 and max_supernodes >= 0");
   for (int32_t g = 0; g < n_graphs; ++g) {
     const bg_graph& gr = graphs[g];
     if (gr.n_nodes < 0 || gr.n_edges < 0)
@@ -198,23 +201,68 @@ int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S
   pl->perm.resize(total);
   pl->bw_before.assign(n_graphs, 0);
   pl->bw_after.assign(n_graphs, 0);
+  pl->nsup.assign(n_graphs, 0);
   std::atomic<int32_t> next{0};
   auto worker = [&]() {
     for (;;) {
       int32_t g = next.fetch_add(1);
       if (g >= n_graphs) return;
       const bg_graph& gr = graphs[g];
+      const int32_t n = gr.n_nodes;
       int32_t* pg = pl->perm.data() + pl->node_base[g];
-      if (flags & BG_RCM) {
-        reverse_cuthill_mckee(gr.n_nodes, gr.n_edges, gr.src, gr.dst,
-                              (flags & BG_KEEP_IF_BETTER) != 0, pg);
-      } else {
-        for (int32_t i = 0; i < gr.n_nodes; ++i) pg[i] = i;
+      // supernodes: degree (distinct neighbours, self-loops not counted) at least the threshold,
+      // highest degree first, ties by id, at most max_super; they take the first positions
+      std::vector<int32_t> sup;
+      if (supernodes && max_super > 0) {
+        Csr c = build_csr(n, gr.n_edges, gr.src, gr.dst);
+        for (int32_t v = 0; v < n; ++v)
+          if (c.deg(v) >= super_min_degree) sup.push_back(v);
+        std::sort(sup.begin(), sup.end(), [&](int32_t a, int32_t b) {
+          return c.deg(a) != c.deg(b) ? c.deg(a) > c.deg(b) : a < b;
+        });
+        if ((int32_t)sup.size() > max_super) sup.resize(max_super);
       }
-      std::vector<int32_t> where(gr.n_nodes);
-      for (int32_t i = 0; i < gr.n_nodes; ++i) where[pg[i]] = i;
+      pl->nsup[g] = (int32_t)sup.size();
+      std::vector<char> is_sup(n, 0);
+      for (int32_t v : sup) is_sup[v] = 1;
+      if (sup.empty()) {
+        if (flags & BG_RCM) {
+          reverse_cuthill_mckee(n, gr.n_edges, gr.src, gr.dst, (flags & BG_KEEP_IF_BETTER) != 0, pg);
+        } else {
+          for (int32_t i = 0; i < n; ++i) pg[i] = i;
+        }
+      } else {
+        // the graph without its supernodes, renumbered in ascending id, ordered on its own
+        std::vector<int32_t> rest, rid(n, -1), rs, rd;
+        for (int32_t v = 0; v < n; ++v)
+          if (!is_sup[v]) { rid[v] = (int32_t)rest.size(); rest.push_back(v); }
+        for (int64_t e = 0; e < gr.n_edges; ++e)
+          if (!is_sup[gr.src[e]] && !is_sup[gr.dst[e]]) { rs.push_back(rid[gr.src[e]]); rd.push_back(rid[gr.dst[e]]); }
+        const int32_t nr = (int32_t)rest.size();
+        std::vector<int32_t> pr(nr);
+        if (flags & BG_RCM) {
+          reverse_cuthill_mckee(nr, (int64_t)rs.size(), rs.data(), rd.data(),
+                                (flags & BG_KEEP_IF_BETTER) != 0, pr.data());
+        } else {
+          for (int32_t i = 0; i < nr; ++i) pr[i] = i;
+        }
+        for (size_t i = 0; i < sup.size(); ++i) pg[i] = sup[i];
+        for (int32_t i = 0; i < nr; ++i) pg[sup.size() + i] = rest[pr[i]];
+      }
+      std::vector<int32_t> where(n);
+      for (int32_t i = 0; i < n; ++i) where[pg[i]] = i;
       pl->bw_before[g] = bandwidth_of(gr.n_edges, gr.src, gr.dst, nullptr);
-      pl->bw_after[g] = bandwidth_of(gr.n_edges, gr.src, gr.dst, where.data());
+      if (sup.empty()) {
+        pl->bw_after[g] = bandwidth_of(gr.n_edges, gr.src, gr.dst, where.data());
+      } else {
+        int64_t bw = 0;
+        for (int64_t e = 0; e < gr.n_edges; ++e)
+          if (!is_sup[gr.src[e]] && !is_sup[gr.dst[e]]) {
+            const int64_t a = where[gr.src[e]], b = where[gr.dst[e]];
+            bw = std::max(bw, a > b ? a - b : b - a);
+          }
+        pl->bw_after[g] = bw;
+      }
     }
   };
   unsigned nt = std::max(1u, std::min(std::thread::hardware_concurrency(), 16u));
@@ -236,6 +284,7 @@ int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S
     pl->bw_before_max = std::max(pl->bw_before_max, pl->bw_before[g]);
     pl->bw_after_max = std::max(pl->bw_after_max, pl->bw_after[g]);
     pl->n_edges_in += gr.n_edges;
+    pl->n_super += pl->nsup[g];
   }
 
   // Deduplicated edges in supergraph positions and their bits, graph by graph on the host
@@ -247,6 +296,7 @@ int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S
   pl->masks.assign(nwords, 0u);
   pl->masksT.assign(nwords, 0u);
   std::vector<int64_t> uniq(pl->n_packed, 0), kept(pl->n_packed, 0), dropped(pl->n_packed, 0);
+  std::vector<std::vector<int32_t>> sup_e(pl->n_packed);
   std::atomic<int32_t> next_g{0};
   auto edge_worker = [&]() {
     std::vector<uint64_t> keys;
@@ -269,10 +319,17 @@ int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S
       std::sort(keys.begin(), keys.end());
       keys.erase(std::unique(keys.begin(), keys.end()), keys.end());
       uniq[g] = (int64_t)keys.size();
+      const int64_t sup_end = o + pl->nsup[g];  // the graph's supernodes: positions [o, sup_end)
       for (uint64_t key : keys) {
         const int64_t i = (int64_t)(key >> 34);
         const int64_t j = (int64_t)((key >> 6) & ((1ull << 28) - 1));
         const int32_t p = (int32_t)(key & 63);
+        if (i < sup_end || j < sup_end) {
+          // a supernode end: kept, propagated by the supernode rows and columns
+          ++kept[g];
+          sup_e[g].insert(sup_e[g].end(), {(int32_t)i, (int32_t)j, p});
+          continue;
+        }
         const int64_t bi = i / S, bj = j / S;
         if (bj - bi < -1 || bj - bi > 1) { ++dropped[g]; continue; }
         ++kept[g];
@@ -296,6 +353,8 @@ int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S
     pl->n_unique += uniq[g];
     pl->n_kept += kept[g];
     pl->n_dropped += dropped[g];
+    // graphs occupy ascending position ranges, so the concatenation stays sorted
+    pl->sup_edges.insert(pl->sup_edges.end(), sup_e[g].begin(), sup_e[g].end());
   }
   *out = pl;
   return BG_OK;

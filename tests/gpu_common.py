@@ -66,11 +66,17 @@ def f32_dev(x) -> torch.Tensor:
 class Case:
     """A planned, uploaded supergraph with packed device states and the oracle's view of it."""
 
-    def __init__(self, graphs, P, S, H, dtype, seed=0, cap=0, plain_xavier=False):
+    def __init__(self, graphs, P, S, H, dtype, seed=0, cap=0, plain_xavier=False, sup=None):
         self.P, self.S, self.H, self.dtype = P, S, H, dtype
-        self.plan = L.band_plan(graphs, P, S, cap)
+        if sup:  # (supernode_min_degree, max_supernodes)
+            F = L.BG_RCM | L.BG_KEEP_IF_BETTER | L.BG_SUPERNODES
+            self.plan = L.band_plan(graphs, P, S, cap, F, *sup)
+            self.ref = oracle.layout(graphs, P, S, cap, flags=F, super_min_degree=sup[0],
+                                     max_super=sup[1])
+        else:
+            self.plan = L.band_plan(graphs, P, S, cap)
+            self.ref = oracle.layout(graphs, P, S, cap)
         self.plan.upload()
-        self.ref = oracle.layout(graphs, P, S, cap)
         info = self.plan.info()
         self.info = info
         self.N = info["n_pad"]

@@ -203,3 +203,51 @@ def test_reach_filtered_batch_gives_the_full_graphs_candidate_states():
         got_c.append(got[off[i] + m[cand]])
         want_c.append(Es[T][cand])
     assert_close(np.concatenate(got_c), np.concatenate(want_c), TOL["bf16"], "E(T) at candidates")
+
+
+# ------------------------------------------------------------------------ supernodes (Section 6)
+
+
+def _two_way_hub(n_leaves, seed, back_type=5):
+    """A hub graph whose hub also sends one edge back to every node (a supernode's full row and
+    column)."""
+    h = synth.hub_graph(n_leaves, 20, seed, lam=2.0)
+    hub = int(np.bincount(h.dst[h.etype == 0]).argmax())
+    back = h.src[h.etype == 0]
+    return synth.Graph(h.n_nodes, np.concatenate([h.src, np.full(len(back), hub, np.int32)]),
+                       np.concatenate([h.dst, back]),
+                       np.concatenate([h.etype, np.full(len(back), back_type, np.int32)]), 20)
+
+
+def _super_case(S, H, dtype, seed, leaves=(300, 150)):
+    gs = synth.gen_batch(4, 100, 600, 10, True, S // 2, S // 3, 2.0, seed)
+    gs.insert(1, _two_way_hub(leaves[0], seed + 1))
+    gs.insert(3, _two_way_hub(leaves[1], seed + 2, back_type=13))
+    n = sum(g.n_nodes for g in gs)
+    per = max(1, 128 // S)
+    cap = -(-(-(-n // S)) // per) * per
+    c = Case(gs, 20, S, H, dtype, seed=seed, cap=cap, sup=(100, 2))
+    assert c.plan.info()["n_super"] == 2 and c.plan.info()["n_super_edges"] > 4 * 150
+    return c
+
+
+@pytest.mark.parametrize("dtype,S,H", [("bf16", 128, 64), ("bf16", 32, 128), ("bf16", 128, 256),
+                                       ("bf16", 512, 64), ("f32", 64, 64), ("bf16", 128, 96)])
+def test_supernode_propagation(dtype, S, H):
+    """Supernodes (Section 6): two hub graphs whose hub exchanges edges with every node; the
+    hubs take their graphs' first positions, their edges are kept and propagated beside the band
+    (forward: added to Y; backward: to dE, dW and db), on the tensor-core path, on the fp32 SIMT
+    path and on the bf16 SIMT path (H = 96)."""
+    c = _super_case(S, H, dtype, 700 + S + H)
+    tc = dtype == "bf16" and H != 96
+    assert L.band_uses_tensor_cores(c.plan, dtype, H) == tc
+    _check_propagation(c, 701)
+
+
+@pytest.mark.parametrize("S,H", [(128, 64), (64, 128), (128, 32), (128, 256)])
+def test_supernode_ggnn(S, H):
+    """T = 2 GGNN steps with supernodes, forward and backward: on the fused tensor-core path the
+    supernode rows' messages are added by the band kernel before it rounds Y (H = 32, 64, 128),
+    and their gradients after each step's band backward; H = 256 takes the GEMM path."""
+    c = _super_case(S, H, "bf16", 800 + S + H)
+    _ggnn_check(c, 2, 801)

@@ -277,3 +277,49 @@ def test_reach_filter_bit_exact_against_the_oracle(T):
             np.testing.assert_array_equal(a, b)
     with pytest.raises(L.BandGGNNError):
         L.reach_filter(g, [g.n_nodes], T)
+
+
+def _hub_batch(S, seed):
+    """Program-shaped graphs with hubs: two hub graphs (one node sending to and receiving from
+    every other node) among ordinary ones."""
+    gs = synth.gen_batch(4, 100, max(3 * S, 300), 5, True, max(2, S // 2), max(2, S // 3), 1.5,
+                         seed)
+    for i, k in ((1, 3 * S), (3, S + 7)):
+        h = synth.hub_graph(k, 10, seed + i, lam=1.0)
+        hub = int(np.bincount(h.dst[h.etype == 0]).argmax())
+        back = h.src[h.etype == 0]
+        gs.insert(i, synth.Graph(h.n_nodes, np.concatenate([h.src, np.full(len(back), hub, np.int32)]),
+                                 np.concatenate([h.dst, back]),
+                                 np.concatenate([h.etype, np.full(len(back), 5, np.int32)]), 10))
+    return gs
+
+
+@pytest.mark.parametrize("S,min_deg,max_sup", [(32, 64, 4), (128, 100, 2), (512, 40, 8),
+                                               (64, 1000000, 4)])
+def test_planner_bit_exact_with_supernodes(S, min_deg, max_sup):
+    """Supernodes (Section 6): the library's positions, band tiles, counts and supernode edge
+    list equal the oracle's independent layout; every edge with a supernode end is kept, and the
+    band masks hold the other kept edges only."""
+    gs = _hub_batch(S, 60 + S)
+    F = L.BG_RCM | L.BG_KEEP_IF_BETTER | L.BG_SUPERNODES
+    plan = L.band_plan(gs, 10, S, 0, F, min_deg, max_sup)
+    ref = oracle.layout(gs, 10, S, flags=F, super_min_degree=min_deg, max_super=max_sup)
+    info = plan.info()
+    for k in ("K", "n_packed", "n_real"):
+        assert info[k] == getattr(ref, k)
+    assert info["n_kept"] == ref.n_kept and info["n_dropped"] == ref.n_dropped
+    assert info["bw_after_max"] == ref.bw_after_max and info["n_edges_unique"] == ref.n_unique
+    np.testing.assert_array_equal(plan.export(L.BG_EXPORT_PERM), ref.perm)
+    assert plan.export(L.BG_EXPORT_MASKS).tobytes() == ref.masks.tobytes()
+    sup = plan.export(L.BG_EXPORT_SUPER_EDGES)
+    want = np.stack([ref.kept_dst, ref.kept_src, ref.kept_type], 1)[ref.kept_super]
+    np.testing.assert_array_equal(sup, want)
+    assert info["n_super_edges"] == len(want) and info["n_super"] == ref.is_super.sum()
+    counts = plan.export(L.BG_EXPORT_SUPER_COUNT)
+    assert counts.sum() >= info["n_super"]
+    if min_deg < 1000:
+        assert info["n_super"] > 0 and len(want) > 0
+        plain = L.band_plan(gs, 10, S)
+        assert plain.info()["n_dropped"] > info["n_dropped"]
+    else:
+        assert info["n_super"] == 0 and len(want) == 0

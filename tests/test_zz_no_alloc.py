@@ -113,3 +113,16 @@ def test_noalloc_timeouts_reach_bg_check_device():
     assert "BG_ETIMEOUT" in str(err.value)
     L.band_propagate_fwd_noalloc(c.plan, c.dtype, c.H, c.E_band_dev, c.dprm["W"], c.dprm["b"], Y)
     L.check_device()
+
+
+def test_noalloc_with_supernodes():
+    """A plan with supernodes: their rows and columns are added to Y in place, with no scratch;
+    the result equals the workspace entry point's, on two calls in a row."""
+    gs = synth.gen_batch(4, 100, 500, 10, True, 48, 32, 2.0, 21)
+    g = synth.hub_graph(260, 20, 22, lam=2.0)
+    gs.insert(1, g)
+    c = Case(gs, 20, 128, 64, "bf16", seed=8, sup=(100, 1))
+    assert c.plan.info()["n_super"] == 1
+    for E_dev, b in ((c.E_band_dev, c.dprm["b"]), (c.E_band_dev, None)):
+        got, want, grew = _both(c, E_dev, b)
+        assert _rel(got, want) < TOL["bf16"] and grew == 0
