@@ -152,6 +152,34 @@ double bg_plan_flops(const bg_plan* plan, int32_t H, int32_t which);
 size_t bg_plan_export_bytes(const bg_plan* plan, int32_t which);
 int bg_plan_export(const bg_plan* plan, int32_t which, void* out, size_t out_bytes);
 
+/* Block-row partition for running one supergraph on several GPUs (Eq. 3: block-row k couples
+ * only to block-rows k - 1 and k + 1).  Part `part` of n_parts owns a contiguous range of whole
+ * 128-row tiles (max(1, 128 / S) block-rows each; ranges as equal as the tile count allows) and
+ * gets a local plan (free it with bg_plan_free; upload it like any plan) over that range plus one
+ * tile of halo on each side, clipped at the supergraph's ends.  Local row i is supergraph
+ * position row0 + i.  The local forward tiles keep only the rows the part owns as targets, the
+ * transposed tiles only the rows it owns as sources.  Used with bg_band_propagate_fwd/bwd:
+ *   forward:  fill the local E with rows [row0, row0 + n_local) of the full E -- the halo rows
+ *             [0, own_begin) and [own_end, n_local) from the neighbouring parts -- and the own
+ *             rows of Y are exact (the halo rows of Y come out 0);
+ *   backward: likewise for dY; the own rows of dE are exact (halo rows 0), and dW, db are the
+ *             sums over the part's own source rows, so their sum over all parts (an all-reduce)
+ *             is the whole plan's.
+ * One halo exchange per direction per step: halo_lo rows from part - 1, halo_hi rows from
+ * part + 1 (0 at the ends).  The local plan has no graph table (no pack/unpack or readout) and
+ * n_real = the real positions of its range.  Plans with supernodes are not partitioned
+ * (BG_EINVAL).  Host only. */
+typedef struct bg_part_info {
+  int32_t row0;      /* supergraph position of local row 0 */
+  int32_t n_local;   /* local rows (the local plan's n_pad) */
+  int32_t own_begin; /* local rows [own_begin, own_end) are the part's own */
+  int32_t own_end;
+  int32_t halo_lo;   /* rows before own_begin (from part - 1), = own_begin */
+  int32_t halo_hi;   /* rows from own_end on (from part + 1), = n_local - own_end */
+} bg_part_info;
+int bg_plan_partition(const bg_plan* full, int32_t n_parts, int32_t part, bg_plan** out,
+                      bg_part_info* info);
+
 /* Copy the plan's tiles and index tables to the current CUDA device (plan-owned memory, freed by
  * bg_plan_free).  Must precede every device call with this plan; a plan serves one device. */
 int bg_plan_upload(bg_plan* plan, void* stream);

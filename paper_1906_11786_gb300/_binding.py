@@ -53,6 +53,11 @@ class bg_plan_opts(ctypes.Structure):
                 ("max_supernodes", ctypes.c_int32)]
 
 
+class bg_part_info(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in ("row0", "n_local", "own_begin", "own_end", "halo_lo",
+                                              "halo_hi")]
+
+
 class bg_params(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in ("W", "b", "W_ih", "W_hh", "b_ih", "b_hh")]
 
@@ -106,6 +111,7 @@ def load(path: str = LIB_PATH):
         "bg_launch_count": (i64, []),
         "bg_band_uses_tensor_cores": (c.c_int, [vp, c.c_int, i32]),
         "bg_reach_filter": (c.c_int, [vp, vp, i32, i32, vp, vp, vp, vp, vp, vp]),
+        "bg_plan_partition": (c.c_int, [vp, i32, i32, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -242,6 +248,14 @@ def band_plan(graphs, n_types, block_S, capacity_blocks=0, flags=BG_RCM | BG_KEE
         _check(lib.bg_band_plan(arr, len(graphs), n_types, block_S, capacity_blocks, flags,
                                 ctypes.byref(h)))
     return Plan(h.value, n_types)
+
+
+def plan_partition(plan, n_parts, part):
+    """bg_plan_partition: (local Plan, info dict) of part `part` of a block-row split."""
+    h = ctypes.c_void_p()
+    info = bg_part_info()
+    _check(load().bg_plan_partition(plan.handle, n_parts, part, ctypes.byref(h), ctypes.byref(info)))
+    return Plan(h.value, plan.P), {f: getattr(info, f) for f, _ in bg_part_info._fields_}
 
 
 def reach_filter(graph, candidates, T):

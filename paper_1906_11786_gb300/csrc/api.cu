@@ -208,6 +208,16 @@ extern "C" int bg_band_plan_opts(const bg_graph* graphs, int32_t n_graphs, int32
   }
 }
 
+extern "C" int bg_plan_partition(const bg_plan* full, int32_t n_parts, int32_t part,
+                                 bg_plan** out, bg_part_info* info) {
+  bg_clear_error();
+  try {
+    return bg_plan_partition_build(full, n_parts, part, out, info);
+  } catch (const std::bad_alloc&) {
+    return bg_fail(BG_ENOMEM, "host allocation failed");
+  }
+}
+
 static void free_device(bg_plan* p) {
   if (p->device < 0) return;
   int prev = 0;

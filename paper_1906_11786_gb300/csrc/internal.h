@@ -77,6 +77,10 @@ int* bg_status_word_if_created(int dev);
 // size.  Called by bg_plan_upload, which allocates anyway.
 int bg_noalloc_prepare(const bg_plan* p);
 
+// block-row partition (plan.cpp)
+int bg_plan_partition_build(const bg_plan* full, int32_t n_parts, int32_t part, bg_plan** out,
+                            bg_part_info* info);
+
 // planner entry (plan.cpp)
 int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S, int32_t cap,
                   uint32_t flags, int32_t super_min_degree, int32_t max_super, bg_plan** out);

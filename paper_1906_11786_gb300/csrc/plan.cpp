@@ -359,3 +359,51 @@ int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S
   *out = pl;
   return BG_OK;
 }
+
+// Block-row partition of a plan (Eq. 3: block-row k couples only to block-rows k - 1 and k + 1).
+// Part `part` of n_parts owns a contiguous range of whole 128-row tiles (of max(1, 128 / S)
+// block-rows each); its local plan spans that range plus one tile of halo on each side (clipped
+// at the ends).  The forward tiles keep only the rows the part owns as targets and the
+// transposed tiles only the rows it owns as sources, so with the halo rows of E (forward) or dY
+// (backward) copied in from the neighbours the part's own rows of Y and dE are exact, the halo
+// rows of Y and dE come out 0, and its dW, db are the sums over its own source rows: summed over
+// the parts they give the whole plan's.
+int bg_plan_partition_build(const bg_plan* full, int32_t n_parts, int32_t part, bg_plan** out,
+                            bg_part_info* info) {
+  if (!full || !out || !info) return bg_fail(BG_EINVAL, "NULL argument");
+  *out = nullptr;
+  if (full->n_super > 0) return bg_fail(BG_EINVAL, "plans with supernodes cannot be partitioned");
+  const int32_t S = full->S, K = full->K, P = full->P;
+  const int32_t unit = S >= 128 ? 1 : 128 / S;  // block-rows per tile
+  const int32_t n_units = (K + unit - 1) / unit;
+  if (n_parts < 1 || n_parts > n_units) return bg_fail(BG_EINVAL, "n_parts must be in [1, tiles]");
+  if (part < 0 || part >= n_parts) return bg_fail(BG_EINVAL, "part out of range");
+  const int32_t u0 = (int32_t)((int64_t)n_units * part / n_parts);
+  const int32_t u1 = (int32_t)((int64_t)n_units * (part + 1) / n_parts);
+  const int32_t k0 = u0 * unit, k1 = std::min(K, u1 * unit);  // own block-rows [k0, k1)
+  const int32_t kb0 = std::max(0, k0 - unit), kb1 = std::min(K, k1 + unit);  // with the halo
+  bg_plan* pl = new (std::nothrow) bg_plan();
+  if (!pl) return bg_fail(BG_ENOMEM, "host allocation failed");
+  pl->S = S; pl->P = P; pl->W32 = full->W32; pl->K = kb1 - kb0;
+  pl->n_graphs = 0; pl->n_packed = 0;
+  const int64_t row0 = (int64_t)kb0 * S;
+  pl->n_real = (int32_t)std::max<int64_t>(0, std::min<int64_t>((int64_t)pl->K * S, full->n_real - row0));
+  const size_t tile_words = (size_t)3 * P * S * full->W32;  // one block-row of tiles
+  pl->masks.assign((size_t)pl->K * tile_words, 0u);
+  pl->masksT.assign((size_t)pl->K * tile_words, 0u);
+  for (int32_t k = k0; k < k1; ++k) {
+    const size_t src = (size_t)k * tile_words, dst = (size_t)(k - kb0) * tile_words;
+    std::memcpy(pl->masks.data() + dst, full->masks.data() + src, tile_words * 4);
+    std::memcpy(pl->masksT.data() + dst, full->masksT.data() + src, tile_words * 4);
+  }
+  for (uint32_t w : pl->masks) pl->n_kept += __builtin_popcount(w);
+  pl->n_unique = pl->n_kept;
+  info->row0 = (int32_t)row0;
+  info->n_local = pl->K * S;
+  info->own_begin = (k0 - kb0) * S;
+  info->own_end = (k1 - kb0) * S;
+  info->halo_lo = (k0 - kb0) * S;
+  info->halo_hi = (kb1 - k1) * S;
+  *out = pl;
+  return BG_OK;
+}

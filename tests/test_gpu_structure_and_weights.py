@@ -255,3 +255,62 @@ def test_supernode_ggnn(S, H):
     itself stayed at 5e-5 (measured)."""
     c = _super_case(S, H, "bf16", 800 + S + H, leaves=(160, 100))
     _ggnn_check(c, 2, 801)
+
+
+# ------------------------------------------------------------------------ block-row split
+
+
+@pytest.mark.parametrize("S,H,n_parts", [(128, 64, 2), (32, 128, 3), (256, 64, 2)])
+def test_block_row_split_on_one_gpu_matches_the_unsplit_launch(S, H, n_parts):
+    """Several parts of one plan (bg_plan_partition) run on one GPU one after another, their
+    halo rows of E (forward) and dY (backward) copied from the neighbouring parts' own rows: the
+    own rows of Y and dE equal the unsplit launch's (same tiles, same sums), the halo rows of Y
+    come out 0, and the parts' dW, db sum to the unsplit ones."""
+    from paper_1906_11786_gb300 import halo
+    gs = synth.gen_batch(12, 200, 1200, 10, True, S // 2, S // 3, 2.0, 900 + S)
+    n = sum(g.n_nodes for g in gs)
+    unit = max(1, 128 // S)
+    c = Case(gs, 20, S, H, "bf16", seed=9, cap=-(-(-(-n // S)) // unit) * unit)
+    dY, (Y, dE, dW, db) = _propagate(c, 901)
+    parts = [L.plan_partition(c.plan, n_parts, r) for r in range(n_parts)]
+    for sub, _ in parts:
+        sub.upload()
+    infos = [inf for _, inf in parts]
+    E_all = c.E_band_dev
+    Ys, dEs, sW, sb = [], [], np.zeros_like(dW), np.zeros_like(db)
+    El = [torch.zeros((inf["n_local"], H), dtype=E_all.dtype, device="cuda") for inf in infos]
+    dYl = [torch.zeros((inf["n_local"], H), dtype=torch.float32, device="cuda") for inf in infos]
+    dY_dev = f32_dev(dY)
+    for inf, e, g in zip(infos, El, dYl):
+        r0, ob, oe = inf["row0"], inf["own_begin"], inf["own_end"]
+        e[ob:oe] = E_all[r0 + ob:r0 + oe]
+        g[ob:oe] = dY_dev[r0 + ob:r0 + oe]
+    # the halo exchange: one copy per neighbour and direction (here within one device)
+    for r, cps in enumerate(halo.halo_plan(infos)):
+        for src, s0, d0, rows in cps:
+            El[r][d0:d0 + rows] = El[src][s0:s0 + rows]
+            dYl[r][d0:d0 + rows] = dYl[src][s0:s0 + rows]
+    for (sub, inf), e, g in zip(parts, El, dYl):
+        assert L.band_uses_tensor_cores(sub, "bf16", H)
+        nl = inf["n_local"]
+        Yl = torch.empty((nl, H), device="cuda")
+        L.band_propagate_fwd(sub, "bf16", H, e, c.dprm["W"], c.dprm["b"], Yl,
+                             torch.empty(L.workspace_bytes(sub, "bf16", H, L.BG_OP_PROPAGATE_FWD),
+                                         dtype=torch.uint8, device="cuda"))
+        dEl = torch.empty((nl, H), device="cuda")
+        dWl = torch.empty((c.P, H, H), device="cuda")
+        dbl = torch.empty((c.P, H), device="cuda")
+        L.band_propagate_bwd(sub, "bf16", H, e, c.dprm["W"], g, dEl, dWl, dbl,
+                             torch.empty(L.workspace_bytes(sub, "bf16", H, L.BG_OP_PROPAGATE_BWD),
+                                         dtype=torch.uint8, device="cuda"))
+        torch.cuda.synchronize()
+        L.check_device()
+        Yl, dEl = Yl.cpu().numpy(), dEl.cpu().numpy()
+        r0, ob, oe = inf["row0"], inf["own_begin"], inf["own_end"]
+        np.testing.assert_allclose(Yl[ob:oe], Y[r0 + ob:r0 + oe], rtol=1e-6, atol=1e-5)
+        np.testing.assert_allclose(dEl[ob:oe], dE[r0 + ob:r0 + oe], rtol=1e-6, atol=1e-5)
+        assert not Yl[:ob].any() and not Yl[oe:].any()
+        sW += dWl.cpu().numpy()
+        sb += dbl.cpu().numpy()
+    np.testing.assert_allclose(sW, dW, rtol=1e-4, atol=1e-3 * np.abs(dW).max())
+    np.testing.assert_allclose(sb, db, rtol=1e-4, atol=1e-3 * np.abs(db).max())

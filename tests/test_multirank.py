@@ -99,3 +99,78 @@ def test_single_process_gradients_untouched():
     flat = torch.arange(5, dtype=torch.float32)
     bench.allreduce_grads(None, flat)
     assert flat.tolist() == [0.0, 1.0, 2.0, 3.0, 4.0]
+
+
+def _split_worker(rank, world, port, out):
+    """One rank of a block-row split: plans the whole supergraph, takes its part, fills its own
+    rows of E and dY, exchanges the halo rows with its neighbour, propagates its part forward and
+    backward with the oracle on its local tiles, sums dW and db over the ranks."""
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    import numpy as np
+
+    import oracle
+    from paper_1906_11786_gb300 import _binding as L
+    from paper_1906_11786_gb300 import halo, synth
+    from test_plan_abi import edges_from_masks
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        P, S, H = 8, 64, 16
+        gs = synth.gen_batch(10, 100, 500, 4, True, 32, 20, 2.0, 808)
+        n = sum(g.n_nodes for g in gs)
+        cap = -(-(-(-n // S)) // 2) * 2
+        full = L.band_plan(gs, P, S, cap)
+        N = full.info()["n_pad"]
+        rng = np.random.default_rng(1)
+        E = rng.standard_normal((N, H)); dY = rng.standard_normal((N, H))
+        prm = synth.gen_params(P, H, 2)
+        sub, inf = L.plan_partition(full, world, rank)
+        r0, nl, ob, oe = inf["row0"], inf["n_local"], inf["own_begin"], inf["own_end"]
+        El = torch.zeros((nl, H), dtype=torch.float64)
+        El[ob:oe] = torch.from_numpy(E[r0 + ob:r0 + oe])
+        halo.exchange(El, inf, rank, world)
+        dYl = torch.zeros((nl, H), dtype=torch.float64)
+        dYl[ob:oe] = torch.from_numpy(dY[r0 + ob:r0 + oe])
+        halo.exchange(dYl, inf, rank, world)
+        # the halo rows now hold the neighbours' rows of the full arrays
+        halo_ok = bool(np.array_equal(El.numpy(), E[r0:r0 + nl]) and
+                       np.array_equal(dYl.numpy(), dY[r0:r0 + nl]))
+        fe = edges_from_masks(sub.export(L.BG_EXPORT_MASKS), S)
+        Yl = oracle.propagate_fwd(nl, P, H, *fe, El.numpy(), prm["W"], prm["b"])
+        te = edges_from_masks(sub.export(L.BG_EXPORT_MASKS_T), S, transposed=True)
+        dEl, dWl, dbl = oracle.propagate_bwd(nl, P, H, *te, El.numpy(), prm["W"], dYl.numpy())
+        dW_t, db_t = torch.from_numpy(dWl), torch.from_numpy(dbl)
+        halo.allreduce_sum([dW_t, db_t])
+        # the whole plan, on every rank, for comparison
+        ge = edges_from_masks(full.export(L.BG_EXPORT_MASKS), S)
+        Y = oracle.propagate_fwd(N, P, H, *ge, E, prm["W"], prm["b"])
+        dE, dW, db = oracle.propagate_bwd(N, P, H, *ge, E, prm["W"], dY)
+        own = slice(r0 + ob, r0 + oe)
+        out[rank] = (halo_ok,
+                     float(np.max(np.abs(Yl[ob:oe] - Y[own]))),
+                     float(np.max(np.abs(Yl[:ob])) if ob else 0.0) + float(np.max(np.abs(Yl[oe:])) if oe < nl else 0.0),
+                     float(np.max(np.abs(dEl[ob:oe] - dE[own]))),
+                     float(np.max(np.abs(dW_t.numpy() - dW))), float(np.max(np.abs(db_t.numpy() - db))),
+                     oe - ob)
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.timeout(300)
+def test_block_row_split_two_ranks_matches_the_whole_plan():
+    """The block-row split (bg_plan_partition) on two gloo ranks with halo.exchange: each rank's
+    own rows of Y and dE equal the whole plan's, its halo rows of Y are 0, and the all-reduced
+    dW, db equal the whole plan's (fp64 oracle arithmetic on both sides)."""
+    world = 2
+    port = _free_port()
+    mgr = mp.get_context("spawn").Manager()
+    out = mgr.dict()
+    mp.start_processes(_split_worker, args=(world, port, out), nprocs=world, start_method="spawn")
+    rows = 0
+    for r in range(world):
+        halo_ok, eY, eYhalo, edE, edW, edb, own = out[r]
+        assert halo_ok
+        assert eY < 1e-12 and eYhalo == 0.0 and edE < 1e-12
+        assert edW < 1e-9 and edb < 1e-9
+        rows += own
+    assert rows > 0

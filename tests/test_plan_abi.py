@@ -323,3 +323,54 @@ def test_planner_bit_exact_with_supernodes(S, min_deg, max_sup):
         assert plain.info()["n_dropped"] > info["n_dropped"]
     else:
         assert info["n_super"] == 0 and len(want) == 0
+
+
+def edges_from_masks(m, S, transposed=False):
+    """(dst, src, type) of the set bits of exported forward (or transposed) band masks."""
+    bits = np.unpackbits(m, axis=-1, bitorder="little")
+    k, d, p, r, c = np.nonzero(bits)
+    a, b = k.astype(np.int64) * S + r, (k.astype(np.int64) + d - 1) * S + c
+    return (b, a, p) if transposed else (a, b, p)
+
+
+@pytest.mark.parametrize("S,n_parts", [(32, 2), (128, 3), (256, 2), (64, 5)])
+def test_partition_tiles_rows_and_halos(S, n_parts):
+    """Block-row split (Eq. 3): the parts own contiguous whole-tile ranges covering the
+    supergraph; each local plan spans its range plus one tile of halo per side; its forward
+    tiles hold exactly the kept edges whose target it owns and its transposed tiles those whose
+    source it owns, in local positions."""
+    gs = synth.gen_batch(8, 100, 600, 4, True, max(2, S // 2), max(2, S // 3), 1.5, 5 + S)
+    n = sum(g.n_nodes for g in gs)
+    unit = max(1, 128 // S)
+    cap = -(-(-(-n // S)) // unit) * unit
+    full = L.band_plan(gs, 8, S, cap)
+    fi = full.info()
+    d, s_, t = edges_from_masks(full.export(L.BG_EXPORT_MASKS), S)
+    pos_all = []
+    for part in range(n_parts):
+        sub, inf = L.plan_partition(full, n_parts, part)
+        si = sub.info()
+        assert si["n_pad"] == inf["n_local"] and inf["n_local"] % 128 == 0
+        assert inf["halo_lo"] == inf["own_begin"] and inf["halo_hi"] == inf["n_local"] - inf["own_end"]
+        assert inf["halo_lo"] == (0 if part == 0 else max(S, 128))
+        assert inf["halo_hi"] == (0 if part == n_parts - 1 else max(S, 128))
+        own = np.arange(inf["own_begin"], inf["own_end"]) + inf["row0"]
+        pos_all.append(own)
+        r0 = inf["row0"]
+        ld, ls, lt = edges_from_masks(sub.export(L.BG_EXPORT_MASKS), S)
+        sel = np.isin(d, own)
+        got = sorted(zip((ld + r0).tolist(), (ls + r0).tolist(), lt.tolist()))
+        assert got == sorted(zip(d[sel].tolist(), s_[sel].tolist(), t[sel].tolist()))
+        ld, ls, lt = edges_from_masks(sub.export(L.BG_EXPORT_MASKS_T), S, transposed=True)
+        sel = np.isin(s_, own)
+        got = sorted(zip((ld + r0).tolist(), (ls + r0).tolist(), lt.tolist()))
+        assert got == sorted(zip(d[sel].tolist(), s_[sel].tolist(), t[sel].tolist()))
+        assert si["n_real"] == max(0, min(inf["n_local"], fi["n_real"] - r0))
+    pos_all = np.concatenate(pos_all)
+    np.testing.assert_array_equal(pos_all, np.arange(fi["n_pad"]))
+    with pytest.raises(L.BandGGNNError):
+        L.plan_partition(full, 0, 0)
+    sup = L.band_plan([synth.hub_graph(300, 8, 1)], 8, S, 0,
+                      L.BG_RCM | L.BG_KEEP_IF_BETTER | L.BG_SUPERNODES, 100, 1)
+    with pytest.raises(L.BandGGNNError):
+        L.plan_partition(sup, 2, 0)
