@@ -267,13 +267,14 @@ __global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
     // ------------------------------------------------------------------ TMA producer
     tma_prefetch_desc(&tm_x);
     tma_prefetch_desc(&tm_w);
+    if (has_bias) tma_prefetch_desc(&tm_deg);
+    // the state windows, W and the bias split may be the previous kernel's output (the bit tiles
+    // and in-degrees are plan data)
+    grid_dep_wait();
     if (has_bias) {
-      tma_prefetch_desc(&tm_deg);
       mbar_expect_tx(&bars->b2_full, C::B2);
       tma_load_2d(b2s, &tm_b2, &bars->b2_full, 0, 0);
     }
-    // the state windows are the previous kernel's output (bit tiles, W, deg and b2 are not)
-    grid_dep_wait();
     uint32_t widx = 0, xi = 0, di = 0;
     uint32_t n_x[2] = {0, 0}, n_deg[2] = {0, 0}, n_w[4] = {0, 0, 0, 0};
     bool ok = true;

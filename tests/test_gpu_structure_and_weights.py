@@ -264,8 +264,10 @@ def test_supernode_ggnn(S, H):
 def test_block_row_split_on_one_gpu_matches_the_unsplit_launch(S, H, n_parts):
     """Several parts of one plan (bg_plan_partition) run on one GPU one after another, their
     halo rows of E (forward) and dY (backward) copied from the neighbouring parts' own rows: the
-    own rows of Y and dE equal the unsplit launch's (same tiles, same sums), the halo rows of Y
-    come out 0, and the parts' dW, db sum to the unsplit ones."""
+    own rows of Y and dE equal the unsplit launch's up to fp32 reassociation (the same tiles and
+    products; a part with fewer tiles than SMs splits its tiles over several CTAs and sums their
+    partial results in another order), the halo rows of Y come out 0, and the parts' dW, db sum
+    to the unsplit ones."""
     from paper_1906_11786_gb300 import halo
     gs = synth.gen_batch(12, 200, 1200, 10, True, S // 2, S // 3, 2.0, 900 + S)
     n = sum(g.n_nodes for g in gs)
@@ -307,10 +309,12 @@ def test_block_row_split_on_one_gpu_matches_the_unsplit_launch(S, H, n_parts):
         L.check_device()
         Yl, dEl = Yl.cpu().numpy(), dEl.cpu().numpy()
         r0, ob, oe = inf["row0"], inf["own_begin"], inf["own_end"]
-        np.testing.assert_allclose(Yl[ob:oe], Y[r0 + ob:r0 + oe], rtol=1e-6, atol=1e-5)
-        np.testing.assert_allclose(dEl[ob:oe], dE[r0 + ob:r0 + oe], rtol=1e-6, atol=1e-5)
+        np.testing.assert_allclose(Yl[ob:oe], Y[r0 + ob:r0 + oe], rtol=0,
+                                   atol=1e-5 * np.abs(Y).max())
+        np.testing.assert_allclose(dEl[ob:oe], dE[r0 + ob:r0 + oe], rtol=0,
+                                   atol=1e-5 * np.abs(dE).max())
         assert not Yl[:ob].any() and not Yl[oe:].any()
         sW += dWl.cpu().numpy()
         sb += dbl.cpu().numpy()
-    np.testing.assert_allclose(sW, dW, rtol=1e-4, atol=1e-3 * np.abs(dW).max())
-    np.testing.assert_allclose(sb, db, rtol=1e-4, atol=1e-3 * np.abs(db).max())
+    np.testing.assert_allclose(sW, dW, rtol=0, atol=1e-5 * np.abs(dW).max())
+    np.testing.assert_allclose(sb, db, rtol=0, atol=1e-5 * np.abs(db).max())
