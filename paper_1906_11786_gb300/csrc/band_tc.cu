@@ -69,7 +69,7 @@ constexpr int kAtom = 64;      // bf16 per 128-byte swizzle row
 //   S <= 64: C1 = 2 (the tile spans 128 / S block-rows);  S = 128: 3;  S = 256: 6;  S = 512: 12.
 __host__ __device__ constexpr int band_chunks(int S) { return S <= 64 ? 2 : 3 * (S / 128); }
 
-template <int H, int S>
+template <int H, int S, bool BWD = false>
 struct Cfg {
   // H > SW runs as H / SW passes over SW-column slices of the state: pass hh contracts the band
   // with columns SW hh .. SW hh + SW - 1 of E and multiplies the result by rows SW hh .. of W_p,
@@ -103,6 +103,8 @@ struct Cfg {
   static constexpr int SMEM = OFF_BAR + 1024 + 1024;          // barriers + 1 KB alignment slack
   // TMEM columns: Y (H), two 64-column pre_p units used by the jobs (half, type) in turn, so that
   // a job's band products overlap the previous job's W product, then the A-tile slots
+  // (a third unit for the backward at H <= 64, so that the converters' read of one job's dM_p
+  // overlaps the band products of the next two, measured 2% slower at packed64: 85.7 vs 84.1 us)
   static constexpr int NB = 2;
   static constexpr int YCOL = 0;
   static constexpr int D1COL0 = H < 64 ? 64 : H;              // units start 64-column aligned
@@ -117,6 +119,9 @@ struct Cfg {
   static constexpr int THREADS = 128 * (2 + NE);
   static_assert(H == 32 || H == 64 || H == 128 || H == 256, "state size");
   static_assert(C1 % CG == 0 && NT % G == 0, "chunk groups");
+  // the release of a job's pre_p unit is signalled on the barrier of job + NB's first group: the
+  // ring must hold NB jobs' groups, or that barrier would still serve a pending job
+  static_assert(NT / G >= NB, "barrier ring");
   static_assert(NA >= CG + 1 && NA <= 8, "one group of A tiles and one more must fit");
   static_assert(NM >= 2 && NM <= 8, "mask ring");
   static_assert(SMEM <= 232448, "shared memory");
@@ -202,14 +207,14 @@ __device__ __forceinline__ void item_of(const Sched& sc, int w, int jobs, int& t
 }
 
 template <int H, int S, bool BWD>
-__global__ void __launch_bounds__(Cfg<H, S>::THREADS, 1)
+__global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
     k_band_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
               const __grid_constant__ CUtensorMap tm_deg, const __grid_constant__ CUtensorMap tm_b2,
               const uint32_t* __restrict__ maskI, float* __restrict__ out,
               __nv_bfloat16* __restrict__ outb, __nv_bfloat16* __restrict__ outT, int64_t ld_outT,
               __nv_bfloat16* __restrict__ dMT, int64_t ld_mt, const Sched sc, int P, int has_bias,
               int bias_f16, int accumulate, int* status) {
-  using C = Cfg<H, S>;
+  using C = Cfg<H, S, BWD>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -830,7 +835,7 @@ cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap&
                      __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
                      __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate,
                      float* split, const float* addend, int* status, cudaStream_t st) {
-  using C = Cfg<H, S>;
+  using C = Cfg<H, S, BWD>;
   cudaError_t e = cudaFuncSetAttribute(k_band_tc<H, S, BWD>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
