@@ -872,8 +872,8 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
       {
         KTimer tm(BG_KID_BAND_FWD, st);
         BG_CUDA(bg::band_tc_fwd_core(p, H, ETa + (size_t)t * n, (int64_t)TN, WT,
-                                     prm->b ? b2T : nullptr, nullptr, Yi(t), YTa + (size_t)t * n,
-                                     (int64_t)TN, split, addend, status, st));
+                                     prm->b ? b2T : nullptr, prm->b, nullptr, Yi(t),
+                                     YTa + (size_t)t * n, (int64_t)TN, split, addend, status, st));
       }
       KTimer tm(BG_KID_GRU_FWD, st);
       BG_CUDA(bg::gru_fwd_tc(

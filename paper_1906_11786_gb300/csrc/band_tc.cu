@@ -73,23 +73,27 @@ template <int H, int S, bool BWD = false>
 struct Cfg {
   // H > SW runs as H / SW passes over SW-column slices of the state: pass hh contracts the band
   // with columns SW hh .. SW hh + SW - 1 of E and multiplies the result by rows SW hh .. of W_p,
-  // into Y.  SW = 64, or 32 at H = 32 and at S = 512 (whose 1536-node window of 64 columns would
-  // take 192 KB)
-  static constexpr int SW = (H < 64 || S == 512) ? 32 : 64;   // state columns per pass
+  // into Y.  SW = 64, or 32 at H = 32.
+  static constexpr int SW = H < 64 ? 32 : 64;                 // state columns per pass
+  // S = 512 at SW = 64: the 1536-node window takes 192 KB, so the kernel keeps nothing else of
+  // size in shared memory: the expanders read their mask words straight from global memory (L2)
+  // instead of a staged ring, W has one stage, and the bias is added in the epilogue (in-degree
+  // times b in fp32) instead of by a product with staged operands
+  static constexpr bool GM = S == 512 && SW == 64;
   static constexpr int NH = H / SW;
   static constexpr int C1 = band_chunks(S);                   // 128-column chunks per type
   static constexpr int ATOM_X = SW * 128;                     // 64 nodes x SW state columns
   static constexpr int XWIN = 2 * C1 * ATOM_X;                // one half's window, 64-node atoms
   static constexpr int NXB = XWIN <= 48 * 1024 ? 2 : 1;       // state-window buffers
-  static constexpr int NW = 2;                                // W ring stages
+  static constexpr int NW = GM ? 1 : 2;                       // W ring stages
   // W stages hold K-columns of W_p^T as fp32 (tf32 operand) in 32-column atoms of H rows: a job's
   // 64 K-columns in one stage, or at H = 256 (64 KB) in two stages of one atom
   static constexpr int WK = H <= 128 ? SW : 32;               // K-columns per stage
   static constexpr int WJ = SW / WK;                          // stages per job
   static constexpr int WSTAGE = (WK / 32) * H * 128;
   static constexpr int DEG = kTile * 128;                     // 128 rows x 64 bf16
-  static constexpr int NDEG = NH > 1 ? 1 : 2;                 // deg buffers
-  static constexpr int B2 = H * 128;                          // H rows x 64 bf16
+  static constexpr int NDEG = GM ? 0 : (NH > 1 ? 1 : 2);      // deg buffers
+  static constexpr int B2 = GM ? 0 : H * 128;                 // H rows x 64 bf16
   static constexpr int OFF_X = 0;
   static constexpr int OFF_W = OFF_X + NXB * XWIN;
   static constexpr int OFF_DEG = OFF_W + NW * WSTAGE;
@@ -97,7 +101,9 @@ struct Cfg {
   static constexpr int MSTAGE = C1 * kTile * 16;              // C1 chunks x 128 rows x 128 bits
   // mask ring stages (one job each): as many as fit beside the window, at least two
   static constexpr int NM0 = (C1 <= 3 ? 8 : 4) / NH;
-  static constexpr int NM = C1 > 6 ? 2 : (NM0 > 2 ? NM0 : 2);
+  static constexpr int NM = GM ? 0 : (C1 > 6 ? 2 : (NM0 > 2 ? NM0 : 2));
+  // ring sizes as divisors (the GM shapes have no deg or mask ring; their code paths are off)
+  static constexpr int NDEGD = NDEG > 0 ? NDEG : 1, NMD = NM > 0 ? NM : 1;
   static constexpr int OFF_M = OFF_B2 + B2;
   static constexpr int OFF_BAR = OFF_M + NM * MSTAGE;
   static constexpr int SMEM = OFF_BAR + 1024 + 1024;          // barriers + 1 KB alignment slack
@@ -123,7 +129,7 @@ struct Cfg {
   // ring must hold NB jobs' groups, or that barrier would still serve a pending job
   static_assert(NT / G >= NB, "barrier ring");
   static_assert(NA >= CG + 1 && NA <= 8, "one group of A tiles and one more must fit");
-  static_assert(NM >= 2 && NM <= 8, "mask ring");
+  static_assert(GM || (NM >= 2 && NM <= 8), "mask ring");
   static_assert(SMEM <= 232448, "shared memory");
 };
 
@@ -190,6 +196,11 @@ struct Sched {
   // are written (the supernode rows' messages); NULL for none
   const float* addend;
   const int32_t* slot;
+  // epilogue bias (shapes without the bias product): Y[r] += sum_p deg[r][p] b[p], the in-degrees
+  // as 16-bit integers ([n][64], bf16 or, bias_f16, fp16) and b fp32 [P][H]; NULL for none
+  const uint16_t* deg;
+  const float* bias;
+  int bias_f16;
 };
 
 // Tile and job range [j0, j1) of item w; part -1 for a whole tile, else its slice.
@@ -231,6 +242,7 @@ __global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
   // issuer's commit and, backward, the 4 converter warps.
   constexpr int kFree = 1 + (BWD ? 4 : 0);
   const int jobs = C::NH * P;  // per tile
+  if (C::GM) has_bias = 0;     // the bias enters in the epilogue (sc.bias), not as a product
   // bias: once per tile, by the whole tile or its first slice
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -288,8 +300,8 @@ __global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
       item_of(sc, w, jobs, k, j0, j1, part);
       const int row0 = k * kTile, ws = (row0 / S) * S - S;
       if (has_bias && part <= 0) {
-        const int db = di % C::NDEG;
-        if (!mbar_wait(&bars->deg_empty[db], ((di / C::NDEG) & 1) ^ 1, status, 102, abort, 64)) break;
+        const int db = di % C::NDEGD;
+        if (!mbar_wait(&bars->deg_empty[db], ((di / C::NDEGD) & 1) ^ 1, status, 102, abort, 64)) break;
         ++n_deg[db];
         ++di;
         mbar_expect_tx(&bars->deg_full[db], C::DEG);
@@ -341,7 +353,7 @@ __global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
       for (int q = 0; q < 4; ++q) settle(&bars->w_full[q], n_w[q]);
       if (has_bias) settle(&bars->b2_full, 1);
     }
-  } else if (warp == 2 && lane == 0) {
+  } else if (warp == 2 && lane == 0 && !C::GM) {
     // ------------------------------------------------------------------ mask producer
     // each job's C1 bit chunks (contiguous [C1][128][4] words of its type), NM jobs ahead of the
     // expanders; both halves of a tile read the same bits
@@ -352,8 +364,8 @@ __global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
       bool ok = true;
       int p = j0 % P;
       for (int jb = j0; jb < j1; ++jb, ++midx, p = p + 1 == P ? 0 : p + 1) {
-        const int ms = midx % C::NM;
-        if (!mbar_wait(&bars->m_empty[ms], ((midx / C::NM) & 1) ^ 1, status, 104, abort, 64)) {
+        const int ms = midx % C::NMD;
+        if (!mbar_wait(&bars->m_empty[ms], ((midx / C::NMD) & 1) ^ 1, status, 104, abort, 64)) {
           ok = false;
           break;
         }
@@ -463,8 +475,8 @@ __global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
       }
       if (!ok) break;
       if (has_bias && part <= 0) {
-        const int db = di % C::NDEG;
-        if (!mbar_wait(&bars->deg_full[db], (di / C::NDEG) & 1, status, 206, abort)) break;
+        const int db = di % C::NDEGD;
+        if (!mbar_wait(&bars->deg_full[db], (di / C::NDEGD) & 1, status, 206, abort)) break;
         if (di == 0 && !mbar_wait(&bars->b2_full, 0, status, 207, abort)) break;
         ++di;
         tc_fence_after();
@@ -498,14 +510,33 @@ __global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
           aidx += C::C1;  // the other group's job
           continue;
         }
-        const int ms = midx % C::NM;
-        if (!mbar_wait(&bars->m_full[ms], (midx / C::NM) & 1, status, 302, abort, 32)) {
-          ok = false;
-          break;
+        // this row's mask words of the job's chunks: from the staged ring, or (GM) straight from
+        // global memory, all of the job's chunks requested at once (the other group's job and
+        // the MMAs run meanwhile)
+        const int ms = C::GM ? 0 : midx % C::NMD;
+        const uint8_t* mrow = nullptr;
+        uint4 mm[C::GM ? C::C1 : 1];
+        if constexpr (C::GM) {
+          const uint4* mg = reinterpret_cast<const uint4*>(maskI) +
+                            ((size_t)k * P + (jb % P)) * C::C1 * kTile + r;
+#pragma unroll
+          for (int j = 0; j < C::C1; ++j) mm[j] = __ldg(mg + (size_t)j * kTile);
+        } else {
+          if (!mbar_wait(&bars->m_full[ms], (midx / C::NMD) & 1, status, 302, abort, 32)) {
+            ok = false;
+            break;
+          }
+          mrow = mring + ms * C::MSTAGE + r * 16;
         }
-        const uint8_t* mrow = mring + ms * C::MSTAGE + r * 16;
+        // unrolled where the words sit in registers (a rolled loop measured faster otherwise)
+#pragma unroll(C::GM ? C::C1 : 1)
         for (int j = 0; j < C::C1; ++j) {
-          const uint4 m = *reinterpret_cast<const uint4*>(mrow + j * kTile * 16);
+          uint4 m;
+          if constexpr (C::GM) {
+            m = mm[j];
+          } else {
+            m = *reinterpret_cast<const uint4*>(mrow + j * kTile * 16);
+          }
           const int slot = aidx % C::NA;
           if (!mbar_wait(&bars->a_empty[slot][eg], (par >> slot) & 1, status, 301, abort)) {
             ok = false;
@@ -530,7 +561,7 @@ __global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
           ++aidx;
         }
         if (!ok) break;
-        warp_arrive(&bars->m_empty[ms]);
+        if (!C::GM) warp_arrive(&bars->m_empty[ms]);
       }
       if (!ok) break;
     }
@@ -598,6 +629,19 @@ __global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
           const float* ad = sc.addend + (size_t)asl * H + g0;
 #pragma unroll
           for (int j = 0; j < YG; ++j) vg[j] = __float_as_uint(__uint_as_float(vg[j]) + ad[j]);
+        }
+        if (C::GM && !BWD && sc.bias && part <= 0) {
+          // the bias: in-degree of each type (an exact 16-bit integer) times b_p, in fp32
+          const uint16_t* dr = sc.deg + (size_t)row * 64;
+          for (int q = 0; q < P; ++q) {
+            const uint32_t bits = dr[q];
+            if (!bits) continue;
+            const float d = sc.bias_f16 ? __half2float(__ushort_as_half((unsigned short)bits))
+                                        : __uint_as_float(bits << 16);
+            const float* bq = sc.bias + (size_t)q * H + g0;
+#pragma unroll
+            for (int j = 0; j < YG; ++j) vg[j] = __float_as_uint(fmaf(d, bq[j], __uint_as_float(vg[j])));
+          }
         }
 #pragma unroll
         for (int h1 = 0; h1 < YG; h1 += 32) {
@@ -801,7 +845,10 @@ int num_sms() {
 inline size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 // State columns per pass of the band kernel (Cfg::SW) and so its jobs per tile.
-int band_jobs(int H, int S, int P) { return H / ((H < 64 || S == 512) ? 32 : 64) * P; }
+int band_jobs(int H, int S, int P) {
+  (void)S;
+  return H / (H < 64 ? 32 : 64) * P;
+}
 
 // Work items of a launch over n_tiles tiles on `sms` SMs, one CTA per SM: whole tiles, and when
 // the last round of the grid would be mostly idle, its tiles split over k in {2, 4} job ranges
@@ -834,7 +881,8 @@ cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap&
                      const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
                      __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
                      __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate,
-                     float* split, const float* addend, int* status, cudaStream_t st) {
+                     float* split, const float* addend, const float* b32, int* status,
+                     cudaStream_t st) {
   using C = Cfg<H, S, BWD>;
   cudaError_t e = cudaFuncSetAttribute(k_band_tc<H, S, BWD>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
@@ -844,6 +892,9 @@ cudaError_t launch_s(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap&
   sc.part = split;
   sc.addend = BWD ? nullptr : addend;
   sc.slot = p->d_sin_slot;
+  sc.deg = reinterpret_cast<const uint16_t*>(p->d_deg2);
+  sc.bias = (C::GM && !BWD && has_bias) ? b32 : nullptr;
+  sc.bias_f16 = p->max_deg > 256 ? 1 : 0;
   const int grid = std::min(sc.n_items, sms);
   e = launch_pdl(k_band_tc<H, S, BWD>, dim3(grid), dim3(C::THREADS), C::SMEM, st, tx, tw, tdeg,
                  tb2, BWD ? p->d_maskTI : p->d_maskI, out, outb, outT, ld_outT, dMT, ld_mt, sc,
@@ -865,10 +916,10 @@ cudaError_t launch(const bg_plan* p, const CUtensorMap& tx, const CUtensorMap& t
                    const CUtensorMap& tdeg, const CUtensorMap& tb2, float* out,
                    __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
                    __nv_bfloat16* dMT, int64_t ld_mt, int has_bias, int accumulate, float* split,
-                   const float* addend, int* status, cudaStream_t st) {
+                   const float* addend, const float* b32, int* status, cudaStream_t st) {
 #define BG_BAND_S(SV)                                                                            \
   return launch_s<H, SV, BWD>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, dMT, ld_mt,      \
-                              has_bias, accumulate, split, addend, status, st);
+                              has_bias, accumulate, split, addend, b32, status, st);
   switch (p->S) {
     case 32: BG_BAND_S(32)
     case 64: BG_BAND_S(64)
@@ -975,19 +1026,20 @@ size_t band_tc_split_floats(const bg_plan* p, int H) {
 }
 
 cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, int64_t ld_x,
-                             const void* Wk, const __nv_bfloat16* b2T, float* out,
-                             __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
-                             float* split, const float* addend, int* status, cudaStream_t st) {
+                             const void* Wk, const __nv_bfloat16* b2T, const float* b32,
+                             float* out, __nv_bfloat16* outb, __nv_bfloat16* outT,
+                             int64_t ld_outT, float* split, const float* addend, int* status,
+                             cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw, tdeg, tb2;
-  if (!make_map_ld(&tx, XT, H, n, ld_x, (H < 64 || p->S == 512) ? 32 : 64) ||
+  if (!make_map_ld(&tx, XT, H, n, ld_x, H < 64 ? 32 : 64) ||
       !make_map_w(&tw, Wk, P, H) || !make_map(&tdeg, p->d_deg2, n, 64, kTile) ||
       !make_map(&tb2, b2T ? b2T : XT, H, 64, H))
     return cudaErrorInvalidValue;
   const int hb = b2T != nullptr;
 #define BG_FWD(HV)                                                                                \
   return launch<HV, false>(p, tx, tw, tdeg, tb2, out, outb, outT, ld_outT, nullptr, 0, hb, 0,     \
-                           split, addend, status, st);
+                           split, addend, b32, status, st);
   switch (H) {
     case 32: BG_FWD(32)
     case 64: BG_FWD(64)
@@ -1002,12 +1054,12 @@ cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, 
                              int64_t ld_mt, float* split, int* status, cudaStream_t st) {
   const int n = p->n_pad(), P = p->P;
   CUtensorMap tx, tw;
-  if (!make_map_ld(&tx, dYT, H, n, ld_y, (H < 64 || p->S == 512) ? 32 : 64) ||
+  if (!make_map_ld(&tx, dYT, H, n, ld_y, H < 64 ? 32 : 64) ||
       !make_map_w(&tw, Wk, P, H))
     return cudaErrorInvalidValue;
 #define BG_BWD(HV)                                                                                \
   return launch<HV, true>(p, tx, tw, tw, tw, dE, nullptr, nullptr, 0, dMT, ld_mt, 0, accumulate,  \
-                          split, nullptr, status, st);
+                          split, nullptr, nullptr, status, st);
   switch (H) {
     case 32: BG_BWD(32)
     case 64: BG_BWD(64)
@@ -1056,7 +1108,7 @@ cudaError_t band_tc_fwd(const bg_plan* p, int H, const void* E, const void* W, c
   if (e == cudaSuccess && b) e = prep_bias_split(p, b, b2T, H, status, st);
   if (e != cudaSuccess) return e;
   ProfSpan span(BG_KID_BAND_FWD, st);
-  return band_tc_fwd_core(p, H, ET, n, WT, b ? b2T : nullptr, Y, nullptr, nullptr, 0,
+  return band_tc_fwd_core(p, H, ET, n, WT, b ? b2T : nullptr, b, Y, nullptr, nullptr, 0,
                           band_tc_split_floats(p, H) ? split : nullptr, nullptr, status, st);
 }
 

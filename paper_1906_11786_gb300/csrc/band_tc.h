@@ -33,10 +33,13 @@ cudaError_t band_tc_prep_w(const bg_plan* p, int H, const void* W, int bwd, void
 //   addend (may be NULL): fp32 [rows_in][H], added to the Y rows of the plan's supernode in-edge
 //   targets (row r gets addend[p->d_sin_slot[r]]) before the outputs are written.
 size_t band_tc_split_floats(const bg_plan* p, int H);
+//   b32: the fp32 bias [P][H] (or NULL) beside its split b2T; the S = 512 kernels at 64-column
+//   slices add the bias in their epilogue from it.
 cudaError_t band_tc_fwd_core(const bg_plan* p, int H, const __nv_bfloat16* XT, int64_t ld_x,
-                             const void* Wk, const __nv_bfloat16* b2T, float* out,
-                             __nv_bfloat16* outb, __nv_bfloat16* outT, int64_t ld_outT,
-                             float* split, const float* addend, int* status, cudaStream_t st);
+                             const void* Wk, const __nv_bfloat16* b2T, const float* b32,
+                             float* out, __nv_bfloat16* outb, __nv_bfloat16* outT,
+                             int64_t ld_outT, float* split, const float* addend, int* status,
+                             cudaStream_t st);
 //   dYT: [H][>= n_pad] bf16; Wk: band_tc_prep_w(bwd = 1); dE fp32 (+)=; dMT: [P*H][ld_mt] bf16.
 cudaError_t band_tc_bwd_core(const bg_plan* p, int H, const __nv_bfloat16* dYT, int64_t ld_y,
                              const void* Wk, float* dE, int accumulate, __nv_bfloat16* dMT,
