@@ -510,38 +510,12 @@ __global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
           aidx += C::C1;  // the other group's job
           continue;
         }
-        // this row's mask words of the job's chunks: from the staged ring, or (GM) straight from
-        // global memory, all of the job's chunks requested at once (the other group's job and
-        // the MMAs run meanwhile)
-        const int ms = C::GM ? 0 : midx % C::NMD;
-        const uint8_t* mrow = nullptr;
-        uint4 mm[C::GM ? C::C1 : 1];
-        if constexpr (C::GM) {
-          const uint4* mg = reinterpret_cast<const uint4*>(maskI) +
-                            ((size_t)k * P + (jb % P)) * C::C1 * kTile + r;
-#pragma unroll
-          for (int j = 0; j < C::C1; ++j) mm[j] = __ldg(mg + (size_t)j * kTile);
-        } else {
-          if (!mbar_wait(&bars->m_full[ms], (midx / C::NMD) & 1, status, 302, abort, 32)) {
-            ok = false;
-            break;
-          }
-          mrow = mring + ms * C::MSTAGE + r * 16;
-        }
-        // unrolled where the words sit in registers (a rolled loop measured faster otherwise)
-#pragma unroll(C::GM ? C::C1 : 1)
-        for (int j = 0; j < C::C1; ++j) {
-          uint4 m;
-          if constexpr (C::GM) {
-            m = mm[j];
-          } else {
-            m = *reinterpret_cast<const uint4*>(mrow + j * kTile * 16);
-          }
+        // one chunk: wait for its A slot, expand the row's 128 bits into bf16 pairs in TMEM, and
+        // after the last chunk of a group signal the band-product issuer
+        auto expand_chunk = [&](int j, const uint4& m) -> bool {
           const int slot = aidx % C::NA;
-          if (!mbar_wait(&bars->a_empty[slot][eg], (par >> slot) & 1, status, 301, abort)) {
-            ok = false;
-            break;
-          }
+          if (!mbar_wait(&bars->a_empty[slot][eg], (par >> slot) & 1, status, 301, abort))
+            return false;
           par ^= 1u << slot;
           tc_fence_after();
           uint32_t v[32];
@@ -559,6 +533,44 @@ __global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
             warp_arrive(&bars->t_full[gi % C::NT]);
           }
           ++aidx;
+          return true;
+        };
+        // this row's mask words of the job's chunks: from the staged ring, or (GM) straight from
+        // global memory in groups of four chunks, the next group requested while the current one
+        // is expanded (a rolled group loop keeps the code small enough for the instruction cache)
+        const int ms = C::GM ? 0 : midx % C::NMD;
+        if constexpr (C::GM) {
+          constexpr int QG = 4;
+          static_assert(C::C1 % QG == 0, "mask prefetch groups");
+          const uint4* mg = reinterpret_cast<const uint4*>(maskI) +
+                            ((size_t)k * P + (jb % P)) * C::C1 * kTile + r;
+          uint4 cur[QG], nxt[QG];
+#pragma unroll
+          for (int q = 0; q < QG; ++q) cur[q] = __ldg(mg + (size_t)q * kTile);
+#pragma unroll 1
+          for (int g0 = 0; g0 < C::C1 && ok; g0 += QG) {
+            if (g0 + QG < C::C1) {
+#pragma unroll
+              for (int q = 0; q < QG; ++q) nxt[q] = __ldg(mg + (size_t)(g0 + QG + q) * kTile);
+            }
+#pragma unroll
+            for (int q = 0; q < QG; ++q)
+              if (ok && !expand_chunk(g0 + q, cur[q])) ok = false;
+#pragma unroll
+            for (int q = 0; q < QG; ++q) cur[q] = nxt[q];
+          }
+        } else {
+          if (!mbar_wait(&bars->m_full[ms], (midx / C::NMD) & 1, status, 302, abort, 32)) {
+            ok = false;
+            break;
+          }
+          const uint8_t* mrow = mring + ms * C::MSTAGE + r * 16;
+#pragma unroll 1
+          for (int j = 0; j < C::C1; ++j)
+            if (!expand_chunk(j, *reinterpret_cast<const uint4*>(mrow + j * kTile * 16))) {
+              ok = false;
+              break;
+            }
         }
         if (!ok) break;
         if (!C::GM) warp_arrive(&bars->m_empty[ms]);
