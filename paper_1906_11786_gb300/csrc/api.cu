@@ -442,8 +442,16 @@ BwdWs bwd_ws(const bg_plan* p, bg_dtype dt, int H) {
   return w;
 }
 
+// The GEMM-path GGNN steps of a shape whose band runs on the tensor cores and whose GRU forward
+// has a fused kernel but no fused backward (bf16, H = 256): the band kernel writes Y in bf16 and
+// the fused GRU forward reads it; Y is saved in bf16 (in the fp32 slot) for the backward.
+bool y_bf16_path(const bg_plan* p, bg_dtype dt, int H) {
+  return dt == BG_BF16 && tc_gemm_path(dt, H) && !bg::gru_tc_supported(H) &&
+         bg::gru_fwd_tc_supported(H) && bg::band_tc_supported(p, (int)dt, H);
+}
+
 struct GgnnFwdWs {
-  size_t gi, gh, Ybf, prop, part, total;
+  size_t gi, gh, Ybf, prop, part, addend, total;
 };
 GgnnFwdWs ggnn_fwd_ws(const bg_plan* p, bg_dtype dt, int H) {
   GgnnFwdWs w{};
@@ -454,6 +462,7 @@ GgnnFwdWs ggnn_fwd_ws(const bg_plan* p, bg_dtype dt, int H) {
   w.Ybf = o; o += al(n * H * 2);
   w.part = o; o += al(sizeof(float) * part_floats(p, H));
   w.prop = o; o += al(fwd_ws(p, dt, H).total);
+  w.addend = o; o += al(sizeof(float) * (size_t)p->sup_rows_in * H);
   w.total = o;
   return w;
 }
@@ -800,7 +809,8 @@ static int check_params(const bg_params* prm) {
 }
 
 // gi = X W_ih^T + b_ih, gh = Hs W_hh^T + b_hh  ([n, 3H] fp32).  With Xb (bf16 scratch [n][H]) the
-// products run on the tensor cores (W_ih, W_hh are already K-major [3H][H] operands).
+// products run on the tensor cores (W_ih, W_hh are already K-major [3H][H] operands); X NULL means
+// Xb already holds the messages in bf16.
 static int gru_gates_in(const bg_plan* p, int bf, int H, const float* X, const void* Hs,
                         const bg_params* prm, float* gi, float* gh, float* part, size_t pf,
                         cudaStream_t st, __nv_bfloat16* Xb = nullptr) {
@@ -808,7 +818,7 @@ static int gru_gates_in(const bg_plan* p, int bf, int H, const float* X, const v
   if (Xb) {
     int* status = nullptr;
     BG_TRY(status_word_ptr(&status));
-    BG_CUDA(bg::f32_to_bf16(X, Xb, (int64_t)n * H, st));
+    if (X) BG_CUDA(bg::f32_to_bf16(X, Xb, (int64_t)n * H, st));
     BG_CUDA(bg::gemm_bf16_tn(Xb, H, 0, prm->W_ih, H, 0, n, 3 * H, H, 1, gi, 3 * H, 0, prm->b_ih, 0,
                              0, status, st));
     BG_CUDA(bg::gemm_bf16_tn(Hs, H, 0, prm->W_hh, H, 0, n, 3 * H, H, 1, gh, 3 * H, 0, prm->b_hh, 0,
@@ -894,6 +904,42 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
   const size_t pf = part_floats(p, H);
   const size_t ebytes = esz(dt) * (size_t)p->n_pad() * H;
   BG_CUDA(cudaMemcpyAsync(sv + saved_E_off(p, dt, H, 0), E0, ebytes, cudaMemcpyDeviceToDevice, st));
+  if (y_bf16_path(p, dt, H)) {
+    // band kernel (bf16 Y) and the fused GRU forward; operands as band_tc_fwd lays them out
+    int* status = nullptr;
+    BG_TRY(status_word_ptr(&status));
+    const size_t n = (size_t)p->n_pad();
+    char* pw = wsc + w.prop;
+    auto* ETb = reinterpret_cast<__nv_bfloat16*>(pw);
+    void* WT = pw + al(n * H * 2);
+    auto* b2T = reinterpret_cast<__nv_bfloat16*>(pw + al(n * H * 2) + bg::band_tc_w_bytes(p, H));
+    float* split = reinterpret_cast<float*>(pw + al(n * H * 2) + bg::band_tc_w_bytes(p, H) +
+                                            al((size_t)H * 64 * 2));
+    float* addend = p->sup_rows_in ? reinterpret_cast<float*>(wsc + w.addend) : nullptr;
+    BG_CUDA(bg::band_tc_prep_w(p, H, prm->W, 0, WT, st));
+    if (prm->b) BG_CUDA(bg::prep_bias_split(p, prm->b, b2T, H, status, st));
+    for (int t = 0; t < T; ++t) {
+      const auto* Et = reinterpret_cast<const __nv_bfloat16*>(sv + saved_E_off(p, dt, H, t));
+      auto* En = reinterpret_cast<__nv_bfloat16*>(sv + saved_E_off(p, dt, H, t + 1));
+      auto* Yb = reinterpret_cast<__nv_bfloat16*>(sv + saved_Y_off(p, dt, H, T, t));
+      BG_CUDA(bg::prep_transpose_bf16(Et, 0, ETb, (int)n, H, 1, st));
+      if (addend) BG_CUDA(bg::super_fwd(p, 1, H, Et, prm->W, prm->b, addend, 1, st));
+      {
+        KTimer tm(BG_KID_BAND_FWD, st);
+        BG_CUDA(bg::band_tc_fwd_core(p, H, ETb, (int64_t)n, WT, prm->b ? b2T : nullptr, prm->b,
+                                     nullptr, Yb, nullptr, 0,
+                                     bg::band_tc_split_floats(p, H) ? split : nullptr, addend,
+                                     status, st));
+      }
+      KTimer tm(BG_KID_GRU_FWD, st);
+      BG_CUDA(bg::gru_fwd_tc(H, (int)n, p->n_real, Yb, Et,
+                             static_cast<const __nv_bfloat16*>(prm->W_ih),
+                             static_cast<const __nv_bfloat16*>(prm->W_hh), prm->b_ih, prm->b_hh, En,
+                             nullptr, 0, status, st));
+    }
+    if (ET) BG_CUDA(cudaMemcpyAsync(ET, sv + saved_E_off(p, dt, H, T), ebytes, cudaMemcpyDeviceToDevice, st));
+    return BG_OK;
+  }
   for (int t = 0; t < T; ++t) {
     const void* Et = sv + saved_E_off(p, dt, H, t);
     void* En = sv + saved_E_off(p, dt, H, t + 1);
@@ -1042,23 +1088,38 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     BG_CUDA(bg::fill_ones_rows(YTa, H, TN, TN, st));
     BG_CUDA(bg::fill_ones_rows(ETa, H, TN, TN, st));
   }
+  const bool ybf = y_bf16_path(p, dt, H);  // Y(t) saved in bf16 by the forward
   for (int t = T - 1; t >= 0; --t) {
     const void* Et = sv + saved_E_off(p, dt, H, t);
     const float* Yt = reinterpret_cast<const float*>(sv + saved_Y_off(p, dt, H, T, t));
     if (tcg) {
       KTimer tm(BG_KID_GRU_BWD, st);
-      BG_TRY(gru_gates_in(p, bf, H, Yt, Et, prm, gi, gh, part, pf, st, Ybf));
-      BG_CUDA(bg::gru_bwd_gates(bf, gi, gh, Et, gin, dgi, dgh, g, p->n_real, n, H, st));
-      BG_CUDA(bg::f32_to_bf16(dgi, dgib, (int64_t)n * 3 * H, st));
-      BG_CUDA(bg::f32_to_bf16(dgh, dghb, (int64_t)n * 3 * H, st));
+      if (ybf) {
+        // gates recomputed and their gradients formed in one kernel: bf16 row-major (the
+        // GEMMs' A operands) and transposed (step t's columns of the weight-gradient operands),
+        // g = the direct term
+        BG_CUDA(bg::gru_bwd_gates_tc(H, n, p->n_real, reinterpret_cast<const __nv_bfloat16*>(Yt),
+                                     static_cast<const __nv_bfloat16*>(Et),
+                                     static_cast<const __nv_bfloat16*>(prm->W_ih),
+                                     static_cast<const __nv_bfloat16*>(prm->W_hh), prm->b_ih,
+                                     prm->b_hh, gin, g, dgib, dghb, dgiT + (size_t)t * n,
+                                     dghT + (size_t)t * n, TN, status, st));
+      } else {
+        BG_TRY(gru_gates_in(p, bf, H, Yt, Et, prm, gi, gh, part, pf, st, Ybf));
+        BG_CUDA(bg::gru_bwd_gates(bf, gi, gh, Et, gin, dgi, dgh, g, p->n_real, n, H, st));
+        BG_CUDA(bg::f32_to_bf16(dgi, dgib, (int64_t)n * 3 * H, st));
+        BG_CUDA(bg::f32_to_bf16(dgh, dghb, (int64_t)n * 3 * H, st));
+      }
       BG_CUDA(bg::gemm_bf16_tn(dgib, 3 * H, 0, WihT, 3 * H, 0, n, H, 3 * H, 1, dX, H, 0, nullptr,
                                0, 0, status, st));
       BG_CUDA(bg::gemm_bf16_tn(dghb, 3 * H, 0, WhhT, 3 * H, 0, n, H, 3 * H, 1, g, H, 0, nullptr,
                                0, 1, status, st));
       // step t's columns of the weight-gradient operands (reduced after the loop)
-      BG_CUDA(bg::prep_transpose_bf16(dgib, 0, dgiT + (size_t)t * n, n, 3 * H, 1, st, TN));
-      BG_CUDA(bg::prep_transpose_bf16(dghb, 0, dghT + (size_t)t * n, n, 3 * H, 1, st, TN));
-      BG_CUDA(bg::prep_transpose_bf16(Yt, 1, YTa + (size_t)t * n, n, H, 1, st, TN));
+      if (!ybf) {
+        BG_CUDA(bg::prep_transpose_bf16(dgib, 0, dgiT + (size_t)t * n, n, 3 * H, 1, st, TN));
+        BG_CUDA(bg::prep_transpose_bf16(dghb, 0, dghT + (size_t)t * n, n, 3 * H, 1, st, TN));
+      }
+      BG_CUDA(bg::prep_transpose_bf16(Yt, ybf ? 0 : 1, YTa + (size_t)t * n, n, H, 1, st, TN));
       BG_CUDA(bg::prep_transpose_bf16(Et, 0, ETa + (size_t)t * n, n, H, 1, st, TN));
     } else {
       KTimer tm(BG_KID_GRU_BWD, st);

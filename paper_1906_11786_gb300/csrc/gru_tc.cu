@@ -597,6 +597,19 @@ constexpr int kSlotsB = 5;                   // backward piece ring
 constexpr int kGin = 128 * 64 * 4;           // one half of the incoming gradient: 2 boxes of 16 KB
 constexpr int kGates = 4 * 64;               // TMEM columns of one job's gate pre-activations
 
+// The forward takes H = 128 or 256 (HW): HW / 64 jobs per tile, one 64-column slice each; the tile
+// ring holds two stages at H = 128 and one at H = 256 (a 128-row tile of Y and E is 128 KB there).
+template <int HW>
+struct FwdCfg {
+  static constexpr int NH = HW / 64;
+  static constexpr int kTileB = 128 * HW * 2;
+  static constexpr int NS = HW <= 128 ? 2 : 1;  // tile stages
+  static constexpr int STAGE = 2 * kTileB;      // Y, E
+  static constexpr int PIECES = NS * STAGE;
+  static constexpr int SMEM = PIECES + kSlots * kPiece + 1024;
+  static_assert(SMEM + 8192 <= 232448, "shared memory");
+};
+
 struct Smem {
   static constexpr int FWD_STAGE = 2 * kTileB;  // Y, E
   static constexpr int FWD_PIECES = 2 * FWD_STAGE;
@@ -616,8 +629,8 @@ struct Bars {
 };
 
 __device__ __forceinline__ void setup(Bars* b, float* bias, const float* b_ih, const float* b_hh,
-                                      int warp) {
-  fill_gate_bias(bias, b_ih, b_hh, H);
+                                      int warp, int Hb = H) {
+  fill_gate_bias(bias, b_ih, b_hh, Hb);
   if (threadIdx.x == 0) {
     for (int i = 0; i < 2; ++i) {
       mbar_init(&b->t_full[i], 1);
@@ -648,7 +661,7 @@ __device__ __forceinline__ void setup(Bars* b, float* bias, const float* b_ih, c
 // Piece producer: for every job, the 2 NH gate pieces and (backward) the 6 backward pieces, in
 // the order the MMA issuer uses them.  The weights are not written by the kernels this one may
 // overlap under programmatic dependent launch (they change only between training steps).
-template <int NS>
+template <int NS, int HW = H>
 __device__ __forceinline__ void produce_pieces(Bars* b, uint8_t* ring, const CUtensorMap* tWih,
                                                const CUtensorMap* tWhh, const CUtensorMap* tWihT,
                                                const CUtensorMap* tWhhT, bool bwd, int n_tiles,
@@ -663,14 +676,15 @@ __device__ __forceinline__ void produce_pieces(Bars* b, uint8_t* ring, const CUt
     ++pc;
     return ring + s * kPiece;
   };
+  constexpr int NHW = HW / 64;
   for (int t = blockIdx.x; t < n_tiles && ok && !*abort; t += gridDim.x) {
-    for (int hh = 0; hh < NH && ok; ++hh) {
-      for (int q = 0; q < 2 * NH && ok; ++q) {
-        const int m = q / NH, ka = q % NH, s = pc % NS;
+    for (int hh = 0; hh < NHW && ok; ++hh) {
+      for (int q = 0; q < 2 * NHW && ok; ++q) {
+        const int m = q / NHW, ka = q % NHW, s = pc % NS;
         uint8_t* dst = next(kPiece);
         if (!dst) { ok = false; break; }
         for (int g = 0; g < 3; ++g)
-          tma_load_2d(dst + g * 64 * 128, m ? tWhh : tWih, &b->p_full[s], 64 * ka, g * H + 64 * hh);
+          tma_load_2d(dst + g * 64 * 128, m ? tWhh : tWih, &b->p_full[s], 64 * ka, g * HW + 64 * hh);
       }
       for (int q = 0; bwd && q < 6 && ok; ++q) {
         const int m = q / 3, g = q % 3, s = pc % NS;
@@ -688,13 +702,14 @@ __device__ __forceinline__ void produce_pieces(Bars* b, uint8_t* ring, const CUt
 
 // Gate pre-activations of job (tile in `stage`, half hh) into TMEM columns g0 .. g0 + 255,
 // consuming 2 NH gate pieces.
-template <int NS>
+template <int NS, int HW = H>
 __device__ __forceinline__ bool gate_mmas(Bars* b, bool leader, uint32_t g0, uint32_t sY,
                                           uint32_t sE, uint8_t* ring, uint32_t& pc, int* status,
                                           volatile int* abort) {
   constexpr uint32_t id_rz = idesc_bf16_f32(128, 128), id_n = idesc_bf16_f32(128, 64);
-  for (int q = 0; q < 2 * NH; ++q, ++pc) {
-    const int m = q / NH, ka = q % NH, s = pc % NS;
+  constexpr int NHW = HW / 64;
+  for (int q = 0; q < 2 * NHW; ++q, ++pc) {
+    const int m = q / NHW, ka = q % NHW, s = pc % NS;
     if (!mbar_wait(&b->p_full[s], (pc / NS) & 1, status, 632, abort)) return false;
     tc_fence_after();
     const uint32_t a0 = (m ? sE : sY) + ka * kAtomB, p0 = smem_u32(ring + s * kPiece);
@@ -713,6 +728,7 @@ __device__ __forceinline__ bool gate_mmas(Bars* b, bool leader, uint32_t g0, uin
   return true;
 }
 
+template <int HW>
 __global__ void __launch_bounds__(kThreads, 1)
     k_gru_fwd(const __grid_constant__ CUtensorMap tY, const __grid_constant__ CUtensorMap tE,
               const __grid_constant__ CUtensorMap tWih, const __grid_constant__ CUtensorMap tWhh,
@@ -723,12 +739,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   __shared__ Bars bars;
-  __shared__ __align__(16) float bias[4 * H];
+  using FC = FwdCfg<HW>;
+  __shared__ __align__(16) float bias[4 * HW];
   volatile int* abort = &bars.abort;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  setup(&bars, bias, b_ih, b_hh, warp);
+  setup(&bars, bias, b_ih, b_hh, warp, HW);
   const uint32_t tmem = bars.tmem_slot;
-  uint8_t* pieces = smem + Smem::FWD_PIECES;
+  uint8_t* pieces = smem + FC::PIECES;
 
   if (warp == 0 && lane == 0) {
     // ------------------------------------------------------------------ tile producer
@@ -736,23 +753,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t issued[2] = {0, 0};
     int i = 0;
     for (int t = blockIdx.x; t < n_tiles && !*abort; t += gridDim.x, ++i) {
-      const int s = i & 1;
-      if (!mbar_wait(&bars.t_empty[s], ((i >> 1) & 1) ^ 1, status, 633, abort, 64)) break;
+      const int s = i % FC::NS;
+      if (!mbar_wait(&bars.t_empty[s], ((i / FC::NS) & 1) ^ 1, status, 633, abort, 64)) break;
       ++issued[s];
-      uint8_t* st = smem + s * Smem::FWD_STAGE;
-      mbar_expect_tx(&bars.t_full[s], 2 * kTileB);
-      for (int a = 0; a < NH; ++a) {
+      uint8_t* st = smem + s * FC::STAGE;
+      mbar_expect_tx(&bars.t_full[s], 2 * FC::kTileB);
+      for (int a = 0; a < FC::NH; ++a) {
         tma_load_2d(st + a * kAtomB, &tY, &bars.t_full[s], 64 * a, t * 128);
-        tma_load_2d(st + kTileB + a * kAtomB, &tE, &bars.t_full[s], 64 * a, t * 128);
+        tma_load_2d(st + FC::kTileB + a * kAtomB, &tE, &bars.t_full[s], 64 * a, t * 128);
       }
     }
     if (*abort)
-      for (int s = 0; s < 2; ++s)
+      for (int s = 0; s < FC::NS; ++s)
         for (uint32_t k = 0; issued[s] && k < (1u << 22) && !mbar_try(&bars.t_full[s], (issued[s] - 1) & 1); ++k) {
         }
   } else if (warp == 2 && lane == 0) {
-    produce_pieces<kSlots>(&bars, pieces, &tWih, &tWhh, nullptr, nullptr, false, n_tiles, status,
-                           abort);
+    produce_pieces<kSlots, HW>(&bars, pieces, &tWih, &tWhh, nullptr, nullptr, false, n_tiles,
+                               status, abort);
   } else if (warp == 1) {
     // ------------------------------------------------------------------ MMA issuer
     const bool leader = elect_one_sync();
@@ -760,15 +777,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     int i = 0;
     for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++i) {
-      const int s = i & 1;
-      if (!mbar_wait(&bars.t_full[s], (i >> 1) & 1, status, 634, abort)) break;
-      const uint32_t sY = smem_u32(smem + s * Smem::FWD_STAGE);
-      for (int hh = 0; hh < NH && ok; ++hh, ++jn) {
+      const int s = i % FC::NS;
+      if (!mbar_wait(&bars.t_full[s], (i / FC::NS) & 1, status, 634, abort)) break;
+      const uint32_t sY = smem_u32(smem + s * FC::STAGE);
+      for (int hh = 0; hh < FC::NH && ok; ++hh, ++jn) {
         const int gb = jn & 1;
         if (!mbar_wait(&bars.g_empty[gb], ((jn >> 1) & 1) ^ 1, status, 635, abort)) { ok = false; break; }
         tc_fence_after();
-        if (!gate_mmas<kSlots>(&bars, leader, tmem + gb * kGates, sY, sY + kTileB, pieces, pc,
-                               status, abort)) {
+        if (!gate_mmas<kSlots, HW>(&bars, leader, tmem + gb * kGates, sY, sY + FC::kTileB, pieces,
+                                   pc, status, abort)) {
           ok = false;
           break;
         }
@@ -790,11 +807,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     int i = 0;
     bool ok = true;
     for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++i) {
-      const int s = i & 1;
+      const int s = i % FC::NS;
       const int row = t * 128 + r;
       const bool real = row < n_real;
-      const uint8_t* etile = smem + s * Smem::FWD_STAGE + kTileB;
-      for (int hh = 0; hh < NH; ++hh, ++jn) {
+      const uint8_t* etile = smem + s * FC::STAGE + FC::kTileB;
+      for (int hh = 0; hh < FC::NH; ++hh, ++jn) {
         const int gb = jn & 1;
         if (!mbar_wait(&bars.g_full[gb], (jn >> 1) & 1, status, 636, abort, 64)) { ok = false; break; }
         tc_fence_after();
@@ -813,12 +830,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (h8 == 1) {
             tc_fence_before();
             warp_arrive(&bars.g_empty[gb]);
-            if (hh == NH - 1) warp_arrive(&bars.t_empty[s]);
+            if (hh == FC::NH - 1) warp_arrive(&bars.t_empty[s]);
           }
           uint32_t pk[4];
 #pragma unroll
           for (int q = 0; q < 2; ++q) {
-            const GateBias gb = gate_bias(bias, H, h + 4 * q);
+            const GateBias gb = gate_bias(bias, HW, h + 4 * q);
             float o[4];
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
@@ -832,8 +849,183 @@ __global__ void __launch_bounds__(kThreads, 1)
             pk[2 * q] = pk2(o[0], o[1]);
             pk[2 * q + 1] = pk2(o[2], o[3]);
           }
-          *reinterpret_cast<uint4*>(En + (size_t)row * H + h) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          *reinterpret_cast<uint4*>(En + (size_t)row * HW + h) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
           if (EnT) store_T4(EnT, ld_T, row, h, pk);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// Gate gradients of the GRU backward at H = 256 (the GEMM path's backward: dX = dgi W_ih and
+// dH += dgh W_hh then run as tensor-core GEMMs).  Per job (tile, 64-column slice hh), as in the
+// forward: the gate pre-activations of the slice from streamed weight pieces into TMEM; the
+// epilogue recomputes the gates, reads the incoming gradient dE(t+1) of its row and columns, and
+// writes the gate gradients bf16 row-major (dgi, dgh [n][3H], the GEMMs' A operands) and
+// transposed (dgi^T, dgh^T [3H][ld_T], the weight-gradient operands), and the direct term
+// z * dE(t+1) (fp32, overwritten).  Padding rows get zeros.
+template <int HW>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_gru_bwd_gates(const __grid_constant__ CUtensorMap tY, const __grid_constant__ CUtensorMap tE,
+                    const __grid_constant__ CUtensorMap tWih,
+                    const __grid_constant__ CUtensorMap tWhh, const float* __restrict__ b_ih,
+                    const float* __restrict__ b_hh, const float* __restrict__ gin,
+                    float* __restrict__ gout, __nv_bfloat16* __restrict__ dgi,
+                    __nv_bfloat16* __restrict__ dgh, __nv_bfloat16* __restrict__ dgiT,
+                    __nv_bfloat16* __restrict__ dghT, int64_t ld_T, int n_tiles, int n_real,
+                    int* status) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  __shared__ Bars bars;
+  using FC = FwdCfg<HW>;
+  __shared__ __align__(16) float bias[4 * HW];
+  volatile int* abort = &bars.abort;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  setup(&bars, bias, b_ih, b_hh, warp, HW);
+  const uint32_t tmem = bars.tmem_slot;
+  uint8_t* pieces = smem + FC::PIECES;
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------------------ tile producer
+    grid_dep_wait();  // Y, E and the incoming gradient may be the previous kernels' output
+    uint32_t issued[2] = {0, 0};
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles && !*abort; t += gridDim.x, ++i) {
+      const int s = i % FC::NS;
+      if (!mbar_wait(&bars.t_empty[s], ((i / FC::NS) & 1) ^ 1, status, 641, abort, 64)) break;
+      ++issued[s];
+      uint8_t* st = smem + s * FC::STAGE;
+      mbar_expect_tx(&bars.t_full[s], 2 * FC::kTileB);
+      for (int a = 0; a < FC::NH; ++a) {
+        tma_load_2d(st + a * kAtomB, &tY, &bars.t_full[s], 64 * a, t * 128);
+        tma_load_2d(st + FC::kTileB + a * kAtomB, &tE, &bars.t_full[s], 64 * a, t * 128);
+      }
+    }
+    if (*abort)
+      for (int s = 0; s < FC::NS; ++s)
+        for (uint32_t k = 0; issued[s] && k < (1u << 22) && !mbar_try(&bars.t_full[s], (issued[s] - 1) & 1); ++k) {
+        }
+  } else if (warp == 2 && lane == 0) {
+    produce_pieces<kSlots, HW>(&bars, pieces, &tWih, &tWhh, nullptr, nullptr, false, n_tiles,
+                               status, abort);
+  } else if (warp == 1) {
+    // ------------------------------------------------------------------ MMA issuer
+    const bool leader = elect_one_sync();
+    uint32_t pc = 0, jn = 0;
+    bool ok = true;
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++i) {
+      const int s = i % FC::NS;
+      if (!mbar_wait(&bars.t_full[s], (i / FC::NS) & 1, status, 642, abort)) break;
+      const uint32_t sY = smem_u32(smem + s * FC::STAGE);
+      for (int hh = 0; hh < FC::NH && ok; ++hh, ++jn) {
+        const int gb = jn & 1;
+        if (!mbar_wait(&bars.g_empty[gb], ((jn >> 1) & 1) ^ 1, status, 643, abort)) { ok = false; break; }
+        tc_fence_after();
+        if (!gate_mmas<kSlots, HW>(&bars, leader, tmem + gb * kGates, sY, sY + FC::kTileB, pieces,
+                                   pc, status, abort)) {
+          ok = false;
+          break;
+        }
+        if (leader) tc_commit(&bars.g_full[gb]);
+        __syncwarp();
+      }
+    }
+    if (leader) tc_commit(&bars.drain);
+    __syncwarp();
+    for (uint32_t k = 0; k < (1u << 24) && !mbar_try(&bars.drain, 0); ++k) {
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------------------------ epilogue
+    grid_dep_wait();  // the outputs may still be in use by the previous kernel
+    const int g = (warp - 4) / 4;
+    const int r = (warp & 3) * 32 + lane;
+    const uint32_t lb = (uint32_t)((warp & 3) * 32) << 16;
+    uint32_t jn = 0;
+    int i = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++i) {
+      const int s = i % FC::NS;
+      const int row = t * 128 + r;
+      const bool real = row < n_real;
+      const uint8_t* etile = smem + s * FC::STAGE + FC::kTileB;
+      for (int hh = 0; hh < FC::NH; ++hh, ++jn) {
+        const int gb = jn & 1;
+        if (!mbar_wait(&bars.g_full[gb], (jn >> 1) & 1, status, 644, abort, 64)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t acc = tmem + lb + gb * kGates;
+#pragma unroll
+        for (int h8 = 0; h8 < 2; ++h8) {
+          const int hs = 16 * g + 8 * h8, h = 64 * hh + hs;  // column within the slice; global
+          uint32_t vr[8], vz[8], vn[8], vh[8];
+          tmem_ld8(acc + hs, vr);
+          tmem_ld8(acc + 64 + hs, vz);
+          tmem_ld8(acc + 128 + hs, vn);
+          tmem_ld8(acc + 192 + hs, vh);
+          tmem_wait_ld();
+          float e[8];
+          read_sw128_row8(etile, r, h, e);
+          if (h8 == 1) {
+            tc_fence_before();
+            warp_arrive(&bars.g_empty[gb]);
+            if (hh == FC::NH - 1) warp_arrive(&bars.t_empty[s]);
+          }
+          const float4* gp = reinterpret_cast<const float4*>(gin + (size_t)row * HW + h);
+          const float4 g0 = gp[0], g1 = gp[1];
+          const float gv[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+          uint32_t pr[4], pz[4], pn[4], ph[4];
+          float dd[8];
+#pragma unroll
+          for (int q = 0; q < 2; ++q) {
+            const GateBias gb4 = gate_bias(bias, HW, h + 4 * q);
+            float ar[4], az[4], an[4], ahn[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const int j = 4 * q + u;
+              const float rr = sigm(__uint_as_float(vr[j]) + f4(gb4.r, u));
+              const float zz = sigm(__uint_as_float(vz[j]) + f4(gb4.z, u));
+              const float ghn = __uint_as_float(vh[j]) + f4(gb4.hn, u);
+              const float nn = tanh_fast(__uint_as_float(vn[j]) + f4(gb4.in, u) + rr * ghn);
+              const float gg = real ? gv[j] : 0.f;
+              const float dn = gg * (1.f - zz);
+              const float dz = gg * (e[j] - nn);
+              const float dan = dn * (1.f - nn * nn);
+              ar[u] = dan * ghn * rr * (1.f - rr);
+              az[u] = dz * zz * (1.f - zz);
+              an[u] = dan;
+              ahn[u] = dan * rr;
+              dd[j] = gg * zz;
+            }
+            pr[2 * q] = pk2(ar[0], ar[1]); pr[2 * q + 1] = pk2(ar[2], ar[3]);
+            pz[2 * q] = pk2(az[0], az[1]); pz[2 * q + 1] = pk2(az[2], az[3]);
+            pn[2 * q] = pk2(an[0], an[1]); pn[2 * q + 1] = pk2(an[2], an[3]);
+            ph[2 * q] = pk2(ahn[0], ahn[1]); ph[2 * q + 1] = pk2(ahn[2], ahn[3]);
+          }
+          __nv_bfloat16* di = dgi + (size_t)row * 3 * HW;
+          __nv_bfloat16* dh = dgh + (size_t)row * 3 * HW;
+          *reinterpret_cast<uint4*>(di + h) = make_uint4(pr[0], pr[1], pr[2], pr[3]);
+          *reinterpret_cast<uint4*>(di + HW + h) = make_uint4(pz[0], pz[1], pz[2], pz[3]);
+          *reinterpret_cast<uint4*>(di + 2 * HW + h) = make_uint4(pn[0], pn[1], pn[2], pn[3]);
+          *reinterpret_cast<uint4*>(dh + h) = make_uint4(pr[0], pr[1], pr[2], pr[3]);
+          *reinterpret_cast<uint4*>(dh + HW + h) = make_uint4(pz[0], pz[1], pz[2], pz[3]);
+          *reinterpret_cast<uint4*>(dh + 2 * HW + h) = make_uint4(ph[0], ph[1], ph[2], ph[3]);
+          store_T4(dgiT, ld_T, row, h, pr);
+          store_T4(dgiT, ld_T, row, HW + h, pz);
+          store_T4(dgiT, ld_T, row, 2 * HW + h, pn);
+          store_T4(dghT, ld_T, row, h, pr);
+          store_T4(dghT, ld_T, row, HW + h, pz);
+          store_T4(dghT, ld_T, row, 2 * HW + h, ph);
+          float4* go = reinterpret_cast<float4*>(gout + (size_t)row * HW + h);
+          go[0] = make_float4(dd[0], dd[1], dd[2], dd[3]);
+          go[1] = make_float4(dd[4], dd[5], dd[6], dd[7]);
         }
       }
     }
@@ -1095,27 +1287,53 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace
 
 bool gru_tc_supported(int H) { return H == 32 || H == 64 || H == wide::H; }
+bool gru_fwd_tc_supported(int H) { return gru_tc_supported(H) || H == 256; }
 
 cudaError_t gru_fwd_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y,
                        const __nv_bfloat16* E, const __nv_bfloat16* W_ih,
                        const __nv_bfloat16* W_hh, const float* b_ih, const float* b_hh,
                        __nv_bfloat16* En, __nv_bfloat16* EnT, int64_t ld_T, int* status,
                        cudaStream_t st) {
-  if (!gru_tc_supported(H) || n_pad % 128) return cudaErrorInvalidValue;
-  const bool w = H == wide::H;
+  if (!gru_fwd_tc_supported(H) || n_pad % 128) return cudaErrorInvalidValue;
+  const bool w = H >= 128;
   CUtensorMap tY, tE, tWi, tWh;
   if (!make_map_ld(&tY, Y, n_pad, H, H, 128) || !make_map_ld(&tE, E, n_pad, H, H, 128) ||
       !make_map_ld(&tWi, W_ih, 3 * H, H, H, w ? 64 : 3 * H) ||
       !make_map_ld(&tWh, W_hh, 3 * H, H, H, w ? 64 : 3 * H))
     return cudaErrorInvalidValue;
-  auto kern = w ? wide::k_gru_fwd : H == 32 ? k_gru_fwd_tc<32> : k_gru_fwd_tc<64>;
-  const int smem = w ? wide::Smem::FWD : H == 32 ? GruSmem<32>::FWD : GruSmem<64>::FWD;
+  auto kern = H == 256 ? wide::k_gru_fwd<256> : H == 128 ? wide::k_gru_fwd<128>
+            : H == 32 ? k_gru_fwd_tc<32> : k_gru_fwd_tc<64>;
+  const int smem = H == 256 ? wide::FwdCfg<256>::SMEM : H == 128 ? wide::FwdCfg<128>::SMEM
+                 : H == 32 ? GruSmem<32>::FWD : GruSmem<64>::FWD;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const int n_tiles = n_pad / 128;
   const int grid = std::min(n_tiles, gemm_tn_num_sms());
   e = launch_pdl(kern, dim3(grid), dim3(kThreads), smem, st, tY, tE, tWi, tWh, b_ih, b_hh, En, EnT,
                  ld_T, n_tiles, n_real, status);
+  note_launch();
+  return e;
+}
+
+cudaError_t gru_bwd_gates_tc(int H, int n_pad, int n_real, const __nv_bfloat16* Y,
+                             const __nv_bfloat16* E, const __nv_bfloat16* W_ih,
+                             const __nv_bfloat16* W_hh, const float* b_ih, const float* b_hh,
+                             const float* gin, float* gout, __nv_bfloat16* dgi,
+                             __nv_bfloat16* dgh, __nv_bfloat16* dgiT, __nv_bfloat16* dghT,
+                             int64_t ld_T, int* status, cudaStream_t st) {
+  if (H != 256 || n_pad % 128) return cudaErrorInvalidValue;
+  CUtensorMap tY, tE, tWi, tWh;
+  if (!make_map_ld(&tY, Y, n_pad, H, H, 128) || !make_map_ld(&tE, E, n_pad, H, H, 128) ||
+      !make_map_ld(&tWi, W_ih, 3 * H, H, H, 64) || !make_map_ld(&tWh, W_hh, 3 * H, H, H, 64))
+    return cudaErrorInvalidValue;
+  auto kern = wide::k_gru_bwd_gates<256>;
+  const int smem = wide::FwdCfg<256>::SMEM;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  const int n_tiles = n_pad / 128;
+  const int grid = std::min(n_tiles, gemm_tn_num_sms());
+  e = launch_pdl(kern, dim3(grid), dim3(kThreads), smem, st, tY, tE, tWi, tWh, b_ih, b_hh, gin, gout,
+                 dgi, dgh, dgiT, dghT, ld_T, n_tiles, n_real, status);
   note_launch();
   return e;
 }
