@@ -512,7 +512,7 @@ __global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
         }
         // one chunk: wait for its A slot, expand the row's 128 bits into bf16 pairs in TMEM, and
         // after the last chunk of a group signal the band-product issuer
-        auto expand_chunk = [&](int j, const uint4& m) -> bool {
+        auto expand_chunk = [&](int j, const uint4 m) -> bool {
           const int slot = aidx % C::NA;
           if (!mbar_wait(&bars->a_empty[slot][eg], (par >> slot) & 1, status, 301, abort))
             return false;
@@ -565,12 +565,15 @@ __global__ void __launch_bounds__(Cfg<H, S, BWD>::THREADS, 1)
             break;
           }
           const uint8_t* mrow = mring + ms * C::MSTAGE + r * 16;
-#pragma unroll 1
-          for (int j = 0; j < C::C1; ++j)
-            if (!expand_chunk(j, *reinterpret_cast<const uint4*>(mrow + j * kTile * 16))) {
+          for (int j = 0; j < C::C1; ++j) {
+            // the words are read into registers before the slot wait, so that the shared-memory
+            // load overlaps it
+            const uint4 m = *reinterpret_cast<const uint4*>(mrow + j * kTile * 16);
+            if (!expand_chunk(j, m)) {
               ok = false;
               break;
             }
+          }
         }
         if (!ok) break;
         if (!C::GM) warp_arrive(&bars->m_empty[ms]);
