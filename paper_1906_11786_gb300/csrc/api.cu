@@ -470,8 +470,10 @@ GgnnFwdWs ggnn_fwd_ws(const bg_plan* p, bg_dtype dt, int H) {
 struct GgnnBwdWs {
   size_t gi, gh, dgi, dgh, dX, g, part, prop;
   size_t Ybf, dgib, dghb, dgiT, dghT, YTa, ETa, WihT, WhhT, tpart;  // tensor-core GEMM path
+  size_t dXT, dMT, Wk, tcpart, split, sup, dWs, dbs;  // and with the band kernel (bf16 Y saved)
   size_t total;
 };
+size_t tc_part_floats(const bg_plan* p, int H, int T);
 // The GRU weight gradients of the GEMM path are reduced once over all T steps: the gate gradients
 // and the [Y^T; 1; 0], [E^T; 1; 0] operands of every step are kept side by side, [rows][T n].
 size_t gru_tpart_floats(const bg_plan* p, int H, int T) {
@@ -482,16 +484,29 @@ GgnnBwdWs ggnn_bwd_ws(const bg_plan* p, bg_dtype dt, int H, int T) {
   size_t n = (size_t)p->n_pad(), TN = (size_t)T * n;
   size_t o = 0;
   if (tc_gemm_path(dt, H)) {
+    const bool ybf = y_bf16_path(p, dt, H);
     w.Ybf = o; o += al(n * H * 2);
     w.dgib = o; o += al(n * 3 * H * 2);
     w.dghb = o; o += al(n * 3 * H * 2);
     w.dgiT = o; o += al(TN * 3 * H * 2);
     w.dghT = o; o += al(TN * 3 * H * 2);
-    w.YTa = o; o += al((size_t)(H + 16) * TN * 2);
-    w.ETa = o; o += al((size_t)(H + 16) * TN * 2);
+    // with the band kernel the forward keeps [Y^T; 1] and [E^T; 1] among the saved activations
+    w.YTa = o; o += ybf ? 0 : al((size_t)(H + 16) * TN * 2);
+    w.ETa = o; o += ybf ? 0 : al((size_t)(H + 16) * TN * 2);
     w.WihT = o; o += al((size_t)3 * H * H * 2);
     w.WhhT = o; o += al((size_t)3 * H * H * 2);
     w.tpart = o; o += al(sizeof(float) * gru_tpart_floats(p, H, T));
+    if (ybf) {
+      w.dXT = o; o += al(n * H * 2);
+      w.dMT = o; o += al((size_t)p->P * H * n * 2);
+      w.Wk = o; o += bg::band_tc_w_bytes(p, H);
+      w.tcpart = o; o += al(sizeof(float) * tc_part_floats(p, H, T));
+      w.split = o; o += al(sizeof(float) * bg::band_tc_split_floats(p, H));
+      const bool sup = p->n_super_edges() > 0;
+      w.sup = o; o += bg::super_bwd_ws_bytes(p, H);
+      w.dWs = o; o += sup ? al(sizeof(float) * (size_t)p->P * H * H) : 0;
+      w.dbs = o; o += sup ? al(sizeof(float) * (size_t)p->P * H) : 0;
+    }
   }
   w.gi = o; o += al(sizeof(float) * n * 3 * H);
   w.gh = o; o += al(sizeof(float) * n * 3 * H);
@@ -510,6 +525,21 @@ size_t saved_E_off(const bg_plan* p, bg_dtype dt, int H, int t) {
 }
 size_t saved_Y_off(const bg_plan* p, bg_dtype dt, int H, int T, int t) {
   return saved_E_off(p, dt, H, T + 1) + (size_t)t * al(sizeof(float) * (size_t)p->n_pad() * H);
+}
+// With the band kernel and bf16 Y (H = 256): after E(0..T) and Y(0..T-1), [E(0..T-1)^T; 1; 0] and
+// [Y(0..T-1)^T; 1; 0] as [H+16][T n] bf16, written by the forward's GRU and band kernels: the band
+// products' operands and the weight-gradient GEMMs' (ones row -> bias gradient).
+struct YbSaved {
+  size_t ETa, YTa, total;
+};
+YbSaved yb_saved(const bg_plan* p, bg_dtype dt, int H, int T) {
+  const size_t TN = (size_t)T * p->n_pad();
+  YbSaved s{};
+  size_t o = saved_Y_off(p, dt, H, T, T);
+  s.ETa = o; o += al((size_t)(H + 16) * TN * 2);
+  s.YTa = o; o += al((size_t)(H + 16) * TN * 2);
+  s.total = o;
+  return s;
 }
 
 // ---- fused tensor-core GGNN steps (bf16, H in {32, 64, 128}, P <= 32)
@@ -609,6 +639,7 @@ extern "C" size_t bg_ggnn_workspace_bytes(const bg_plan* p, bg_dtype dt, int32_t
 extern "C" size_t bg_ggnn_saved_bytes(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T) {
   if (!p || H <= 0 || T < 0) return 0;
   const size_t simt = saved_Y_off(p, dt, H, T, T);
+  if (T >= 1 && y_bf16_path(p, dt, H)) return yb_saved(p, dt, H, T).total;
   return tc_shape(p, dt, H) && T >= 1 ? std::max(simt, tc_saved(p, H, T).total) : simt;
 }
 
@@ -905,29 +936,36 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
   const size_t ebytes = esz(dt) * (size_t)p->n_pad() * H;
   BG_CUDA(cudaMemcpyAsync(sv + saved_E_off(p, dt, H, 0), E0, ebytes, cudaMemcpyDeviceToDevice, st));
   if (y_bf16_path(p, dt, H)) {
-    // band kernel (bf16 Y) and the fused GRU forward; operands as band_tc_fwd lays them out
+    // band kernel (bf16 Y and Y^T) and the fused GRU forward (E(t+1) and E(t+1)^T): the
+    // transposed copies go to the saved [E^T; 1] and [Y^T; 1] for the band products of the next
+    // step and for the backward's weight gradients
     int* status = nullptr;
     BG_TRY(status_word_ptr(&status));
-    const size_t n = (size_t)p->n_pad();
+    const size_t n = (size_t)p->n_pad(), TN = (size_t)T * n;
+    const YbSaved ys = yb_saved(p, dt, H, T);
+    auto* ETa = reinterpret_cast<__nv_bfloat16*>(sv + ys.ETa);
+    auto* YTa = reinterpret_cast<__nv_bfloat16*>(sv + ys.YTa);
     char* pw = wsc + w.prop;
-    auto* ETb = reinterpret_cast<__nv_bfloat16*>(pw);
     void* WT = pw + al(n * H * 2);
     auto* b2T = reinterpret_cast<__nv_bfloat16*>(pw + al(n * H * 2) + bg::band_tc_w_bytes(p, H));
     float* split = reinterpret_cast<float*>(pw + al(n * H * 2) + bg::band_tc_w_bytes(p, H) +
                                             al((size_t)H * 64 * 2));
     float* addend = p->sup_rows_in ? reinterpret_cast<float*>(wsc + w.addend) : nullptr;
+    BG_CUDA(bg::prep_transpose_bf16(E0, 0, ETa, (int)n, H, 1, st, (int64_t)TN));
+    BG_CUDA(bg::fill_ones_rows(ETa, H, (int64_t)TN, (int64_t)TN, st));
+    BG_CUDA(bg::fill_ones_rows(YTa, H, (int64_t)TN, (int64_t)TN, st));
     BG_CUDA(bg::band_tc_prep_w(p, H, prm->W, 0, WT, st));
     if (prm->b) BG_CUDA(bg::prep_bias_split(p, prm->b, b2T, H, status, st));
     for (int t = 0; t < T; ++t) {
       const auto* Et = reinterpret_cast<const __nv_bfloat16*>(sv + saved_E_off(p, dt, H, t));
       auto* En = reinterpret_cast<__nv_bfloat16*>(sv + saved_E_off(p, dt, H, t + 1));
       auto* Yb = reinterpret_cast<__nv_bfloat16*>(sv + saved_Y_off(p, dt, H, T, t));
-      BG_CUDA(bg::prep_transpose_bf16(Et, 0, ETb, (int)n, H, 1, st));
       if (addend) BG_CUDA(bg::super_fwd(p, 1, H, Et, prm->W, prm->b, addend, 1, st));
       {
         KTimer tm(BG_KID_BAND_FWD, st);
-        BG_CUDA(bg::band_tc_fwd_core(p, H, ETb, (int64_t)n, WT, prm->b ? b2T : nullptr, prm->b,
-                                     nullptr, Yb, nullptr, 0,
+        BG_CUDA(bg::band_tc_fwd_core(p, H, ETa + (size_t)t * n, (int64_t)TN, WT,
+                                     prm->b ? b2T : nullptr, prm->b, nullptr, Yb,
+                                     YTa + (size_t)t * n, (int64_t)TN,
                                      bg::band_tc_split_floats(p, H) ? split : nullptr, addend,
                                      status, st));
       }
@@ -935,7 +973,8 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
       BG_CUDA(bg::gru_fwd_tc(H, (int)n, p->n_real, Yb, Et,
                              static_cast<const __nv_bfloat16*>(prm->W_ih),
                              static_cast<const __nv_bfloat16*>(prm->W_hh), prm->b_ih, prm->b_hh, En,
-                             nullptr, 0, status, st));
+                             t + 1 < T ? ETa + (size_t)(t + 1) * n : nullptr, (int64_t)TN, status,
+                             st));
     }
     if (ET) BG_CUDA(cudaMemcpyAsync(ET, sv + saved_E_off(p, dt, H, T), ebytes, cudaMemcpyDeviceToDevice, st));
     return BG_OK;
@@ -1058,6 +1097,90 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
   float* g = reinterpret_cast<float*>(wsc + w.g);
   float* part = reinterpret_cast<float*>(wsc + w.part);
   const size_t pf = part_floats(p, H);
+  if (y_bf16_path(p, dt, H)) {
+    // H = 256 with the band kernel: per step the gate gradients (one kernel), dX^T = (dgi W_ih)^T
+    // straight into the band backward's operand, g += dgh W_hh, the transposed-band backward and
+    // the band's weight gradients from its dM_p^T (one step's K range of [E^T; 1] stays in L2
+    // across the M tiles, which a product over all T steps at once does not); the GRU's weight
+    // gradients in one grouped product over all T steps at the end (operands [E^T; 1], [Y^T; 1]
+    // saved by the forward).  The running state gradient alternates between two buffers.
+    int* status = nullptr;
+    BG_TRY(status_word_ptr(&status));
+    const size_t nn = (size_t)n, TN = (size_t)T * nn;
+    const YbSaved ys = yb_saved(p, dt, H, T);
+    const auto* ETa = reinterpret_cast<const __nv_bfloat16*>(sv + ys.ETa);
+    const auto* YTa = reinterpret_cast<const __nv_bfloat16*>(sv + ys.YTa);
+    auto* dgib = reinterpret_cast<__nv_bfloat16*>(wsc + w.dgib);
+    auto* dghb = reinterpret_cast<__nv_bfloat16*>(wsc + w.dghb);
+    auto* dgiT = reinterpret_cast<__nv_bfloat16*>(wsc + w.dgiT);
+    auto* dghT = reinterpret_cast<__nv_bfloat16*>(wsc + w.dghT);
+    auto* WihT = reinterpret_cast<__nv_bfloat16*>(wsc + w.WihT);
+    auto* WhhT = reinterpret_cast<__nv_bfloat16*>(wsc + w.WhhT);
+    auto* dXT = reinterpret_cast<__nv_bfloat16*>(wsc + w.dXT);
+    auto* dMT = reinterpret_cast<__nv_bfloat16*>(wsc + w.dMT);
+    void* Wk = wsc + w.Wk;
+    float* tcpart = reinterpret_cast<float*>(wsc + w.tcpart);
+    float* split = bg::band_tc_split_floats(p, H) ? reinterpret_cast<float*>(wsc + w.split)
+                                                   : nullptr;
+    const auto* Wih = static_cast<const __nv_bfloat16*>(prm->W_ih);
+    const auto* Whh = static_cast<const __nv_bfloat16*>(prm->W_hh);
+    BG_CUDA(bg::prep_transpose_bf16(Wih, 0, WihT, 3 * H, H, 1, st));
+    BG_CUDA(bg::prep_transpose_bf16(Whh, 0, WhhT, 3 * H, H, 1, st));
+    BG_CUDA(bg::band_tc_prep_w(p, H, prm->W, 1, Wk, st));
+    const bool sup = p->n_super_edges() > 0;
+    float* dWs = reinterpret_cast<float*>(wsc + w.dWs);
+    float* dbs = reinterpret_cast<float*>(wsc + w.dbs);
+    if (sup) {
+      BG_CUDA(bg::fill_zero_f32(dWs, (int64_t)p->P * H * H, st));
+      BG_CUDA(bg::fill_zero_f32(dbs, (int64_t)p->P * H, st));
+    }
+    const int acc = (flags & BG_ACCUM) ? 1 : 0;
+    const float* gin = dET;
+    float* gout = dX;
+    for (int t = T - 1; t >= 0; --t) {
+      const auto* Et = reinterpret_cast<const __nv_bfloat16*>(sv + saved_E_off(p, dt, H, t));
+      const auto* Yt = reinterpret_cast<const __nv_bfloat16*>(sv + saved_Y_off(p, dt, H, T, t));
+      {
+        KTimer tm(BG_KID_GRU_BWD, st);
+        BG_CUDA(bg::gru_bwd_gates_tc(H, n, p->n_real, Yt, Et, Wih, Whh, prm->b_ih, prm->b_hh, gin,
+                                     gout, dgib, dghb, dgiT + (size_t)t * nn,
+                                     dghT + (size_t)t * nn, (int64_t)TN, status, st));
+        BG_CUDA(bg::gemm_bf16_tn_outT(dgib, 3 * H, WihT, 3 * H, n, H, 3 * H, dXT, (int64_t)nn,
+                                      status, st));
+        BG_CUDA(bg::gemm_bf16_tn(dghb, 3 * H, 0, WhhT, 3 * H, 0, n, H, 3 * H, 1, gout, H, 0,
+                                 nullptr, 0, 1, status, st));
+      }
+      {
+        KTimer tm(BG_KID_BAND_BWD, st);
+        BG_CUDA(bg::band_tc_bwd_core(p, H, dXT, (int64_t)nn, Wk, gout, 1, dMT, (int64_t)nn, split,
+                                     status, st));
+      }
+      {
+        KTimer tm(BG_KID_DW, st);
+        BG_CUDA(bg::gemm_tn(dMT, (int64_t)nn, ETa + (size_t)t * nn, (int64_t)TN, p->P * H, H,
+                            (int64_t)nn, 1, gr->dW, gr->db, t == T - 1 ? acc : 1, tcpart,
+                            tc_part_floats(p, H, T), status, st));
+      }
+      // the supernode rows and columns: dE(t) and their share of dW, db (summed over the steps)
+      if (sup)
+        BG_CUDA(bg::super_bwd(p, 1, H, Et, prm->W, nullptr, dXT, (int64_t)nn, gout, dWs, dbs,
+                              wsc + w.sup, st, t < T - 1));
+      gin = gout;
+      gout = gout == dX ? g : dX;
+    }
+    KTimer tm(BG_KID_DW, st);
+    const bg::TNProblem probs[2] = {
+        {dgiT, (int64_t)TN, YTa, (int64_t)TN, 3 * H, 0, gr->dW_ih, gr->db_ih},
+        {dghT, (int64_t)TN, ETa, (int64_t)TN, 3 * H, 0, gr->dW_hh, gr->db_hh}};
+    BG_CUDA(bg::gemm_tn_multi(probs, 2, H, (int64_t)TN, acc, tcpart, tc_part_floats(p, H, T),
+                              status, st));
+    if (sup) {
+      BG_CUDA(bg::add_inplace_f32(gr->dW, dWs, (int64_t)p->P * H * H, st));
+      if (gr->db) BG_CUDA(bg::add_inplace_f32(gr->db, dbs, (int64_t)p->P * H, st));
+    }
+    BG_CUDA(cudaMemcpyAsync(dE0, gin, sizeof(float) * nn * H, cudaMemcpyDeviceToDevice, st));
+    return BG_OK;
+  }
   if (!(flags & BG_ACCUM)) {
     BG_CUDA(bg::fill_zero_f32(gr->dW, (int64_t)p->P * H * H, st));
     if (gr->db) BG_CUDA(bg::fill_zero_f32(gr->db, (int64_t)p->P * H, st));

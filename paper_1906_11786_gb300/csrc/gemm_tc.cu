@@ -272,6 +272,11 @@ struct BatchArgs {
   const float* bias;
   int64_t sBias;
   int accumulate;
+  int vec;  // C rows (and bias) 16-byte aligned: each thread stores its row as float4
+  // instead of C: the product rounded to bf16 and stored transposed, CT[n * ldT + m] (batch 1,
+  // no bias, no accumulation; M even, N a multiple of 32, ldT even)
+  __nv_bfloat16* CT;
+  int64_t ldT;
 };
 
 template <int BN>
@@ -346,6 +351,81 @@ __global__ void __launch_bounds__(192, 2)
     __syncwarp();
     for (uint32_t t = 0; t < (1u << 24) && !mbar_try(drain, 0); ++t) {
     }
+  } else if (warp >= 2 && g.CT) {
+    // thread = row m, 32 consecutive columns per round; a lane pair (rows m, m + 1) swaps its
+    // packed column pairs so that each lane stores 4-byte words of two rows of one column
+    const int q = warp & 3;
+    if (mbar_wait(done, 0, status, 513, abort, 128)) {
+      tc_fence_after();
+      const int m = mt * 128 + q * 32 + lane;
+      const bool odd = lane & 1;
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        const int n0 = nt * BN + c0;
+        if (n0 >= g.N) break;  // the same for the whole warp
+        uint32_t v[32];
+        tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + c0, v);
+        tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + c0 + 16, v + 16);
+        tmem_wait_ld();
+        __nv_bfloat16* base = g.CT + (size_t)(n0 + odd) * g.ldT + (m & ~1);
+        const bool live = (m & ~1) < g.M;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          __nv_bfloat162 h2 = __floats2bfloat162_rn(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+          const uint32_t pk = *reinterpret_cast<uint32_t*>(&h2);
+          const uint32_t other = __shfl_xor_sync(0xffffffffu, pk, 1);
+          const uint32_t word = odd ? __byte_perm(other, pk, 0x7632) : __byte_perm(pk, other, 0x5410);
+          if (live) *reinterpret_cast<uint32_t*>(base + (size_t)(2 * j) * g.ldT) = word;
+        }
+      }
+    }
+  } else if (warp >= 2 && g.vec) {
+    // each warp drains its 32 TMEM lanes (rows), 32 columns at a time: a thread holds 32
+    // consecutive columns of its own row and writes them as 8 float4; the accumulating form reads
+    // the 8 previous float4 first, all in flight at once
+    const int q = warp & 3;
+    if (mbar_wait(done, 0, status, 513, abort, 128)) {
+      tc_fence_after();
+      const float* brow = g.bias ? g.bias + (size_t)b * g.sBias : nullptr;
+      float* cbase = g.C + (size_t)b * g.sC;
+      const int m = mt * 128 + q * 32 + lane;
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        const int n0 = nt * BN + c0;
+        if (n0 >= g.N) break;  // the same for the whole warp
+        uint32_t v[32];
+        tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + c0, v);
+        tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + c0 + 16, v + 16);
+        tmem_wait_ld();
+        if (m >= g.M) continue;
+        float* dst = cbase + (size_t)m * g.ldc + n0;
+        if (n0 + 32 <= g.N) {
+          float4 prev[8];
+          if (g.accumulate) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) prev[j] = reinterpret_cast<const float4*>(dst)[j];
+          }
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            float4 o = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                   __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+            if (brow) {
+              const float4 bv = reinterpret_cast<const float4*>(brow + n0)[j];
+              o.x += bv.x; o.y += bv.y; o.z += bv.z; o.w += bv.w;
+            }
+            if (g.accumulate) { o.x += prev[j].x; o.y += prev[j].y; o.z += prev[j].z; o.w += prev[j].w; }
+            reinterpret_cast<float4*>(dst)[j] = o;
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (n0 + j < g.N) {
+              const float x = __uint_as_float(v[j]) + (brow ? brow[n0 + j] : 0.f);
+              dst[j] = g.accumulate ? dst[j] + x : x;
+            }
+        }
+      }
+    }
   } else if (warp >= 2) {
     // each warp drains its 32 TMEM lanes (rows) 32 columns at a time through a padded SMEM
     // transpose so that every global store instruction writes 32 consecutive columns of one row
@@ -413,10 +493,11 @@ cudaError_t fill_ones_rows(__nv_bfloat16* base, int H, int64_t n, int64_t ld, cu
   return cudaGetLastError();
 }
 
-cudaError_t gemm_bf16_tn(const void* A, int64_t lda, int64_t sA, const void* B, int64_t ldb,
-                         int64_t sB, int M, int N, int K, int batch, float* Cout, int64_t ldc,
-                         int64_t sC, const float* bias, int64_t sBias, int accumulate, int* status,
-                         cudaStream_t st) {
+namespace {
+cudaError_t gemm_bf16_tn_any(const void* A, int64_t lda, int64_t sA, const void* B, int64_t ldb,
+                             int64_t sB, int M, int N, int K, int batch, float* Cout, int64_t ldc,
+                             int64_t sC, const float* bias, int64_t sBias, int accumulate,
+                             __nv_bfloat16* CT, int64_t ldT, int* status, cudaStream_t st) {
   if (M <= 0 || N <= 0 || batch <= 0) return cudaSuccess;
   if (K <= 0 || (lda % 8) || (ldb % 8) || (sA % 8) || (sB % 8)) return cudaErrorInvalidValue;
   const int BN = N <= 64 ? 64 : N <= 128 ? 128 : N <= 192 ? 192 : 256;
@@ -425,7 +506,10 @@ cudaError_t gemm_bf16_tn(const void* A, int64_t lda, int64_t sA, const void* B, 
   if (!(a3 ? make_map_3d(&ta, A, batch, M, K, lda, sA, 128) : make_map_ld(&ta, A, M, K, lda, 128)) ||
       !(b3 ? make_map_3d(&tb, B, batch, N, K, ldb, sB, BN) : make_map_ld(&tb, B, N, K, ldb, BN)))
     return cudaErrorInvalidValue;
-  BatchArgs g{M, N, (K + 63) / 64, a3 ? 1 : 0, b3 ? 1 : 0, Cout, ldc, sC, bias, sBias, accumulate};
+  const int vec = (reinterpret_cast<uintptr_t>(Cout) % 16 == 0) && ldc % 4 == 0 && sC % 4 == 0 &&
+                  (!bias || (reinterpret_cast<uintptr_t>(bias) % 16 == 0 && sBias % 4 == 0));
+  BatchArgs g{M, N, (K + 63) / 64, a3 ? 1 : 0, b3 ? 1 : 0, Cout, ldc, sC, bias, sBias, accumulate,
+              vec, CT, ldT};
   dim3 grid((M + 127) / 128, (N + BN - 1) / BN, batch);
   cudaError_t e;
 #define BG_GEMM16_CASE(BNV)                                                                    \
@@ -442,6 +526,24 @@ cudaError_t gemm_bf16_tn(const void* A, int64_t lda, int64_t sA, const void* B, 
 #undef BG_GEMM16_CASE
   note_launch();
   return cudaGetLastError();
+}
+}  // namespace
+
+cudaError_t gemm_bf16_tn(const void* A, int64_t lda, int64_t sA, const void* B, int64_t ldb,
+                         int64_t sB, int M, int N, int K, int batch, float* Cout, int64_t ldc,
+                         int64_t sC, const float* bias, int64_t sBias, int accumulate, int* status,
+                         cudaStream_t st) {
+  return gemm_bf16_tn_any(A, lda, sA, B, ldb, sB, M, N, K, batch, Cout, ldc, sC, bias, sBias,
+                          accumulate, nullptr, 0, status, st);
+}
+
+cudaError_t gemm_bf16_tn_outT(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int N,
+                              int K, __nv_bfloat16* CT, int64_t ldT, int* status, cudaStream_t st) {
+  if (!CT || (M % 2) || (N % 32) || (ldT % 2) || ldT < M ||
+      (reinterpret_cast<uintptr_t>(CT) % 4))
+    return cudaErrorInvalidValue;
+  return gemm_bf16_tn_any(A, lda, 0, B, ldb, 0, M, N, K, 1, nullptr, 0, 0, nullptr, 0, 0, CT, ldT,
+                          status, st);
 }
 
 size_t gemm_tn_part_floats(int M, int N, int64_t K) {

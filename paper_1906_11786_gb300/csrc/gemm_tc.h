@@ -3,6 +3,7 @@
 
 #include <cuda.h>
 #include <cuda_runtime.h>
+#include <cuda_bf16.h>
 
 #include <cstddef>
 #include <cstdint>
@@ -47,6 +48,10 @@ cudaError_t gemm_bf16_tn(const void* A, int64_t lda, int64_t sA, const void* B, 
                          int64_t sB, int M, int N, int K, int batch, float* C, int64_t ldc,
                          int64_t sC, const float* bias, int64_t sBias, int accumulate, int* status,
                          cudaStream_t st);
+// The same product (batch 1, no bias) rounded to bf16 and stored transposed: CT[n * ldT + m].  M
+// even, N a multiple of 32, ldT even and >= M, CT 4-byte aligned.
+cudaError_t gemm_bf16_tn_outT(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int N,
+                              int K, __nv_bfloat16* CT, int64_t ldT, int* status, cudaStream_t st);
 
 // 2-D bf16 tensor map over row-major [rows][cols] with row stride ld elements; box {64, box_rows};
 // 128-byte swizzle; reads outside the array return zero.
