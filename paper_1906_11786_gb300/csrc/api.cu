@@ -1211,38 +1211,23 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     BG_CUDA(bg::fill_ones_rows(YTa, H, TN, TN, st));
     BG_CUDA(bg::fill_ones_rows(ETa, H, TN, TN, st));
   }
-  const bool ybf = y_bf16_path(p, dt, H);  // Y(t) saved in bf16 by the forward
   for (int t = T - 1; t >= 0; --t) {
     const void* Et = sv + saved_E_off(p, dt, H, t);
     const float* Yt = reinterpret_cast<const float*>(sv + saved_Y_off(p, dt, H, T, t));
     if (tcg) {
       KTimer tm(BG_KID_GRU_BWD, st);
-      if (ybf) {
-        // gates recomputed and their gradients formed in one kernel: bf16 row-major (the
-        // GEMMs' A operands) and transposed (step t's columns of the weight-gradient operands),
-        // g = the direct term
-        BG_CUDA(bg::gru_bwd_gates_tc(H, n, p->n_real, reinterpret_cast<const __nv_bfloat16*>(Yt),
-                                     static_cast<const __nv_bfloat16*>(Et),
-                                     static_cast<const __nv_bfloat16*>(prm->W_ih),
-                                     static_cast<const __nv_bfloat16*>(prm->W_hh), prm->b_ih,
-                                     prm->b_hh, gin, g, dgib, dghb, dgiT + (size_t)t * n,
-                                     dghT + (size_t)t * n, TN, status, st));
-      } else {
-        BG_TRY(gru_gates_in(p, bf, H, Yt, Et, prm, gi, gh, part, pf, st, Ybf));
-        BG_CUDA(bg::gru_bwd_gates(bf, gi, gh, Et, gin, dgi, dgh, g, p->n_real, n, H, st));
-        BG_CUDA(bg::f32_to_bf16(dgi, dgib, (int64_t)n * 3 * H, st));
-        BG_CUDA(bg::f32_to_bf16(dgh, dghb, (int64_t)n * 3 * H, st));
-      }
+      BG_TRY(gru_gates_in(p, bf, H, Yt, Et, prm, gi, gh, part, pf, st, Ybf));
+      BG_CUDA(bg::gru_bwd_gates(bf, gi, gh, Et, gin, dgi, dgh, g, p->n_real, n, H, st));
+      BG_CUDA(bg::f32_to_bf16(dgi, dgib, (int64_t)n * 3 * H, st));
+      BG_CUDA(bg::f32_to_bf16(dgh, dghb, (int64_t)n * 3 * H, st));
       BG_CUDA(bg::gemm_bf16_tn(dgib, 3 * H, 0, WihT, 3 * H, 0, n, H, 3 * H, 1, dX, H, 0, nullptr,
                                0, 0, status, st));
       BG_CUDA(bg::gemm_bf16_tn(dghb, 3 * H, 0, WhhT, 3 * H, 0, n, H, 3 * H, 1, g, H, 0, nullptr,
                                0, 1, status, st));
       // step t's columns of the weight-gradient operands (reduced after the loop)
-      if (!ybf) {
-        BG_CUDA(bg::prep_transpose_bf16(dgib, 0, dgiT + (size_t)t * n, n, 3 * H, 1, st, TN));
-        BG_CUDA(bg::prep_transpose_bf16(dghb, 0, dghT + (size_t)t * n, n, 3 * H, 1, st, TN));
-      }
-      BG_CUDA(bg::prep_transpose_bf16(Yt, ybf ? 0 : 1, YTa + (size_t)t * n, n, H, 1, st, TN));
+      BG_CUDA(bg::prep_transpose_bf16(dgib, 0, dgiT + (size_t)t * n, n, 3 * H, 1, st, TN));
+      BG_CUDA(bg::prep_transpose_bf16(dghb, 0, dghT + (size_t)t * n, n, 3 * H, 1, st, TN));
+      BG_CUDA(bg::prep_transpose_bf16(Yt, 1, YTa + (size_t)t * n, n, H, 1, st, TN));
       BG_CUDA(bg::prep_transpose_bf16(Et, 0, ETa + (size_t)t * n, n, H, 1, st, TN));
     } else {
       KTimer tm(BG_KID_GRU_BWD, st);
