@@ -85,7 +85,11 @@ struct Cfg {
   static constexpr int ATOM_X = SW * 128;                     // 64 nodes x SW state columns
   static constexpr int XWIN = 2 * C1 * ATOM_X;                // one half's window, 64-node atoms
   static constexpr int NXB = XWIN <= 48 * 1024 ? 2 : 1;       // state-window buffers
-  static constexpr int NW = GM ? 1 : 2;                       // W ring stages
+  // W ring stages: at H <= 64, S <= 128 the small window leaves room for a deeper ring (the second
+  // issuer's W stages come from L2, and it gates the release of the pre_p units); measured best
+  // with four stages forward and three backward, the mask ring giving up the space
+  static constexpr bool DW = H <= 64 && S <= 128;
+  static constexpr int NW = GM ? 1 : (DW ? (BWD ? 3 : 4) : 2);
   // W stages hold K-columns of W_p^T as fp32 (tf32 operand) in 32-column atoms of H rows: a job's
   // 64 K-columns in one stage, or at H = 256 (64 KB) in two stages of one atom
   static constexpr int WK = H <= 128 ? SW : 32;               // K-columns per stage
@@ -100,7 +104,7 @@ struct Cfg {
   static constexpr int OFF_B2 = OFF_DEG + NDEG * DEG;
   static constexpr int MSTAGE = C1 * kTile * 16;              // C1 chunks x 128 rows x 128 bits
   // mask ring stages (one job each): as many as fit beside the window, at least two
-  static constexpr int NM0 = (C1 <= 3 ? 8 : 4) / NH;
+  static constexpr int NM0 = (C1 <= 3 ? (DW ? (BWD ? 6 : 4) : 8) : 4) / NH;
   static constexpr int NM = GM ? 0 : (C1 > 6 ? 2 : (NM0 > 2 ? NM0 : 2));
   // ring sizes as divisors (the GM shapes have no deg or mask ring; their code paths are off)
   static constexpr int NDEGD = NDEG > 0 ? NDEG : 1, NMD = NM > 0 ? NM : 1;
