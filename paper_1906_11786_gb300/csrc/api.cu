@@ -782,7 +782,6 @@ static int propagate_bwd_band(const bg_plan* p, bg_dtype dt, int H, const void* 
     // dW_p, db_p from one split-K product of dM^T with [E^T; 1; 0]
     BG_CUDA(bg::prep_transpose_bf16(dMb, 0, dMT, (int)n, PH, 1, st));
     BG_CUDA(bg::prep_transpose_bf16(E, 0, ETa, (int)n, H, 1, st));
-    BG_CUDA(bg::fill_ones_rows(ETa, H, (int64_t)n, (int64_t)n, st));
     BG_CUDA(bg::gemm_tn(dMT, (int64_t)n, ETa, (int64_t)n, PH, H, (int64_t)n, 1, dW, db, accum,
                         tpart, tpf, status, st));
     return BG_OK;
@@ -903,8 +902,6 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
     float* addend = p->sup_rows_in ? reinterpret_cast<float*>(wsc + wl.addend) : nullptr;
     BG_CUDA(cudaMemcpyAsync(Ei(0), E0, n * H * 2, cudaMemcpyDeviceToDevice, st));
     BG_CUDA(bg::prep_transpose_bf16(E0, 0, ETa, (int)n, H, 1, st, (int64_t)TN));
-    BG_CUDA(bg::fill_ones_rows(ETa, H, (int64_t)TN, (int64_t)TN, st));
-    BG_CUDA(bg::fill_ones_rows(YTa, H, (int64_t)TN, (int64_t)TN, st));
     BG_CUDA(bg::band_tc_prep_w(p, H, prm->W, 0, WT, st));
     if (prm->b) BG_CUDA(bg::prep_bias_split(p, prm->b, b2T, H, status, st));
     for (int t = 0; t < T; ++t) {
@@ -952,8 +949,6 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
                                             al((size_t)H * 64 * 2));
     float* addend = p->sup_rows_in ? reinterpret_cast<float*>(wsc + w.addend) : nullptr;
     BG_CUDA(bg::prep_transpose_bf16(E0, 0, ETa, (int)n, H, 1, st, (int64_t)TN));
-    BG_CUDA(bg::fill_ones_rows(ETa, H, (int64_t)TN, (int64_t)TN, st));
-    BG_CUDA(bg::fill_ones_rows(YTa, H, (int64_t)TN, (int64_t)TN, st));
     BG_CUDA(bg::band_tc_prep_w(p, H, prm->W, 0, WT, st));
     if (prm->b) BG_CUDA(bg::prep_bias_split(p, prm->b, b2T, H, status, st));
     for (int t = 0; t < T; ++t) {
@@ -1208,8 +1203,6 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     // [E^T; 1; 0] over all T steps (their bias-gradient column)
     BG_CUDA(bg::prep_transpose_bf16(prm->W_ih, 0, WihT, 3 * H, H, 1, st));
     BG_CUDA(bg::prep_transpose_bf16(prm->W_hh, 0, WhhT, 3 * H, H, 1, st));
-    BG_CUDA(bg::fill_ones_rows(YTa, H, TN, TN, st));
-    BG_CUDA(bg::fill_ones_rows(ETa, H, TN, TN, st));
   }
   for (int t = T - 1; t >= 0; --t) {
     const void* Et = sv + saved_E_off(p, dt, H, t);

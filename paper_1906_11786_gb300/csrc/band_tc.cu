@@ -1156,9 +1156,9 @@ cudaError_t band_tc_bwd(const bg_plan* p, int H, const void* E, const void* W, c
     e = band_tc_bwd_core(p, H, dYT, n, Wk, dE, accum, dMT, n, split, status, st);
   }
   if (e != cudaSuccess) return e;
-  // [E^T; 1; 0]: the ones row turns the bias gradient into column H of the same product
+  // E^T; the weight-gradient product appends its ones row, which turns the bias gradient into
+  // column H of the same product
   e = prep_transpose_bf16(E, 0, ETa, n, H, 1, st);
-  if (e == cudaSuccess) e = fill_ones_rows(ETa, H, n, n, st);
   if (e != cudaSuccess) return e;
   // dW_p[h][h'] (+)= sum_nodes E[node][h] dM_p[node][h'],  db_p[h'] (+)= sum_nodes dM_p[node][h']
   ProfSpan span(BG_KID_DW, st);

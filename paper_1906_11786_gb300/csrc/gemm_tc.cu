@@ -28,8 +28,10 @@ constexpr int kStages = 4;
 // MT = 2 consecutive 128-row M tiles of one problem (MT = 1 at BN = 272, whose accumulator takes all
 // 512 TMEM columns), so that each K chunk of B, which every M tile of the problem reads, is loaded
 // once per two tiles: the pass moves A once and B once per tile pair, instead of once per tile.
-// B boxes are at most 256 rows: BN = 272 loads two boxes of 136 rows and issues an N = 256 and an
-// N = 16 MMA per K step.
+// B is [X^T; 1; 0]: its Hout = BN - 16 data rows come by TMA (one box of at most 256 rows), and
+// its last 16 rows, a ones row (the bias column of the product) and zeros, are the same for every K
+// chunk, so the kernel writes them once into each stage at its start.  BN = 272 issues an N = 256
+// and an N = 16 MMA per K step.
 template <int BN>
 struct GCfg {
   static constexpr int MT = BN <= 256 ? 2 : 1;
@@ -39,12 +41,12 @@ struct GCfg {
   static constexpr int STAGES = 4;
   static constexpr int SMEM = STAGES * STAGE + 1024 + 1024;
   static constexpr int TCOLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : BN <= 256 ? 256 : 512;
-  static constexpr int BOX = BN <= 256 ? BN : BN / 2;  // B rows per TMA box
+  static constexpr int BROWS = BN - 16;                 // B rows loaded per K chunk (one box)
   static constexpr int N1 = BN <= 256 ? BN : 256;      // first MMA's N
   static_assert(BN % 16 == 0 && BN <= 512, "tile width");
   static_assert(SMEM + 512 <= 232448, "shared memory");
   static_assert(MT * TCOLS <= 512, "tensor memory");
-  static_assert(BOX * 128 % 1024 == 0 && A_BYTES % 1024 == 0, "box alignment");
+  static_assert(BROWS <= 256 && BROWS * 128 % 1024 == 0 && A_BYTES % 1024 == 0, "box alignment");
   static_assert(STAGES <= kStages, "stage count");
 };
 
@@ -95,6 +97,15 @@ __global__ void __launch_bounds__(192, 1)
   const CUtensorMap* tmB = &grp.b[g];
   const int kc0 = split * per_split;
   const int kc1 = min(kchunks, kc0 + per_split);
+  // the last 16 rows of every stage's B: row Hout all bf16 ones, the rest zeros (128 bytes a row;
+  // all 16-byte chunks of a row equal, so the 128-byte swizzle leaves them in place)
+  for (int i = threadIdx.x; i < C::STAGES * 16 * 8; i += blockDim.x) {
+    const int s = i / 128, r = (i / 8) % 16, c = i % 8;
+    const uint32_t v = r == 0 ? 0x3F803F80u : 0u;
+    *reinterpret_cast<uint4*>(smem + s * C::STAGE + C::MT * C::A_BYTES + (C::BROWS + r) * 128 + c * 16) =
+        make_uint4(v, v, v, v);
+  }
+  fence_proxy_async();  // visible to the tensor cores' shared-memory reads
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
     mbar_init(done, 1);
@@ -121,12 +132,11 @@ __global__ void __launch_bounds__(192, 1)
       const int s = it % C::STAGES;
       if (!mbar_wait(&empty[s], ((it / C::STAGES) & 1) ^ 1, status, 501, abort, 32)) break;
       ++issued[s];
-      mbar_expect_tx(&full[s], ntiles * C::A_BYTES + C::B_BYTES);
+      mbar_expect_tx(&full[s], ntiles * C::A_BYTES + C::BROWS * 128);
       uint8_t* st = smem + s * C::STAGE;
       for (int m = 0; m < ntiles; ++m)
         tma_load_2d(st + m * C::A_BYTES, tmA, &full[s], kc * 64, (mt0 + m) * 128);
-      for (int r = 0; r < BN; r += C::BOX)
-        tma_load_2d(st + C::MT * C::A_BYTES + r * 128, tmB, &full[s], kc * 64, blockIdx.y * BN + r);
+      tma_load_2d(st + C::MT * C::A_BYTES, tmB, &full[s], kc * 64, blockIdx.y * BN);
     }
     if (*abort)
       for (int s = 0; s < C::STAGES; ++s)
@@ -471,29 +481,6 @@ __global__ void __launch_bounds__(192, 2)
 }  // namespace
 
 namespace {
-__global__ void k_fill_ones_rows(__nv_bfloat16* base, int H, int64_t n, int64_t ld) {
-  // row H: ones, rows H+1 .. H+15: zeros; 16-byte stores (ld and n are multiples of 8 elements)
-  const int64_t per_row = n / 8, total = 16 * per_row;
-  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total;
-       t += (int64_t)gridDim.x * blockDim.x) {
-    const int r = (int)(t / per_row);
-    const int64_t c = (t - r * per_row) * 8;
-    const uint32_t v = r == 0 ? 0x3F803F80u : 0u;  // bf16 1.0 pairs
-    *reinterpret_cast<uint4*>(base + (int64_t)(H + r) * ld + c) = make_uint4(v, v, v, v);
-  }
-}
-}  // namespace
-
-cudaError_t fill_ones_rows(__nv_bfloat16* base, int H, int64_t n, int64_t ld, cudaStream_t st) {
-  if ((n % 8) || (ld % 8) || (reinterpret_cast<uintptr_t>(base) % 16)) return cudaErrorInvalidValue;
-  const int64_t total = 2 * n;  // 16 rows x n / 8 vectors
-  k_fill_ones_rows<<<(unsigned)std::min<int64_t>((total + 255) / 256, 8192), 256, 0, st>>>(base, H,
-                                                                                          n, ld);
-  note_launch();
-  return cudaGetLastError();
-}
-
-namespace {
 cudaError_t gemm_bf16_tn_any(const void* A, int64_t lda, int64_t sA, const void* B, int64_t ldb,
                              int64_t sB, int M, int N, int K, int batch, float* Cout, int64_t ldc,
                              int64_t sC, const float* bias, int64_t sBias, int accumulate,
@@ -565,7 +552,7 @@ cudaError_t gemm_tn_multi(const TNProblem* pr, int n, int Hout, int64_t K, int a
   int mt = 0, Mtot = 0;
   for (int g = 0; g < n; ++g) {
     if (!make_map_ld(&grp.a[g], pr[g].A, pr[g].M, K, pr[g].lda, 128) ||
-        !make_map_ld(&grp.b[g], pr[g].B, N, K, pr[g].ldb, N <= 256 ? N : N / 2))
+        !make_map_ld(&grp.b[g], pr[g].B, N - 16, K, pr[g].ldb, N - 16))
       return cudaErrorInvalidValue;
     mt += ((pr[g].M + 127) / 128 + MT - 1) / MT;
     grp.it_end[g] = mt;

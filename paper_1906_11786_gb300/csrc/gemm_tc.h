@@ -14,9 +14,9 @@ namespace bg {
 size_t gemm_tn_part_floats(int M, int N, int64_t K);
 
 // Reduces over K (nodes, possibly several steps concatenated) the outer products
-//   G[m][n] = sum_k A[m][k] B[n][k]    A: [M][K] bf16 (row stride lda), B: [Hout+16][K] bf16
-// where B's row Hout is all ones and rows Hout+1.. are zero, so column Hout of G is the row sum
-// of A (a bias gradient).  Output (accumulate != 0 adds):
+//   G[m][n] = sum_k A[m][k] B'[n][k]    A: [M][K] bf16 (row stride lda), B: [Hout][K] bf16
+// where B' is B with a row of ones (row Hout) and 15 zero rows appended by the kernel, so column
+// Hout of G is the row sum of A (a bias gradient).  Output (accumulate != 0 adds):
 //   mode 0: out[m][n] = G[m][n] (n < Hout), bias[m] = G[m][Hout]
 //   mode 1: m = p*Hout + o: out[p][n][o] = G[m][n], bias[m] = G[m][Hout]   (bias may be NULL)
 // Hout in {32, 64, 128, 256}.  Deterministic: fixed split layout and summation order.
@@ -68,8 +68,5 @@ bool make_map_3d(CUtensorMap* m, const void* base, uint64_t batch, uint64_t rows
 // One block whose bounded mbarrier wait is never satisfied: it gives up after the poll cap and
 // records a timeout (site 901) in `status`, the path every stalled pipeline role takes.
 cudaError_t wait_selftest(int* status, cudaStream_t st);
-
-// rows [H, H+16) of a [H+16][ld] bf16 array: row H = 1.0, the rest 0 (cols [0, n)).
-cudaError_t fill_ones_rows(__nv_bfloat16* base, int H, int64_t n, int64_t ld, cudaStream_t st);
 
 }  // namespace bg
