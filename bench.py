@@ -467,10 +467,18 @@ def oracle_sample(name: str, c, budget_s: float = 15.0, parallel: bool = False,
 
 
 def fixed_config(name, graphs, c, world, n_packed, n_real, n_pad, K):
-    """The workload's identity, the same for both arms: what ran, not how fast."""
+    """The workload's identity, the same for both arms: what ran, not how fast.  `l2` states
+    whether one step's working set (the band's bit tiles in both orientations and the states and
+    saved activations, estimated from the shapes) exceeds the 129 MB L2 or is timed L2-resident."""
+    tiles = 2 * K * 3 * c["P"] * c["S"] * c["S"] // 8
+    acts = (2 * c["T"] + 1) * n_pad * c["H"] * 2
+    mb = (tiles + acts) / 1e6
+    l2 = (f"per-step working set ~{mb:.0f} MB (band tiles + activations) > 129 MB L2" if mb > 129
+          else f"per-step working set ~{mb:.1f} MB fits the 129 MB L2: repeated steps run "
+               "L2-resident (not flushed)")
     return {"workload": name, "graphs": len(graphs), "packed": n_packed, "n_real": n_real,
             "n_pad": n_pad, "K": K, "S": c["S"], "P": c["P"], "H": c["H"], "T": c["T"],
-            "l2": "per-step working set (band tiles + saved activations) > 129 MB L2",
+            "l2": l2,
             "parallelism": f"dp{world} (one supergraph per GPU"
                            + (", gradient all-reduce)" if world > 1 else ")")}
 
