@@ -275,7 +275,10 @@ typedef struct bg_grads {
 } bg_grads;
 
 /* Bytes of the activation buffer the forward fills and the backward reads: E(0..T) in dtype and
- * the messages Y(0..T-1) in fp32 (the (T+1) N H embeddings of Appendix A.1 plus T message sums). */
+ * the messages Y(0..T-1) in fp32 (the (T+1) N H embeddings of Appendix A.1 plus T message sums);
+ * on the tensor-core paths (bf16 with a band kernel for the plan's S and H) the messages are kept
+ * in bf16 and transposed bf16 copies of E(0..T-1) and Y(0..T-1) are added, the backward's
+ * operands.  The layout is the library's own: callers pass the buffer through unchanged. */
 size_t bg_ggnn_saved_bytes(const bg_plan* plan, bg_dtype dtype, int32_t H, int32_t T);
 /* E0 [n_pad, H] dtype; ET [n_pad, H] dtype or NULL; saved: device buffer of
  * bg_ggnn_saved_bytes. */

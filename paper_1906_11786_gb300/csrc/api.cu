@@ -475,7 +475,8 @@ struct GgnnBwdWs {
 };
 size_t tc_part_floats(const bg_plan* p, int H, int T);
 // The GRU weight gradients of the GEMM path are reduced once over all T steps: the gate gradients
-// and the [Y^T; 1; 0], [E^T; 1; 0] operands of every step are kept side by side, [rows][T n].
+// and the Y^T, E^T operands of every step are kept side by side, [rows][T n]; the GEMM appends a
+// ones row to its operand (the bias-gradient column H of a product of width H + 16).
 size_t gru_tpart_floats(const bg_plan* p, int H, int T) {
   return bg::gemm_tn_part_floats(6 * H, H + 16, (int64_t)T * p->n_pad());
 }
@@ -526,9 +527,10 @@ size_t saved_E_off(const bg_plan* p, bg_dtype dt, int H, int t) {
 size_t saved_Y_off(const bg_plan* p, bg_dtype dt, int H, int T, int t) {
   return saved_E_off(p, dt, H, T + 1) + (size_t)t * al(sizeof(float) * (size_t)p->n_pad() * H);
 }
-// With the band kernel and bf16 Y (H = 256): after E(0..T) and Y(0..T-1), [E(0..T-1)^T; 1; 0] and
-// [Y(0..T-1)^T; 1; 0] as [H+16][T n] bf16, written by the forward's GRU and band kernels: the band
-// products' operands and the weight-gradient GEMMs' (ones row -> bias gradient).
+// With the band kernel and bf16 Y (H = 256): after E(0..T) and Y(0..T-1), E(0..T-1)^T and
+// Y(0..T-1)^T in [H+16][T n] bf16 arrays, written by the forward's GRU and band kernels: the band
+// products' operands and the weight-gradient GEMMs', which read the first H rows and append the
+// ones row (-> bias gradient) in shared memory; the last 16 rows are not written.
 struct YbSaved {
   size_t ETa, YTa, total;
 };
@@ -553,9 +555,10 @@ bool tc_ggnn(const bg_plan* p, bg_dtype dt, int H) {
   return tc_shape(p, dt, H) && bg::band_tc_supported(p, (int)dt, H) && bg::gru_tc_supported(H);
 }
 
-// Saved activations: E(0..T) [n][H]; [E(0..T-1)^T; 1; 0] as [H+16][T n]; Y(0..T-1) [n][H];
-// [Y(0..T-1)^T; 1; 0] as [H+16][T n]  (all bf16).  The transposed copies are the operands of the
-// band products (TMA, K contiguous) and of the weight-gradient GEMMs (ones row -> bias gradient).
+// Saved activations: E(0..T) [n][H]; E(0..T-1)^T in an [H+16][T n] array; Y(0..T-1) [n][H];
+// Y(0..T-1)^T in an [H+16][T n] array (all bf16).  The transposed copies are the operands of the
+// band products (TMA, K contiguous) and of the weight-gradient GEMMs, which append the ones row
+// (-> bias gradient) in shared memory; the last 16 rows of each array are not written.
 struct TcSaved {
   size_t E, ETa, Y, YTa, total;
 };
@@ -779,7 +782,7 @@ static int propagate_bwd_band(const bg_plan* p, bg_dtype dt, int H, const void* 
                                accum, status, st));
     }
     KTimer t(BG_KID_DW, st);
-    // dW_p, db_p from one split-K product of dM^T with [E^T; 1; 0]
+    // dW_p, db_p from one split-K product of dM^T with E^T and the GEMM's appended ones row
     BG_CUDA(bg::prep_transpose_bf16(dMb, 0, dMT, (int)n, PH, 1, st));
     BG_CUDA(bg::prep_transpose_bf16(E, 0, ETa, (int)n, H, 1, st));
     BG_CUDA(bg::gemm_tn(dMT, (int64_t)n, ETa, (int64_t)n, PH, H, (int64_t)n, 1, dW, db, accum,
@@ -1199,8 +1202,7 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
   auto* WhhT = reinterpret_cast<__nv_bfloat16*>(wsc + w.WhhT);
   if (tcg) {
     BG_TRY(status_word_ptr(&status));
-    // B operands W^T [H][3H] of dX = dgi W_ih and g += dgh W_hh; the ones rows of [Y^T; 1; 0] and
-    // [E^T; 1; 0] over all T steps (their bias-gradient column)
+    // B operands W^T [H][3H] of dX = dgi W_ih and g += dgh W_hh
     BG_CUDA(bg::prep_transpose_bf16(prm->W_ih, 0, WihT, 3 * H, H, 1, st));
     BG_CUDA(bg::prep_transpose_bf16(prm->W_hh, 0, WhhT, 3 * H, H, 1, st));
   }
