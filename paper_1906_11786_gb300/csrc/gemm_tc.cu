@@ -570,6 +570,8 @@ cudaError_t gemm_tn_multi(const TNProblem* pr, int n, int Hout, int64_t K, int a
   // few CTAs would nearly double the time of this HBM-bound pass)
   int splits = (int)std::max<int64_t>(1, std::min<int64_t>(kchunks, std::max(1, sms / mt)));
   while (splits > 1 && (size_t)splits * Mtot * N > part_floats) --splits;
+  // the kernel writes its partial sums even when it does not split K
+  if ((size_t)splits * Mtot * N > part_floats) return cudaErrorInvalidValue;
   const int per = (int)((kchunks + splits - 1) / splits);
   splits = (int)((kchunks + per - 1) / per);
   dim3 grid(mt, 1, splits);

@@ -565,6 +565,7 @@ cudaError_t colsum(const float* X, int64_t rows, int cols, float* out, int accum
   if (splits > 256) splits = 256;
   while (splits > 1 && (size_t)splits * cols > part_floats) --splits;
   if (splits < 1) splits = 1;
+  if ((size_t)splits * cols > part_floats) return cudaErrorInvalidValue;  // partials always used
   int64_t chunk = (rows + splits - 1) / splits;
   dim3 grid((cols + 255) / 256, splits);
   k_colsum_part<<<grid, 256, 0, st>>>(X, rows, cols, chunk, part);
