@@ -9,7 +9,8 @@ per second = real (non-padding) nodes x T / step time.  Default workload: 64 pro
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload packed64] [--impl ours|reference]
 
 Under torchrun every rank plans its own supergraph (different seeds; the paper gives each core its
-own supergraph) and runs with no data-path collective (weak scaling); rank 0 prints one JSON line.
+own supergraph: weak scaling); the step's one collective is the mean of the ranks' gradients after
+the backward (the paper's synchronous data-parallel update); rank 0 prints one JSON line.
 """
 from __future__ import annotations
 
