@@ -1,7 +1,9 @@
 """Multi-GPU logic of the benchmark on CPU ranks (gloo, world size 2): every rank plans its own
 supergraph of the same shape (the paper gives each core its own supergraph), the whole-job
 figures are the slowest rank's time and the sum of all ranks' node-steps, and the data-parallel
-gradient exchange leaves every rank with the mean of all ranks' gradients.  No GPU is used."""
+gradient exchange leaves every rank with the mean of all ranks' gradients, which equals the
+gradient of the union of the ranks' graphs divided by the number of ranks.  The block-row split
+of one supergraph exchanges halos and sums dW, db.  No GPU is used."""
 import os
 import socket
 
@@ -174,3 +176,76 @@ def test_block_row_split_two_ranks_matches_the_whole_plan():
         assert edW < 1e-9 and edb < 1e-9
         rows += own
     assert rows > 0
+
+
+
+DP_P, DP_S, DP_H, DP_T = 4, 64, 8, 2
+
+
+def _dp_grads(graphs, seeds):
+    """Oracle GGNN forward + backward (T = 2) over one supergraph of `graphs`, nothing dropped,
+    graph i's states and incoming gradient drawn from seeds[i] in its original node order: the
+    parameter gradients as one flat fp64 vector."""
+    import numpy as np
+
+    import oracle
+    from paper_1906_11786_gb300 import synth
+    P, S, H, T = DP_P, DP_S, DP_H, DP_T
+    lay = oracle.layout(graphs, P, S)
+    assert lay.n_dropped == 0 and lay.n_packed == len(graphs)
+    E_orig = np.concatenate([synth.gen_states(g.n_nodes, H, s) for g, s in zip(graphs, seeds)])
+    dET_orig = np.concatenate([synth.gen_states(g.n_nodes, H, s + 7)
+                               for g, s in zip(graphs, seeds)])
+    N, gi = lay.n_pad, lay.gather_index()
+    E0 = np.zeros((N, H)); E0[:lay.n_real] = E_orig[gi]
+    dET = np.zeros((N, H)); dET[:lay.n_real] = dET_orig[gi]
+    prm = synth.gen_params(P, H, 4242)
+    edges = (lay.kept_dst, lay.kept_src, lay.kept_type)
+    Es, Ys = oracle.ggnn_fwd(N, P, H, T, lay.n_real, *edges, E0, prm)
+    g = oracle.ggnn_bwd(N, P, H, T, lay.n_real, *edges, prm, Es, Ys, dET)
+    return np.concatenate([g[k].ravel() for k in ("dW", "db", "dW_ih", "dW_hh", "db_ih", "db_hh")])
+
+
+def _dp_graphs(rank):
+    from paper_1906_11786_gb300 import synth
+    gs = synth.gen_batch(3, 30, 60, 2, True, 6, 6, 1.0, 900 + rank)
+    return gs, [1000 * (rank + 1) + 31 * i for i in range(len(gs))]
+
+
+def _dp_worker(rank, world, port, out):
+    """One data-parallel rank: its own supergraph's gradients (the oracle standing in for the
+    device step on CPU), then the benchmark's gradient exchange."""
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    import bench
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        own = _dp_grads(*_dp_graphs(rank))
+        flat = torch.from_numpy(own.copy())
+        bench.allreduce_grads(dist, flat)
+        out[rank] = (own.tolist(), flat.tolist())
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.timeout(300)
+def test_data_parallel_mean_equals_the_union_batch_gradient():
+    """The synchronous data-parallel step (each rank its own supergraph, as the paper trains on
+    several cores; gradients averaged by the exchange) equals one step over the union of the
+    ranks' graphs with its gradient divided by the number of ranks: the graphs share no edge, so
+    their gradient contributions add.  fp64 oracle arithmetic throughout; gloo ranks."""
+    import numpy as np
+    world = 2
+    port = _free_port()
+    mgr = mp.get_context("spawn").Manager()
+    out = mgr.dict()
+    mp.start_processes(_dp_worker, args=(world, port, out), nprocs=world, start_method="spawn")
+    parts = [_dp_graphs(r) for r in range(world)]
+    union = _dp_grads([g for gs, _ in parts for g in gs], [s for _, ss in parts for s in ss])
+    own = [np.array(out[r][0]) for r in range(world)]
+    assert np.max(np.abs(own[0] - own[1])) > 1e-3  # the ranks' supergraphs differ
+    for r in range(world):
+        got = np.array(out[r][1])
+        np.testing.assert_allclose(got, (own[0] + own[1]) / world, rtol=0, atol=1e-12)
+        np.testing.assert_allclose(got, union / world, rtol=1e-10,
+                                   atol=1e-10 * np.max(np.abs(union)))
