@@ -284,6 +284,45 @@ def test_ggnn_bwd_finite_differences():
         np.testing.assert_allclose(out[gk], _fd(f, prm[k]), rtol=1e-6, atol=1e-8, err_msg=k)
 
 
+
+def _ggnn(N, P, H, T, g_dst, g_src, g_typ, E0, G, prm):
+    args = (N, P, H, T, N, g_dst, g_src, g_typ)
+    Es, Ys = oracle.ggnn_fwd(*args, E0, prm)
+    return Es[T], oracle.ggnn_bwd(*args, prm, Es, Ys, G)
+
+
+def test_ggnn_relabelling_and_disjoint_graphs():
+    """T = 3 GGNN steps over the exact edge list: relabelling the nodes relabels E(T) and dE(0)
+    and leaves every parameter gradient unchanged (Eq. 1 has no node order); a union of two graphs
+    that share no edge gives each graph's own E(T) and dE(0), and parameter gradients that are the
+    sum of the two graphs' (they share only the parameters)."""
+    rng = np.random.default_rng(21)
+    P, H, T = 3, 4, 3
+    prm = synth.gen_params(P, H, 8, bias_scale=0.3)
+    keys = ("dW", "db", "dW_ih", "dW_hh", "db_ih", "db_hh")
+    a = synth.gen_graph(25, 3, False, 6, 4, 1.0, 41)
+    E0 = rng.standard_normal((25, H)); G = rng.standard_normal((25, H))
+    ET, gr = _ggnn(25, P, H, T, a.dst, a.src, a.etype, E0, G, prm)
+    pi = rng.permutation(25)  # node v becomes pi[v]
+    Ep = np.zeros_like(E0); Ep[pi] = E0
+    Gp = np.zeros_like(G); Gp[pi] = G
+    ETp, grp = _ggnn(25, P, H, T, pi[a.dst], pi[a.src], a.etype, Ep, Gp, prm)
+    np.testing.assert_allclose(ETp[pi], ET, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(grp["dE0"][pi], gr["dE0"], rtol=0, atol=1e-12)
+    for k in keys:
+        np.testing.assert_allclose(grp[k], gr[k], rtol=1e-12, atol=1e-12, err_msg=k)
+    b = synth.gen_graph(17, 3, False, 6, 4, 1.0, 42)
+    Eb = rng.standard_normal((17, H)); Gb = rng.standard_normal((17, H))
+    ETb, grb = _ggnn(17, P, H, T, b.dst, b.src, b.etype, Eb, Gb, prm)
+    ETu, gru = _ggnn(42, P, H, T, np.concatenate([a.dst, b.dst + 25]),
+                     np.concatenate([a.src, b.src + 25]), np.concatenate([a.etype, b.etype]),
+                     np.concatenate([E0, Eb]), np.concatenate([G, Gb]), prm)
+    np.testing.assert_allclose(ETu, np.concatenate([ET, ETb]), rtol=0, atol=1e-12)
+    np.testing.assert_allclose(gru["dE0"], np.concatenate([gr["dE0"], grb["dE0"]]), rtol=0,
+                               atol=1e-12)
+    for k in keys:
+        np.testing.assert_allclose(gru[k], gr[k] + grb[k], rtol=1e-12, atol=1e-12, err_msg=k)
+
 def test_readout_loss_matches_autograd():
     rng = np.random.default_rng(15)
     N, H = 20, 5
