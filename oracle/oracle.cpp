@@ -181,12 +181,14 @@ int32_t orc_reach(int32_t n, int64_t m, const int32_t* src, const int32_t* dst,
   return kept;
 }
 
-// Number of blocks K the supergraph gets: capacity_blocks, or ceil(sum n / S) when 0.
+// Number of blocks K the supergraph gets: capacity_blocks, or ceil(sum n / S) when 0, and at
+// least one (reading c9: a batch with no nodes is one block of padding).
 int32_t orc_num_blocks(int32_t n_graphs, const int32_t* n_nodes, int32_t S, int32_t capacity_blocks) {
   if (capacity_blocks > 0) return capacity_blocks;
   int64_t tot = 0;
   for (int32_t g = 0; g < n_graphs; ++g) tot += n_nodes[g];
-  return (int32_t)((tot + S - 1) / S);
+  const int64_t k = (tot + S - 1) / S;
+  return (int32_t)(k > 0 ? k : 1);
 }
 
 // Sparse batching into one supergraph (Section 2 "Sparse batching", Section 3.1) and the

@@ -460,6 +460,19 @@ def test_layout_masks_agree_with_kept_edges_and_packing_rule():
     assert not bits[0, 0].any() and not bits[-1, 2].any()
 
 
+
+def test_batch_without_nodes_is_one_padding_block():
+    """Reading c9: K = ceil(sum n / S), at least one block; graphs with no nodes are packed at the
+    current offset and take no positions."""
+    e = np.zeros(0, np.int32)
+    empty = synth.Graph(0, e, e, e, 2)
+    lay = oracle.layout([empty, empty], 2, 32)
+    assert lay.K == 1 and lay.n_packed == 2 and lay.n_real == 0 and lay.offset.tolist() == [0, 0]
+    assert lay.n_kept == 0 and not lay.masks.any()
+    g = _graph(40, [(0, 1), (1, 2)], P=2)
+    lay = oracle.layout([g, empty, g], 2, 32)
+    assert lay.K == 3 and lay.offset.tolist() == [0, 40, 40] and lay.n_real == 80
+
 def test_duplicate_edges_count_once():
     g = _graph(4, [(0, 1), (0, 1), (0, 1), (2, 3)])
     L = oracle.layout([g], 1, 8, flags=0)

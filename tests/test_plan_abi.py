@@ -374,3 +374,47 @@ def test_partition_tiles_rows_and_halos(S, n_parts):
                       L.BG_RCM | L.BG_KEEP_IF_BETTER | L.BG_SUPERNODES, 100, 1)
     with pytest.raises(L.BandGGNNError):
         L.plan_partition(sup, 2, 0)
+
+
+def _random_graph(rng, n, P):
+    """Arbitrary (not program-shaped) typed edges: uniform pairs, a dense clump, duplicates,
+    self-loops and isolated nodes."""
+    m = int(rng.integers(0, 4 * n + 1)) if n else 0
+    src = rng.integers(0, max(n, 1), m)
+    dst = rng.integers(0, max(n, 1), m)
+    if n >= 8 and rng.random() < 0.5:  # a dense clump of 8 nodes somewhere in the graph
+        c = rng.choice(n, 8, replace=False)
+        a, b = np.meshgrid(c, c)
+        src, dst = np.concatenate([src, a.ravel()]), np.concatenate([dst, b.ravel()])
+    if len(src) and rng.random() < 0.5:  # duplicates
+        k = rng.integers(0, len(src), len(src) // 4 + 1)
+        src, dst = np.concatenate([src, src[k]]), np.concatenate([dst, dst[k]])
+    typ = rng.integers(0, P, len(src))
+    return synth.Graph(n, src.astype(np.int32), dst.astype(np.int32), typ.astype(np.int32), P)
+
+
+@pytest.mark.parametrize("seed", range(48))
+def test_planner_bit_exact_on_arbitrary_graphs(seed):
+    """Random batches of arbitrary graphs (0 to 400 nodes, up to 4n random typed edges plus dense
+    clumps, duplicates and self-loops), every block size, random capacities (the batch may not
+    fit) and every ordering flag: the planner stays bit-exact against the oracle."""
+    rng = np.random.default_rng(7000 + seed)
+    P = int(rng.integers(1, 7))
+    S = int(rng.choice([32, 64, 128, 256, 512]))
+    sizes = [0 if rng.random() < 0.1 else int(rng.integers(1, 401))
+             for _ in range(int(rng.integers(1, 7)))]
+    gs = [_random_graph(rng, n, P) for n in sizes]
+    total = sum(g.n_nodes for g in gs)
+    cap = 0 if rng.random() < 0.5 else int(rng.integers(1, max(1, -(-total // S)) + 1))
+    if cap and gs[0].n_nodes > cap * S:
+        cap = max(1, -(-gs[0].n_nodes // S))  # at least the first graph fits
+    flags = [0, L.BG_RCM, L.BG_RCM | L.BG_KEEP_IF_BETTER][int(rng.integers(0, 3))]
+    _compare(gs, P, S, cap, flags)
+
+
+def test_planner_bit_exact_on_batches_without_nodes():
+    e = np.zeros(0, np.int32)
+    empty = synth.Graph(0, e, e, e, 3)
+    plan, ref = _compare([empty], 3, 64)
+    assert ref.K == 1 and ref.n_real == 0
+    _compare([empty, synth.gen_graph(70, 3, False, 6, 4, 1.0, 2), empty], 3, 32)
