@@ -418,3 +418,48 @@ def test_planner_bit_exact_on_batches_without_nodes():
     plan, ref = _compare([empty], 3, 64)
     assert ref.K == 1 and ref.n_real == 0
     _compare([empty, synth.gen_graph(70, 3, False, 6, 4, 1.0, 2), empty], 3, 32)
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_reach_filter_bit_exact_on_arbitrary_graphs(seed):
+    """Reachability preprocessing on arbitrary graphs (duplicates, self-loops, isolated nodes,
+    repeated candidates, T from 0 to 6): the library's kept nodes, renumbering and kept edges
+    equal the oracle's."""
+    rng = np.random.default_rng(8100 + seed)
+    g = _random_graph(rng, int(rng.integers(1, 301)), int(rng.integers(1, 5)))
+    cand = rng.integers(0, g.n_nodes, int(rng.integers(1, 6))).astype(np.int32)
+    T = int(rng.integers(0, 7))
+    got = L.reach_filter(g, cand, T)
+    want = oracle.reach_filter(g, cand, T)
+    np.testing.assert_array_equal(got[0], want[0])
+    assert got[1] == want[1]
+    for a, b in zip(got[2:], want[2:]):
+        np.testing.assert_array_equal(a, b)
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_planner_bit_exact_with_supernodes_on_arbitrary_graphs(seed):
+    """Supernodes on arbitrary graphs with random thresholds and caps (including none found and
+    more candidates than the cap): positions, band tiles, counts and the supernode edge list equal
+    the oracle's."""
+    rng = np.random.default_rng(8200 + seed)
+    P = int(rng.integers(1, 6))
+    S = int(rng.choice([32, 64, 128, 256, 512]))
+    gs = [_random_graph(rng, int(rng.integers(0, 301)), P) for _ in range(int(rng.integers(1, 5)))]
+    min_deg = int(rng.integers(1, 40))
+    max_sup = int(rng.integers(0, 6))
+    F = L.BG_RCM | L.BG_KEEP_IF_BETTER | L.BG_SUPERNODES
+    plan = L.band_plan(gs, P, S, 0, F, min_deg, max_sup)
+    ref = oracle.layout(gs, P, S, flags=F, super_min_degree=min_deg, max_super=max_sup)
+    info = plan.info()
+    for k in ("K", "n_packed", "n_real"):
+        assert info[k] == getattr(ref, k)
+    assert info["n_kept"] == ref.n_kept and info["n_dropped"] == ref.n_dropped
+    assert info["bw_after_max"] == ref.bw_after_max and info["n_edges_unique"] == ref.n_unique
+    np.testing.assert_array_equal(plan.export(L.BG_EXPORT_PERM), ref.perm)
+    np.testing.assert_array_equal(plan.export(L.BG_EXPORT_OFFSETS), ref.offset)
+    assert plan.export(L.BG_EXPORT_MASKS).tobytes() == ref.masks.tobytes()
+    sup = plan.export(L.BG_EXPORT_SUPER_EDGES)
+    want = np.stack([ref.kept_dst, ref.kept_src, ref.kept_type], 1)[ref.kept_super]
+    np.testing.assert_array_equal(sup.reshape(-1, 3), want.reshape(-1, 3))
+    assert info["n_super_edges"] == len(want) and info["n_super"] == ref.is_super.sum()
