@@ -153,10 +153,12 @@ size_t bg_plan_export_bytes(const bg_plan* plan, int32_t which);
 int bg_plan_export(const bg_plan* plan, int32_t which, void* out, size_t out_bytes);
 
 /* Block-row partition for running one supergraph on several GPUs (Eq. 3: block-row k couples
- * only to block-rows k - 1 and k + 1).  Part `part` of n_parts owns a contiguous range of whole
- * 128-row tiles (max(1, 128 / S) block-rows each; ranges as equal as the tile count allows) and
- * gets a local plan (free it with bg_plan_free; upload it like any plan) over that range plus one
- * tile of halo on each side, clipped at the supergraph's ends.  Local row i is supergraph
+ * only to block-rows k - 1 and k + 1).  The supergraph is cut into units of max(128, S) rows (a
+ * 128-row tile of 128 / S block-rows when S <= 128, one block-row when S > 128).  Part `part` of
+ * n_parts (1 <= n_parts <= the number of units, else BG_EINVAL) owns a contiguous range of whole
+ * units (ranges as equal as the unit count allows) and gets a local plan (free it with
+ * bg_plan_free; upload it like any plan) over that range plus one unit of halo on each side,
+ * clipped at the supergraph's ends.  Local row i is supergraph
  * position row0 + i.  The local forward tiles keep only the rows the part owns as targets, the
  * transposed tiles only the rows it owns as sources.  Used with bg_band_propagate_fwd/bwd:
  *   forward:  fill the local E with rows [row0, row0 + n_local) of the full E -- the halo rows

@@ -361,9 +361,9 @@ int bg_plan_build(const bg_graph* graphs, int32_t n_graphs, int32_t P, int32_t S
 }
 
 // Block-row partition of a plan (Eq. 3: block-row k couples only to block-rows k - 1 and k + 1).
-// Part `part` of n_parts owns a contiguous range of whole 128-row tiles (of max(1, 128 / S)
-// block-rows each); its local plan spans that range plus one tile of halo on each side (clipped
-// at the ends).  The forward tiles keep only the rows the part owns as targets and the
+// Part `part` of n_parts owns a contiguous range of whole units of max(128, S) rows (a 128-row
+// tile of 128 / S block-rows when S <= 128, one block-row otherwise); its local plan spans that
+// range plus one unit of halo on each side (clipped at the ends).  The forward tiles keep only the rows the part owns as targets and the
 // transposed tiles only the rows it owns as sources, so with the halo rows of E (forward) or dY
 // (backward) copied in from the neighbours the part's own rows of Y and dE are exact, the halo
 // rows of Y and dE come out 0, and its dW, db are the sums over its own source rows: summed over
@@ -374,9 +374,9 @@ int bg_plan_partition_build(const bg_plan* full, int32_t n_parts, int32_t part, 
   *out = nullptr;
   if (full->n_super > 0) return bg_fail(BG_EINVAL, "plans with supernodes cannot be partitioned");
   const int32_t S = full->S, K = full->K, P = full->P;
-  const int32_t unit = S >= 128 ? 1 : 128 / S;  // block-rows per tile
+  const int32_t unit = S >= 128 ? 1 : 128 / S;  // block-rows per unit
   const int32_t n_units = (K + unit - 1) / unit;
-  if (n_parts < 1 || n_parts > n_units) return bg_fail(BG_EINVAL, "n_parts must be in [1, tiles]");
+  if (n_parts < 1 || n_parts > n_units) return bg_fail(BG_EINVAL, "n_parts must be in [1, units of max(128, S) rows]");
   if (part < 0 || part >= n_parts) return bg_fail(BG_EINVAL, "part out of range");
   const int32_t u0 = (int32_t)((int64_t)n_units * part / n_parts);
   const int32_t u1 = (int32_t)((int64_t)n_units * (part + 1) / n_parts);

@@ -204,6 +204,13 @@ def test_tensor_core_upload_layout_from_the_bit_tiles(S, hub, tmp_path_factory, 
     gs = synth.gen_batch(5, 40, 3 * S, 6, False, max(2, S // 2), max(2, S // 3), 1.5, 300 + S)
     if hub:  # in-degrees above 256: the table switches to fp16
         gs.insert(1, synth.hub_graph(S + S // 4, 2, 7 + S))
+    max_deg = _check_upload(exe, gs, P, S, tmp_path)
+    assert (max_deg > 256) == bool(hub)
+
+
+def _check_upload(exe, gs, P, S, tmp_path):
+    """Runs the probe on `gs` (padded with an edgeless graph to whole 128-row tiles) and checks
+    the tensor-core operands it writes against the ones rebuilt here from its bit tiles."""
     n = sum(g.n_nodes for g in gs)
     K0 = -(-n // S)
     if K0 * S % 128:  # whole 128-row tiles, as the tensor-core path requires: pad with a graph
@@ -260,7 +267,7 @@ def test_tensor_core_upload_layout_from_the_bit_tiles(S, hub, tmp_path_factory, 
     exp_deg[:, 32:32 + P] = exp_deg[:, :P]
     np.testing.assert_array_equal(deg.reshape(N, 64), exp_deg)
     assert max_deg == cnt.max()
-    assert (max_deg > 256) == bool(hub)
+    return int(max_deg)
 
 
 @pytest.mark.parametrize("T", [0, 1, 3, 8])
@@ -335,15 +342,27 @@ def edges_from_masks(m, S, transposed=False):
 
 @pytest.mark.parametrize("S,n_parts", [(32, 2), (128, 3), (256, 2), (64, 5)])
 def test_partition_tiles_rows_and_halos(S, n_parts):
-    """Block-row split (Eq. 3): the parts own contiguous whole-tile ranges covering the
-    supergraph; each local plan spans its range plus one tile of halo per side; its forward
+    """Block-row split (Eq. 3): the parts own contiguous ranges of whole units (max(128, S) rows)
+    covering the supergraph; each local plan spans its range plus one unit of halo per side; its forward
     tiles hold exactly the kept edges whose target it owns and its transposed tiles those whose
     source it owns, in local positions."""
     gs = synth.gen_batch(8, 100, 600, 4, True, max(2, S // 2), max(2, S // 3), 1.5, 5 + S)
+    full = _check_partition(gs, 8, S, n_parts)
+    with pytest.raises(L.BandGGNNError):
+        L.plan_partition(full, 0, 0)
+    sup = L.band_plan([synth.hub_graph(300, 8, 1)], 8, S, 0,
+                      L.BG_RCM | L.BG_KEEP_IF_BETTER | L.BG_SUPERNODES, 100, 1)
+    with pytest.raises(L.BandGGNNError):
+        L.plan_partition(sup, 2, 0)
+
+
+def _check_partition(gs, P, S, n_parts):
+    """Plans `gs` at whole 128-row tiles, splits the plan into n_parts and checks every part
+    (own ranges, halos, local forward and transposed tiles, real rows); returns the plan."""
     n = sum(g.n_nodes for g in gs)
     unit = max(1, 128 // S)
     cap = -(-(-(-n // S)) // unit) * unit
-    full = L.band_plan(gs, 8, S, cap)
+    full = L.band_plan(gs, P, S, cap)
     fi = full.info()
     d, s_, t = edges_from_masks(full.export(L.BG_EXPORT_MASKS), S)
     pos_all = []
@@ -368,12 +387,7 @@ def test_partition_tiles_rows_and_halos(S, n_parts):
         assert si["n_real"] == max(0, min(inf["n_local"], fi["n_real"] - r0))
     pos_all = np.concatenate(pos_all)
     np.testing.assert_array_equal(pos_all, np.arange(fi["n_pad"]))
-    with pytest.raises(L.BandGGNNError):
-        L.plan_partition(full, 0, 0)
-    sup = L.band_plan([synth.hub_graph(300, 8, 1)], 8, S, 0,
-                      L.BG_RCM | L.BG_KEEP_IF_BETTER | L.BG_SUPERNODES, 100, 1)
-    with pytest.raises(L.BandGGNNError):
-        L.plan_partition(sup, 2, 0)
+    return full
 
 
 def _random_graph(rng, n, P):
@@ -463,3 +477,31 @@ def test_planner_bit_exact_with_supernodes_on_arbitrary_graphs(seed):
     want = np.stack([ref.kept_dst, ref.kept_src, ref.kept_type], 1)[ref.kept_super]
     np.testing.assert_array_equal(sup.reshape(-1, 3), want.reshape(-1, 3))
     assert info["n_super_edges"] == len(want) and info["n_super"] == ref.is_super.sum()
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_tensor_core_upload_layout_on_arbitrary_graphs(seed, tmp_path_factory, tmp_path):
+    """The tensor-core operands on arbitrary graphs (dropped edges, duplicates, self-loops, dense
+    clumps), every block size."""
+    rng = np.random.default_rng(8300 + seed)
+    P = int(rng.integers(1, 7))
+    S = int(rng.choice([32, 64, 128, 256, 512]))
+    gs = [_random_graph(rng, int(rng.integers(1, 401)), P) for _ in range(int(rng.integers(1, 5)))]
+    _check_upload(_probe_binary(tmp_path_factory), gs, P, S, tmp_path)
+
+
+@pytest.mark.parametrize("seed", range(16))
+def test_partition_on_arbitrary_graphs(seed):
+    """The block-row split on arbitrary graphs (dropped edges, duplicates, self-loops), every block
+    size, from two parts up to one part per unit of max(128, S) rows."""
+    rng = np.random.default_rng(8400 + seed)
+    P = int(rng.integers(1, 7))
+    S = int(rng.choice([32, 64, 128, 256, 512]))
+    gs = [_random_graph(rng, int(rng.integers(1, 401)), P) for _ in range(int(rng.integers(2, 7)))]
+    n = sum(g.n_nodes for g in gs)
+    rows = max(128, S)  # the partition's unit: a 128-row tile, or one block-row when S > 128
+    if -(-n // rows) < 2:
+        gs.append(_random_graph(rng, rows, P))
+        n += rows
+    units = -(-n // rows)
+    _check_partition(gs, P, S, int(rng.integers(2, min(units, 6) + 1)))
