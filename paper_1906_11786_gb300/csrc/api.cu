@@ -491,7 +491,7 @@ GgnnBwdWs ggnn_bwd_ws(const bg_plan* p, bg_dtype dt, int H, int T) {
     w.dghb = o; o += al(n * 3 * H * 2);
     w.dgiT = o; o += al(TN * 3 * H * 2);
     w.dghT = o; o += al(TN * 3 * H * 2);
-    // with the band kernel the forward keeps [Y^T; 1] and [E^T; 1] among the saved activations
+    // with the band kernel the forward keeps Y^T and E^T among the saved activations
     w.YTa = o; o += ybf ? 0 : al((size_t)(H + 16) * TN * 2);
     w.ETa = o; o += ybf ? 0 : al((size_t)(H + 16) * TN * 2);
     w.WihT = o; o += al((size_t)3 * H * H * 2);
@@ -937,7 +937,7 @@ extern "C" int bg_ggnn_step(const bg_plan* p, bg_dtype dt, int32_t H, int32_t T,
   BG_CUDA(cudaMemcpyAsync(sv + saved_E_off(p, dt, H, 0), E0, ebytes, cudaMemcpyDeviceToDevice, st));
   if (y_bf16_path(p, dt, H)) {
     // band kernel (bf16 Y and Y^T) and the fused GRU forward (E(t+1) and E(t+1)^T): the
-    // transposed copies go to the saved [E^T; 1] and [Y^T; 1] for the band products of the next
+    // transposed copies go to the saved E^T and Y^T arrays for the band products of the next
     // step and for the backward's weight gradients
     int* status = nullptr;
     BG_TRY(status_word_ptr(&status));
@@ -1098,9 +1098,9 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
   if (y_bf16_path(p, dt, H)) {
     // H = 256 with the band kernel: per step the gate gradients (one kernel), dX^T = (dgi W_ih)^T
     // straight into the band backward's operand, g += dgh W_hh, the transposed-band backward and
-    // the band's weight gradients from its dM_p^T (one step's K range of [E^T; 1] stays in L2
+    // the band's weight gradients from its dM_p^T (one step's K range of E^T stays in L2
     // across the M tiles, which a product over all T steps at once does not); the GRU's weight
-    // gradients in one grouped product over all T steps at the end (operands [E^T; 1], [Y^T; 1]
+    // gradients in one grouped product over all T steps at the end (operands E^T, Y^T
     // saved by the forward).  The running state gradient alternates between two buffers.
     int* status = nullptr;
     BG_TRY(status_word_ptr(&status));
@@ -1262,7 +1262,8 @@ extern "C" int bg_ggnn_step_bwd(const bg_plan* p, bg_dtype dt, int32_t H, int32_
     }
   }
   if (tcg) {
-    // dW_ih, db_ih += dgi^T [Y; 1] and dW_hh, db_hh += dgh^T [E; 1] over all T steps at once
+    // dW_ih, db_ih += dgi^T [Y 1] and dW_hh, db_hh += dgh^T [E 1] over all T steps at once (the
+    // GEMM appends the ones column)
     KTimer tm(BG_KID_DW, st);
     const bg::TNProblem probs[2] = {
         {dgiT, TN, YTa, TN, 3 * H, 0, gr->dW_ih, gr->db_ih},
