@@ -525,6 +525,34 @@ def test_parallel_oracle_equals_the_oracle_to_the_last_bit():
     assert oracle.par_max_threads() >= 1
 
 
+
+@pytest.mark.parametrize("seed", range(6))
+def test_parallel_oracle_equals_the_oracle_on_unsorted_edge_lists(seed):
+    """The same on raw edge lists in arbitrary order, with repeated edges and self-loops and thread
+    counts from 1 to 7: the pull-based gather visits each target's and each source's edges in
+    list order, as the scatter does."""
+    rng = np.random.default_rng(600 + seed)
+    N, P, H, T = int(rng.integers(5, 80)), int(rng.integers(1, 5)), int(rng.integers(1, 9)), 2
+    m = int(rng.integers(0, 6 * N))
+    e = (rng.integers(0, N, m), rng.integers(0, N, m), rng.integers(0, P, m))
+    threads = int(rng.integers(1, 8))
+    E = rng.standard_normal((N, H)); dY = rng.standard_normal((N, H))
+    prm = synth.gen_params(P, H, 9 + seed)
+    np.testing.assert_array_equal(
+        oracle.par_propagate_fwd(N, P, H, *e, E, prm["W"], prm["b"], threads),
+        oracle.propagate_fwd(N, P, H, *e, E, prm["W"], prm["b"]))
+    for a, b in zip(oracle.par_propagate_bwd(N, P, H, *e, E, prm["W"], dY, threads),
+                    oracle.propagate_bwd(N, P, H, *e, E, prm["W"], dY)):
+        np.testing.assert_array_equal(a, b)
+    n_real = N - int(rng.integers(0, 3))
+    Es, Ys = oracle.ggnn_fwd(N, P, H, T, n_real, *e, E, prm)
+    Es2, Ys2 = oracle.par_ggnn_fwd(N, P, H, T, n_real, *e, E, prm, threads)
+    np.testing.assert_array_equal(Es2, Es)
+    r = oracle.ggnn_bwd(N, P, H, T, n_real, *e, prm, Es, Ys, dY)
+    r2 = oracle.par_ggnn_bwd(N, P, H, T, n_real, *e, prm, Es, Ys, dY, threads)
+    for k in r:
+        np.testing.assert_array_equal(r2[k], r[k], err_msg=k)
+
 # ------------------------------------------------------------------------ reachability (Section 4)
 
 
