@@ -32,3 +32,26 @@ def test_reference_arm_json_line():
     assert c["workload"] == "single512" and c["n_real"] == 512 and c["T"] == 1
     # a 512-node step fits the L2: the line says so instead of claiming a working set above it
     assert "fits the 129 MB L2" in c["l2"]
+
+
+def test_reference_arm_under_two_ranks_prints_one_line():
+    """Launched as the multi-GPU runs launch it (torchrun, two ranks): rank 0 alone runs the
+    oracle and prints one JSON line; the other rank exits 0 without work."""
+    import socket
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    out = subprocess.run(
+        [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+         "--master-addr", "127.0.0.1", "--master-port", str(port), os.path.join(ROOT, "bench.py"),
+         "--impl", "reference", "--gpus", "2", "--steps", "1", "--warmup", "3", "--ref-budget",
+         "1", "--workload", "single512"],
+        cwd=ROOT, capture_output=True, text=True, timeout=600,
+        env=dict(os.environ, OMP_NUM_THREADS="1"))
+    assert out.returncode == 0, out.stderr[-2000:]
+    lines = [l for l in out.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, out.stdout[-2000:]
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["warmup"] == 3
+    assert d["config"]["parallelism"].startswith("dp2")
