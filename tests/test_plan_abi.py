@@ -505,3 +505,61 @@ def test_partition_on_arbitrary_graphs(seed):
         n += rows
     units = -(-n // rows)
     _check_partition(gs, P, S, int(rng.integers(2, min(units, 6) + 1)))
+
+
+def _header_prototypes():
+    """(return type, [argument types]) of every function the C header declares."""
+    import re
+    src = open(L.HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", "", src)
+    out = {}
+    for m in re.finditer(r"([A-Za-z_][\w\s\*]*?)\s*\b(bg_\w+)\s*\(([^;{]*?)\)\s*;", src):
+        ret, name, args = m.group(1).strip(), m.group(2), m.group(3).strip()
+        ret = ret.split("\n")[-1].strip()
+        params = [] if args in ("", "void") else [a.strip() for a in args.split(",")]
+        # drop the parameter name: the type is everything before the last identifier
+        types = [re.sub(r"\s*\b\w+$", "", a) if not a.endswith("*") else a for a in params]
+        out[name] = (ret, types)
+    return out
+
+
+def _ctype_of(ctype: str):
+    t = " ".join(ctype.replace("const ", "").split())
+    if "*" in t:
+        return "char_p" if t.replace(" ", "") == "char*" else "pointer"
+    return {"int": ctypes.c_int, "int32_t": ctypes.c_int32, "uint32_t": ctypes.c_uint32,
+            "int64_t": ctypes.c_int64, "size_t": ctypes.c_size_t, "float": ctypes.c_float,
+            "double": ctypes.c_double, "bg_dtype": ctypes.c_int, "void": None}[t]
+
+
+def test_binding_signatures_match_the_header():
+    """Every function the header declares is bound with the same number of arguments and
+    matching types (pointer, 32/64-bit integer, size, float, double) and return type: a
+    mismatch would hand the library shifted or truncated arguments."""
+    lib = L.load()
+    protos = _header_prototypes()
+    assert set(protos) == set(L.declared_symbols())
+    for name, (ret, args) in protos.items():
+        fn = getattr(lib, name)
+        assert fn.argtypes is not None, f"{name} has no bound signature"
+        assert len(fn.argtypes) == len(args), (name, len(fn.argtypes), args)
+        for i, (a, b) in enumerate(zip(args, fn.argtypes)):
+            want = _ctype_of(a)
+            if want == "pointer":
+                assert b in (ctypes.c_void_p, ctypes.c_char_p), (name, i, a, b)
+            else:
+                assert b is want or ctypes.sizeof(b) == ctypes.sizeof(want) and \
+                    (b in (ctypes.c_float, ctypes.c_double)) == (want in (ctypes.c_float,
+                                                                          ctypes.c_double)), \
+                    (name, i, a, b)
+        want = _ctype_of(ret)
+        if want == "pointer":
+            assert fn.restype == ctypes.c_void_p, (name, ret)
+        elif want == "char_p":
+            assert fn.restype == ctypes.c_char_p, (name, ret)
+        elif want is None:
+            assert fn.restype is None, (name, ret)
+        else:
+            assert fn.restype is want or ctypes.sizeof(fn.restype) == ctypes.sizeof(want), \
+                (name, ret, fn.restype)
