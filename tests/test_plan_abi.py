@@ -563,3 +563,44 @@ def test_binding_signatures_match_the_header():
         else:
             assert fn.restype is want or ctypes.sizeof(fn.restype) == ctypes.sizeof(want), \
                 (name, ret, fn.restype)
+
+
+def test_binding_structs_match_the_c_layout(tmp_path):
+    """The ctypes structures of the binding have the header's fields in its order, at the offsets
+    and total size the C compiler gives them (a small C program compiled against the header
+    prints them)."""
+    import re
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    src = re.sub(r"/\*.*?\*/", "", open(L.HEADER).read(), flags=re.S)
+    structs = {}
+    for m in re.finditer(r"typedef struct (bg_\w+) \{(.*?)\} \1;", src, flags=re.S):
+        fields = re.findall(r"(\w+)\s*;", m.group(2))
+        structs[m.group(1)] = fields
+    assert set(structs) == {"bg_graph", "bg_info", "bg_plan_opts", "bg_part_info", "bg_params",
+                            "bg_grads"}
+    lines = ['#include <stddef.h>', '#include <stdio.h>', '#include "bandggnn.h"', "int main(void) {"]
+    for s, fields in structs.items():
+        lines.append(f'  printf("{s} . %zu\\n", sizeof({s}));')
+        for f in fields:
+            lines.append(f'  printf("{s} {f} %zu\\n", offsetof({s}, {f}));')
+    lines += ["  return 0;", "}"]
+    (tmp_path / "layout.c").write_text("\n".join(lines))
+    exe = str(tmp_path / "layout")
+    import os
+    inc = os.path.dirname(L.HEADER)
+    subprocess.run([cc, "-std=c99", "-I", inc, str(tmp_path / "layout.c"), "-o", exe], check=True)
+    got = {}
+    for line in subprocess.run([exe], capture_output=True, text=True, check=True).stdout.split("\n"):
+        if line:
+            s, f, v = line.split()
+            got[(s, f)] = int(v)
+    for s, fields in structs.items():
+        cls = getattr(L, s)
+        assert [f for f, _ in cls._fields_] == fields, s
+        assert ctypes.sizeof(cls) == got[(s, ".")], s
+        for f in fields:
+            assert getattr(cls, f).offset == got[(s, f)], (s, f)
