@@ -604,3 +604,27 @@ def test_binding_structs_match_the_c_layout(tmp_path):
         assert ctypes.sizeof(cls) == got[(s, ".")], s
         for f in fields:
             assert getattr(cls, f).offset == got[(s, f)], (s, f)
+
+
+def test_binding_constants_match_the_header():
+    """Every constant of the header (status codes, flags, dtype values, export, op and kernel ids)
+    has the same value in the binding; the status names cover every code."""
+    import re
+    src = re.sub(r"/\*.*?\*/", "", open(L.HEADER).read(), flags=re.S)
+    consts = {m.group(1): int(m.group(2))
+              for m in re.finditer(r"#define (BG_\w+)\s+\(?(-?\d+)u?\)?", src)}
+    for m in re.finditer(r"(BG_\w+)\s*=\s*(-?\d+)", src):
+        consts[m.group(1)] = int(m.group(2))
+    assert len(consts) >= 30
+    status = {k: v for k, v in consts.items() if k in ("BG_OK",) or k.startswith("BG_E") and
+              not k.startswith("BG_EXPORT")}
+    assert {v: k for k, v in status.items()} == L.STATUS
+    missing = []
+    for k, v in consts.items():
+        if k in status or k == "BG_KID_COUNT":
+            continue
+        if not hasattr(L, k):
+            missing.append(k)
+        else:
+            assert getattr(L, k) == v, (k, getattr(L, k), v)
+    assert not missing, missing
