@@ -142,6 +142,15 @@ MUTANTS = [
     ("parallel oracle: sigmoid of the negated argument", "oracle_par.cpp",
      "double sigmoid_p(double x) { return 1.0 / (1.0 + std::exp(-x)); }",
      "double sigmoid_p(double x) { return 1.0 / (1.0 + std::exp(x)); }", 0),
+    # summation order alone: the same terms added in another order must not pass as bit-equal
+    ("parallel oracle: a target's messages summed last edge first", "oracle_par.cpp",
+     "    for (int64_t i = off[v]; i < off[v + 1]; ++i) {\n      const int64_t e = ids[(size_t)i];",
+     "    for (int64_t i = off[v]; i < off[v + 1]; ++i) {\n"
+     "      const int64_t e = ids[(size_t)(off[v] + off[v + 1] - 1 - i)];", 0),
+    ("parallel oracle: dE summed over the types in descending order", "oracle_par.cpp",
+     "      for (int32_t p = 0; p < P; ++p) {\n        const double* g = &dM[((size_t)p * N + u) * H];",
+     "      for (int32_t p = P - 1; p >= 0; --p) {\n"
+     "        const double* g = &dM[((size_t)p * N + u) * H];", 0),
 ]
 
 
